@@ -1,0 +1,168 @@
+/*
+ * htam.h -- C ABI of the GB300 hierarchical transition-attended memory lookup
+ * (HTAM, arxiv 2605.29734).
+ *
+ * The memory follows the paper's Hierarchical Transition Graph (Eq. 6, §4.1):
+ * coarse *groups* stand for the global nodes V_G, fine *entries* (transition
+ * embeddings) stand for the local nodes V_GL, and every entry has one parent
+ * group (par(l) in Eq. 12).  Each group's key is the mean of its entries.
+ *
+ * A query runs the read side of one evolution step (§4.3, Algorithm 1 steps 2
+ * and 3) for a batch of state embeddings q:
+ *   1. score every non-empty group key with the linear scorer (Eq. 9 with
+ *      phi = w^T z of App. B.6; in embedding space the dot product q . c_g)
+ *      and keep the k_groups best groups (ties to the lower group id);
+ *   2. restrict the candidates to the entries of the selected groups (Eq. 12),
+ *      score them (q . k_e) and return the k_entries best (Eq. 13 as a top-k,
+ *      ties to the lower entry id), with
+ *      lse = log sum_{e in C} exp(s_e / tau) over the WHOLE candidate set C
+ *      and weight w_e = eps/|C| + (1 - eps) * exp(s_e / tau - lse)
+ *      (the eps-uniform / tau-softmax mixture of Eq. 11).
+ * Appending entries is the memory update of Eq. 15: rows are filed under
+ * their groups and the group keys are updated in place.
+ *
+ * Conventions for every function below:
+ *  - Array pointers are DEVICE pointers (except in htam_query_host and the
+ *    host-output helpers), row-major and contiguous, 16-byte aligned.
+ *  - Entry and query rows are of the memory's dtype (fp32 or bf16).
+ *  - Entry ids are the caller's numbering: the rows passed to
+ *    htam_build_memory are ids 0..n-1, appended rows continue from the current
+ *    entry count.  Ids are int32, so the capacity is below 2^31.
+ *  - Work is queued on `cuda_stream` (a cudaStream_t; NULL = legacy default
+ *    stream).  Inputs must stay valid until the queued work has finished;
+ *    the library copies entries into its own storage.
+ *  - Functions return a status and never abort or throw.  Argument errors are
+ *    detected before anything is launched and leave the memory unchanged.
+ *  - One memory object is used from one stream at a time: htam_query does
+ *    not modify the stored entries or keys, but it uses scratch space owned by
+ *    the memory object, so two queries on the same object must not overlap.
+ */
+#ifndef HTAM_H_
+#define HTAM_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct htam_memory htam_memory; /* opaque, owns all its device storage */
+
+typedef enum {
+  HTAM_OK = 0,
+  HTAM_EINVAL = 1,    /* bad argument (null, misaligned, out of range) */
+  HTAM_ENOMEM = 2,    /* device or host allocation failed */
+  HTAM_ECAPACITY = 3, /* append would exceed the memory's capacity */
+  HTAM_ECUDA = 4,     /* a CUDA call or kernel launch failed */
+  HTAM_ETIMEOUT = 5,  /* a bounded device-side wait gave up (kernel returned early) */
+  HTAM_ENODEV = 6     /* no usable CUDA device */
+} htam_status;
+
+typedef enum { HTAM_F32 = 0, HTAM_BF16 = 1 } htam_dtype;
+
+/* Query parameters.
+ *  k_groups : groups kept per query, 1 <= k_groups <= min(n_groups, 64)
+ *  k_entries: entries returned per query, 1 <= k_entries <= 64
+ *  tau      : softmax temperature of Eq. 11, tau > 0 (the paper gives no
+ *             value; 1 is the neutral choice)
+ *  epsilon  : uniform-exploration mass of Eq. 11, 0 <= epsilon <= 1 */
+typedef struct {
+  int32_t k_groups;
+  int32_t k_entries;
+  float tau;
+  float epsilon;
+} htam_query_params;
+
+/* Builds a memory from n entries (the initial memory M_0 of Algorithm 1).
+ *  entries  : [n, d] of dtype, device
+ *  group_ids: [n] int32 in [0, n_groups), device
+ *  d        : embedding dimension, multiple of 8, 8 <= d <= 16384
+ *  n_groups : number of groups, 1 <= n_groups <= 65536
+ *  capacity : most entries the memory will ever hold (>= n, < 2^31); storage
+ *             is reserved up front so that appends never reallocate
+ *  out      : receives the new memory (NULL on failure)
+ * Synchronises `cuda_stream` once (the group sizes are read back to lay out
+ * the pages).  Errors: EINVAL (arguments, a group id out of range), ENOMEM,
+ * ECUDA, ENODEV. */
+htam_status htam_build_memory(const void *entries, const int32_t *group_ids,
+                              int64_t n, int32_t d, int32_t n_groups,
+                              htam_dtype dtype, int64_t capacity,
+                              void *cuda_stream, htam_memory **out);
+
+/* Appends `count` entries (the memory update of Eq. 15) and updates the keys
+ * of the groups they join in place.  New entries get ids n, n+1, ...
+ *  entries  : [count, d] of the memory's dtype, device
+ *  group_ids: [count] int32 in [0, n_groups), device
+ * Synchronises `cuda_stream` once.  Errors: EINVAL (a group id out of range),
+ * ECAPACITY (n + count would exceed the capacity, or the page pool is full);
+ * the memory is unchanged on any error. */
+htam_status htam_append_transitions(htam_memory *m, const void *entries,
+                                    const int32_t *group_ids, int64_t count,
+                                    void *cuda_stream);
+
+/* Answers b queries (device pointers; all outputs caller-allocated):
+ *  queries     : [b, d] of the memory's dtype
+ *  group_idx   : [b, k_groups] int32, selected groups best first, -1 padding
+ *                when fewer than k_groups groups are non-empty
+ *  group_score : [b, k_groups] fp32, q . c_g (-inf for padding)
+ *  entry_idx   : [b, k_entries] int32 entry ids best first, -1 padding when
+ *                the candidate set holds fewer than k_entries entries
+ *  entry_score : [b, k_entries] fp32, q . k_e (-inf for padding)
+ *  entry_weight: [b, k_entries] fp32, w_e as above (0 for padding)
+ *  lse         : [b] fp32 or NULL, log-sum-exp of s/tau over the candidates
+ * Fully asynchronous: nothing is read back.  b may be 0.  A device-side
+ * timeout is reported by htam_device_status.  Errors: EINVAL, ENOMEM (scratch
+ * growth), ECUDA. */
+htam_status htam_query(htam_memory *m, const void *queries, int32_t b,
+                       const htam_query_params *p, int32_t *group_idx,
+                       float *group_score, int32_t *entry_idx,
+                       float *entry_score, float *entry_weight, float *lse,
+                       void *cuda_stream);
+
+/* The same lookup with every array in HOST memory (pageable or pinned): the
+ * queries are copied to the device, htam_query runs, and the outputs are
+ * copied back; returns after the stream has finished.  lse may be NULL. */
+htam_status htam_query_host(htam_memory *m, const void *queries, int32_t b,
+                            const htam_query_params *p, int32_t *group_idx,
+                            float *group_score, int32_t *entry_idx,
+                            float *entry_score, float *entry_weight,
+                            float *lse, void *cuda_stream);
+
+/* Sizes of a memory; any output pointer may be NULL (host pointers). */
+htam_status htam_memory_info(const htam_memory *m, int64_t *n, int32_t *d,
+                             int32_t *n_groups, int64_t *capacity);
+
+/* Copies the current group sizes n_g into counts[n_groups] (host). */
+htam_status htam_memory_group_counts(const htam_memory *m, int64_t *counts);
+
+/* Copies the current group keys (fp32 means, [n_groups, d]) into host
+ * memory; rows of empty groups are zero.  Synchronises `cuda_stream`. */
+htam_status htam_memory_group_keys(const htam_memory *m, float *keys,
+                                   void *cuda_stream);
+
+/* Synchronises `cuda_stream`, reads and clears the memory's device status
+ * word.  Returns ETIMEOUT if a bounded device wait gave up since the last
+ * check, ECUDA if the stream reports an error, OK otherwise. */
+htam_status htam_device_status(htam_memory *m, void *cuda_stream);
+
+/* Releases the memory and all its device storage (NULL is a no-op).  The
+ * caller must make sure no queued work still uses it. */
+void htam_free_memory(htam_memory *m);
+
+/* Human-readable name of a status code (static string). */
+const char *htam_status_string(htam_status s);
+
+/* Diagnostic for the bounded-wait machinery: launches one kernel that waits
+ * for a device flag that nothing sets, giving up after `max_iters` polls; the
+ * kernel records the give-up in a status word and returns.  Returns ETIMEOUT
+ * when the wait gave up (the expected result), OK if it did not, ECUDA on a
+ * launch error.  Synchronises `cuda_stream`.  The paper has no counterpart;
+ * it exists to test failure reporting without faulting the GPU. */
+htam_status htam_selftest_wait_timeout(int64_t max_iters, void *cuda_stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* HTAM_H_ */

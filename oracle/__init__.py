@@ -1,0 +1,187 @@
+"""Float64 CPU oracle for the hierarchical transition-attended memory lookup.
+
+TEST INFRASTRUCTURE ONLY.  The oracle is the plain definition of what the
+lookup computes (group keys, Eq. 9 scoring with the linear scorer of App. B.6,
+the Eq. 12 candidate restriction, the Eq. 11 tau-softmax / eps-uniform policy
+and the Eq. 13 pick, generalised to top-k).  Only ``tests/``,
+``__graft_entry__.smoke()`` and the CPU-baseline leg of ``bench.py`` may import
+it.  It shares no code with the CUDA library and never imports it.
+
+The arithmetic lives in ``htam_oracle.c`` (plain C, double precision,
+sequential sums).  This module compiles it with gcc on first use and wraps it
+with ctypes; numpy arrays in, numpy arrays out.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "htam_oracle.c")
+_BUILD_DIR = os.path.join(_HERE, "_build")
+_LIB_PATH = os.path.join(_BUILD_DIR, "libhtam_oracle.so")
+_lock = threading.Lock()
+_lib = None
+
+F32 = 0
+BF16 = 1
+
+
+def build(force: bool = False) -> str:
+    """Compile the oracle shared library (gcc, -O2, IEEE semantics kept)."""
+    os.makedirs(_BUILD_DIR, exist_ok=True)
+    if (not force and os.path.exists(_LIB_PATH)
+            and os.path.getmtime(_LIB_PATH) >= os.path.getmtime(_SRC)):
+        return _LIB_PATH
+    tmp = _LIB_PATH + f".tmp{os.getpid()}"
+    cmd = ["gcc", "-O2", "-std=c11", "-fPIC", "-shared", "-fno-fast-math",
+           "-ffp-contract=off", "-o", tmp, _SRC, "-lpthread", "-lm"]
+    subprocess.run(cmd, check=True)
+    os.replace(tmp, _LIB_PATH)
+    return _LIB_PATH
+
+
+def _load():
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        lib = ctypes.CDLL(build())
+        P = ctypes.c_void_p
+        i32, i64, dbl = ctypes.c_int32, ctypes.c_int64, ctypes.c_double
+        lib.htam_oracle_centroid_accumulate.argtypes = [P, ctypes.c_int, P, i64, i32, i32, P, P]
+        lib.htam_oracle_centroid_accumulate.restype = ctypes.c_int
+        lib.htam_oracle_centroid_finalize.argtypes = [P, P, i32, i32, P]
+        lib.htam_oracle_centroid_finalize.restype = None
+        lib.htam_oracle_stage1.argtypes = [P, ctypes.c_int, i32, i32, P, P, i32, i32, P, P, ctypes.c_int]
+        lib.htam_oracle_stage1.restype = ctypes.c_int
+        lib.htam_oracle_stage2.argtypes = [P, ctypes.c_int, P, i64, i32, i32, P, ctypes.c_int, i32, P,
+                                           i32, i32, dbl, dbl, P, P, P, P, P, ctypes.c_int]
+        lib.htam_oracle_stage2.restype = ctypes.c_int
+        _lib = lib
+        return lib
+
+
+def _ptr(a: np.ndarray):
+    return a.ctypes.data_as(ctypes.c_void_p)
+
+
+def _as_input(x: np.ndarray):
+    """Return (contiguous array, dtype code). bf16 arrives as uint16 bits."""
+    x = np.ascontiguousarray(x)
+    if x.dtype == np.float32:
+        return x, F32
+    if x.dtype == np.uint16:
+        return x, BF16
+    raise TypeError(f"oracle inputs are float32 or bf16 bits (uint16), got {x.dtype}")
+
+
+def default_threads() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:  # pragma: no cover
+        return os.cpu_count() or 1
+
+
+class CentroidAccumulator:
+    """Group sums and counts fed in chunks (for memories too big to pass at once)."""
+
+    def __init__(self, n_groups: int, d: int):
+        self.n_groups, self.d = int(n_groups), int(d)
+        self.sums = np.zeros((self.n_groups, self.d), dtype=np.float64)
+        self.counts = np.zeros(self.n_groups, dtype=np.int64)
+
+    def add(self, entries: np.ndarray, gid: np.ndarray) -> None:
+        lib = _load()
+        entries, dt = _as_input(entries)
+        gid = np.ascontiguousarray(gid, dtype=np.int32)
+        n = gid.shape[0]
+        if entries.shape != (n, self.d):
+            raise ValueError("entries must be [n, d]")
+        rc = lib.htam_oracle_centroid_accumulate(_ptr(entries), dt, _ptr(gid), n, self.d,
+                                                 self.n_groups, _ptr(self.sums), _ptr(self.counts))
+        if rc != 0:
+            raise ValueError("group id out of range")
+
+    def finalize(self):
+        lib = _load()
+        cent = np.empty((self.n_groups, self.d), dtype=np.float64)
+        lib.htam_oracle_centroid_finalize(_ptr(self.sums), _ptr(self.counts), self.d,
+                                          self.n_groups, _ptr(cent))
+        return cent, self.counts.copy()
+
+
+def centroids(entries: np.ndarray, gid: np.ndarray, n_groups: int):
+    """Group keys c_g = mean of the group's entries (float64), and counts n_g."""
+    acc = CentroidAccumulator(n_groups, entries.shape[1])
+    acc.add(entries, gid)
+    return acc.finalize()
+
+
+def stage1(queries: np.ndarray, centroid: np.ndarray, counts: np.ndarray, k_groups: int,
+           nthreads: int | None = None):
+    """Coarse scores against every non-empty group key and the top-k_g groups."""
+    lib = _load()
+    queries, qdt = _as_input(queries)
+    centroid = np.ascontiguousarray(centroid, dtype=np.float64)
+    counts = np.ascontiguousarray(counts, dtype=np.int64)
+    b, d = queries.shape
+    g = centroid.shape[0]
+    gi = np.empty((b, k_groups), dtype=np.int32)
+    gs = np.empty((b, k_groups), dtype=np.float64)
+    rc = lib.htam_oracle_stage1(_ptr(queries), qdt, b, d, _ptr(centroid), _ptr(counts), g,
+                                int(k_groups), _ptr(gi), _ptr(gs), nthreads or default_threads())
+    if rc != 0:
+        raise RuntimeError(f"oracle stage1 failed ({rc})")
+    return gi, gs
+
+
+def stage2(entries: np.ndarray, gid: np.ndarray, n_groups: int, queries: np.ndarray,
+           groups: np.ndarray, k_entries: int, tau: float = 1.0, eps: float = 0.0,
+           nthreads: int | None = None):
+    """Fine scores over the selected groups' entries, softmax and top-k_e.
+
+    ``groups`` is [B, k_g] int32 (-1 = empty slot): the groups each query
+    selected.  Returns a dict with entry_idx, entry_score, entry_weight, lse and
+    n_cand (the candidate-set size |C_b|).
+    """
+    lib = _load()
+    entries, edt = _as_input(entries)
+    queries, qdt = _as_input(queries)
+    gid = np.ascontiguousarray(gid, dtype=np.int32)
+    groups = np.ascontiguousarray(groups, dtype=np.int32)
+    n, d = entries.shape
+    b = queries.shape[0]
+    kg = groups.shape[1]
+    out = {
+        "entry_idx": np.empty((b, k_entries), dtype=np.int32),
+        "entry_score": np.empty((b, k_entries), dtype=np.float64),
+        "entry_weight": np.empty((b, k_entries), dtype=np.float64),
+        "lse": np.empty(b, dtype=np.float64),
+        "n_cand": np.empty(b, dtype=np.int64),
+    }
+    rc = lib.htam_oracle_stage2(_ptr(entries), edt, _ptr(gid), n, d, int(n_groups), _ptr(queries),
+                                qdt, b, _ptr(groups), kg, int(k_entries), float(tau), float(eps),
+                                _ptr(out["entry_idx"]), _ptr(out["entry_score"]),
+                                _ptr(out["entry_weight"]), _ptr(out["lse"]), _ptr(out["n_cand"]),
+                                nthreads or default_threads())
+    if rc != 0:
+        raise RuntimeError(f"oracle stage2 failed ({rc})")
+    return out
+
+
+def query(entries: np.ndarray, gid: np.ndarray, n_groups: int, queries: np.ndarray,
+          k_groups: int, k_entries: int, tau: float = 1.0, eps: float = 0.0,
+          centroid=None, counts=None, nthreads: int | None = None):
+    """Full two-level lookup: stage 1 then stage 2 on the groups it selected."""
+    if centroid is None or counts is None:
+        centroid, counts = centroids(entries, gid, n_groups)
+    gi, gs = stage1(queries, centroid, counts, k_groups, nthreads)
+    out = stage2(entries, gid, n_groups, queries, gi, k_entries, tau, eps, nthreads)
+    out["group_idx"] = gi
+    out["group_score"] = gs
+    return out

@@ -1,0 +1,324 @@
+/*
+ * htam_oracle.c -- float64 brute-force CPU oracle for HTAM's hierarchical
+ * transition-attended memory lookup (arxiv 2605.29734).
+ *
+ * TEST INFRASTRUCTURE ONLY.  This file is the plain, slow definition that the
+ * CUDA path is checked against.  Only the tests, the package smoke check and
+ * the benchmark's CPU-baseline leg may load it; the product path never does.
+ * It shares no code, header, table or helper with the CUDA library.
+ *
+ * What it computes (one query q, memory of n entries k_e with group ids):
+ *   Memory (Eq. 6, §4.1): global nodes V_G = groups, local nodes V_GL =
+ *     entries, each entry tagged with its parent group par(e) (Eq. 12).
+ *   Group key: c_g = (1/n_g) * sum_{e: par(e)=g} k_e   (mean of its entries;
+ *     the paper leaves the embedding of a global node open, the workload
+ *     definition fixes it as the mean).
+ *   Stage 1 (Eq. 9 with the linear scorer of App. B.6, phi = w^T z; in
+ *     embedding space the linear scorer is the dot product):
+ *       s1[g] = q . c_g for every non-empty g; S = the k_g best groups,
+ *       ordered by score descending, ties to the lower group id.  Empty groups
+ *       (n_g = 0) are never candidates (App. B.7: a direction with no valid
+ *       local node gives no candidate).
+ *   Stage 2 (Eq. 12 restriction, Eq. 13 pick, Eq. 11 policy):
+ *       C = { e : par(e) in S }  (candidate restriction L(g_t)),
+ *       s2[e] = q . k_e for e in C,
+ *       lse = log sum_{e in C} exp(s2[e]/tau),
+ *       w[e] = eps/|C| + (1-eps) * exp(s2[e]/tau - lse)   (the eps-uniform /
+ *         tau-softmax mixture of Eq. 11, normalised over the whole candidate
+ *         set C),
+ *       output: the k_e best e of C by s2 descending, ties to the lower entry
+ *       id, with s2 and w; slots beyond |C| are padded with id -1, score
+ *       -inf, weight 0.
+ *
+ * Everything is double precision, sequential sums in index order, brute force
+ * over the caller's arrays in their original (unsorted) order.  Inputs are
+ * float32 (dtype 0) or bfloat16 bit patterns (dtype 1, uint16), converted
+ * exactly to double.
+ */
+#include <math.h>
+#include <pthread.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+#define ORACLE_F32 0
+#define ORACLE_BF16 1
+
+/* Exact conversion of element idx of an fp32 or bf16 array to double. */
+static double load_elem(const void *base, int dtype, int64_t idx) {
+  if (dtype == ORACLE_F32) {
+    return (double)((const float *)base)[idx];
+  }
+  uint16_t bits = ((const uint16_t *)base)[idx];
+  uint32_t wide = ((uint32_t)bits) << 16;
+  float f;
+  memcpy(&f, &wide, sizeof f);
+  return (double)f;
+}
+
+/* ---------------------------------------------------------------- centroids
+ * Adds every entry of the chunk into sums[gid][:] and counts[gid].  Callers
+ * zero sums/counts first and may feed the entries in several chunks.
+ * Returns 0, or -1 when a group id is outside [0, n_groups). */
+int htam_oracle_centroid_accumulate(const void *entries, int dtype,
+                                    const int32_t *gid, int64_t n, int32_t d,
+                                    int32_t n_groups, double *sums,
+                                    int64_t *counts) {
+  for (int64_t e = 0; e < n; ++e) {
+    int32_t g = gid[e];
+    if (g < 0 || g >= n_groups) return -1;
+    double *row = sums + (int64_t)g * d;
+    for (int32_t j = 0; j < d; ++j) {
+      row[j] += load_elem(entries, dtype, e * (int64_t)d + j);
+    }
+    counts[g] += 1;
+  }
+  return 0;
+}
+
+/* c_g = sums_g / n_g; groups with n_g = 0 are left as NaN (never used). */
+void htam_oracle_centroid_finalize(const double *sums, const int64_t *counts,
+                                   int32_t d, int32_t n_groups,
+                                   double *centroid) {
+  for (int32_t g = 0; g < n_groups; ++g) {
+    for (int32_t j = 0; j < d; ++j) {
+      centroid[(int64_t)g * d + j] =
+          counts[g] > 0 ? sums[(int64_t)g * d + j] / (double)counts[g] : NAN;
+    }
+  }
+}
+
+/* ------------------------------------------------------------- ordering */
+typedef struct {
+  double score;
+  int64_t id;
+} scored_t;
+
+/* Score descending, then id ascending. */
+static int by_score_then_id(const void *pa, const void *pb) {
+  const scored_t *a = (const scored_t *)pa;
+  const scored_t *b = (const scored_t *)pb;
+  if (a->score > b->score) return -1;
+  if (a->score < b->score) return 1;
+  if (a->id < b->id) return -1;
+  if (a->id > b->id) return 1;
+  return 0;
+}
+
+/* ------------------------------------------------------------- stage 1 */
+typedef struct {
+  const void *queries;
+  int q_dtype;
+  int32_t n_queries, d;
+  const double *centroid;
+  const int64_t *counts;
+  int32_t n_groups, k_groups;
+  int32_t *group_idx;
+  double *group_score;
+  int tid, nthreads;
+  int status;
+} stage1_job;
+
+static void *stage1_worker(void *arg) {
+  stage1_job *job = (stage1_job *)arg;
+  scored_t *cand = (scored_t *)malloc(sizeof(scored_t) * (size_t)job->n_groups);
+  if (!cand) {
+    job->status = -2;
+    return NULL;
+  }
+  for (int32_t b = job->tid; b < job->n_queries; b += job->nthreads) {
+    int32_t n_cand = 0;
+    for (int32_t g = 0; g < job->n_groups; ++g) {
+      if (job->counts[g] == 0) continue;
+      double s = 0.0;
+      for (int32_t j = 0; j < job->d; ++j) {
+        s += load_elem(job->queries, job->q_dtype, (int64_t)b * job->d + j) *
+             job->centroid[(int64_t)g * job->d + j];
+      }
+      cand[n_cand].score = s;
+      cand[n_cand].id = g;
+      ++n_cand;
+    }
+    qsort(cand, (size_t)n_cand, sizeof(scored_t), by_score_then_id);
+    for (int32_t j = 0; j < job->k_groups; ++j) {
+      int64_t o = (int64_t)b * job->k_groups + j;
+      if (j < n_cand) {
+        job->group_idx[o] = (int32_t)cand[j].id;
+        job->group_score[o] = cand[j].score;
+      } else {
+        job->group_idx[o] = -1;
+        job->group_score[o] = -INFINITY;
+      }
+    }
+  }
+  free(cand);
+  return NULL;
+}
+
+/* ------------------------------------------------------------- stage 2 */
+typedef struct {
+  const void *entries;
+  int e_dtype;
+  const int32_t *gid;
+  int64_t n;
+  int32_t d, n_groups;
+  const void *queries;
+  int q_dtype;
+  int32_t n_queries;
+  const int32_t *groups; /* [n_queries, k_groups], -1 = unused slot */
+  int32_t k_groups, k_entries;
+  double tau, eps;
+  int32_t *entry_idx;
+  double *entry_score, *entry_weight, *lse;
+  int64_t *n_cand_out;
+  int tid, nthreads;
+  int status;
+} stage2_job;
+
+static void *stage2_worker(void *arg) {
+  stage2_job *job = (stage2_job *)arg;
+  unsigned char *selected = (unsigned char *)malloc((size_t)job->n_groups);
+  scored_t *cand = (scored_t *)malloc(sizeof(scored_t) * (size_t)(job->n > 0 ? job->n : 1));
+  if (!selected || !cand) {
+    free(selected);
+    free(cand);
+    job->status = -2;
+    return NULL;
+  }
+  for (int32_t b = job->tid; b < job->n_queries; b += job->nthreads) {
+    memset(selected, 0, (size_t)job->n_groups);
+    for (int32_t j = 0; j < job->k_groups; ++j) {
+      int32_t g = job->groups[(int64_t)b * job->k_groups + j];
+      if (g >= 0 && g < job->n_groups) selected[g] = 1;
+    }
+    /* Candidate restriction: entries whose parent group was selected. */
+    int64_t n_cand = 0;
+    for (int64_t e = 0; e < job->n; ++e) {
+      if (!selected[job->gid[e]]) continue;
+      double s = 0.0;
+      for (int32_t j = 0; j < job->d; ++j) {
+        s += load_elem(job->queries, job->q_dtype, (int64_t)b * job->d + j) *
+             load_elem(job->entries, job->e_dtype, e * (int64_t)job->d + j);
+      }
+      cand[n_cand].score = s;
+      cand[n_cand].id = e;
+      ++n_cand;
+    }
+    /* Softmax over the whole candidate set, max-shifted. */
+    double lse_b = -INFINITY;
+    if (n_cand > 0) {
+      double m = -INFINITY;
+      for (int64_t i = 0; i < n_cand; ++i) {
+        double z = cand[i].score / job->tau;
+        if (z > m) m = z;
+      }
+      double sum = 0.0;
+      for (int64_t i = 0; i < n_cand; ++i) {
+        sum += exp(cand[i].score / job->tau - m);
+      }
+      lse_b = m + log(sum);
+    }
+    qsort(cand, (size_t)n_cand, sizeof(scored_t), by_score_then_id);
+    for (int32_t j = 0; j < job->k_entries; ++j) {
+      int64_t o = (int64_t)b * job->k_entries + j;
+      if (j < n_cand) {
+        job->entry_idx[o] = (int32_t)cand[j].id;
+        job->entry_score[o] = cand[j].score;
+        job->entry_weight[o] =
+            job->eps / (double)n_cand +
+            (1.0 - job->eps) * exp(cand[j].score / job->tau - lse_b);
+      } else {
+        job->entry_idx[o] = -1;
+        job->entry_score[o] = -INFINITY;
+        job->entry_weight[o] = 0.0;
+      }
+    }
+    job->lse[b] = lse_b;
+    job->n_cand_out[b] = n_cand;
+  }
+  free(selected);
+  free(cand);
+  return NULL;
+}
+
+static int clamp_threads(int nthreads, int32_t n_queries) {
+  if (nthreads < 1) nthreads = 1;
+  if (nthreads > 256) nthreads = 256;
+  if (n_queries > 0 && nthreads > n_queries) nthreads = n_queries;
+  return nthreads;
+}
+
+/* Stage 1 for n_queries queries.  centroid [n_groups, d], counts [n_groups].
+ * Outputs group_idx [n_queries, k_groups] and group_score (same shape).
+ * Returns 0, -1 on bad arguments, -2 on allocation failure. */
+int htam_oracle_stage1(const void *queries, int q_dtype, int32_t n_queries,
+                       int32_t d, const double *centroid,
+                       const int64_t *counts, int32_t n_groups,
+                       int32_t k_groups, int32_t *group_idx,
+                       double *group_score, int nthreads) {
+  if (n_queries < 0 || d <= 0 || n_groups <= 0 || k_groups <= 0) return -1;
+  nthreads = clamp_threads(nthreads, n_queries);
+  stage1_job jobs[256];
+  pthread_t threads[256];
+  for (int t = 0; t < nthreads; ++t) {
+    stage1_job j = {queries, q_dtype, n_queries, d, centroid, counts,
+                    n_groups, k_groups, group_idx, group_score, t, nthreads, 0};
+    jobs[t] = j;
+  }
+  for (int t = 1; t < nthreads; ++t) {
+    if (pthread_create(&threads[t], NULL, stage1_worker, &jobs[t]) != 0) {
+      jobs[t].status = -3;
+    }
+  }
+  stage1_worker(&jobs[0]);
+  int status = jobs[0].status;
+  for (int t = 1; t < nthreads; ++t) {
+    if (jobs[t].status != -3) pthread_join(threads[t], NULL);
+    if (jobs[t].status != 0) status = jobs[t].status;
+  }
+  return status;
+}
+
+/* Stage 2 for n_queries queries given each query's selected groups
+ * (groups [n_queries, k_groups], -1 for unused slots).  Outputs entry_idx,
+ * entry_score, entry_weight [n_queries, k_entries], lse [n_queries] and the
+ * candidate-set size n_cand [n_queries].  Returns 0, -1 on bad arguments
+ * (including a group id outside [0, n_groups)), -2 on allocation failure. */
+int htam_oracle_stage2(const void *entries, int e_dtype, const int32_t *gid,
+                       int64_t n, int32_t d, int32_t n_groups,
+                       const void *queries, int q_dtype, int32_t n_queries,
+                       const int32_t *groups, int32_t k_groups,
+                       int32_t k_entries, double tau, double eps,
+                       int32_t *entry_idx, double *entry_score,
+                       double *entry_weight, double *lse, int64_t *n_cand,
+                       int nthreads) {
+  if (n < 0 || d <= 0 || n_groups <= 0 || n_queries < 0 || k_groups <= 0 ||
+      k_entries <= 0 || !(tau > 0.0) || !(eps >= 0.0 && eps <= 1.0)) {
+    return -1;
+  }
+  for (int64_t e = 0; e < n; ++e) {
+    if (gid[e] < 0 || gid[e] >= n_groups) return -1;
+  }
+  nthreads = clamp_threads(nthreads, n_queries);
+  stage2_job jobs[256];
+  pthread_t threads[256];
+  for (int t = 0; t < nthreads; ++t) {
+    stage2_job j = {entries, e_dtype, gid, n, d, n_groups, queries, q_dtype,
+                    n_queries, groups, k_groups, k_entries, tau, eps,
+                    entry_idx, entry_score, entry_weight, lse, n_cand, t,
+                    nthreads, 0};
+    jobs[t] = j;
+  }
+  for (int t = 1; t < nthreads; ++t) {
+    if (pthread_create(&threads[t], NULL, stage2_worker, &jobs[t]) != 0) {
+      jobs[t].status = -3;
+    }
+  }
+  stage2_worker(&jobs[0]);
+  int status = jobs[0].status;
+  for (int t = 1; t < nthreads; ++t) {
+    if (jobs[t].status != -3) pthread_join(threads[t], NULL);
+    if (jobs[t].status != 0) status = jobs[t].status;
+  }
+  return status;
+}

@@ -1,0 +1,337 @@
+"""Pins for the float64 oracle (CPU only).
+
+Each test ties the oracle to something other than itself: a closed form
+worked out from the equations, a library routine that computes the same
+quantity a different way (numpy matmul / lexsort, scipy logsumexp), an
+invariant the paper's definitions imply, or brute force on a tiny memory.
+Together they are chosen so that a plausible slip (a dropped term, a wrong
+sign, a transposed operand, a missing 1/n, tau multiplied instead of divided,
+a wrong tie order, a leak outside the selected groups) fails at least one.
+"""
+import math
+
+import numpy as np
+import pytest
+from scipy.special import logsumexp
+
+import oracle
+
+
+def _unit_rows(rng, n, d):
+    x = rng.standard_normal((n, d))
+    x /= np.linalg.norm(x, axis=1, keepdims=True)
+    return x.astype(np.float32)
+
+
+def _bf16_bits(x: np.ndarray) -> np.ndarray:
+    """float32 -> bf16 bit pattern with round-to-nearest-even (finite inputs)."""
+    u = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32).astype(np.uint64)
+    rounded = (u + 0x7FFF + ((u >> 16) & 1)) >> 16
+    return rounded.astype(np.uint16)
+
+
+def _bf16_to_f64(bits: np.ndarray) -> np.ndarray:
+    return (bits.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+
+
+# ---------------------------------------------------------------- closed forms
+
+def test_one_hot_memory_by_counting():
+    """Entries are unit axis vectors, so a group key's d-th coordinate is the
+    fraction of its entries on axis d (the mean, c_g = sum/n_g) and a one-hot
+    query e_d scores an entry 1 if it lies on axis d, else 0 (Eq. 9 with the
+    linear scorer).  Every expected number below comes from counting."""
+    d, n_groups = 4, 3
+    gid = np.array([0, 0, 0, 1, 1, 2, 2, 2, 2, 0], dtype=np.int32)
+    axis = np.array([0, 1, 0, 2, 2, 3, 1, 3, 3, 3])
+    entries = np.zeros((gid.size, d), dtype=np.float32)
+    entries[np.arange(gid.size), axis] = 1.0
+    cent, counts = oracle.centroids(entries, gid, n_groups)
+    for g in range(n_groups):
+        members = axis[gid == g]
+        for a in range(d):
+            assert cent[g, a] == np.count_nonzero(members == a) / members.size
+    assert list(counts) == [4, 2, 4]
+
+    for query_axis in range(d):
+        q = np.zeros((1, d), dtype=np.float32)
+        q[0, query_axis] = 1.0
+        frac = [np.count_nonzero(axis[gid == g] == query_axis) / np.count_nonzero(gid == g)
+                for g in range(n_groups)]
+        want_groups = sorted(range(n_groups), key=lambda g: (-frac[g], g))[:2]
+        out = oracle.query(entries, gid, n_groups, q, k_groups=2, k_entries=4, tau=1.0)
+        assert list(out["group_idx"][0]) == want_groups
+        assert list(out["group_score"][0]) == [frac[g] for g in want_groups]
+        cand = [e for e in range(gid.size) if gid[e] in want_groups]
+        hit = [e for e in cand if axis[e] == query_axis]
+        miss = [e for e in cand if axis[e] != query_axis]
+        want_ids = (hit + miss)[:4]          # score 1 before 0, ties to lower id
+        assert list(out["entry_idx"][0]) == want_ids
+        assert list(out["entry_score"][0]) == [1.0 if axis[e] == query_axis else 0.0 for e in want_ids]
+        lse = math.log(len(hit) * math.e + len(miss))
+        assert out["lse"][0] == pytest.approx(lse, rel=0, abs=1e-15)
+        for e, w in zip(want_ids, out["entry_weight"][0]):
+            s = 1.0 if axis[e] == query_axis else 0.0
+            assert w == pytest.approx(math.exp(s - lse), rel=1e-15)
+        assert out["n_cand"][0] == len(cand)
+
+
+@pytest.mark.parametrize("tau,eps", [(0.5, 0.0), (0.5, 0.2), (2.0, 0.7)])
+def test_two_candidates_closed_form(tau, eps):
+    """With two candidates a, b the Eq. 11 mixture is
+    w_a = eps/2 + (1-eps) / (1 + exp((s_b - s_a)/tau))."""
+    entries = np.array([[0.6, 0.8, 0, 0], [1.0, 0, 0, 0], [0, 0, 1.0, 0]], dtype=np.float32)
+    gid = np.array([1, 1, 0], dtype=np.int32)
+    q = np.array([[0.28, 0.96, 0, 0]], dtype=np.float32)
+    out = oracle.query(entries, gid, 2, q, k_groups=1, k_entries=2, tau=tau, eps=eps)
+    assert list(out["group_idx"][0]) == [1]
+    s0 = float(np.dot(entries[0].astype(np.float64), q[0].astype(np.float64)))
+    s1 = float(np.dot(entries[1].astype(np.float64), q[0].astype(np.float64)))
+    assert s0 > s1
+    assert list(out["entry_idx"][0]) == [0, 1]
+    w0 = eps / 2 + (1 - eps) / (1 + math.exp((s1 - s0) / tau))
+    w1 = eps / 2 + (1 - eps) / (1 + math.exp((s0 - s1) / tau))
+    assert out["entry_weight"][0][0] == pytest.approx(w0, rel=1e-14)
+    assert out["entry_weight"][0][1] == pytest.approx(w1, rel=1e-14)
+    assert out["lse"][0] == pytest.approx(math.log(math.exp(s0 / tau) + math.exp(s1 / tau)), rel=1e-14)
+
+
+def test_single_candidate_has_weight_one():
+    entries = np.array([[0.0, 1.0], [1.0, 0.0]], dtype=np.float32)
+    gid = np.array([0, 1], dtype=np.int32)
+    q = np.array([[0.25, 0.75]], dtype=np.float32)
+    out = oracle.query(entries, gid, 2, q, k_groups=1, k_entries=3, tau=0.3, eps=0.5)
+    assert list(out["group_idx"][0]) == [0]
+    assert list(out["entry_idx"][0]) == [0, -1, -1]
+    assert out["entry_weight"][0][0] == pytest.approx(1.0, rel=1e-15)
+    assert out["lse"][0] == pytest.approx(0.75 / 0.3, rel=1e-15)
+    assert list(out["entry_weight"][0][1:]) == [0.0, 0.0]
+    assert np.isneginf(out["entry_score"][0][1:]).all()
+
+
+# ---------------------------------------------------- library-routine special cases
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_all_groups_selected_equals_flat_scan(dtype):
+    """k_groups = G selects every non-empty group, so the two-level lookup is
+    the flat retrieval of App. C.4 / C.8: a full top-k over all entries, which
+    numpy computes independently (matmul + lexsort); lse is scipy's."""
+    rng = np.random.default_rng(11)
+    n, d, g = 300, 24, 7
+    x = _unit_rows(rng, n, d)
+    q32 = _unit_rows(rng, 5, d)
+    gid = rng.integers(0, g, n).astype(np.int32)
+    if dtype == "bf16":
+        entries, queries = _bf16_bits(x), _bf16_bits(q32)
+        e64, q64 = _bf16_to_f64(entries), _bf16_to_f64(queries)
+    else:
+        entries, queries = x, q32
+        e64, q64 = x.astype(np.float64), q32.astype(np.float64)
+    tau = 0.07
+    out = oracle.query(entries, gid, g, queries, k_groups=g, k_entries=40, tau=tau, eps=0.0)
+    scores = q64 @ e64.T
+    for b in range(queries.shape[0]):
+        order = np.lexsort((np.arange(n), -scores[b]))[:40]
+        assert list(out["entry_idx"][b]) == list(order)
+        np.testing.assert_allclose(out["entry_score"][b], scores[b][order], rtol=0, atol=1e-12)
+        assert out["lse"][b] == pytest.approx(logsumexp(scores[b] / tau), rel=1e-12)
+        np.testing.assert_allclose(out["entry_weight"][b], np.exp(scores[b][order] / tau - logsumexp(scores[b] / tau)),
+                                   rtol=1e-11)
+        assert out["n_cand"][b] == n
+
+
+def test_stage1_matches_numpy_brute_force():
+    """Group keys by numpy (bincount means), coarse scores by matmul, top-k by
+    lexsort: an independent computation of centroids + stage 1."""
+    rng = np.random.default_rng(5)
+    n, d, g, kg = 500, 16, 12, 5
+    x = _unit_rows(rng, n, d)
+    gid = rng.integers(0, g, n).astype(np.int32)
+    q = _unit_rows(rng, 9, d)
+    cent, counts = oracle.centroids(x, gid, g)
+    want_counts = np.bincount(gid, minlength=g)
+    assert list(counts) == list(want_counts)
+    want_cent = np.stack([x[gid == j].astype(np.float64).mean(axis=0) for j in range(g)])
+    np.testing.assert_allclose(cent, want_cent, rtol=0, atol=1e-15)
+    gi, gs = oracle.stage1(q, cent, counts, kg)
+    s1 = q.astype(np.float64) @ want_cent.T
+    for b in range(q.shape[0]):
+        order = np.lexsort((np.arange(g), -s1[b]))[:kg]
+        assert list(gi[b]) == list(order)
+        np.testing.assert_allclose(gs[b], s1[b][order], rtol=0, atol=1e-14)
+
+
+def test_two_level_matches_numpy_brute_force():
+    """Whole lookup on a tiny clustered memory against an independent numpy
+    brute force (mask by selected groups, lexsort, logsumexp)."""
+    rng = np.random.default_rng(7)
+    n, d, g, kg, ke = 400, 32, 10, 3, 6
+    centres = rng.standard_normal((g, d))
+    gid = rng.integers(0, g, n).astype(np.int32)
+    x = centres[gid] + 0.3 * rng.standard_normal((n, d))
+    x = (x / np.linalg.norm(x, axis=1, keepdims=True)).astype(np.float32)
+    q = centres[rng.integers(0, g, 6)] + 0.3 * rng.standard_normal((6, d))
+    q = (q / np.linalg.norm(q, axis=1, keepdims=True)).astype(np.float32)
+    tau, eps = 0.25, 0.1
+    out = oracle.query(x, gid, g, q, kg, ke, tau, eps)
+    e64, q64 = x.astype(np.float64), q.astype(np.float64)
+    cent = np.stack([e64[gid == j].mean(axis=0) for j in range(g)])
+    for b in range(q.shape[0]):
+        s1 = cent @ q64[b]
+        sel = np.lexsort((np.arange(g), -s1))[:kg]
+        mask = np.isin(gid, sel)
+        ids = np.nonzero(mask)[0]
+        s2 = e64[ids] @ q64[b]
+        order = np.lexsort((ids, -s2))[:ke]
+        lse = logsumexp(s2 / tau)
+        assert list(out["group_idx"][b]) == list(sel)
+        assert list(out["entry_idx"][b]) == list(ids[order])
+        np.testing.assert_allclose(out["entry_score"][b], s2[order], atol=1e-13, rtol=0)
+        np.testing.assert_allclose(out["entry_weight"][b],
+                                   eps / ids.size + (1 - eps) * np.exp(s2[order] / tau - lse), rtol=1e-11)
+        assert out["lse"][b] == pytest.approx(lse, rel=1e-13)
+
+
+# ------------------------------------------------------------------ invariants
+
+@pytest.mark.parametrize("tau,eps", [(1.0, 0.0), (0.05, 0.0), (1.0, 0.1), (0.3, 1.0)])
+def test_weights_over_full_candidate_set_sum_to_one(tau, eps):
+    rng = np.random.default_rng(3)
+    n, d, g = 200, 8, 6
+    x = _unit_rows(rng, n, d)
+    gid = rng.integers(0, g, n).astype(np.int32)
+    q = _unit_rows(rng, 4, d)
+    out = oracle.query(x, gid, g, q, k_groups=3, k_entries=n, tau=tau, eps=eps)
+    for b in range(4):
+        nb = out["n_cand"][b]
+        w = out["entry_weight"][b][:nb]
+        assert math.fsum(w) == pytest.approx(1.0, abs=1e-12)
+        assert (out["entry_idx"][b][nb:] == -1).all()
+        if eps == 1.0:
+            np.testing.assert_allclose(w, 1.0 / nb, rtol=1e-15)
+
+
+def test_restriction_to_selected_groups():
+    """Eq. 12: every returned entry belongs to a selected group, and the
+    candidate count is the selected groups' total size."""
+    rng = np.random.default_rng(9)
+    n, d, g = 1000, 16, 20
+    x = _unit_rows(rng, n, d)
+    gid = rng.integers(0, g, n).astype(np.int32)
+    q = _unit_rows(rng, 12, d)
+    out = oracle.query(x, gid, g, q, k_groups=4, k_entries=25)
+    counts = np.bincount(gid, minlength=g)
+    for b in range(12):
+        sel = set(out["group_idx"][b])
+        assert all(gid[e] in sel for e in out["entry_idx"][b])
+        assert out["n_cand"][b] == sum(counts[s] for s in sel)
+
+
+def test_entry_permutation_only_relabels():
+    rng = np.random.default_rng(2)
+    n, d, g = 256, 12, 8
+    x = _unit_rows(rng, n, d)
+    gid = rng.integers(0, g, n).astype(np.int32)
+    q = _unit_rows(rng, 5, d)
+    perm = rng.permutation(n)
+    a = oracle.query(x, gid, g, q, 3, 10)
+    b = oracle.query(x[perm], gid[perm], g, q, 3, 10)
+    assert (a["group_idx"] == b["group_idx"]).all()
+    np.testing.assert_array_equal(a["entry_idx"], perm[b["entry_idx"]])
+    np.testing.assert_array_equal(a["entry_score"], b["entry_score"])
+    np.testing.assert_allclose(a["lse"], b["lse"], rtol=1e-14)
+
+
+def test_empty_groups_never_selected_and_padding():
+    rng = np.random.default_rng(4)
+    d, g = 8, 8
+    gid = np.array([0, 2, 3, 4, 6, 7] * 5, dtype=np.int32)  # groups 1 and 5 empty
+    x = _unit_rows(rng, gid.size, d)
+    q = _unit_rows(rng, 3, d)
+    out = oracle.query(x, gid, g, q, k_groups=8, k_entries=gid.size + 5)
+    for b in range(3):
+        assert sorted(out["group_idx"][b][:6]) == [0, 2, 3, 4, 6, 7]
+        assert list(out["group_idx"][b][6:]) == [-1, -1]
+        assert np.isneginf(out["group_score"][b][6:]).all()
+        assert list(out["entry_idx"][b][-5:]) == [-1] * 5
+        assert (out["entry_weight"][b][-5:] == 0).all()
+
+
+def test_ties_go_to_lower_index():
+    d = 4
+    row = np.array([0.5, 0.5, 0.5, 0.5], dtype=np.float32)
+    other = np.array([1.0, 0, 0, 0], dtype=np.float32)
+    # groups 0 and 2 hold identical rows (equal keys and scores), group 1 differs
+    entries = np.stack([row, other, row, row, other, row])
+    gid = np.array([2, 1, 0, 2, 1, 0], dtype=np.int32)
+    q = np.array([[0.5, 0.5, 0.5, 0.5]], dtype=np.float32)
+    out = oracle.query(entries, gid, 3, q, k_groups=2, k_entries=4)
+    assert list(out["group_idx"][0]) == [0, 2]
+    assert out["group_score"][0][0] == out["group_score"][0][1]
+    assert list(out["entry_idx"][0]) == [0, 2, 3, 5]
+
+
+def test_tau_changes_weights_not_ranking():
+    rng = np.random.default_rng(8)
+    x = _unit_rows(rng, 300, 16)
+    gid = rng.integers(0, 6, 300).astype(np.int32)
+    q = _unit_rows(rng, 4, 16)
+    base = oracle.query(x, gid, 6, q, 2, 12, tau=1.0)
+    for tau in (0.05, 20.0):
+        out = oracle.query(x, gid, 6, q, 2, 12, tau=tau)
+        np.testing.assert_array_equal(out["entry_idx"], base["entry_idx"])
+        assert (np.diff(out["entry_weight"], axis=1) <= 0).all()
+    flat = oracle.query(x, gid, 6, q, 2, 12, tau=1e7)
+    for b in range(4):
+        np.testing.assert_allclose(flat["entry_weight"][b], 1.0 / flat["n_cand"][b], rtol=1e-6)
+
+
+def test_query_scale_doubles_scores_exactly():
+    rng = np.random.default_rng(6)
+    x = _unit_rows(rng, 100, 8)
+    gid = rng.integers(0, 4, 100).astype(np.int32)
+    q = _unit_rows(rng, 3, 8)
+    a = oracle.query(x, gid, 4, q, 2, 5)
+    b = oracle.query(x, gid, 4, 2 * q, 2, 5)
+    np.testing.assert_array_equal(b["entry_idx"], a["entry_idx"])
+    np.testing.assert_array_equal(b["entry_score"], 2 * a["entry_score"])
+    np.testing.assert_array_equal(b["group_score"], 2 * a["group_score"])
+
+
+def test_bf16_bits_read_exactly():
+    rng = np.random.default_rng(1)
+    bits = _bf16_bits(_unit_rows(rng, 64, 16))
+    qbits = _bf16_bits(_unit_rows(rng, 2, 16))
+    gid = rng.integers(0, 4, 64).astype(np.int32)
+    a = oracle.query(bits, gid, 4, qbits, 2, 8)
+    b = oracle.query(_bf16_to_f64(bits).astype(np.float32), gid, 4,
+                     _bf16_to_f64(qbits).astype(np.float32), 2, 8)
+    for k in ("group_idx", "entry_idx", "entry_score", "entry_weight", "lse"):
+        np.testing.assert_array_equal(a[k], b[k])
+
+
+def test_centroid_chunks_and_incremental_mean():
+    """Feeding entries in chunks gives the same sums; the mean after an
+    append equals (n_g c_g + sum of new rows) / (n_g + m_g), the in-place
+    update rule the CUDA path uses for Eq. 15."""
+    rng = np.random.default_rng(12)
+    x = _unit_rows(rng, 90, 8)
+    gid = rng.integers(0, 5, 90).astype(np.int32)
+    whole, counts = oracle.centroids(x, gid, 5)
+    acc = oracle.CentroidAccumulator(5, 8)
+    for s in range(0, 90, 40):
+        acc.add(x[s:s + 40], gid[s:s + 40])
+    chunked, counts2 = acc.finalize()
+    np.testing.assert_array_equal(chunked, whole)
+    old, old_n = oracle.centroids(x[:60], gid[:60], 5)
+    new_sum = np.zeros((5, 8))
+    np.add.at(new_sum, gid[60:], x[60:].astype(np.float64))
+    new_n = np.bincount(gid[60:], minlength=5)
+    inc = (old * old_n[:, None] + new_sum) / (old_n + new_n)[:, None]
+    np.testing.assert_allclose(inc, whole, rtol=1e-14, atol=1e-15)
+
+
+def test_bad_group_id_rejected():
+    x = np.zeros((3, 8), dtype=np.float32)
+    with pytest.raises(ValueError):
+        oracle.centroids(x, np.array([0, 5, 1], dtype=np.int32), 3)

@@ -1,0 +1,49 @@
+"""Planted mistakes in the oracle must be caught by its pins (CPU only).
+
+Each case copies the oracle's C source into a temporary directory, plants one
+plausible slip (tau multiplied instead of divided, the eps/|C| term dropped,
+the tie order reversed, the mean not divided by n_g, the ranking sign flipped,
+a transposed operand, a leak of entries outside the selected groups, empty
+groups allowed into stage 1), builds it there and runs ``test_oracle.py``
+against the mutant: at least one pin has to fail.
+"""
+import os
+import shutil
+import subprocess
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+MUTANTS = {
+    "tau_multiplied": ("cand[i].score / job->tau - m", "cand[i].score * job->tau - m"),
+    "eps_term_dropped": ("job->eps / (double)n_cand +", "0.0 +"),
+    "tie_order_reversed": ("if (a->id < b->id) return -1;\n  if (a->id > b->id) return 1;",
+                           "if (a->id < b->id) return 1;\n  if (a->id > b->id) return -1;"),
+    "mean_not_divided": ("sums[(int64_t)g * d + j] / (double)counts[g]", "sums[(int64_t)g * d + j]"),
+    "ranking_sign_flipped": ("if (a->score > b->score) return -1;\n  if (a->score < b->score) return 1;",
+                             "if (a->score < b->score) return -1;\n  if (a->score > b->score) return 1;"),
+    "operand_transposed": ("load_elem(job->entries, job->e_dtype, e * (int64_t)job->d + j)",
+                           "load_elem(job->entries, job->e_dtype, j * (int64_t)job->d + (e % job->d))"),
+    "restriction_leaks": ("if (!selected[job->gid[e]]) continue;",
+                          "if (!selected[job->gid[e]] && e % 7) continue;"),
+    "empty_groups_scored": ("if (job->counts[g] == 0) continue;", ""),
+}
+
+
+@pytest.mark.parametrize("name", sorted(MUTANTS))
+def test_pins_catch_planted_mistake(name, tmp_path):
+    before, after = MUTANTS[name]
+    src = open(os.path.join(ROOT, "oracle", "htam_oracle.c")).read()
+    assert before in src, "mutation site moved; update the mutant"
+    (tmp_path / "oracle").mkdir()
+    (tmp_path / "tests").mkdir()
+    (tmp_path / "oracle" / "htam_oracle.c").write_text(src.replace(before, after))
+    shutil.copy(os.path.join(ROOT, "oracle", "__init__.py"), tmp_path / "oracle" / "__init__.py")
+    shutil.copy(os.path.join(ROOT, "tests", "test_oracle.py"), tmp_path / "tests" / "test_oracle.py")
+    (tmp_path / "pytest.ini").write_text("[pytest]\naddopts = -p no:cacheprovider\n")
+    env = dict(os.environ, PYTHONPATH=str(tmp_path))
+    r = subprocess.run([sys.executable, "-m", "pytest", "-q", "-x", "tests/test_oracle.py"],
+                       cwd=tmp_path, env=env, capture_output=True, text=True, timeout=300)
+    assert r.returncode == 1, f"mutant {name} survived the pins:\n{r.stdout[-2000:]}"
