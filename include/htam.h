@@ -153,6 +153,10 @@ void htam_free_memory(htam_memory *m);
 /* Human-readable name of a status code (static string). */
 const char *htam_status_string(htam_status s);
 
+/* Text of the last failing CUDA call made by this thread ("" if none); the
+ * string stays valid until the thread's next failing call. */
+const char *htam_last_error(void);
+
 /* Diagnostic for the bounded-wait machinery: launches one kernel that waits
  * for a device flag that nothing sets, giving up after `max_iters` polls; the
  * kernel records the give-up in a status word and returns.  Returns ETIMEOUT

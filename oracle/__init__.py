@@ -53,7 +53,7 @@ def _load():
         lib = ctypes.CDLL(build())
         P = ctypes.c_void_p
         i32, i64, dbl = ctypes.c_int32, ctypes.c_int64, ctypes.c_double
-        lib.htam_oracle_centroid_accumulate.argtypes = [P, ctypes.c_int, P, i64, i32, i32, P, P]
+        lib.htam_oracle_centroid_accumulate.argtypes = [P, ctypes.c_int, P, i64, i32, i32, P, P, ctypes.c_int]
         lib.htam_oracle_centroid_accumulate.restype = ctypes.c_int
         lib.htam_oracle_centroid_finalize.argtypes = [P, P, i32, i32, P]
         lib.htam_oracle_centroid_finalize.restype = None
@@ -95,7 +95,7 @@ class CentroidAccumulator:
         self.sums = np.zeros((self.n_groups, self.d), dtype=np.float64)
         self.counts = np.zeros(self.n_groups, dtype=np.int64)
 
-    def add(self, entries: np.ndarray, gid: np.ndarray) -> None:
+    def add(self, entries: np.ndarray, gid: np.ndarray, nthreads: int | None = None) -> None:
         lib = _load()
         entries, dt = _as_input(entries)
         gid = np.ascontiguousarray(gid, dtype=np.int32)
@@ -103,7 +103,8 @@ class CentroidAccumulator:
         if entries.shape != (n, self.d):
             raise ValueError("entries must be [n, d]")
         rc = lib.htam_oracle_centroid_accumulate(_ptr(entries), dt, _ptr(gid), n, self.d,
-                                                 self.n_groups, _ptr(self.sums), _ptr(self.counts))
+                                                 self.n_groups, _ptr(self.sums), _ptr(self.counts),
+                                                 nthreads or default_threads())
         if rc != 0:
             raise ValueError("group id out of range")
 
@@ -115,10 +116,10 @@ class CentroidAccumulator:
         return cent, self.counts.copy()
 
 
-def centroids(entries: np.ndarray, gid: np.ndarray, n_groups: int):
+def centroids(entries: np.ndarray, gid: np.ndarray, n_groups: int, nthreads: int | None = None):
     """Group keys c_g = mean of the group's entries (float64), and counts n_g."""
     acc = CentroidAccumulator(n_groups, entries.shape[1])
-    acc.add(entries, gid)
+    acc.add(entries, gid, nthreads)
     return acc.finalize()
 
 
@@ -179,7 +180,7 @@ def query(entries: np.ndarray, gid: np.ndarray, n_groups: int, queries: np.ndarr
           centroid=None, counts=None, nthreads: int | None = None):
     """Full two-level lookup: stage 1 then stage 2 on the groups it selected."""
     if centroid is None or counts is None:
-        centroid, counts = centroids(entries, gid, n_groups)
+        centroid, counts = centroids(entries, gid, n_groups, nthreads)
     gi, gs = stage1(queries, centroid, counts, k_groups, nthreads)
     out = stage2(entries, gid, n_groups, queries, gi, k_entries, tau, eps, nthreads)
     out["group_idx"] = gi

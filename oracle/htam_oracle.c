@@ -58,21 +58,57 @@ static double load_elem(const void *base, int dtype, int64_t idx) {
 
 /* ---------------------------------------------------------------- centroids
  * Adds every entry of the chunk into sums[gid][:] and counts[gid].  Callers
- * zero sums/counts first and may feed the entries in several chunks.
+ * zero sums/counts first and may feed the entries in several chunks.  Threads
+ * split the coordinates, so each sums[g][j] is still added in entry order.
  * Returns 0, or -1 when a group id is outside [0, n_groups). */
+typedef struct {
+  const void *entries;
+  int dtype;
+  const int32_t *gid;
+  int64_t n;
+  int32_t d, j0, j1;
+  double *sums;
+} centroid_job;
+
+static void *centroid_worker(void *arg) {
+  centroid_job *job = (centroid_job *)arg;
+  for (int64_t e = 0; e < job->n; ++e) {
+    double *row = job->sums + (int64_t)job->gid[e] * job->d;
+    for (int32_t j = job->j0; j < job->j1; ++j) {
+      row[j] += load_elem(job->entries, job->dtype, e * (int64_t)job->d + j);
+    }
+  }
+  return NULL;
+}
+
 int htam_oracle_centroid_accumulate(const void *entries, int dtype,
                                     const int32_t *gid, int64_t n, int32_t d,
                                     int32_t n_groups, double *sums,
-                                    int64_t *counts) {
+                                    int64_t *counts, int nthreads) {
   for (int64_t e = 0; e < n; ++e) {
-    int32_t g = gid[e];
-    if (g < 0 || g >= n_groups) return -1;
-    double *row = sums + (int64_t)g * d;
-    for (int32_t j = 0; j < d; ++j) {
-      row[j] += load_elem(entries, dtype, e * (int64_t)d + j);
-    }
-    counts[g] += 1;
+    if (gid[e] < 0 || gid[e] >= n_groups) return -1;
   }
+  if (nthreads < 1) nthreads = 1;
+  if (nthreads > 256) nthreads = 256;
+  if (nthreads > d) nthreads = d;
+  centroid_job jobs[256];
+  pthread_t threads[256];
+  int started[256];
+  for (int t = 0; t < nthreads; ++t) {
+    centroid_job j = {entries, dtype, gid, n, d, (int32_t)((int64_t)d * t / nthreads),
+                      (int32_t)((int64_t)d * (t + 1) / nthreads), sums};
+    jobs[t] = j;
+    started[t] = 0;
+  }
+  for (int t = 1; t < nthreads; ++t) {
+    started[t] = pthread_create(&threads[t], NULL, centroid_worker, &jobs[t]) == 0;
+    if (!started[t]) centroid_worker(&jobs[t]);
+  }
+  centroid_worker(&jobs[0]);
+  for (int t = 1; t < nthreads; ++t) {
+    if (started[t]) pthread_join(threads[t], NULL);
+  }
+  for (int64_t e = 0; e < n; ++e) counts[gid[e]] += 1;
   return 0;
 }
 

@@ -1,0 +1,218 @@
+// api.cu -- the C ABI declared in include/htam.h: argument checks, status
+// codes, and the bounded-wait self test.  Every argument error is detected
+// here, before anything is launched.
+
+#include <cstdio>
+#include <cstring>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace htam {
+
+static thread_local char g_last_error[256] = "";
+
+void set_last_error(const char *what, cudaError_t err) {
+  std::snprintf(g_last_error, sizeof g_last_error, "%s: %s", what, cudaGetErrorString(err));
+}
+
+static bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// Waits for a flag that nothing sets, giving up after max_iters polls; the
+// give-up is recorded in *status and the kernel returns normally.
+__global__ void wait_timeout_selftest_kernel(const volatile unsigned int *flag, long long max_iters,
+                                             unsigned int *status) {
+  if (threadIdx.x != 0 || blockIdx.x != 0) return;
+  long long it = 0;
+  while (*flag == 0u) {
+    if (++it > max_iters) {
+      atomicOr(status, 1u);
+      return;
+    }
+    __nanosleep(64);
+  }
+}
+
+}  // namespace htam
+
+using namespace htam;
+
+extern "C" {
+
+const char *htam_status_string(htam_status s) {
+  switch (s) {
+    case HTAM_OK: return "HTAM_OK";
+    case HTAM_EINVAL: return "HTAM_EINVAL: invalid argument";
+    case HTAM_ENOMEM: return "HTAM_ENOMEM: allocation failed";
+    case HTAM_ECAPACITY: return "HTAM_ECAPACITY: memory capacity exceeded";
+    case HTAM_ECUDA: return "HTAM_ECUDA: CUDA error";
+    case HTAM_ETIMEOUT: return "HTAM_ETIMEOUT: a device-side wait gave up";
+    case HTAM_ENODEV: return "HTAM_ENODEV: no CUDA device";
+  }
+  return "unknown htam_status";
+}
+
+const char *htam_last_error(void) { return g_last_error; }
+
+static htam_status check_device() {
+  int n = 0;
+  if (cudaGetDeviceCount(&n) != cudaSuccess || n == 0) {
+    cudaGetLastError();
+    return HTAM_ENODEV;
+  }
+  return HTAM_OK;
+}
+
+htam_status htam_build_memory(const void *entries, const int32_t *group_ids, int64_t n, int32_t d,
+                              int32_t n_groups, htam_dtype dtype, int64_t capacity, void *cuda_stream,
+                              htam_memory **out) {
+  if (!out) return HTAM_EINVAL;
+  *out = nullptr;
+  if (dtype != HTAM_F32 && dtype != HTAM_BF16) return HTAM_EINVAL;
+  if (d < 8 || d > 16384 || d % 8 != 0) return HTAM_EINVAL;
+  if (n_groups < 1 || n_groups > 65536) return HTAM_EINVAL;
+  if (n < 0 || capacity < n || capacity < 1 || capacity >= (int64_t(1) << 31) - kPageRows) return HTAM_EINVAL;
+  if (n > 0 && (!entries || !group_ids || !aligned16(entries) || !aligned16(group_ids))) return HTAM_EINVAL;
+  htam_status s = check_device();
+  if (s != HTAM_OK) return s;
+  return build_impl(entries, group_ids, n, d, n_groups, dtype, capacity,
+                    static_cast<cudaStream_t>(cuda_stream), out);
+}
+
+htam_status htam_append_transitions(htam_memory *m, const void *entries, const int32_t *group_ids,
+                                    int64_t count, void *cuda_stream) {
+  if (!m || count < 0) return HTAM_EINVAL;
+  if (count == 0) return HTAM_OK;
+  if (!entries || !group_ids || !aligned16(entries) || !aligned16(group_ids)) return HTAM_EINVAL;
+  if (m->n + count > m->capacity) return HTAM_ECAPACITY;
+  return append_impl(m, entries, group_ids, count, static_cast<cudaStream_t>(cuda_stream));
+}
+
+static htam_status check_query_args(const htam_memory *m, const void *queries, int32_t b,
+                                    const htam_query_params *p, const int32_t *group_idx,
+                                    const float *group_score, const int32_t *entry_idx,
+                                    const float *entry_score, const float *entry_weight) {
+  if (!m || !p || b < 0) return HTAM_EINVAL;
+  if (p->k_groups < 1 || p->k_groups > kMaxK || p->k_groups > m->n_groups) return HTAM_EINVAL;
+  if (p->k_entries < 1 || p->k_entries > kMaxK) return HTAM_EINVAL;
+  if (!(p->tau > 0.0f) || !(p->epsilon >= 0.0f && p->epsilon <= 1.0f)) return HTAM_EINVAL;
+  if (!std::isfinite(1.0f / p->tau)) return HTAM_EINVAL;
+  if (b > (1 << 24)) return HTAM_EINVAL;
+  if (b > 0 && (!queries || !group_idx || !group_score || !entry_idx || !entry_score || !entry_weight)) {
+    return HTAM_EINVAL;
+  }
+  return HTAM_OK;
+}
+
+htam_status htam_query(htam_memory *m, const void *queries, int32_t b, const htam_query_params *p,
+                       int32_t *group_idx, float *group_score, int32_t *entry_idx, float *entry_score,
+                       float *entry_weight, float *lse, void *cuda_stream) {
+  htam_status s = check_query_args(m, queries, b, p, group_idx, group_score, entry_idx, entry_score, entry_weight);
+  if (s != HTAM_OK) return s;
+  if (b > 0 && !aligned16(queries)) return HTAM_EINVAL;
+  return query_impl(m, queries, b, *p, group_idx, group_score, entry_idx, entry_score, entry_weight, lse,
+                    static_cast<cudaStream_t>(cuda_stream));
+}
+
+htam_status htam_query_host(htam_memory *m, const void *queries, int32_t b, const htam_query_params *p,
+                            int32_t *group_idx, float *group_score, int32_t *entry_idx, float *entry_score,
+                            float *entry_weight, float *lse, void *cuda_stream) {
+  htam_status s = check_query_args(m, queries, b, p, group_idx, group_score, entry_idx, entry_score, entry_weight);
+  if (s != HTAM_OK) return s;
+  if (b == 0) return HTAM_OK;
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  const int kg = p->k_groups, ke = p->k_entries;
+  const size_t qbytes = (size_t)b * m->d * m->elem_bytes;
+  const size_t bytes = Carver::round(qbytes) + 2 * Carver::round((size_t)b * kg * 4) +
+                       3 * Carver::round((size_t)b * ke * 4) + Carver::round((size_t)b * 4) + 1024;
+  if (bytes > m->stage_bytes) {
+    if (m->stage) cudaFree(m->stage);
+    m->stage = nullptr;
+    m->stage_bytes = 0;
+    if (cudaMalloc(&m->stage, bytes) != cudaSuccess) {
+      cudaGetLastError();
+      return HTAM_ENOMEM;
+    }
+    m->stage_bytes = bytes;
+  }
+  Carver cv(m->stage);
+  void *dq = cv.take<char>(qbytes);
+  int32_t *dgi = cv.take<int32_t>((size_t)b * kg);
+  float *dgs = cv.take<float>((size_t)b * kg);
+  int32_t *dei = cv.take<int32_t>((size_t)b * ke);
+  float *des = cv.take<float>((size_t)b * ke);
+  float *dew = cv.take<float>((size_t)b * ke);
+  float *dl = cv.take<float>((size_t)b);
+  HTAM_CK(cudaMemcpyAsync(dq, queries, qbytes, cudaMemcpyHostToDevice, st));
+  s = query_impl(m, dq, b, *p, dgi, dgs, dei, des, dew, lse ? dl : nullptr, st);
+  if (s != HTAM_OK) return s;
+  HTAM_CK(cudaMemcpyAsync(group_idx, dgi, (size_t)b * kg * 4, cudaMemcpyDeviceToHost, st));
+  HTAM_CK(cudaMemcpyAsync(group_score, dgs, (size_t)b * kg * 4, cudaMemcpyDeviceToHost, st));
+  HTAM_CK(cudaMemcpyAsync(entry_idx, dei, (size_t)b * ke * 4, cudaMemcpyDeviceToHost, st));
+  HTAM_CK(cudaMemcpyAsync(entry_score, des, (size_t)b * ke * 4, cudaMemcpyDeviceToHost, st));
+  HTAM_CK(cudaMemcpyAsync(entry_weight, dew, (size_t)b * ke * 4, cudaMemcpyDeviceToHost, st));
+  if (lse) HTAM_CK(cudaMemcpyAsync(lse, dl, (size_t)b * 4, cudaMemcpyDeviceToHost, st));
+  HTAM_CK(cudaStreamSynchronize(st));
+  return HTAM_OK;
+}
+
+htam_status htam_memory_info(const htam_memory *m, int64_t *n, int32_t *d, int32_t *n_groups,
+                             int64_t *capacity) {
+  if (!m) return HTAM_EINVAL;
+  if (n) *n = m->n;
+  if (d) *d = m->d;
+  if (n_groups) *n_groups = m->n_groups;
+  if (capacity) *capacity = m->capacity;
+  return HTAM_OK;
+}
+
+htam_status htam_memory_group_counts(const htam_memory *m, int64_t *counts) {
+  if (!m || !counts) return HTAM_EINVAL;
+  std::memcpy(counts, m->h_count.data(), sizeof(int64_t) * m->n_groups);
+  return HTAM_OK;
+}
+
+htam_status htam_memory_group_keys(const htam_memory *m, float *keys, void *cuda_stream) {
+  if (!m || !keys) return HTAM_EINVAL;
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  HTAM_CK(cudaMemcpyAsync(keys, m->cent, sizeof(float) * (size_t)m->n_groups * m->d, cudaMemcpyDeviceToHost, st));
+  HTAM_CK(cudaStreamSynchronize(st));
+  return HTAM_OK;
+}
+
+htam_status htam_device_status(htam_memory *m, void *cuda_stream) {
+  if (!m) return HTAM_EINVAL;
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  unsigned int word = 0;
+  HTAM_CK(cudaMemcpyAsync(&word, m->status, sizeof word, cudaMemcpyDeviceToHost, st));
+  HTAM_CK(cudaMemsetAsync(m->status, 0, sizeof(unsigned int), st));
+  HTAM_CK(cudaStreamSynchronize(st));
+  return word ? HTAM_ETIMEOUT : HTAM_OK;
+}
+
+void htam_free_memory(htam_memory *m) { free_impl(m); }
+
+htam_status htam_selftest_wait_timeout(int64_t max_iters, void *cuda_stream) {
+  htam_status s = check_device();
+  if (s != HTAM_OK) return s;
+  if (max_iters < 0) return HTAM_EINVAL;
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  unsigned int *buf = nullptr;  // [0] flag nobody sets, [1] status
+  HTAM_CK(cudaMalloc(&buf, 2 * sizeof(unsigned int)));
+  unsigned int host[2] = {0, 0};
+  cudaError_t e = cudaMemsetAsync(buf, 0, 2 * sizeof(unsigned int), st);
+  if (e == cudaSuccess) {
+    wait_timeout_selftest_kernel<<<1, 32, 0, st>>>(buf, (long long)max_iters, buf + 1);
+    e = cudaGetLastError();
+  }
+  if (e == cudaSuccess) e = cudaMemcpyAsync(host, buf, sizeof host, cudaMemcpyDeviceToHost, st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  cudaFree(buf);
+  if (e != cudaSuccess) {
+    set_last_error("htam_selftest_wait_timeout", e);
+    return HTAM_ECUDA;
+  }
+  return host[1] ? HTAM_ETIMEOUT : HTAM_OK;
+}
+
+}  // extern "C"

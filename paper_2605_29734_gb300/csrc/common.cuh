@@ -1,0 +1,119 @@
+// common.cuh -- shared device/host helpers of the HTAM lookup library.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <climits>
+#include <cmath>
+
+#include "htam.h"
+
+namespace htam {
+
+constexpr int kPageRows = 128;       // entry rows per storage page
+constexpr unsigned kFullMask = 0xffffffffu;
+constexpr int kMaxK = 64;            // largest k_groups / k_entries
+
+// Records the failing call for htam_last_error-style diagnostics.
+void set_last_error(const char *what, cudaError_t err);
+
+#define HTAM_CK(call)                                   \
+  do {                                                  \
+    cudaError_t err__ = (call);                         \
+    if (err__ != cudaSuccess) {                         \
+      ::htam::set_last_error(#call, err__);             \
+      return HTAM_ECUDA;                                \
+    }                                                   \
+  } while (0)
+
+#define HTAM_CK_LAUNCH(what)                            \
+  do {                                                  \
+    cudaError_t err__ = cudaGetLastError();             \
+    if (err__ != cudaSuccess) {                         \
+      ::htam::set_last_error(what, err__);              \
+      return HTAM_ECUDA;                                \
+    }                                                   \
+  } while (0)
+
+// ------------------------------------------------------------ element access
+__device__ __forceinline__ float to_f32(float x) { return x; }
+__device__ __forceinline__ float to_f32(__nv_bfloat16 x) { return __bfloat162float(x); }
+
+// Low / high bf16 halves of a 32-bit word as fp32 (exact: a bf16 is the top
+// 16 bits of the fp32 with the same value).
+__device__ __forceinline__ float bf16lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
+
+// ------------------------------------------------------------ ordering
+// Score descending, then id ascending (the tie rule of both levels).
+__device__ __forceinline__ bool better(float a, int ia, float b, int ib) {
+  return a > b || (a == b && ia < ib);
+}
+
+// A sorted list of up to 64 (score, id) pairs spread over one warp: lane l
+// holds positions l (half 0) and l + 32 (half 1).  Empty slots hold
+// (-inf, INT_MAX), worse than any real candidate.
+struct WarpList {
+  float s0, s1;
+  int i0, i1;
+
+  __device__ __forceinline__ void init() {
+    s0 = s1 = -INFINITY;
+    i0 = i1 = INT_MAX;
+  }
+
+  // The element at position k-1 (the admission threshold), broadcast.
+  __device__ __forceinline__ void kth(int k, float &ts, int &ti) const {
+    int pos = k - 1;
+    int src = pos & 31;
+    float a = __shfl_sync(kFullMask, pos < 32 ? s0 : s1, src);
+    int b = __shfl_sync(kFullMask, pos < 32 ? i0 : i1, src);
+    ts = a;
+    ti = b;
+  }
+
+  // Inserts a warp-uniform candidate, keeping the 64 slots sorted.  All
+  // lanes must call it with the same (s, id).
+  __device__ __forceinline__ void insert(int k, float s, int id) {
+    const int lane = threadIdx.x & 31;
+    int p = __popc(__ballot_sync(kFullMask, better(s0, i0, s, id)));
+    if (k > 32) p += __popc(__ballot_sync(kFullMask, better(s1, i1, s, id)));
+    if (p >= k) return;
+    float s0u = __shfl_up_sync(kFullMask, s0, 1);
+    int i0u = __shfl_up_sync(kFullMask, i0, 1);
+    float s1u = __shfl_up_sync(kFullMask, s1, 1);
+    int i1u = __shfl_up_sync(kFullMask, i1, 1);
+    float s31 = __shfl_sync(kFullMask, s0, 31);
+    int i31 = __shfl_sync(kFullMask, i0, 31);
+    if (lane == 0) {
+      s1u = s31;
+      i1u = i31;
+    }
+    if (lane > p) {
+      s0 = s0u;
+      i0 = i0u;
+    } else if (lane == p) {
+      s0 = s;
+      i0 = id;
+    }
+    if (lane + 32 > p) {
+      s1 = s1u;
+      i1 = i1u;
+    } else if (lane + 32 == p) {
+      s1 = s;
+      i1 = id;
+    }
+  }
+};
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(kFullMask, v, o);
+  return v;
+}
+
+__host__ __device__ inline int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
+
+}  // namespace htam

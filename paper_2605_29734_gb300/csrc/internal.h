@@ -1,0 +1,87 @@
+// internal.h -- the memory object behind the opaque htam_memory handle.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <vector>
+
+#include "htam.h"
+
+struct htam_memory {
+  int device = 0;
+  int sm_count = 0;
+  int32_t d = 0;
+  int32_t n_groups = 0;
+  htam_dtype dtype = HTAM_BF16;
+  int elem_bytes = 2;
+  int64_t n = 0;           // entries stored
+  int64_t capacity = 0;    // most entries ever stored
+  int64_t n_pages_max = 0; // pages reserved: ceil(capacity/128) + n_groups
+  int64_t n_pages_used = 0;
+
+  // Paged storage: page p holds rows [p*128, p*128+128) of `pool`; each row
+  // is d elements of dtype.  Group g owns pages page_list[page_off[g] ..
+  // page_off[g+1]) in order, filled front to back; its i-th entry sits in
+  // page page_list[page_off[g] + i/128], row i%128.
+  void *pool = nullptr;
+  int32_t *slot_id = nullptr;    // [n_pages_max*128] entry id of each row, -1 if empty
+  int32_t *page_list = nullptr;  // [n_pages_max]
+  int32_t *page_off = nullptr;   // [n_groups+1]
+  int32_t *count = nullptr;      // [n_groups] entries per group (device copy)
+
+  // Group keys: fp64 running sums (exact enough to update in place), the
+  // fp32 mean, and the mean split into bf16 hi + lo parts.
+  double *csum = nullptr;           // [n_groups*d]
+  float *cent = nullptr;            // [n_groups*d]
+  __nv_bfloat16 *cent_hi = nullptr; // [n_groups*d]
+  __nv_bfloat16 *cent_lo = nullptr; // [n_groups*d]
+
+  unsigned int *status = nullptr;   // device status word (bit 0: a wait gave up)
+
+  // Host mirrors of the layout.
+  std::vector<int64_t> h_count;
+  std::vector<std::vector<int32_t>> h_pages;
+
+  // Scratch owned by the object, grown on demand (never shrinks).
+  void *scratch = nullptr;
+  size_t scratch_bytes = 0;
+  // Device staging for htam_query_host.
+  void *stage = nullptr;
+  size_t stage_bytes = 0;
+};
+
+namespace htam {
+
+// Grows m->scratch to at least `bytes` (synchronising the device when it has
+// to reallocate).  Returns HTAM_OK / HTAM_ENOMEM.
+htam_status ensure_scratch(htam_memory *m, size_t bytes);
+
+// Bump allocator over a scratch buffer (256-byte aligned pieces).
+struct Carver {
+  char *base;
+  size_t off = 0;
+  explicit Carver(void *b) : base(static_cast<char *>(b)) {}
+  template <typename T>
+  T *take(size_t count) {
+    off = (off + 255) & ~size_t(255);
+    T *p = reinterpret_cast<T *>(base + off);
+    off += count * sizeof(T);
+    return p;
+  }
+  static size_t round(size_t bytes) { return (bytes + 255) & ~size_t(255); }
+};
+
+htam_status build_impl(const void *entries, const int32_t *group_ids, int64_t n, int32_t d,
+                       int32_t n_groups, htam_dtype dtype, int64_t capacity, cudaStream_t st,
+                       htam_memory **out);
+htam_status append_impl(htam_memory *m, const void *entries, const int32_t *group_ids,
+                        int64_t count, cudaStream_t st);
+htam_status query_impl(htam_memory *m, const void *queries, int32_t b,
+                       const htam_query_params &p, int32_t *group_idx, float *group_score,
+                       int32_t *entry_idx, float *entry_score, float *entry_weight, float *lse,
+                       cudaStream_t st);
+void free_impl(htam_memory *m);
+
+}  // namespace htam

@@ -1,0 +1,423 @@
+// memory.cu -- building and appending to the paged group memory.
+//
+// The memory mirrors the paper's Hierarchical Transition Graph (Eq. 6, §4.1):
+// entries (local nodes) are filed under their parent group (global node), and
+// each group keeps a key equal to the mean of its entries.  Appending is the
+// memory update of Eq. 15: new rows go to the tail of their group's pages and
+// the touched groups' keys are updated in place from fp64 running sums.
+//
+// Every step is deterministic: rows are placed by a stable counting sort (the
+// i-th row of a group in input order lands at the group's next free slot), and
+// key sums are taken over rows in slot order, in fixed-size row segments whose
+// fp32 partials are added to the fp64 sum in segment order.
+
+#include <algorithm>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <vector>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace htam {
+
+namespace {
+
+constexpr int kKeySegRows = 1024;  // rows per key partial-sum segment
+
+__global__ void count_groups_kernel(const int32_t *__restrict__ gid, int64_t n, int32_t n_groups,
+                                    int32_t *__restrict__ counts, int32_t *__restrict__ bad) {
+  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < n;
+       e += (int64_t)gridDim.x * blockDim.x) {
+    int32_t g = gid[e];
+    if (g < 0 || g >= n_groups) {
+      atomicOr(bad, 1);
+    } else {
+      atomicAdd(&counts[g], 1);
+    }
+  }
+}
+
+// hist[g * n_chunks + c] = number of rows of group g in chunk c.
+__global__ void chunk_hist_kernel(const int32_t *__restrict__ gid, int64_t n, int64_t chunk,
+                                  int64_t n_chunks, int32_t *__restrict__ hist) {
+  int64_t c = blockIdx.x;
+  int64_t lo = c * chunk, hi = min(n, lo + chunk);
+  for (int64_t e = lo + threadIdx.x; e < hi; e += blockDim.x) {
+    atomicAdd(&hist[(int64_t)gid[e] * n_chunks + c], 1);
+  }
+}
+
+// Per group (one warp each): hist[g][c] <- base[g] + sum_{c' < c} hist[g][c'].
+__global__ void chunk_scan_kernel(int32_t *__restrict__ hist, int64_t n_chunks, int32_t n_groups,
+                                  const int32_t *__restrict__ base) {
+  int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  int lane = threadIdx.x & 31;
+  if (warp >= n_groups) return;
+  int32_t *row = hist + (int64_t)warp * n_chunks;
+  int32_t running = base[warp];
+  for (int64_t c0 = 0; c0 < n_chunks; c0 += 32) {
+    int64_t c = c0 + lane;
+    int32_t v = c < n_chunks ? row[c] : 0;
+    int32_t incl = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      int32_t t = __shfl_up_sync(kFullMask, incl, o);
+      if (lane >= o) incl += t;
+    }
+    if (c < n_chunks) row[c] = running + incl - v;
+    running += __shfl_sync(kFullMask, incl, 31);
+  }
+}
+
+// One warp per chunk walks its rows in order; rows of the same group take
+// consecutive slots (stable), so pos[e] = slot of row e within its group.
+__global__ void chunk_place_kernel(const int32_t *__restrict__ gid, int64_t n, int64_t chunk,
+                                   int64_t n_chunks, int32_t *__restrict__ hist,
+                                   int32_t *__restrict__ pos) {
+  int64_t c = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+  int lane = threadIdx.x & 31;
+  if (c >= n_chunks) return;
+  int64_t lo = c * chunk, hi = min(n, lo + chunk);
+  unsigned lt = (1u << lane) - 1u;
+  for (int64_t b0 = lo; b0 < hi; b0 += 32) {
+    int64_t e = b0 + lane;
+    unsigned act = __ballot_sync(kFullMask, e < hi);
+    if (e < hi) {
+      int32_t g = gid[e];
+      unsigned peers = __match_any_sync(act, g);
+      int leader = __ffs(peers) - 1;
+      int rank = __popc(peers & lt);
+      int32_t old = 0;
+      int32_t *slot = &hist[(int64_t)g * n_chunks + c];
+      if (lane == leader) {
+        old = *slot;
+        *slot = old + __popc(peers);
+      }
+      old = __shfl_sync(act, old, leader);
+      pos[e] = old + rank;
+    }
+    __syncwarp();
+  }
+}
+
+// One warp per row: copy into its page slot, record its entry id.
+__global__ void place_rows_kernel(const uint4 *__restrict__ src, const int32_t *__restrict__ gid,
+                                  const int32_t *__restrict__ pos, int64_t n, int vec_per_row,
+                                  const int32_t *__restrict__ page_list,
+                                  const int32_t *__restrict__ page_off, uint4 *__restrict__ pool,
+                                  int32_t *__restrict__ slot_id, int64_t id_base) {
+  int64_t e = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+  int lane = threadIdx.x & 31;
+  if (e >= n) return;
+  int32_t g = gid[e];
+  int32_t p = pos[e];
+  int64_t page = page_list[page_off[g] + p / kPageRows];
+  int64_t slot = page * kPageRows + (p % kPageRows);
+  const uint4 *s = src + e * vec_per_row;
+  uint4 *dst = pool + slot * vec_per_row;
+  for (int v = lane; v < vec_per_row; v += 32) dst[v] = s[v];
+  if (lane == 0) slot_id[slot] = (int32_t)(id_base + e);
+}
+
+struct KeySeg {
+  int32_t g, r0, r1, pad;
+};
+struct KeyGroup {
+  int32_t g, seg0, seg1, count;
+};
+
+// partial[s][j] = sum over rows r0..r1-1 of group g of row[j] (fp32).
+template <typename T>
+__global__ void key_partial_kernel(const T *__restrict__ pool, int32_t d,
+                                   const int32_t *__restrict__ page_list,
+                                   const int32_t *__restrict__ page_off,
+                                   const KeySeg *__restrict__ segs, float *__restrict__ partial) {
+  KeySeg sg = segs[blockIdx.x];
+  int j0 = (blockIdx.y * blockDim.x + threadIdx.x) * 8;
+  if (j0 >= d) return;
+  float acc[8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) acc[i] = 0.f;
+  const int32_t *pages = page_list + page_off[sg.g];
+  for (int r = sg.r0; r < sg.r1; ++r) {
+    int64_t slot = (int64_t)pages[r / kPageRows] * kPageRows + (r % kPageRows);
+    const T *row = pool + slot * d + j0;
+    if constexpr (sizeof(T) == 2) {
+      uint4 v = *reinterpret_cast<const uint4 *>(row);
+      acc[0] += bf16lo(v.x); acc[1] += bf16hi(v.x);
+      acc[2] += bf16lo(v.y); acc[3] += bf16hi(v.y);
+      acc[4] += bf16lo(v.z); acc[5] += bf16hi(v.z);
+      acc[6] += bf16lo(v.w); acc[7] += bf16hi(v.w);
+    } else {
+      float4 a = *reinterpret_cast<const float4 *>(row);
+      float4 b = *reinterpret_cast<const float4 *>(row + 4);
+      acc[0] += a.x; acc[1] += a.y; acc[2] += a.z; acc[3] += a.w;
+      acc[4] += b.x; acc[5] += b.y; acc[6] += b.z; acc[7] += b.w;
+    }
+  }
+  float *out = partial + (int64_t)blockIdx.x * d + j0;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) out[i] = acc[i];
+}
+
+// csum[g] += partials in segment order; refresh the fp32 mean and its bf16
+// hi/lo split for the group.
+__global__ void key_finalize_kernel(const KeyGroup *__restrict__ groups,
+                                    const float *__restrict__ partial, int32_t d,
+                                    double *__restrict__ csum, float *__restrict__ cent,
+                                    __nv_bfloat16 *__restrict__ hi, __nv_bfloat16 *__restrict__ lo) {
+  KeyGroup kg = groups[blockIdx.x];
+  for (int j = blockIdx.y * blockDim.x + threadIdx.x; j < d; j += gridDim.y * blockDim.x) {
+    double add = 0.0;
+    for (int s = kg.seg0; s < kg.seg1; ++s) add += (double)partial[(int64_t)s * d + j];
+    int64_t o = (int64_t)kg.g * d + j;
+    double sum = csum[o] + add;
+    csum[o] = sum;
+    double mean = kg.count > 0 ? sum / (double)kg.count : 0.0;
+    cent[o] = (float)mean;
+    __nv_bfloat16 h = __double2bfloat16(mean);
+    hi[o] = h;
+    lo[o] = __double2bfloat16(mean - (double)__bfloat162float(h));
+  }
+}
+
+}  // namespace
+
+htam_status ensure_scratch(htam_memory *m, size_t bytes) {
+  if (bytes <= m->scratch_bytes) return HTAM_OK;
+  if (m->scratch) {
+    cudaFree(m->scratch);  // implicit device synchronisation: no queued work still uses it
+    m->scratch = nullptr;
+    m->scratch_bytes = 0;
+  }
+  size_t want = std::max(bytes, size_t(1) << 20);
+  if (cudaMalloc(&m->scratch, want) != cudaSuccess) {
+    cudaGetLastError();
+    m->scratch = nullptr;
+    return HTAM_ENOMEM;
+  }
+  m->scratch_bytes = want;
+  return HTAM_OK;
+}
+
+// Files `count` rows (ids id_base..) under their groups and updates the keys
+// of the groups they join.  Arguments are already validated except the group
+// id range, which is checked on the device before anything is written.
+static htam_status add_rows(htam_memory *m, const void *entries, const int32_t *gid, int64_t count,
+                            cudaStream_t st) {
+  if (count == 0) return HTAM_OK;
+  const int32_t G = m->n_groups, d = m->d;
+
+  // Chunking of the stable sort: at most ~16M (group, chunk) counters.
+  int64_t chunk = std::max<int64_t>(256, ceil_div((int64_t)count * G, int64_t(1) << 24));
+  chunk = ceil_div(chunk, 32) * 32;
+  int64_t n_chunks = ceil_div(count, chunk);
+
+  // Key segments need the final layout; their number is bounded by
+  // count/kKeySegRows + number of groups.
+  int64_t max_segs = count / kKeySegRows + G + 1;
+
+  size_t need = Carver::round(sizeof(int32_t) * (G + 1)) + Carver::round(sizeof(int32_t) * count) +
+                Carver::round(sizeof(int32_t) * (size_t)G * n_chunks) +
+                Carver::round(sizeof(KeySeg) * max_segs) + Carver::round(sizeof(KeyGroup) * G) +
+                Carver::round(sizeof(float) * (size_t)max_segs * d) + 4096;
+  htam_status s = ensure_scratch(m, need);
+  if (s != HTAM_OK) return s;
+  Carver cv(m->scratch);
+  int32_t *bcount = cv.take<int32_t>(G + 1);  // [G] counts + [1] bad flag
+  int32_t *pos = cv.take<int32_t>(count);
+  int32_t *hist = cv.take<int32_t>((size_t)G * n_chunks);
+  KeySeg *segs = cv.take<KeySeg>(max_segs);
+  KeyGroup *kgroups = cv.take<KeyGroup>(G);
+  float *partial = cv.take<float>((size_t)max_segs * d);
+
+  // 1. Per-group counts of the batch and the group-id range check.
+  HTAM_CK(cudaMemsetAsync(bcount, 0, sizeof(int32_t) * (G + 1), st));
+  {
+    int blocks = (int)std::min<int64_t>(ceil_div(count, 256), 4096);
+    count_groups_kernel<<<blocks, 256, 0, st>>>(gid, count, G, bcount, bcount + G);
+    HTAM_CK_LAUNCH("count_groups_kernel");
+  }
+  std::vector<int32_t> h_b(G + 1);
+  HTAM_CK(cudaMemcpyAsync(h_b.data(), bcount, sizeof(int32_t) * (G + 1), cudaMemcpyDeviceToHost, st));
+  HTAM_CK(cudaStreamSynchronize(st));
+  if (h_b[G] != 0) return HTAM_EINVAL;
+
+  // 2. Page layout on the host.
+  std::vector<int64_t> new_count(G);
+  int64_t new_pages = 0;
+  for (int32_t g = 0; g < G; ++g) {
+    new_count[g] = m->h_count[g] + h_b[g];
+    new_pages += ceil_div(new_count[g], kPageRows) - ceil_div(m->h_count[g], kPageRows);
+  }
+  if (m->n + count > m->capacity || m->n_pages_used + new_pages > m->n_pages_max) {
+    return HTAM_ECAPACITY;
+  }
+  std::vector<std::vector<int32_t>> pages = m->h_pages;
+  int64_t next_page = m->n_pages_used;
+  std::vector<int32_t> h_off(G + 1), h_list;
+  h_list.reserve((size_t)(m->n_pages_used + new_pages));
+  for (int32_t g = 0; g < G; ++g) {
+    int64_t want = ceil_div(new_count[g], kPageRows);
+    while ((int64_t)pages[g].size() < want) pages[g].push_back((int32_t)next_page++);
+    h_off[g] = (int32_t)h_list.size();
+    h_list.insert(h_list.end(), pages[g].begin(), pages[g].end());
+  }
+  h_off[G] = (int32_t)h_list.size();
+
+  // Key segments over the new rows of every touched group.
+  std::vector<KeySeg> h_segs;
+  std::vector<KeyGroup> h_kg;
+  for (int32_t g = 0; g < G; ++g) {
+    if (h_b[g] == 0) continue;
+    KeyGroup kg{g, (int32_t)h_segs.size(), 0, (int32_t)new_count[g]};
+    for (int64_t r = m->h_count[g]; r < new_count[g]; r += kKeySegRows) {
+      h_segs.push_back(KeySeg{g, (int32_t)r, (int32_t)std::min<int64_t>(new_count[g], r + kKeySegRows), 0});
+    }
+    kg.seg1 = (int32_t)h_segs.size();
+    h_kg.push_back(kg);
+  }
+
+  // From here on the memory is modified.  Upload the layout (stream
+  // ordered after any earlier query on this stream).
+  HTAM_CK(cudaMemcpyAsync(m->page_off, h_off.data(), sizeof(int32_t) * (G + 1), cudaMemcpyHostToDevice, st));
+  if (!h_list.empty()) {
+    HTAM_CK(cudaMemcpyAsync(m->page_list, h_list.data(), sizeof(int32_t) * h_list.size(),
+                            cudaMemcpyHostToDevice, st));
+  }
+  HTAM_CK(cudaMemcpyAsync(segs, h_segs.data(), sizeof(KeySeg) * h_segs.size(), cudaMemcpyHostToDevice, st));
+  HTAM_CK(cudaMemcpyAsync(kgroups, h_kg.data(), sizeof(KeyGroup) * h_kg.size(), cudaMemcpyHostToDevice, st));
+
+  // 3. Stable slot assignment: pos[e] = old count of its group + rank among
+  //    earlier rows of the batch with the same group.
+  HTAM_CK(cudaMemsetAsync(hist, 0, sizeof(int32_t) * (size_t)G * n_chunks, st));
+  chunk_hist_kernel<<<(unsigned)n_chunks, 256, 0, st>>>(gid, count, chunk, n_chunks, hist);
+  HTAM_CK_LAUNCH("chunk_hist_kernel");
+  chunk_scan_kernel<<<(unsigned)ceil_div((int64_t)G * 32, 256), 256, 0, st>>>(hist, n_chunks, G, m->count);
+  HTAM_CK_LAUNCH("chunk_scan_kernel");
+  chunk_place_kernel<<<(unsigned)ceil_div(n_chunks * 32, 256), 256, 0, st>>>(gid, count, chunk, n_chunks, hist, pos);
+  HTAM_CK_LAUNCH("chunk_place_kernel");
+
+  // 4. Copy rows into their slots.
+  int vec_per_row = d * m->elem_bytes / 16;
+  place_rows_kernel<<<(unsigned)ceil_div(count * 32, 256), 256, 0, st>>>(
+      static_cast<const uint4 *>(entries), gid, pos, count, vec_per_row, m->page_list, m->page_off,
+      static_cast<uint4 *>(m->pool), m->slot_id, m->n);
+  HTAM_CK_LAUNCH("place_rows_kernel");
+
+  // 5. Keys of the touched groups.
+  if (!h_segs.empty()) {
+    dim3 grid((unsigned)h_segs.size(), (unsigned)ceil_div(d, 256 * 8));
+    if (m->dtype == HTAM_BF16) {
+      key_partial_kernel<__nv_bfloat16><<<grid, 256, 0, st>>>(
+          static_cast<const __nv_bfloat16 *>(m->pool), d, m->page_list, m->page_off, segs, partial);
+    } else {
+      key_partial_kernel<float><<<grid, 256, 0, st>>>(static_cast<const float *>(m->pool), d,
+                                                      m->page_list, m->page_off, segs, partial);
+    }
+    HTAM_CK_LAUNCH("key_partial_kernel");
+    dim3 g2((unsigned)h_kg.size(), (unsigned)std::min<int64_t>(ceil_div(d, 256), 16));
+    key_finalize_kernel<<<g2, 256, 0, st>>>(kgroups, partial, d, m->csum, m->cent, m->cent_hi, m->cent_lo);
+    HTAM_CK_LAUNCH("key_finalize_kernel");
+  }
+
+  // 6. New device counts and host mirrors.
+  std::vector<int32_t> h_c32(G);
+  for (int32_t g = 0; g < G; ++g) h_c32[g] = (int32_t)new_count[g];
+  HTAM_CK(cudaMemcpyAsync(m->count, h_c32.data(), sizeof(int32_t) * G, cudaMemcpyHostToDevice, st));
+  // The host vectors above are pageable: cudaMemcpyAsync has staged them
+  // before returning, but the key/segment tables live in scratch that the
+  // next call may reuse, so finish the queued work before returning.
+  HTAM_CK(cudaStreamSynchronize(st));
+  m->h_count.swap(new_count);
+  m->h_pages.swap(pages);
+  m->n_pages_used = next_page;
+  m->n += count;
+  return HTAM_OK;
+}
+
+void free_impl(htam_memory *m) {
+  if (!m) return;
+  int prev = 0;
+  cudaGetDevice(&prev);
+  cudaSetDevice(m->device);
+  cudaFree(m->pool);
+  cudaFree(m->slot_id);
+  cudaFree(m->page_list);
+  cudaFree(m->page_off);
+  cudaFree(m->count);
+  cudaFree(m->csum);
+  cudaFree(m->cent);
+  cudaFree(m->cent_hi);
+  cudaFree(m->cent_lo);
+  cudaFree(m->status);
+  cudaFree(m->scratch);
+  cudaFree(m->stage);
+  cudaGetLastError();
+  cudaSetDevice(prev);
+  delete m;
+}
+
+htam_status build_impl(const void *entries, const int32_t *gid, int64_t n, int32_t d,
+                       int32_t n_groups, htam_dtype dtype, int64_t capacity, cudaStream_t st,
+                       htam_memory **out) {
+  htam_memory *m = new (std::nothrow) htam_memory();
+  if (!m) return HTAM_ENOMEM;
+  HTAM_CK(cudaGetDevice(&m->device));
+  HTAM_CK(cudaDeviceGetAttribute(&m->sm_count, cudaDevAttrMultiProcessorCount, m->device));
+  m->d = d;
+  m->n_groups = n_groups;
+  m->dtype = dtype;
+  m->elem_bytes = dtype == HTAM_BF16 ? 2 : 4;
+  m->capacity = capacity;
+  m->n_pages_max = ceil_div(capacity, kPageRows) + n_groups;
+  m->h_count.assign(n_groups, 0);
+  m->h_pages.assign(n_groups, {});
+
+  auto fail = [&](htam_status s) {
+    free_impl(m);
+    return s;
+  };
+  size_t pool_bytes = (size_t)m->n_pages_max * kPageRows * d * m->elem_bytes;
+  size_t gd = (size_t)n_groups * d;
+  if (cudaMalloc(&m->pool, pool_bytes) != cudaSuccess ||
+      cudaMalloc(&m->slot_id, sizeof(int32_t) * m->n_pages_max * kPageRows) != cudaSuccess ||
+      cudaMalloc(&m->page_list, sizeof(int32_t) * m->n_pages_max) != cudaSuccess ||
+      cudaMalloc(&m->page_off, sizeof(int32_t) * (n_groups + 1)) != cudaSuccess ||
+      cudaMalloc(&m->count, sizeof(int32_t) * n_groups) != cudaSuccess ||
+      cudaMalloc(&m->csum, sizeof(double) * gd) != cudaSuccess ||
+      cudaMalloc(&m->cent, sizeof(float) * gd) != cudaSuccess ||
+      cudaMalloc(&m->cent_hi, sizeof(__nv_bfloat16) * gd) != cudaSuccess ||
+      cudaMalloc(&m->cent_lo, sizeof(__nv_bfloat16) * gd) != cudaSuccess ||
+      cudaMalloc(&m->status, sizeof(unsigned int)) != cudaSuccess) {
+    cudaGetLastError();
+    return fail(HTAM_ENOMEM);
+  }
+  // Empty rows are zero (never NaN), empty slots have id -1, keys start at 0.
+  if (cudaMemsetAsync(m->pool, 0, pool_bytes, st) != cudaSuccess ||
+      cudaMemsetAsync(m->slot_id, 0xff, sizeof(int32_t) * m->n_pages_max * kPageRows, st) != cudaSuccess ||
+      cudaMemsetAsync(m->page_off, 0, sizeof(int32_t) * (n_groups + 1), st) != cudaSuccess ||
+      cudaMemsetAsync(m->count, 0, sizeof(int32_t) * n_groups, st) != cudaSuccess ||
+      cudaMemsetAsync(m->csum, 0, sizeof(double) * gd, st) != cudaSuccess ||
+      cudaMemsetAsync(m->cent, 0, sizeof(float) * gd, st) != cudaSuccess ||
+      cudaMemsetAsync(m->cent_hi, 0, sizeof(__nv_bfloat16) * gd, st) != cudaSuccess ||
+      cudaMemsetAsync(m->cent_lo, 0, sizeof(__nv_bfloat16) * gd, st) != cudaSuccess ||
+      cudaMemsetAsync(m->status, 0, sizeof(unsigned int), st) != cudaSuccess) {
+    set_last_error("cudaMemsetAsync", cudaGetLastError());
+    return fail(HTAM_ECUDA);
+  }
+  htam_status s = add_rows(m, entries, gid, n, st);
+  if (s != HTAM_OK) return fail(s);
+  *out = m;
+  return HTAM_OK;
+}
+
+htam_status append_impl(htam_memory *m, const void *entries, const int32_t *gid, int64_t count,
+                        cudaStream_t st) {
+  if (m->n + count > m->capacity) return HTAM_ECAPACITY;
+  return add_rows(m, entries, gid, count, st);
+}
+
+}  // namespace htam

@@ -1,0 +1,677 @@
+// query.cu -- the two-level lookup (read side of one evolution step, §4.3).
+//
+//   1. coarse scores s1[b][g] = q_b . c_g against every group key (Eq. 9
+//      with the linear scorer of App. B.6) and the k_groups best groups;
+//   2. bucketing: invert query -> selected groups into group -> queries so
+//      that each selected group's pages are streamed once per bucket chunk;
+//   3. fine scores over the entries of the selected groups only (the Eq. 12
+//      restriction), with the per-query online softmax statistics (Eq. 11)
+//      and a running top-k_entries (Eq. 13 as a top-k) fused in;
+//   4. merge of the per-unit partial results per query: log-sum-exp combine,
+//      final top-k, weights eps/|C| + (1-eps) exp(s/tau - lse).
+// Nothing is read back to the host; every size that depends on the data
+// lives on the device and the kernels loop over it.
+
+#include <algorithm>
+#include <cstring>
+#include <vector>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace htam {
+
+namespace {
+
+// ------------------------------------------------------------------ stage 1
+
+// s1[b][g] = q_b . cent_g in fp32; -inf for empty groups.  64x64 tile per
+// block, 16x16 threads with 4x4 outputs each, k-slices of 32 staged in
+// shared memory.
+template <typename T>
+__global__ void __launch_bounds__(256) coarse_scores_simt_kernel(
+    const T *__restrict__ Q, int B, int d, const float *__restrict__ cent,
+    const int32_t *__restrict__ count, int G, float *__restrict__ s1) {
+  __shared__ float qs[32][68];
+  __shared__ float cs[32][68];
+  const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
+  const int b0 = blockIdx.y * 64, g0 = blockIdx.x * 64;
+  float acc[4][4] = {};
+  const int lr = tid >> 2, lc = (tid & 3) * 8;  // loader: row, 8 columns
+  for (int k0 = 0; k0 < d; k0 += 32) {
+    {
+      int b = b0 + lr, k = k0 + lc;
+      float v[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+      if (b < B && k < d) {
+        const T *p = Q + (int64_t)b * d + k;
+        if constexpr (sizeof(T) == 2) {
+          uint4 w = *reinterpret_cast<const uint4 *>(p);
+          v[0] = bf16lo(w.x); v[1] = bf16hi(w.x); v[2] = bf16lo(w.y); v[3] = bf16hi(w.y);
+          v[4] = bf16lo(w.z); v[5] = bf16hi(w.z); v[6] = bf16lo(w.w); v[7] = bf16hi(w.w);
+        } else {
+          float4 a = *reinterpret_cast<const float4 *>(p);
+          float4 c = *reinterpret_cast<const float4 *>(p + 4);
+          v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = c.x; v[5] = c.y; v[6] = c.z; v[7] = c.w;
+        }
+      }
+#pragma unroll
+      for (int i = 0; i < 8; ++i) qs[lc + i][lr] = v[i];
+    }
+    {
+      int g = g0 + lr, k = k0 + lc;
+      float v[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+      if (g < G && k < d) {
+        const float *p = cent + (int64_t)g * d + k;
+        float4 a = *reinterpret_cast<const float4 *>(p);
+        float4 c = *reinterpret_cast<const float4 *>(p + 4);
+        v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = c.x; v[5] = c.y; v[6] = c.z; v[7] = c.w;
+      }
+#pragma unroll
+      for (int i = 0; i < 8; ++i) cs[lc + i][lr] = v[i];
+    }
+    __syncthreads();
+#pragma unroll 8
+    for (int k = 0; k < 32; ++k) {
+      float4 a = *reinterpret_cast<const float4 *>(&qs[k][ty * 4]);
+      float4 c = *reinterpret_cast<const float4 *>(&cs[k][tx * 4]);
+      float av[4] = {a.x, a.y, a.z, a.w}, cv[4] = {c.x, c.y, c.z, c.w};
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(av[i], cv[j], acc[i][j]);
+    }
+    __syncthreads();
+  }
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    int b = b0 + ty * 4 + i;
+    if (b >= B) continue;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      int g = g0 + tx * 4 + j;
+      if (g < G) s1[(int64_t)b * G + g] = count[g] > 0 ? acc[i][j] : -INFINITY;
+    }
+  }
+}
+
+// One warp per query: top-k_groups of s1[b][:] (score desc, lower g on ties),
+// empty groups excluded; -1 / -inf padding.
+__global__ void group_topk_kernel(const float *__restrict__ s1, int B, int G,
+                                  const int32_t *__restrict__ count, int kg,
+                                  int32_t *__restrict__ gidx, float *__restrict__ gscore) {
+  int b = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  int lane = threadIdx.x & 31;
+  if (b >= B) return;
+  WarpList L;
+  L.init();
+  float ts = -INFINITY;
+  int ti = INT_MAX;
+  for (int g0 = 0; g0 < G; g0 += 32) {
+    int g = g0 + lane;
+    bool valid = g < G && count[g] > 0;
+    float s = valid ? s1[(int64_t)b * G + g] : -INFINITY;
+    unsigned mask = __ballot_sync(kFullMask, valid && better(s, g, ts, ti));
+    while (mask) {
+      int src = __ffs(mask) - 1;
+      mask &= mask - 1;
+      float cs = __shfl_sync(kFullMask, s, src);
+      L.insert(kg, cs, g0 + src);
+      L.kth(kg, ts, ti);
+    }
+  }
+  if (lane < kg) {
+    gidx[(int64_t)b * kg + lane] = L.i0 == INT_MAX ? -1 : L.i0;
+    gscore[(int64_t)b * kg + lane] = L.i0 == INT_MAX ? -INFINITY : L.s0;
+  }
+  if (lane + 32 < kg) {
+    gidx[(int64_t)b * kg + lane + 32] = L.i1 == INT_MAX ? -1 : L.i1;
+    gscore[(int64_t)b * kg + lane + 32] = L.i1 == INT_MAX ? -INFINITY : L.s1;
+  }
+}
+
+// ---------------------------------------------------------------- bucketing
+
+__global__ void bucket_bits_kernel(const int32_t *__restrict__ gidx, int B, int kg, int W,
+                                   uint32_t *__restrict__ bits) {
+  int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  if (t >= (int64_t)B * kg) return;
+  int b = (int)(t / kg);
+  int32_t g = gidx[t];
+  if (g >= 0) atomicOr(&bits[(int64_t)g * W + (b >> 5)], 1u << (b & 31));
+}
+
+__global__ void bucket_count_kernel(const uint32_t *__restrict__ bits, int G, int W,
+                                    int32_t *__restrict__ cnt) {
+  int g = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  int lane = threadIdx.x & 31;
+  if (g >= G) return;
+  int c = 0;
+  for (int w = lane; w < W; w += 32) c += __popc(bits[(int64_t)g * W + w]);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(kFullMask, c, o);
+  if (lane == 0) cnt[g] = c;
+}
+
+// Single block: per group the bucket size c_g, its work units
+// ceil(c_g/qc) * nseg_g and partial records c_g * nseg_g, with exclusive
+// scans over the groups.  nseg_g = ceil(pages_g / seg_pages).
+__global__ void __launch_bounds__(1024) bucket_scan_kernel(
+    const int32_t *__restrict__ cnt, const int32_t *__restrict__ page_off, int G, int qc,
+    int seg_pages, int32_t *__restrict__ bucket_off, int32_t *__restrict__ unit_off,
+    int64_t *__restrict__ part_off, int32_t *__restrict__ n_units) {
+  __shared__ int64_t sh[3][1024];
+  const int tid = threadIdx.x;
+  const int per = (G + 1023) / 1024;
+  const int lo = min(G, tid * per), hi = min(G, lo + per);
+  int64_t a = 0, u = 0, p = 0;
+  for (int g = lo; g < hi; ++g) {
+    int c = cnt[g];
+    int nseg = (page_off[g + 1] - page_off[g] + seg_pages - 1) / seg_pages;
+    a += c;
+    u += c > 0 ? (int64_t)((c + qc - 1) / qc) * nseg : 0;
+    p += (int64_t)c * nseg;
+  }
+  sh[0][tid] = a;
+  sh[1][tid] = u;
+  sh[2][tid] = p;
+  __syncthreads();
+  for (int o = 1; o < 1024; o <<= 1) {
+    int64_t va = 0, vu = 0, vp = 0;
+    if (tid >= o) {
+      va = sh[0][tid - o];
+      vu = sh[1][tid - o];
+      vp = sh[2][tid - o];
+    }
+    __syncthreads();
+    sh[0][tid] += va;
+    sh[1][tid] += vu;
+    sh[2][tid] += vp;
+    __syncthreads();
+  }
+  a = sh[0][tid] - a;
+  u = sh[1][tid] - u;
+  p = sh[2][tid] - p;
+  for (int g = lo; g < hi; ++g) {
+    int c = cnt[g];
+    int nseg = (page_off[g + 1] - page_off[g] + seg_pages - 1) / seg_pages;
+    bucket_off[g] = (int32_t)a;
+    unit_off[g] = (int32_t)u;
+    part_off[g] = p;
+    a += c;
+    u += c > 0 ? (int64_t)((c + qc - 1) / qc) * nseg : 0;
+    p += (int64_t)c * nseg;
+  }
+  if (tid == 1023) {
+    bucket_off[G] = (int32_t)a;
+    unit_off[G] = (int32_t)u;
+    part_off[G] = p;
+    *n_units = (int32_t)u;
+  }
+}
+
+// One warp per group: bucket[g] lists its queries in increasing order;
+// pos[b][j] = rank of query b in the bucket of its j-th selected group.
+// Also writes the group's work units (group, chunk, segment).
+__global__ void bucket_fill_kernel(const uint32_t *__restrict__ bits, int G, int W,
+                                   const int32_t *__restrict__ bucket_off,
+                                   const int32_t *__restrict__ gidx, int kg,
+                                   const int32_t *__restrict__ cnt,
+                                   const int32_t *__restrict__ page_off, int qc, int seg_pages,
+                                   const int32_t *__restrict__ unit_off,
+                                   int32_t *__restrict__ bucket, int32_t *__restrict__ pos,
+                                   int4 *__restrict__ units) {
+  int g = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  int lane = threadIdx.x & 31;
+  if (g >= G) return;
+  int running = 0;
+  const int base = bucket_off[g];
+  for (int w0 = 0; w0 < W; w0 += 32) {
+    uint32_t word = w0 + lane < W ? bits[(int64_t)g * W + w0 + lane] : 0u;
+    int pc = __popc(word), incl = pc;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      int t = __shfl_up_sync(kFullMask, incl, o);
+      if (lane >= o) incl += t;
+    }
+    int r = running + incl - pc;
+    while (word) {
+      int bit = __ffs(word) - 1;
+      word &= word - 1;
+      int b = (w0 + lane) * 32 + bit;
+      bucket[base + r] = b;
+      for (int j = 0; j < kg; ++j) {
+        if (gidx[(int64_t)b * kg + j] == g) pos[(int64_t)b * kg + j] = r;
+      }
+      ++r;
+    }
+    running += __shfl_sync(kFullMask, incl, 31);
+  }
+  int c = cnt[g];
+  if (c == 0) return;
+  int nseg = (page_off[g + 1] - page_off[g] + seg_pages - 1) / seg_pages;
+  int n_u = ((c + qc - 1) / qc) * nseg;
+  for (int u = lane; u < n_u; u += 32) units[unit_off[g] + u] = make_int4(g, u / nseg, u % nseg, 0);
+}
+
+// ------------------------------------------------------------ fine (SIMT)
+
+struct FineArgs {
+  const void *pool;
+  int d;
+  const int32_t *slot_id;
+  const int32_t *page_list;
+  const int32_t *page_off;
+  const int32_t *count;
+  const void *Q;
+  const int32_t *bucket;
+  const int32_t *bucket_off;
+  const int32_t *cnt;
+  const int4 *units;
+  const int32_t *n_units;
+  const int64_t *part_off;
+  int ke;
+  float inv_tau;
+  int seg_pages;
+  float2 *part_ml;
+  float *part_s;
+  int32_t *part_id;
+};
+
+constexpr int kFineWarps = 8;
+
+// 16 bytes of entry data as fp32 values.
+template <typename T>
+struct Unpack;
+template <>
+struct Unpack<__nv_bfloat16> {
+  static constexpr int kN = 8;
+  __device__ static void run(const uint4 &w, float *f) {
+    f[0] = bf16lo(w.x); f[1] = bf16hi(w.x); f[2] = bf16lo(w.y); f[3] = bf16hi(w.y);
+    f[4] = bf16lo(w.z); f[5] = bf16hi(w.z); f[6] = bf16lo(w.w); f[7] = bf16hi(w.w);
+  }
+};
+template <>
+struct Unpack<float> {
+  static constexpr int kN = 4;
+  __device__ static void run(const uint4 &w, float *f) {
+    f[0] = __uint_as_float(w.x); f[1] = __uint_as_float(w.y);
+    f[2] = __uint_as_float(w.z); f[3] = __uint_as_float(w.w);
+  }
+};
+
+// Work unit = (group g, bucket chunk c, page segment s): the up-to-QC queries
+// bucket[g][c*QC ...] against the rows of pages [s*seg, (s+1)*seg) of g.
+// Each warp streams rows (coalesced 16-byte loads), reduces the dot products
+// with shuffles and keeps, per query, the online softmax state (max, sum of
+// exp) and a warp-distributed top-k; the warps are merged in shared memory
+// and one partial record per (query, unit) is written.
+template <typename T, int QC>
+__global__ void __launch_bounds__(kFineWarps * 32) fine_simt_kernel(FineArgs a) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  constexpr int kN = Unpack<T>::kN;
+  const int d = a.d;
+  float *qs = reinterpret_cast<float *>(smem_raw);              // [QC][d]
+  float *ws = qs + QC * d;                                       // [warps][QC][64]
+  int *wi = reinterpret_cast<int *>(ws + kFineWarps * QC * 64);  // [warps][QC][64]
+  float *wm = reinterpret_cast<float *>(wi + kFineWarps * QC * 64);  // [warps][QC]
+  float *wl = wm + kFineWarps * QC;                                   // [warps][QC]
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int n_vec = d / kN;  // 16-byte vectors per row
+  const int ke = a.ke;
+  const int n_units = *a.n_units;
+  const uint4 *pool = static_cast<const uint4 *>(a.pool);
+  const T *Q = static_cast<const T *>(a.Q);
+
+  for (int u = blockIdx.x; u < n_units; u += gridDim.x) {
+    const int4 U = a.units[u];
+    const int g = U.x, c = U.y, s = U.z;
+    const int cg = a.cnt[g];
+    const int q0 = c * QC;
+    const int nq = min(QC, cg - q0);
+    const int *bq = a.bucket + a.bucket_off[g] + q0;
+
+    __syncthreads();  // the previous unit is done with shared memory
+    for (int i = tid; i < nq * (d / 4); i += blockDim.x) {
+      int j = i / (d / 4), k = (i % (d / 4)) * 4;
+      const T *src = Q + (int64_t)bq[j] * d + k;
+      float4 v;
+      if constexpr (sizeof(T) == 2) {
+        uint2 w = *reinterpret_cast<const uint2 *>(src);
+        v = make_float4(bf16lo(w.x), bf16hi(w.x), bf16lo(w.y), bf16hi(w.y));
+      } else {
+        v = *reinterpret_cast<const float4 *>(src);
+      }
+      *reinterpret_cast<float4 *>(qs + j * d + k) = v;
+    }
+    __syncthreads();
+
+    const int pg0 = a.page_off[g];
+    const int npages = a.page_off[g + 1] - pg0;
+    const int p_beg = s * a.seg_pages;
+    const int p_end = min(npages, p_beg + a.seg_pages);
+    const int r0 = p_beg * kPageRows;
+    const int r1 = min(p_end * kPageRows, a.count[g]);
+
+    float m[QC], l[QC], ts[QC];
+    int ti[QC];
+    WarpList lst[QC];
+#pragma unroll
+    for (int j = 0; j < QC; ++j) {
+      m[j] = -INFINITY;
+      l[j] = 0.f;
+      ts[j] = -INFINITY;
+      ti[j] = INT_MAX;
+      lst[j].init();
+    }
+
+    for (int r = r0 + warp; r < r1; r += kFineWarps) {
+      const int64_t slot = (int64_t)a.page_list[pg0 + r / kPageRows] * kPageRows + (r % kPageRows);
+      const int id = a.slot_id[slot];
+      const uint4 *row = pool + slot * n_vec;
+      float acc[QC];
+#pragma unroll
+      for (int j = 0; j < QC; ++j) acc[j] = 0.f;
+      for (int v = lane; v < n_vec; v += 32) {
+        uint4 w = row[v];
+        float f[kN];
+        Unpack<T>::run(w, f);
+#pragma unroll
+        for (int j = 0; j < QC; ++j) {
+          if (j < nq) {
+            const float *q = qs + j * d + v * kN;
+#pragma unroll
+            for (int t = 0; t < kN; t += 4) {
+              float4 qq = *reinterpret_cast<const float4 *>(q + t);
+              acc[j] = fmaf(f[t], qq.x, acc[j]);
+              acc[j] = fmaf(f[t + 1], qq.y, acc[j]);
+              acc[j] = fmaf(f[t + 2], qq.z, acc[j]);
+              acc[j] = fmaf(f[t + 3], qq.w, acc[j]);
+            }
+          }
+        }
+      }
+#pragma unroll
+      for (int j = 0; j < QC; ++j) {
+        if (j < nq) {
+          float sc = warp_sum(acc[j]);
+          float z = sc * a.inv_tau;
+          if (z > m[j]) {
+            l[j] = l[j] * expf(m[j] - z) + 1.f;
+            m[j] = z;
+          } else {
+            l[j] += expf(z - m[j]);
+          }
+          if (better(sc, id, ts[j], ti[j])) {
+            lst[j].insert(ke, sc, id);
+            lst[j].kth(ke, ts[j], ti[j]);
+          }
+        }
+      }
+    }
+
+    // Hand each warp's state to shared memory, then warp j merges query j.
+#pragma unroll
+    for (int j = 0; j < QC; ++j) {
+      if (j < nq) {
+        int o = (warp * QC + j) * 64;
+        ws[o + lane] = lst[j].s0;
+        wi[o + lane] = lst[j].i0;
+        ws[o + 32 + lane] = lst[j].s1;
+        wi[o + 32 + lane] = lst[j].i1;
+        if (lane == 0) {
+          wm[warp * QC + j] = m[j];
+          wl[warp * QC + j] = l[j];
+        }
+      }
+    }
+    __syncthreads();
+    for (int j = warp; j < nq; j += kFineWarps) {
+      float M = -INFINITY;
+      for (int w = 0; w < kFineWarps; ++w) M = fmaxf(M, wm[w * QC + j]);
+      float Ls = 0.f;
+      for (int w = 0; w < kFineWarps; ++w) {
+        float mw = wm[w * QC + j];
+        if (mw != -INFINITY) Ls += wl[w * QC + j] * expf(mw - M);
+      }
+      WarpList F;
+      F.init();
+      float fs = -INFINITY;
+      int fi = INT_MAX;
+      for (int w = 0; w < kFineWarps; ++w) {
+        for (int h = 0; h < 2; ++h) {
+          if (h * 32 >= ke) break;
+          int o = (w * QC + j) * 64 + h * 32;
+          float cs = ws[o + lane];
+          int ci = wi[o + lane];
+          unsigned mask = __ballot_sync(kFullMask, h * 32 + lane < ke && ci != INT_MAX && better(cs, ci, fs, fi));
+          while (mask) {
+            int src = __ffs(mask) - 1;
+            mask &= mask - 1;
+            float vs = __shfl_sync(kFullMask, cs, src);
+            int vi = __shfl_sync(kFullMask, ci, src);
+            F.insert(ke, vs, vi);
+            F.kth(ke, fs, fi);
+          }
+        }
+      }
+      const int64_t pidx = a.part_off[g] + (int64_t)s * cg + q0 + j;
+      if (lane == 0) a.part_ml[pidx] = make_float2(M, Ls);
+      if (lane < ke) {
+        a.part_s[pidx * ke + lane] = F.s0;
+        a.part_id[pidx * ke + lane] = F.i0;
+      }
+      if (lane + 32 < ke) {
+        a.part_s[pidx * ke + lane + 32] = F.s1;
+        a.part_id[pidx * ke + lane + 32] = F.i1;
+      }
+    }
+  }
+}
+
+// ------------------------------------------------------------------- merge
+
+struct MergeArgs {
+  const int32_t *gidx;
+  int B, kg, ke;
+  const int32_t *count;
+  const int32_t *pos;
+  const int32_t *cnt;
+  const int32_t *page_off;
+  int seg_pages;
+  const int64_t *part_off;
+  const float2 *part_ml;
+  const float *part_s;
+  const int32_t *part_id;
+  float inv_tau, eps;
+  int32_t *entry_idx;
+  float *entry_score, *entry_weight, *lse;
+};
+
+// One warp per query: combine its partial records (one per selected group and
+// page segment): log-sum-exp of the softmax statistics and the final top-k.
+__global__ void merge_kernel(MergeArgs a) {
+  int b = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  int lane = threadIdx.x & 31;
+  if (b >= a.B) return;
+  const int ke = a.ke;
+  float M = -INFINITY, L = 0.f;
+  int64_t nb = 0;
+  WarpList F;
+  F.init();
+  float fs = -INFINITY;
+  int fi = INT_MAX;
+  for (int j = 0; j < a.kg; ++j) {
+    int g = a.gidx[(int64_t)b * a.kg + j];
+    if (g < 0) continue;
+    int p = a.pos[(int64_t)b * a.kg + j];
+    int cg = a.cnt[g];
+    int nseg = (a.page_off[g + 1] - a.page_off[g] + a.seg_pages - 1) / a.seg_pages;
+    nb += a.count[g];
+    for (int s = 0; s < nseg; ++s) {
+      int64_t pidx = a.part_off[g] + (int64_t)s * cg + p;
+      float2 ml = a.part_ml[pidx];
+      if (ml.x != -INFINITY) {
+        float Mn = fmaxf(M, ml.x);
+        L = L * expf(M - Mn) + ml.y * expf(ml.x - Mn);
+        M = Mn;
+      }
+      for (int h = 0; h < 2; ++h) {
+        if (h * 32 >= ke) break;
+        int t = h * 32 + lane;
+        float cs = t < ke ? a.part_s[pidx * ke + t] : -INFINITY;
+        int ci = t < ke ? a.part_id[pidx * ke + t] : INT_MAX;
+        unsigned mask = __ballot_sync(kFullMask, ci != INT_MAX && better(cs, ci, fs, fi));
+        while (mask) {
+          int src = __ffs(mask) - 1;
+          mask &= mask - 1;
+          float vs = __shfl_sync(kFullMask, cs, src);
+          int vi = __shfl_sync(kFullMask, ci, src);
+          F.insert(ke, vs, vi);
+          F.kth(ke, fs, fi);
+        }
+      }
+    }
+  }
+  const float lse_b = nb > 0 ? M + logf(L) : -INFINITY;
+  const float unif = nb > 0 ? a.eps / (float)nb : 0.f;
+  auto emit = [&](int t, float s, int id) {
+    int64_t o = (int64_t)b * ke + t;
+    if (id == INT_MAX) {
+      a.entry_idx[o] = -1;
+      a.entry_score[o] = -INFINITY;
+      a.entry_weight[o] = 0.f;
+    } else {
+      a.entry_idx[o] = id;
+      a.entry_score[o] = s;
+      a.entry_weight[o] = unif + (1.f - a.eps) * expf(s * a.inv_tau - lse_b);
+    }
+  };
+  if (lane < ke) emit(lane, F.s0, F.i0);
+  if (lane + 32 < ke) emit(lane + 32, F.s1, F.i1);
+  if (a.lse && lane == 0) a.lse[b] = lse_b;
+}
+
+template <typename T, int QC>
+htam_status launch_fine_simt(const FineArgs &fa, int sm_count, int64_t max_units, cudaStream_t st) {
+  const int d = fa.d;
+  size_t smem = sizeof(float) * QC * d + (sizeof(float) + sizeof(int)) * kFineWarps * QC * 64 +
+                sizeof(float) * 2 * kFineWarps * QC;
+  HTAM_CK(cudaFuncSetAttribute(fine_simt_kernel<T, QC>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+  int per_sm = 0;
+  HTAM_CK(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fine_simt_kernel<T, QC>, kFineWarps * 32, smem));
+  per_sm = std::max(per_sm, 1);
+  int64_t grid = std::min<int64_t>(max_units, (int64_t)sm_count * per_sm);
+  if (grid <= 0) return HTAM_OK;
+  fine_simt_kernel<T, QC><<<(unsigned)grid, kFineWarps * 32, smem, st>>>(fa);
+  HTAM_CK_LAUNCH("fine_simt_kernel");
+  return HTAM_OK;
+}
+
+template <typename T>
+htam_status dispatch_fine_simt(int qc, const FineArgs &fa, int sm_count, int64_t max_units, cudaStream_t st) {
+  switch (qc) {
+    case 8: return launch_fine_simt<T, 8>(fa, sm_count, max_units, st);
+    case 4: return launch_fine_simt<T, 4>(fa, sm_count, max_units, st);
+    case 2: return launch_fine_simt<T, 2>(fa, sm_count, max_units, st);
+    default: return launch_fine_simt<T, 1>(fa, sm_count, max_units, st);
+  }
+}
+
+}  // namespace
+
+// Queries per SIMT work unit: the staged query block (fp32) stays within
+// 64 KiB of shared memory.
+static int simt_query_chunk(int d) {
+  int qc = 8;
+  while (qc > 1 && (size_t)qc * d * sizeof(float) > 64 * 1024) qc >>= 1;
+  return qc;
+}
+
+constexpr int kSimtSegPages = 4;
+
+htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const htam_query_params &p,
+                       int32_t *group_idx, float *group_score, int32_t *entry_idx,
+                       float *entry_score, float *entry_weight, float *lse, cudaStream_t st) {
+  if (B == 0) return HTAM_OK;
+  const int G = m->n_groups, d = m->d, kg = p.k_groups, ke = p.k_entries;
+  const int qc = simt_query_chunk(d);
+  const int seg = kSimtSegPages;
+
+  // Upper bound of the partial records: every query in the buckets of the
+  // k_g groups with the most page segments.
+  std::vector<int64_t> nseg(G);
+  for (int g = 0; g < G; ++g) nseg[g] = ceil_div((int64_t)m->h_pages[g].size(), seg);
+  std::vector<int64_t> top = nseg;
+  std::nth_element(top.begin(), top.begin() + (kg - 1), top.end(), std::greater<int64_t>());
+  int64_t seg_sum = 0;
+  for (int i = 0; i < kg; ++i) seg_sum += top[i];
+  const int64_t max_parts = std::max<int64_t>(1, (int64_t)B * seg_sum);
+  const int64_t max_units = max_parts;
+  const int W = (int)ceil_div(B, 32);
+
+  size_t need = Carver::round(sizeof(float) * (size_t)B * G) + Carver::round(sizeof(uint32_t) * (size_t)G * W) +
+                4 * Carver::round(sizeof(int32_t) * (G + 1)) + Carver::round(sizeof(int64_t) * (G + 1)) +
+                2 * Carver::round(sizeof(int32_t) * (size_t)B * kg) + Carver::round(sizeof(int4) * max_units) +
+                Carver::round(sizeof(float2) * max_parts) + Carver::round(sizeof(float) * max_parts * ke) +
+                Carver::round(sizeof(int32_t) * max_parts * ke) + Carver::round(64) + 4096;
+  htam_status s = ensure_scratch(m, need);
+  if (s != HTAM_OK) return s;
+  Carver cv(m->scratch);
+  float *s1 = cv.take<float>((size_t)B * G);
+  uint32_t *bits = cv.take<uint32_t>((size_t)G * W);
+  int32_t *cnt = cv.take<int32_t>(G + 1);
+  int32_t *bucket_off = cv.take<int32_t>(G + 1);
+  int32_t *unit_off = cv.take<int32_t>(G + 1);
+  int64_t *part_off = cv.take<int64_t>(G + 1);
+  int32_t *n_units = cv.take<int32_t>(G + 1);
+  int32_t *bucket = cv.take<int32_t>((size_t)B * kg);
+  int32_t *pos = cv.take<int32_t>((size_t)B * kg);
+  int4 *units = cv.take<int4>(max_units);
+  float2 *part_ml = cv.take<float2>(max_parts);
+  float *part_s = cv.take<float>(max_parts * ke);
+  int32_t *part_id = cv.take<int32_t>(max_parts * ke);
+
+  // 1. Coarse scores and the selected groups.
+  {
+    dim3 grid((unsigned)ceil_div(G, 64), (unsigned)ceil_div(B, 64));
+    if (m->dtype == HTAM_BF16) {
+      coarse_scores_simt_kernel<__nv_bfloat16><<<grid, 256, 0, st>>>(
+          static_cast<const __nv_bfloat16 *>(queries), B, d, m->cent, m->count, G, s1);
+    } else {
+      coarse_scores_simt_kernel<float><<<grid, 256, 0, st>>>(static_cast<const float *>(queries), B, d,
+                                                             m->cent, m->count, G, s1);
+    }
+    HTAM_CK_LAUNCH("coarse_scores_simt_kernel");
+    group_topk_kernel<<<(unsigned)ceil_div((int64_t)B * 32, 256), 256, 0, st>>>(s1, B, G, m->count, kg,
+                                                                                group_idx, group_score);
+    HTAM_CK_LAUNCH("group_topk_kernel");
+  }
+
+  // 2. Buckets: group -> queries, work units, partial-record offsets.
+  HTAM_CK(cudaMemsetAsync(bits, 0, sizeof(uint32_t) * (size_t)G * W, st));
+  bucket_bits_kernel<<<(unsigned)ceil_div((int64_t)B * kg, 256), 256, 0, st>>>(group_idx, B, kg, W, bits);
+  HTAM_CK_LAUNCH("bucket_bits_kernel");
+  bucket_count_kernel<<<(unsigned)ceil_div((int64_t)G * 32, 256), 256, 0, st>>>(bits, G, W, cnt);
+  HTAM_CK_LAUNCH("bucket_count_kernel");
+  bucket_scan_kernel<<<1, 1024, 0, st>>>(cnt, m->page_off, G, qc, seg, bucket_off, unit_off, part_off, n_units);
+  HTAM_CK_LAUNCH("bucket_scan_kernel");
+  bucket_fill_kernel<<<(unsigned)ceil_div((int64_t)G * 32, 256), 256, 0, st>>>(
+      bits, G, W, bucket_off, group_idx, kg, cnt, m->page_off, qc, seg, unit_off, bucket, pos, units);
+  HTAM_CK_LAUNCH("bucket_fill_kernel");
+
+  // 3. Fine scores with fused softmax statistics and top-k.
+  FineArgs fa{m->pool, d, m->slot_id, m->page_list, m->page_off, m->count, queries, bucket, bucket_off,
+              cnt, units, n_units, part_off, ke, 1.0f / p.tau, seg, part_ml, part_s, part_id};
+  s = m->dtype == HTAM_BF16 ? dispatch_fine_simt<__nv_bfloat16>(qc, fa, m->sm_count, max_units, st)
+                            : dispatch_fine_simt<float>(qc, fa, m->sm_count, max_units, st);
+  if (s != HTAM_OK) return s;
+
+  // 4. Merge per query.
+  MergeArgs ma{group_idx, B, kg, ke, m->count, pos, cnt, m->page_off, seg, part_off, part_ml, part_s,
+               part_id, 1.0f / p.tau, p.epsilon, entry_idx, entry_score, entry_weight, lse};
+  merge_kernel<<<(unsigned)ceil_div((int64_t)B * 32, 256), 256, 0, st>>>(ma);
+  HTAM_CK_LAUNCH("merge_kernel");
+  return HTAM_OK;
+}
+
+}  // namespace htam

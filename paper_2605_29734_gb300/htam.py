@@ -1,0 +1,220 @@
+"""Python binding of the C ABI in include/htam.h (argument marshalling only).
+
+Every step of the lookup runs in the CUDA library ``_lib/libhtam.so``; this
+module passes torch tensors' device pointers and the current CUDA stream
+through ctypes.  There is no fallback: if the library is missing the import
+fails, and every call raises on a non-OK status.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "_lib", "libhtam.so")
+
+HTAM_OK, HTAM_EINVAL, HTAM_ENOMEM, HTAM_ECAPACITY, HTAM_ECUDA, HTAM_ETIMEOUT, HTAM_ENODEV = range(7)
+HTAM_F32, HTAM_BF16 = 0, 1
+
+# Every symbol include/htam.h declares, in declaration order.
+EXPORTS = (
+    "htam_build_memory", "htam_append_transitions", "htam_query", "htam_query_host",
+    "htam_memory_info", "htam_memory_group_counts", "htam_memory_group_keys",
+    "htam_device_status", "htam_free_memory", "htam_status_string", "htam_last_error",
+    "htam_selftest_wait_timeout",
+)
+
+
+class HtamError(RuntimeError):
+    def __init__(self, status: int, what: str):
+        self.status = status
+        msg = _lib.htam_status_string(status).decode()
+        detail = _lib.htam_last_error().decode()
+        super().__init__(f"{what}: {msg}" + (f" ({detail})" if detail and status == HTAM_ECUDA else ""))
+
+
+class QueryParams(ctypes.Structure):
+    _fields_ = [("k_groups", ctypes.c_int32), ("k_entries", ctypes.c_int32),
+                ("tau", ctypes.c_float), ("epsilon", ctypes.c_float)]
+
+
+def _load() -> ctypes.CDLL:
+    if not os.path.exists(LIB_PATH):
+        raise ImportError(f"{LIB_PATH} is missing: build it with paper_2605_29734_gb300.build.build()")
+    lib = ctypes.CDLL(LIB_PATH)
+    P, i32, i64, st = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_int
+    PP = ctypes.POINTER(ctypes.c_void_p)
+    lib.htam_build_memory.argtypes = [P, P, i64, i32, i32, ctypes.c_int, i64, P, PP]
+    lib.htam_append_transitions.argtypes = [P, P, P, i64, P]
+    qargs = [P, P, i32, ctypes.POINTER(QueryParams), P, P, P, P, P, P, P]
+    lib.htam_query.argtypes = qargs
+    lib.htam_query_host.argtypes = qargs
+    lib.htam_memory_info.argtypes = [P, P, P, P, P]
+    lib.htam_memory_group_counts.argtypes = [P, P]
+    lib.htam_memory_group_keys.argtypes = [P, P, P]
+    lib.htam_device_status.argtypes = [P, P]
+    lib.htam_free_memory.argtypes = [P]
+    lib.htam_free_memory.restype = None
+    lib.htam_status_string.argtypes = [st]
+    lib.htam_status_string.restype = ctypes.c_char_p
+    lib.htam_last_error.argtypes = []
+    lib.htam_last_error.restype = ctypes.c_char_p
+    lib.htam_selftest_wait_timeout.argtypes = [i64, P]
+    for name in ("htam_build_memory", "htam_append_transitions", "htam_query", "htam_query_host",
+                 "htam_memory_info", "htam_memory_group_counts", "htam_memory_group_keys",
+                 "htam_device_status", "htam_selftest_wait_timeout"):
+        getattr(lib, name).restype = st
+    return lib
+
+
+_lib = _load()
+
+
+def lib() -> ctypes.CDLL:
+    return _lib
+
+
+def _check(status: int, what: str) -> None:
+    if status != HTAM_OK:
+        raise HtamError(status, what)
+
+
+def _stream_ptr(stream) -> ctypes.c_void_p:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(int(stream.cuda_stream))
+
+
+def _dev_ptr(t: torch.Tensor | None) -> ctypes.c_void_p:
+    if t is None:
+        return ctypes.c_void_p(0)
+    if not t.is_cuda or not t.is_contiguous():
+        raise ValueError("expected a contiguous CUDA tensor")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _dtype_code(dt: torch.dtype) -> int:
+    if dt == torch.bfloat16:
+        return HTAM_BF16
+    if dt == torch.float32:
+        return HTAM_F32
+    raise TypeError(f"entries must be bfloat16 or float32, got {dt}")
+
+
+class Memory:
+    """A device-resident two-level memory (groups of transition entries)."""
+
+    def __init__(self, entries: torch.Tensor, group_ids: torch.Tensor, n_groups: int,
+                 capacity: int | None = None, stream=None):
+        if entries.dim() != 2 or group_ids.dim() != 1 or group_ids.dtype != torch.int32:
+            raise ValueError("entries [n, d] and int32 group_ids [n] expected")
+        n, d = entries.shape
+        self.dtype = entries.dtype
+        self.d = int(d)
+        self.n_groups = int(n_groups)
+        handle = ctypes.c_void_p()
+        cap = int(capacity if capacity is not None else max(n, 1))
+        _check(_lib.htam_build_memory(_dev_ptr(entries), _dev_ptr(group_ids), n, d, n_groups,
+                                      _dtype_code(entries.dtype), cap, _stream_ptr(stream),
+                                      ctypes.byref(handle)), "htam_build_memory")
+        self._h = handle
+
+    @property
+    def handle(self) -> ctypes.c_void_p:
+        if not self._h:
+            raise RuntimeError("memory already freed")
+        return self._h
+
+    def append(self, entries: torch.Tensor, group_ids: torch.Tensor, stream=None) -> None:
+        if entries.dtype != self.dtype or group_ids.dtype != torch.int32:
+            raise TypeError("entries must match the memory dtype; group_ids int32")
+        if entries.dim() != 2 or entries.shape[1] != self.d or group_ids.shape[0] != entries.shape[0]:
+            raise ValueError("entries [count, d] and group_ids [count] expected")
+        _check(_lib.htam_append_transitions(self.handle, _dev_ptr(entries), _dev_ptr(group_ids),
+                                            entries.shape[0], _stream_ptr(stream)),
+               "htam_append_transitions")
+
+    def query(self, queries: torch.Tensor, k_groups: int, k_entries: int, tau: float = 1.0,
+              epsilon: float = 0.0, stream=None, out: dict | None = None) -> dict:
+        """Device lookup; returns (or fills) a dict of device tensors."""
+        if queries.dtype != self.dtype or queries.dim() != 2 or queries.shape[1] != self.d:
+            raise ValueError("queries must be [b, d] of the memory dtype")
+        b = queries.shape[0]
+        dev = queries.device
+        if out is None:
+            out = {
+                "group_idx": torch.empty(b, k_groups, dtype=torch.int32, device=dev),
+                "group_score": torch.empty(b, k_groups, dtype=torch.float32, device=dev),
+                "entry_idx": torch.empty(b, k_entries, dtype=torch.int32, device=dev),
+                "entry_score": torch.empty(b, k_entries, dtype=torch.float32, device=dev),
+                "entry_weight": torch.empty(b, k_entries, dtype=torch.float32, device=dev),
+                "lse": torch.empty(b, dtype=torch.float32, device=dev),
+            }
+        p = QueryParams(k_groups, k_entries, tau, epsilon)
+        _check(_lib.htam_query(self.handle, _dev_ptr(queries), b, ctypes.byref(p),
+                               _dev_ptr(out["group_idx"]), _dev_ptr(out["group_score"]),
+                               _dev_ptr(out["entry_idx"]), _dev_ptr(out["entry_score"]),
+                               _dev_ptr(out["entry_weight"]), _dev_ptr(out.get("lse")),
+                               _stream_ptr(stream)), "htam_query")
+        return out
+
+    def query_host(self, queries: torch.Tensor, k_groups: int, k_entries: int, tau: float = 1.0,
+                   epsilon: float = 0.0, stream=None, out: dict | None = None) -> dict:
+        """Lookup with host (CPU, ideally pinned) tensors in and out; the copies
+        to and from the device happen inside the library call."""
+        if queries.is_cuda or not queries.is_contiguous():
+            raise ValueError("query_host takes a contiguous CPU tensor")
+        b = queries.shape[0]
+        pin = queries.is_pinned()
+        if out is None:
+            def mk(shape, dt):
+                return torch.empty(shape, dtype=dt, pin_memory=pin)
+            out = {"group_idx": mk((b, k_groups), torch.int32), "group_score": mk((b, k_groups), torch.float32),
+                   "entry_idx": mk((b, k_entries), torch.int32), "entry_score": mk((b, k_entries), torch.float32),
+                   "entry_weight": mk((b, k_entries), torch.float32), "lse": mk((b,), torch.float32)}
+        p = QueryParams(k_groups, k_entries, tau, epsilon)
+        hp = lambda t: ctypes.c_void_p(t.data_ptr()) if t is not None else ctypes.c_void_p(0)
+        _check(_lib.htam_query_host(self.handle, hp(queries), b, ctypes.byref(p), hp(out["group_idx"]),
+                                    hp(out["group_score"]), hp(out["entry_idx"]), hp(out["entry_score"]),
+                                    hp(out["entry_weight"]), hp(out.get("lse")), _stream_ptr(stream)),
+               "htam_query_host")
+        return out
+
+    def info(self) -> dict:
+        n, d, g, cap = ctypes.c_int64(), ctypes.c_int32(), ctypes.c_int32(), ctypes.c_int64()
+        _check(_lib.htam_memory_info(self.handle, ctypes.byref(n), ctypes.byref(d), ctypes.byref(g),
+                                     ctypes.byref(cap)), "htam_memory_info")
+        return {"n": n.value, "d": d.value, "n_groups": g.value, "capacity": cap.value}
+
+    def group_counts(self) -> torch.Tensor:
+        out = torch.empty(self.n_groups, dtype=torch.int64)
+        _check(_lib.htam_memory_group_counts(self.handle, ctypes.c_void_p(out.data_ptr())),
+               "htam_memory_group_counts")
+        return out
+
+    def group_keys(self, stream=None) -> torch.Tensor:
+        out = torch.empty(self.n_groups, self.d, dtype=torch.float32)
+        _check(_lib.htam_memory_group_keys(self.handle, ctypes.c_void_p(out.data_ptr()), _stream_ptr(stream)),
+               "htam_memory_group_keys")
+        return out
+
+    def device_status(self, stream=None) -> int:
+        return _lib.htam_device_status(self.handle, _stream_ptr(stream))
+
+    def close(self) -> None:
+        if self._h:
+            _lib.htam_free_memory(self._h)
+            self._h = ctypes.c_void_p()
+
+    def __del__(self):  # pragma: no cover - best effort
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def selftest_wait_timeout(max_iters: int, stream=None) -> int:
+    """Runs the bounded-wait diagnostic; returns the status code."""
+    return _lib.htam_selftest_wait_timeout(int(max_iters), _stream_ptr(stream))

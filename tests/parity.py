@@ -1,0 +1,133 @@
+"""GPU-vs-oracle comparison rules shared by the parity tests.
+
+Index rule: with t_k and t_{k+1} the oracle's k-th and (k+1)-th scores, the
+returned set must equal the oracle's when t_k - t_{k+1} > 1e-3; otherwise every
+oracle index scoring above t_k + 1e-3 must be returned and every returned
+index must score at least t_k - 1e-3 (exact oracle scores).  The order must
+agree wherever adjacent scores differ by more than 1e-3.  Padding (-1) must
+match exactly.
+
+Value rule: |gpu - ref| <= rtol * |ref| + atol with (rtol, atol) =
+(2e-2, 1e-4) for bf16 inputs and (1e-5, 1e-7) for fp32 inputs.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+GAP = 1e-3
+TOL = {"bf16": (2e-2, 1e-4), "f32": (1e-5, 1e-7)}
+
+
+def close(gpu, ref, dtype) -> bool:
+    rtol, atol = TOL[dtype]
+    gpu, ref = float(gpu), float(ref)
+    if np.isneginf(ref):
+        return np.isneginf(gpu)
+    return abs(gpu - ref) <= rtol * abs(ref) + atol
+
+
+def check_ranked(what, gpu_ids, gpu_scores, ref_ids, ref_scores, k, exact_score, dtype):
+    """gpu_ids/gpu_scores: length k.  ref_ids/ref_scores: the oracle's ranking
+    of length >= k+1 (padded with -1 / -inf).  exact_score(id) gives the
+    oracle's (float64) score of any id.  Returns a list of problems."""
+    bad = []
+    gpu_ids = [int(x) for x in gpu_ids[:k]]
+    ref_ids = [int(x) for x in ref_ids]
+    v_ref = sum(1 for x in ref_ids[:k] if x >= 0)
+    v_gpu = sum(1 for x in gpu_ids if x >= 0)
+    if v_ref != v_gpu or any(x < 0 for x in gpu_ids[:v_gpu]) or any(x >= 0 for x in gpu_ids[v_gpu:]):
+        return [f"{what}: padding differs (gpu {gpu_ids}, oracle {ref_ids[:k]})"]
+    if len(set(gpu_ids[:v_gpu])) != v_gpu:
+        return [f"{what}: duplicate ids {gpu_ids}"]
+    if v_ref < k:
+        if set(gpu_ids[:v_gpu]) != set(ref_ids[:v_ref]):
+            bad.append(f"{what}: candidate set differs")
+    else:
+        t_k = float(ref_scores[k - 1])
+        t_next = float(ref_scores[k]) if len(ref_scores) > k else -np.inf
+        if t_k - t_next > GAP:
+            if set(gpu_ids) != set(ref_ids[:k]):
+                bad.append(f"{what}: set differs with a clear gap ({t_k - t_next:.3g}): "
+                           f"gpu {sorted(set(gpu_ids) - set(ref_ids[:k]))} oracle {sorted(set(ref_ids[:k]) - set(gpu_ids))}")
+        else:
+            must = {ref_ids[i] for i in range(k) if float(ref_scores[i]) > t_k + GAP}
+            if not must <= set(gpu_ids):
+                bad.append(f"{what}: missing clearly-better ids {sorted(must - set(gpu_ids))}")
+            for x in gpu_ids:
+                if exact_score(x) < t_k - GAP:
+                    bad.append(f"{what}: id {x} scores {exact_score(x):.6g} < t_k - gap ({t_k:.6g})")
+    es = [exact_score(x) for x in gpu_ids[:v_gpu]]
+    run_min = np.inf
+    for i in range(v_gpu):
+        if es[i] > run_min + GAP:
+            bad.append(f"{what}: order differs at position {i}")
+            break
+        run_min = min(run_min, es[i])
+    for i in range(v_gpu):
+        if not close(gpu_scores[i], es[i], dtype):
+            bad.append(f"{what}: score of id {gpu_ids[i]} gpu {float(gpu_scores[i]):.7g} oracle {es[i]:.7g}")
+            break
+    return bad
+
+
+def compare_lookup(out, entries_np, gid_np, n_groups, queries_np, k_groups, k_entries, tau, eps, dtype,
+                   rows=None, centroid=None, counts=None, nthreads=None):
+    """Checks the GPU outputs of the queries listed in `rows` (all by default)
+    against the oracle: stage 1 directly, stage 2 given the groups the GPU
+    selected (so that a near-tie at the group level cannot cascade)."""
+    import oracle
+
+    gi = out["group_idx"].cpu().numpy()
+    gs = out["group_score"].cpu().numpy()
+    ei = out["entry_idx"].cpu().numpy()
+    es = out["entry_score"].cpu().numpy()
+    ew = out["entry_weight"].cpu().numpy()
+    lse = out["lse"].cpu().numpy()
+    B = queries_np.shape[0]
+    rows = np.arange(B) if rows is None else np.asarray(rows)
+    q = queries_np[rows]
+    if centroid is None:
+        centroid, counts = oracle.centroids(entries_np, gid_np, n_groups, nthreads)
+    ref_gi, ref_gs = oracle.stage1(q, centroid, counts, min(k_groups + 1, n_groups), nthreads)
+    if ref_gi.shape[1] == k_groups:  # k_groups == n_groups: pad the (k+1)-th
+        ref_gi = np.concatenate([ref_gi, -np.ones((len(rows), 1), np.int32)], axis=1)
+        ref_gs = np.concatenate([ref_gs, np.full((len(rows), 1), -np.inf)], axis=1)
+    n_extra = 16
+    ref2 = oracle.stage2(entries_np, gid_np, n_groups, q, gi[rows], k_entries + n_extra, tau, eps, nthreads)
+    qf = _as_f64(q)
+    problems = []
+    for r, b in enumerate(rows):
+        cent_score = lambda g, r=r: float(centroid[g] @ qf[r])
+        problems += check_ranked(f"query {b} groups", gi[b], gs[b], ref_gi[r], ref_gs[r], k_groups,
+                                 cent_score, dtype)
+        ref_map = {int(i): (float(s), float(w)) for i, s, w in
+                   zip(ref2["entry_idx"][r], ref2["entry_score"][r], ref2["entry_weight"][r]) if i >= 0}
+
+        def entry_score(e, r=r):
+            if e in ref_map:
+                return ref_map[e][0]
+            return float(_as_f64(entries_np[e:e + 1])[0] @ qf[r])
+
+        problems += check_ranked(f"query {b} entries", ei[b], es[b], ref2["entry_idx"][r],
+                                 ref2["entry_score"][r], k_entries, entry_score, dtype)
+        nb = int(ref2["n_cand"][r])
+        for i in range(k_entries):
+            e = int(ei[b][i])
+            if e < 0:
+                if ew[b][i] != 0:
+                    problems.append(f"query {b}: padded weight not 0")
+                continue
+            s_ref = entry_score(e)
+            w_ref = ref_map[e][1] if e in ref_map else eps / nb + (1 - eps) * np.exp(s_ref / tau - ref2["lse"][r])
+            if not close(ew[b][i], w_ref, dtype):
+                problems.append(f"query {b}: weight of id {e} gpu {ew[b][i]:.7g} oracle {w_ref:.7g}")
+                break
+        if not close(lse[b], ref2["lse"][r], dtype):
+            problems.append(f"query {b}: lse gpu {lse[b]:.7g} oracle {ref2['lse'][r]:.7g}")
+    return problems
+
+
+def _as_f64(x: np.ndarray) -> np.ndarray:
+    if x.dtype == np.uint16:
+        return (x.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+    return x.astype(np.float64)

@@ -1,0 +1,325 @@
+"""Parity of the CUDA lookup with the float64 oracle, through the C ABI (GPU)."""
+import numpy as np
+import pytest
+import torch
+
+from parity import compare_lookup
+from paper_2605_29734_gb300 import workloads
+from paper_2605_29734_gb300.workloads import to_numpy
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def htam():
+    import __graft_entry__
+
+    __graft_entry__.build()
+    from paper_2605_29734_gb300 import htam as mod
+
+    return mod
+
+
+DEV = "cuda"
+
+
+def _unit(x):
+    return x / torch.linalg.vector_norm(x, dim=1, keepdim=True)
+
+
+def _rand_memory(n, d, g, dtype, seed, clustered=True, gid=None):
+    gen = torch.Generator(device=DEV).manual_seed(seed)
+    if gid is None:
+        gid = torch.randint(0, g, (n,), generator=gen, device=DEV, dtype=torch.int64).to(torch.int32)
+    if clustered:
+        centres = torch.randn(g, d, generator=gen, device=DEV)
+        x = centres[gid.long()] + 0.3 * torch.randn(n, d, generator=gen, device=DEV)
+    else:
+        centres = None
+        x = torch.randn(n, d, generator=gen, device=DEV)
+    return _unit(x).to(dtype).contiguous(), gid.contiguous(), centres
+
+
+def _rand_queries(b, d, dtype, seed, centres=None):
+    gen = torch.Generator(device=DEV).manual_seed(seed + 7)
+    if centres is not None:
+        pick = torch.randint(0, centres.shape[0], (b,), generator=gen, device=DEV)
+        x = centres[pick] + 0.3 * torch.randn(b, d, generator=gen, device=DEV)
+    else:
+        x = torch.randn(b, d, generator=gen, device=DEV)
+    return _unit(x).to(dtype).contiguous()
+
+
+def _check(htam, mem, entries, gid, g, queries, kg, ke, tau=1.0, eps=0.0, rows=None, **kw):
+    out = mem.query(queries, kg, ke, tau=tau, epsilon=eps)
+    torch.cuda.synchronize()
+    dt = "bf16" if queries.dtype == torch.bfloat16 else "f32"
+    problems = compare_lookup(out, to_numpy(entries), to_numpy(gid), g, to_numpy(queries), kg, ke, tau, eps,
+                              dt, rows=rows, **kw)
+    assert not problems, "\n".join(problems[:20])
+    assert mem.device_status() == htam.HTAM_OK
+    return out
+
+
+# ------------------------------------------------------------- workload sizes
+
+@pytest.mark.parametrize("tau,eps", [(1.0, 0.0), (0.05, 0.0), (1.0, 0.1), (0.5, 1.0)])
+def test_tiny_fp32_workload(htam, tau, eps):
+    w = workloads.WORKLOADS["tiny_f32_1k"]
+    entries, gid, centres = workloads.make_memory(w, seed=0, device=DEV)
+    q = workloads.make_queries(w, gid, centres, seed=0)
+    mem = htam.Memory(entries, gid, w.g)
+    _check(htam, mem, entries, gid, w.g, q, w.k_groups, w.k_entries, tau, eps)
+
+
+def test_zipf_65k_workload(htam):
+    w = workloads.WORKLOADS["zipf_bf16_65k"]
+    entries, gid, centres = workloads.make_memory(w, seed=0, device=DEV)
+    q = workloads.make_queries(w, gid, centres, seed=0)
+    mem = htam.Memory(entries, gid, w.g)
+    _check(htam, mem, entries, gid, w.g, q, w.k_groups, w.k_entries)
+
+
+def test_zipf_1m_workload_sampled(htam):
+    """Full size, full batch, as the benchmark runs it; the oracle checks a
+    sample of the queries (stage 2 given the GPU's groups)."""
+    w = workloads.WORKLOADS["zipf_bf16_1m"]
+    entries, gid, centres = workloads.make_memory(w, seed=0, device=DEV)
+    q = workloads.make_queries(w, gid, centres, seed=0)
+    mem = htam.Memory(entries, gid, w.g)
+    rows = np.linspace(0, w.b - 1, 48).astype(int)
+    _check(htam, mem, entries, gid, w.g, q, w.k_groups, w.k_entries, rows=rows)
+
+
+def test_uniform_4m_workload_sampled(htam):
+    """The largest memory (4,194,304 x 4,096 bf16, 32 GiB of keys), full batch;
+    the oracle's group keys are accumulated from device chunks and a sample of
+    queries is checked."""
+    import oracle
+
+    w = workloads.WORKLOADS["uniform_bf16_4m"]
+    entries, gid, centres = workloads.make_memory(w, seed=0, device=DEV)
+    q = workloads.make_queries(w, gid, centres, seed=0)
+    mem = htam.Memory(entries, gid, w.g)
+    out = mem.query(q, w.k_groups, w.k_entries)
+    torch.cuda.synchronize()
+    entries_np = to_numpy(entries)
+    gid_np = to_numpy(gid)
+    del entries
+    cent, counts = oracle.centroids(entries_np, gid_np, w.g)
+    rows = np.linspace(0, w.b - 1, 16).astype(int)
+    problems = compare_lookup(out, entries_np, gid_np, w.g, to_numpy(q), w.k_groups, w.k_entries, 1.0, 0.0,
+                              "bf16", rows=rows, centroid=cent, counts=counts)
+    assert not problems, "\n".join(problems[:20])
+
+
+# ------------------------------------------------------------------ edge cases
+
+@pytest.mark.parametrize("b", [1, 31, 33, 100])
+def test_ragged_batches(htam, b):
+    entries, gid, centres = _rand_memory(5000, 64, 40, torch.bfloat16, seed=b)
+    q = _rand_queries(b, 64, torch.bfloat16, seed=b, centres=centres)
+    mem = htam.Memory(entries, gid, 40)
+    _check(htam, mem, entries, gid, 40, q, 5, 7)
+
+
+def test_empty_batch(htam):
+    entries, gid, _ = _rand_memory(300, 32, 4, torch.float32, seed=1)
+    mem = htam.Memory(entries, gid, 4)
+    out = mem.query(torch.empty(0, 32, device=DEV), 2, 3)
+    torch.cuda.synchronize()
+    assert out["entry_idx"].shape == (0, 3)
+
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+def test_all_groups_selected_is_flat_scan(htam, dtype):
+    entries, gid, centres = _rand_memory(3000, 48, 16, dtype, seed=3)
+    q = _rand_queries(20, 48, dtype, seed=3, centres=centres)
+    mem = htam.Memory(entries, gid, 16)
+    out = _check(htam, mem, entries, gid, 16, q, 16, 64)
+    assert (out["entry_idx"] >= 0).all()
+
+
+def test_k_max_both_levels(htam):
+    entries, gid, centres = _rand_memory(20000, 128, 100, torch.bfloat16, seed=4)
+    q = _rand_queries(64, 128, torch.bfloat16, seed=4, centres=centres)
+    mem = htam.Memory(entries, gid, 100)
+    _check(htam, mem, entries, gid, 100, q, 64, 64, tau=0.2, eps=0.05)
+
+
+def test_empty_groups_and_short_candidate_sets(htam):
+    # 50 groups declared, only 6 hold entries; k_groups above the non-empty
+    # count and k_entries above the candidate-set size both pad.
+    gid = torch.tensor([3, 7, 11, 19, 23, 42] * 5, dtype=torch.int32, device=DEV)
+    entries, gid, _ = _rand_memory(30, 16, 50, torch.float32, seed=5, clustered=False, gid=gid)
+    q = _rand_queries(9, 16, torch.float32, seed=5)
+    mem = htam.Memory(entries, gid, 50)
+    out = _check(htam, mem, entries, gid, 50, q, 8, 40)
+    assert (out["group_idx"][:, 6:] == -1).all()
+    assert (out["entry_idx"][:, 30:] == -1).all()
+
+
+def test_duplicate_rows_tie_to_lower_id(htam):
+    base, _, _ = _rand_memory(10, 32, 1, torch.float32, seed=6, clustered=False)
+    entries = base.repeat(30, 1).contiguous()  # every row appears 30 times
+    gid = (torch.arange(300, device=DEV) % 3).to(torch.int32)
+    q = _rand_queries(4, 32, torch.float32, seed=6)
+    mem = htam.Memory(entries, gid, 3)
+    out = mem.query(q, 3, 20)
+    torch.cuda.synchronize()
+    ids = out["entry_idx"].cpu().numpy()
+    sc = out["entry_score"].cpu().numpy()
+    for b in range(4):
+        for i in range(19):
+            if sc[b, i] == sc[b, i + 1]:
+                assert ids[b, i] < ids[b, i + 1]
+
+
+@pytest.mark.parametrize("d", [8, 24, 4096, 16384])
+def test_dimension_extremes(htam, d):
+    n = 2000 if d <= 4096 else 400
+    entries, gid, centres = _rand_memory(n, d, 12, torch.bfloat16, seed=d)
+    q = _rand_queries(10, d, torch.bfloat16, seed=d, centres=centres)
+    mem = htam.Memory(entries, gid, 12)
+    _check(htam, mem, entries, gid, 12, q, 3, 9)
+
+
+def test_large_groups_many_segments_ragged_tail(htam):
+    # one group of 5,000 rows (40 pages, ragged last page) and a few small ones
+    gid = torch.cat([torch.zeros(5000, dtype=torch.int32), torch.arange(1, 6, dtype=torch.int32).repeat(7)])
+    gid = gid[torch.randperm(gid.numel(), generator=torch.Generator().manual_seed(0))].to(DEV)
+    entries, gid, centres = _rand_memory(gid.numel(), 96, 6, torch.bfloat16, seed=8, gid=gid)
+    q = _rand_queries(40, 96, torch.bfloat16, seed=8, centres=centres)
+    mem = htam.Memory(entries, gid, 6)
+    _check(htam, mem, entries, gid, 6, q, 2, 33)
+
+
+# ---------------------------------------------------------------- append path
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+def test_append_rounds_match_rebuilt_oracle(htam, dtype):
+    entries, gid, centres = _rand_memory(4000, 64, 30, dtype, seed=9)
+    mem = htam.Memory(entries, gid, 30, capacity=4000 + 3 * 700)
+    q = _rand_queries(50, 64, dtype, seed=9, centres=centres)
+    all_e, all_g = entries, gid
+    for r in range(3):
+        new_e, new_g, _ = _rand_memory(700, 64, 30, dtype, seed=100 + r)
+        mem.append(new_e, new_g)
+        all_e = torch.cat([all_e, new_e])
+        all_g = torch.cat([all_g, new_g])
+        assert mem.info()["n"] == all_e.shape[0]
+        assert (mem.group_counts().numpy() == np.bincount(to_numpy(all_g), minlength=30)).all()
+        _check(htam, mem, all_e, all_g, 30, q, 4, 12, tau=0.3)
+
+
+def test_append_updates_group_keys_in_place(htam):
+    import oracle
+
+    entries, gid, _ = _rand_memory(3000, 32, 8, torch.float32, seed=10)
+    mem = htam.Memory(entries, gid, 8, capacity=6000)
+    new_e, new_g, _ = _rand_memory(2500, 32, 8, torch.float32, seed=11)
+    mem.append(new_e, new_g)
+    keys = mem.group_keys().numpy()
+    ref, _ = oracle.centroids(to_numpy(torch.cat([entries, new_e])), to_numpy(torch.cat([gid, new_g])), 8)
+    np.testing.assert_allclose(keys, ref, rtol=1e-6, atol=1e-7)
+
+
+def test_append_errors_leave_memory_unchanged(htam):
+    entries, gid, centres = _rand_memory(1000, 32, 10, torch.bfloat16, seed=12)
+    mem = htam.Memory(entries, gid, 10, capacity=1100)
+    q = _rand_queries(8, 32, torch.bfloat16, seed=12, centres=centres)
+    before = {k: v.clone() for k, v in mem.query(q, 3, 5).items()}
+    bad_e, bad_g, _ = _rand_memory(50, 32, 10, torch.bfloat16, seed=13)
+    bad_g[17] = 10  # out of range
+    with pytest.raises(htam.HtamError) as err:
+        mem.append(bad_e, bad_g)
+    assert err.value.status == htam.HTAM_EINVAL
+    big_e, big_g, _ = _rand_memory(101, 32, 10, torch.bfloat16, seed=14)
+    with pytest.raises(htam.HtamError) as err:
+        mem.append(big_e, big_g)
+    assert err.value.status == htam.HTAM_ECAPACITY
+    after = mem.query(q, 3, 5)
+    torch.cuda.synchronize()
+    assert mem.info()["n"] == 1000
+    for k in before:
+        assert torch.equal(before[k], after[k])
+
+
+def test_stream_workload_rounds(htam):
+    """The streaming workload at full size for its first rounds (append 4,096
+    clustered rows, then 1,024 queries), oracle-checked on sampled queries."""
+    import oracle
+
+    w = workloads.WORKLOADS["stream_bf16_512k"]
+    entries, gid, centres = workloads.make_memory(w, seed=0, device=DEV)
+    mem = htam.Memory(entries, gid, w.g, capacity=w.capacity)
+    all_e, all_g = [to_numpy(entries)], [to_numpy(gid)]
+    acc = oracle.CentroidAccumulator(w.g, w.d)
+    acc.add(all_e[0], all_g[0])
+    for r in range(3):
+        new_e, new_g = workloads.make_append_batch(w, centres, r, seed=0, device=DEV)
+        mem.append(new_e, new_g)
+        all_e.append(to_numpy(new_e))
+        all_g.append(to_numpy(new_g))
+        acc.add(all_e[-1], all_g[-1])
+        q = workloads.make_queries(w, gid, centres, seed=0, stream=200 + r)
+        out = mem.query(q, w.k_groups, w.k_entries)
+        torch.cuda.synchronize()
+        cent, counts = acc.finalize()
+        rows = np.linspace(0, w.b - 1, 24).astype(int)
+        problems = compare_lookup(out, np.concatenate(all_e), np.concatenate(all_g), w.g, to_numpy(q),
+                                  w.k_groups, w.k_entries, 1.0, 0.0, "bf16", rows=rows,
+                                  centroid=cent, counts=counts)
+        assert not problems, "\n".join(problems[:20])
+
+
+# ------------------------------------------------------------------ interfaces
+
+def test_host_buffer_query_matches_device_query(htam):
+    entries, gid, centres = _rand_memory(8000, 128, 20, torch.bfloat16, seed=15)
+    q = _rand_queries(70, 128, torch.bfloat16, seed=15, centres=centres)
+    mem = htam.Memory(entries, gid, 20)
+    dev = mem.query(q, 4, 10, tau=0.7, epsilon=0.2)
+    host = mem.query_host(q.cpu().pin_memory(), 4, 10, tau=0.7, epsilon=0.2)
+    for k in dev:
+        assert torch.equal(dev[k].cpu(), host[k]), k
+
+
+def test_repeated_queries_are_bitwise_deterministic(htam):
+    entries, gid, centres = _rand_memory(30000, 256, 64, torch.bfloat16, seed=16)
+    q = _rand_queries(200, 256, torch.bfloat16, seed=16, centres=centres)
+    mem = htam.Memory(entries, gid, 64)
+    a = {k: v.clone() for k, v in mem.query(q, 8, 16).items()}
+    mem2 = htam.Memory(entries, gid, 64)
+    b = mem2.query(q, 8, 16)
+    c = mem.query(q, 8, 16)
+    torch.cuda.synchronize()
+    for k in a:
+        assert torch.equal(a[k], b[k]) and torch.equal(a[k], c[k]), k
+
+
+def test_bad_query_arguments(htam):
+    entries, gid, _ = _rand_memory(100, 16, 4, torch.float32, seed=17)
+    mem = htam.Memory(entries, gid, 4)
+    q = _rand_queries(2, 16, torch.float32, seed=17)
+    for kw in (dict(k_groups=0, k_entries=1), dict(k_groups=5, k_entries=1), dict(k_groups=1, k_entries=65),
+               dict(k_groups=1, k_entries=1, tau=0.0), dict(k_groups=1, k_entries=1, epsilon=1.5)):
+        with pytest.raises(htam.HtamError) as err:
+            mem.query(q, **kw)
+        assert err.value.status == htam.HTAM_EINVAL
+
+
+def test_bounded_wait_gives_up_and_context_survives(htam):
+    assert htam.selftest_wait_timeout(1000) == htam.HTAM_ETIMEOUT
+    entries, gid, _ = _rand_memory(500, 16, 4, torch.float32, seed=18)
+    mem = htam.Memory(entries, gid, 4)
+    q = _rand_queries(3, 16, torch.float32, seed=18)
+    _check(htam, mem, entries, gid, 4, q, 2, 4)
+
+
+def test_build_rejects_out_of_range_group_ids(htam):
+    entries, gid, _ = _rand_memory(100, 16, 4, torch.float32, seed=19)
+    gid[5] = -1
+    with pytest.raises(htam.HtamError) as err:
+        htam.Memory(entries, gid, 4)
+    assert err.value.status == htam.HTAM_EINVAL
