@@ -9,7 +9,7 @@
 // Every step is deterministic: rows are placed by a stable counting sort (the
 // i-th row of a group in input order lands at the group's next free slot), and
 // key sums are taken over rows in slot order, in fixed-size row segments whose
-// fp32 partials are added to the fp64 sum in segment order.
+// compensated fp32 partials are added to the fp64 sum in segment order.
 
 #include <algorithm>
 #include <cstdio>
@@ -128,50 +128,57 @@ struct KeyGroup {
   int32_t g, seg0, seg1, count;
 };
 
-// partial[s][j] = sum over rows r0..r1-1 of group g of row[j] (fp32).
+// partial[s][j] = sum over rows r0..r1-1 of group g of row[j], accumulated
+// in fp32 with Kahan compensation and returned as fp64 (sum + compensation),
+// so the key error does not grow with the segment length.
 template <typename T>
 __global__ void key_partial_kernel(const T *__restrict__ pool, int32_t d,
                                    const int32_t *__restrict__ page_list,
                                    const int32_t *__restrict__ page_off,
-                                   const KeySeg *__restrict__ segs, float *__restrict__ partial) {
+                                   const KeySeg *__restrict__ segs, double *__restrict__ partial) {
   KeySeg sg = segs[blockIdx.x];
   int j0 = (blockIdx.y * blockDim.x + threadIdx.x) * 8;
   if (j0 >= d) return;
-  float acc[8];
+  float acc[8], comp[8];
 #pragma unroll
-  for (int i = 0; i < 8; ++i) acc[i] = 0.f;
+  for (int i = 0; i < 8; ++i) acc[i] = comp[i] = 0.f;
   const int32_t *pages = page_list + page_off[sg.g];
   for (int r = sg.r0; r < sg.r1; ++r) {
     int64_t slot = (int64_t)pages[r / kPageRows] * kPageRows + (r % kPageRows);
     const T *row = pool + slot * d + j0;
+    float x[8];
     if constexpr (sizeof(T) == 2) {
       uint4 v = *reinterpret_cast<const uint4 *>(row);
-      acc[0] += bf16lo(v.x); acc[1] += bf16hi(v.x);
-      acc[2] += bf16lo(v.y); acc[3] += bf16hi(v.y);
-      acc[4] += bf16lo(v.z); acc[5] += bf16hi(v.z);
-      acc[6] += bf16lo(v.w); acc[7] += bf16hi(v.w);
+      x[0] = bf16lo(v.x); x[1] = bf16hi(v.x); x[2] = bf16lo(v.y); x[3] = bf16hi(v.y);
+      x[4] = bf16lo(v.z); x[5] = bf16hi(v.z); x[6] = bf16lo(v.w); x[7] = bf16hi(v.w);
     } else {
       float4 a = *reinterpret_cast<const float4 *>(row);
       float4 b = *reinterpret_cast<const float4 *>(row + 4);
-      acc[0] += a.x; acc[1] += a.y; acc[2] += a.z; acc[3] += a.w;
-      acc[4] += b.x; acc[5] += b.y; acc[6] += b.z; acc[7] += b.w;
+      x[0] = a.x; x[1] = a.y; x[2] = a.z; x[3] = a.w; x[4] = b.x; x[5] = b.y; x[6] = b.z; x[7] = b.w;
+    }
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      float y = x[i] - comp[i];
+      float t = acc[i] + y;
+      comp[i] = (t - acc[i]) - y;
+      acc[i] = t;
     }
   }
-  float *out = partial + (int64_t)blockIdx.x * d + j0;
+  double *out = partial + (int64_t)blockIdx.x * d + j0;
 #pragma unroll
-  for (int i = 0; i < 8; ++i) out[i] = acc[i];
+  for (int i = 0; i < 8; ++i) out[i] = (double)acc[i] - (double)comp[i];
 }
 
 // csum[g] += partials in segment order; refresh the fp32 mean and its bf16
 // hi/lo split for the group.
 __global__ void key_finalize_kernel(const KeyGroup *__restrict__ groups,
-                                    const float *__restrict__ partial, int32_t d,
+                                    const double *__restrict__ partial, int32_t d,
                                     double *__restrict__ csum, float *__restrict__ cent,
                                     __nv_bfloat16 *__restrict__ hi, __nv_bfloat16 *__restrict__ lo) {
   KeyGroup kg = groups[blockIdx.x];
   for (int j = blockIdx.y * blockDim.x + threadIdx.x; j < d; j += gridDim.y * blockDim.x) {
     double add = 0.0;
-    for (int s = kg.seg0; s < kg.seg1; ++s) add += (double)partial[(int64_t)s * d + j];
+    for (int s = kg.seg0; s < kg.seg1; ++s) add += partial[(int64_t)s * d + j];
     int64_t o = (int64_t)kg.g * d + j;
     double sum = csum[o] + add;
     csum[o] = sum;
@@ -222,7 +229,7 @@ static htam_status add_rows(htam_memory *m, const void *entries, const int32_t *
   size_t need = Carver::round(sizeof(int32_t) * (G + 1)) + Carver::round(sizeof(int32_t) * count) +
                 Carver::round(sizeof(int32_t) * (size_t)G * n_chunks) +
                 Carver::round(sizeof(KeySeg) * max_segs) + Carver::round(sizeof(KeyGroup) * G) +
-                Carver::round(sizeof(float) * (size_t)max_segs * d) + 4096;
+                Carver::round(sizeof(double) * (size_t)max_segs * d) + 4096;
   htam_status s = ensure_scratch(m, need);
   if (s != HTAM_OK) return s;
   Carver cv(m->scratch);
@@ -231,7 +238,7 @@ static htam_status add_rows(htam_memory *m, const void *entries, const int32_t *
   int32_t *hist = cv.take<int32_t>((size_t)G * n_chunks);
   KeySeg *segs = cv.take<KeySeg>(max_segs);
   KeyGroup *kgroups = cv.take<KeyGroup>(G);
-  float *partial = cv.take<float>((size_t)max_segs * d);
+  double *partial = cv.take<double>((size_t)max_segs * d);
 
   // 1. Per-group counts of the batch and the group-id range check.
   HTAM_CK(cudaMemsetAsync(bcount, 0, sizeof(int32_t) * (G + 1), st));
