@@ -1,0 +1,414 @@
+#!/usr/bin/env python
+"""Benchmark of the GB300 memory lookup: queries/s and roofline fraction.
+
+One step = one htam_query over a batch of the workload's queries (coarse
+scores, group top-k, bucketing, fine scores with fused softmax statistics and
+top-k, merge) on a prebuilt memory; for the streaming workload a step is one
+round (append, then query).  Prints ONE JSON line on rank 0.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+  python bench.py --impl reference ...   # the float64 CPU oracle arm
+
+Multi-GPU (launched by torchrun): every rank holds its own replica of the
+memory and answers its own query batches; nothing crosses ranks on the data
+path (a barrier and a max-reduction of the timing only), so scaling is weak.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import re
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2605_29734_gb300 import workloads  # noqa: E402
+
+METRIC = "memory-lookup queries/sec at 1 GB300 and % of roofline (tensor peak or HBM GB/s)"
+UNIT = "queries/s"
+DEFAULT_WORKLOAD = "uniform_bf16_4m"   # the largest configuration (4,194,304 entries, 32 GiB of keys)
+FP32_ALU_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12   # SMs x FP32 lanes x FMA x max clock
+
+
+def parse_args():
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(workloads.WORKLOADS))
+    ap.add_argument("--impl", default="htam", choices=["htam", "reference"])
+    ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--batches", type=int, default=4, help="distinct resident query batches cycled over")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=10.0, help="target length of the oracle sample")
+    return ap.parse_args()
+
+
+# ----------------------------------------------------------------- plumbing
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    elif torch.cuda.is_available():
+        torch.cuda.set_device(local)
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.barrier()
+
+
+def max_over_ranks(x: float, world: int) -> float:
+    if world == 1:
+        return x
+    import torch.distributed as dist
+
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        p = json.load(open(path))
+        return {"hbm_gbs": p["hbm_gbs"], "bf16_tflops": p["bf16_tflops"],
+                "bf16_tflops_sustained": p.get("bf16_tflops_sustained"), "source": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "source": "fallback"}
+
+
+class ClockSampler:
+    """nvidia-smi sampling of SM clocks and throttle reasons while running."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index: int):
+        self.proc = None
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "50",
+                 "-i", str(device_index)], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (OSError, ValueError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, mx, reasons = [], [], set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for line in out.splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for name, val in zip(names, f[5:9]):
+                if val.lower() == "active":
+                    reasons.add(name)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def source_sha(*names) -> str:
+    h = hashlib.sha256()
+    for n in names:
+        h.update(open(os.path.join(ROOT, "paper_2605_29734_gb300", "csrc", n), "rb").read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(kernel: str, workload: str):
+    """Per-launch DRAM bytes of `kernel` on `workload` from a committed ncu
+    summary, if the kernel's source is unchanged since the capture."""
+    path = os.path.join(ROOT, "profiles", f"{kernel}_{workload}.md")
+    if not os.path.exists(path):
+        return None
+    text = open(path).read()
+    m_sha = re.search(r"kernel_source_sha:\s*([0-9a-f]+)", text)
+    m_tr = re.search(r"traffic_bytes_per_launch:\s*([0-9.eE+]+)", text)
+    m_files = re.search(r"kernel_sources:\s*([\w., ]+)", text)
+    if not (m_sha and m_tr and m_files):
+        return None
+    files = [f.strip() for f in m_files.group(1).split(",") if f.strip()]
+    if source_sha(*files) != m_sha.group(1):
+        return None
+    return float(m_tr.group(1))
+
+
+# ------------------------------------------------------------- algorithmic work
+
+def step_work(w, counts: np.ndarray, group_idx: np.ndarray):
+    """Algorithmic bytes / flops of one query batch, from the groups it selected."""
+    s = 2 if w.dtype == "bf16" else 4
+    sel = np.unique(group_idx[group_idx >= 0])
+    entries_read = float(counts[sel].sum())
+    n_b = np.where(group_idx >= 0, counts[np.clip(group_idx, 0, None)], 0).sum(axis=1)
+    B, D, G = group_idx.shape[0], w.d, w.g
+    fine_bytes = entries_read * D * s + B * D * s
+    fine_flops = 2.0 * D * float(n_b.sum())
+    coarse_flops = 2.0 * D * B * G
+    out_bytes = B * (w.k_groups * 8 + w.k_entries * 12 + 4)
+    step_bytes = fine_bytes + G * D * 4 + out_bytes
+    return {"fine_bytes": fine_bytes, "fine_flops": fine_flops, "step_bytes": step_bytes,
+            "step_flops": fine_flops + coarse_flops, "mean_candidates": float(n_b.mean())}
+
+
+# --------------------------------------------------------------------- arms
+
+def make_workload(w, seed, device, rank):
+    entries, gid, centres = workloads.make_memory(w, seed=seed, device=device)
+    return entries, gid, centres
+
+
+def oracle_rate(w, entries_np, gid_np, queries_np, target_s, cent=None, counts=None):
+    """Times the oracle (as it stands) on a bounded sample of the queries."""
+    import oracle
+
+    threads = oracle.default_threads()
+    if cent is None:
+        cent, counts = oracle.centroids(entries_np, gid_np, w.g, threads)
+    probe = min(threads, queries_np.shape[0])
+    t0 = time.perf_counter()
+    oracle.query(entries_np, gid_np, w.g, queries_np[:probe], w.k_groups, w.k_entries, centroid=cent,
+                 counts=counts, nthreads=threads)
+    t_probe = max(time.perf_counter() - t0, 1e-6)
+    n = int(min(queries_np.shape[0], max(probe, probe * target_s / t_probe)))
+    n = max(probe, (n // threads) * threads) if n >= threads else n
+    t0 = time.perf_counter()
+    oracle.query(entries_np, gid_np, w.g, queries_np[:n], w.k_groups, w.k_entries, centroid=cent,
+                 counts=counts, nthreads=threads)
+    dt = time.perf_counter() - t0
+    return n / dt, n, dt, threads, cent, counts
+
+
+def run_reference(args, world, rank):
+    """The float64 oracle on the host cores, same workload, metric and unit."""
+    if rank != 0:
+        return
+    w = workloads.WORKLOADS[args.workload]
+    device = "cuda" if torch.cuda.is_available() else "cpu"
+    entries, gid, centres = make_workload(w, args.seed, device, rank)
+    qs = [workloads.make_queries(w, gid, centres, seed=args.seed, stream=4 + 10 * i) for i in range(args.batches)]
+    entries_np, gid_np = workloads.to_numpy(entries), workloads.to_numpy(gid)
+    del entries
+    q_np = np.concatenate([workloads.to_numpy(q) for q in qs])
+    import oracle
+
+    threads = oracle.default_threads()
+    cent, counts = oracle.centroids(entries_np, gid_np, w.g, threads)
+    per_step_target = max(0.5, 120.0 / max(1, args.steps + args.warmup))
+    _, n_sample, _, _, _, _ = oracle_rate(w, entries_np, gid_np, q_np, per_step_target, cent, counts)
+    times = []
+    for i in range(args.warmup + args.steps):
+        off = (i * n_sample) % max(1, q_np.shape[0] - n_sample + 1)
+        t0 = time.perf_counter()
+        oracle.query(entries_np, gid_np, w.g, q_np[off:off + n_sample], w.k_groups, w.k_entries, centroid=cent,
+                     counts=counts, nthreads=threads)
+        if i >= args.warmup:
+            times.append(time.perf_counter() - t0)
+    total = sum(times)
+    value = n_sample * len(times) / total
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * total / len(times),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic",
+        "config": {"workload": w.name, "queries_per_step": n_sample, "d": w.d, "groups": w.g, "entries": w.n,
+                   "k_groups": w.k_groups, "k_entries": w.k_entries},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle",
+                         "sample": f"{n_sample} queries of {w.name} per step, float64 brute force, "
+                                   f"group keys precomputed"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def run_htam(args, world, rank, local):
+    from paper_2605_29734_gb300 import htam
+
+    w = workloads.WORKLOADS[args.workload]
+    dev = torch.device("cuda", local)
+    stream = torch.cuda.current_stream(dev)
+    props = torch.cuda.get_device_properties(dev)
+    l2_bytes = int(getattr(props, "L2_cache_size", 128 << 20))
+
+    entries, gid, centres = make_workload(w, args.seed, dev, rank)
+    # The streaming workload appends once per step (warm-up, timed, end-to-end).
+    capacity = w.n + (args.warmup + 2 * args.steps + 60) * w.append_per_round if w.rounds else w.n
+    mem = htam.Memory(entries, gid, w.g, capacity=capacity)
+    q_seed = args.seed + 1000 * rank
+    batches = [workloads.make_queries(w, gid, centres, seed=q_seed, stream=4 + 10 * i) for i in range(args.batches)]
+    append_batches = []
+    if w.rounds:
+        n_rounds = args.warmup + args.steps
+        append_batches = [workloads.make_append_batch(w, centres, r, seed=args.seed, device=dev)
+                          for r in range(min(n_rounds, w.rounds))]
+    out = mem.query(batches[0], w.k_groups, w.k_entries)
+    torch.cuda.synchronize()
+
+    # Work per batch (the selected groups decide the bytes).
+    counts = mem.group_counts().numpy()
+    work = []
+    for q in batches:
+        o = mem.query(q, w.k_groups, w.k_entries)
+        work.append(step_work(w, counts, o["group_idx"].cpu().numpy()))
+    flush_l2 = work[0]["step_bytes"] < 4 * l2_bytes
+    flush = torch.empty(2 * l2_bytes, dtype=torch.uint8, device=dev) if flush_l2 else None
+
+    def one_step(i):
+        if w.rounds:
+            e, g = append_batches[i % len(append_batches)]
+            mem.append(e, g)
+        return mem.query(batches[i % len(batches)], w.k_groups, w.k_entries, out=out)
+
+    for i in range(args.warmup):
+        one_step(i)
+    torch.cuda.synchronize()
+    mem.read_phase_timing()          # reset counters
+    mem.set_phase_timing(True)
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    sampler = ClockSampler(local)
+    time.sleep(0.05)
+    barrier(world)
+    torch.cuda.synchronize()
+    wall0 = time.perf_counter()
+    for i in range(args.steps):
+        if flush is not None:
+            flush.fill_(i & 0xFF)
+        starts[i].record(stream)
+        one_step(args.warmup + i)
+        ends[i].record(stream)
+    torch.cuda.synchronize()
+    barrier(world)
+    wall = time.perf_counter() - wall0
+    clocks = sampler.stop()
+    mem.set_phase_timing(False)
+    phases = mem.read_phase_timing()
+    step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
+    total_s = max_over_ranks(sum(step_ms) / 1e3, world)
+    queries_total = w.b * args.steps * world
+    value = queries_total / total_s
+
+    # Dominant kernel roofline (live CUDA events on the launching stream).
+    peaks = load_peaks()
+    per_batch = [work[(args.warmup + i) % len(work)] for i in range(args.steps)]
+    fine_bytes = float(np.mean([x["fine_bytes"] for x in per_batch]))
+    fine_flops = float(np.mean([x["fine_flops"] for x in per_batch]))
+    step_bytes = float(np.mean([x["step_bytes"] for x in per_batch]))
+    step_flops = float(np.mean([x["step_flops"] for x in per_batch]))
+    fine_ms, fine_launches = phases["fine"]
+    fine_s = fine_ms / 1e3 / max(1, fine_launches)
+    achieved = fine_bytes / fine_s / 1e9
+    kernel = "fine_simt"
+    roofline = {"kernel": kernel, "bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                "frac": achieved / peaks["hbm_gbs"],
+                "traffic": profiled_traffic(kernel, w.name), "peak_source": peaks["source"],
+                "algorithmic_bytes_per_launch": fine_bytes, "mean_launch_ms": fine_s * 1e3,
+                "flops_per_launch": fine_flops,
+                "alu_frac": fine_flops / fine_s / 1e12 / FP32_ALU_TFLOPS}
+    t_roof = max(step_bytes / (peaks["hbm_gbs"] * 1e9), step_flops / (FP32_ALU_TFLOPS * 1e12))
+    step_s = total_s / args.steps
+    launches = sum(v[1] for k, v in phases.items() if k != "queries")
+
+    # End to end: host (pinned) queries in, host results out, through the C ABI.
+    host_q = [b.cpu().pin_memory() for b in batches]
+    host_out = mem.query_host(host_q[0], w.k_groups, w.k_entries)
+    e2e_steps = max(3, min(args.steps, 50))
+    torch.cuda.synchronize()
+    barrier(world)
+    t0 = time.perf_counter()
+    for i in range(e2e_steps):
+        if w.rounds:
+            e, g = append_batches[i % len(append_batches)]
+            mem.append(e, g)
+        mem.query_host(host_q[i % len(host_q)], w.k_groups, w.k_entries, out=host_out)
+    barrier(world)
+    e2e_s = max_over_ranks(time.perf_counter() - t0, world)
+    s_elem = 2 if w.dtype == "bf16" else 4
+    e2e = {"value": w.b * e2e_steps * world / e2e_s, "unit": UNIT, "h2d_bytes_per_step": w.b * w.d * s_elem,
+           "d2h_bytes_per_step": w.b * (w.k_groups * 8 + w.k_entries * 12 + 4), "steps": e2e_steps,
+           "path": "htam_query_host (pinned host buffers, copies inside the call)"}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        entries_np, gid_np = workloads.to_numpy(entries), workloads.to_numpy(gid)
+        q_np = np.concatenate([workloads.to_numpy(q) for q in batches])
+        rate, n, dt, threads, _, _ = oracle_rate(w, entries_np, gid_np, q_np, args.cpu_seconds)
+        cpu = {"value": rate, "unit": UNIT, "cores": threads, "kind": "oracle",
+               "sample": f"{n} queries of {w.name} ({dt:.1f} s), float64 brute force over the same memory, "
+                         f"group keys precomputed"}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": 1e3 * step_s, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
+            "config": {"workload": w.name, "queries_per_step": w.b, "d": w.d, "groups": w.g, "entries": w.n,
+                       "k_groups": w.k_groups, "k_entries": w.k_entries, "query_batches": len(batches),
+                       "mean_candidates_per_query": float(np.mean([x["mean_candidates"] for x in work])),
+                       "l2": ("flushed between steps (2x L2 buffer write, outside the step events)" if flush_l2 else
+                              f"inputs larger than L2 ({work[0]['step_bytes'] / 1e9:.2f} GB touched per step)"),
+                       "parallelism": f"replicas{world}" if world > 1 else "single GPU"},
+            "roofline": roofline,
+            "step_roofline": {"algorithmic_bytes": step_bytes, "algorithmic_flops": step_flops,
+                              "t_roof_ms": 1e3 * t_roof, "frac": t_roof / step_s,
+                              "phase_ms_per_step": {k: v[0] / args.steps for k, v in phases.items() if k != "queries"}},
+            "e2e": e2e,
+            "cpu_baseline": cpu,
+            "clocks": clocks,
+            "gpu_launches": launches,
+            "wall_s_timed_region": wall,
+        }
+        print(json.dumps(line), flush=True)
+    mem.close()
+
+
+def main():
+    args = parse_args()
+    world, rank, local = dist_setup()
+    try:
+        if args.impl == "reference":
+            run_reference(args, world, rank)
+        else:
+            run_htam(args, world, rank, local)
+    finally:
+        if world > 1:
+            import torch.distributed as dist
+
+            dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

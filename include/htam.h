@@ -146,6 +146,28 @@ htam_status htam_memory_group_keys(const htam_memory *m, float *keys,
  * check, ECUDA if the stream reports an error, OK otherwise. */
 htam_status htam_device_status(htam_memory *m, void *cuda_stream);
 
+/* Phases of htam_query, for the timing counters below. */
+typedef enum {
+  HTAM_PHASE_COARSE = 0, /* group-key scores */
+  HTAM_PHASE_SELECT = 1, /* top-k_groups per query */
+  HTAM_PHASE_BUCKET = 2, /* group -> queries buckets and work units */
+  HTAM_PHASE_FINE = 3,   /* entry scores, softmax statistics, partial top-k */
+  HTAM_PHASE_MERGE = 4,  /* per-query merge, weights, outputs */
+  HTAM_N_PHASES = 5
+} htam_phase;
+
+/* Turns CUDA-event timing of each htam_query phase on (1) or off (0).  While
+ * on, every query records a pair of events around each phase on its stream
+ * (a few microseconds of host work per query). */
+htam_status htam_set_phase_timing(htam_memory *m, int enable);
+
+/* Synchronises `cuda_stream`, then writes, for the htam_query calls since the
+ * previous read: ms[p] = summed device time of phase p (0 unless timing was
+ * on), launches[p] = kernels phase p launched, *queries = calls.  Any output
+ * may be NULL; arrays hold HTAM_N_PHASES values (host).  Resets the counts. */
+htam_status htam_read_phase_timing(htam_memory *m, double *ms, int64_t *launches,
+                                   int64_t *queries, void *cuda_stream);
+
 /* Releases the memory and all its device storage (NULL is a no-op).  The
  * caller must make sure no queued work still uses it. */
 void htam_free_memory(htam_memory *m);

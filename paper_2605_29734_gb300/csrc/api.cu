@@ -33,6 +33,27 @@ __global__ void wait_timeout_selftest_kernel(const volatile unsigned int *flag, 
   }
 }
 
+void PhaseMark::begin(int p) {
+  phase = p;
+  if (!m->timing) return;
+  while (m->ev_pool.size() < m->ev_used + 2) {
+    cudaEvent_t e;
+    if (cudaEventCreate(&e) != cudaSuccess) {
+      cudaGetLastError();
+      return;
+    }
+    m->ev_pool.push_back(e);
+  }
+  cudaEventRecord(m->ev_pool[m->ev_used], st);
+  m->ev_phase.push_back(p);
+}
+
+void PhaseMark::end() {
+  if (!m->timing || m->ev_phase.size() * 2 != m->ev_used + 2) return;
+  cudaEventRecord(m->ev_pool[m->ev_used + 1], st);
+  m->ev_used += 2;
+}
+
 }  // namespace htam
 
 using namespace htam;
@@ -188,6 +209,35 @@ htam_status htam_device_status(htam_memory *m, void *cuda_stream) {
   HTAM_CK(cudaMemsetAsync(m->status, 0, sizeof(unsigned int), st));
   HTAM_CK(cudaStreamSynchronize(st));
   return word ? HTAM_ETIMEOUT : HTAM_OK;
+}
+
+htam_status htam_set_phase_timing(htam_memory *m, int enable) {
+  if (!m) return HTAM_EINVAL;
+  m->timing = enable != 0;
+  return HTAM_OK;
+}
+
+htam_status htam_read_phase_timing(htam_memory *m, double *ms, int64_t *launches, int64_t *queries,
+                                   void *cuda_stream) {
+  if (!m) return HTAM_EINVAL;
+  HTAM_CK(cudaStreamSynchronize(static_cast<cudaStream_t>(cuda_stream)));
+  double acc[HTAM_N_PHASES] = {};
+  for (size_t i = 0; i < m->ev_used / 2; ++i) {
+    float t = 0.f;
+    HTAM_CK(cudaEventSynchronize(m->ev_pool[2 * i + 1]));
+    HTAM_CK(cudaEventElapsedTime(&t, m->ev_pool[2 * i], m->ev_pool[2 * i + 1]));
+    acc[m->ev_phase[i]] += t;
+  }
+  for (int p = 0; p < HTAM_N_PHASES; ++p) {
+    if (ms) ms[p] = acc[p];
+    if (launches) launches[p] = m->phase_launches[p];
+    m->phase_launches[p] = 0;
+  }
+  if (queries) *queries = m->n_queries;
+  m->n_queries = 0;
+  m->ev_used = 0;
+  m->ev_phase.clear();
+  return HTAM_OK;
 }
 
 void htam_free_memory(htam_memory *m) { free_impl(m); }

@@ -50,6 +50,14 @@ struct htam_memory {
   // Device staging for htam_query_host.
   void *stage = nullptr;
   size_t stage_bytes = 0;
+
+  // Phase timing and launch counters (htam_set_phase_timing / _read_).
+  bool timing = false;
+  std::vector<cudaEvent_t> ev_pool;    // created on demand, reused
+  std::vector<int> ev_phase;           // phase of each recorded pair
+  size_t ev_used = 0;                  // events in use (2 per pair)
+  int64_t n_queries = 0;
+  int64_t phase_launches[HTAM_N_PHASES] = {};
 };
 
 namespace htam {
@@ -83,5 +91,17 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t b,
                        int32_t *entry_idx, float *entry_score, float *entry_weight, float *lse,
                        cudaStream_t st);
 void free_impl(htam_memory *m);
+
+// Records the start / end of a query phase when timing is on, and counts
+// kernel launches per phase.
+struct PhaseMark {
+  htam_memory *m;
+  cudaStream_t st;
+  int phase = -1;
+  PhaseMark(htam_memory *mem, cudaStream_t s) : m(mem), st(s) {}
+  void begin(int p);
+  void end();
+  void launched(int n = 1) { m->phase_launches[phase] += n; }
+};
 
 }  // namespace htam

@@ -362,6 +362,7 @@ void free_impl(htam_memory *m) {
   cudaFree(m->status);
   cudaFree(m->scratch);
   cudaFree(m->stage);
+  for (cudaEvent_t e : m->ev_pool) cudaEventDestroy(e);
   cudaGetLastError();
   cudaSetDevice(prev);
   delete m;

@@ -593,6 +593,8 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
                        int32_t *group_idx, float *group_score, int32_t *entry_idx,
                        float *entry_score, float *entry_weight, float *lse, cudaStream_t st) {
   if (B == 0) return HTAM_OK;
+  m->n_queries += 1;
+  PhaseMark mark(m, st);
   const int G = m->n_groups, d = m->d, kg = p.k_groups, ke = p.k_entries;
   const int qc = simt_query_chunk(d);
   const int seg = kSimtSegPages;
@@ -633,6 +635,7 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
 
   // 1. Coarse scores and the selected groups.
   {
+    mark.begin(HTAM_PHASE_COARSE);
     dim3 grid((unsigned)ceil_div(G, 64), (unsigned)ceil_div(B, 64));
     if (m->dtype == HTAM_BF16) {
       coarse_scores_simt_kernel<__nv_bfloat16><<<grid, 256, 0, st>>>(
@@ -642,12 +645,18 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
                                                              m->cent, m->count, G, s1);
     }
     HTAM_CK_LAUNCH("coarse_scores_simt_kernel");
+    mark.launched();
+    mark.end();
+    mark.begin(HTAM_PHASE_SELECT);
     group_topk_kernel<<<(unsigned)ceil_div((int64_t)B * 32, 256), 256, 0, st>>>(s1, B, G, m->count, kg,
                                                                                 group_idx, group_score);
     HTAM_CK_LAUNCH("group_topk_kernel");
+    mark.launched();
+    mark.end();
   }
 
   // 2. Buckets: group -> queries, work units, partial-record offsets.
+  mark.begin(HTAM_PHASE_BUCKET);
   HTAM_CK(cudaMemsetAsync(bits, 0, sizeof(uint32_t) * (size_t)G * W, st));
   bucket_bits_kernel<<<(unsigned)ceil_div((int64_t)B * kg, 256), 256, 0, st>>>(group_idx, B, kg, W, bits);
   HTAM_CK_LAUNCH("bucket_bits_kernel");
@@ -658,19 +667,27 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   bucket_fill_kernel<<<(unsigned)ceil_div((int64_t)G * 32, 256), 256, 0, st>>>(
       bits, G, W, bucket_off, group_idx, kg, cnt, m->page_off, qc, seg, unit_off, bucket, pos, units);
   HTAM_CK_LAUNCH("bucket_fill_kernel");
+  mark.launched(4);
+  mark.end();
 
   // 3. Fine scores with fused softmax statistics and top-k.
+  mark.begin(HTAM_PHASE_FINE);
   FineArgs fa{m->pool, d, m->slot_id, m->page_list, m->page_off, m->count, queries, bucket, bucket_off,
               cnt, units, n_units, part_off, ke, 1.0f / p.tau, seg, part_ml, part_s, part_id};
   s = m->dtype == HTAM_BF16 ? dispatch_fine_simt<__nv_bfloat16>(qc, fa, m->sm_count, max_units, st)
                             : dispatch_fine_simt<float>(qc, fa, m->sm_count, max_units, st);
   if (s != HTAM_OK) return s;
+  mark.launched();
+  mark.end();
 
   // 4. Merge per query.
+  mark.begin(HTAM_PHASE_MERGE);
   MergeArgs ma{group_idx, B, kg, ke, m->count, pos, cnt, m->page_off, seg, part_off, part_ml, part_s,
                part_id, 1.0f / p.tau, p.epsilon, entry_idx, entry_score, entry_weight, lse};
   merge_kernel<<<(unsigned)ceil_div((int64_t)B * 32, 256), 256, 0, st>>>(ma);
   HTAM_CK_LAUNCH("merge_kernel");
+  mark.launched();
+  mark.end();
   return HTAM_OK;
 }
 

@@ -22,9 +22,10 @@ HTAM_F32, HTAM_BF16 = 0, 1
 EXPORTS = (
     "htam_build_memory", "htam_append_transitions", "htam_query", "htam_query_host",
     "htam_memory_info", "htam_memory_group_counts", "htam_memory_group_keys",
-    "htam_device_status", "htam_free_memory", "htam_status_string", "htam_last_error",
-    "htam_selftest_wait_timeout",
+    "htam_device_status", "htam_set_phase_timing", "htam_read_phase_timing", "htam_free_memory",
+    "htam_status_string", "htam_last_error", "htam_selftest_wait_timeout",
 )
+PHASES = ("coarse", "select", "bucket", "fine", "merge")
 
 
 class HtamError(RuntimeError):
@@ -62,9 +63,12 @@ def _load() -> ctypes.CDLL:
     lib.htam_last_error.argtypes = []
     lib.htam_last_error.restype = ctypes.c_char_p
     lib.htam_selftest_wait_timeout.argtypes = [i64, P]
+    lib.htam_set_phase_timing.argtypes = [P, ctypes.c_int]
+    lib.htam_read_phase_timing.argtypes = [P, P, P, P, P]
     for name in ("htam_build_memory", "htam_append_transitions", "htam_query", "htam_query_host",
                  "htam_memory_info", "htam_memory_group_counts", "htam_memory_group_keys",
-                 "htam_device_status", "htam_selftest_wait_timeout"):
+                 "htam_device_status", "htam_selftest_wait_timeout", "htam_set_phase_timing",
+                 "htam_read_phase_timing"):
         getattr(lib, name).restype = st
     return lib
 
@@ -202,6 +206,21 @@ class Memory:
 
     def device_status(self, stream=None) -> int:
         return _lib.htam_device_status(self.handle, _stream_ptr(stream))
+
+    def set_phase_timing(self, enable: bool) -> None:
+        _check(_lib.htam_set_phase_timing(self.handle, int(bool(enable))), "htam_set_phase_timing")
+
+    def read_phase_timing(self, stream=None) -> dict:
+        """{phase: (device ms summed, kernel launches)} plus 'queries', since the last read."""
+        n = len(PHASES)
+        ms = (ctypes.c_double * n)()
+        launches = (ctypes.c_int64 * n)()
+        queries = ctypes.c_int64()
+        _check(_lib.htam_read_phase_timing(self.handle, ms, launches, ctypes.byref(queries), _stream_ptr(stream)),
+               "htam_read_phase_timing")
+        out = {p: (ms[i], launches[i]) for i, p in enumerate(PHASES)}
+        out["queries"] = queries.value
+        return out
 
     def close(self) -> None:
         if self._h:
