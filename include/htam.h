@@ -129,6 +129,42 @@ htam_status htam_query_host(htam_memory *m, const void *queries, int32_t b,
                             float *entry_score, float *entry_weight,
                             float *lse, void *cuda_stream);
 
+/* Bytes of the fixed device scratch used by htam_select_groups_static. */
+#define HTAM_STATIC_SCRATCH_BYTES (16u << 20)
+
+/* Group selection that allocates nothing.  The paper has no counterpart: this
+ * is an extra entry point for callers that cannot allocate device memory
+ * while they run -- a server whose device memory is fully reserved up front
+ * (an allocation could fail or fragment its pool), code running inside an
+ * allocator callback that must not re-enter the allocator, and latency-
+ * critical loops that cannot absorb the device-wide synchronisation that
+ * cudaFree implies.  htam_query may grow the memory object's scratch with
+ * cudaMalloc; this call never calls cudaMalloc, cudaFree or any allocating
+ * library routine.
+ *
+ * It returns the same group_idx / group_score as htam_query (stage 1: the
+ * coarse scores q . c_g against every non-empty group key and the k_groups
+ * best groups, ties to the lower id, -1 / -inf padding).  Arguments are those
+ * of htam_query: device pointers, queries [b, d] of the memory's dtype,
+ * outputs [b, k_groups].
+ *
+ * Scratch: the [b, n_groups] fp32 score matrix lives in one fixed array of
+ * HTAM_STATIC_SCRATCH_BYTES compiled into the library; every GPU that loads
+ * the library keeps it until the process exits.  Calls with
+ * b * n_groups * 4 > HTAM_STATIC_SCRATCH_BYTES are rejected with HTAM_EINVAL
+ * before anything is launched.  The first call on a device looks up the
+ * array's device address (cudaGetSymbolAddress, with that device current);
+ * make that first call before any stream capture.  The current device must be
+ * the memory's device.  All calls share the array and it keeps the previous
+ * call's contents (each call writes what it reads, so nothing needs to start
+ * at zero); calls whose GPU work overlaps -- on different streams or from
+ * different host threads -- race on it and must be serialised by the caller.
+ * Errors: EINVAL, ECUDA. */
+htam_status htam_select_groups_static(const htam_memory *m, const void *queries,
+                                      int32_t b, int32_t k_groups,
+                                      int32_t *group_idx, float *group_score,
+                                      void *cuda_stream);
+
 /* Sizes of a memory; any output pointer may be NULL (host pointers). */
 htam_status htam_memory_info(const htam_memory *m, int64_t *n, int32_t *d,
                              int32_t *n_groups, int64_t *capacity);

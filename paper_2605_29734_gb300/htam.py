@@ -21,7 +21,7 @@ HTAM_F32, HTAM_BF16 = 0, 1
 # Every symbol include/htam.h declares, in declaration order.
 EXPORTS = (
     "htam_build_memory", "htam_append_transitions", "htam_query", "htam_query_host",
-    "htam_memory_info", "htam_memory_group_counts", "htam_memory_group_keys",
+    "htam_select_groups_static", "htam_memory_info", "htam_memory_group_counts", "htam_memory_group_keys",
     "htam_device_status", "htam_set_phase_timing", "htam_read_phase_timing", "htam_free_memory",
     "htam_status_string", "htam_last_error", "htam_selftest_wait_timeout",
 )
@@ -63,6 +63,8 @@ def _load() -> ctypes.CDLL:
     lib.htam_last_error.argtypes = []
     lib.htam_last_error.restype = ctypes.c_char_p
     lib.htam_selftest_wait_timeout.argtypes = [i64, P]
+    lib.htam_select_groups_static.argtypes = [P, P, i32, i32, P, P, P]
+    lib.htam_select_groups_static.restype = st
     lib.htam_set_phase_timing.argtypes = [P, ctypes.c_int]
     lib.htam_read_phase_timing.argtypes = [P, P, P, P, P]
     for name in ("htam_build_memory", "htam_append_transitions", "htam_query", "htam_query_host",
