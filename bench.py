@@ -51,7 +51,20 @@ def parse_args():
     ap.add_argument("--batches", type=int, default=4, help="distinct resident query batches cycled over")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=10.0, help="target length of the oracle sample")
+    ap.add_argument("--shrink", type=int, default=1,
+                    help="divide the workload's groups and entries by this factor (same group sizes); "
+                         "for small profiling captures only")
     return ap.parse_args()
+
+
+def workload_of(args):
+    w = workloads.WORKLOADS[args.workload]
+    if args.shrink > 1:
+        import dataclasses
+
+        w = dataclasses.replace(w, name=f"{w.name}_div{args.shrink}", g=w.g // args.shrink, n=w.n // args.shrink,
+                                k_groups=min(w.k_groups, w.g // args.shrink))
+    return w
 
 
 # ----------------------------------------------------------------- plumbing
@@ -216,7 +229,7 @@ def run_reference(args, world, rank):
     """The float64 oracle on the host cores, same workload, metric and unit."""
     if rank != 0:
         return
-    w = workloads.WORKLOADS[args.workload]
+    w = workload_of(args)
     device = "cuda" if torch.cuda.is_available() else "cpu"
     entries, gid, centres = make_workload(w, args.seed, device, rank)
     qs = [workloads.make_queries(w, gid, centres, seed=args.seed, stream=4 + 10 * i) for i in range(args.batches)]
@@ -257,7 +270,7 @@ def run_reference(args, world, rank):
 def run_htam(args, world, rank, local):
     from paper_2605_29734_gb300 import htam
 
-    w = workloads.WORKLOADS[args.workload]
+    w = workload_of(args)
     dev = torch.device("cuda", local)
     stream = torch.cuda.current_stream(dev)
     props = torch.cuda.get_device_properties(dev)
@@ -267,6 +280,9 @@ def run_htam(args, world, rank, local):
     # The streaming workload appends once per step (warm-up, timed, end-to-end).
     capacity = w.n + (args.warmup + 2 * args.steps + 60) * w.append_per_round if w.rounds else w.n
     mem = htam.Memory(entries, gid, w.g, capacity=capacity)
+    if args.no_cpu_baseline:
+        del entries                  # the memory holds its own copy
+        torch.cuda.empty_cache()
     q_seed = args.seed + 1000 * rank
     batches = [workloads.make_queries(w, gid, centres, seed=q_seed, stream=4 + 10 * i) for i in range(args.batches)]
     append_batches = []
