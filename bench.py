@@ -181,20 +181,33 @@ def profiled_traffic(kernel: str, workload: str):
 
 # ------------------------------------------------------------- algorithmic work
 
+TC_MIN_BUCKET = 16   # the library's default: buckets this large go to the tensor-core kernel
+
+
 def step_work(w, counts: np.ndarray, group_idx: np.ndarray):
-    """Algorithmic bytes / flops of one query batch, from the groups it selected."""
+    """Algorithmic bytes / flops of one query batch, from the groups it selected:
+    each selected group's entries read once, the queries read once, and
+    2*D flops per (query, candidate entry); split between the CUDA-core kernel
+    (small buckets) and the tensor-core kernel (buckets of >= 16 queries)."""
     s = 2 if w.dtype == "bf16" else 4
-    sel = np.unique(group_idx[group_idx >= 0])
-    entries_read = float(counts[sel].sum())
-    n_b = np.where(group_idx >= 0, counts[np.clip(group_idx, 0, None)], 0).sum(axis=1)
     B, D, G = group_idx.shape[0], w.d, w.g
-    fine_bytes = entries_read * D * s + B * D * s
-    fine_flops = 2.0 * D * float(n_b.sum())
+    sel = group_idx[group_idx >= 0]
+    bucket = np.bincount(sel, minlength=G)                # queries per group
+    tc_on = w.dtype == "bf16" and w.k_entries <= 32 and TC_MIN_BUCKET <= B
+    is_tc = (bucket >= TC_MIN_BUCKET) & tc_on
+    touched = bucket > 0
+    n_b = np.where(group_idx >= 0, counts[np.clip(group_idx, 0, None)], 0).sum(axis=1)
+    work = {}
+    for name, mask in (("fine", touched & ~is_tc), ("fine_tc", touched & is_tc)):
+        entries_read = float(counts[mask].sum())
+        queries_read = float(bucket[mask].sum())          # bucket rows staged per kernel
+        work[name] = {"bytes": entries_read * D * s + min(B, queries_read) * D * s,
+                      "flops": 2.0 * D * float((bucket[mask] * counts[mask]).sum())}
     coarse_flops = 2.0 * D * B * G
     out_bytes = B * (w.k_groups * 8 + w.k_entries * 12 + 4)
-    step_bytes = fine_bytes + G * D * 4 + out_bytes
-    return {"fine_bytes": fine_bytes, "fine_flops": fine_flops, "step_bytes": step_bytes,
-            "step_flops": fine_flops + coarse_flops, "mean_candidates": float(n_b.mean())}
+    step_bytes = float(counts[touched].sum()) * D * s + B * D * s + G * D * 4 + out_bytes
+    return {"kernels": work, "step_bytes": step_bytes,
+            "step_flops": 2.0 * D * float(n_b.sum()) + coarse_flops, "mean_candidates": float(n_b.mean())}
 
 
 # --------------------------------------------------------------------- arms
@@ -340,21 +353,36 @@ def run_htam(args, world, rank, local):
     # Dominant kernel roofline (live CUDA events on the launching stream).
     peaks = load_peaks()
     per_batch = [work[(args.warmup + i) % len(work)] for i in range(args.steps)]
-    fine_bytes = float(np.mean([x["fine_bytes"] for x in per_batch]))
-    fine_flops = float(np.mean([x["fine_flops"] for x in per_batch]))
     step_bytes = float(np.mean([x["step_bytes"] for x in per_batch]))
     step_flops = float(np.mean([x["step_flops"] for x in per_batch]))
-    fine_ms, fine_launches = phases["fine"]
-    fine_s = fine_ms / 1e3 / max(1, fine_launches)
-    achieved = fine_bytes / fine_s / 1e9
-    kernel = "fine_simt"
-    roofline = {"kernel": kernel, "bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
-                "frac": achieved / peaks["hbm_gbs"],
-                "traffic": profiled_traffic(kernel, w.name), "peak_source": peaks["source"],
-                "algorithmic_bytes_per_launch": fine_bytes, "mean_launch_ms": fine_s * 1e3,
-                "flops_per_launch": fine_flops,
-                "alu_frac": fine_flops / fine_s / 1e12 / FP32_ALU_TFLOPS}
-    t_roof = max(step_bytes / (peaks["hbm_gbs"] * 1e9), step_flops / (FP32_ALU_TFLOPS * 1e12))
+    # The dominant kernel: the fine kernel (CUDA-core or tensor-core) with the
+    # most device time in the timed region.
+    phase = max(("fine", "fine_tc"), key=lambda k: phases[k][0])
+    kernel = {"fine": "fine_simt", "fine_tc": "fine_tc"}[phase]
+    k_ms, k_launches = phases[phase]
+    k_s = k_ms / 1e3 / max(1, k_launches)
+    k_bytes = float(np.mean([x["kernels"][phase]["bytes"] for x in per_batch]))
+    k_flops = float(np.mean([x["kernels"][phase]["flops"] for x in per_batch]))
+    if phase == "fine_tc":
+        tensor_peak = peaks["bf16_tflops_sustained"] or peaks["bf16_tflops"]
+        t_hbm = k_bytes / (peaks["hbm_gbs"] * 1e9)
+        t_tc = k_flops / (tensor_peak * 1e12)
+        if t_tc > t_hbm:
+            roofline = {"kernel": kernel, "bound": "tensor", "achieved": k_flops / k_s / 1e12, "peak": tensor_peak,
+                        "unit": "TFLOP/s", "peak_note": "measured sustained bf16"}
+        else:
+            roofline = {"kernel": kernel, "bound": "hbm", "achieved": k_bytes / k_s / 1e9, "peak": peaks["hbm_gbs"],
+                        "unit": "GB/s"}
+        roofline["tensor_frac"] = k_flops / k_s / 1e12 / tensor_peak
+    else:
+        roofline = {"kernel": kernel, "bound": "hbm", "achieved": k_bytes / k_s / 1e9, "peak": peaks["hbm_gbs"],
+                    "unit": "GB/s", "alu_frac": k_flops / k_s / 1e12 / FP32_ALU_TFLOPS}
+    roofline["frac"] = roofline["achieved"] / roofline["peak"]
+    roofline.update({"traffic": profiled_traffic(kernel, w.name), "peak_source": peaks["source"],
+                     "algorithmic_bytes_per_launch": k_bytes, "flops_per_launch": k_flops,
+                     "mean_launch_ms": k_s * 1e3, "hbm_frac": k_bytes / k_s / 1e9 / peaks["hbm_gbs"]})
+    t_roof = max(step_bytes / (peaks["hbm_gbs"] * 1e9),
+                 step_flops / ((peaks["bf16_tflops_sustained"] or peaks["bf16_tflops"]) * 1e12))
     step_s = total_s / args.steps
     launches = sum(v[1] for k, v in phases.items() if k != "queries")
 

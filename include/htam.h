@@ -187,10 +187,20 @@ typedef enum {
   HTAM_PHASE_COARSE = 0, /* group-key scores */
   HTAM_PHASE_SELECT = 1, /* top-k_groups per query */
   HTAM_PHASE_BUCKET = 2, /* group -> queries buckets and work units */
-  HTAM_PHASE_FINE = 3,   /* entry scores, softmax statistics, partial top-k */
-  HTAM_PHASE_MERGE = 4,  /* per-query merge, weights, outputs */
-  HTAM_N_PHASES = 5
+  HTAM_PHASE_FINE = 3,    /* entry scores of small buckets on the CUDA cores */
+  HTAM_PHASE_FINE_TC = 4, /* entry scores of large buckets on the tensor cores */
+  HTAM_PHASE_MERGE = 5,   /* per-query merge, weights, outputs */
+  HTAM_N_PHASES = 6
 } htam_phase;
+
+/* Tuning: when a group was selected by at least `min_bucket` queries of a
+ * batch, its entries are scored against those queries on the tensor cores
+ * (tcgen05, 128 queries per tile); smaller buckets are scored on the CUDA
+ * cores.  The tensor-core path needs a bf16 memory and k_entries <= 32.
+ * Default 16; a value above the batch size turns the tensor-core path off.
+ * Both paths return the same results within the fp32 rounding of the
+ * scores.  Errors: EINVAL (m NULL or min_bucket < 1). */
+htam_status htam_set_tensor_core_min_bucket(htam_memory *m, int32_t min_bucket);
 
 /* Turns CUDA-event timing of each htam_query phase on (1) or off (0).  While
  * on, every query records a pair of events around each phase on its stream

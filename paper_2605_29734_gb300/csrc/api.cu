@@ -211,6 +211,12 @@ htam_status htam_device_status(htam_memory *m, void *cuda_stream) {
   return word ? HTAM_ETIMEOUT : HTAM_OK;
 }
 
+htam_status htam_set_tensor_core_min_bucket(htam_memory *m, int32_t min_bucket) {
+  if (!m || min_bucket < 1) return HTAM_EINVAL;
+  m->tc_min = min_bucket;
+  return HTAM_OK;
+}
+
 htam_status htam_set_phase_timing(htam_memory *m, int enable) {
   if (!m) return HTAM_EINVAL;
   m->timing = enable != 0;

@@ -1,0 +1,51 @@
+// fine_tc.h -- tensor-core (tcgen05) fine-score kernel of the lookup.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "htam.h"
+
+namespace htam {
+
+constexpr int kTcRows = 128;      // queries per tensor-core work unit (MMA M)
+constexpr int kTcMaxK = 32;       // largest k_entries the tensor-core path keeps
+
+struct TcFineArgs {
+  const int4 *units;          // (group, bucket chunk, page segment)
+  const int32_t *n_units;     // device count of units
+  const int32_t *bucket;      // bucket rows -> query id
+  const int32_t *bucket_off;  // [G+1]
+  const int32_t *cnt;         // [G] bucket sizes
+  const int32_t *page_list;
+  const int32_t *page_off;
+  const int32_t *count;       // [G] entries per group
+  const int32_t *slot_id;
+  const int64_t *part_off;
+  int d;
+  int seg_pages;
+  int ke;
+  float k2;                   // log2(e) / tau
+  float2 *part_ml;
+  float *part_s;
+  int32_t *part_id;
+  unsigned *thr_enc;          // [B] order-preserving encoding of a lower bound of the k-th best score
+  unsigned *status;           // memory status word
+  uint32_t max_polls;
+};
+
+// Encodes a 2-D bf16 row-major [rows, cols] tensor for TMA tile loads of
+// box {64 columns, box_rows rows} with the 128-byte swizzle.
+htam_status make_bf16_tile_map(CUtensorMap *map, const void *base, uint64_t rows, uint64_t cols,
+                               uint32_t box_rows);
+
+// Queries gathered into bucket order, as the A operand of the kernel.
+htam_status launch_gather_queries(const void *Q, int d, const int32_t *bucket, const int32_t *bucket_group,
+                                  const int32_t *cnt, int tc_min, const int32_t *total_rows, int64_t max_rows,
+                                  void *Qg, cudaStream_t st);
+
+htam_status launch_fine_tc(const TcFineArgs &a, const CUtensorMap &q_map, const CUtensorMap &pool_map, int grid,
+                           cudaStream_t st);
+
+}  // namespace htam

@@ -1,6 +1,7 @@
 // internal.h -- the memory object behind the opaque htam_memory handle.
 #pragma once
 
+#include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -58,6 +59,12 @@ struct htam_memory {
   size_t ev_used = 0;                  // events in use (2 per pair)
   int64_t n_queries = 0;
   int64_t phase_launches[HTAM_N_PHASES] = {};
+
+  // Tensor-core fine path: smallest bucket it takes, and the TMA map of the
+  // page pool (built on first use).
+  int tc_min = 16;
+  CUtensorMap pool_map;
+  bool pool_map_ready = false;
 };
 
 namespace htam {

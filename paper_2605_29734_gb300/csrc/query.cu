@@ -17,6 +17,7 @@
 #include <vector>
 
 #include "common.cuh"
+#include "fine_tc.h"
 #include "internal.h"
 
 namespace htam {
@@ -152,74 +153,91 @@ __global__ void bucket_count_kernel(const uint32_t *__restrict__ bits, int G, in
   if (lane == 0) cnt[g] = c;
 }
 
-// Single block: per group the bucket size c_g, its work units
-// ceil(c_g/qc) * nseg_g and partial records c_g * nseg_g, with exclusive
-// scans over the groups.  nseg_g = ceil(pages_g / seg_pages).
+// Which fine kernel scores a group's bucket: buckets of at least tc_min
+// queries go to the tensor-core kernel in chunks of 128 queries and page
+// segments of seg_tc pages, smaller ones to the SIMT kernel in chunks of
+// qc_simt queries and segments of seg_simt pages.
+struct Route {
+  int tc_min, qc_simt, seg_simt, seg_tc;
+  __host__ __device__ bool tc(int c) const { return c >= tc_min; }
+  __host__ __device__ int qc(int c) const { return tc(c) ? kTcRows : qc_simt; }
+  __host__ __device__ int seg(int c) const { return tc(c) ? seg_tc : seg_simt; }
+  __host__ __device__ int nseg(int c, int pages) const { return (pages + seg(c) - 1) / seg(c); }
+  __host__ __device__ int64_t units(int c, int pages) const {
+    return c > 0 ? (int64_t)((c + qc(c) - 1) / qc(c)) * nseg(c, pages) : 0;
+  }
+};
+
+// Single block: per group the bucket size c_g, its work units (in the SIMT or
+// the tensor-core list) and its partial records c_g * nseg_g, with exclusive
+// scans over the groups.  n_units = {SIMT units, tensor-core units}.
 __global__ void __launch_bounds__(1024) bucket_scan_kernel(
-    const int32_t *__restrict__ cnt, const int32_t *__restrict__ page_off, int G, int qc,
-    int seg_pages, int32_t *__restrict__ bucket_off, int32_t *__restrict__ unit_off,
+    const int32_t *__restrict__ cnt, const int32_t *__restrict__ page_off, int G, Route rt,
+    int32_t *__restrict__ bucket_off, int32_t *__restrict__ unit_off, int32_t *__restrict__ unit_off_tc,
     int64_t *__restrict__ part_off, int32_t *__restrict__ n_units) {
-  __shared__ int64_t sh[3][1024];
+  __shared__ int64_t sh[4][1024];
   const int tid = threadIdx.x;
   const int per = (G + 1023) / 1024;
   const int lo = min(G, tid * per), hi = min(G, lo + per);
-  int64_t a = 0, u = 0, p = 0;
+  int64_t a = 0, u = 0, t = 0, p = 0;
   for (int g = lo; g < hi; ++g) {
-    int c = cnt[g];
-    int nseg = (page_off[g + 1] - page_off[g] + seg_pages - 1) / seg_pages;
+    int c = cnt[g], pages = page_off[g + 1] - page_off[g];
     a += c;
-    u += c > 0 ? (int64_t)((c + qc - 1) / qc) * nseg : 0;
-    p += (int64_t)c * nseg;
+    (rt.tc(c) ? t : u) += rt.units(c, pages);
+    p += (int64_t)c * rt.nseg(c, pages);
   }
   sh[0][tid] = a;
   sh[1][tid] = u;
-  sh[2][tid] = p;
+  sh[2][tid] = t;
+  sh[3][tid] = p;
   __syncthreads();
   for (int o = 1; o < 1024; o <<= 1) {
-    int64_t va = 0, vu = 0, vp = 0;
+    int64_t v[4] = {0, 0, 0, 0};
     if (tid >= o) {
-      va = sh[0][tid - o];
-      vu = sh[1][tid - o];
-      vp = sh[2][tid - o];
+      for (int i = 0; i < 4; ++i) v[i] = sh[i][tid - o];
     }
     __syncthreads();
-    sh[0][tid] += va;
-    sh[1][tid] += vu;
-    sh[2][tid] += vp;
+    for (int i = 0; i < 4; ++i) sh[i][tid] += v[i];
     __syncthreads();
   }
   a = sh[0][tid] - a;
   u = sh[1][tid] - u;
-  p = sh[2][tid] - p;
+  t = sh[2][tid] - t;
+  p = sh[3][tid] - p;
   for (int g = lo; g < hi; ++g) {
-    int c = cnt[g];
-    int nseg = (page_off[g + 1] - page_off[g] + seg_pages - 1) / seg_pages;
+    int c = cnt[g], pages = page_off[g + 1] - page_off[g];
     bucket_off[g] = (int32_t)a;
     unit_off[g] = (int32_t)u;
+    unit_off_tc[g] = (int32_t)t;
     part_off[g] = p;
     a += c;
-    u += c > 0 ? (int64_t)((c + qc - 1) / qc) * nseg : 0;
-    p += (int64_t)c * nseg;
+    (rt.tc(c) ? t : u) += rt.units(c, pages);
+    p += (int64_t)c * rt.nseg(c, pages);
   }
   if (tid == 1023) {
     bucket_off[G] = (int32_t)a;
     unit_off[G] = (int32_t)u;
+    unit_off_tc[G] = (int32_t)t;
     part_off[G] = p;
-    *n_units = (int32_t)u;
+    n_units[0] = (int32_t)u;
+    n_units[1] = (int32_t)t;
   }
 }
 
 // One warp per group: bucket[g] lists its queries in increasing order;
 // pos[b][j] = rank of query b in the bucket of its j-th selected group.
-// Also writes the group's work units (group, chunk, segment).
+// Also writes the group's work units (group, chunk, segment) to the list of
+// the kernel that will score them, and the group of every bucket row.
 __global__ void bucket_fill_kernel(const uint32_t *__restrict__ bits, int G, int W,
                                    const int32_t *__restrict__ bucket_off,
                                    const int32_t *__restrict__ gidx, int kg,
                                    const int32_t *__restrict__ cnt,
-                                   const int32_t *__restrict__ page_off, int qc, int seg_pages,
+                                   const int32_t *__restrict__ page_off, Route rt,
                                    const int32_t *__restrict__ unit_off,
-                                   int32_t *__restrict__ bucket, int32_t *__restrict__ pos,
-                                   int4 *__restrict__ units) {
+                                   const int32_t *__restrict__ unit_off_tc,
+                                   int32_t *__restrict__ bucket, int32_t *__restrict__ bucket_group,
+                                   int32_t *__restrict__ pos, int4 *__restrict__ units,
+                                   int4 *__restrict__ units_tc) {
   int g = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   int lane = threadIdx.x & 31;
   if (g >= G) return;
@@ -239,6 +257,7 @@ __global__ void bucket_fill_kernel(const uint32_t *__restrict__ bits, int G, int
       word &= word - 1;
       int b = (w0 + lane) * 32 + bit;
       bucket[base + r] = b;
+      bucket_group[base + r] = g;
       for (int j = 0; j < kg; ++j) {
         if (gidx[(int64_t)b * kg + j] == g) pos[(int64_t)b * kg + j] = r;
       }
@@ -248,9 +267,11 @@ __global__ void bucket_fill_kernel(const uint32_t *__restrict__ bits, int G, int
   }
   int c = cnt[g];
   if (c == 0) return;
-  int nseg = (page_off[g + 1] - page_off[g] + seg_pages - 1) / seg_pages;
-  int n_u = ((c + qc - 1) / qc) * nseg;
-  for (int u = lane; u < n_u; u += 32) units[unit_off[g] + u] = make_int4(g, u / nseg, u % nseg, 0);
+  const int pages = page_off[g + 1] - page_off[g];
+  const int nseg = rt.nseg(c, pages);
+  const int n_u = (int)rt.units(c, pages);
+  int4 *dst = rt.tc(c) ? units_tc + unit_off_tc[g] : units + unit_off[g];
+  for (int u = lane; u < n_u; u += 32) dst[u] = make_int4(g, u / nseg, u % nseg, 0);
 }
 
 // ------------------------------------------------------------ fine (SIMT)
@@ -477,7 +498,7 @@ struct MergeArgs {
   const int32_t *pos;
   const int32_t *cnt;
   const int32_t *page_off;
-  int seg_pages;
+  Route rt;
   const int64_t *part_off;
   const float2 *part_ml;
   const float *part_s;
@@ -505,7 +526,7 @@ __global__ void merge_kernel(MergeArgs a) {
     if (g < 0) continue;
     int p = a.pos[(int64_t)b * a.kg + j];
     int cg = a.cnt[g];
-    int nseg = (a.page_off[g + 1] - a.page_off[g] + a.seg_pages - 1) / a.seg_pages;
+    int nseg = a.rt.nseg(cg, a.page_off[g + 1] - a.page_off[g]);
     nb += a.count[g];
     for (int s = 0; s < nseg; ++s) {
       int64_t pidx = a.part_off[g] + (int64_t)s * cg + p;
@@ -588,6 +609,8 @@ static int simt_query_chunk(int d) {
 }
 
 constexpr int kSimtSegPages = 4;
+constexpr int kTcSegPages = 16;
+constexpr uint32_t kMaxPolls = 1u << 24;
 
 htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const htam_query_params &p,
                        int32_t *group_idx, float *group_score, int32_t *entry_idx,
@@ -597,25 +620,31 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   PhaseMark mark(m, st);
   const int G = m->n_groups, d = m->d, kg = p.k_groups, ke = p.k_entries;
   const int qc = simt_query_chunk(d);
-  const int seg = kSimtSegPages;
+  // The tensor-core path takes bf16 memories and k_entries <= 32.
+  const bool tc_ok = m->dtype == HTAM_BF16 && ke <= kTcMaxK && m->tc_min <= B;
+  const Route rt{tc_ok ? m->tc_min : INT_MAX, qc, kSimtSegPages, kTcSegPages};
 
   // Upper bound of the partial records: every query in the buckets of the
-  // k_g groups with the most page segments.
+  // k_g groups with the most page segments (counted with the shorter
+  // segments of the two kernels).
+  const int seg_min = std::min(kSimtSegPages, kTcSegPages);
   std::vector<int64_t> nseg(G);
-  for (int g = 0; g < G; ++g) nseg[g] = ceil_div((int64_t)m->h_pages[g].size(), seg);
-  std::vector<int64_t> top = nseg;
-  std::nth_element(top.begin(), top.begin() + (kg - 1), top.end(), std::greater<int64_t>());
+  for (int g = 0; g < G; ++g) nseg[g] = ceil_div((int64_t)m->h_pages[g].size(), seg_min);
+  std::nth_element(nseg.begin(), nseg.begin() + (kg - 1), nseg.end(), std::greater<int64_t>());
   int64_t seg_sum = 0;
-  for (int i = 0; i < kg; ++i) seg_sum += top[i];
+  for (int i = 0; i < kg; ++i) seg_sum += nseg[i];
   const int64_t max_parts = std::max<int64_t>(1, (int64_t)B * seg_sum);
   const int64_t max_units = max_parts;
+  const int64_t rows = (int64_t)B * kg;  // bucket rows
   const int W = (int)ceil_div(B, 32);
+  const size_t qg_bytes = tc_ok ? sizeof(__nv_bfloat16) * (size_t)rows * d : 0;
 
   size_t need = Carver::round(sizeof(float) * (size_t)B * G) + Carver::round(sizeof(uint32_t) * (size_t)G * W) +
-                4 * Carver::round(sizeof(int32_t) * (G + 1)) + Carver::round(sizeof(int64_t) * (G + 1)) +
-                2 * Carver::round(sizeof(int32_t) * (size_t)B * kg) + Carver::round(sizeof(int4) * max_units) +
+                5 * Carver::round(sizeof(int32_t) * (G + 1)) + Carver::round(sizeof(int64_t) * (G + 1)) +
+                3 * Carver::round(sizeof(int32_t) * rows) + 2 * Carver::round(sizeof(int4) * max_units) +
                 Carver::round(sizeof(float2) * max_parts) + Carver::round(sizeof(float) * max_parts * ke) +
-                Carver::round(sizeof(int32_t) * max_parts * ke) + Carver::round(64) + 4096;
+                Carver::round(sizeof(int32_t) * max_parts * ke) + Carver::round(sizeof(unsigned) * B) +
+                Carver::round(qg_bytes) + 8192;
   htam_status s = ensure_scratch(m, need);
   if (s != HTAM_OK) return s;
   Carver cv(m->scratch);
@@ -624,14 +653,19 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   int32_t *cnt = cv.take<int32_t>(G + 1);
   int32_t *bucket_off = cv.take<int32_t>(G + 1);
   int32_t *unit_off = cv.take<int32_t>(G + 1);
+  int32_t *unit_off_tc = cv.take<int32_t>(G + 1);
   int64_t *part_off = cv.take<int64_t>(G + 1);
-  int32_t *n_units = cv.take<int32_t>(G + 1);
-  int32_t *bucket = cv.take<int32_t>((size_t)B * kg);
-  int32_t *pos = cv.take<int32_t>((size_t)B * kg);
+  int32_t *n_units = cv.take<int32_t>(G + 1);  // [0] SIMT units, [1] tensor-core units
+  int32_t *bucket = cv.take<int32_t>(rows);
+  int32_t *bucket_group = cv.take<int32_t>(rows);
+  int32_t *pos = cv.take<int32_t>(rows);
   int4 *units = cv.take<int4>(max_units);
+  int4 *units_tc = cv.take<int4>(max_units);
   float2 *part_ml = cv.take<float2>(max_parts);
   float *part_s = cv.take<float>(max_parts * ke);
   int32_t *part_id = cv.take<int32_t>(max_parts * ke);
+  unsigned *thr_enc = cv.take<unsigned>(B);
+  void *qg = tc_ok ? static_cast<void *>(cv.take<char>(qg_bytes)) : nullptr;
 
   // 1. Coarse scores and the selected groups.
   {
@@ -658,31 +692,61 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   // 2. Buckets: group -> queries, work units, partial-record offsets.
   mark.begin(HTAM_PHASE_BUCKET);
   HTAM_CK(cudaMemsetAsync(bits, 0, sizeof(uint32_t) * (size_t)G * W, st));
-  bucket_bits_kernel<<<(unsigned)ceil_div((int64_t)B * kg, 256), 256, 0, st>>>(group_idx, B, kg, W, bits);
+  bucket_bits_kernel<<<(unsigned)ceil_div(rows, 256), 256, 0, st>>>(group_idx, B, kg, W, bits);
   HTAM_CK_LAUNCH("bucket_bits_kernel");
   bucket_count_kernel<<<(unsigned)ceil_div((int64_t)G * 32, 256), 256, 0, st>>>(bits, G, W, cnt);
   HTAM_CK_LAUNCH("bucket_count_kernel");
-  bucket_scan_kernel<<<1, 1024, 0, st>>>(cnt, m->page_off, G, qc, seg, bucket_off, unit_off, part_off, n_units);
+  bucket_scan_kernel<<<1, 1024, 0, st>>>(cnt, m->page_off, G, rt, bucket_off, unit_off, unit_off_tc, part_off,
+                                         n_units);
   HTAM_CK_LAUNCH("bucket_scan_kernel");
   bucket_fill_kernel<<<(unsigned)ceil_div((int64_t)G * 32, 256), 256, 0, st>>>(
-      bits, G, W, bucket_off, group_idx, kg, cnt, m->page_off, qc, seg, unit_off, bucket, pos, units);
+      bits, G, W, bucket_off, group_idx, kg, cnt, m->page_off, rt, unit_off, unit_off_tc, bucket, bucket_group,
+      pos, units, units_tc);
   HTAM_CK_LAUNCH("bucket_fill_kernel");
   mark.launched(4);
+  CUtensorMap q_map;
+  if (tc_ok) {
+    // Queries of tensor-core buckets in bucket order (the MMA's A operand),
+    // and the per-query score bounds the tensor-core units share.
+    if (!m->pool_map_ready) {
+      s = make_bf16_tile_map(&m->pool_map, m->pool, (uint64_t)m->n_pages_max * kPageRows, d, kPageRows);
+      if (s != HTAM_OK) return s;
+      m->pool_map_ready = true;
+    }
+    s = make_bf16_tile_map(&q_map, qg, rows, d, kTcRows);
+    if (s != HTAM_OK) return s;
+    HTAM_CK(cudaMemsetAsync(thr_enc, 0, sizeof(unsigned) * B, st));
+    s = launch_gather_queries(queries, d, bucket, bucket_group, cnt, rt.tc_min, bucket_off + G, rows, qg, st);
+    if (s != HTAM_OK) return s;
+    mark.launched();
+  }
   mark.end();
 
-  // 3. Fine scores with fused softmax statistics and top-k.
+  // 3a. Fine scores of small buckets on the CUDA cores.
   mark.begin(HTAM_PHASE_FINE);
   FineArgs fa{m->pool, d, m->slot_id, m->page_list, m->page_off, m->count, queries, bucket, bucket_off,
-              cnt, units, n_units, part_off, ke, 1.0f / p.tau, seg, part_ml, part_s, part_id};
+              cnt, units, n_units, part_off, ke, 1.0f / p.tau, kSimtSegPages, part_ml, part_s, part_id};
   s = m->dtype == HTAM_BF16 ? dispatch_fine_simt<__nv_bfloat16>(qc, fa, m->sm_count, max_units, st)
                             : dispatch_fine_simt<float>(qc, fa, m->sm_count, max_units, st);
   if (s != HTAM_OK) return s;
   mark.launched();
   mark.end();
 
+  // 3b. Fine scores of large buckets on the tensor cores.
+  if (tc_ok) {
+    mark.begin(HTAM_PHASE_FINE_TC);
+    TcFineArgs ta{units_tc, n_units + 1, bucket, bucket_off, cnt, m->page_list, m->page_off, m->count, m->slot_id,
+                  part_off, d, kTcSegPages, ke, 1.4426950408889634f / p.tau, part_ml, part_s, part_id, thr_enc,
+                  m->status, kMaxPolls};
+    s = launch_fine_tc(ta, q_map, m->pool_map, (int)std::min<int64_t>(max_units, m->sm_count), st);
+    if (s != HTAM_OK) return s;
+    mark.launched();
+    mark.end();
+  }
+
   // 4. Merge per query.
   mark.begin(HTAM_PHASE_MERGE);
-  MergeArgs ma{group_idx, B, kg, ke, m->count, pos, cnt, m->page_off, seg, part_off, part_ml, part_s,
+  MergeArgs ma{group_idx, B, kg, ke, m->count, pos, cnt, m->page_off, rt, part_off, part_ml, part_s,
                part_id, 1.0f / p.tau, p.epsilon, entry_idx, entry_score, entry_weight, lse};
   merge_kernel<<<(unsigned)ceil_div((int64_t)B * 32, 256), 256, 0, st>>>(ma);
   HTAM_CK_LAUNCH("merge_kernel");

@@ -194,6 +194,52 @@ def test_large_groups_many_segments_ragged_tail(htam):
     _check(htam, mem, entries, gid, 6, q, 2, 33)
 
 
+# ------------------------------------------- tensor-core and CUDA-core paths
+
+TC_CASES = [
+    # n, groups, d, batch, k_groups, k_entries: several 128-query chunks per
+    # bucket, groups spanning several 16-page segments, ragged last pages
+    (60000, 8, 256, 300, 3, 20),
+    # d not a multiple of the 64-column K slice; k_entries at the tensor-core limit
+    (20000, 50, 1000, 130, 10, 32),
+    # one group, one page: a single tile of one page
+    (100, 1, 64, 40, 1, 5),
+]
+
+
+@pytest.mark.parametrize("case", TC_CASES)
+@pytest.mark.parametrize("min_bucket", [1, 16, 1 << 30])
+def test_tensor_core_and_cuda_core_paths(htam, case, min_bucket):
+    n, g, d, b, kg, ke = case
+    entries, gid, centres = _rand_memory(n, d, g, torch.bfloat16, seed=n + d)
+    q = _rand_queries(b, d, torch.bfloat16, seed=n + d, centres=centres)
+    mem = htam.Memory(entries, gid, g)
+    mem.set_tensor_core_min_bucket(min_bucket)
+    mem.read_phase_timing()
+    _check(htam, mem, entries, gid, g, q, kg, ke, tau=0.5, eps=0.05)
+    ran = mem.read_phase_timing()
+    if min_bucket == 1:
+        assert ran["fine_tc"][1] > 0
+    if min_bucket == 1 << 30:
+        assert ran["fine_tc"][1] == 0
+
+
+def test_paths_agree_on_the_zipf_65k_workload(htam):
+    w = workloads.WORKLOADS["zipf_bf16_65k"]
+    entries, gid, centres = workloads.make_memory(w, seed=0, device=DEV)
+    q = workloads.make_queries(w, gid, centres, seed=0)
+    mem = htam.Memory(entries, gid, w.g)
+    outs = []
+    for min_bucket in (1, 1 << 30):
+        mem.set_tensor_core_min_bucket(min_bucket)
+        outs.append({k: v.clone() for k, v in mem.query(q, w.k_groups, w.k_entries).items()})
+    torch.cuda.synchronize()
+    assert torch.equal(outs[0]["group_idx"], outs[1]["group_idx"])
+    same = (outs[0]["entry_idx"] == outs[1]["entry_idx"]).float().mean().item()
+    assert same > 0.99
+    torch.testing.assert_close(outs[0]["lse"], outs[1]["lse"], rtol=1e-4, atol=1e-4)
+
+
 # ---------------------------------------------------------------- append path
 
 @pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
