@@ -127,18 +127,22 @@ struct RowTopK {
     }
   }
 
-  // Inserts one pair; the worst pair falls off the end.
+  // Inserts one pair; the worst pair falls off the end.  The list is sorted,
+  // so "slot i stays better than x" holds for a prefix of the slots: slot i
+  // keeps its pair, takes x, or takes slot i-1's pair depending only on its
+  // own and its neighbour's comparison -- no dependency chain through the
+  // list.
   __device__ __forceinline__ void insert(float xs, int xc) {
+    bool keep[K];
 #pragma unroll
-    for (int i = 0; i < K; ++i) {
-      const bool sw = better(xs, xc, s[i], c[i]);
-      const float ts = s[i];
-      const int tc = c[i];
-      s[i] = sw ? xs : s[i];
-      c[i] = sw ? xc : c[i];
-      xs = sw ? ts : xs;
-      xc = sw ? tc : xc;
+    for (int i = 0; i < K; ++i) keep[i] = better(s[i], c[i], xs, xc);
+#pragma unroll
+    for (int i = K - 1; i >= 1; --i) {
+      s[i] = keep[i] ? s[i] : (keep[i - 1] ? xs : s[i - 1]);
+      c[i] = keep[i] ? c[i] : (keep[i - 1] ? xc : c[i - 1]);
     }
+    s[0] = keep[0] ? s[0] : xs;
+    c[0] = keep[0] ? c[0] : xc;
   }
 
   // Merges 32 pairs sorted best first: the K best of the union are the
@@ -399,18 +403,21 @@ __global__ void __launch_bounds__(kThreads, 1)
             } else {
               // Sparse chunk: insert the flagged pairs one by one.
               for (int it = 0; it < most; ++it) {
-                const int j = flagged ? __ffs(flagged) - 1 : -1;
+                const bool any = flagged != 0u;
+                const int j = any ? __ffs(flagged) - 1 : 0;
                 flagged &= flagged - 1;
-                float xs = -INFINITY;
-                int xc = INT_MAX;
+                // r[j] through a 5-level select tree on the bits of j.
+                uint32_t t16[16], t8[8], t4[4], t2[2];
 #pragma unroll
-                for (int jj = 0; jj < 32; ++jj) {
-                  if (jj == j) {
-                    xs = __uint_as_float(r[jj]);
-                    xc = cbase + jj;
-                  }
-                }
-                top.insert(xs, xc);
+                for (int i = 0; i < 16; ++i) t16[i] = (j & 1) ? r[2 * i + 1] : r[2 * i];
+#pragma unroll
+                for (int i = 0; i < 8; ++i) t8[i] = (j & 2) ? t16[2 * i + 1] : t16[2 * i];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) t4[i] = (j & 4) ? t8[2 * i + 1] : t8[2 * i];
+#pragma unroll
+                for (int i = 0; i < 2; ++i) t2[i] = (j & 8) ? t4[2 * i + 1] : t4[2 * i];
+                const uint32_t xv = (j & 16) ? t2[1] : t2[0];
+                top.insert(any ? __uint_as_float(xv) : -INFINITY, any ? cbase + j : INT_MAX);
               }
             }
             if (valid) thr = fmaxf(thr, top.kth(k));
