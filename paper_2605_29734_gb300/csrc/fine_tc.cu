@@ -127,15 +127,17 @@ struct RowTopK {
     }
   }
 
-  // Inserts one pair; the worst pair falls off the end.  The list is sorted,
-  // so "slot i stays better than x" holds for a prefix of the slots: slot i
-  // keeps its pair, takes x, or takes slot i-1's pair depending only on its
-  // own and its neighbour's comparison -- no dependency chain through the
-  // list.
-  __device__ __forceinline__ void insert(float xs, int xc) {
+  // Inserts one pair whose column is above every column in the list (the
+  // epilogue visits columns in increasing order), so on equal scores the
+  // pair already in the list wins, which is the lower-column (lower-id) rule;
+  // the worst pair falls off the end.  The list is sorted, so "slot i stays
+  // ahead of x" holds for a prefix of the slots: slot i keeps its pair, takes
+  // x, or takes slot i-1's pair depending only on its own and its
+  // neighbour's comparison -- no dependency chain through the list.
+  __device__ __forceinline__ void insert_later(float xs, int xc) {
     bool keep[K];
 #pragma unroll
-    for (int i = 0; i < K; ++i) keep[i] = better(s[i], c[i], xs, xc);
+    for (int i = 0; i < K; ++i) keep[i] = s[i] >= xs;
 #pragma unroll
     for (int i = K - 1; i >= 1; --i) {
       s[i] = keep[i] ? s[i] : (keep[i - 1] ? xs : s[i - 1]);
@@ -417,7 +419,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                 for (int i = 0; i < 2; ++i) t2[i] = (j & 8) ? t4[2 * i + 1] : t4[2 * i];
                 const uint32_t xv = (j & 16) ? t2[1] : t2[0];
-                top.insert(any ? __uint_as_float(xv) : -INFINITY, any ? cbase + j : INT_MAX);
+                if (any) top.insert_later(__uint_as_float(xv), cbase + j);
               }
             }
             if (valid) thr = fmaxf(thr, top.kth(k));

@@ -224,6 +224,25 @@ def test_tensor_core_and_cuda_core_paths(htam, case, min_bucket):
         assert ran["fine_tc"][1] == 0
 
 
+@pytest.mark.parametrize("min_bucket", [1, 1 << 30])
+def test_duplicate_bf16_rows_tie_to_lower_id_on_both_paths(htam, min_bucket):
+    """Exactly equal scores (duplicate rows spread over pages and chunks)
+    must come out in entry-id order on both fine kernels."""
+    base, _, _ = _rand_memory(40, 128, 1, torch.bfloat16, seed=22, clustered=False)
+    entries = base.repeat(100, 1).contiguous()            # 4,000 rows, each value 100 times
+    gid = (torch.arange(4000, device=DEV) % 2).to(torch.int32)
+    q = _rand_queries(50, 128, torch.bfloat16, seed=22)
+    mem = htam.Memory(entries, gid, 2)
+    mem.set_tensor_core_min_bucket(min_bucket)
+    _check(htam, mem, entries, gid, 2, q, 2, 32)
+    out = mem.query(q, 2, 32)
+    torch.cuda.synchronize()
+    ids, sc = out["entry_idx"].cpu().numpy(), out["entry_score"].cpu().numpy()
+    for b in range(50):
+        for i in range(31):
+            assert sc[b, i] > sc[b, i + 1] or (sc[b, i] == sc[b, i + 1] and ids[b, i] < ids[b, i + 1])
+
+
 def test_paths_agree_on_the_zipf_65k_workload(htam):
     w = workloads.WORKLOADS["zipf_bf16_65k"]
     entries, gid, centres = workloads.make_memory(w, seed=0, device=DEV)
