@@ -326,8 +326,8 @@ struct Unpack<float> {
 // with shuffles and keeps, per query, the online softmax state (max, sum of
 // exp) and a warp-distributed top-k; the warps are merged in shared memory
 // and one partial record per (query, unit) is written.
-template <typename T, int QC>
-__global__ void __launch_bounds__(kFineWarps * 32) fine_simt_kernel(FineArgs a) {
+template <typename T, int QC, int B>
+__global__ void __launch_bounds__(kFineWarps * 32, 2) fine_simt_kernel(FineArgs a) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   constexpr int kN = Unpack<T>::kN;
   const int d = a.d;
@@ -392,21 +392,33 @@ __global__ void __launch_bounds__(kFineWarps * 32) fine_simt_kernel(FineArgs a) 
       float acc[QC];
 #pragma unroll
       for (int j = 0; j < QC; ++j) acc[j] = 0.f;
-      for (int v = lane; v < n_vec; v += 32) {
-        uint4 w = row[v];
-        float f[kN];
-        Unpack<T>::run(w, f);
+      // B 16-byte loads per lane are issued before any is used, so each warp
+      // keeps B * 512 bytes of the row in flight.
+      for (int v0 = lane; v0 < n_vec; v0 += 32 * B) {
+        uint4 w[B];
 #pragma unroll
-        for (int j = 0; j < QC; ++j) {
-          if (j < nq) {
-            const float *q = qs + j * d + v * kN;
+        for (int i = 0; i < B; ++i) {
+          const int v = v0 + 32 * i;
+          w[i] = v < n_vec ? row[v] : make_uint4(0u, 0u, 0u, 0u);
+        }
 #pragma unroll
-            for (int t = 0; t < kN; t += 4) {
-              float4 qq = *reinterpret_cast<const float4 *>(q + t);
-              acc[j] = fmaf(f[t], qq.x, acc[j]);
-              acc[j] = fmaf(f[t + 1], qq.y, acc[j]);
-              acc[j] = fmaf(f[t + 2], qq.z, acc[j]);
-              acc[j] = fmaf(f[t + 3], qq.w, acc[j]);
+        for (int i = 0; i < B; ++i) {
+          const int v = v0 + 32 * i;
+          if (v >= n_vec) break;
+          float f[kN];
+          Unpack<T>::run(w[i], f);
+#pragma unroll
+          for (int j = 0; j < QC; ++j) {
+            if (j < nq) {
+              const float *q = qs + j * d + v * kN;
+#pragma unroll
+              for (int t = 0; t < kN; t += 4) {
+                float4 qq = *reinterpret_cast<const float4 *>(q + t);
+                acc[j] = fmaf(f[t], qq.x, acc[j]);
+                acc[j] = fmaf(f[t + 1], qq.y, acc[j]);
+                acc[j] = fmaf(f[t + 2], qq.z, acc[j]);
+                acc[j] = fmaf(f[t + 3], qq.w, acc[j]);
+              }
             }
           }
         }
@@ -572,29 +584,46 @@ __global__ void merge_kernel(MergeArgs a) {
   if (a.lse && lane == 0) a.lse[b] = lse_b;
 }
 
-template <typename T, int QC>
+template <typename T, int QC, int B>
 htam_status launch_fine_simt(const FineArgs &fa, int sm_count, int64_t max_units, cudaStream_t st) {
   const int d = fa.d;
   size_t smem = sizeof(float) * QC * d + (sizeof(float) + sizeof(int)) * kFineWarps * QC * 64 +
                 sizeof(float) * 2 * kFineWarps * QC;
-  HTAM_CK(cudaFuncSetAttribute(fine_simt_kernel<T, QC>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+  auto kernel = fine_simt_kernel<T, QC, B>;
+  HTAM_CK(cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
   int per_sm = 0;
-  HTAM_CK(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fine_simt_kernel<T, QC>, kFineWarps * 32, smem));
+  HTAM_CK(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, kFineWarps * 32, smem));
   per_sm = std::max(per_sm, 1);
   int64_t grid = std::min<int64_t>(max_units, (int64_t)sm_count * per_sm);
   if (grid <= 0) return HTAM_OK;
-  fine_simt_kernel<T, QC><<<(unsigned)grid, kFineWarps * 32, smem, st>>>(fa);
+  kernel<<<(unsigned)grid, kFineWarps * 32, smem, st>>>(fa);
   HTAM_CK_LAUNCH("fine_simt_kernel");
   return HTAM_OK;
+}
+
+// Loads in flight per lane: enough 16-byte vectors for one row, at most
+// 32 / QC (so that two blocks of 256 threads fit an SM's registers).
+template <typename T, int QC>
+htam_status dispatch_batch(const FineArgs &fa, int sm_count, int64_t max_units, cudaStream_t st) {
+  const int per_lane = (int)ceil_div((int64_t)fa.d * (int)sizeof(T) / 16, 32);
+  if constexpr (QC <= 2) {
+    if (per_lane >= 16) return launch_fine_simt<T, QC, 16>(fa, sm_count, max_units, st);
+  }
+  if constexpr (QC <= 4) {
+    if (per_lane > 4) return launch_fine_simt<T, QC, 8>(fa, sm_count, max_units, st);
+  }
+  if (per_lane > 2) return launch_fine_simt<T, QC, 4>(fa, sm_count, max_units, st);
+  if (per_lane > 1) return launch_fine_simt<T, QC, 2>(fa, sm_count, max_units, st);
+  return launch_fine_simt<T, QC, 1>(fa, sm_count, max_units, st);
 }
 
 template <typename T>
 htam_status dispatch_fine_simt(int qc, const FineArgs &fa, int sm_count, int64_t max_units, cudaStream_t st) {
   switch (qc) {
-    case 8: return launch_fine_simt<T, 8>(fa, sm_count, max_units, st);
-    case 4: return launch_fine_simt<T, 4>(fa, sm_count, max_units, st);
-    case 2: return launch_fine_simt<T, 2>(fa, sm_count, max_units, st);
-    default: return launch_fine_simt<T, 1>(fa, sm_count, max_units, st);
+    case 8: return dispatch_batch<T, 8>(fa, sm_count, max_units, st);
+    case 4: return dispatch_batch<T, 4>(fa, sm_count, max_units, st);
+    case 2: return dispatch_batch<T, 2>(fa, sm_count, max_units, st);
+    default: return dispatch_batch<T, 1>(fa, sm_count, max_units, st);
   }
 }
 
