@@ -54,6 +54,11 @@ def parse_args():
     ap.add_argument("--shrink", type=int, default=1,
                     help="divide the workload's groups and entries by this factor (same group sizes); "
                          "for small profiling captures only")
+    ap.add_argument("--stream-rows", type=int, default=None, choices=[0, 1],
+                    help="CUDA-core path: stream rows through shared memory (1, library default) or load "
+                         "them directly (0)")
+    ap.add_argument("--tc-min-bucket", type=int, default=None,
+                    help="smallest bucket scored on the tensor cores (library default 16)")
     return ap.parse_args()
 
 
@@ -184,7 +189,7 @@ def profiled_traffic(kernel: str, workload: str):
 TC_MIN_BUCKET = 16   # the library's default: buckets this large go to the tensor-core kernel
 
 
-def step_work(w, counts: np.ndarray, group_idx: np.ndarray):
+def step_work(w, counts: np.ndarray, group_idx: np.ndarray, tc_min: int = TC_MIN_BUCKET):
     """Algorithmic bytes / flops of one query batch, from the groups it selected:
     each selected group's entries read once, the queries read once, and
     2*D flops per (query, candidate entry); split between the CUDA-core kernel
@@ -193,8 +198,8 @@ def step_work(w, counts: np.ndarray, group_idx: np.ndarray):
     B, D, G = group_idx.shape[0], w.d, w.g
     sel = group_idx[group_idx >= 0]
     bucket = np.bincount(sel, minlength=G)                # queries per group
-    tc_on = w.dtype == "bf16" and w.k_entries <= 32 and TC_MIN_BUCKET <= B
-    is_tc = (bucket >= TC_MIN_BUCKET) & tc_on
+    tc_on = w.dtype == "bf16" and w.k_entries <= 32 and tc_min <= B
+    is_tc = (bucket >= tc_min) & tc_on
     touched = bucket > 0
     n_b = np.where(group_idx >= 0, counts[np.clip(group_idx, 0, None)], 0).sum(axis=1)
     work = {}
@@ -293,6 +298,10 @@ def run_htam(args, world, rank, local):
     # The streaming workload appends once per step (warm-up, timed, end-to-end).
     capacity = w.n + (args.warmup + 2 * args.steps + 60) * w.append_per_round if w.rounds else w.n
     mem = htam.Memory(entries, gid, w.g, capacity=capacity)
+    if args.stream_rows is not None:
+        mem.set_stream_rows(args.stream_rows)
+    if args.tc_min_bucket is not None:
+        mem.set_tensor_core_min_bucket(args.tc_min_bucket)
     if args.no_cpu_baseline:
         del entries                  # the memory holds its own copy
         torch.cuda.empty_cache()
@@ -311,7 +320,7 @@ def run_htam(args, world, rank, local):
     work = []
     for q in batches:
         o = mem.query(q, w.k_groups, w.k_entries)
-        work.append(step_work(w, counts, o["group_idx"].cpu().numpy()))
+        work.append(step_work(w, counts, o["group_idx"].cpu().numpy(), args.tc_min_bucket or TC_MIN_BUCKET))
     flush_l2 = work[0]["step_bytes"] < 4 * l2_bytes
     flush = torch.empty(2 * l2_bytes, dtype=torch.uint8, device=dev) if flush_l2 else None
 

@@ -193,14 +193,19 @@ typedef enum {
   HTAM_N_PHASES = 6
 } htam_phase;
 
-/* Tuning: when a group was selected by at least `min_bucket` queries of a
- * batch, its entries are scored against those queries on the tensor cores
- * (tcgen05, 128 queries per tile); smaller buckets are scored on the CUDA
- * cores.  The tensor-core path needs a bf16 memory and k_entries <= 32.
- * Default 16; a value above the batch size turns the tensor-core path off.
- * Both paths return the same results within the fp32 rounding of the
- * scores.  Errors: EINVAL (m NULL or min_bucket < 1). */
-htam_status htam_set_tensor_core_min_bucket(htam_memory *m, int32_t min_bucket);
+/* Tuning knobs of htam_query (all paths return the same results within the
+ * fp32 rounding of the scores):
+ *  HTAM_TUNE_TC_MIN_BUCKET: when a group was selected by at least this many
+ *    queries of a batch, its entries are scored against them on the tensor
+ *    cores (tcgen05, 128 queries per tile); smaller buckets are scored on the
+ *    CUDA cores.  Needs a bf16 memory and k_entries <= 32.  Default 16; a
+ *    value above the batch size turns the tensor-core path off.  >= 1.
+ *  HTAM_TUNE_STREAM_ROWS: 1 (default) streams the CUDA-core path's entry rows
+ *    through shared memory with bulk asynchronous copies (rows up to 8 KiB);
+ *    0 loads them directly into registers.
+ * Errors: EINVAL (m NULL, unknown key, value out of range). */
+typedef enum { HTAM_TUNE_TC_MIN_BUCKET = 0, HTAM_TUNE_STREAM_ROWS = 1 } htam_tuning;
+htam_status htam_set_tuning(htam_memory *m, htam_tuning key, int32_t value);
 
 /* Turns CUDA-event timing of each htam_query phase on (1) or off (0).  While
  * on, every query records a pair of events around each phase on its stream

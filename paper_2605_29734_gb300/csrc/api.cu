@@ -211,10 +211,19 @@ htam_status htam_device_status(htam_memory *m, void *cuda_stream) {
   return word ? HTAM_ETIMEOUT : HTAM_OK;
 }
 
-htam_status htam_set_tensor_core_min_bucket(htam_memory *m, int32_t min_bucket) {
-  if (!m || min_bucket < 1) return HTAM_EINVAL;
-  m->tc_min = min_bucket;
-  return HTAM_OK;
+htam_status htam_set_tuning(htam_memory *m, htam_tuning key, int32_t value) {
+  if (!m) return HTAM_EINVAL;
+  switch (key) {
+    case HTAM_TUNE_TC_MIN_BUCKET:
+      if (value < 1) return HTAM_EINVAL;
+      m->tc_min = value;
+      return HTAM_OK;
+    case HTAM_TUNE_STREAM_ROWS:
+      if (value != 0 && value != 1) return HTAM_EINVAL;
+      m->stream_rows = value;
+      return HTAM_OK;
+  }
+  return HTAM_EINVAL;
 }
 
 htam_status htam_set_phase_timing(htam_memory *m, int enable) {

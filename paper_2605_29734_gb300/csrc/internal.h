@@ -63,6 +63,9 @@ struct htam_memory {
   // Tensor-core fine path: smallest bucket it takes, and the TMA map of the
   // page pool (built on first use).
   int tc_min = 16;
+  // CUDA-core fine path: stream rows through shared memory (1) or load them
+  // directly (0).
+  int stream_rows = 1;
   CUtensorMap pool_map;
   bool pool_map_ready = false;
 };

@@ -17,6 +17,7 @@
 #include <vector>
 
 #include "common.cuh"
+#include "fine_stream.h"
 #include "fine_tc.h"
 #include "internal.h"
 
@@ -629,11 +630,12 @@ htam_status dispatch_fine_simt(int qc, const FineArgs &fa, int sm_count, int64_t
 
 }  // namespace
 
-// Queries per SIMT work unit: the staged query block (fp32) stays within
-// 64 KiB of shared memory.
+// Queries per CUDA-core work unit: qc * d <= 8192 (at most 8), which keeps
+// the staged fp32 query block within 32 KiB and leaves the direct-load
+// kernel registers for a long row's loads in flight.
 static int simt_query_chunk(int d) {
   int qc = 8;
-  while (qc > 1 && (size_t)qc * d * sizeof(float) > 64 * 1024) qc >>= 1;
+  while (qc > 1 && (size_t)qc * d > 8192) qc >>= 1;
   return qc;
 }
 
@@ -753,10 +755,20 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
 
   // 3a. Fine scores of small buckets on the CUDA cores.
   mark.begin(HTAM_PHASE_FINE);
-  FineArgs fa{m->pool, d, m->slot_id, m->page_list, m->page_off, m->count, queries, bucket, bucket_off,
-              cnt, units, n_units, part_off, ke, 1.0f / p.tau, kSimtSegPages, part_ml, part_s, part_id};
-  s = m->dtype == HTAM_BF16 ? dispatch_fine_simt<__nv_bfloat16>(qc, fa, m->sm_count, max_units, st)
-                            : dispatch_fine_simt<float>(qc, fa, m->sm_count, max_units, st);
+  {
+    // Rows streamed through shared memory by bulk asynchronous copies; rows
+    // or query blocks too large for its ring take direct 16-byte loads.
+    StreamArgs sa{m->pool, d, m->slot_id, m->page_list, m->page_off, m->count, queries, bucket, bucket_off,
+                  cnt, units, n_units, part_off, ke, 1.0f / p.tau, kSimtSegPages, part_ml, part_s, part_id,
+                  m->status, kMaxPolls};
+    s = m->stream_rows ? launch_fine_stream(sa, qc, m->dtype, m->sm_count, st) : HTAM_EINVAL;
+    if (s == HTAM_EINVAL) {
+      FineArgs fa{m->pool, d, m->slot_id, m->page_list, m->page_off, m->count, queries, bucket, bucket_off,
+                  cnt, units, n_units, part_off, ke, 1.0f / p.tau, kSimtSegPages, part_ml, part_s, part_id};
+      s = m->dtype == HTAM_BF16 ? dispatch_fine_simt<__nv_bfloat16>(qc, fa, m->sm_count, max_units, st)
+                                : dispatch_fine_simt<float>(qc, fa, m->sm_count, max_units, st);
+    }
+  }
   if (s != HTAM_OK) return s;
   mark.launched();
   mark.end();

@@ -17,12 +17,13 @@ LIB_PATH = os.path.join(_PKG, "_lib", "libhtam.so")
 
 HTAM_OK, HTAM_EINVAL, HTAM_ENOMEM, HTAM_ECAPACITY, HTAM_ECUDA, HTAM_ETIMEOUT, HTAM_ENODEV = range(7)
 HTAM_F32, HTAM_BF16 = 0, 1
+HTAM_TUNE_TC_MIN_BUCKET, HTAM_TUNE_STREAM_ROWS = 0, 1
 
 # Every symbol include/htam.h declares, in declaration order.
 EXPORTS = (
     "htam_build_memory", "htam_append_transitions", "htam_query", "htam_query_host",
     "htam_select_groups_static", "htam_memory_info", "htam_memory_group_counts", "htam_memory_group_keys",
-    "htam_device_status", "htam_set_tensor_core_min_bucket", "htam_set_phase_timing",
+    "htam_device_status", "htam_set_tuning", "htam_set_phase_timing",
     "htam_read_phase_timing", "htam_free_memory", "htam_status_string", "htam_last_error",
     "htam_selftest_wait_timeout",
 )
@@ -66,8 +67,8 @@ def _load() -> ctypes.CDLL:
     lib.htam_selftest_wait_timeout.argtypes = [i64, P]
     lib.htam_select_groups_static.argtypes = [P, P, i32, i32, P, P, P]
     lib.htam_select_groups_static.restype = st
-    lib.htam_set_tensor_core_min_bucket.argtypes = [P, i32]
-    lib.htam_set_tensor_core_min_bucket.restype = st
+    lib.htam_set_tuning.argtypes = [P, ctypes.c_int, i32]
+    lib.htam_set_tuning.restype = st
     lib.htam_set_phase_timing.argtypes = [P, ctypes.c_int]
     lib.htam_read_phase_timing.argtypes = [P, P, P, P, P]
     for name in ("htam_build_memory", "htam_append_transitions", "htam_query", "htam_query_host",
@@ -212,10 +213,17 @@ class Memory:
     def device_status(self, stream=None) -> int:
         return _lib.htam_device_status(self.handle, _stream_ptr(stream))
 
+    def set_tuning(self, key: int, value: int) -> None:
+        _check(_lib.htam_set_tuning(self.handle, int(key), int(value)), "htam_set_tuning")
+
     def set_tensor_core_min_bucket(self, min_bucket: int) -> None:
         """Buckets of at least `min_bucket` queries go to the tensor-core kernel."""
-        _check(_lib.htam_set_tensor_core_min_bucket(self.handle, int(min_bucket)),
-               "htam_set_tensor_core_min_bucket")
+        self.set_tuning(HTAM_TUNE_TC_MIN_BUCKET, min_bucket)
+
+    def set_stream_rows(self, enable: bool) -> None:
+        """CUDA-core path: stream rows through shared memory (True) or load
+        them directly (False)."""
+        self.set_tuning(HTAM_TUNE_STREAM_ROWS, int(bool(enable)))
 
     def set_phase_timing(self, enable: bool) -> None:
         _check(_lib.htam_set_phase_timing(self.handle, int(bool(enable))), "htam_set_phase_timing")

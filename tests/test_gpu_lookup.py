@@ -224,6 +224,29 @@ def test_tensor_core_and_cuda_core_paths(htam, case, min_bucket):
         assert ran["fine_tc"][1] == 0
 
 
+STREAM_CASES = [
+    # n, groups, d, dtype, batch, k_groups, k_entries
+    (6000, 30, 4096, torch.bfloat16, 20, 3, 16),   # 8 KiB rows: one row per ring stage
+    (9000, 40, 1024, torch.bfloat16, 70, 5, 33),   # 2 KiB rows, k_entries above the tensor-core limit
+    (5000, 20, 256, torch.float32, 25, 4, 10),     # fp32 rows
+    (3000, 12, 2048, torch.float32, 9, 2, 8),      # fp32 8 KiB rows
+    (2000, 10, 8192, torch.bfloat16, 6, 2, 5),     # 16 KiB rows: direct loads either way
+    (700, 7, 24, torch.bfloat16, 30, 3, 9),        # tiny rows, many per stage
+]
+
+
+@pytest.mark.parametrize("case", STREAM_CASES)
+@pytest.mark.parametrize("stream", [0, 1])
+def test_cuda_core_rows_streamed_and_loaded_directly(htam, case, stream):
+    n, g, d, dtype, b, kg, ke = case
+    entries, gid, centres = _rand_memory(n, d, g, dtype, seed=n + d)
+    q = _rand_queries(b, d, dtype, seed=n + d, centres=centres)
+    mem = htam.Memory(entries, gid, g)
+    mem.set_tensor_core_min_bucket(1 << 30)
+    mem.set_stream_rows(stream)
+    _check(htam, mem, entries, gid, g, q, kg, ke, tau=0.4, eps=0.02)
+
+
 @pytest.mark.parametrize("min_bucket", [1, 1 << 30])
 def test_duplicate_bf16_rows_tie_to_lower_id_on_both_paths(htam, min_bucket):
     """Exactly equal scores (duplicate rows spread over pages and chunks)
