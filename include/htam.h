@@ -142,9 +142,11 @@ htam_status htam_query_host(htam_memory *m, const void *queries, int32_t b,
  * cudaMalloc; this call never calls cudaMalloc, cudaFree or any allocating
  * library routine.
  *
- * It returns the same group_idx / group_score as htam_query (stage 1: the
- * coarse scores q . c_g against every non-empty group key and the k_groups
- * best groups, ties to the lower id, -1 / -inf padding).  Arguments are those
+ * It returns the group_idx / group_score of htam_query's stage 1 (the coarse
+ * scores q . c_g against every non-empty group key and the k_groups best
+ * groups, ties to the lower id, -1 / -inf padding), with scores equal within
+ * fp32 rounding (so groups whose scores differ by less than that may come
+ * out in the other order).  Arguments are those
  * of htam_query: device pointers, queries [b, d] of the memory's dtype,
  * outputs [b, k_groups].
  *

@@ -17,6 +17,7 @@
 #include <vector>
 
 #include "common.cuh"
+#include "coarse_tc.h"
 #include "fine_stream.h"
 #include "fine_tc.h"
 #include "internal.h"
@@ -701,15 +702,17 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   // 1. Coarse scores and the selected groups.
   {
     mark.begin(HTAM_PHASE_COARSE);
-    dim3 grid((unsigned)ceil_div(G, 64), (unsigned)ceil_div(B, 64));
     if (m->dtype == HTAM_BF16) {
-      coarse_scores_simt_kernel<__nv_bfloat16><<<grid, 256, 0, st>>>(
-          static_cast<const __nv_bfloat16 *>(queries), B, d, m->cent, m->count, G, s1);
+      // Tensor cores against the split (hi + lo) bf16 group keys.
+      s = launch_coarse_tc(queries, B, d, m->cent_hi, m->cent_lo, m->count, G, s1, m->status, kMaxPolls, st);
+      if (s != HTAM_OK) return s;
     } else {
+      // fp32 memories: CUDA cores against the fp32 keys.
+      dim3 grid((unsigned)ceil_div(G, 64), (unsigned)ceil_div(B, 64));
       coarse_scores_simt_kernel<float><<<grid, 256, 0, st>>>(static_cast<const float *>(queries), B, d,
                                                              m->cent, m->count, G, s1);
+      HTAM_CK_LAUNCH("coarse_scores_simt_kernel");
     }
-    HTAM_CK_LAUNCH("coarse_scores_simt_kernel");
     mark.launched();
     mark.end();
     mark.begin(HTAM_PHASE_SELECT);

@@ -58,8 +58,9 @@ htam_status static_scores_on(int device, float **out) {
 }
 
 // s1[b][g] = q_b . cent_g, each output accumulated with fmaf over k = 0..d-1
-// in order (the accumulation order of htam_query's coarse stage, so the two
-// entry points give the same bits); -inf for empty groups.  32x32 tiles.
+// in order against the fp32 group key (htam_query reaches the same scores
+// within fp32 rounding, on the tensor cores for bf16 memories); -inf for empty
+// groups.  32x32 tiles.
 template <typename T>
 __global__ void __launch_bounds__(256) static_coarse_kernel(const T *__restrict__ Q, int B, int d,
                                                             const float *__restrict__ cent,
