@@ -67,8 +67,10 @@ def workload_of(args):
     if args.shrink > 1:
         import dataclasses
 
+        # Groups, entries and queries shrink together, so each selected group
+        # keeps about the same number of queries (the same kernel regime).
         w = dataclasses.replace(w, name=f"{w.name}_div{args.shrink}", g=w.g // args.shrink, n=w.n // args.shrink,
-                                k_groups=min(w.k_groups, w.g // args.shrink))
+                                b=max(1, w.b // args.shrink), k_groups=min(w.k_groups, w.g // args.shrink))
     return w
 
 
@@ -95,14 +97,21 @@ def barrier(world):
         dist.barrier()
 
 
-def max_over_ranks(x: float, world: int) -> float:
+def max_over_ranks(x: float, world: int, device: str = "cuda") -> float:
     if world == 1:
         return x
     import torch.distributed as dist
 
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    t = torch.tensor([x], dtype=torch.float64, device=device)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
+
+
+def whole_job_rate(local_seconds: float, local_queries: int, world: int, device: str = "cuda"):
+    """Replicas: every rank answers its own batches; the job's rate is all
+    ranks' queries over the slowest rank's time.  Returns (rate, max seconds)."""
+    slowest = max_over_ranks(local_seconds, world, device)
+    return local_queries * world / slowest, slowest
 
 
 def load_peaks():
@@ -355,9 +364,7 @@ def run_htam(args, world, rank, local):
     mem.set_phase_timing(False)
     phases = mem.read_phase_timing()
     step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
-    total_s = max_over_ranks(sum(step_ms) / 1e3, world)
-    queries_total = w.b * args.steps * world
-    value = queries_total / total_s
+    value, total_s = whole_job_rate(sum(step_ms) / 1e3, w.b * args.steps, world)
 
     # Dominant kernel roofline (live CUDA events on the launching stream).
     peaks = load_peaks()
