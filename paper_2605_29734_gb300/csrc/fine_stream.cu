@@ -1,356 +1,364 @@
-// fine_stream.cu -- fine scores of small buckets on the CUDA cores, with the
-// selected groups' entry rows streamed through a shared-memory ring.
+// fine_stream.cu -- fine scores of small buckets on the CUDA cores (bf16
+// memories), with the selected groups' entry rows prefetched into per-warp
+// shared-memory rings.
 //
 // Work unit = (group g, bucket chunk c, page segment s): up to QC queries
 // that selected g (the Eq. 12 restriction) against the rows of a few pages of
-// g.  The rows are read from HBM exactly once per unit by one producer thread
-// issuing bulk asynchronous copies (cp.async.bulk, completion counted on an
-// mbarrier) into a ring of 20 stages of up to 8 KiB (160 KiB in flight per
-// SM, independent of registers); eight consumer warps take the stages
-// round-robin, and the copies of later stages -- including those of the
-// CTA's next unit -- are in flight while earlier ones are being scored.
+// g, each row read from HBM once per unit.  Warp w of the block scores rows
+// w, w+8, ... of the unit.
 //
-// A consumer warp scores one row at a time: each lane reads 16-byte slices of
-// the row and of the queries (kept in shared memory in the rows' own layout,
-// so both reads are conflict-free), accumulates four independent partial dot
-// products per query, and the warp reduces them with shuffles.  Per query the
-// warp keeps the online softmax statistics of s/tau (the Eq. 11 normaliser)
-// and a warp-distributed sorted top-k (the Eq. 13 pick as a top-k).  At the
-// end of a unit the eight warps' states are merged per query and one partial
-// record per (query, unit) is written for the merge kernel.  Every mbarrier
-// wait is bounded.
+// Rows: every lane copies its own 16-byte slices of the warp's upcoming rows
+// into the warp's ring with cp.async (L1 bypassed) a few rows ahead of the
+// row it is scoring, then reads back exactly those slices: no lane waits for
+// another lane's copy, no barrier guards a ring slot, and the bytes in flight
+// sit in shared memory, not in registers.  Lane 0 copies each row's entry id
+// along with the row.  The ring depth is a compile-time function of the
+// query block and of the longest row the instantiation serves, so the waits
+// and slot indices are constants.  The copies of a unit's first rows are
+// issued before the previous unit's warps are merged, so the row stream
+// does not pause between units.
+//
+// Queries: the registers left free by the ring hold each lane's slices of
+// the unit's queries as packed bf16 (QC x KV x 16 bytes), so scoring a row
+// reads shared memory once per row slice; the products go through the
+// mixed-precision fma.rn.f32.bf16 (bf16 operands, fp32 accumulator).  A
+// product of two bf16 values is exact in fp32, so this rounds exactly like
+// widening both operands and calling fmaf.  The partial sums of a query (one
+// per slice of the lane, or two for 8-query blocks) are reduced across the warp with shuffles; per query the warp keeps the online
+// softmax statistics of s/tau (the Eq. 11 normaliser) and a warp-distributed
+// sorted top-k (the Eq. 13 pick as a top-k).  At the end of a unit the eight
+// warps' states are merged per query and one partial record per (query,
+// unit) is written for the merge kernel.
 
 #include <algorithm>
 
 #include "common.cuh"
 #include "fine_stream.h"
-#include "sm100.cuh"
 
 namespace htam {
 
 namespace {
 
-using namespace sm100;
+constexpr int kWarps = 8;
+constexpr int kMaxSlots = 16;           // rows per warp ring: cp.async.wait_group takes at most 15 pending
+constexpr int kMaxSegPages = 4;         // pages of a unit, held in registers
+constexpr int kSmemLimit = 227 * 1024;  // opt-in dynamic shared memory per block
+constexpr int kMaxQueryVecs = 32;       // QC x KV: 128 registers of packed queries
 
-constexpr int kConsumers = 8;                     // consumer warps
-constexpr int kThreadsS = (kConsumers + 1) * 32;  // + one producer warp
-constexpr int kRing = 20;                         // stages
-constexpr int kStageBytes = kStreamMaxRowBytes;   // 8 KiB
-
-template <typename T>
-struct Vec16;
-template <>
-struct Vec16<__nv_bfloat16> {
-  static constexpr int kN = 8;
-  __device__ static void run(const uint4 &w, float *f) {
-    f[0] = bf16lo(w.x); f[1] = bf16hi(w.x); f[2] = bf16lo(w.y); f[3] = bf16hi(w.y);
-    f[4] = bf16lo(w.z); f[5] = bf16hi(w.z); f[6] = bf16lo(w.w); f[7] = bf16hi(w.w);
-  }
-};
-template <>
-struct Vec16<float> {
-  static constexpr int kN = 4;
-  __device__ static void run(const uint4 &w, float *f) {
-    f[0] = __uint_as_float(w.x); f[1] = __uint_as_float(w.y);
-    f[2] = __uint_as_float(w.z); f[3] = __uint_as_float(w.w);
-  }
-};
-
-struct __align__(8) StreamBars {
-  uint64_t full[kRing];
-  uint64_t empty[kRing];
-  int abort;
-};
-
-// Rows per stage: a power of two dividing the 128-row page, at most 32.
-__host__ __device__ inline int rows_per_stage(int row_bytes) {
-  int r = 1;
-  while (r < 32 && (r * 2) * row_bytes <= kStageBytes) r *= 2;
-  return r;
+// Shared memory besides the row rings: row ids, per-warp top-k lists and
+// softmax statistics.
+__host__ __device__ constexpr size_t side_bytes(int qc) {
+  return sizeof(int) * kWarps * kMaxSlots + (sizeof(float) + sizeof(int)) * kWarps * qc * 64 +
+         sizeof(float) * 2 * kWarps * qc;
 }
 
-__host__ __device__ inline size_t stream_smem_bytes(int qc, int row_bytes) {
-  return (size_t)kRing * kStageBytes + (size_t)qc * row_bytes +
-         (sizeof(float) + sizeof(int)) * kConsumers * qc * 64 + sizeof(float) * 2 * kConsumers * qc +
-         sizeof(StreamBars);
+// Ring depth (rows per warp) for QC queries per unit and rows of up to
+// 32 * KV 16-byte slices: as many as the shared memory holds, at most 16.
+template <int QC, int KV>
+__host__ __device__ constexpr int ring_slots() {
+  const size_t per_slot = (size_t)kWarps * KV * 32 * 16;
+  const size_t n = (kSmemLimit - side_bytes(QC)) / per_slot;
+  return n < (size_t)kMaxSlots ? (int)n : kMaxSlots;
 }
 
-// acc += <16 bytes of row, 16 bytes of query>, element by element.
-template <typename T>
-__device__ __forceinline__ float dot16(const uint4 &row, const uint4 &q, float acc) {
-  float f[Vec16<T>::kN], g[Vec16<T>::kN];
-  Vec16<T>::run(row, f);
-  Vec16<T>::run(q, g);
-#pragma unroll
-  for (int t = 0; t < Vec16<T>::kN; ++t) acc = fmaf(f[t], g[t], acc);
+__device__ __forceinline__ void cp_async16(void *smem_dst, const void *gmem_src) {
+  const uint32_t d = static_cast<uint32_t>(__cvta_generic_to_shared(smem_dst));
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(d), "l"(gmem_src) : "memory");
+}
+__device__ __forceinline__ void cp_async4(void *smem_dst, const void *gmem_src) {
+  const uint32_t d = static_cast<uint32_t>(__cvta_generic_to_shared(smem_dst));
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(d), "l"(gmem_src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+// acc + x.lo * y.lo + x.hi * y.hi for two packed bf16 pairs, fp32 accumulate.
+__device__ __forceinline__ float fma_bf16x2(uint32_t x, uint32_t y, float acc) {
+  asm("{\n\t.reg .b16 xl, xh, yl, yh;\n\t"
+      "mov.b32 {xl, xh}, %1;\n\t"
+      "mov.b32 {yl, yh}, %2;\n\t"
+      "fma.rn.f32.bf16 %0, xl, yl, %0;\n\t"
+      "fma.rn.f32.bf16 %0, xh, yh, %0;\n\t}"
+      : "+f"(acc)
+      : "r"(x), "r"(y));
   return acc;
 }
 
-template <typename T, int QC>
-__global__ void __launch_bounds__(kThreadsS, 1) fine_stream_kernel(StreamArgs a) {
+// acc + <8 bf16 of a row, 8 bf16 of a query>, in element order.
+__device__ __forceinline__ float dot8_bf16(const uint4 &w, const uint4 &q, float acc) {
+  acc = fma_bf16x2(w.x, q.x, acc);
+  acc = fma_bf16x2(w.y, q.y, acc);
+  acc = fma_bf16x2(w.z, q.z, acc);
+  return fma_bf16x2(w.w, q.w, acc);
+}
+
+// Where one warp's rows of one unit are.
+struct UnitRows {
+  int g, q0, nq, cg, s, r0, my_rows;
+  int pg[kMaxSegPages];  // storage pages of the unit's segment
+};
+
+template <int QC>
+__device__ __forceinline__ UnitRows unit_rows(const StreamArgs &a, int u, int warp) {
+  const int4 U = a.units[u];
+  UnitRows r;
+  r.g = U.x;
+  r.s = U.z;
+  r.cg = a.cnt[r.g];
+  r.q0 = U.y * QC;
+  r.nq = min(QC, r.cg - r.q0);
+  const int pg0 = a.page_off[r.g];
+  const int npages = a.page_off[r.g + 1] - pg0;
+  const int p_beg = r.s * a.seg_pages;
+  const int p_end = min(npages, p_beg + a.seg_pages);
+#pragma unroll
+  for (int k = 0; k < kMaxSegPages; ++k) r.pg[k] = p_beg + k < p_end ? a.page_list[pg0 + p_beg + k] : 0;
+  r.r0 = p_beg * kPageRows;
+  const int r1 = min(p_end * kPageRows, a.count[r.g]);
+  r.my_rows = r1 - r.r0 > warp ? (r1 - r.r0 - warp + kWarps - 1) / kWarps : 0;
+  return r;
+}
+
+template <int QC, int KV>
+__global__ void __launch_bounds__(kWarps * 32, 1) fine_ring_kernel(StreamArgs a) {
+  // Slice t of a lane is row slice lane + 32 t, and query register qr[j][t]
+  // holds the same slice of query j.
+  constexpr int S = ring_slots<QC, KV>();
+  constexpr int AHEAD = S - 1;  // rows in flight beyond the one being scored
+  // Partial sums per query: one per slice, two when eight queries already
+  // fill the registers.
+  constexpr int NP = QC >= 8 && KV > 2 ? 2 : KV;
+  static_assert(S >= kStreamMinSlots, "ring too shallow");
   extern __shared__ __align__(128) unsigned char smem_raw[];
-  const int d = a.d;
-  const int row_bytes = d * (int)sizeof(T);
-  const int n_vec = row_bytes / 16;
-  const int R = rows_per_stage(row_bytes);
-  uint8_t *ring = smem_raw;                                           // [kRing][kStageBytes]
-  uint4 *qv = reinterpret_cast<uint4 *>(ring + kRing * kStageBytes);  // [QC][n_vec], rows' layout
-  float *ws = reinterpret_cast<float *>(qv + QC * n_vec);             // [warps][QC][64]
-  int *wi = reinterpret_cast<int *>(ws + kConsumers * QC * 64);       // [warps][QC][64]
-  float *wm = reinterpret_cast<float *>(wi + kConsumers * QC * 64);   // [warps][QC]
-  float *wl = wm + kConsumers * QC;                                   // [warps][QC]
-  StreamBars *bars = reinterpret_cast<StreamBars *>(wl + kConsumers * QC);
-  volatile int *abort = &bars->abort;
-
+  const int n_vec = a.d / 8;  // 16-byte slices per row, at most 32 * KV
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  if (tid == 0) {
-    for (int s = 0; s < kRing; ++s) {
-      mbar_init(&bars->full[s], 1);
-      mbar_init(&bars->empty[s], 1);
-    }
-    bars->abort = 0;
-    fence_barrier_init();
-  }
-  __syncthreads();
+  uint4 *ring = reinterpret_cast<uint4 *>(smem_raw) + (size_t)warp * S * n_vec;  // this warp's ring
+  int *ids_all = reinterpret_cast<int *>(reinterpret_cast<uint4 *>(smem_raw) + (size_t)kWarps * S * n_vec);
+  int *ids = ids_all + warp * kMaxSlots;                             // this warp's row ids
+  float *ws = reinterpret_cast<float *>(ids_all + kWarps * kMaxSlots);  // [warps][QC][64]
+  int *wi = reinterpret_cast<int *>(ws + kWarps * QC * 64);            // [warps][QC][64]
+  float *wm = reinterpret_cast<float *>(wi + kWarps * QC * 64);        // [warps][QC]
+  float *wl = wm + kWarps * QC;                                        // [warps][QC]
   const int n_units = *a.n_units;
-  const uint8_t *pool = static_cast<const uint8_t *>(a.pool);
+  const uint4 *pool = static_cast<const uint4 *>(a.pool);
+  const uint4 *Q = static_cast<const uint4 *>(a.Q);
+  const int ke = a.ke;
 
-  if (warp == kConsumers) {
-    // ----------------------------------------------------------- producer
-    uint32_t t = 0;  // stage batches issued by this CTA
-    bool ok = true;
-    for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
-      const int4 U = a.units[u];
-      const int g = U.x;
-      const int pg0 = a.page_off[g];
-      const int npg = a.page_off[g + 1] - pg0;
-      const int p_beg = U.z * a.seg_pages, p_end = min(npg, p_beg + a.seg_pages);
-      const int cnt_rows = a.count[g];
-      for (int p = p_beg; ok && p < p_end; ++p) {
-        const int fill = min(kPageRows, cnt_rows - p * kPageRows);
-        const int64_t page_row = (int64_t)a.page_list[pg0 + p] * kPageRows;
-        for (int r0 = 0; r0 < fill; r0 += R, ++t) {
-          const int slot = t % kRing;
-          if (!mbar_wait(&bars->empty[slot], ((t / kRing) & 1u) ^ 1u, abort, a.max_polls)) {
-            ok = false;
-            break;
-          }
-          if (lane == 0) {
-            const uint32_t bytes = (uint32_t)(min(R, fill - r0) * row_bytes);
-            mbar_arrive_expect_tx(&bars->full[slot], bytes);
-            bulk_load(smem_addr(ring + slot * kStageBytes), pool + (page_row + r0) * row_bytes, bytes,
-                      &bars->full[slot]);
-          }
-          __syncwarp();
-        }
+  // Copies this lane's slices of row i of unit U, and on lane 0 the row's
+  // entry id, into ring slot i % S.  One copy group per row, empty past the
+  // unit's last row, keeps the count of groups equal to the count of rows.
+  auto prefetch = [&](const UnitRows &U, int i) {
+    if (i < U.my_rows) {
+      const int r = U.r0 + warp + i * kWarps;  // row of the group; r0 is page-aligned
+      const int pi = (r - U.r0) / kPageRows;
+      const int page = pi == 0 ? U.pg[0] : pi == 1 ? U.pg[1] : pi == 2 ? U.pg[2] : U.pg[3];
+      const int64_t slot = (int64_t)page * kPageRows + (r % kPageRows);
+      const int k = i % S;
+      const uint4 *src = pool + slot * n_vec;
+      uint4 *dst = ring + k * n_vec;
+#pragma unroll
+      for (int t = 0; t < KV; ++t) {
+        const int o = lane + 32 * t;
+        if (o < n_vec) cp_async16(dst + o, src + o);
       }
+      if (lane == 0) cp_async4(ids + k, a.slot_id + slot);
     }
-    if (!ok && lane == 0) {
-      atomicOr(a.status, 1u);
-      bars->abort = 1;
-    }
-    // Drain: the copies of the last kRing batches have landed.
-    for (uint32_t back = 1; back <= kRing && back <= t; ++back) {
-      const uint32_t tt = t - back;
-      for (uint32_t i = 0; i < a.max_polls && !mbar_try_wait(&bars->full[tt % kRing], (tt / kRing) & 1u); ++i) {
-      }
-    }
-    __syncwarp();
-  } else {
-    // ---------------------------------------------------------- consumers
-    // After a give-up (ok == false) a warp keeps walking the same units and
-    // batches -- its waits then return at once -- so that every consumer
-    // warp reaches every named barrier.
-    const T *Q = static_cast<const T *>(a.Q);
-    const int ke = a.ke;
-    uint32_t t = 0;  // stage batches seen by this CTA (all consumer warps count them all)
-    bool ok = true;
-    for (int u = blockIdx.x; u < n_units; u += gridDim.x) {
-      const int4 U = a.units[u];
-      const int g = U.x, c = U.y, s = U.z;
-      const int cg = a.cnt[g];
-      const int q0 = c * QC;
-      const int nq = min(QC, cg - q0);
-      const int *bq = a.bucket + a.bucket_off[g] + q0;
+    cp_async_commit();
+  };
 
-      // Stage the unit's queries in the rows' layout (the previous unit is
-      // done with them).
-      for (int i = tid; i < nq * n_vec; i += kConsumers * 32) {
-        const int j = i / n_vec, v = i % n_vec;
-        qv[j * n_vec + v] = reinterpret_cast<const uint4 *>(Q + (int64_t)bq[j] * d)[v];
-      }
-      named_sync(1, kConsumers * 32);
-
-      float m[QC], l[QC], ts[QC];
-      int ti[QC];
-      WarpList lst[QC];
+  int u = blockIdx.x;
+  UnitRows cur{};
+  if (u < n_units) {
+    cur = unit_rows<QC>(a, u, warp);
+#pragma unroll
+    for (int i = 0; i < AHEAD; ++i) prefetch(cur, i);
+  }
+  for (; u < n_units; u += gridDim.x) {
+    const int nq = cur.nq;
+    uint4 qr[QC][KV];
+    {
+      const int *bq = a.bucket + a.bucket_off[cur.g] + cur.q0;
 #pragma unroll
       for (int j = 0; j < QC; ++j) {
-        m[j] = -INFINITY;
-        l[j] = 0.f;
-        ts[j] = -INFINITY;
-        ti[j] = INT_MAX;
-        lst[j].init();
-      }
-
-      const int pg0 = a.page_off[g];
-      const int npg = a.page_off[g + 1] - pg0;
-      const int p_beg = s * a.seg_pages, p_end = min(npg, p_beg + a.seg_pages);
-      const int cnt_rows = a.count[g];
-      for (int p = p_beg; p < p_end; ++p) {
-        const int fill = min(kPageRows, cnt_rows - p * kPageRows);
-        const int64_t page_row = (int64_t)a.page_list[pg0 + p] * kPageRows;
-        for (int r0 = 0; r0 < fill; r0 += R, ++t) {
-          if ((int)(t % kConsumers) != warp) continue;
-          const int slot = t % kRing;
-          const int nrows = min(R, fill - r0);
-          const int my_id = lane < nrows ? a.slot_id[page_row + r0 + lane] : INT_MAX;
-          if (ok && !mbar_wait(&bars->full[slot], (t / kRing) & 1u, abort, a.max_polls)) ok = false;
-          if (!ok) continue;
-          const uint4 *stage = reinterpret_cast<const uint4 *>(ring + slot * kStageBytes);
-          for (int rr = 0; rr < nrows; ++rr) {
-            const uint4 *row = stage + rr * n_vec;
-            const int id = __shfl_sync(kFullMask, my_id, rr);
-            // Four independent partial sums per query (vectors v, v+32, v+64,
-            // v+96 of each group of 128) keep the FMA pipeline busy.
-            float acc[QC][4];
+        const int64_t qrow = j < nq ? (int64_t)bq[j] * n_vec : 0;
 #pragma unroll
-            for (int j = 0; j < QC; ++j)
-#pragma unroll
-              for (int k = 0; k < 4; ++k) acc[j][k] = 0.f;
-            for (int v0 = lane; v0 < n_vec; v0 += 128) {
-#pragma unroll
-              for (int k = 0; k < 4; ++k) {
-                const int v = v0 + 32 * k;
-                if (v < n_vec) {
-                  const uint4 w = row[v];
-#pragma unroll
-                  for (int j = 0; j < QC; ++j) {
-                    if (j < nq) acc[j][k] = dot16<T>(w, qv[j * n_vec + v], acc[j][k]);
-                  }
-                }
-              }
-            }
-#pragma unroll
-            for (int j = 0; j < QC; ++j) {
-              if (j < nq) {
-                const float sc = warp_sum((acc[j][0] + acc[j][1]) + (acc[j][2] + acc[j][3]));
-                const float z = sc * a.inv_tau;
-                if (z > m[j]) {
-                  l[j] = l[j] * expf(m[j] - z) + 1.f;
-                  m[j] = z;
-                } else {
-                  l[j] += expf(z - m[j]);
-                }
-                if (better(sc, id, ts[j], ti[j])) {
-                  lst[j].insert(ke, sc, id);
-                  lst[j].kth(ke, ts[j], ti[j]);
-                }
-              }
-            }
-          }
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&bars->empty[slot]);
+        for (int t = 0; t < KV; ++t) {
+          const int o = lane + 32 * t;
+          qr[j][t] = j < nq && o < n_vec ? Q[qrow + o] : make_uint4(0u, 0u, 0u, 0u);
         }
       }
+    }
 
-      // Merge the eight warps' states per query and write the partial records.
+    float m[QC], l[QC], ts[QC];
+    int ti[QC];
+    WarpList lst[QC];
+#pragma unroll
+    for (int j = 0; j < QC; ++j) {
+      m[j] = -INFINITY;
+      l[j] = 0.f;
+      ts[j] = -INFINITY;
+      ti[j] = INT_MAX;
+      lst[j].init();
+    }
+    for (int i = 0; i < cur.my_rows; ++i) {
+      prefetch(cur, i + AHEAD);
+      cp_async_wait<AHEAD>();  // row i has landed; rows i+1 .. i+AHEAD may still be pending
+      const int ks = i % S;
+      const uint4 *row = ring + ks * n_vec;
+      const int id = __shfl_sync(kFullMask, lane == 0 ? ids[ks] : 0, 0);
+      float acc[QC][NP];
+#pragma unroll
+      for (int j = 0; j < QC; ++j)
+#pragma unroll
+        for (int t = 0; t < NP; ++t) acc[j][t] = 0.f;
+#pragma unroll
+      for (int t = 0; t < KV; ++t) {
+        const int o = lane + 32 * t;
+        if (o < n_vec) {
+          const uint4 w = row[o];
+#pragma unroll
+          for (int j = 0; j < QC; ++j) {
+            if (j < nq) acc[j][t % NP] = dot8_bf16(w, qr[j][t], acc[j][t % NP]);
+          }
+        }
+      }
 #pragma unroll
       for (int j = 0; j < QC; ++j) {
         if (j < nq) {
-          const int o = (warp * QC + j) * 64;
-          ws[o + lane] = lst[j].s0;
-          wi[o + lane] = lst[j].i0;
-          ws[o + 32 + lane] = lst[j].s1;
-          wi[o + 32 + lane] = lst[j].i1;
-          if (lane == 0) {
-            wm[warp * QC + j] = m[j];
-            wl[warp * QC + j] = l[j];
+#pragma unroll
+          for (int h = NP / 2; h >= 1; h /= 2)
+#pragma unroll
+            for (int t = 0; t < h; ++t) acc[j][t] += acc[j][t + h];
+          const float sc = warp_sum(acc[j][0]);
+          const float z = sc * a.inv_tau;
+          if (z > m[j]) {
+            l[j] = l[j] * expf(m[j] - z) + 1.f;
+            m[j] = z;
+          } else {
+            l[j] += expf(z - m[j]);
+          }
+          if (better(sc, id, ts[j], ti[j])) {
+            lst[j].insert(ke, sc, id);
+            lst[j].kth(ke, ts[j], ti[j]);
           }
         }
       }
-      named_sync(1, kConsumers * 32);
-      for (int j = warp; ok && j < nq; j += kConsumers) {
-        float M = -INFINITY;
-        for (int w = 0; w < kConsumers; ++w) M = fmaxf(M, wm[w * QC + j]);
-        float Ls = 0.f;
-        for (int w = 0; w < kConsumers; ++w) {
-          const float mw = wm[w * QC + j];
-          if (mw != -INFINITY) Ls += wl[w * QC + j] * expf(mw - M);
-        }
-        WarpList F;
-        F.init();
-        float fs = -INFINITY;
-        int fi = INT_MAX;
-        for (int w = 0; w < kConsumers; ++w) {
-          for (int h = 0; h < 2; ++h) {
-            if (h * 32 >= ke) break;
-            const int o = (w * QC + j) * 64 + h * 32;
-            const float cs = ws[o + lane];
-            const int ci = wi[o + lane];
-            unsigned mask = __ballot_sync(kFullMask, h * 32 + lane < ke && ci != INT_MAX && better(cs, ci, fs, fi));
-            while (mask) {
-              const int src = __ffs(mask) - 1;
-              mask &= mask - 1;
-              const float vs = __shfl_sync(kFullMask, cs, src);
-              const int vi = __shfl_sync(kFullMask, ci, src);
-              F.insert(ke, vs, vi);
-              F.kth(ke, fs, fi);
-            }
-          }
-        }
-        const int64_t pidx = a.part_off[g] + (int64_t)s * cg + q0 + j;
-        if (lane == 0) a.part_ml[pidx] = make_float2(M, Ls);
-        if (lane < ke) {
-          a.part_s[pidx * ke + lane] = F.s0;
-          a.part_id[pidx * ke + lane] = F.i0;
-        }
-        if (lane + 32 < ke) {
-          a.part_s[pidx * ke + lane + 32] = F.s1;
-          a.part_id[pidx * ke + lane + 32] = F.i1;
-        }
-      }
-      named_sync(1, kConsumers * 32);  // shared state is free for the next unit
     }
-    if (!ok && lane == 0) {
-      atomicOr(a.status, 1u);
-      bars->abort = 1;
+
+    // Every copy still pending belongs to an empty group, and this lane has
+    // read all of its slices: start the next unit's rows now.
+    const UnitRows done = cur;
+    if (u + (int)gridDim.x < n_units) {
+      cur = unit_rows<QC>(a, u + gridDim.x, warp);
+#pragma unroll
+      for (int i = 0; i < AHEAD; ++i) prefetch(cur, i);
+    }
+
+    // Hand each warp's state to shared memory, then warp j merges query j.
+    __syncthreads();  // the previous unit's merge is done reading
+#pragma unroll
+    for (int j = 0; j < QC; ++j) {
+      if (j < nq) {
+        const int o = (warp * QC + j) * 64;
+        ws[o + lane] = lst[j].s0;
+        wi[o + lane] = lst[j].i0;
+        ws[o + 32 + lane] = lst[j].s1;
+        wi[o + 32 + lane] = lst[j].i1;
+        if (lane == 0) {
+          wm[warp * QC + j] = m[j];
+          wl[warp * QC + j] = l[j];
+        }
+      }
+    }
+    __syncthreads();
+    for (int j = warp; j < nq; j += kWarps) {
+      float M = -INFINITY;
+      for (int w = 0; w < kWarps; ++w) M = fmaxf(M, wm[w * QC + j]);
+      float Ls = 0.f;
+      for (int w = 0; w < kWarps; ++w) {
+        const float mw = wm[w * QC + j];
+        if (mw != -INFINITY) Ls += wl[w * QC + j] * expf(mw - M);
+      }
+      WarpList F;
+      F.init();
+      float fs = -INFINITY;
+      int fi = INT_MAX;
+      for (int w = 0; w < kWarps; ++w) {
+        for (int h = 0; h < 2; ++h) {
+          if (h * 32 >= ke) break;
+          const int o = (w * QC + j) * 64 + h * 32;
+          const float cs = ws[o + lane];
+          const int ci = wi[o + lane];
+          unsigned mask =
+              __ballot_sync(kFullMask, h * 32 + lane < ke && ci != INT_MAX && better(cs, ci, fs, fi));
+          while (mask) {
+            const int src = __ffs(mask) - 1;
+            mask &= mask - 1;
+            const float vs = __shfl_sync(kFullMask, cs, src);
+            const int vi = __shfl_sync(kFullMask, ci, src);
+            F.insert(ke, vs, vi);
+            F.kth(ke, fs, fi);
+          }
+        }
+      }
+      const int64_t pidx = a.part_off[done.g] + (int64_t)done.s * done.cg + done.q0 + j;
+      if (lane == 0) a.part_ml[pidx] = make_float2(M, Ls);
+      if (lane < ke) {
+        a.part_s[pidx * ke + lane] = F.s0;
+        a.part_id[pidx * ke + lane] = F.i0;
+      }
+      if (lane + 32 < ke) {
+        a.part_s[pidx * ke + lane + 32] = F.s1;
+        a.part_id[pidx * ke + lane + 32] = F.i1;
+      }
     }
   }
-  __syncthreads();
+  cp_async_wait<0>();
 }
 
-template <typename T, int QC>
-htam_status launch_qc(const StreamArgs &a, int sm_count, cudaStream_t st) {
-  const size_t smem = stream_smem_bytes(QC, a.d * (int)sizeof(T));
-  if (smem > 227 * 1024) return HTAM_EINVAL;
-  auto kernel = fine_stream_kernel<T, QC>;
+template <int QC, int KV>
+htam_status launch_qk(const StreamArgs &a, int sm_count, cudaStream_t st) {
+  const size_t smem = (size_t)kWarps * ring_slots<QC, KV>() * (a.d / 8) * 16 + side_bytes(QC);
+  auto kernel = fine_ring_kernel<QC, KV>;
   HTAM_CK(cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
-  kernel<<<sm_count, kThreadsS, smem, st>>>(a);
-  HTAM_CK_LAUNCH("fine_stream_kernel");
+  kernel<<<sm_count, kWarps * 32, smem, st>>>(a);
+  HTAM_CK_LAUNCH("fine_ring_kernel");
   return HTAM_OK;
 }
 
-template <typename T>
-htam_status launch_t(const StreamArgs &a, int qc, int sm_count, cudaStream_t st) {
-  switch (qc) {
-    case 8: return launch_qc<T, 8>(a, sm_count, st);
-    case 4: return launch_qc<T, 4>(a, sm_count, st);
-    case 2: return launch_qc<T, 2>(a, sm_count, st);
-    default: return launch_qc<T, 1>(a, sm_count, st);
+template <int QC>
+htam_status launch_q(const StreamArgs &a, int kv, int sm_count, cudaStream_t st) {
+  switch (kv) {
+    case 1: return launch_qk<QC, 1>(a, sm_count, st);
+    case 2: return launch_qk<QC, 2>(a, sm_count, st);
+    case 4: return launch_qk<QC, 4>(a, sm_count, st);
+    case 8:
+      if constexpr (QC * 8 <= kMaxQueryVecs) return launch_qk<QC, 8>(a, sm_count, st);
+      break;
+    case 16:
+      if constexpr (QC * 16 <= kMaxQueryVecs) return launch_qk<QC, 16>(a, sm_count, st);
+      break;
   }
+  return HTAM_EINVAL;
 }
 
 }  // namespace
 
 htam_status launch_fine_stream(const StreamArgs &a, int qc, htam_dtype dtype, int sm_count, cudaStream_t st) {
-  const int row_bytes = a.d * (dtype == HTAM_BF16 ? 2 : 4);
-  if (row_bytes > kStreamMaxRowBytes || row_bytes % 16 != 0) return HTAM_EINVAL;
-  // With one row per stage each consumer warp has too little prefetched
-  // (measured slower than direct loads on 8 KiB rows): stream only when a
-  // stage holds at least two rows.
-  if (rows_per_stage(row_bytes) < 2) return HTAM_EINVAL;
-  return dtype == HTAM_BF16 ? launch_t<__nv_bfloat16>(a, qc, sm_count, st) : launch_t<float>(a, qc, sm_count, st);
+  if (dtype != HTAM_BF16 || a.d % 8 != 0 || a.seg_pages < 1 || a.seg_pages > kMaxSegPages) return HTAM_EINVAL;
+  const int per_lane = (a.d / 8 + 31) / 32;  // 16-byte query slices per lane
+  int kv = 1;
+  while (kv < per_lane) kv *= 2;
+  if (kv * qc > kMaxQueryVecs) return HTAM_EINVAL;
+  switch (qc) {
+    case 8: return launch_q<8>(a, kv, sm_count, st);
+    case 4: return launch_q<4>(a, kv, sm_count, st);
+    case 2: return launch_q<2>(a, kv, sm_count, st);
+    case 1: return launch_q<1>(a, kv, sm_count, st);
+  }
+  return HTAM_EINVAL;
 }
 
 }  // namespace htam

@@ -1,5 +1,5 @@
 // fine_stream.h -- CUDA-core fine-score kernel for small buckets, with the
-// entry rows streamed through shared memory by bulk asynchronous copies.
+// entry rows prefetched into per-warp shared-memory rings by cp.async.
 #pragma once
 
 #include <cuda_runtime.h>
@@ -29,17 +29,16 @@ struct StreamArgs {
   float2 *part_ml;
   float *part_s;
   int32_t *part_id;
-  unsigned *status;
-  uint32_t max_polls;
 };
 
-// Rows up to this many bytes are streamed (a ring stage holds at least one).
-constexpr int kStreamMaxRowBytes = 8192;
+// Every ring holds at least this many rows per warp (two in flight while the
+// third is scored).
+constexpr int kStreamMinSlots = 3;
 
-// Launches the streaming kernel for `qc` queries per unit (1, 2, 4 or 8) on
-// bf16 or fp32 rows.  Returns HTAM_EINVAL without launching when the row is
-// longer than a stage or the shared memory would not fit (the caller then
-// uses the direct-load kernel).
+// Launches the ring kernel for `qc` queries per unit (1, 2, 4 or 8) on bf16
+// rows.  Returns HTAM_EINVAL without launching for fp32 rows, when the
+// unit's queries do not fit in 128 registers per lane, i.e. for rows longer
+// than 8 KiB (the caller then uses the direct-load kernel).
 htam_status launch_fine_stream(const StreamArgs &a, int qc, htam_dtype dtype, int sm_count, cudaStream_t st);
 
 }  // namespace htam

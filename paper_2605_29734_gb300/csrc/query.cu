@@ -759,11 +759,10 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   // 3a. Fine scores of small buckets on the CUDA cores.
   mark.begin(HTAM_PHASE_FINE);
   {
-    // Rows streamed through shared memory by bulk asynchronous copies; rows
-    // or query blocks too large for its ring take direct 16-byte loads.
+    // Rows prefetched into per-warp shared-memory rings; rows or query
+    // blocks too large for the rings take direct 16-byte loads.
     StreamArgs sa{m->pool, d, m->slot_id, m->page_list, m->page_off, m->count, queries, bucket, bucket_off,
-                  cnt, units, n_units, part_off, ke, 1.0f / p.tau, kSimtSegPages, part_ml, part_s, part_id,
-                  m->status, kMaxPolls};
+                  cnt, units, n_units, part_off, ke, 1.0f / p.tau, kSimtSegPages, part_ml, part_s, part_id};
     s = m->stream_rows ? launch_fine_stream(sa, qc, m->dtype, m->sm_count, st) : HTAM_EINVAL;
     if (s == HTAM_EINVAL) {
       FineArgs fa{m->pool, d, m->slot_id, m->page_list, m->page_off, m->count, queries, bucket, bucket_off,

@@ -226,7 +226,8 @@ def test_tensor_core_and_cuda_core_paths(htam, case, min_bucket):
 
 STREAM_CASES = [
     # n, groups, d, dtype, batch, k_groups, k_entries
-    (6000, 30, 4096, torch.bfloat16, 20, 3, 16),   # 8 KiB rows: one row per ring stage
+    (6000, 30, 4096, torch.bfloat16, 20, 3, 16),   # 8 KiB rows: three ring slots per warp
+    (60000, 300, 512, torch.bfloat16, 200, 4, 16), # more work units than SMs: next unit's rows fetched early
     (9000, 40, 1024, torch.bfloat16, 70, 5, 33),   # 2 KiB rows, k_entries above the tensor-core limit
     (5000, 20, 256, torch.float32, 25, 4, 10),     # fp32 rows
     (3000, 12, 2048, torch.float32, 9, 2, 8),      # fp32 8 KiB rows
