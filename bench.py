@@ -195,6 +195,15 @@ def profiled_traffic(kernel: str, workload: str):
 
 # ------------------------------------------------------------- algorithmic work
 
+def cuda_core_kernel(w, stream_rows) -> str:
+    """Which CUDA-core fine kernel the library runs for this workload: the
+    shared-memory row ring for bf16 rows up to 8 KiB (unless turned off),
+    otherwise the direct-load kernel."""
+    if w.dtype == "bf16" and w.d <= 4096 and stream_rows != 0:
+        return "fine_ring"
+    return "fine_simt"
+
+
 TC_MIN_BUCKET = 16   # the library's default: buckets this large go to the tensor-core kernel
 
 
@@ -374,7 +383,7 @@ def run_htam(args, world, rank, local):
     # The dominant kernel: the fine kernel (CUDA-core or tensor-core) with the
     # most device time in the timed region.
     phase = max(("fine", "fine_tc"), key=lambda k: phases[k][0])
-    kernel = {"fine": "fine_simt", "fine_tc": "fine_tc"}[phase]
+    kernel = {"fine": cuda_core_kernel(w, args.stream_rows), "fine_tc": "fine_tc"}[phase]
     k_ms, k_launches = phases[phase]
     k_s = k_ms / 1e3 / max(1, k_launches)
     k_bytes = float(np.mean([x["kernels"][phase]["bytes"] for x in per_batch]))

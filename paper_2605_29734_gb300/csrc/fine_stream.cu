@@ -31,6 +31,7 @@
 // unit) is written for the merge kernel.
 
 #include <algorithm>
+#include <type_traits>
 
 #include "common.cuh"
 #include "fine_stream.h"
@@ -130,12 +131,15 @@ __global__ void __launch_bounds__(kWarps * 32, 1) fine_ring_kernel(StreamArgs a)
   // Partial sums per query: one per slice, two when eight queries already
   // fill the registers.
   constexpr int NP = QC >= 8 && KV > 2 ? 2 : KV;
+  // Ring slots are 32 * KV slices long whatever the row length; the slices
+  // past the row stay zero, so scoring needs no bounds test.
+  constexpr int RS = 32 * KV;
   static_assert(S >= kStreamMinSlots, "ring too shallow");
   extern __shared__ __align__(128) unsigned char smem_raw[];
-  const int n_vec = a.d / 8;  // 16-byte slices per row, at most 32 * KV
+  const int n_vec = a.d / 8;  // 16-byte slices per row, at most RS
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  uint4 *ring = reinterpret_cast<uint4 *>(smem_raw) + (size_t)warp * S * n_vec;  // this warp's ring
-  int *ids_all = reinterpret_cast<int *>(reinterpret_cast<uint4 *>(smem_raw) + (size_t)kWarps * S * n_vec);
+  uint4 *ring = reinterpret_cast<uint4 *>(smem_raw) + (size_t)warp * S * RS;  // this warp's ring
+  int *ids_all = reinterpret_cast<int *>(reinterpret_cast<uint4 *>(smem_raw) + (size_t)kWarps * S * RS);
   int *ids = ids_all + warp * kMaxSlots;                             // this warp's row ids
   float *ws = reinterpret_cast<float *>(ids_all + kWarps * kMaxSlots);  // [warps][QC][64]
   int *wi = reinterpret_cast<int *>(ws + kWarps * QC * 64);            // [warps][QC][64]
@@ -157,7 +161,7 @@ __global__ void __launch_bounds__(kWarps * 32, 1) fine_ring_kernel(StreamArgs a)
       const int64_t slot = (int64_t)page * kPageRows + (r % kPageRows);
       const int k = i % S;
       const uint4 *src = pool + slot * n_vec;
-      uint4 *dst = ring + k * n_vec;
+      uint4 *dst = ring + k * RS;
 #pragma unroll
       for (int t = 0; t < KV; ++t) {
         const int o = lane + 32 * t;
@@ -167,6 +171,18 @@ __global__ void __launch_bounds__(kWarps * 32, 1) fine_ring_kernel(StreamArgs a)
     }
     cp_async_commit();
   };
+
+  // Zero the slices past the row once; copies never write them, and each is
+  // read only by the lane that zeroed it.
+  if (n_vec < RS) {
+#pragma unroll
+    for (int k = 0; k < S; ++k)
+#pragma unroll
+      for (int t = 0; t < KV; ++t) {
+        const int o = lane + 32 * t;
+        if (o >= n_vec) ring[k * RS + o] = make_uint4(0u, 0u, 0u, 0u);
+      }
+  }
 
   int u = blockIdx.x;
   UnitRows cur{};
@@ -202,31 +218,29 @@ __global__ void __launch_bounds__(kWarps * 32, 1) fine_ring_kernel(StreamArgs a)
       ti[j] = INT_MAX;
       lst[j].init();
     }
-    for (int i = 0; i < cur.my_rows; ++i) {
-      prefetch(cur, i + AHEAD);
-      cp_async_wait<AHEAD>();  // row i has landed; rows i+1 .. i+AHEAD may still be pending
-      const int ks = i % S;
-      const uint4 *row = ring + ks * n_vec;
-      const int id = __shfl_sync(kFullMask, lane == 0 ? ids[ks] : 0, 0);
-      float acc[QC][NP];
+    // The row loop with the unit's query count NQ as a constant, so the
+    // slices of a row feed NQ x KV independent FMA chains in one block.
+    auto score_rows = [&](auto nq_c) {
+      constexpr int NQ = decltype(nq_c)::value;
+      for (int i = 0; i < cur.my_rows; ++i) {
+        prefetch(cur, i + AHEAD);
+        cp_async_wait<AHEAD>();  // row i has landed; rows i+1 .. i+AHEAD may still be pending
+        const int ks = i % S;
+        const uint4 *row = ring + ks * RS;
+        const int id = __shfl_sync(kFullMask, lane == 0 ? ids[ks] : 0, 0);
+        float acc[NQ][NP];
 #pragma unroll
-      for (int j = 0; j < QC; ++j)
+        for (int j = 0; j < NQ; ++j)
 #pragma unroll
-        for (int t = 0; t < NP; ++t) acc[j][t] = 0.f;
+          for (int t = 0; t < NP; ++t) acc[j][t] = 0.f;
 #pragma unroll
-      for (int t = 0; t < KV; ++t) {
-        const int o = lane + 32 * t;
-        if (o < n_vec) {
-          const uint4 w = row[o];
+        for (int t = 0; t < KV; ++t) {
+          const uint4 w = row[lane + 32 * t];
 #pragma unroll
-          for (int j = 0; j < QC; ++j) {
-            if (j < nq) acc[j][t % NP] = dot8_bf16(w, qr[j][t], acc[j][t % NP]);
-          }
+          for (int j = 0; j < NQ; ++j) acc[j][t % NP] = dot8_bf16(w, qr[j][t], acc[j][t % NP]);
         }
-      }
 #pragma unroll
-      for (int j = 0; j < QC; ++j) {
-        if (j < nq) {
+        for (int j = 0; j < NQ; ++j) {
 #pragma unroll
           for (int h = NP / 2; h >= 1; h /= 2)
 #pragma unroll
@@ -245,6 +259,16 @@ __global__ void __launch_bounds__(kWarps * 32, 1) fine_ring_kernel(StreamArgs a)
           }
         }
       }
+    };
+    switch (nq) {
+      case 1: score_rows(std::integral_constant<int, 1>{}); break;
+      case 2: if constexpr (QC >= 2) score_rows(std::integral_constant<int, 2>{}); break;
+      case 3: if constexpr (QC >= 4) score_rows(std::integral_constant<int, 3>{}); break;
+      case 4: if constexpr (QC >= 4) score_rows(std::integral_constant<int, 4>{}); break;
+      case 5: if constexpr (QC >= 8) score_rows(std::integral_constant<int, 5>{}); break;
+      case 6: if constexpr (QC >= 8) score_rows(std::integral_constant<int, 6>{}); break;
+      case 7: if constexpr (QC >= 8) score_rows(std::integral_constant<int, 7>{}); break;
+      case 8: if constexpr (QC >= 8) score_rows(std::integral_constant<int, 8>{}); break;
     }
 
     // Every copy still pending belongs to an empty group, and this lane has
@@ -320,7 +344,7 @@ __global__ void __launch_bounds__(kWarps * 32, 1) fine_ring_kernel(StreamArgs a)
 
 template <int QC, int KV>
 htam_status launch_qk(const StreamArgs &a, int sm_count, cudaStream_t st) {
-  const size_t smem = (size_t)kWarps * ring_slots<QC, KV>() * (a.d / 8) * 16 + side_bytes(QC);
+  const size_t smem = (size_t)kWarps * ring_slots<QC, KV>() * 32 * KV * 16 + side_bytes(QC);
   auto kernel = fine_ring_kernel<QC, KV>;
   HTAM_CK(cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
   kernel<<<sm_count, kWarps * 32, smem, st>>>(a);
