@@ -9,7 +9,12 @@
 // lo (128-byte swizzle), one thread issues per slice four MMAs against hi and
 // four against lo into the same fp32 accumulator in tensor memory, and four
 // epilogue warps write the scores (-inf for empty groups) for the top-k
-// kernel.  Every mbarrier wait is bounded.
+// kernel.  When the tiles alone would leave SMs idle (few queries), the K
+// slices are split over blockIdx.z: split z writes its partial dot products
+// to plane z of the output, and the top-k kernel adds the planes in order.
+// Every mbarrier wait is bounded.
+
+#include <algorithm>
 
 #include "coarse_tc.h"
 #include "common.cuh"
@@ -43,8 +48,8 @@ constexpr size_t kCSmem = 1024 + kCStages * (kCABytes + 2 * kCBBytes) + sizeof(C
 
 __global__ void __launch_bounds__(kCThreads, 1)
     coarse_tc_kernel(const __grid_constant__ CUtensorMap q_map, const __grid_constant__ CUtensorMap hi_map,
-                     const __grid_constant__ CUtensorMap lo_map, int d, const int32_t *__restrict__ count, int B,
-                     int G, float *__restrict__ s1, unsigned *status, uint32_t max_polls) {
+                     const __grid_constant__ CUtensorMap lo_map, int d, int kb_per, const int32_t *__restrict__ count,
+                     int B, int G, float *__restrict__ s1, unsigned *status, uint32_t max_polls) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t *smem = smem_raw + ((1024 - (smem_addr(smem_raw) & 1023)) & 1023);
   uint8_t *st_a = smem;
@@ -55,7 +60,10 @@ __global__ void __launch_bounds__(kCThreads, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int m0 = blockIdx.x * kCM, n0 = blockIdx.y * kCN;
   const bool two = n0 + kPageRows < G;  // second half of the group tile exists
-  const int nk = (d + kCKBlock - 1) / kCKBlock;
+  const int nk_all = (d + kCKBlock - 1) / kCKBlock;
+  const int kb0 = blockIdx.z * kb_per;                // this split's K slices: [kb0, kb0 + nk)
+  const int nk = min(nk_all, kb0 + kb_per) - kb0;     // >= 1 by the launch
+  s1 += (int64_t)blockIdx.z * B * G;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kCStages; ++s) {
@@ -84,7 +92,7 @@ __global__ void __launch_bounds__(kCThreads, 1)
       if (lane == 0) {
         const uint32_t bytes = kCABytes + 2u * (two ? kCBBytes : kCHalf);
         mbar_arrive_expect_tx(&sh->full[st], bytes);
-        const int x = kb * kCKBlock;
+        const int x = (kb0 + kb) * kCKBlock;
         tma_load_2d(smem_addr(st_a + st * kCABytes), &q_map, x, m0, &sh->full[st]);
         tma_load_2d(smem_addr(st_hi + st * kCBBytes), &hi_map, x, n0, &sh->full[st]);
         tma_load_2d(smem_addr(st_lo + st * kCBBytes), &lo_map, x, n0, &sh->full[st]);
@@ -172,9 +180,17 @@ __global__ void __launch_bounds__(kCThreads, 1)
 
 }  // namespace
 
+int coarse_tc_splits(int B, int d, int G, int sm_count) {
+  const int64_t tiles = ceil_div((int64_t)B, kCM) * ceil_div((int64_t)G, kCN);
+  const int nk = (int)ceil_div((int64_t)d, kCKBlock);
+  const int want = (int)std::max<int64_t>(1, std::min<int64_t>(nk, sm_count / std::max<int64_t>(1, tiles)));
+  const int kb_per = (int)ceil_div((int64_t)nk, want);
+  return (int)ceil_div((int64_t)nk, kb_per);
+}
+
 htam_status launch_coarse_tc(const void *queries, int B, int d, const __nv_bfloat16 *hi, const __nv_bfloat16 *lo,
-                             const int32_t *count, int G, float *s1, unsigned *status, uint32_t max_polls,
-                             cudaStream_t st) {
+                             const int32_t *count, int G, int splits, float *s1, unsigned *status,
+                             uint32_t max_polls, cudaStream_t st) {
   CUtensorMap q_map, hi_map, lo_map;
   htam_status s = make_bf16_tile_map(&q_map, queries, B, d, kCM);
   if (s == HTAM_OK) s = make_bf16_tile_map(&hi_map, hi, G, d, kPageRows);
@@ -185,8 +201,12 @@ htam_status launch_coarse_tc(const void *queries, int B, int d, const __nv_bfloa
     HTAM_CK(cudaFuncSetAttribute(coarse_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kCSmem));
     attr_set = true;
   }
-  dim3 grid((unsigned)ceil_div(B, kCM), (unsigned)ceil_div(G, kCN));
-  coarse_tc_kernel<<<grid, kCThreads, kCSmem, st>>>(q_map, hi_map, lo_map, d, count, B, G, s1, status, max_polls);
+  const int nk = (int)ceil_div((int64_t)d, kCKBlock);
+  const int kb_per = (int)ceil_div((int64_t)nk, splits);
+  if (splits < 1 || (int)ceil_div((int64_t)nk, kb_per) != splits) return HTAM_EINVAL;  // no empty split
+  dim3 grid((unsigned)ceil_div(B, kCM), (unsigned)ceil_div(G, kCN), (unsigned)splits);
+  coarse_tc_kernel<<<grid, kCThreads, kCSmem, st>>>(q_map, hi_map, lo_map, d, kb_per, count, B, G, s1, status,
+                                                     max_polls);
   HTAM_CK_LAUNCH("coarse_tc_kernel");
   return HTAM_OK;
 }

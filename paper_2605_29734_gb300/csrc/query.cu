@@ -97,31 +97,90 @@ __global__ void __launch_bounds__(256) coarse_scores_simt_kernel(
   }
 }
 
-// One warp per query: top-k_groups of s1[b][:] (score desc, lower g on ties),
-// empty groups excluded; -1 / -inf padding.
-__global__ void group_topk_kernel(const float *__restrict__ s1, int B, int G,
-                                  const int32_t *__restrict__ count, int kg,
-                                  int32_t *__restrict__ gidx, float *__restrict__ gscore) {
-  int b = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  int lane = threadIdx.x & 31;
-  if (b >= B) return;
+// A team of WPQ warps per query (8 warps per block): top-k_groups of
+// sum_z s1[z][b][:] (score desc, lower g on ties), empty groups excluded;
+// -1 / -inf padding.  Each warp keeps the top-k of its share of the groups,
+// loading kSelBatch chunks of 32 scores per lane before comparing any; the
+// team's first warp then merges the team's lists.  Few queries take teams of
+// eight warps so that the grid fills the GPU; many take one warp each.
+constexpr int kSelWarps = 8;
+constexpr int kSelBatch = 8;
+
+template <int WPQ>
+__global__ void __launch_bounds__(kSelWarps * 32) group_topk_kernel(const float *__restrict__ s1, int planes,
+                                                                    int B, int G,
+                                                                    const int32_t *__restrict__ count, int kg,
+                                                                    int32_t *__restrict__ gidx,
+                                                                    float *__restrict__ gscore) {
+  __shared__ float ls[kSelWarps][64];
+  __shared__ int li[kSelWarps][64];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int b = blockIdx.x * (kSelWarps / WPQ) + warp / WPQ;
+  const int sw = warp % WPQ;  // this warp's place in the team
+  const bool live = b < B;    // uniform per warp
+  const int64_t plane = (int64_t)B * G;
+  const float *row = s1 + (int64_t)(live ? b : 0) * G;
+  constexpr int kStep = WPQ * 32;
   WarpList L;
   L.init();
   float ts = -INFINITY;
   int ti = INT_MAX;
-  for (int g0 = 0; g0 < G; g0 += 32) {
-    int g = g0 + lane;
-    bool valid = g < G && count[g] > 0;
-    float s = valid ? s1[(int64_t)b * G + g] : -INFINITY;
-    unsigned mask = __ballot_sync(kFullMask, valid && better(s, g, ts, ti));
-    while (mask) {
-      int src = __ffs(mask) - 1;
-      mask &= mask - 1;
-      float cs = __shfl_sync(kFullMask, s, src);
-      L.insert(kg, cs, g0 + src);
-      L.kth(kg, ts, ti);
+  for (int base = sw * 32; live && base < G; base += kStep * kSelBatch) {
+    float sv[kSelBatch];
+    int cv[kSelBatch];
+#pragma unroll
+    for (int u = 0; u < kSelBatch; ++u) {
+      const int g = base + u * kStep + lane;
+      cv[u] = g < G ? count[g] : 0;
+      sv[u] = g < G ? row[g] : -INFINITY;
+    }
+    for (int z = 1; z < planes; ++z) {
+#pragma unroll
+      for (int u = 0; u < kSelBatch; ++u) {
+        const int g = base + u * kStep + lane;
+        if (g < G) sv[u] += row[z * plane + g];
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kSelBatch; ++u) {
+      const int g0 = base + u * kStep;
+      const bool valid = cv[u] > 0;
+      const float sc = valid ? sv[u] : -INFINITY;
+      unsigned mask = __ballot_sync(kFullMask, valid && better(sc, g0 + lane, ts, ti));
+      while (mask) {
+        const int src = __ffs(mask) - 1;
+        mask &= mask - 1;
+        const float cs = __shfl_sync(kFullMask, sc, src);
+        L.insert(kg, cs, g0 + src);
+        L.kth(kg, ts, ti);
+      }
     }
   }
+  if constexpr (WPQ > 1) {
+    ls[warp][lane] = L.s0;
+    li[warp][lane] = L.i0;
+    ls[warp][lane + 32] = L.s1;
+    li[warp][lane + 32] = L.i1;
+    __syncthreads();
+    if (sw != 0 || !live) return;
+    L.init();
+    ts = -INFINITY;
+    ti = INT_MAX;
+    for (int w = warp; w < warp + WPQ; ++w) {
+      for (int h = 0; h < 2 && h * 32 < kg; ++h) {
+        const float cs = ls[w][h * 32 + lane];
+        const int ci = li[w][h * 32 + lane];
+        unsigned mask = __ballot_sync(kFullMask, h * 32 + lane < kg && ci != INT_MAX && better(cs, ci, ts, ti));
+        while (mask) {
+          const int src = __ffs(mask) - 1;
+          mask &= mask - 1;
+          L.insert(kg, __shfl_sync(kFullMask, cs, src), __shfl_sync(kFullMask, ci, src));
+          L.kth(kg, ts, ti);
+        }
+      }
+    }
+  }
+  if (!live) return;
   if (lane < kg) {
     gidx[(int64_t)b * kg + lane] = L.i0 == INT_MAX ? -1 : L.i0;
     gscore[(int64_t)b * kg + lane] = L.i0 == INT_MAX ? -INFINITY : L.s0;
@@ -131,6 +190,10 @@ __global__ void group_topk_kernel(const float *__restrict__ s1, int B, int G,
     gscore[(int64_t)b * kg + lane + 32] = L.i1 == INT_MAX ? -INFINITY : L.s1;
   }
 }
+
+// Warps per query for B queries: eight while B * 8 warps stay under about
+// two full waves of the GPU (16 warps per SM), else one.
+static int warps_per_query(int B, int sm_count) { return (int64_t)B * 8 <= 2LL * 16 * sm_count ? 8 : 1; }
 
 // ---------------------------------------------------------------- bucketing
 
@@ -522,12 +585,23 @@ struct MergeArgs {
   float *entry_score, *entry_weight, *lse;
 };
 
-// One warp per query: combine its partial records (one per selected group and
-// page segment): log-sum-exp of the softmax statistics and the final top-k.
-__global__ void merge_kernel(MergeArgs a) {
-  int b = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  int lane = threadIdx.x & 31;
-  if (b >= a.B) return;
+// A team of WPQ warps per query (8 warps per block): combine its partial
+// records (one per selected group and page segment) -- log-sum-exp of the
+// softmax statistics and the final top-k.  Warp w of a team takes the
+// selected groups j = w, w + WPQ, ...; the team's first warp then combines
+// the team's statistics and lists.
+constexpr int kMergeWarps = 8;
+
+template <int WPQ>
+__global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(MergeArgs a) {
+  __shared__ float ls[kMergeWarps][64];
+  __shared__ int li[kMergeWarps][64];
+  __shared__ float wM[kMergeWarps], wL[kMergeWarps];
+  __shared__ long long wN[kMergeWarps];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int b = blockIdx.x * (kMergeWarps / WPQ) + warp / WPQ;
+  const int sw = warp % WPQ;
+  const bool live = b < a.B;  // uniform per warp
   const int ke = a.ke;
   float M = -INFINITY, L = 0.f;
   int64_t nb = 0;
@@ -535,38 +609,68 @@ __global__ void merge_kernel(MergeArgs a) {
   F.init();
   float fs = -INFINITY;
   int fi = INT_MAX;
-  for (int j = 0; j < a.kg; ++j) {
-    int g = a.gidx[(int64_t)b * a.kg + j];
+  auto offer = [&](float cs, int ci, int limit) {
+    unsigned mask = __ballot_sync(kFullMask, lane < limit && ci != INT_MAX && better(cs, ci, fs, fi));
+    while (mask) {
+      const int src = __ffs(mask) - 1;
+      mask &= mask - 1;
+      F.insert(ke, __shfl_sync(kFullMask, cs, src), __shfl_sync(kFullMask, ci, src));
+      F.kth(ke, fs, fi);
+    }
+  };
+  for (int j = sw; live && j < a.kg; j += WPQ) {
+    const int g = a.gidx[(int64_t)b * a.kg + j];
     if (g < 0) continue;
-    int p = a.pos[(int64_t)b * a.kg + j];
-    int cg = a.cnt[g];
-    int nseg = a.rt.nseg(cg, a.page_off[g + 1] - a.page_off[g]);
+    const int p = a.pos[(int64_t)b * a.kg + j];
+    const int cg = a.cnt[g];
+    const int nseg = a.rt.nseg(cg, a.page_off[g + 1] - a.page_off[g]);
     nb += a.count[g];
     for (int s = 0; s < nseg; ++s) {
-      int64_t pidx = a.part_off[g] + (int64_t)s * cg + p;
-      float2 ml = a.part_ml[pidx];
+      const int64_t pidx = a.part_off[g] + (int64_t)s * cg + p;
+      const float2 ml = a.part_ml[pidx];
       if (ml.x != -INFINITY) {
-        float Mn = fmaxf(M, ml.x);
+        const float Mn = fmaxf(M, ml.x);
         L = L * expf(M - Mn) + ml.y * expf(ml.x - Mn);
         M = Mn;
       }
-      for (int h = 0; h < 2; ++h) {
-        if (h * 32 >= ke) break;
-        int t = h * 32 + lane;
-        float cs = t < ke ? a.part_s[pidx * ke + t] : -INFINITY;
-        int ci = t < ke ? a.part_id[pidx * ke + t] : INT_MAX;
-        unsigned mask = __ballot_sync(kFullMask, ci != INT_MAX && better(cs, ci, fs, fi));
-        while (mask) {
-          int src = __ffs(mask) - 1;
-          mask &= mask - 1;
-          float vs = __shfl_sync(kFullMask, cs, src);
-          int vi = __shfl_sync(kFullMask, ci, src);
-          F.insert(ke, vs, vi);
-          F.kth(ke, fs, fi);
-        }
+      for (int h = 0; h * 32 < ke; ++h) {
+        const int t = h * 32 + lane;
+        const float cs = t < ke ? a.part_s[pidx * ke + t] : -INFINITY;
+        const int ci = t < ke ? a.part_id[pidx * ke + t] : INT_MAX;
+        offer(cs, ci, ke - h * 32);
       }
     }
   }
+  if constexpr (WPQ > 1) {
+    ls[warp][lane] = F.s0;
+    li[warp][lane] = F.i0;
+    ls[warp][lane + 32] = F.s1;
+    li[warp][lane + 32] = F.i1;
+    if (lane == 0) {
+      wM[warp] = M;
+      wL[warp] = L;
+      wN[warp] = nb;
+    }
+    __syncthreads();
+    if (sw != 0 || !live) return;
+    M = -INFINITY;
+    L = 0.f;
+    nb = 0;
+    for (int w = warp; w < warp + WPQ; ++w) {
+      nb += wN[w];
+      if (wM[w] != -INFINITY) {
+        const float Mn = fmaxf(M, wM[w]);
+        L = L * expf(M - Mn) + wL[w] * expf(wM[w] - Mn);
+        M = Mn;
+      }
+    }
+    F.init();
+    fs = -INFINITY;
+    fi = INT_MAX;
+    for (int w = warp; w < warp + WPQ; ++w)
+      for (int h = 0; h * 32 < ke; ++h) offer(ls[w][h * 32 + lane], li[w][h * 32 + lane], ke - h * 32);
+  }
+  if (!live) return;
   const float lse_b = nb > 0 ? M + logf(L) : -INFINITY;
   const float unif = nb > 0 ? a.eps / (float)nb : 0.f;
   auto emit = [&](int t, float s, int id) {
@@ -671,7 +775,10 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   const int W = (int)ceil_div(B, 32);
   const size_t qg_bytes = tc_ok ? sizeof(__nv_bfloat16) * (size_t)rows * d : 0;
 
-  size_t need = Carver::round(sizeof(float) * (size_t)B * G) + Carver::round(sizeof(uint32_t) * (size_t)G * W) +
+  // Coarse scores: one plane per K split of the tensor-core kernel.
+  const int planes = m->dtype == HTAM_BF16 ? coarse_tc_splits(B, d, G, m->sm_count) : 1;
+  const int wpq = warps_per_query(B, m->sm_count);  // warps per query in top-k and merge
+  size_t need = Carver::round(sizeof(float) * (size_t)planes * B * G) + Carver::round(sizeof(uint32_t) * (size_t)G * W) +
                 5 * Carver::round(sizeof(int32_t) * (G + 1)) + Carver::round(sizeof(int64_t) * (G + 1)) +
                 3 * Carver::round(sizeof(int32_t) * rows) + 2 * Carver::round(sizeof(int4) * max_units) +
                 Carver::round(sizeof(float2) * max_parts) + Carver::round(sizeof(float) * max_parts * ke) +
@@ -680,7 +787,7 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   htam_status s = ensure_scratch(m, need);
   if (s != HTAM_OK) return s;
   Carver cv(m->scratch);
-  float *s1 = cv.take<float>((size_t)B * G);
+  float *s1 = cv.take<float>((size_t)planes * B * G);
   uint32_t *bits = cv.take<uint32_t>((size_t)G * W);
   int32_t *cnt = cv.take<int32_t>(G + 1);
   int32_t *bucket_off = cv.take<int32_t>(G + 1);
@@ -704,7 +811,8 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
     mark.begin(HTAM_PHASE_COARSE);
     if (m->dtype == HTAM_BF16) {
       // Tensor cores against the split (hi + lo) bf16 group keys.
-      s = launch_coarse_tc(queries, B, d, m->cent_hi, m->cent_lo, m->count, G, s1, m->status, kMaxPolls, st);
+      s = launch_coarse_tc(queries, B, d, m->cent_hi, m->cent_lo, m->count, G, planes, s1, m->status, kMaxPolls,
+                           st);
       if (s != HTAM_OK) return s;
     } else {
       // fp32 memories: CUDA cores against the fp32 keys.
@@ -716,8 +824,13 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
     mark.launched();
     mark.end();
     mark.begin(HTAM_PHASE_SELECT);
-    group_topk_kernel<<<(unsigned)ceil_div((int64_t)B * 32, 256), 256, 0, st>>>(s1, B, G, m->count, kg,
-                                                                                group_idx, group_score);
+    if (wpq == 8) {
+      group_topk_kernel<8><<<(unsigned)B, kSelWarps * 32, 0, st>>>(s1, planes, B, G, m->count, kg, group_idx,
+                                                                   group_score);
+    } else {
+      group_topk_kernel<1><<<(unsigned)ceil_div(B, kSelWarps), kSelWarps * 32, 0, st>>>(
+          s1, planes, B, G, m->count, kg, group_idx, group_score);
+    }
     HTAM_CK_LAUNCH("group_topk_kernel");
     mark.launched();
     mark.end();
@@ -791,7 +904,11 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   mark.begin(HTAM_PHASE_MERGE);
   MergeArgs ma{group_idx, B, kg, ke, m->count, pos, cnt, m->page_off, rt, part_off, part_ml, part_s,
                part_id, 1.0f / p.tau, p.epsilon, entry_idx, entry_score, entry_weight, lse};
-  merge_kernel<<<(unsigned)ceil_div((int64_t)B * 32, 256), 256, 0, st>>>(ma);
+  if (wpq == 8) {
+    merge_kernel<8><<<(unsigned)B, kMergeWarps * 32, 0, st>>>(ma);
+  } else {
+    merge_kernel<1><<<(unsigned)ceil_div(B, kMergeWarps), kMergeWarps * 32, 0, st>>>(ma);
+  }
   HTAM_CK_LAUNCH("merge_kernel");
   mark.launched();
   mark.end();
