@@ -14,10 +14,8 @@
 //     log2 domain with ex2.approx;
 //   * the row's K best (score, column) pairs so far, sorted, in registers
 //     (the Eq. 13 pick as a top-k, K = k_entries rounded up to 8/16/32).
-//     Scores that reach the admission bound are inserted: when a warp has few
-//     of them in a 32-column chunk, one at a time through an unrolled
-//     compare-and-swap chain; when it has many, the chunk is sorted with a
-//     register bitonic network and bitonic-merged into the list.  The bound
+//     Scores that reach the admission bound are inserted one at a time
+//     through an unrolled compare-and-swap pass over the list.  The bound
 //     is the list's k-th score, raised by a per-query value that all units
 //     of the query share through atomicMax after every tile: an entry below
 //     it cannot reach the final top-k, since k other candidates score at
@@ -57,7 +55,6 @@ constexpr int kHalfB = kBBytes / 2;
 constexpr int kThreads = 192;
 constexpr uint32_t kAccCols = 256;                 // fp32 columns per accumulator
 constexpr unsigned kFull = 0xffffffffu;
-constexpr int kDenseChunk = 8;  // flagged scores per lane above which a chunk is merged as a whole
 
 struct __align__(8) TcSmem {
   uint64_t full[kStages];
@@ -78,39 +75,6 @@ __device__ __forceinline__ unsigned enc_score(float f) {
 __device__ __forceinline__ float dec_score(unsigned u) {
   if (u == 0u) return -INFINITY;
   return __uint_as_float((u & 0x80000000u) ? (u & 0x7fffffffu) : ~u);
-}
-
-// Orders (s[i], c[i]) before (s[j], c[j]) (better first).
-__device__ __forceinline__ void order_pair(float &si, int &ci, float &sj, int &cj) {
-  const bool sw = better(sj, cj, si, ci);
-  const float ts = si;
-  const int tc = ci;
-  si = sw ? sj : si;
-  ci = sw ? cj : ci;
-  sj = sw ? ts : sj;
-  cj = sw ? tc : cj;
-}
-
-// Bitonic sort, best first, of N register pairs (indices fold at compile time).
-template <int N>
-__device__ __forceinline__ void bitonic_sort(float (&s)[N], int (&c)[N]) {
-#pragma unroll
-  for (int size = 2; size <= N; size <<= 1) {
-#pragma unroll
-    for (int stride = size / 2; stride > 0; stride >>= 1) {
-#pragma unroll
-      for (int i = 0; i < N; ++i) {
-        const int j = i ^ stride;
-        if (j > i) {
-          if ((i & size) == 0) {
-            order_pair(s[i], c[i], s[j], c[j]);
-          } else {
-            order_pair(s[j], c[j], s[i], c[i]);
-          }
-        }
-      }
-    }
-  }
 }
 
 // A row's K best (score, column) pairs, best first, in registers.
@@ -147,26 +111,6 @@ struct RowTopK {
     c[0] = keep[0] ? c[0] : xc;
   }
 
-  // Merges 32 pairs sorted best first: the K best of the union are the
-  // better of s[i] and n[K-1-i] (a bitonic sequence), then a bitonic merge.
-  __device__ __forceinline__ void merge_sorted32(const float (&ns)[32], const int (&nc)[32]) {
-#pragma unroll
-    for (int i = 0; i < K; ++i) {
-      if (better(ns[K - 1 - i], nc[K - 1 - i], s[i], c[i])) {
-        s[i] = ns[K - 1 - i];
-        c[i] = nc[K - 1 - i];
-      }
-    }
-#pragma unroll
-    for (int stride = K / 2; stride > 0; stride >>= 1) {
-#pragma unroll
-      for (int i = 0; i < K; ++i) {
-        const int j = i ^ stride;
-        if (j > i) order_pair(s[i], c[i], s[j], c[j]);
-      }
-    }
-  }
-
   // The score at position k-1 (k <= K): the list is sorted, so it is the
   // smallest of the first k (a form that keeps the list in registers).
   __device__ __forceinline__ float kth(int k) const {
@@ -196,7 +140,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&sh->acc_full[i], 1);
-      mbar_init(&sh->acc_empty[i], 1);
+      mbar_init(&sh->acc_empty[i], 4);
     }
     mbar_init(&sh->drain, 1);
     sh->abort = 0;
@@ -390,45 +334,32 @@ __global__ void __launch_bounds__(kThreads, 1)
             int most = __popc(flagged);
 #pragma unroll
             for (int o = 16; o > 0; o >>= 1) most = max(most, __shfl_xor_sync(kFull, most, o));
-            if (most > kDenseChunk) {
-              // Dense chunk: sort its flagged pairs and merge them in.
-              float ns[32];
-              int nc[32];
+            // Insert the flagged pairs one at a time.  (A sorting network over
+            // the chunk costs more here: its unrolled code is large and runs
+            // rarely, while this loop body is small.)
+            for (int it = 0; it < most; ++it) {
+              const bool any = flagged != 0u;
+              const int j = any ? __ffs(flagged) - 1 : 0;
+              flagged &= flagged - 1;
+              // r[j] through a 5-level select tree on the bits of j.
+              uint32_t t16[16], t8[8], t4[4], t2[2];
 #pragma unroll
-              for (int j = 0; j < 32; ++j) {
-                const bool f = (flagged >> j) & 1u;
-                ns[j] = f ? __uint_as_float(r[j]) : -INFINITY;
-                nc[j] = f ? cbase + j : INT_MAX;
-              }
-              bitonic_sort<32>(ns, nc);
-              top.merge_sorted32(ns, nc);
-            } else {
-              // Sparse chunk: insert the flagged pairs one by one.
-              for (int it = 0; it < most; ++it) {
-                const bool any = flagged != 0u;
-                const int j = any ? __ffs(flagged) - 1 : 0;
-                flagged &= flagged - 1;
-                // r[j] through a 5-level select tree on the bits of j.
-                uint32_t t16[16], t8[8], t4[4], t2[2];
+              for (int i = 0; i < 16; ++i) t16[i] = (j & 1) ? r[2 * i + 1] : r[2 * i];
 #pragma unroll
-                for (int i = 0; i < 16; ++i) t16[i] = (j & 1) ? r[2 * i + 1] : r[2 * i];
+              for (int i = 0; i < 8; ++i) t8[i] = (j & 2) ? t16[2 * i + 1] : t16[2 * i];
 #pragma unroll
-                for (int i = 0; i < 8; ++i) t8[i] = (j & 2) ? t16[2 * i + 1] : t16[2 * i];
+              for (int i = 0; i < 4; ++i) t4[i] = (j & 4) ? t8[2 * i + 1] : t8[2 * i];
 #pragma unroll
-                for (int i = 0; i < 4; ++i) t4[i] = (j & 4) ? t8[2 * i + 1] : t8[2 * i];
-#pragma unroll
-                for (int i = 0; i < 2; ++i) t2[i] = (j & 8) ? t4[2 * i + 1] : t4[2 * i];
-                const uint32_t xv = (j & 16) ? t2[1] : t2[0];
-                if (any) top.insert_later(__uint_as_float(xv), cbase + j);
-              }
+              for (int i = 0; i < 2; ++i) t2[i] = (j & 8) ? t4[2 * i + 1] : t4[2 * i];
+              const uint32_t xv = (j & 16) ? t2[1] : t2[0];
+              if (any) top.insert_later(__uint_as_float(xv), cbase + j);
             }
             if (valid) thr = fmaxf(thr, top.kth(k));
           }
         }
         tc_fence_before();
         __syncwarp();
-        named_sync(1, 128);
-        if (e == 0) mbar_arrive(&sh->acc_empty[acc]);
+        if (lane == 0) mbar_arrive(&sh->acc_empty[acc]);
         if (++acc == 2) {
           acc = 0;
           aph ^= 1u;
@@ -440,16 +371,22 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (valid) {
         const int64_t pidx = a.part_off[g] + (int64_t)sg * cg + c * kTcRows + e;
         a.part_ml[pidx] = make_float2(m2 * 0.69314718055994531f, l);
+        // Unit columns -> entry ids: all page lookups, then all id loads,
+        // then the stores, so the loads of a row overlap.
+        int idv[K];
+#pragma unroll
+        for (int i = 0; i < K; ++i) {
+          idv[i] = i < k && top.c[i] != INT_MAX ? a.page_list[pg0 + p_beg + top.c[i] / kPageRows] : -1;
+        }
+#pragma unroll
+        for (int i = 0; i < K; ++i) {
+          idv[i] = idv[i] >= 0 ? a.slot_id[(int64_t)idv[i] * kPageRows + top.c[i] % kPageRows] : INT_MAX;
+        }
 #pragma unroll
         for (int i = 0; i < K; ++i) {
           if (i < k) {
-            int id = INT_MAX;
-            if (top.c[i] != INT_MAX) {
-              const int pg = p_beg + top.c[i] / kPageRows;
-              id = a.slot_id[(int64_t)a.page_list[pg0 + pg] * kPageRows + top.c[i] % kPageRows];
-            }
             a.part_s[pidx * k + i] = top.s[i];
-            a.part_id[pidx * k + i] = id;
+            a.part_id[pidx * k + i] = idv[i];
           }
         }
       }
