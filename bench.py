@@ -453,7 +453,10 @@ def run_htam(args, world, rank, local):
             "roofline": roofline,
             "step_roofline": {"algorithmic_bytes": step_bytes, "algorithmic_flops": step_flops,
                               "t_roof_ms": 1e3 * t_roof, "frac": t_roof / step_s,
-                              "phase_ms_per_step": {k: v[0] / args.steps for k, v in phases.items() if k != "queries"}},
+                              "phase_ms_per_step": {k: v[0] / args.steps for k, v in phases.items() if k != "queries"},
+                              "fine_kernels": {k: {"bytes": float(np.mean([x["kernels"][k]["bytes"] for x in per_batch])),
+                                                   "flops": float(np.mean([x["kernels"][k]["flops"] for x in per_batch]))}
+                                               for k in ("fine", "fine_tc")}},
             "e2e": e2e,
             "cpu_baseline": cpu,
             "clocks": clocks,

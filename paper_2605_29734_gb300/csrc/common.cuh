@@ -74,6 +74,31 @@ struct WarpList {
     ti = b;
   }
 
+  // Merges a list sorted best first and held one pair per lane (lane t: the
+  // t-th best) into slots 0..31; for k <= 32 only (slots 32..63 are not
+  // touched).  The 32 best of two sorted lists A, B are better(A[i],
+  // B[31-i]) for each i, a bitonic sequence, which five shuffle stages of
+  // compare-and-exchange sort (better pair to the lower lane).
+  __device__ __forceinline__ void merge32(float cs, int ci) {
+    const int lane = threadIdx.x & 31;
+    const float rs = __shfl_sync(kFullMask, cs, 31 - lane);
+    const int ri = __shfl_sync(kFullMask, ci, 31 - lane);
+    if (better(rs, ri, s0, i0)) {
+      s0 = rs;
+      i0 = ri;
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float ps = __shfl_xor_sync(kFullMask, s0, o);
+      const int pi = __shfl_xor_sync(kFullMask, i0, o);
+      const bool low = (lane & o) == 0;  // the lower lane of the pair keeps the better pair
+      if (low == better(ps, pi, s0, i0)) {
+        s0 = ps;
+        i0 = pi;
+      }
+    }
+  }
+
   // Inserts a warp-uniform candidate, keeping the 64 slots sorted.  All
   // lanes must call it with the same (s, id).
   __device__ __forceinline__ void insert(int k, float s, int id) {

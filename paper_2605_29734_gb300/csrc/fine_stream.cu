@@ -310,6 +310,20 @@ __global__ void __launch_bounds__(kWarps * 32, 1) fine_ring_kernel(StreamArgs a)
       float fs = -INFINITY;
       int fi = INT_MAX;
       for (int w = 0; w < kWarps; ++w) {
+        if (ke <= 32) {
+          // The warps' lists are sorted: merge each whole unless its best
+          // cannot enter the top-ke.
+          const int o = (w * QC + j) * 64;
+          const float cs = ws[o + lane];
+          const int ci = wi[o + lane];
+          const float bs = __shfl_sync(kFullMask, cs, 0);
+          const int bi = __shfl_sync(kFullMask, ci, 0);
+          if (bi != INT_MAX && better(bs, bi, fs, fi)) {
+            F.merge32(cs, ci);
+            F.kth(ke, fs, fi);
+          }
+          continue;
+        }
         for (int h = 0; h < 2; ++h) {
           if (h * 32 >= ke) break;
           const int o = (w * QC + j) * 64 + h * 32;

@@ -107,7 +107,7 @@ constexpr int kSelWarps = 8;
 constexpr int kSelBatch = 8;
 
 template <int WPQ>
-__global__ void __launch_bounds__(kSelWarps * 32) group_topk_kernel(const float *__restrict__ s1, int planes,
+__global__ void __launch_bounds__(kSelWarps * 32, 1) group_topk_kernel(const float *__restrict__ s1, int planes,
                                                                     int B, int G,
                                                                     const int32_t *__restrict__ count, int kg,
                                                                     int32_t *__restrict__ gidx,
@@ -167,6 +167,19 @@ __global__ void __launch_bounds__(kSelWarps * 32) group_topk_kernel(const float 
     ts = -INFINITY;
     ti = INT_MAX;
     for (int w = warp; w < warp + WPQ; ++w) {
+      if (kg <= 32) {
+        // The team's lists are sorted: merge each whole unless its best
+        // cannot enter the top-kg.
+        const float cs = ls[w][lane];
+        const int ci = li[w][lane];
+        const float bs = __shfl_sync(kFullMask, cs, 0);
+        const int bi = __shfl_sync(kFullMask, ci, 0);
+        if (bi != INT_MAX && better(bs, bi, ts, ti)) {
+          L.merge32(cs, ci);
+          L.kth(kg, ts, ti);
+        }
+        continue;
+      }
       for (int h = 0; h < 2 && h * 32 < kg; ++h) {
         const float cs = ls[w][h * 32 + lane];
         const int ci = li[w][h * 32 + lane];
@@ -593,7 +606,7 @@ struct MergeArgs {
 constexpr int kMergeWarps = 8;
 
 template <int WPQ>
-__global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(MergeArgs a) {
+__global__ void __launch_bounds__(kMergeWarps * 32, 1) merge_kernel(MergeArgs a) {
   __shared__ float ls[kMergeWarps][64];
   __shared__ int li[kMergeWarps][64];
   __shared__ float wM[kMergeWarps], wL[kMergeWarps];
@@ -618,29 +631,84 @@ __global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(MergeArgs a) {
       F.kth(ke, fs, fi);
     }
   };
-  for (int j = sw; live && j < a.kg; j += WPQ) {
-    const int g = a.gidx[(int64_t)b * a.kg + j];
-    if (g < 0) continue;
-    const int p = a.pos[(int64_t)b * a.kg + j];
-    const int cg = a.cnt[g];
-    const int nseg = a.rt.nseg(cg, a.page_off[g + 1] - a.page_off[g]);
-    nb += a.count[g];
-    for (int s = 0; s < nseg; ++s) {
-      const int64_t pidx = a.part_off[g] + (int64_t)s * cg + p;
-      const float2 ml = a.part_ml[pidx];
-      if (ml.x != -INFINITY) {
-        const float Mn = fmaxf(M, ml.x);
-        L = L * expf(M - Mn) + ml.y * expf(ml.x - Mn);
-        M = Mn;
+  // Takes in a sorted list of ke <= 32 pairs held one per lane (padding past
+  // ke): skipped when its best pair cannot enter the top-ke, else merged.
+  auto take32 = [&](float cs, int ci) {
+    const float bs = __shfl_sync(kFullMask, cs, 0);
+    const int bi = __shfl_sync(kFullMask, ci, 0);
+    if (bi != INT_MAX && better(bs, bi, fs, fi)) {
+      F.merge32(cs, ci);
+      F.kth(ke, fs, fi);
+    }
+  };
+  // The index data of this warp's groups j = sw + t * WPQ, loaded by lane
+  // t % 32 (slot t / 32) in parallel, then handed round by shuffles.
+  struct GroupRecs {
+    int g, p, cg, nseg;
+    long long base;
+  };
+  auto load_group = [&](int t) {
+    GroupRecs r{-1, 0, 0, 0, 0};
+    const int j = sw + t * WPQ;
+    if (live && j < a.kg) {
+      r.g = a.gidx[(int64_t)b * a.kg + j];
+      if (r.g >= 0) {
+        r.p = a.pos[(int64_t)b * a.kg + j];
+        r.cg = a.cnt[r.g];
+        r.nseg = a.rt.nseg(r.cg, a.page_off[r.g + 1] - a.page_off[r.g]);
+        r.base = a.part_off[r.g];
+        nb += a.count[r.g];
       }
-      for (int h = 0; h * 32 < ke; ++h) {
-        const int t = h * 32 + lane;
-        const float cs = t < ke ? a.part_s[pidx * ke + t] : -INFINITY;
-        const int ci = t < ke ? a.part_id[pidx * ke + t] : INT_MAX;
-        offer(cs, ci, ke - h * 32);
+    }
+    return r;
+  };
+  const GroupRecs gr0 = load_group(lane), gr1 = load_group(lane + 32);
+  constexpr int kBatch = 4;  // records fetched before any is combined
+  const int n_t = live ? (a.kg - sw + WPQ - 1) / WPQ : 0;
+  for (int t = 0; t < n_t; ++t) {
+    const bool lo = t < 32;
+    const int g = __shfl_sync(kFullMask, lo ? gr0.g : gr1.g, t & 31);
+    if (g < 0) continue;  // uniform
+    const int p = __shfl_sync(kFullMask, lo ? gr0.p : gr1.p, t & 31);
+    const int cg = __shfl_sync(kFullMask, lo ? gr0.cg : gr1.cg, t & 31);
+    const int nseg = __shfl_sync(kFullMask, lo ? gr0.nseg : gr1.nseg, t & 31);
+    const long long base = __shfl_sync(kFullMask, lo ? gr0.base : gr1.base, t & 31);
+    for (int s0 = 0; s0 < nseg; s0 += kBatch) {
+      float2 ml[kBatch];
+      float cs[kBatch][2];
+      int ci[kBatch][2];
+#pragma unroll
+      for (int i = 0; i < kBatch; ++i) {
+        const bool v = s0 + i < nseg;
+        const int64_t pidx = base + (int64_t)(s0 + i) * cg + p;
+        ml[i] = v ? a.part_ml[pidx] : make_float2(-INFINITY, 0.f);
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          const int tt = h * 32 + lane;
+          const bool in = v && tt < ke;
+          cs[i][h] = in ? a.part_s[pidx * ke + tt] : -INFINITY;
+          ci[i][h] = in ? a.part_id[pidx * ke + tt] : INT_MAX;
+        }
+      }
+#pragma unroll
+      for (int i = 0; i < kBatch; ++i) {
+        if (ml[i].x != -INFINITY) {
+          const float Mn = fmaxf(M, ml[i].x);
+          L = L * expf(M - Mn) + ml[i].y * expf(ml[i].x - Mn);
+          M = Mn;
+        }
+        if (ke <= 32) {
+          take32(cs[i][0], ci[i][0]);
+        } else {
+#pragma unroll
+          for (int h = 0; h < 2; ++h) offer(cs[i][h], ci[i][h], ke - h * 32);
+        }
       }
     }
   }
+  // Entries behind this warp's groups (each lane counted its own groups).
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) nb += __shfl_xor_sync(kFullMask, nb, o);
   if constexpr (WPQ > 1) {
     ls[warp][lane] = F.s0;
     li[warp][lane] = F.i0;
@@ -667,8 +735,13 @@ __global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(MergeArgs a) {
     F.init();
     fs = -INFINITY;
     fi = INT_MAX;
-    for (int w = warp; w < warp + WPQ; ++w)
-      for (int h = 0; h * 32 < ke; ++h) offer(ls[w][h * 32 + lane], li[w][h * 32 + lane], ke - h * 32);
+    for (int w = warp; w < warp + WPQ; ++w) {
+      if (ke <= 32) {
+        take32(ls[w][lane], li[w][lane]);
+      } else {
+        for (int h = 0; h * 32 < ke; ++h) offer(ls[w][h * 32 + lane], li[w][h * 32 + lane], ke - h * 32);
+      }
+    }
   }
   if (!live) return;
   const float lse_b = nb > 0 ? M + logf(L) : -INFINITY;
