@@ -133,6 +133,32 @@ struct WarpList {
   }
 };
 
+// Sorts one (score, id) pair per lane across the warp, best first, with a
+// bitonic network of shuffle compare-and-exchange stages.
+__device__ __forceinline__ void warp_sort32(float &s, int &i) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int k = 2; k <= 32; k <<= 1) {
+#pragma unroll
+    for (int o = k >> 1; o > 0; o >>= 1) {
+      const float ps = __shfl_xor_sync(kFullMask, s, o);
+      const int pi = __shfl_xor_sync(kFullMask, i, o);
+      const bool desc = (lane & k) == 0;  // this k-block ends up best first
+      const bool low = (lane & o) == 0;
+      if ((low == desc) == better(ps, pi, s, i)) {
+        s = ps;
+        i = pi;
+      }
+    }
+  }
+}
+
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(kFullMask, v, o));
+  return v;
+}
+
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(kFullMask, v, o);

@@ -26,7 +26,8 @@
 // widening both operands and calling fmaf.  The partial sums of a query (one
 // per slice of the lane, or two for 8-query blocks) are reduced across the warp with shuffles; per query the warp keeps the online
 // softmax statistics of s/tau (the Eq. 11 normaliser) and a warp-distributed
-// sorted top-k (the Eq. 13 pick as a top-k).  At the end of a unit the eight
+// sorted top-k (the Eq. 13 pick as a top-k, k_entries <= 32), both updated
+// 32 rows at a time.  At the end of a unit the eight
 // warps' states are merged per query and one partial record per (query,
 // unit) is written for the merge kernel.
 
@@ -46,10 +47,10 @@ constexpr int kMaxSegPages = 4;         // pages of a unit, held in registers
 constexpr int kSmemLimit = 227 * 1024;  // opt-in dynamic shared memory per block
 constexpr int kMaxQueryVecs = 32;       // QC x KV: 128 registers of packed queries
 
-// Shared memory besides the row rings: row ids, per-warp top-k lists and
-// softmax statistics.
+// Shared memory besides the row rings: row ids, per-warp top-k lists (32
+// slots: k_entries <= 32) and softmax statistics.
 __host__ __device__ constexpr size_t side_bytes(int qc) {
-  return sizeof(int) * kWarps * kMaxSlots + (sizeof(float) + sizeof(int)) * kWarps * qc * 64 +
+  return sizeof(int) * kWarps * kMaxSlots + (sizeof(float) + sizeof(int)) * kWarps * qc * 32 +
          sizeof(float) * 2 * kWarps * qc;
 }
 
@@ -141,9 +142,9 @@ __global__ void __launch_bounds__(kWarps * 32, 1) fine_ring_kernel(StreamArgs a)
   uint4 *ring = reinterpret_cast<uint4 *>(smem_raw) + (size_t)warp * S * RS;  // this warp's ring
   int *ids_all = reinterpret_cast<int *>(reinterpret_cast<uint4 *>(smem_raw) + (size_t)kWarps * S * RS);
   int *ids = ids_all + warp * kMaxSlots;                             // this warp's row ids
-  float *ws = reinterpret_cast<float *>(ids_all + kWarps * kMaxSlots);  // [warps][QC][64]
-  int *wi = reinterpret_cast<int *>(ws + kWarps * QC * 64);            // [warps][QC][64]
-  float *wm = reinterpret_cast<float *>(wi + kWarps * QC * 64);        // [warps][QC]
+  float *ws = reinterpret_cast<float *>(ids_all + kWarps * kMaxSlots);  // [warps][QC][32]
+  int *wi = reinterpret_cast<int *>(ws + kWarps * QC * 32);            // [warps][QC][32]
+  float *wm = reinterpret_cast<float *>(wi + kWarps * QC * 32);        // [warps][QC]
   float *wl = wm + kWarps * QC;                                        // [warps][QC]
   const int n_units = *a.n_units;
   const uint4 *pool = static_cast<const uint4 *>(a.pool);
@@ -219,9 +220,35 @@ __global__ void __launch_bounds__(kWarps * 32, 1) fine_ring_kernel(StreamArgs a)
       lst[j].init();
     }
     // The row loop with the unit's query count NQ as a constant, so the
-    // slices of a row feed NQ x KV independent FMA chains in one block.
+    // slices of a row feed NQ x KV independent FMA chains in one block.  Row
+    // scores are buffered one row per lane and taken in 32 rows at a time:
+    // one warp max and one warp sum update the softmax statistics, and only
+    // if some buffered row can enter the top-k (k_entries <= 32) are the 32
+    // sorted across the warp and merged into the list.
     auto score_rows = [&](auto nq_c) {
       constexpr int NQ = decltype(nq_c)::value;
+      float bs[NQ];  // lane r: the score of buffered row r
+      int bid = INT_MAX;
+      auto flush = [&](int nv) {
+        const bool in = lane < nv;
+#pragma unroll
+        for (int j = 0; j < NQ; ++j) {
+          const float z = in ? bs[j] * a.inv_tau : -INFINITY;
+          const float zm = warp_max(z);
+          if (zm > m[j]) {
+            l[j] *= expf(m[j] - zm);
+            m[j] = zm;
+          }
+          l[j] += warp_sum(in ? expf(z - m[j]) : 0.f);
+          float cs = in ? bs[j] : -INFINITY;
+          int ci = in ? bid : INT_MAX;
+          if (__any_sync(kFullMask, in && better(cs, ci, ts[j], ti[j]))) {
+            warp_sort32(cs, ci);
+            lst[j].merge32(cs, ci);
+            lst[j].kth(ke, ts[j], ti[j]);
+          }
+        }
+      };
       for (int i = 0; i < cur.my_rows; ++i) {
         prefetch(cur, i + AHEAD);
         cp_async_wait<AHEAD>();  // row i has landed; rows i+1 .. i+AHEAD may still be pending
@@ -239,6 +266,7 @@ __global__ void __launch_bounds__(kWarps * 32, 1) fine_ring_kernel(StreamArgs a)
 #pragma unroll
           for (int j = 0; j < NQ; ++j) acc[j][t % NP] = dot8_bf16(w, qr[j][t], acc[j][t % NP]);
         }
+        const bool mine = lane == (i & 31);
 #pragma unroll
         for (int j = 0; j < NQ; ++j) {
 #pragma unroll
@@ -246,18 +274,10 @@ __global__ void __launch_bounds__(kWarps * 32, 1) fine_ring_kernel(StreamArgs a)
 #pragma unroll
             for (int t = 0; t < h; ++t) acc[j][t] += acc[j][t + h];
           const float sc = warp_sum(acc[j][0]);
-          const float z = sc * a.inv_tau;
-          if (z > m[j]) {
-            l[j] = l[j] * expf(m[j] - z) + 1.f;
-            m[j] = z;
-          } else {
-            l[j] += expf(z - m[j]);
-          }
-          if (better(sc, id, ts[j], ti[j])) {
-            lst[j].insert(ke, sc, id);
-            lst[j].kth(ke, ts[j], ti[j]);
-          }
+          if (mine) bs[j] = sc;
         }
+        if (mine) bid = id;
+        if ((i & 31) == 31 || i + 1 == cur.my_rows) flush((i & 31) + 1);
       }
     };
     switch (nq) {
@@ -285,11 +305,9 @@ __global__ void __launch_bounds__(kWarps * 32, 1) fine_ring_kernel(StreamArgs a)
 #pragma unroll
     for (int j = 0; j < QC; ++j) {
       if (j < nq) {
-        const int o = (warp * QC + j) * 64;
+        const int o = (warp * QC + j) * 32;
         ws[o + lane] = lst[j].s0;
         wi[o + lane] = lst[j].i0;
-        ws[o + 32 + lane] = lst[j].s1;
-        wi[o + 32 + lane] = lst[j].i1;
         if (lane == 0) {
           wm[warp * QC + j] = m[j];
           wl[warp * QC + j] = l[j];
@@ -310,35 +328,16 @@ __global__ void __launch_bounds__(kWarps * 32, 1) fine_ring_kernel(StreamArgs a)
       float fs = -INFINITY;
       int fi = INT_MAX;
       for (int w = 0; w < kWarps; ++w) {
-        if (ke <= 32) {
-          // The warps' lists are sorted: merge each whole unless its best
-          // cannot enter the top-ke.
-          const int o = (w * QC + j) * 64;
-          const float cs = ws[o + lane];
-          const int ci = wi[o + lane];
-          const float bs = __shfl_sync(kFullMask, cs, 0);
-          const int bi = __shfl_sync(kFullMask, ci, 0);
-          if (bi != INT_MAX && better(bs, bi, fs, fi)) {
-            F.merge32(cs, ci);
-            F.kth(ke, fs, fi);
-          }
-          continue;
-        }
-        for (int h = 0; h < 2; ++h) {
-          if (h * 32 >= ke) break;
-          const int o = (w * QC + j) * 64 + h * 32;
-          const float cs = ws[o + lane];
-          const int ci = wi[o + lane];
-          unsigned mask =
-              __ballot_sync(kFullMask, h * 32 + lane < ke && ci != INT_MAX && better(cs, ci, fs, fi));
-          while (mask) {
-            const int src = __ffs(mask) - 1;
-            mask &= mask - 1;
-            const float vs = __shfl_sync(kFullMask, cs, src);
-            const int vi = __shfl_sync(kFullMask, ci, src);
-            F.insert(ke, vs, vi);
-            F.kth(ke, fs, fi);
-          }
+        // The warps' lists are sorted: merge each whole unless its best
+        // cannot enter the top-ke.
+        const int o = (w * QC + j) * 32;
+        const float cs = ws[o + lane];
+        const int ci = wi[o + lane];
+        const float bs = __shfl_sync(kFullMask, cs, 0);
+        const int bi = __shfl_sync(kFullMask, ci, 0);
+        if (bi != INT_MAX && better(bs, bi, fs, fi)) {
+          F.merge32(cs, ci);
+          F.kth(ke, fs, fi);
         }
       }
       const int64_t pidx = a.part_off[done.g] + (int64_t)done.s * done.cg + done.q0 + j;
@@ -346,10 +345,6 @@ __global__ void __launch_bounds__(kWarps * 32, 1) fine_ring_kernel(StreamArgs a)
       if (lane < ke) {
         a.part_s[pidx * ke + lane] = F.s0;
         a.part_id[pidx * ke + lane] = F.i0;
-      }
-      if (lane + 32 < ke) {
-        a.part_s[pidx * ke + lane + 32] = F.s1;
-        a.part_id[pidx * ke + lane + 32] = F.i1;
       }
     }
   }
@@ -385,7 +380,9 @@ htam_status launch_q(const StreamArgs &a, int kv, int sm_count, cudaStream_t st)
 }  // namespace
 
 htam_status launch_fine_stream(const StreamArgs &a, int qc, htam_dtype dtype, int sm_count, cudaStream_t st) {
-  if (dtype != HTAM_BF16 || a.d % 8 != 0 || a.seg_pages < 1 || a.seg_pages > kMaxSegPages) return HTAM_EINVAL;
+  if (dtype != HTAM_BF16 || a.d % 8 != 0 || a.seg_pages < 1 || a.seg_pages > kMaxSegPages || a.ke > 32) {
+    return HTAM_EINVAL;
+  }
   const int per_lane = (a.d / 8 + 31) / 32;  // 16-byte query slices per lane
   int kv = 1;
   while (kv < per_lane) kv *= 2;

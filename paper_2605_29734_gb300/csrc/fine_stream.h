@@ -36,9 +36,10 @@ struct StreamArgs {
 constexpr int kStreamMinSlots = 3;
 
 // Launches the ring kernel for `qc` queries per unit (1, 2, 4 or 8) on bf16
-// rows.  Returns HTAM_EINVAL without launching for fp32 rows, when the
-// unit's queries do not fit in 128 registers per lane, i.e. for rows longer
-// than 8 KiB (the caller then uses the direct-load kernel).
+// rows.  Returns HTAM_EINVAL without launching for fp32 rows, for
+// k_entries > 32, or when the unit's queries do not fit in 128 registers
+// per lane, i.e. for rows longer than 8 KiB (the caller then uses the
+// direct-load kernel).
 htam_status launch_fine_stream(const StreamArgs &a, int qc, htam_dtype dtype, int sm_count, cudaStream_t st);
 
 }  // namespace htam
