@@ -155,6 +155,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tbase = sh->tmem_base;
   const int n_units = *a.n_units;
   const int nk = (a.d + kKBlock - 1) / kKBlock;
+  const int seg_pages = *a.seg_pages;
 
   // The producer and MMA warps run their loops with all 32 lanes (so every
   // warp reaches the final barrier converged); lane 0 issues the copies and
@@ -171,7 +172,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int a_row = a.bucket_off[g] + U.y * kTcRows;
       const int pg0 = a.page_off[g];
       const int npg = a.page_off[g + 1] - pg0;
-      const int p_beg = U.z * a.seg_pages, p_end = min(npg, p_beg + a.seg_pages);
+      const int p_beg = U.z * seg_pages, p_end = min(npg, p_beg + seg_pages);
       for (int p = p_beg; ok && p < p_end; p += 2) {
         const bool two = p + 1 < p_end;
         const int y0 = a.page_list[pg0 + p] * kPageRows;
@@ -220,7 +221,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int4 U = a.units[u];
       const int g = U.x;
       const int npg = a.page_off[g + 1] - a.page_off[g];
-      const int p_beg = U.z * a.seg_pages, p_end = min(npg, p_beg + a.seg_pages);
+      const int p_beg = U.z * seg_pages, p_end = min(npg, p_beg + seg_pages);
       for (int p = p_beg; ok && p < p_end; p += 2) {
         if (!mbar_wait(&sh->acc_empty[acc], aph ^ 1u, abort, a.max_polls)) {
           ok = false;
@@ -292,7 +293,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int pg0 = a.page_off[g];
       const int npg = a.page_off[g + 1] - pg0;
       const int cnt_rows = a.count[g];
-      const int p_beg = sg * a.seg_pages, p_end = min(npg, p_beg + a.seg_pages);
+      const int p_beg = sg * seg_pages, p_end = min(npg, p_beg + seg_pages);
       for (int p = p_beg; ok && p < p_end; p += 2) {
         const int f0 = min(kPageRows, cnt_rows - p * kPageRows);
         const int f1 = p + 1 < p_end ? min(kPageRows, cnt_rows - (p + 1) * kPageRows) : 0;

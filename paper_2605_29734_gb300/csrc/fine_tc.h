@@ -24,7 +24,7 @@ struct TcFineArgs {
   const int32_t *slot_id;
   const int64_t *part_off;
   int d;
-  int seg_pages;
+  const int32_t *seg_pages;  // device: pages per unit (even), chosen by the bucketing
   int ke;
   float k2;                   // log2(e) / tau
   float2 *part_ml;

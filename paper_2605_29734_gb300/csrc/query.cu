@@ -244,19 +244,51 @@ struct Route {
   __host__ __device__ int64_t units(int c, int pages) const {
     return c > 0 ? (int64_t)((c + qc(c) - 1) / qc(c)) * nseg(c, pages) : 0;
   }
+  // Tensor-core tiles (two pages each) of a group: every chunk of the bucket
+  // against every page pair.
+  __host__ __device__ int64_t tc_tiles(int c, int pages) const {
+    return tc(c) ? (int64_t)((c + kTcRows - 1) / kTcRows) * ((pages + 1) / 2) : 0;
+  }
 };
 
-// Single block: per group the bucket size c_g, its work units (in the SIMT or
-// the tensor-core list) and its partial records c_g * nseg_g, with exclusive
-// scans over the groups.  n_units = {SIMT units, tensor-core units}.
+// Pages per tensor-core unit: the power of two nearest below the tiles per
+// SM, as pages, within [kTcSegPagesMin, kTcSegPagesMax].  Long segments mean
+// fewer cold top-k lists and fewer partial records; short ones keep every SM
+// busy when the tensor-core work is small.
+constexpr int kTcSegPagesMin = 16;
+constexpr int kTcSegPagesMax = 64;
+__device__ __forceinline__ int tc_seg_pages(int64_t tiles, int sms) {
+  int seg = kTcSegPagesMin;
+  while (seg < kTcSegPagesMax && (int64_t)seg * sms <= tiles) seg *= 2;  // seg/2 tiles <= tiles per SM
+  return seg;
+}
+
+// Single block: chooses the pages per tensor-core unit from the total
+// tensor-core tiles (written to seg_tc_dev), then per group the bucket size
+// c_g, its work units (in the SIMT or the tensor-core list) and its partial
+// records c_g * nseg_g, with exclusive scans over the groups.
+// n_units = {SIMT units, tensor-core units}.
 __global__ void __launch_bounds__(1024) bucket_scan_kernel(
-    const int32_t *__restrict__ cnt, const int32_t *__restrict__ page_off, int G, Route rt,
+    const int32_t *__restrict__ cnt, const int32_t *__restrict__ page_off, int G, Route rt, int sms,
     int32_t *__restrict__ bucket_off, int32_t *__restrict__ unit_off, int32_t *__restrict__ unit_off_tc,
-    int64_t *__restrict__ part_off, int32_t *__restrict__ n_units) {
+    int64_t *__restrict__ part_off, int32_t *__restrict__ n_units, int32_t *__restrict__ seg_tc_dev) {
   __shared__ int64_t sh[4][1024];
   const int tid = threadIdx.x;
   const int per = (G + 1023) / 1024;
   const int lo = min(G, tid * per), hi = min(G, lo + per);
+  {
+    int64_t x = 0;
+    for (int g = lo; g < hi; ++g) x += rt.tc_tiles(cnt[g], page_off[g + 1] - page_off[g]);
+    sh[0][tid] = x;
+    __syncthreads();
+    for (int o = 512; o > 0; o >>= 1) {
+      if (tid < o) sh[0][tid] += sh[0][tid + o];
+      __syncthreads();
+    }
+    rt.seg_tc = tc_seg_pages(sh[0][0], sms);
+    __syncthreads();  // sh is reused below
+    if (tid == 0) *seg_tc_dev = rt.seg_tc;
+  }
   int64_t a = 0, u = 0, t = 0, p = 0;
   for (int g = lo; g < hi; ++g) {
     int c = cnt[g], pages = page_off[g + 1] - page_off[g];
@@ -311,6 +343,7 @@ __global__ void bucket_fill_kernel(const uint32_t *__restrict__ bits, int G, int
                                    const int32_t *__restrict__ gidx, int kg,
                                    const int32_t *__restrict__ cnt,
                                    const int32_t *__restrict__ page_off, Route rt,
+                                   const int32_t *__restrict__ seg_tc_dev,
                                    const int32_t *__restrict__ unit_off,
                                    const int32_t *__restrict__ unit_off_tc,
                                    int32_t *__restrict__ bucket, int32_t *__restrict__ bucket_group,
@@ -319,6 +352,7 @@ __global__ void bucket_fill_kernel(const uint32_t *__restrict__ bits, int G, int
   int g = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   int lane = threadIdx.x & 31;
   if (g >= G) return;
+  rt.seg_tc = *seg_tc_dev;
   int running = 0;
   const int base = bucket_off[g];
   for (int w0 = 0; w0 < W; w0 += 32) {
@@ -588,7 +622,8 @@ struct MergeArgs {
   const int32_t *pos;
   const int32_t *cnt;
   const int32_t *page_off;
-  Route rt;
+  Route rt;                  // seg_tc is replaced by *seg_tc_dev
+  const int32_t *seg_tc_dev;
   const int64_t *part_off;
   const float2 *part_ml;
   const float *part_s;
@@ -647,6 +682,8 @@ __global__ void __launch_bounds__(kMergeWarps * 32, 1) merge_kernel(MergeArgs a)
     int g, p, cg, nseg;
     long long base;
   };
+  Route rt = a.rt;
+  rt.seg_tc = *a.seg_tc_dev;
   auto load_group = [&](int t) {
     GroupRecs r{-1, 0, 0, 0, 0};
     const int j = sw + t * WPQ;
@@ -655,7 +692,7 @@ __global__ void __launch_bounds__(kMergeWarps * 32, 1) merge_kernel(MergeArgs a)
       if (r.g >= 0) {
         r.p = a.pos[(int64_t)b * a.kg + j];
         r.cg = a.cnt[r.g];
-        r.nseg = a.rt.nseg(r.cg, a.page_off[r.g + 1] - a.page_off[r.g]);
+        r.nseg = rt.nseg(r.cg, a.page_off[r.g + 1] - a.page_off[r.g]);
         r.base = a.part_off[r.g];
         nb += a.count[r.g];
       }
@@ -818,7 +855,7 @@ static int simt_query_chunk(int d) {
 }
 
 constexpr int kSimtSegPages = 4;
-constexpr int kTcSegPages = 16;
+
 constexpr uint32_t kMaxPolls = 1u << 24;
 
 htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const htam_query_params &p,
@@ -831,12 +868,14 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   const int qc = simt_query_chunk(d);
   // The tensor-core path takes bf16 memories and k_entries <= 32.
   const bool tc_ok = m->dtype == HTAM_BF16 && ke <= kTcMaxK && m->tc_min <= B;
-  const Route rt{tc_ok ? m->tc_min : INT_MAX, qc, kSimtSegPages, kTcSegPages};
+  // seg_tc here is the shortest tensor-core segment (for the bounds below);
+  // the kernels take the one bucket_scan_kernel chooses.
+  const Route rt{tc_ok ? m->tc_min : INT_MAX, qc, kSimtSegPages, kTcSegPagesMin};
 
   // Upper bound of the partial records: every query in the buckets of the
   // k_g groups with the most page segments (counted with the shorter
   // segments of the two kernels).
-  const int seg_min = std::min(kSimtSegPages, kTcSegPages);
+  const int seg_min = std::min(kSimtSegPages, kTcSegPagesMin);
   std::vector<int64_t> nseg(G);
   for (int g = 0; g < G; ++g) nseg[g] = ceil_div((int64_t)m->h_pages[g].size(), seg_min);
   std::nth_element(nseg.begin(), nseg.begin() + (kg - 1), nseg.end(), std::greater<int64_t>());
@@ -853,6 +892,7 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   const int wpq = warps_per_query(B, m->sm_count);  // warps per query in top-k and merge
   size_t need = Carver::round(sizeof(float) * (size_t)planes * B * G) + Carver::round(sizeof(uint32_t) * (size_t)G * W) +
                 5 * Carver::round(sizeof(int32_t) * (G + 1)) + Carver::round(sizeof(int64_t) * (G + 1)) +
+                Carver::round(sizeof(int32_t)) +
                 3 * Carver::round(sizeof(int32_t) * rows) + 2 * Carver::round(sizeof(int4) * max_units) +
                 Carver::round(sizeof(float2) * max_parts) + Carver::round(sizeof(float) * max_parts * ke) +
                 Carver::round(sizeof(int32_t) * max_parts * ke) + Carver::round(sizeof(unsigned) * B) +
@@ -868,6 +908,7 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   int32_t *unit_off_tc = cv.take<int32_t>(G + 1);
   int64_t *part_off = cv.take<int64_t>(G + 1);
   int32_t *n_units = cv.take<int32_t>(G + 1);  // [0] SIMT units, [1] tensor-core units
+  int32_t *seg_tc = cv.take<int32_t>(1);        // pages per tensor-core unit, chosen on the device
   int32_t *bucket = cv.take<int32_t>(rows);
   int32_t *bucket_group = cv.take<int32_t>(rows);
   int32_t *pos = cv.take<int32_t>(rows);
@@ -916,12 +957,12 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   HTAM_CK_LAUNCH("bucket_bits_kernel");
   bucket_count_kernel<<<(unsigned)ceil_div((int64_t)G * 32, 256), 256, 0, st>>>(bits, G, W, cnt);
   HTAM_CK_LAUNCH("bucket_count_kernel");
-  bucket_scan_kernel<<<1, 1024, 0, st>>>(cnt, m->page_off, G, rt, bucket_off, unit_off, unit_off_tc, part_off,
-                                         n_units);
+  bucket_scan_kernel<<<1, 1024, 0, st>>>(cnt, m->page_off, G, rt, m->sm_count, bucket_off, unit_off,
+                                         unit_off_tc, part_off, n_units, seg_tc);
   HTAM_CK_LAUNCH("bucket_scan_kernel");
   bucket_fill_kernel<<<(unsigned)ceil_div((int64_t)G * 32, 256), 256, 0, st>>>(
-      bits, G, W, bucket_off, group_idx, kg, cnt, m->page_off, rt, unit_off, unit_off_tc, bucket, bucket_group,
-      pos, units, units_tc);
+      bits, G, W, bucket_off, group_idx, kg, cnt, m->page_off, rt, seg_tc, unit_off, unit_off_tc, bucket,
+      bucket_group, pos, units, units_tc);
   HTAM_CK_LAUNCH("bucket_fill_kernel");
   mark.launched(4);
   CUtensorMap q_map;
@@ -965,7 +1006,7 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   if (tc_ok) {
     mark.begin(HTAM_PHASE_FINE_TC);
     TcFineArgs ta{units_tc, n_units + 1, bucket, bucket_off, cnt, m->page_list, m->page_off, m->count, m->slot_id,
-                  part_off, d, kTcSegPages, ke, 1.4426950408889634f / p.tau, part_ml, part_s, part_id, thr_enc,
+                  part_off, d, seg_tc, ke, 1.4426950408889634f / p.tau, part_ml, part_s, part_id, thr_enc,
                   m->status, kMaxPolls};
     s = launch_fine_tc(ta, q_map, m->pool_map, (int)std::min<int64_t>(max_units, m->sm_count), st);
     if (s != HTAM_OK) return s;
@@ -975,7 +1016,7 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
 
   // 4. Merge per query.
   mark.begin(HTAM_PHASE_MERGE);
-  MergeArgs ma{group_idx, B, kg, ke, m->count, pos, cnt, m->page_off, rt, part_off, part_ml, part_s,
+  MergeArgs ma{group_idx, B, kg, ke, m->count, pos, cnt, m->page_off, rt, seg_tc, part_off, part_ml, part_s,
                part_id, 1.0f / p.tau, p.epsilon, entry_idx, entry_score, entry_weight, lse};
   if (wpq == 8) {
     merge_kernel<8><<<(unsigned)B, kMergeWarps * 32, 0, st>>>(ma);
