@@ -203,8 +203,8 @@ typedef enum {
  *    CUDA cores.  Needs a bf16 memory and k_entries <= 32.  Default 16; a
  *    value above the batch size turns the tensor-core path off.  >= 1.
  *  HTAM_TUNE_STREAM_ROWS: 1 (default) prefetches the CUDA-core path's entry
- *    rows into per-warp shared-memory rings (when three rows per warp fit);
- *    0 loads them directly into registers.
+ *    rows into per-warp shared-memory rings (bf16 memories with rows up to
+ *    8 KiB and k_entries <= 32); 0 loads them directly into registers.
  * Errors: EINVAL (m NULL, unknown key, value out of range). */
 typedef enum { HTAM_TUNE_TC_MIN_BUCKET = 0, HTAM_TUNE_STREAM_ROWS = 1 } htam_tuning;
 htam_status htam_set_tuning(htam_memory *m, htam_tuning key, int32_t value);
