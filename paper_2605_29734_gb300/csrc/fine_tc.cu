@@ -25,6 +25,13 @@
 // else.  At the end of a unit each row writes one partial record (max, sum
 // of exp, its top-k entry ids and scores) that the merge kernel combines.
 //
+// Units are taken dynamically (unit i by CTA i first, then from a global
+// counter), so neighbouring units run at the same time -- the CTAs on the
+// chunks of a large group read its pages at about the same moment -- and a
+// CTA that drew short units takes more.  The producer warp takes each unit
+// and passes its index to the MMA and epilogue warps through a small
+// shared-memory queue guarded by mbarriers.
+//
 // Warp roles (192 threads, one CTA per SM, persistent over units):
 //   warp 0   TMA producer (lane 0 issues)
 //   warp 1   TMEM owner, MMA issuer (lane 0 issues)
@@ -56,15 +63,34 @@ constexpr int kThreads = 192;
 constexpr uint32_t kAccCols = 256;                 // fp32 columns per accumulator
 constexpr unsigned kFull = 0xffffffffu;
 
+constexpr int kUQ = 4;  // unit queue slots (producer -> MMA and epilogue warps)
+
 struct __align__(8) TcSmem {
   uint64_t full[kStages];
   uint64_t empty[kStages];
   uint64_t acc_full[2];
   uint64_t acc_empty[2];
   uint64_t drain;
+  uint64_t uq_full[kUQ];   // a unit index was written
+  uint64_t uq_empty[kUQ];  // the MMA warp and the 4 epilogue warps have read it
   uint32_t tmem_base;
   int abort;
+  int uq[kUQ];             // unit indices in the order the producer took them; -1 = no more
 };
+
+// The j-th unit of this CTA, from the producer's queue, for a whole warp:
+// -1 when there are no more units, or when the wait gave up (ok cleared).
+__device__ __forceinline__ int take_unit(TcSmem *sh, int j, volatile int *abort, uint32_t max_polls, bool &ok) {
+  const int slot = j % kUQ;
+  if (!mbar_wait(&sh->uq_full[slot], (uint32_t)(j / kUQ) & 1u, abort, max_polls)) {
+    ok = false;
+    return -1;
+  }
+  const int u = *reinterpret_cast<volatile int *>(&sh->uq[slot]);
+  __syncwarp();
+  if ((threadIdx.x & 31) == 0) mbar_arrive(&sh->uq_empty[slot]);
+  return u;
+}
 
 constexpr size_t kSmemBytes = 1024 /* alignment slack */ + kStages * (kABytes + kBBytes) + sizeof(TcSmem);
 
@@ -143,6 +169,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&sh->acc_empty[i], 4);
     }
     mbar_init(&sh->drain, 1);
+    for (int i = 0; i < kUQ; ++i) {
+      mbar_init(&sh->uq_full[i], 1);
+      mbar_init(&sh->uq_empty[i], 5);
+    }
     sh->abort = 0;
     fence_barrier_init();
     prefetch_tensormap(&q_map);
@@ -166,7 +196,22 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t ph = 0;
     uint32_t issued = 0, issued_phase = 0;  // per stage: a copy was issued / its phase parity
     bool ok = true;
-    for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
+    // Units are taken dynamically: unit blockIdx.x first, then the next one
+    // from a global counter, so CTAs that drew short units take more.  Each
+    // index goes through the queue to the MMA and epilogue warps.
+    int u = blockIdx.x;
+    for (int j = 0; ok; ++j) {
+      const int slot = j % kUQ;
+      if (!mbar_wait(&sh->uq_empty[slot], ((uint32_t)(j / kUQ) & 1u) ^ 1u, abort, a.max_polls)) {
+        ok = false;
+        break;
+      }
+      if (lane == 0) {
+        sh->uq[slot] = u < n_units ? u : -1;
+        mbar_arrive(&sh->uq_full[slot]);
+      }
+      __syncwarp();
+      if (u >= n_units) break;
       const int4 U = a.units[u];
       const int g = U.x;
       const int a_row = a.bucket_off[g] + U.y * kTcRows;
@@ -198,6 +243,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
       }
+      int next = 0;
+      if (lane == 0) next = (int)gridDim.x + atomicAdd(a.unit_ctr, 1);
+      u = __shfl_sync(kFull, next, 0);
     }
     if (!ok && lane == 0) {
       atomicOr(a.status, 1u);
@@ -217,7 +265,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     int st = 0, acc = 0;
     uint32_t ph = 0, aph = 0;
     bool ok = true;
-    for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
+    for (int j = 0; ok; ++j) {
+      const int u = take_unit(sh, j, abort, a.max_polls, ok);
+      if (u < 0) break;
       const int4 U = a.units[u];
       const int g = U.x;
       const int npg = a.page_off[g + 1] - a.page_off[g];
@@ -280,7 +330,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t aph = 0;
     bool ok = true;
     RowTopK<K> top;
-    for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
+    for (int j = 0; ok; ++j) {
+      const int u = take_unit(sh, j, abort, a.max_polls, ok);
+      if (u < 0) break;
       const int4 U = a.units[u];
       const int g = U.x, c = U.y, sg = U.z;
       const int cg = a.cnt[g];
@@ -355,7 +407,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               const uint32_t xv = (j & 16) ? t2[1] : t2[0];
               if (any) top.insert_later(__uint_as_float(xv), cbase + j);
             }
-            if (valid) thr = fmaxf(thr, top.kth(k));
+            if (valid && most > 0) thr = fmaxf(thr, top.kth(k));
           }
         }
         tc_fence_before();

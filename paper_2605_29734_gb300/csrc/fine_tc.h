@@ -15,6 +15,7 @@ constexpr int kTcMaxK = 32;       // largest k_entries the tensor-core path keep
 struct TcFineArgs {
   const int4 *units;          // (group, bucket chunk, page segment)
   const int32_t *n_units;     // device count of units
+  int32_t *unit_ctr;          // units taken beyond the first per CTA; zero before the launch
   const int32_t *bucket;      // bucket rows -> query id
   const int32_t *bucket_off;  // [G+1]
   const int32_t *cnt;         // [G] bucket sizes

@@ -892,7 +892,7 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   const int wpq = warps_per_query(B, m->sm_count);  // warps per query in top-k and merge
   size_t need = Carver::round(sizeof(float) * (size_t)planes * B * G) + Carver::round(sizeof(uint32_t) * (size_t)G * W) +
                 5 * Carver::round(sizeof(int32_t) * (G + 1)) + Carver::round(sizeof(int64_t) * (G + 1)) +
-                Carver::round(sizeof(int32_t)) +
+                2 * Carver::round(sizeof(int32_t)) +
                 3 * Carver::round(sizeof(int32_t) * rows) + 2 * Carver::round(sizeof(int4) * max_units) +
                 Carver::round(sizeof(float2) * max_parts) + Carver::round(sizeof(float) * max_parts * ke) +
                 Carver::round(sizeof(int32_t) * max_parts * ke) + Carver::round(sizeof(unsigned) * B) +
@@ -909,6 +909,7 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   int64_t *part_off = cv.take<int64_t>(G + 1);
   int32_t *n_units = cv.take<int32_t>(G + 1);  // [0] SIMT units, [1] tensor-core units
   int32_t *seg_tc = cv.take<int32_t>(1);        // pages per tensor-core unit, chosen on the device
+  int32_t *tc_ctr = cv.take<int32_t>(1);        // tensor-core units taken from the shared counter
   int32_t *bucket = cv.take<int32_t>(rows);
   int32_t *bucket_group = cv.take<int32_t>(rows);
   int32_t *pos = cv.take<int32_t>(rows);
@@ -977,6 +978,7 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
     s = make_bf16_tile_map(&q_map, qg, rows, d, kTcRows);
     if (s != HTAM_OK) return s;
     HTAM_CK(cudaMemsetAsync(thr_enc, 0, sizeof(unsigned) * B, st));
+    HTAM_CK(cudaMemsetAsync(tc_ctr, 0, sizeof(int32_t), st));
     s = launch_gather_queries(queries, d, bucket, bucket_group, cnt, rt.tc_min, bucket_off + G, rows, qg, st);
     if (s != HTAM_OK) return s;
     mark.launched();
@@ -1005,7 +1007,7 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   // 3b. Fine scores of large buckets on the tensor cores.
   if (tc_ok) {
     mark.begin(HTAM_PHASE_FINE_TC);
-    TcFineArgs ta{units_tc, n_units + 1, bucket, bucket_off, cnt, m->page_list, m->page_off, m->count, m->slot_id,
+    TcFineArgs ta{units_tc, n_units + 1, tc_ctr, bucket, bucket_off, cnt, m->page_list, m->page_off, m->count, m->slot_id,
                   part_off, d, seg_tc, ke, 1.4426950408889634f / p.tau, part_ml, part_s, part_id, thr_enc,
                   m->status, kMaxPolls};
     s = launch_fine_tc(ta, q_map, m->pool_map, (int)std::min<int64_t>(max_units, m->sm_count), st);
