@@ -251,12 +251,13 @@ struct Route {
   }
 };
 
-// Pages per tensor-core unit: the power of two nearest below the tiles per
-// SM, as pages, within [kTcSegPagesMin, kTcSegPagesMax].  Long segments mean
-// fewer cold top-k lists and fewer partial records; short ones keep every SM
-// busy when the tensor-core work is small.
+// Pages per tensor-core unit: the smallest power of two whose tiles (two
+// pages each) are at least half the tiles per SM, within [kTcSegPagesMin,
+// kTcSegPagesMax].  Long segments mean fewer cold top-k lists and fewer
+// partial records; short ones keep every SM busy when the tensor-core work
+// is small (units are taken dynamically, so a few long ones balance out).
 constexpr int kTcSegPagesMin = 16;
-constexpr int kTcSegPagesMax = 64;
+constexpr int kTcSegPagesMax = 256;
 __device__ __forceinline__ int tc_seg_pages(int64_t tiles, int sms) {
   int seg = kTcSegPagesMin;
   while (seg < kTcSegPagesMax && (int64_t)seg * sms <= tiles) seg *= 2;  // seg/2 tiles <= tiles per SM
