@@ -204,14 +204,12 @@ def cuda_core_kernel(w, stream_rows) -> str:
     return "fine_simt"
 
 
-TC_MIN_BUCKET = 16   # the library's default: buckets this large go to the tensor-core kernel
-
-
-def step_work(w, counts: np.ndarray, group_idx: np.ndarray, tc_min: int = TC_MIN_BUCKET):
+def step_work(w, counts: np.ndarray, group_idx: np.ndarray, tc_min: int):
     """Algorithmic bytes / flops of one query batch, from the groups it selected:
     each selected group's entries read once, the queries read once, and
     2*D flops per (query, candidate entry); split between the CUDA-core kernel
-    (small buckets) and the tensor-core kernel (buckets of >= 16 queries)."""
+    (small buckets) and the tensor-core kernel (buckets of >= tc_min queries,
+    the memory's routing threshold)."""
     s = 2 if w.dtype == "bf16" else 4
     B, D, G = group_idx.shape[0], w.d, w.g
     sel = group_idx[group_idx >= 0]
@@ -320,6 +318,7 @@ def run_htam(args, world, rank, local):
         mem.set_stream_rows(args.stream_rows)
     if args.tc_min_bucket is not None:
         mem.set_tensor_core_min_bucket(args.tc_min_bucket)
+    tc_min = mem.get_tuning(htam.HTAM_TUNE_TC_MIN_BUCKET)
     if args.no_cpu_baseline:
         del entries                  # the memory holds its own copy
         torch.cuda.empty_cache()
@@ -338,7 +337,7 @@ def run_htam(args, world, rank, local):
     work = []
     for q in batches:
         o = mem.query(q, w.k_groups, w.k_entries)
-        work.append(step_work(w, counts, o["group_idx"].cpu().numpy(), args.tc_min_bucket or TC_MIN_BUCKET))
+        work.append(step_work(w, counts, o["group_idx"].cpu().numpy(), tc_min))
     flush_l2 = work[0]["step_bytes"] < 4 * l2_bytes
     flush = torch.empty(2 * l2_bytes, dtype=torch.uint8, device=dev) if flush_l2 else None
 

@@ -226,6 +226,19 @@ htam_status htam_set_tuning(htam_memory *m, htam_tuning key, int32_t value) {
   return HTAM_EINVAL;
 }
 
+htam_status htam_get_tuning(const htam_memory *m, htam_tuning key, int32_t *value) {
+  if (!m || !value) return HTAM_EINVAL;
+  switch (key) {
+    case HTAM_TUNE_TC_MIN_BUCKET:
+      *value = m->tc_min;
+      return HTAM_OK;
+    case HTAM_TUNE_STREAM_ROWS:
+      *value = m->stream_rows;
+      return HTAM_OK;
+  }
+  return HTAM_EINVAL;
+}
+
 htam_status htam_set_phase_timing(htam_memory *m, int enable) {
   if (!m) return HTAM_EINVAL;
   m->timing = enable != 0;

@@ -60,8 +60,8 @@ struct htam_memory {
   int64_t n_queries = 0;
   int64_t phase_launches[HTAM_N_PHASES] = {};
 
-  // Tensor-core fine path: smallest bucket it takes, and the TMA map of the
-  // page pool (built on first use).
+  // Tensor-core fine path: smallest bucket it takes (set at build from d),
+  // and the TMA map of the page pool (built on first use).
   int tc_min = 16;
   // CUDA-core fine path: stream rows through shared memory (1) or load them
   // directly (0).

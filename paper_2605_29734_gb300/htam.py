@@ -23,7 +23,7 @@ HTAM_TUNE_TC_MIN_BUCKET, HTAM_TUNE_STREAM_ROWS = 0, 1
 EXPORTS = (
     "htam_build_memory", "htam_append_transitions", "htam_query", "htam_query_host",
     "htam_select_groups_static", "htam_memory_info", "htam_memory_group_counts", "htam_memory_group_keys",
-    "htam_device_status", "htam_set_tuning", "htam_set_phase_timing",
+    "htam_device_status", "htam_set_tuning", "htam_get_tuning", "htam_set_phase_timing",
     "htam_read_phase_timing", "htam_free_memory", "htam_status_string", "htam_last_error",
     "htam_selftest_wait_timeout",
 )
@@ -69,6 +69,8 @@ def _load() -> ctypes.CDLL:
     lib.htam_select_groups_static.restype = st
     lib.htam_set_tuning.argtypes = [P, ctypes.c_int, i32]
     lib.htam_set_tuning.restype = st
+    lib.htam_get_tuning.argtypes = [P, ctypes.c_int, ctypes.POINTER(i32)]
+    lib.htam_get_tuning.restype = st
     lib.htam_set_phase_timing.argtypes = [P, ctypes.c_int]
     lib.htam_read_phase_timing.argtypes = [P, P, P, P, P]
     for name in ("htam_build_memory", "htam_append_transitions", "htam_query", "htam_query_host",
@@ -215,6 +217,11 @@ class Memory:
 
     def set_tuning(self, key: int, value: int) -> None:
         _check(_lib.htam_set_tuning(self.handle, int(key), int(value)), "htam_set_tuning")
+
+    def get_tuning(self, key: int) -> int:
+        v = ctypes.c_int32()
+        _check(_lib.htam_get_tuning(self.handle, int(key), ctypes.byref(v)), "htam_get_tuning")
+        return v.value
 
     def set_tensor_core_min_bucket(self, min_bucket: int) -> None:
         """Buckets of at least `min_bucket` queries go to the tensor-core kernel."""
