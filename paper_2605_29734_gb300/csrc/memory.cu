@@ -24,7 +24,18 @@ namespace htam {
 
 namespace {
 
-constexpr int kKeySegRows = 1024;  // rows per key partial-sum segment
+constexpr int kKeySegRowsMin = 64;     // rows per key partial-sum segment: at least this,
+constexpr int kKeySegRowsMax = 1024;   // at most this,
+constexpr int64_t kKeySegTarget = 4096;  // and about count / this (bounds the partial-sum buffer)
+
+// Rows per key segment for a batch of `count` rows: short segments for
+// appends (many blocks in parallel), long ones for large builds (a partial
+// sum buffer of about kKeySegTarget + n_groups segments).
+static int key_seg_rows(int64_t count) {
+  int r = kKeySegRowsMin;
+  while (r < kKeySegRowsMax && (int64_t)r * kKeySegTarget < count) r *= 2;
+  return r;
+}
 
 __global__ void count_groups_kernel(const int32_t *__restrict__ gid, int64_t n, int32_t n_groups,
                                     int32_t *__restrict__ counts, int32_t *__restrict__ bad) {
@@ -130,38 +141,50 @@ struct KeyGroup {
 
 // partial[s][j] = sum over rows r0..r1-1 of group g of row[j], accumulated
 // in fp32 with Kahan compensation and returned as fp64 (sum + compensation),
-// so the key error does not grow with the segment length.
+// so the key error does not grow with the segment length.  Rows are loaded
+// eight at a time before any is added, so the loads of a thread overlap.
 template <typename T>
 __global__ void key_partial_kernel(const T *__restrict__ pool, int32_t d,
                                    const int32_t *__restrict__ page_list,
                                    const int32_t *__restrict__ page_off,
                                    const KeySeg *__restrict__ segs, double *__restrict__ partial) {
-  KeySeg sg = segs[blockIdx.x];
-  int j0 = (blockIdx.y * blockDim.x + threadIdx.x) * 8;
+  constexpr int kBatch = 8;
+  const KeySeg sg = segs[blockIdx.x];
+  const int j0 = (blockIdx.y * blockDim.x + threadIdx.x) * 8;
   if (j0 >= d) return;
   float acc[8], comp[8];
 #pragma unroll
   for (int i = 0; i < 8; ++i) acc[i] = comp[i] = 0.f;
   const int32_t *pages = page_list + page_off[sg.g];
-  for (int r = sg.r0; r < sg.r1; ++r) {
-    int64_t slot = (int64_t)pages[r / kPageRows] * kPageRows + (r % kPageRows);
-    const T *row = pool + slot * d + j0;
-    float x[8];
-    if constexpr (sizeof(T) == 2) {
-      uint4 v = *reinterpret_cast<const uint4 *>(row);
-      x[0] = bf16lo(v.x); x[1] = bf16hi(v.x); x[2] = bf16lo(v.y); x[3] = bf16hi(v.y);
-      x[4] = bf16lo(v.z); x[5] = bf16hi(v.z); x[6] = bf16lo(v.w); x[7] = bf16hi(v.w);
-    } else {
-      float4 a = *reinterpret_cast<const float4 *>(row);
-      float4 b = *reinterpret_cast<const float4 *>(row + 4);
-      x[0] = a.x; x[1] = a.y; x[2] = a.z; x[3] = a.w; x[4] = b.x; x[5] = b.y; x[6] = b.z; x[7] = b.w;
+  for (int r = sg.r0; r < sg.r1; r += kBatch) {
+    float x[kBatch][8];
+#pragma unroll
+    for (int u = 0; u < kBatch; ++u) {
+      const int rr = min(r + u, sg.r1 - 1);  // rows past the segment are loaded but not added
+      const int64_t slot = (int64_t)pages[rr / kPageRows] * kPageRows + (rr % kPageRows);
+      const T *row = pool + slot * d + j0;
+      if constexpr (sizeof(T) == 2) {
+        const uint4 v = *reinterpret_cast<const uint4 *>(row);
+        x[u][0] = bf16lo(v.x); x[u][1] = bf16hi(v.x); x[u][2] = bf16lo(v.y); x[u][3] = bf16hi(v.y);
+        x[u][4] = bf16lo(v.z); x[u][5] = bf16hi(v.z); x[u][6] = bf16lo(v.w); x[u][7] = bf16hi(v.w);
+      } else {
+        const float4 a = *reinterpret_cast<const float4 *>(row);
+        const float4 b = *reinterpret_cast<const float4 *>(row + 4);
+        x[u][0] = a.x; x[u][1] = a.y; x[u][2] = a.z; x[u][3] = a.w;
+        x[u][4] = b.x; x[u][5] = b.y; x[u][6] = b.z; x[u][7] = b.w;
+      }
     }
 #pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      float y = x[i] - comp[i];
-      float t = acc[i] + y;
-      comp[i] = (t - acc[i]) - y;
-      acc[i] = t;
+    for (int u = 0; u < kBatch; ++u) {
+      if (r + u < sg.r1) {  // uniform across the block
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const float y = x[u][i] - comp[i];
+          const float t = acc[i] + y;
+          comp[i] = (t - acc[i]) - y;
+          acc[i] = t;
+        }
+      }
     }
   }
   double *out = partial + (int64_t)blockIdx.x * d + j0;
@@ -199,7 +222,10 @@ htam_status ensure_scratch(htam_memory *m, size_t bytes) {
     m->scratch = nullptr;
     m->scratch_bytes = 0;
   }
-  size_t want = std::max(bytes, size_t(1) << 20);
+  // Half again as much as asked: a memory that grows by appends asks for a
+  // little more scratch every query, and each reallocation costs a device
+  // synchronisation (cudaFree) and an allocation.
+  size_t want = std::max(bytes + bytes / 2, size_t(1) << 20);
   if (cudaMalloc(&m->scratch, want) != cudaSuccess) {
     cudaGetLastError();
     m->scratch = nullptr;
@@ -223,8 +249,9 @@ static htam_status add_rows(htam_memory *m, const void *entries, const int32_t *
   int64_t n_chunks = ceil_div(count, chunk);
 
   // Key segments need the final layout; their number is bounded by
-  // count/kKeySegRows + number of groups.
-  int64_t max_segs = count / kKeySegRows + G + 1;
+  // count/seg_rows + number of groups.
+  const int seg_rows = key_seg_rows(count);
+  int64_t max_segs = count / seg_rows + G + 1;
 
   size_t need = Carver::round(sizeof(int32_t) * (G + 1)) + Carver::round(sizeof(int32_t) * count) +
                 Carver::round(sizeof(int32_t) * (size_t)G * n_chunks) +
@@ -280,8 +307,8 @@ static htam_status add_rows(htam_memory *m, const void *entries, const int32_t *
   for (int32_t g = 0; g < G; ++g) {
     if (h_b[g] == 0) continue;
     KeyGroup kg{g, (int32_t)h_segs.size(), 0, (int32_t)new_count[g]};
-    for (int64_t r = m->h_count[g]; r < new_count[g]; r += kKeySegRows) {
-      h_segs.push_back(KeySeg{g, (int32_t)r, (int32_t)std::min<int64_t>(new_count[g], r + kKeySegRows), 0});
+    for (int64_t r = m->h_count[g]; r < new_count[g]; r += seg_rows) {
+      h_segs.push_back(KeySeg{g, (int32_t)r, (int32_t)std::min<int64_t>(new_count[g], r + seg_rows), 0});
     }
     kg.seg1 = (int32_t)h_segs.size();
     h_kg.push_back(kg);
