@@ -289,7 +289,8 @@ static htam_status add_rows(htam_memory *m, const void *entries, const int32_t *
   if (m->n + count > m->capacity || m->n_pages_used + new_pages > m->n_pages_max) {
     return HTAM_ECAPACITY;
   }
-  std::vector<std::vector<int32_t>> pages = m->h_pages;
+  // Every check has passed: from here on the layout is extended in place.
+  std::vector<std::vector<int32_t>> &pages = m->h_pages;
   int64_t next_page = m->n_pages_used;
   std::vector<int32_t> h_off(G + 1), h_list;
   h_list.reserve((size_t)(m->n_pages_used + new_pages));
@@ -361,12 +362,12 @@ static htam_status add_rows(htam_memory *m, const void *entries, const int32_t *
   std::vector<int32_t> h_c32(G);
   for (int32_t g = 0; g < G; ++g) h_c32[g] = (int32_t)new_count[g];
   HTAM_CK(cudaMemcpyAsync(m->count, h_c32.data(), sizeof(int32_t) * G, cudaMemcpyHostToDevice, st));
-  // The host vectors above are pageable: cudaMemcpyAsync has staged them
-  // before returning, but the key/segment tables live in scratch that the
-  // next call may reuse, so finish the queued work before returning.
-  HTAM_CK(cudaStreamSynchronize(st));
+  // The host vectors above are pageable, so cudaMemcpyAsync staged them
+  // before returning; the key and segment tables in scratch are read by the
+  // kernels above in stream order, before any later call on the stream can
+  // reuse the scratch (a reallocation frees it only after a device
+  // synchronisation).  Nothing here needs to wait for the GPU.
   m->h_count.swap(new_count);
-  m->h_pages.swap(pages);
   m->n_pages_used = next_page;
   m->n += count;
   return HTAM_OK;

@@ -248,6 +248,36 @@ def test_cuda_core_rows_streamed_and_loaded_directly(htam, case, stream):
     _check(htam, mem, entries, gid, g, q, kg, ke, tau=0.4, eps=0.02)
 
 
+def test_tuning_defaults_follow_row_length_and_round_trip(htam):
+    """The tensor-core threshold defaults to 2 queries for rows up to 4 KiB
+    and 16 for longer rows; values set are read back; bad keys and values are
+    refused."""
+    for d, want in ((1024, 2), (2048, 2), (4096, 16)):
+        e, gid, _ = _rand_memory(300, d, 3, torch.bfloat16, seed=d)
+        mem = htam.Memory(e, gid, 3)
+        assert mem.get_tuning(htam.HTAM_TUNE_TC_MIN_BUCKET) == want
+        assert mem.get_tuning(htam.HTAM_TUNE_STREAM_ROWS) == 1
+        mem.set_tensor_core_min_bucket(7)
+        mem.set_stream_rows(False)
+        assert mem.get_tuning(htam.HTAM_TUNE_TC_MIN_BUCKET) == 7
+        assert mem.get_tuning(htam.HTAM_TUNE_STREAM_ROWS) == 0
+        with pytest.raises(htam.HtamError):
+            mem.get_tuning(99)
+        with pytest.raises(htam.HtamError):
+            mem.set_tuning(htam.HTAM_TUNE_TC_MIN_BUCKET, 0)
+
+
+@pytest.mark.parametrize("min_bucket", [2, 1 << 30])
+def test_two_query_buckets_on_both_paths(htam, min_bucket):
+    """Buckets of two or three queries (the smallest the tensor cores take by
+    default) scored on the tensor cores and on the CUDA cores."""
+    entries, gid, centres = _rand_memory(20000, 1024, 400, torch.bfloat16, seed=41)
+    q = _rand_queries(60, 1024, torch.bfloat16, seed=41, centres=centres)
+    mem = htam.Memory(entries, gid, 400)
+    mem.set_tensor_core_min_bucket(min_bucket)
+    _check(htam, mem, entries, gid, 400, q, 6, 24, tau=0.5, eps=0.1)
+
+
 @pytest.mark.parametrize("min_bucket", [1, 1 << 30])
 def test_duplicate_bf16_rows_tie_to_lower_id_on_both_paths(htam, min_bucket):
     """Exactly equal scores (duplicate rows spread over pages and chunks)
