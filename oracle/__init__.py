@@ -62,6 +62,8 @@ def _load():
         lib.htam_oracle_stage2.argtypes = [P, ctypes.c_int, P, i64, i32, i32, P, ctypes.c_int, i32, P,
                                            i32, i32, dbl, dbl, P, P, P, P, P, ctypes.c_int]
         lib.htam_oracle_stage2.restype = ctypes.c_int
+        lib.htam_oracle_prefix_reduce.argtypes = [P, ctypes.c_int, i32, i32, i32, dbl, P]
+        lib.htam_oracle_prefix_reduce.restype = ctypes.c_int
         _lib = lib
         return lib
 
@@ -186,3 +188,30 @@ def query(entries: np.ndarray, gid: np.ndarray, n_groups: int, queries: np.ndarr
     out["group_idx"] = gi
     out["group_score"] = gs
     return out
+
+
+def prefix_reduce(prefix: np.ndarray, lam: float) -> np.ndarray:
+    """Prefix-attended query (Eq. 9 over the prefix of Eq. 8, weights of
+    Eq. 10): prefix [b, P, d] (q_P the most recent) -> qbar [b, d] float64,
+    qbar = sum_i exp(-lam * (P - i)) * q_i.  By linearity of the scorer,
+    qbar . c_g is the prefix score of group g."""
+    lib = _load()
+    prefix, dt = _as_input(prefix)
+    b, p_len, d = prefix.shape
+    out = np.empty((b, d), dtype=np.float64)
+    rc = lib.htam_oracle_prefix_reduce(_ptr(prefix), dt, b, p_len, d, float(lam), _ptr(out))
+    if rc != 0:
+        raise ValueError("oracle prefix_reduce: bad argument")
+    return out
+
+
+def round_query(x: np.ndarray, dtype: str) -> np.ndarray:
+    """A float64 query rounded to the memory's dtype as the lookup consumes
+    it: float32 (round to nearest even), or bf16 bits via float32 (each step
+    round to nearest even)."""
+    f = np.asarray(x, dtype=np.float64).astype(np.float32)
+    if dtype == "f32":
+        return f
+    u = f.view(np.uint32).astype(np.uint64)
+    rounded = (u + 0x7FFF + ((u >> 16) & 1)) >> 16
+    return rounded.astype(np.uint16)

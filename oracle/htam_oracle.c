@@ -358,3 +358,30 @@ int htam_oracle_stage2(const void *entries, int e_dtype, const int32_t *gid,
   }
   return status;
 }
+
+/* ------------------------------------------------------- prefix query (N1)
+ * A prefix-attended query (Eq. 9 summed over the global prefix of
+ * Eq. 8 with the position-aware weights of Eq. 10): for a prefix of P state
+ * embeddings q_1..q_P (q_P the most recent),
+ *   score(g) = sum_{i=1..P} alpha_i * (q_i . c_g),
+ *   alpha_i  = exp(-lambda * (P - i)).
+ * The scorer is linear in the query, so score(g) = qbar . c_g with
+ *   qbar = sum_{i=1..P} alpha_i * q_i,
+ * and the rest of the lookup runs on qbar.  This writes qbar in double:
+ * prefix [n_queries, p_len, d] (dtype 0 fp32, 1 bf16 bits), out
+ * [n_queries, d]; the sum runs over i = 1..P in order.  Returns 0, or -1 on a
+ * bad argument. */
+int htam_oracle_prefix_reduce(const void *prefix, int dtype, int32_t n_queries, int32_t p_len, int32_t d,
+                              double lambda, double *out) {
+  if (n_queries < 0 || p_len < 1 || d < 1 || !(lambda >= 0.0)) return -1;
+  for (int32_t b = 0; b < n_queries; ++b) {
+    double *o = out + (int64_t)b * d;
+    for (int32_t j = 0; j < d; ++j) o[j] = 0.0;
+    for (int32_t i = 1; i <= p_len; ++i) {
+      const double alpha = exp(-lambda * (double)(p_len - i));
+      const int64_t row = ((int64_t)b * p_len + (i - 1)) * d;
+      for (int32_t j = 0; j < d; ++j) o[j] += alpha * load_elem(prefix, dtype, row + j);
+    }
+  }
+  return 0;
+}

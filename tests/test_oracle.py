@@ -335,3 +335,68 @@ def test_bad_group_id_rejected():
     x = np.zeros((3, 8), dtype=np.float32)
     with pytest.raises(ValueError):
         oracle.centroids(x, np.array([0, 5, 1], dtype=np.int32), 3)
+
+
+# ------------------------------------------------ prefix-attended query (N1)
+
+def test_prefix_of_one_is_the_query():
+    """A prefix of length 1 has the single weight exp(0) = 1, so the reduced
+    query is the query itself, for any lambda."""
+    rng = np.random.default_rng(11)
+    q = _unit_rows(rng, 6, 32)[:, None, :]
+    for lam in (0.0, 0.5, 3.0):
+        assert np.array_equal(oracle.prefix_reduce(q, lam), q[:, 0, :].astype(np.float64))
+
+
+@pytest.mark.parametrize("lam", [0.0, 0.5, 1.7])
+def test_prefix_weights_newest_one_and_geometric(lam):
+    """With q_i the i-th unit axis vector, coordinate i of the reduced query is
+    alpha_i: the newest element (i = P) weighs exactly 1, and each older one
+    weighs exp(-lambda) times the next (Eq. 10); lambda = 0 weighs all ones."""
+    P = 7
+    q = np.eye(P, 10, dtype=np.float32)[None, :, :]
+    a = oracle.prefix_reduce(q, lam)[0]
+    assert a[P - 1] == 1.0
+    for i in range(P - 1):
+        assert a[i] == pytest.approx(a[i + 1] * math.exp(-lam), rel=1e-14)
+    assert np.all(a[P:] == 0.0)
+
+
+@pytest.mark.parametrize("lam,P", [(0.0, 5), (0.5, 6), (2.0, 3)])
+def test_constant_prefix_sums_a_geometric_series(lam, P):
+    """P copies of one query reduce to that query times sum_{m=0}^{P-1}
+    exp(-lambda m) = (1 - exp(-lambda P)) / (1 - exp(-lambda)) (P at lambda = 0)."""
+    rng = np.random.default_rng(12)
+    q = _unit_rows(rng, 3, 16)
+    prefix = np.repeat(q[:, None, :], P, axis=1)
+    total = P if lam == 0.0 else (1.0 - math.exp(-lam * P)) / (1.0 - math.exp(-lam))
+    np.testing.assert_allclose(oracle.prefix_reduce(prefix, lam), q.astype(np.float64) * total,
+                               rtol=1e-13, atol=0)
+
+
+def test_prefix_scores_are_weighted_stage1_scores():
+    """Eq. 9 summed over the prefix: the group scores of the reduced query are
+    the alpha-weighted sums of the group scores of the prefix elements, each
+    scored on its own by stage 1 (linearity of the scorer)."""
+    rng = np.random.default_rng(13)
+    G, d, P, lam = 12, 24, 5, 0.7
+    entries = _unit_rows(rng, 300, d)
+    gid = rng.integers(0, G, 300).astype(np.int32)
+    cent, counts = oracle.centroids(entries, gid, G)
+    prefix = _unit_rows(rng, 4 * P, d).reshape(4, P, d)
+    alpha = np.empty(P)
+    alpha[P - 1] = 1.0
+    for i in range(P - 2, -1, -1):
+        alpha[i] = alpha[i + 1] * math.exp(-lam)
+
+    def all_scores(qs):
+        gi, gs = oracle.stage1(qs, cent, counts, G)
+        out = np.empty((qs.shape[0], G))
+        for b in range(qs.shape[0]):
+            out[b, gi[b]] = gs[b]
+        return out
+
+    per_elem = np.stack([all_scores(np.ascontiguousarray(prefix[:, i, :])) for i in range(P)], axis=1)
+    want = np.einsum("i,big->bg", alpha, per_elem)
+    got = all_scores(oracle.round_query(oracle.prefix_reduce(prefix, lam), "f32"))
+    np.testing.assert_allclose(got, want, rtol=0, atol=2e-6)

@@ -4,7 +4,8 @@ Each case copies the oracle's C source into a temporary directory, plants one
 plausible slip (tau multiplied instead of divided, the eps/|C| term dropped,
 the tie order reversed, the mean not divided by n_g, the ranking sign flipped,
 a transposed operand, a leak of entries outside the selected groups, empty
-groups allowed into stage 1), builds it there and runs ``test_oracle.py``
+groups allowed into stage 1, prefix weights reversed, of the wrong sign or
+missing the newest element), builds it there and runs ``test_oracle.py``
 against the mutant: at least one pin has to fail.
 """
 import os
@@ -29,6 +30,9 @@ MUTANTS = {
     "restriction_leaks": ("if (!selected[job->gid[e]]) continue;",
                           "if (!selected[job->gid[e]] && e % 7) continue;"),
     "empty_groups_scored": ("if (job->counts[g] == 0) continue;", ""),
+    "prefix_weights_reversed": ("exp(-lambda * (double)(p_len - i))", "exp(-lambda * (double)(i - 1))"),
+    "prefix_weight_sign_flipped": ("exp(-lambda * (double)(p_len - i))", "exp(lambda * (double)(p_len - i))"),
+    "prefix_newest_dropped": ("for (int32_t i = 1; i <= p_len; ++i) {", "for (int32_t i = 1; i < p_len; ++i) {"),
 }
 
 
