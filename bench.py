@@ -57,6 +57,9 @@ def parse_args():
     ap.add_argument("--stream-rows", type=int, default=None, choices=[0, 1],
                     help="CUDA-core path: stream rows through shared memory (1, library default) or load "
                          "them directly (0)")
+    ap.add_argument("--prefix", type=int, default=0,
+                    help="prefix-attended queries (htam_query_prefix) of this many states per query; 0 = plain")
+    ap.add_argument("--prefix-lambda", type=float, default=0.5, help="position-weight decay of the prefix")
     ap.add_argument("--tc-min-bucket", type=int, default=None,
                     help="smallest bucket scored on the tensor cores (library default 16)")
     return ap.parse_args()
@@ -323,21 +326,38 @@ def run_htam(args, world, rank, local):
         del entries                  # the memory holds its own copy
         torch.cuda.empty_cache()
     q_seed = args.seed + 1000 * rank
-    batches = [workloads.make_queries(w, gid, centres, seed=q_seed, stream=4 + 10 * i) for i in range(args.batches)]
+    P = args.prefix
+    if P > 0:
+        # A prefix of P states per query, each drawn by the workload's query
+        # generator (the most recent last).
+        batches = [workloads.make_queries(w, gid, centres, seed=q_seed, stream=4 + 10 * i, b=w.b * P)
+                   .view(w.b, P, w.d).contiguous() for i in range(args.batches)]
+    else:
+        batches = [workloads.make_queries(w, gid, centres, seed=q_seed, stream=4 + 10 * i)
+                   for i in range(args.batches)]
+
+    def run_query(q, out=None):
+        if P > 0:
+            return mem.query_prefix(q, args.prefix_lambda, w.k_groups, w.k_entries, out=out)
+        return mem.query(q, w.k_groups, w.k_entries, out=out)
+
     append_batches = []
     if w.rounds:
         n_rounds = args.warmup + args.steps
         append_batches = [workloads.make_append_batch(w, centres, r, seed=args.seed, device=dev)
                           for r in range(min(n_rounds, w.rounds))]
-    out = mem.query(batches[0], w.k_groups, w.k_entries)
+    out = run_query(batches[0])
     torch.cuda.synchronize()
 
     # Work per batch (the selected groups decide the bytes).
     counts = mem.group_counts().numpy()
     work = []
     for q in batches:
-        o = mem.query(q, w.k_groups, w.k_entries)
-        work.append(step_work(w, counts, o["group_idx"].cpu().numpy(), tc_min))
+        o = run_query(q)
+        wk = step_work(w, counts, o["group_idx"].cpu().numpy(), tc_min)
+        if P > 0:  # the prefix is read once, in place of the query
+            wk["step_bytes"] += (P - 1) * w.b * w.d * (2 if w.dtype == "bf16" else 4)
+        work.append(wk)
     flush_l2 = work[0]["step_bytes"] < 4 * l2_bytes
     flush = torch.empty(2 * l2_bytes, dtype=torch.uint8, device=dev) if flush_l2 else None
 
@@ -345,7 +365,7 @@ def run_htam(args, world, rank, local):
         if w.rounds:
             e, g = append_batches[i % len(append_batches)]
             mem.append(e, g)
-        return mem.query(batches[i % len(batches)], w.k_groups, w.k_entries, out=out)
+        return run_query(batches[i % len(batches)], out=out)
 
     for i in range(args.warmup):
         one_step(i)
@@ -412,8 +432,27 @@ def run_htam(args, world, rank, local):
 
     # End to end: host (pinned) queries in, host results out, through the C ABI.
     host_q = [b.cpu().pin_memory() for b in batches]
-    host_out = mem.query_host(host_q[0], w.k_groups, w.k_entries)
     e2e_steps = max(3, min(args.steps, 50))
+    s_elem = 2 if w.dtype == "bf16" else 4
+    if P > 0:
+        # No host-buffer prefix entry point: pinned copies on the stream
+        # around htam_query_prefix, outputs read back every step.
+        dev_q = torch.empty_like(batches[0])
+        host_out = {k: torch.empty(v.shape, dtype=v.dtype, pin_memory=True) for k, v in out.items()}
+
+        def e2e_query(i):
+            dev_q.copy_(host_q[i % len(host_q)], non_blocking=True)
+            o = run_query(dev_q, out=out)
+            for k in host_out:
+                host_out[k].copy_(o[k], non_blocking=True)
+            torch.cuda.current_stream().synchronize()
+        path = "pinned host prefix copied in, htam_query_prefix, outputs copied out (torch copies on the stream)"
+    else:
+        host_out = mem.query_host(host_q[0], w.k_groups, w.k_entries)
+
+        def e2e_query(i):
+            mem.query_host(host_q[i % len(host_q)], w.k_groups, w.k_entries, out=host_out)
+        path = "htam_query_host (pinned host buffers, copies inside the call)"
     torch.cuda.synchronize()
     barrier(world)
     t0 = time.perf_counter()
@@ -421,22 +460,27 @@ def run_htam(args, world, rank, local):
         if w.rounds:
             e, g = append_batches[i % len(append_batches)]
             mem.append(e, g)
-        mem.query_host(host_q[i % len(host_q)], w.k_groups, w.k_entries, out=host_out)
+        e2e_query(i)
     barrier(world)
     e2e_s = max_over_ranks(time.perf_counter() - t0, world)
-    s_elem = 2 if w.dtype == "bf16" else 4
-    e2e = {"value": w.b * e2e_steps * world / e2e_s, "unit": UNIT, "h2d_bytes_per_step": w.b * w.d * s_elem,
-           "d2h_bytes_per_step": w.b * (w.k_groups * 8 + w.k_entries * 12 + 4), "steps": e2e_steps,
-           "path": "htam_query_host (pinned host buffers, copies inside the call)"}
+    e2e = {"value": w.b * e2e_steps * world / e2e_s, "unit": UNIT,
+           "h2d_bytes_per_step": w.b * max(P, 1) * w.d * s_elem,
+           "d2h_bytes_per_step": w.b * (w.k_groups * 8 + w.k_entries * 12 + 4), "steps": e2e_steps, "path": path}
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        import oracle
+
         entries_np, gid_np = workloads.to_numpy(entries), workloads.to_numpy(gid)
         q_np = np.concatenate([workloads.to_numpy(q) for q in batches])
+        note = ""
+        if P > 0:  # the oracle's prefix reduction (cheap next to the lookup) happens before the timing
+            q_np = oracle.round_query(oracle.prefix_reduce(q_np, args.prefix_lambda), w.dtype)
+            note = f", prefixes of {P} reduced before timing"
         rate, n, dt, threads, _, _ = oracle_rate(w, entries_np, gid_np, q_np, args.cpu_seconds)
         cpu = {"value": rate, "unit": UNIT, "cores": threads, "kind": "oracle",
                "sample": f"{n} queries of {w.name} ({dt:.1f} s), float64 brute force over the same memory, "
-                         f"group keys precomputed"}
+                         f"group keys precomputed{note}"}
 
     if rank == 0:
         line = {
@@ -448,7 +492,8 @@ def run_htam(args, world, rank, local):
                        "mean_candidates_per_query": float(np.mean([x["mean_candidates"] for x in work])),
                        "l2": ("flushed between steps (2x L2 buffer write, outside the step events)" if flush_l2 else
                               f"inputs larger than L2 ({work[0]['step_bytes'] / 1e9:.2f} GB touched per step)"),
-                       "parallelism": f"replicas{world}" if world > 1 else "single GPU"},
+                       "parallelism": f"replicas{world}" if world > 1 else "single GPU",
+                       **({"prefix": P, "prefix_lambda": args.prefix_lambda} if P > 0 else {})},
             "roofline": roofline,
             "step_roofline": {"algorithmic_bytes": step_bytes, "algorithmic_flops": step_flops,
                               "t_roof_ms": 1e3 * t_roof, "frac": t_roof / step_s,

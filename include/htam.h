@@ -129,6 +129,28 @@ htam_status htam_query_host(htam_memory *m, const void *queries, int32_t b,
                             float *entry_score, float *entry_weight,
                             float *lse, void *cuda_stream);
 
+/* Longest prefix htam_query_prefix takes. */
+#define HTAM_MAX_PREFIX 64
+
+/* Prefix-attended lookup.  The global-direction score of Eq. 9 sums the
+ * transition utility over the prefix of earlier directions (Eq. 8) with the
+ * position-aware weights of Eq. 10:
+ *   score(g) = sum_{i=1..P} alpha_i (q_i . c_g),  alpha_i = exp(-lambda (P - i)),
+ * for a prefix q_1..q_P of state embeddings per query, q_P the most recent.
+ * The scorer is linear in the query, so the call forms the reduced query
+ * qbar = sum_i alpha_i q_i on the device (fp32 accumulation over i = 1..P,
+ * rounded once to the memory's dtype) and runs the htam_query lookup on it:
+ * both levels score qbar.
+ *  prefix : [b, p_len, d] of the memory's dtype, device, 16-byte aligned
+ *  p_len  : 1 <= p_len <= HTAM_MAX_PREFIX (p_len = 1 is htam_query itself)
+ *  lambda : >= 0 and finite (the paper gives no value)
+ * Outputs, asynchrony and errors as htam_query.  The reduced queries are kept
+ * in a buffer the memory object owns, grown with cudaMalloc on demand. */
+htam_status htam_query_prefix(htam_memory *m, const void *prefix, int32_t b, int32_t p_len,
+                              float lambda, const htam_query_params *p, int32_t *group_idx,
+                              float *group_score, int32_t *entry_idx, float *entry_score,
+                              float *entry_weight, float *lse, void *cuda_stream);
+
 /* Bytes of the fixed device scratch used by htam_select_groups_static. */
 #define HTAM_STATIC_SCRATCH_BYTES (16u << 20)
 
@@ -192,7 +214,8 @@ typedef enum {
   HTAM_PHASE_FINE = 3,    /* entry scores of small buckets on the CUDA cores */
   HTAM_PHASE_FINE_TC = 4, /* entry scores of large buckets on the tensor cores */
   HTAM_PHASE_MERGE = 5,   /* per-query merge, weights, outputs */
-  HTAM_N_PHASES = 6
+  HTAM_PHASE_PREFIX = 6,  /* reduced queries of htam_query_prefix */
+  HTAM_N_PHASES = 7
 } htam_phase;
 
 /* Tuning knobs of htam_query (all paths return the same results within the

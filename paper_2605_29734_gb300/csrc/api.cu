@@ -2,6 +2,7 @@
 // codes, and the bounded-wait self test.  Every argument error is detected
 // here, before anything is launched.
 
+#include <cmath>
 #include <cstdio>
 #include <cstring>
 
@@ -133,6 +134,40 @@ htam_status htam_query(htam_memory *m, const void *queries, int32_t b, const hta
   if (b > 0 && !aligned16(queries)) return HTAM_EINVAL;
   return query_impl(m, queries, b, *p, group_idx, group_score, entry_idx, entry_score, entry_weight, lse,
                     static_cast<cudaStream_t>(cuda_stream));
+}
+
+htam_status htam_query_prefix(htam_memory *m, const void *prefix, int32_t b, int32_t p_len, float lambda,
+                              const htam_query_params *p, int32_t *group_idx, float *group_score,
+                              int32_t *entry_idx, float *entry_score, float *entry_weight, float *lse,
+                              void *cuda_stream) {
+  htam_status s = check_query_args(m, prefix, b, p, group_idx, group_score, entry_idx, entry_score, entry_weight);
+  if (s != HTAM_OK) return s;
+  if (p_len < 1 || p_len > HTAM_MAX_PREFIX || !(lambda >= 0.f) || !std::isfinite(lambda)) return HTAM_EINVAL;
+  if (b > 0 && !aligned16(prefix)) return HTAM_EINVAL;
+  if (b == 0) return HTAM_OK;
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  const size_t bytes = (size_t)b * m->d * m->elem_bytes;
+  if (bytes > m->prefix_bytes) {
+    if (m->prefix_buf) cudaFree(m->prefix_buf);  // synchronises: no queued work still reads it
+    m->prefix_buf = nullptr;
+    m->prefix_bytes = 0;
+    const size_t want = bytes + bytes / 2;
+    if (cudaMalloc(&m->prefix_buf, want) != cudaSuccess) {
+      cudaGetLastError();
+      return HTAM_ENOMEM;
+    }
+    m->prefix_bytes = want;
+  }
+  PrefixWeights w;
+  for (int i = 1; i <= p_len; ++i) w.alpha[i - 1] = (float)std::exp(-(double)lambda * (double)(p_len - i));
+  PhaseMark mark(m, st);
+  mark.begin(HTAM_PHASE_PREFIX);
+  s = launch_prefix_reduce(m, prefix, b, p_len, w, m->prefix_buf, st);
+  if (s != HTAM_OK) return s;
+  mark.launched();
+  mark.end();
+  return query_impl(m, m->prefix_buf, b, *p, group_idx, group_score, entry_idx, entry_score, entry_weight, lse,
+                    st);
 }
 
 htam_status htam_query_host(htam_memory *m, const void *queries, int32_t b, const htam_query_params *p,

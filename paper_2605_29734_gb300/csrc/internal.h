@@ -51,6 +51,9 @@ struct htam_memory {
   // Device staging for htam_query_host.
   void *stage = nullptr;
   size_t stage_bytes = 0;
+  // Reduced queries of htam_query_prefix.
+  void *prefix_buf = nullptr;
+  size_t prefix_bytes = 0;
 
   // Phase timing and launch counters (htam_set_phase_timing / _read_).
   bool timing = false;
@@ -101,6 +104,16 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t b,
                        int32_t *entry_idx, float *entry_score, float *entry_weight, float *lse,
                        cudaStream_t st);
 void free_impl(htam_memory *m);
+
+// Weights alpha_1..alpha_P of a prefix (Eq. 10), passed by value to the
+// reduction kernel.
+struct PrefixWeights {
+  float alpha[HTAM_MAX_PREFIX];
+};
+// out[q] = sum_i alpha_i prefix[q][i] for b queries ([b, p_len, d] of the
+// memory's dtype in, [b, d] out), fp32 accumulation, one rounding.
+htam_status launch_prefix_reduce(const htam_memory *m, const void *prefix, int32_t b, int32_t p_len,
+                                 const PrefixWeights &w, void *out, cudaStream_t st);
 
 // Records the start / end of a query phase when timing is on, and counts
 // kernel launches per phase.

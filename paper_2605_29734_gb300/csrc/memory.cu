@@ -390,6 +390,7 @@ void free_impl(htam_memory *m) {
   cudaFree(m->status);
   cudaFree(m->scratch);
   cudaFree(m->stage);
+  cudaFree(m->prefix_buf);
   for (cudaEvent_t e : m->ev_pool) cudaEventDestroy(e);
   cudaGetLastError();
   cudaSetDevice(prev);

@@ -18,16 +18,17 @@ LIB_PATH = os.path.join(_PKG, "_lib", "libhtam.so")
 HTAM_OK, HTAM_EINVAL, HTAM_ENOMEM, HTAM_ECAPACITY, HTAM_ECUDA, HTAM_ETIMEOUT, HTAM_ENODEV = range(7)
 HTAM_F32, HTAM_BF16 = 0, 1
 HTAM_TUNE_TC_MIN_BUCKET, HTAM_TUNE_STREAM_ROWS = 0, 1
+HTAM_MAX_PREFIX = 64  # longest prefix htam_query_prefix takes
 
 # Every symbol include/htam.h declares, in declaration order.
 EXPORTS = (
-    "htam_build_memory", "htam_append_transitions", "htam_query", "htam_query_host",
+    "htam_build_memory", "htam_append_transitions", "htam_query", "htam_query_host", "htam_query_prefix",
     "htam_select_groups_static", "htam_memory_info", "htam_memory_group_counts", "htam_memory_group_keys",
     "htam_device_status", "htam_set_tuning", "htam_get_tuning", "htam_set_phase_timing",
     "htam_read_phase_timing", "htam_free_memory", "htam_status_string", "htam_last_error",
     "htam_selftest_wait_timeout",
 )
-PHASES = ("coarse", "select", "bucket", "fine", "fine_tc", "merge")
+PHASES = ("coarse", "select", "bucket", "fine", "fine_tc", "merge", "prefix")
 
 
 class HtamError(RuntimeError):
@@ -54,6 +55,8 @@ def _load() -> ctypes.CDLL:
     qargs = [P, P, i32, ctypes.POINTER(QueryParams), P, P, P, P, P, P, P]
     lib.htam_query.argtypes = qargs
     lib.htam_query_host.argtypes = qargs
+    lib.htam_query_prefix.argtypes = [P, P, i32, i32, ctypes.c_float, ctypes.POINTER(QueryParams),
+                                      P, P, P, P, P, P, P]
     lib.htam_memory_info.argtypes = [P, P, P, P, P]
     lib.htam_memory_group_counts.argtypes = [P, P]
     lib.htam_memory_group_keys.argtypes = [P, P, P]
@@ -170,6 +173,31 @@ class Memory:
                                _dev_ptr(out["entry_idx"]), _dev_ptr(out["entry_score"]),
                                _dev_ptr(out["entry_weight"]), _dev_ptr(out.get("lse")),
                                _stream_ptr(stream)), "htam_query")
+        return out
+
+    def query_prefix(self, prefix: torch.Tensor, lam: float, k_groups: int, k_entries: int, tau: float = 1.0,
+                     epsilon: float = 0.0, stream=None, out: dict | None = None) -> dict:
+        """Prefix-attended lookup: prefix [b, P, d] of the memory dtype (the
+        most recent state last), position weights exp(-lam * (P - i))."""
+        if prefix.dtype != self.dtype or prefix.dim() != 3 or prefix.shape[2] != self.d:
+            raise ValueError("prefix must be [b, P, d] of the memory dtype")
+        b, p_len = prefix.shape[0], prefix.shape[1]
+        dev = prefix.device
+        if out is None:
+            out = {
+                "group_idx": torch.empty(b, k_groups, dtype=torch.int32, device=dev),
+                "group_score": torch.empty(b, k_groups, dtype=torch.float32, device=dev),
+                "entry_idx": torch.empty(b, k_entries, dtype=torch.int32, device=dev),
+                "entry_score": torch.empty(b, k_entries, dtype=torch.float32, device=dev),
+                "entry_weight": torch.empty(b, k_entries, dtype=torch.float32, device=dev),
+                "lse": torch.empty(b, dtype=torch.float32, device=dev),
+            }
+        p = QueryParams(k_groups, k_entries, tau, epsilon)
+        _check(_lib.htam_query_prefix(self.handle, _dev_ptr(prefix), b, p_len, float(lam), ctypes.byref(p),
+                                      _dev_ptr(out["group_idx"]), _dev_ptr(out["group_score"]),
+                                      _dev_ptr(out["entry_idx"]), _dev_ptr(out["entry_score"]),
+                                      _dev_ptr(out["entry_weight"]), _dev_ptr(out.get("lse")),
+                                      _stream_ptr(stream)), "htam_query_prefix")
         return out
 
     def query_host(self, queries: torch.Tensor, k_groups: int, k_entries: int, tau: float = 1.0,

@@ -248,6 +248,61 @@ def test_cuda_core_rows_streamed_and_loaded_directly(htam, case, stream):
     _check(htam, mem, entries, gid, g, q, kg, ke, tau=0.4, eps=0.02)
 
 
+PREFIX_CASES = [
+    # n, groups, d, dtype, batch, prefix length, lambda, k_groups, k_entries
+    (8000, 40, 256, torch.float32, 30, 4, 0.5, 5, 12),
+    (20000, 100, 1024, torch.bfloat16, 70, 6, 0.5, 6, 24),
+    (6000, 30, 512, torch.bfloat16, 300, 3, 1.3, 4, 16),   # buckets large enough for the tensor cores
+    (3000, 12, 512, torch.bfloat16, 9, 1, 0.0, 3, 8),      # one element: the plain lookup
+]
+
+
+@pytest.mark.parametrize("case", PREFIX_CASES)
+def test_prefix_query_matches_oracle(htam, case):
+    """htam_query_prefix against the oracle's reduced query (Eq. 9 summed over
+    the prefix with the Eq. 10 weights), rounded to the memory's dtype the way
+    the lookup consumes it, then the oracle lookup."""
+    import oracle
+
+    n, g, d, dtype, b, P, lam, kg, ke = case
+    entries, gid, centres = _rand_memory(n, d, g, dtype, seed=n + P)
+    prefix = _rand_queries(b * P, d, dtype, seed=n + P, centres=centres).view(b, P, d).contiguous()
+    mem = htam.Memory(entries, gid, g)
+    out = mem.query_prefix(prefix, lam, kg, ke, tau=0.7, epsilon=0.05)
+    torch.cuda.synchronize()
+    dt = "bf16" if dtype == torch.bfloat16 else "f32"
+    qbar = oracle.round_query(oracle.prefix_reduce(to_numpy(prefix), lam), dt)
+    problems = compare_lookup(out, to_numpy(entries), to_numpy(gid), g, qbar, kg, ke, 0.7, 0.05, dt)
+    assert not problems, "\n".join(problems[:20])
+    assert mem.device_status() == htam.HTAM_OK
+
+
+def test_prefix_of_one_equals_plain_query_bitwise(htam):
+    entries, gid, centres = _rand_memory(5000, 512, 20, torch.bfloat16, seed=3)
+    q = _rand_queries(40, 512, torch.bfloat16, seed=3, centres=centres)
+    mem = htam.Memory(entries, gid, 20)
+    a = mem.query(q, 4, 16, tau=0.5, epsilon=0.1)
+    p = mem.query_prefix(q.view(40, 1, 512).contiguous(), 2.0, 4, 16, tau=0.5, epsilon=0.1)
+    torch.cuda.synchronize()
+    for k in a:
+        assert torch.equal(a[k], p[k]), k
+
+
+def test_prefix_arguments_checked(htam):
+    entries, gid, _ = _rand_memory(500, 64, 4, torch.float32, seed=4)
+    mem = htam.Memory(entries, gid, 4)
+    ok = torch.zeros(3, 2, 64, device=DEV)
+    for bad_len in (0, htam.HTAM_MAX_PREFIX + 1):
+        pre = torch.zeros(3, max(bad_len, 1), 64, device=DEV)
+        if bad_len == 0:
+            pre = pre[:, :0, :].contiguous()
+        with pytest.raises((htam.HtamError, ValueError)):
+            mem.query_prefix(pre, 0.5, 2, 4)
+    for lam in (-0.1, float("inf"), float("nan")):
+        with pytest.raises(htam.HtamError):
+            mem.query_prefix(ok, lam, 2, 4)
+
+
 def test_tuning_defaults_follow_row_length_and_round_trip(htam):
     """The tensor-core threshold defaults to 2 queries for rows up to 4 KiB
     and 16 for longer rows; values set are read back; bad keys and values are
