@@ -64,6 +64,10 @@ def _load():
         lib.htam_oracle_stage2.restype = ctypes.c_int
         lib.htam_oracle_prefix_reduce.argtypes = [P, ctypes.c_int, i32, i32, i32, dbl, P]
         lib.htam_oracle_prefix_reduce.restype = ctypes.c_int
+        lib.htam_oracle_edge_scores.argtypes = [P, i32, i32, P, P, i32, i32, dbl, P]
+        lib.htam_oracle_edge_scores.restype = ctypes.c_int
+        lib.htam_oracle_select.argtypes = [P, P, i32, i32, i32, P, P]
+        lib.htam_oracle_select.restype = ctypes.c_int
         _lib = lib
         return lib
 
@@ -215,3 +219,49 @@ def round_query(x: np.ndarray, dtype: str) -> np.ndarray:
     u = f.view(np.uint32).astype(np.uint64)
     rounded = (u + 0x7FFF + ((u >> 16) & 1)) >> 16
     return rounded.astype(np.uint16)
+
+
+def edge_scores(Z: np.ndarray, w: np.ndarray, prefix: np.ndarray, lam: float) -> np.ndarray:
+    """Edge-table router scores (Eq. 9 with the App. B.6 utility phi = w . z
+    and the Eq. 10 weights): Z [G, G, F] float32 (from, to, feature), w [F],
+    prefix [b, P] int32 group ids (-1 = none) -> [b, G] float64."""
+    lib = _load()
+    Z = np.ascontiguousarray(Z, dtype=np.float32)
+    G, G2, F = Z.shape
+    if G2 != G:
+        raise ValueError("Z must be [G, G, F]")
+    w = np.ascontiguousarray(w, dtype=np.float64)
+    prefix = np.ascontiguousarray(prefix, dtype=np.int32)
+    b, p_len = prefix.shape
+    out = np.empty((b, G), dtype=np.float64)
+    rc = lib.htam_oracle_edge_scores(_ptr(Z), G, F, _ptr(w), _ptr(prefix), b, p_len, float(lam), _ptr(out))
+    if rc != 0:
+        raise ValueError("oracle edge_scores: bad argument")
+    return out
+
+
+def select(scores: np.ndarray, counts: np.ndarray, k: int):
+    """The k best groups of per-group scores, ranked like stage 1 (score
+    descending, ties to the lower id, empty groups excluded, -1/-inf padding)."""
+    lib = _load()
+    scores = np.ascontiguousarray(scores, dtype=np.float64)
+    counts = np.ascontiguousarray(counts, dtype=np.int64)
+    b, G = scores.shape
+    gi = np.empty((b, k), dtype=np.int32)
+    gs = np.empty((b, k), dtype=np.float64)
+    if lib.htam_oracle_select(_ptr(scores), _ptr(counts), b, G, int(k), _ptr(gi), _ptr(gs)) != 0:
+        raise MemoryError("oracle select")
+    return gi, gs
+
+
+def query_edges(entries: np.ndarray, gid: np.ndarray, n_groups: int, Z: np.ndarray, w: np.ndarray,
+                prefix: np.ndarray, lam: float, queries: np.ndarray, k_groups: int, k_entries: int,
+                tau: float = 1.0, eps: float = 0.0, nthreads: int | None = None):
+    """The lookup with the edge-table router as stage 1 (the paper's global
+    direction choice) and the query embeddings for stage 2 (the local pick)."""
+    counts = np.bincount(np.asarray(gid, dtype=np.int64), minlength=n_groups)
+    gi, gs = select(edge_scores(Z, w, prefix, lam), counts, k_groups)
+    out = stage2(entries, gid, n_groups, queries, gi, k_entries, tau, eps, nthreads)
+    out["group_idx"] = gi
+    out["group_score"] = gs
+    return out

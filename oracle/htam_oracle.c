@@ -385,3 +385,62 @@ int htam_oracle_prefix_reduce(const void *prefix, int dtype, int32_t n_queries, 
   }
   return 0;
 }
+
+/* ------------------------------------------------ edge-table routing (N2)
+ * The global router of Eq. 9 with the transition utility of App. B.6: the
+ * utility of moving from direction g_i to direction g is a fixed linear
+ * reward over the edge's feature vector, phi(g_i, g) = w . z(g_i, g).  The
+ * features come from a table Z [G, G, F] of float32 (row = from, column =
+ * to).  For a prefix p_1..p_P of earlier group ids per query (-1 = no
+ * element, contributes nothing) and the weights alpha_i = exp(-lambda (P - i))
+ * of Eq. 10,
+ *   score[b][g] = sum_{i = 1..P, p_i >= 0} alpha_i * sum_{f} w_f Z[p_i][g][f],
+ * summed in index order in double.  Returns 0, or -1 on a bad argument. */
+int htam_oracle_edge_scores(const float *Z, int32_t G, int32_t F, const double *w, const int32_t *prefix,
+                            int32_t n_queries, int32_t p_len, double lambda, double *out) {
+  if (G < 1 || F < 1 || n_queries < 0 || p_len < 1 || !(lambda >= 0.0)) return -1;
+  for (int32_t b = 0; b < n_queries; ++b) {
+    double *o = out + (int64_t)b * G;
+    for (int32_t g = 0; g < G; ++g) o[g] = 0.0;
+    for (int32_t i = 1; i <= p_len; ++i) {
+      const int32_t from = prefix[(int64_t)b * p_len + (i - 1)];
+      if (from < 0) continue;
+      if (from >= G) return -1;
+      const double alpha = exp(-lambda * (double)(p_len - i));
+      for (int32_t g = 0; g < G; ++g) {
+        const float *z = Z + ((int64_t)from * G + g) * F;
+        double phi = 0.0;
+        for (int32_t f = 0; f < F; ++f) phi += w[f] * (double)z[f];
+        o[g] += alpha * phi;
+      }
+    }
+  }
+  return 0;
+}
+
+/* The k best groups of given per-group scores, ranked as stage 1 ranks them:
+ * score descending, ties to the lower group id, empty groups (counts 0)
+ * never candidates, -1 / -inf padding.  Returns 0, or -2 on allocation
+ * failure. */
+int htam_oracle_select(const double *scores, const int64_t *counts, int32_t n_queries, int32_t G, int32_t k,
+                       int32_t *group_idx, double *group_score) {
+  scored_t *cand = (scored_t *)malloc(sizeof(scored_t) * (size_t)G);
+  if (!cand) return -2;
+  for (int32_t b = 0; b < n_queries; ++b) {
+    int32_t n_cand = 0;
+    for (int32_t g = 0; g < G; ++g) {
+      if (counts[g] == 0) continue;
+      cand[n_cand].score = scores[(int64_t)b * G + g];
+      cand[n_cand].id = g;
+      ++n_cand;
+    }
+    qsort(cand, (size_t)n_cand, sizeof(scored_t), by_score_then_id);
+    for (int32_t j = 0; j < k; ++j) {
+      const int64_t o = (int64_t)b * k + j;
+      group_idx[o] = j < n_cand ? (int32_t)cand[j].id : -1;
+      group_score[o] = j < n_cand ? cand[j].score : -INFINITY;
+    }
+  }
+  free(cand);
+  return 0;
+}

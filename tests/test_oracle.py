@@ -400,3 +400,66 @@ def test_prefix_scores_are_weighted_stage1_scores():
     want = np.einsum("i,big->bg", alpha, per_elem)
     got = all_scores(oracle.round_query(oracle.prefix_reduce(prefix, lam), "f32"))
     np.testing.assert_allclose(got, want, rtol=0, atol=2e-6)
+
+
+# ------------------------------------------------ edge-table routing (N2)
+
+def test_edge_scores_one_hot_weights_read_the_feature_slice():
+    """With w the f-th unit vector and a one-element prefix (weight 1), the
+    score of g is the f-th feature of the edge from the prefix group to g:
+    Z[p, g, f] (row = from, column = to)."""
+    rng = np.random.default_rng(21)
+    G, F = 7, 4
+    Z = rng.standard_normal((G, G, F)).astype(np.float32)
+    prefix = np.array([[3], [0], [6]], dtype=np.int32)
+    for f in range(F):
+        w = np.zeros(F)
+        w[f] = 1.0
+        s = oracle.edge_scores(Z, w, prefix, 0.8)
+        for b, p in enumerate(prefix[:, 0]):
+            assert np.array_equal(s[b], Z[p, :, f].astype(np.float64))
+
+
+def test_edge_scores_linear_in_weights():
+    rng = np.random.default_rng(22)
+    G, F = 9, 12
+    Z = rng.standard_normal((G, G, F)).astype(np.float32)
+    prefix = rng.integers(-1, G, (5, 4)).astype(np.int32)
+    w1, w2 = rng.standard_normal(F), rng.standard_normal(F)
+    np.testing.assert_allclose(oracle.edge_scores(Z, w1 + w2, prefix, 0.3),
+                               oracle.edge_scores(Z, w1, prefix, 0.3) + oracle.edge_scores(Z, w2, prefix, 0.3),
+                               rtol=0, atol=1e-12)
+
+
+@pytest.mark.parametrize("lam", [0.0, 0.6])
+def test_edge_prefix_weights_newest_one_and_geometric(lam):
+    """Z has a 1 on every edge leaving group k (feature 0) and 0 elsewhere, so
+    a prefix holding k at one position and nothing (-1) elsewhere scores every
+    group with that position's weight (Eq. 10): 1 for the newest, e^{-lambda}
+    times the next one for each older; an empty prefix scores 0."""
+    G, F, P, k = 6, 2, 5, 4
+    Z = np.zeros((G, G, F), dtype=np.float32)
+    Z[k, :, 0] = 1.0
+    w = np.array([1.0, 0.0])
+    prefix = np.full((P + 1, P), -1, dtype=np.int32)
+    for i in range(P):
+        prefix[i, i] = k
+    s = oracle.edge_scores(Z, w, prefix, lam)
+    assert np.all(s[P - 1] == 1.0)
+    for i in range(P - 1):
+        np.testing.assert_allclose(s[i], s[i + 1] * math.exp(-lam), rtol=1e-14)
+    assert np.all(s[P] == 0.0)
+
+
+def test_select_matches_lexsort_without_empty_groups():
+    rng = np.random.default_rng(23)
+    b, G, k = 6, 30, 8
+    scores = np.round(rng.standard_normal((b, G)), 1)       # many ties
+    counts = rng.integers(0, 3, G)
+    gi, gs = oracle.select(scores, counts, k)
+    for q in range(b):
+        live = np.nonzero(counts > 0)[0]
+        order = live[np.lexsort((live, -scores[q, live]))][:k]
+        assert list(gi[q, :len(order)]) == list(order)
+        assert np.all(gi[q, len(order):] == -1)
+        np.testing.assert_array_equal(gs[q, :len(order)], scores[q, order])

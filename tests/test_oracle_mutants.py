@@ -5,7 +5,8 @@ plausible slip (tau multiplied instead of divided, the eps/|C| term dropped,
 the tie order reversed, the mean not divided by n_g, the ranking sign flipped,
 a transposed operand, a leak of entries outside the selected groups, empty
 groups allowed into stage 1, prefix weights reversed, of the wrong sign or
-missing the newest element), builds it there and runs ``test_oracle.py``
+missing the newest element, edge-table rows and columns swapped, an edge
+feature misread, edge-prefix weights reversed), builds it there and runs ``test_oracle.py``
 against the mutant: at least one pin has to fail.
 """
 import os
@@ -33,6 +34,10 @@ MUTANTS = {
     "prefix_weights_reversed": ("exp(-lambda * (double)(p_len - i))", "exp(-lambda * (double)(i - 1))"),
     "prefix_weight_sign_flipped": ("exp(-lambda * (double)(p_len - i))", "exp(lambda * (double)(p_len - i))"),
     "prefix_newest_dropped": ("for (int32_t i = 1; i <= p_len; ++i) {", "for (int32_t i = 1; i < p_len; ++i) {"),
+    "edge_from_to_transposed": ("Z + ((int64_t)from * G + g) * F", "Z + ((int64_t)g * G + from) * F"),
+    "edge_feature_misread": ("phi += w[f] * (double)z[f];", "phi += w[f] * (double)z[(f + 1) % F];"),
+    "edge_weights_reversed": ("const double alpha = exp(-lambda * (double)(p_len - i));\n      for (int32_t g",
+                              "const double alpha = exp(-lambda * (double)(i - 1));\n      for (int32_t g"),
 }
 
 
