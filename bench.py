@@ -60,6 +60,10 @@ def parse_args():
     ap.add_argument("--prefix", type=int, default=0,
                     help="prefix-attended queries (htam_query_prefix) of this many states per query; 0 = plain")
     ap.add_argument("--prefix-lambda", type=float, default=0.5, help="position-weight decay of the prefix")
+    ap.add_argument("--edges", type=int, default=0,
+                    help="route stage 1 by a transition-edge table (htam_query_edges) with prefixes of this "
+                         "many earlier groups; 0 = group keys")
+    ap.add_argument("--edge-features", type=int, default=12, help="features per edge (12 in App. B.6)")
     ap.add_argument("--tc-min-bucket", type=int, default=None,
                     help="smallest bucket scored on the tensor cores (library default 16)")
     return ap.parse_args()
@@ -336,7 +340,22 @@ def run_htam(args, world, rank, local):
         batches = [workloads.make_queries(w, gid, centres, seed=q_seed, stream=4 + 10 * i)
                    for i in range(args.batches)]
 
+    E = args.edges
+    if E > 0:
+        # A synthetic transition-edge table (features ~ N(0, 1)), a fixed
+        # weight vector, and per batch a prefix of E earlier groups per query
+        # drawn uniformly (the most recent last).
+        rng = np.random.default_rng(args.seed + 7)
+        edge_z = torch.randn(w.g, w.g, args.edge_features, device=dev,
+                             generator=torch.Generator(device=dev).manual_seed(args.seed + 7))
+        edge_w = rng.standard_normal(args.edge_features).astype(np.float32)
+        edge_prefix = [rng.integers(0, w.g, (w.b, E)).astype(np.int32) for _ in range(args.batches)]
+    batch_of = {id(q): i for i, q in enumerate(batches)}
+
     def run_query(q, out=None):
+        if E > 0:
+            return mem.query_edges(edge_z, edge_w, edge_prefix[batch_of.get(id(q), 0)], args.prefix_lambda, q,
+                                   w.k_groups, w.k_entries, out=out)
         if P > 0:
             return mem.query_prefix(q, args.prefix_lambda, w.k_groups, w.k_entries, out=out)
         return mem.query(q, w.k_groups, w.k_entries, out=out)
@@ -357,6 +376,10 @@ def run_htam(args, world, rank, local):
         wk = step_work(w, counts, o["group_idx"].cpu().numpy(), tc_min)
         if P > 0:  # the prefix is read once, in place of the query
             wk["step_bytes"] += (P - 1) * w.b * w.d * (2 if w.dtype == "bf16" else 4)
+        if E > 0:  # stage 1 reads the referenced edge-table rows instead of the group keys
+            rows = len(np.unique(edge_prefix[len(work)]))
+            wk["step_bytes"] += rows * w.g * args.edge_features * 4 - w.g * w.d * 4
+            wk["step_flops"] += 2.0 * args.edge_features * E * w.b * w.g - 2.0 * w.d * w.b * w.g
         work.append(wk)
     flush_l2 = work[0]["step_bytes"] < 4 * l2_bytes
     flush = torch.empty(2 * l2_bytes, dtype=torch.uint8, device=dev) if flush_l2 else None
@@ -434,19 +457,22 @@ def run_htam(args, world, rank, local):
     host_q = [b.cpu().pin_memory() for b in batches]
     e2e_steps = max(3, min(args.steps, 50))
     s_elem = 2 if w.dtype == "bf16" else 4
-    if P > 0:
-        # No host-buffer prefix entry point: pinned copies on the stream
-        # around htam_query_prefix, outputs read back every step.
+    if P > 0 or E > 0:
+        # No host-buffer entry point for these lookups: pinned copies on the
+        # stream around the call, outputs read back every step.
         dev_q = torch.empty_like(batches[0])
+        batch_of[id(dev_q)] = 0
         host_out = {k: torch.empty(v.shape, dtype=v.dtype, pin_memory=True) for k, v in out.items()}
 
         def e2e_query(i):
             dev_q.copy_(host_q[i % len(host_q)], non_blocking=True)
+            batch_of[id(dev_q)] = i % len(host_q)
             o = run_query(dev_q, out=out)
             for k in host_out:
                 host_out[k].copy_(o[k], non_blocking=True)
             torch.cuda.current_stream().synchronize()
-        path = "pinned host prefix copied in, htam_query_prefix, outputs copied out (torch copies on the stream)"
+        path = ("pinned host queries copied in, " + ("htam_query_edges" if E > 0 else "htam_query_prefix") +
+                ", outputs copied out (torch copies on the stream)")
     else:
         host_out = mem.query_host(host_q[0], w.k_groups, w.k_entries)
 
@@ -477,7 +503,22 @@ def run_htam(args, world, rank, local):
         if P > 0:  # the oracle's prefix reduction (cheap next to the lookup) happens before the timing
             q_np = oracle.round_query(oracle.prefix_reduce(q_np, args.prefix_lambda), w.dtype)
             note = f", prefixes of {P} reduced before timing"
-        rate, n, dt, threads, _, _ = oracle_rate(w, entries_np, gid_np, q_np, args.cpu_seconds)
+        if E > 0:  # the oracle's edge-routed lookup on a bounded sample of batch 0
+            threads = oracle.default_threads()
+            z_np, pre_np = edge_z.cpu().numpy(), edge_prefix[0]
+            t0 = time.perf_counter()
+            oracle.query_edges(entries_np, gid_np, w.g, z_np, edge_w, pre_np[:threads], args.prefix_lambda,
+                               q_np[:threads], w.k_groups, w.k_entries, nthreads=threads)
+            t_probe = max(time.perf_counter() - t0, 1e-6)
+            n = int(min(w.b, max(threads, threads * args.cpu_seconds / t_probe)))
+            t0 = time.perf_counter()
+            oracle.query_edges(entries_np, gid_np, w.g, z_np, edge_w, pre_np[:n], args.prefix_lambda, q_np[:n],
+                               w.k_groups, w.k_entries, nthreads=threads)
+            dt = time.perf_counter() - t0
+            rate = n / dt
+            note = ", edge-routed (float64 edge scores over the same table)"
+        else:
+            rate, n, dt, threads, _, _ = oracle_rate(w, entries_np, gid_np, q_np, args.cpu_seconds)
         cpu = {"value": rate, "unit": UNIT, "cores": threads, "kind": "oracle",
                "sample": f"{n} queries of {w.name} ({dt:.1f} s), float64 brute force over the same memory, "
                          f"group keys precomputed{note}"}
@@ -493,7 +534,9 @@ def run_htam(args, world, rank, local):
                        "l2": ("flushed between steps (2x L2 buffer write, outside the step events)" if flush_l2 else
                               f"inputs larger than L2 ({work[0]['step_bytes'] / 1e9:.2f} GB touched per step)"),
                        "parallelism": f"replicas{world}" if world > 1 else "single GPU",
-                       **({"prefix": P, "prefix_lambda": args.prefix_lambda} if P > 0 else {})},
+                       **({"prefix": P, "prefix_lambda": args.prefix_lambda} if P > 0 else {}),
+                       **({"edges_prefix": E, "edge_features": args.edge_features,
+                           "prefix_lambda": args.prefix_lambda} if E > 0 else {})},
             "roofline": roofline,
             "step_roofline": {"algorithmic_bytes": step_bytes, "algorithmic_flops": step_flops,
                               "t_roof_ms": 1e3 * t_roof, "frac": t_roof / step_s,

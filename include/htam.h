@@ -151,6 +151,35 @@ htam_status htam_query_prefix(htam_memory *m, const void *prefix, int32_t b, int
                               float *group_score, int32_t *entry_idx, float *entry_score,
                               float *entry_weight, float *lse, void *cuda_stream);
 
+/* Most features per edge htam_query_edges takes. */
+#define HTAM_MAX_EDGE_FEATURES 32
+
+/* Lookup routed by transition edges: the global router of Eq. 9 with the
+ * transition utility of App. B.6, a fixed linear reward over the features of
+ * the edge between two directions, phi(g_i, g) = w . z(g_i, g), summed over a
+ * prefix of earlier directions with the weights of Eq. 10:
+ *   score(g) = sum_{i=1..P} alpha_i w . Z[p_i][g][:],  alpha_i = exp(-lambda (P - i)).
+ * These scores replace the group-key scores of stage 1 (the top k_groups
+ * groups by score, ties to the lower id, empty groups never chosen,
+ * group_score = these scores); stage 2 scores the selected groups' entries
+ * against `queries` as htam_query does.
+ *  edge_features : [n_groups, n_groups, n_features] fp32, device, 16-byte
+ *                  aligned, row = from, column = to (caller-owned)
+ *  n_features    : 1 <= n_features <= HTAM_MAX_EDGE_FEATURES (12 in App. B.6)
+ *  weights       : [n_features] fp32, HOST, finite
+ *  prefix_groups : [b, p_len] int32, HOST, group ids in [0, n_groups) or -1
+ *                  for no element (contributes nothing); the most recent last
+ *  p_len, lambda : as htam_query_prefix
+ *  queries       : [b, d] of the memory's dtype, device (the stage-2 states)
+ * Outputs, asynchrony and errors as htam_query (EINVAL also for a prefix id
+ * out of range); the prefix is copied to the device inside the call. */
+htam_status htam_query_edges(htam_memory *m, const float *edge_features, int32_t n_features,
+                             const float *weights, const int32_t *prefix_groups, int32_t p_len,
+                             float lambda, const void *queries, int32_t b,
+                             const htam_query_params *p, int32_t *group_idx, float *group_score,
+                             int32_t *entry_idx, float *entry_score, float *entry_weight,
+                             float *lse, void *cuda_stream);
+
 /* Bytes of the fixed device scratch used by htam_select_groups_static. */
 #define HTAM_STATIC_SCRATCH_BYTES (16u << 20)
 

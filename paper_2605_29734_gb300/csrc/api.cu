@@ -170,6 +170,39 @@ htam_status htam_query_prefix(htam_memory *m, const void *prefix, int32_t b, int
                     st);
 }
 
+htam_status htam_query_edges(htam_memory *m, const float *edge_features, int32_t n_features, const float *weights,
+                             const int32_t *prefix_groups, int32_t p_len, float lambda, const void *queries, int32_t b,
+                             const htam_query_params *p, int32_t *group_idx, float *group_score, int32_t *entry_idx,
+                             float *entry_score, float *entry_weight, float *lse, void *cuda_stream) {
+  htam_status s = check_query_args(m, queries, b, p, group_idx, group_score, entry_idx, entry_score, entry_weight);
+  if (s != HTAM_OK) return s;
+  if (b > 0 && !aligned16(queries)) return HTAM_EINVAL;
+  if (!edge_features || !aligned16(edge_features) || !weights || n_features < 1 ||
+      n_features > HTAM_MAX_EDGE_FEATURES) {
+    return HTAM_EINVAL;
+  }
+  if (p_len < 1 || p_len > HTAM_MAX_PREFIX || !(lambda >= 0.f) || !std::isfinite(lambda)) return HTAM_EINVAL;
+  if (b > 0 && !prefix_groups) return HTAM_EINVAL;
+  for (int f = 0; f < n_features; ++f) {
+    if (!std::isfinite(weights[f])) return HTAM_EINVAL;
+  }
+  for (int64_t i = 0; i < (int64_t)b * p_len; ++i) {
+    if (prefix_groups[i] < -1 || prefix_groups[i] >= m->n_groups) return HTAM_EINVAL;
+  }
+  if (b == 0) return HTAM_OK;
+  EdgeRoute er;
+  er.Z = edge_features;
+  er.prefix = prefix_groups;
+  er.F = n_features;
+  er.P = p_len;
+  for (int f = 0; f < HTAM_MAX_EDGE_FEATURES; ++f) er.w[f] = f < n_features ? weights[f] : 0.f;
+  for (int i = 0; i < HTAM_MAX_PREFIX; ++i) {
+    er.alpha[i] = i < p_len ? (float)std::exp(-(double)lambda * (double)(p_len - 1 - i)) : 0.f;
+  }
+  return query_impl(m, queries, b, *p, group_idx, group_score, entry_idx, entry_score, entry_weight, lse,
+                    static_cast<cudaStream_t>(cuda_stream), &er);
+}
+
 htam_status htam_query_host(htam_memory *m, const void *queries, int32_t b, const htam_query_params *p,
                             int32_t *group_idx, float *group_score, int32_t *entry_idx, float *entry_score,
                             float *entry_weight, float *lse, void *cuda_stream) {

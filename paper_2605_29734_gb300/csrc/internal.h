@@ -99,10 +99,19 @@ htam_status build_impl(const void *entries, const int32_t *group_ids, int64_t n,
                        htam_memory **out);
 htam_status append_impl(htam_memory *m, const void *entries, const int32_t *group_ids,
                         int64_t count, cudaStream_t st);
+// Stage 1 from a transition-edge table instead of the group keys
+// (htam_query_edges).
+struct EdgeRoute {
+  const float *Z;          // [G, G, F] device, from x to x feature
+  const int32_t *prefix;   // [B, P] host, ids in [-1, G)
+  int F, P;
+  float w[HTAM_MAX_EDGE_FEATURES];
+  float alpha[HTAM_MAX_PREFIX];
+};
 htam_status query_impl(htam_memory *m, const void *queries, int32_t b,
                        const htam_query_params &p, int32_t *group_idx, float *group_score,
                        int32_t *entry_idx, float *entry_score, float *entry_weight, float *lse,
-                       cudaStream_t st);
+                       cudaStream_t st, const EdgeRoute *er = nullptr);
 void free_impl(htam_memory *m);
 
 // Weights alpha_1..alpha_P of a prefix (Eq. 10), passed by value to the

@@ -208,6 +208,46 @@ __global__ void __launch_bounds__(kSelWarps * 32, 1) group_topk_kernel(const flo
 // two full waves of the GPU (16 warps per SM), else one.
 static int warps_per_query(int B, int sm_count) { return (int64_t)B * 8 <= 2LL * 16 * sm_count ? 8 : 1; }
 
+// Stage-1 scores from a transition-edge table (the router of Eq. 9 with the
+// linear utility of App. B.6 and the weights of Eq. 10): one thread per
+// (query, group), s1[b][g] = sum_i alpha_i sum_f w_f Z[p_i][g][f] over the
+// prefix ids p_i >= 0, in index order with fp32 FMAs.  The threads of a warp
+// read neighbouring groups of the same table row, so the loads coalesce.
+struct EdgeKernelArgs {
+  const float *Z;
+  const int32_t *prefix;
+  int F, P;
+  float w[HTAM_MAX_EDGE_FEATURES];
+  float alpha[HTAM_MAX_PREFIX];
+};
+
+__global__ void __launch_bounds__(256) edge_scores_kernel(EdgeKernelArgs a, int B, int G, float *__restrict__ s1) {
+  const int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  if (t >= (int64_t)B * G) return;
+  const int64_t b = t / G;
+  const int g = (int)(t % G);
+  float acc = 0.f;
+  for (int i = 0; i < a.P; ++i) {
+    const int from = a.prefix[b * a.P + i];
+    if (from < 0) continue;
+    const float *z = a.Z + ((int64_t)from * G + g) * a.F;
+    float phi = 0.f;
+    if ((a.F & 3) == 0) {
+      for (int f = 0; f < a.F; f += 4) {
+        const float4 v = *reinterpret_cast<const float4 *>(z + f);
+        phi = fmaf(a.w[f], v.x, phi);
+        phi = fmaf(a.w[f + 1], v.y, phi);
+        phi = fmaf(a.w[f + 2], v.z, phi);
+        phi = fmaf(a.w[f + 3], v.w, phi);
+      }
+    } else {
+      for (int f = 0; f < a.F; ++f) phi = fmaf(a.w[f], z[f], phi);
+    }
+    acc = fmaf(a.alpha[i], phi, acc);
+  }
+  s1[t] = acc;
+}
+
 // ---------------------------------------------------------------- bucketing
 
 __global__ void bucket_bits_kernel(const int32_t *__restrict__ gidx, int B, int kg, int W,
@@ -861,7 +901,8 @@ constexpr uint32_t kMaxPolls = 1u << 24;
 
 htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const htam_query_params &p,
                        int32_t *group_idx, float *group_score, int32_t *entry_idx,
-                       float *entry_score, float *entry_weight, float *lse, cudaStream_t st) {
+                       float *entry_score, float *entry_weight, float *lse, cudaStream_t st,
+                       const EdgeRoute *er) {
   if (B == 0) return HTAM_OK;
   m->n_queries += 1;
   PhaseMark mark(m, st);
@@ -889,11 +930,11 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   const size_t qg_bytes = tc_ok ? sizeof(__nv_bfloat16) * (size_t)rows * d : 0;
 
   // Coarse scores: one plane per K split of the tensor-core kernel.
-  const int planes = m->dtype == HTAM_BF16 ? coarse_tc_splits(B, d, G, m->sm_count) : 1;
+  const int planes = m->dtype == HTAM_BF16 && !er ? coarse_tc_splits(B, d, G, m->sm_count) : 1;
   const int wpq = warps_per_query(B, m->sm_count);  // warps per query in top-k and merge
   size_t need = Carver::round(sizeof(float) * (size_t)planes * B * G) + Carver::round(sizeof(uint32_t) * (size_t)G * W) +
                 5 * Carver::round(sizeof(int32_t) * (G + 1)) + Carver::round(sizeof(int64_t) * (G + 1)) +
-                2 * Carver::round(sizeof(int32_t)) +
+                2 * Carver::round(sizeof(int32_t)) + (er ? Carver::round(sizeof(int32_t) * (size_t)B * er->P) : 0) +
                 3 * Carver::round(sizeof(int32_t) * rows) + 2 * Carver::round(sizeof(int4) * max_units) +
                 Carver::round(sizeof(float2) * max_parts) + Carver::round(sizeof(float) * max_parts * ke) +
                 Carver::round(sizeof(int32_t) * max_parts * ke) + Carver::round(sizeof(unsigned) * B) +
@@ -911,6 +952,7 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   int32_t *n_units = cv.take<int32_t>(G + 1);  // [0] SIMT units, [1] tensor-core units
   int32_t *seg_tc = cv.take<int32_t>(1);        // pages per tensor-core unit, chosen on the device
   int32_t *tc_ctr = cv.take<int32_t>(1);        // tensor-core units taken from the shared counter
+  int32_t *edge_prefix = er ? cv.take<int32_t>((size_t)B * er->P) : nullptr;
   int32_t *bucket = cv.take<int32_t>(rows);
   int32_t *bucket_group = cv.take<int32_t>(rows);
   int32_t *pos = cv.take<int32_t>(rows);
@@ -925,7 +967,20 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   // 1. Coarse scores and the selected groups.
   {
     mark.begin(HTAM_PHASE_COARSE);
-    if (m->dtype == HTAM_BF16) {
+    if (er) {
+      // Transition-edge scores (the prefix ids were checked on the host).
+      HTAM_CK(cudaMemcpyAsync(edge_prefix, er->prefix, sizeof(int32_t) * (size_t)B * er->P,
+                              cudaMemcpyHostToDevice, st));
+      EdgeKernelArgs ea;
+      ea.Z = er->Z;
+      ea.prefix = edge_prefix;
+      ea.F = er->F;
+      ea.P = er->P;
+      for (int f = 0; f < HTAM_MAX_EDGE_FEATURES; ++f) ea.w[f] = er->w[f];
+      for (int i = 0; i < HTAM_MAX_PREFIX; ++i) ea.alpha[i] = er->alpha[i];
+      edge_scores_kernel<<<(unsigned)ceil_div((int64_t)B * G, 256), 256, 0, st>>>(ea, B, G, s1);
+      HTAM_CK_LAUNCH("edge_scores_kernel");
+    } else if (m->dtype == HTAM_BF16) {
       // Tensor cores against the split (hi + lo) bf16 group keys.
       s = launch_coarse_tc(queries, B, d, m->cent_hi, m->cent_lo, m->count, G, planes, s1, m->status, kMaxPolls,
                            st);

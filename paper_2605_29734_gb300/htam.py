@@ -19,10 +19,12 @@ HTAM_OK, HTAM_EINVAL, HTAM_ENOMEM, HTAM_ECAPACITY, HTAM_ECUDA, HTAM_ETIMEOUT, HT
 HTAM_F32, HTAM_BF16 = 0, 1
 HTAM_TUNE_TC_MIN_BUCKET, HTAM_TUNE_STREAM_ROWS = 0, 1
 HTAM_MAX_PREFIX = 64  # longest prefix htam_query_prefix takes
+HTAM_MAX_EDGE_FEATURES = 32  # most features per edge htam_query_edges takes
 
 # Every symbol include/htam.h declares, in declaration order.
 EXPORTS = (
     "htam_build_memory", "htam_append_transitions", "htam_query", "htam_query_host", "htam_query_prefix",
+    "htam_query_edges",
     "htam_select_groups_static", "htam_memory_info", "htam_memory_group_counts", "htam_memory_group_keys",
     "htam_device_status", "htam_set_tuning", "htam_get_tuning", "htam_set_phase_timing",
     "htam_read_phase_timing", "htam_free_memory", "htam_status_string", "htam_last_error",
@@ -57,6 +59,8 @@ def _load() -> ctypes.CDLL:
     lib.htam_query_host.argtypes = qargs
     lib.htam_query_prefix.argtypes = [P, P, i32, i32, ctypes.c_float, ctypes.POINTER(QueryParams),
                                       P, P, P, P, P, P, P]
+    lib.htam_query_edges.argtypes = [P, P, i32, P, P, i32, ctypes.c_float, P, i32, ctypes.POINTER(QueryParams),
+                                     P, P, P, P, P, P, P]
     lib.htam_memory_info.argtypes = [P, P, P, P, P]
     lib.htam_memory_group_counts.argtypes = [P, P]
     lib.htam_memory_group_keys.argtypes = [P, P, P]
@@ -198,6 +202,41 @@ class Memory:
                                       _dev_ptr(out["entry_idx"]), _dev_ptr(out["entry_score"]),
                                       _dev_ptr(out["entry_weight"]), _dev_ptr(out.get("lse")),
                                       _stream_ptr(stream)), "htam_query_prefix")
+        return out
+
+    def query_edges(self, edge_features: torch.Tensor, weights, prefix_groups, lam: float, queries: torch.Tensor,
+                    k_groups: int, k_entries: int, tau: float = 1.0, epsilon: float = 0.0, stream=None,
+                    out: dict | None = None) -> dict:
+        """Lookup routed by transition edges: edge_features [G, G, F] float32
+        on the device, weights [F] and prefix_groups [b, P] (int32, -1 = none)
+        on the host, queries [b, d] on the device for the entry level."""
+        if edge_features.dtype != torch.float32 or edge_features.dim() != 3:
+            raise ValueError("edge_features must be a [G, G, F] float32 tensor")
+        if queries.dtype != self.dtype or queries.dim() != 2 or queries.shape[1] != self.d:
+            raise ValueError("queries must be [b, d] of the memory dtype")
+        w = torch.as_tensor(weights, dtype=torch.float32).contiguous().cpu()
+        pre = torch.as_tensor(prefix_groups, dtype=torch.int32).contiguous().cpu()
+        b = queries.shape[0]
+        if pre.dim() != 2 or pre.shape[0] != b:
+            raise ValueError("prefix_groups must be [b, P]")
+        dev = queries.device
+        if out is None:
+            out = {
+                "group_idx": torch.empty(b, k_groups, dtype=torch.int32, device=dev),
+                "group_score": torch.empty(b, k_groups, dtype=torch.float32, device=dev),
+                "entry_idx": torch.empty(b, k_entries, dtype=torch.int32, device=dev),
+                "entry_score": torch.empty(b, k_entries, dtype=torch.float32, device=dev),
+                "entry_weight": torch.empty(b, k_entries, dtype=torch.float32, device=dev),
+                "lse": torch.empty(b, dtype=torch.float32, device=dev),
+            }
+        p = QueryParams(k_groups, k_entries, tau, epsilon)
+        _check(_lib.htam_query_edges(self.handle, _dev_ptr(edge_features), edge_features.shape[2],
+                                     ctypes.c_void_p(w.data_ptr()), ctypes.c_void_p(pre.data_ptr()), pre.shape[1],
+                                     float(lam), _dev_ptr(queries), b, ctypes.byref(p),
+                                     _dev_ptr(out["group_idx"]), _dev_ptr(out["group_score"]),
+                                     _dev_ptr(out["entry_idx"]), _dev_ptr(out["entry_score"]),
+                                     _dev_ptr(out["entry_weight"]), _dev_ptr(out.get("lse")),
+                                     _stream_ptr(stream)), "htam_query_edges")
         return out
 
     def query_host(self, queries: torch.Tensor, k_groups: int, k_entries: int, tau: float = 1.0,

@@ -26,10 +26,11 @@ def close(gpu, ref, dtype) -> bool:
     return abs(gpu - ref) <= rtol * abs(ref) + atol
 
 
-def check_ranked(what, gpu_ids, gpu_scores, ref_ids, ref_scores, k, exact_score, dtype):
+def check_ranked(what, gpu_ids, gpu_scores, ref_ids, ref_scores, k, exact_score, dtype, tol=None):
     """gpu_ids/gpu_scores: length k.  ref_ids/ref_scores: the oracle's ranking
     of length >= k+1 (padded with -1 / -inf).  exact_score(id) gives the
-    oracle's (float64) score of any id.  Returns a list of problems."""
+    oracle's (float64) score of any id.  tol(id), when given, replaces the
+    dtype's value tolerance with an absolute bound.  Returns a list of problems."""
     bad = []
     gpu_ids = [int(x) for x in gpu_ids[:k]]
     ref_ids = [int(x) for x in ref_ids]
@@ -64,7 +65,8 @@ def check_ranked(what, gpu_ids, gpu_scores, ref_ids, ref_scores, k, exact_score,
             break
         run_min = min(run_min, es[i])
     for i in range(v_gpu):
-        if not close(gpu_scores[i], es[i], dtype):
+        ok = abs(float(gpu_scores[i]) - es[i]) <= tol(gpu_ids[i]) if tol else close(gpu_scores[i], es[i], dtype)
+        if not ok:
             bad.append(f"{what}: score of id {gpu_ids[i]} gpu {float(gpu_scores[i]):.7g} oracle {es[i]:.7g}")
             break
     return bad
@@ -100,30 +102,68 @@ def compare_lookup(out, entries_np, gid_np, n_groups, queries_np, k_groups, k_en
         cent_score = lambda g, r=r: float(centroid[g] @ qf[r])
         problems += check_ranked(f"query {b} groups", gi[b], gs[b], ref_gi[r], ref_gs[r], k_groups,
                                  cent_score, dtype)
-        ref_map = {int(i): (float(s), float(w)) for i, s, w in
-                   zip(ref2["entry_idx"][r], ref2["entry_score"][r], ref2["entry_weight"][r]) if i >= 0}
+        problems += _check_entries(ei, es, ew, lse, b, r, ref2, entries_np, qf, k_entries, tau, eps, dtype)
+    return problems
 
-        def entry_score(e, r=r):
-            if e in ref_map:
-                return ref_map[e][0]
-            return float(_as_f64(entries_np[e:e + 1])[0] @ qf[r])
 
-        problems += check_ranked(f"query {b} entries", ei[b], es[b], ref2["entry_idx"][r],
-                                 ref2["entry_score"][r], k_entries, entry_score, dtype)
-        nb = int(ref2["n_cand"][r])
-        for i in range(k_entries):
-            e = int(ei[b][i])
-            if e < 0:
-                if ew[b][i] != 0:
-                    problems.append(f"query {b}: padded weight not 0")
-                continue
-            s_ref = entry_score(e)
-            w_ref = ref_map[e][1] if e in ref_map else eps / nb + (1 - eps) * np.exp(s_ref / tau - ref2["lse"][r])
-            if not close(ew[b][i], w_ref, dtype):
-                problems.append(f"query {b}: weight of id {e} gpu {ew[b][i]:.7g} oracle {w_ref:.7g}")
-                break
-        if not close(lse[b], ref2["lse"][r], dtype):
-            problems.append(f"query {b}: lse gpu {lse[b]:.7g} oracle {ref2['lse'][r]:.7g}")
+def _check_entries(ei, es, ew, lse, b, r, ref2, entries_np, qf, k_entries, tau, eps, dtype):
+    """Stage 2 of query b (row r of the oracle's stage-2 results)."""
+    problems = []
+    ref_map = {int(i): (float(s), float(w)) for i, s, w in
+               zip(ref2["entry_idx"][r], ref2["entry_score"][r], ref2["entry_weight"][r]) if i >= 0}
+
+    def entry_score(e, r=r):
+        if e in ref_map:
+            return ref_map[e][0]
+        return float(_as_f64(entries_np[e:e + 1])[0] @ qf[r])
+
+    problems += check_ranked(f"query {b} entries", ei[b], es[b], ref2["entry_idx"][r],
+                             ref2["entry_score"][r], k_entries, entry_score, dtype)
+    nb = int(ref2["n_cand"][r])
+    for i in range(k_entries):
+        e = int(ei[b][i])
+        if e < 0:
+            if ew[b][i] != 0:
+                problems.append(f"query {b}: padded weight not 0")
+            continue
+        s_ref = entry_score(e)
+        w_ref = ref_map[e][1] if e in ref_map else eps / nb + (1 - eps) * np.exp(s_ref / tau - ref2["lse"][r])
+        if not close(ew[b][i], w_ref, dtype):
+            problems.append(f"query {b}: weight of id {e} gpu {ew[b][i]:.7g} oracle {w_ref:.7g}")
+            break
+    if not close(lse[b], ref2["lse"][r], dtype):
+        problems.append(f"query {b}: lse gpu {lse[b]:.7g} oracle {ref2['lse'][r]:.7g}")
+    return problems
+
+
+def compare_edge_lookup(out, entries_np, gid_np, n_groups, Z, w, prefix, lam, queries_np, k_groups, k_entries,
+                        tau, eps, dtype, nthreads=None):
+    """The edge-routed lookup: stage 1 against the oracle's edge-table scores
+    (values within 1e-5 of the sum of the magnitudes of their terms, the fp32
+    rounding bound of the sum, plus 1e-6), stage 2 given the GPU's groups."""
+    import oracle
+
+    gi = out["group_idx"].cpu().numpy()
+    gs = out["group_score"].cpu().numpy()
+    ei = out["entry_idx"].cpu().numpy()
+    es = out["entry_score"].cpu().numpy()
+    ew = out["entry_weight"].cpu().numpy()
+    lse = out["lse"].cpu().numpy()
+    counts = np.bincount(np.asarray(gid_np, dtype=np.int64), minlength=n_groups)
+    scores = oracle.edge_scores(Z, w, prefix, lam)
+    mag = oracle.edge_scores(np.abs(Z), np.abs(np.asarray(w, dtype=np.float64)), prefix, lam)
+    ref_gi, ref_gs = oracle.select(scores, counts, min(k_groups + 1, n_groups))
+    if ref_gi.shape[1] == k_groups:
+        ref_gi = np.concatenate([ref_gi, -np.ones((len(ref_gi), 1), np.int32)], axis=1)
+        ref_gs = np.concatenate([ref_gs, np.full((len(ref_gs), 1), -np.inf)], axis=1)
+    ref2 = oracle.stage2(entries_np, gid_np, n_groups, queries_np, gi, k_entries + 16, tau, eps, nthreads)
+    qf = _as_f64(queries_np)
+    problems = []
+    for b in range(queries_np.shape[0]):
+        problems += check_ranked(f"query {b} groups", gi[b], gs[b], ref_gi[b], ref_gs[b], k_groups,
+                                 lambda g, b=b: float(scores[b, g]), dtype,
+                                 tol=lambda g, b=b: 1e-5 * float(mag[b, g]) + 1e-6)
+        problems += _check_entries(ei, es, ew, lse, b, b, ref2, entries_np, qf, k_entries, tau, eps, dtype)
     return problems
 
 

@@ -303,6 +303,56 @@ def test_prefix_arguments_checked(htam):
             mem.query_prefix(ok, lam, 2, 4)
 
 
+EDGE_CASES = [
+    # n, groups, d, dtype, batch, prefix length, lambda, features, k_groups, k_entries
+    (12000, 60, 256, torch.float32, 40, 4, 0.5, 12, 6, 16),
+    (20000, 100, 1024, torch.bfloat16, 300, 6, 0.5, 12, 8, 24),   # buckets large enough for the tensor cores
+    (5000, 30, 512, torch.bfloat16, 25, 3, 0.0, 5, 4, 8),          # features not a multiple of 4
+]
+
+
+@pytest.mark.parametrize("case", EDGE_CASES)
+def test_edge_routed_lookup_matches_oracle(htam, case):
+    """htam_query_edges against the oracle: stage 1 from the edge table (Eq. 9
+    with the App. B.6 utility and the Eq. 10 weights), stage 2 from the
+    queries on the groups it selected."""
+    from parity import compare_edge_lookup
+
+    n, g, d, dtype, b, P, lam, F, kg, ke = case
+    entries, gid, centres = _rand_memory(n, d, g, dtype, seed=n + F)
+    q = _rand_queries(b, d, dtype, seed=n + F, centres=centres)
+    rng = np.random.default_rng(n + F)
+    Z = rng.standard_normal((g, g, F)).astype(np.float32)
+    w = rng.standard_normal(F).astype(np.float32)
+    prefix = rng.integers(-1, g, (b, P)).astype(np.int32)
+    mem = htam.Memory(entries, gid, g)
+    out = mem.query_edges(torch.from_numpy(Z).to(DEV), w, prefix, lam, q, kg, ke, tau=0.7, epsilon=0.05)
+    torch.cuda.synchronize()
+    dt = "bf16" if dtype == torch.bfloat16 else "f32"
+    problems = compare_edge_lookup(out, to_numpy(entries), to_numpy(gid), g, Z, w.astype(np.float64), prefix, lam,
+                                   to_numpy(q), kg, ke, 0.7, 0.05, dt)
+    assert not problems, "\n".join(problems[:20])
+    assert mem.device_status() == htam.HTAM_OK
+
+
+def test_edge_arguments_checked(htam):
+    entries, gid, _ = _rand_memory(500, 64, 4, torch.float32, seed=6)
+    mem = htam.Memory(entries, gid, 4)
+    q = torch.zeros(2, 64, device=DEV)
+    Z = torch.zeros(4, 4, 12, device=DEV)
+    w = np.ones(12, np.float32)
+    good = np.array([[0, -1], [3, 2]], np.int32)
+    mem.query_edges(Z, w, good, 0.5, q, 2, 4)
+    for bad in (np.array([[0, 4], [1, 2]], np.int32), np.array([[0, -2], [1, 2]], np.int32)):
+        with pytest.raises(htam.HtamError):
+            mem.query_edges(Z, w, bad, 0.5, q, 2, 4)
+    with pytest.raises(htam.HtamError):
+        mem.query_edges(torch.zeros(4, 4, htam.HTAM_MAX_EDGE_FEATURES + 1, device=DEV),
+                        np.ones(htam.HTAM_MAX_EDGE_FEATURES + 1, np.float32), good, 0.5, q, 2, 4)
+    with pytest.raises(htam.HtamError):
+        mem.query_edges(Z, np.array([1.0] * 11 + [np.nan], np.float32), good, 0.5, q, 2, 4)
+
+
 def test_tuning_defaults_follow_row_length_and_round_trip(htam):
     """The tensor-core threshold defaults to 2 queries for rows up to 4 KiB
     and 16 for longer rows; values set are read back; bad keys and values are
