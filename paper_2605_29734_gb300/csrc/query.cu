@@ -221,6 +221,46 @@ struct EdgeKernelArgs {
   float alpha[HTAM_MAX_PREFIX];
 };
 
+// phi(from, to) = w . Z[from][to][:], in the same FMA order as below.
+__device__ __forceinline__ float edge_phi(const EdgeKernelArgs &a, const float *z) {
+  float phi = 0.f;
+  if ((a.F & 3) == 0) {
+    for (int f = 0; f < a.F; f += 4) {
+      const float4 v = *reinterpret_cast<const float4 *>(z + f);
+      phi = fmaf(a.w[f], v.x, phi);
+      phi = fmaf(a.w[f + 1], v.y, phi);
+      phi = fmaf(a.w[f + 2], v.z, phi);
+      phi = fmaf(a.w[f + 3], v.w, phi);
+    }
+  } else {
+    for (int f = 0; f < a.F; ++f) phi = fmaf(a.w[f], z[f], phi);
+  }
+  return phi;
+}
+
+// When a batch references more prefix rows than the table has, the utility
+// of every edge is formed once (U[from][to] = phi) and the scores gather
+// from U: the same products and sums in the same order, so the same results.
+__global__ void __launch_bounds__(256) edge_phi_kernel(EdgeKernelArgs a, int G, float *__restrict__ U) {
+  const int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  if (t >= (int64_t)G * G) return;
+  U[t] = edge_phi(a, a.Z + t * a.F);
+}
+
+__global__ void __launch_bounds__(256) edge_gather_kernel(EdgeKernelArgs a, const float *__restrict__ U, int B, int G,
+                                                          float *__restrict__ s1) {
+  const int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  if (t >= (int64_t)B * G) return;
+  const int64_t b = t / G;
+  const int g = (int)(t % G);
+  float acc = 0.f;
+  for (int i = 0; i < a.P; ++i) {
+    const int from = a.prefix[b * a.P + i];
+    if (from >= 0) acc = fmaf(a.alpha[i], U[(int64_t)from * G + g], acc);
+  }
+  s1[t] = acc;
+}
+
 __global__ void __launch_bounds__(256) edge_scores_kernel(EdgeKernelArgs a, int B, int G, float *__restrict__ s1) {
   const int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   if (t >= (int64_t)B * G) return;
@@ -230,20 +270,7 @@ __global__ void __launch_bounds__(256) edge_scores_kernel(EdgeKernelArgs a, int 
   for (int i = 0; i < a.P; ++i) {
     const int from = a.prefix[b * a.P + i];
     if (from < 0) continue;
-    const float *z = a.Z + ((int64_t)from * G + g) * a.F;
-    float phi = 0.f;
-    if ((a.F & 3) == 0) {
-      for (int f = 0; f < a.F; f += 4) {
-        const float4 v = *reinterpret_cast<const float4 *>(z + f);
-        phi = fmaf(a.w[f], v.x, phi);
-        phi = fmaf(a.w[f + 1], v.y, phi);
-        phi = fmaf(a.w[f + 2], v.z, phi);
-        phi = fmaf(a.w[f + 3], v.w, phi);
-      }
-    } else {
-      for (int f = 0; f < a.F; ++f) phi = fmaf(a.w[f], z[f], phi);
-    }
-    acc = fmaf(a.alpha[i], phi, acc);
+    acc = fmaf(a.alpha[i], edge_phi(a, a.Z + ((int64_t)from * G + g) * a.F), acc);
   }
   s1[t] = acc;
 }
@@ -931,10 +958,14 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
 
   // Coarse scores: one plane per K split of the tensor-core kernel.
   const int planes = m->dtype == HTAM_BF16 && !er ? coarse_tc_splits(B, d, G, m->sm_count) : 1;
+  // Edge routing: form the whole utility table once when the batch references
+  // more prefix rows than the table has.
+  const bool edge_table = er && (int64_t)B * er->P > G;
   const int wpq = warps_per_query(B, m->sm_count);  // warps per query in top-k and merge
   size_t need = Carver::round(sizeof(float) * (size_t)planes * B * G) + Carver::round(sizeof(uint32_t) * (size_t)G * W) +
                 5 * Carver::round(sizeof(int32_t) * (G + 1)) + Carver::round(sizeof(int64_t) * (G + 1)) +
                 2 * Carver::round(sizeof(int32_t)) + (er ? Carver::round(sizeof(int32_t) * (size_t)B * er->P) : 0) +
+                (edge_table ? Carver::round(sizeof(float) * (size_t)G * G) : 0) +
                 3 * Carver::round(sizeof(int32_t) * rows) + 2 * Carver::round(sizeof(int4) * max_units) +
                 Carver::round(sizeof(float2) * max_parts) + Carver::round(sizeof(float) * max_parts * ke) +
                 Carver::round(sizeof(int32_t) * max_parts * ke) + Carver::round(sizeof(unsigned) * B) +
@@ -953,6 +984,7 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   int32_t *seg_tc = cv.take<int32_t>(1);        // pages per tensor-core unit, chosen on the device
   int32_t *tc_ctr = cv.take<int32_t>(1);        // tensor-core units taken from the shared counter
   int32_t *edge_prefix = er ? cv.take<int32_t>((size_t)B * er->P) : nullptr;
+  float *edge_u = edge_table ? cv.take<float>((size_t)G * G) : nullptr;
   int32_t *bucket = cv.take<int32_t>(rows);
   int32_t *bucket_group = cv.take<int32_t>(rows);
   int32_t *pos = cv.take<int32_t>(rows);
@@ -978,8 +1010,16 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
       ea.P = er->P;
       for (int f = 0; f < HTAM_MAX_EDGE_FEATURES; ++f) ea.w[f] = er->w[f];
       for (int i = 0; i < HTAM_MAX_PREFIX; ++i) ea.alpha[i] = er->alpha[i];
-      edge_scores_kernel<<<(unsigned)ceil_div((int64_t)B * G, 256), 256, 0, st>>>(ea, B, G, s1);
-      HTAM_CK_LAUNCH("edge_scores_kernel");
+      if (edge_table) {
+        edge_phi_kernel<<<(unsigned)ceil_div((int64_t)G * G, 256), 256, 0, st>>>(ea, G, edge_u);
+        HTAM_CK_LAUNCH("edge_phi_kernel");
+        edge_gather_kernel<<<(unsigned)ceil_div((int64_t)B * G, 256), 256, 0, st>>>(ea, edge_u, B, G, s1);
+        HTAM_CK_LAUNCH("edge_gather_kernel");
+        mark.launched();
+      } else {
+        edge_scores_kernel<<<(unsigned)ceil_div((int64_t)B * G, 256), 256, 0, st>>>(ea, B, G, s1);
+        HTAM_CK_LAUNCH("edge_scores_kernel");
+      }
     } else if (m->dtype == HTAM_BF16) {
       // Tensor cores against the split (hi + lo) bf16 group keys.
       s = launch_coarse_tc(queries, B, d, m->cent_hi, m->cent_lo, m->count, G, planes, s1, m->status, kMaxPolls,

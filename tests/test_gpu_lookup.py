@@ -305,9 +305,12 @@ def test_prefix_arguments_checked(htam):
 
 EDGE_CASES = [
     # n, groups, d, dtype, batch, prefix length, lambda, features, k_groups, k_entries
+    # (batch x prefix > groups forms the whole utility table first)
     (12000, 60, 256, torch.float32, 40, 4, 0.5, 12, 6, 16),
     (20000, 100, 1024, torch.bfloat16, 300, 6, 0.5, 12, 8, 24),   # buckets large enough for the tensor cores
     (5000, 30, 512, torch.bfloat16, 25, 3, 0.0, 5, 4, 8),          # features not a multiple of 4
+    (12000, 200, 256, torch.float32, 20, 3, 0.5, 12, 6, 16),       # fewer prefix rows than groups: direct scores
+    (12000, 200, 256, torch.float32, 20, 3, 0.5, 7, 6, 16),        # the same with 7 features
 ]
 
 
