@@ -286,16 +286,42 @@ __global__ void bucket_bits_kernel(const int32_t *__restrict__ gidx, int B, int 
   if (g >= 0) atomicOr(&bits[(int64_t)g * W + (b >> 5)], 1u << (b & 31));
 }
 
+// One warp per group: the bucket size c_g and, per bitmap word, how many of
+// the group's queries come before it (wpre[g][w]).
 __global__ void bucket_count_kernel(const uint32_t *__restrict__ bits, int G, int W,
-                                    int32_t *__restrict__ cnt) {
+                                    int32_t *__restrict__ cnt, int32_t *__restrict__ wpre) {
   int g = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   int lane = threadIdx.x & 31;
   if (g >= G) return;
-  int c = 0;
-  for (int w = lane; w < W; w += 32) c += __popc(bits[(int64_t)g * W + w]);
+  int running = 0;
+  for (int w0 = 0; w0 < W; w0 += 32) {
+    const int w = w0 + lane;
+    const int pc = w < W ? __popc(bits[(int64_t)g * W + w]) : 0;
+    int incl = pc;
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(kFullMask, c, o);
-  if (lane == 0) cnt[g] = c;
+    for (int o = 1; o < 32; o <<= 1) {
+      const int t = __shfl_up_sync(kFullMask, incl, o);
+      if (lane >= o) incl += t;
+    }
+    if (w < W) wpre[(int64_t)g * W + w] = running + incl - pc;
+    running += __shfl_sync(kFullMask, incl, 31);
+  }
+  if (lane == 0) cnt[g] = running;
+}
+
+// pos[b][j] = rank of query b in the bucket of its j-th selected group: the
+// group's queries before b's bitmap word plus those before b within it.
+__global__ void bucket_pos_kernel(const uint32_t *__restrict__ bits, const int32_t *__restrict__ wpre, int W,
+                                  const int32_t *__restrict__ gidx, int64_t rows, int kg,
+                                  int32_t *__restrict__ pos) {
+  const int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  if (t >= rows) return;
+  const int g = gidx[t];
+  if (g < 0) return;
+  const int b = (int)(t / kg);
+  const int w = b >> 5;
+  const uint32_t below = bits[(int64_t)g * W + w] & ((1u << (b & 31)) - 1u);
+  pos[t] = wpre[(int64_t)g * W + w] + __popc(below);
 }
 
 // Which fine kernel scores a group's bucket: buckets of at least tc_min
@@ -402,20 +428,18 @@ __global__ void __launch_bounds__(1024) bucket_scan_kernel(
   }
 }
 
-// One warp per group: bucket[g] lists its queries in increasing order;
-// pos[b][j] = rank of query b in the bucket of its j-th selected group.
+// One warp per group: bucket[g] lists its queries in increasing order.
 // Also writes the group's work units (group, chunk, segment) to the list of
 // the kernel that will score them, and the group of every bucket row.
 __global__ void bucket_fill_kernel(const uint32_t *__restrict__ bits, int G, int W,
                                    const int32_t *__restrict__ bucket_off,
-                                   const int32_t *__restrict__ gidx, int kg,
                                    const int32_t *__restrict__ cnt,
                                    const int32_t *__restrict__ page_off, Route rt,
                                    const int32_t *__restrict__ seg_tc_dev,
                                    const int32_t *__restrict__ unit_off,
                                    const int32_t *__restrict__ unit_off_tc,
                                    int32_t *__restrict__ bucket, int32_t *__restrict__ bucket_group,
-                                   int32_t *__restrict__ pos, int4 *__restrict__ units,
+                                   int4 *__restrict__ units,
                                    int4 *__restrict__ units_tc) {
   int g = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   int lane = threadIdx.x & 31;
@@ -438,9 +462,6 @@ __global__ void bucket_fill_kernel(const uint32_t *__restrict__ bits, int G, int
       int b = (w0 + lane) * 32 + bit;
       bucket[base + r] = b;
       bucket_group[base + r] = g;
-      for (int j = 0; j < kg; ++j) {
-        if (gidx[(int64_t)b * kg + j] == g) pos[(int64_t)b * kg + j] = r;
-      }
       ++r;
     }
     running += __shfl_sync(kFullMask, incl, 31);
@@ -767,46 +788,50 @@ __global__ void __launch_bounds__(kMergeWarps * 32, 1) merge_kernel(MergeArgs a)
     }
     return r;
   };
-  const GroupRecs gr0 = load_group(lane), gr1 = load_group(lane + 32);
   constexpr int kBatch = 4;  // records fetched before any is combined
   const int n_t = live ? (a.kg - sw + WPQ - 1) / WPQ : 0;
-  for (int t = 0; t < n_t; ++t) {
-    const bool lo = t < 32;
-    const int g = __shfl_sync(kFullMask, lo ? gr0.g : gr1.g, t & 31);
-    if (g < 0) continue;  // uniform
-    const int p = __shfl_sync(kFullMask, lo ? gr0.p : gr1.p, t & 31);
-    const int cg = __shfl_sync(kFullMask, lo ? gr0.cg : gr1.cg, t & 31);
-    const int nseg = __shfl_sync(kFullMask, lo ? gr0.nseg : gr1.nseg, t & 31);
-    const long long base = __shfl_sync(kFullMask, lo ? gr0.base : gr1.base, t & 31);
-    for (int s0 = 0; s0 < nseg; s0 += kBatch) {
-      float2 ml[kBatch];
-      float cs[kBatch][2];
-      int ci[kBatch][2];
+  for (int t0 = 0; t0 < n_t; t0 += 64) {
+    const GroupRecs gr0 = load_group(t0 + lane), gr1 = load_group(t0 + lane + 32);
+    const int t_end = min(n_t, t0 + 64);
+    for (int t = t0; t < t_end; ++t) {
+      const bool lo = t - t0 < 32;
+      const int src = (t - t0) & 31;
+      const int g = __shfl_sync(kFullMask, lo ? gr0.g : gr1.g, src);
+      if (g < 0) continue;  // uniform
+      const int p = __shfl_sync(kFullMask, lo ? gr0.p : gr1.p, src);
+      const int cg = __shfl_sync(kFullMask, lo ? gr0.cg : gr1.cg, src);
+      const int nseg = __shfl_sync(kFullMask, lo ? gr0.nseg : gr1.nseg, src);
+      const long long base = __shfl_sync(kFullMask, lo ? gr0.base : gr1.base, src);
+      for (int s0 = 0; s0 < nseg; s0 += kBatch) {
+        float2 ml[kBatch];
+        float cs[kBatch][2];
+        int ci[kBatch][2];
 #pragma unroll
-      for (int i = 0; i < kBatch; ++i) {
-        const bool v = s0 + i < nseg;
-        const int64_t pidx = base + (int64_t)(s0 + i) * cg + p;
-        ml[i] = v ? a.part_ml[pidx] : make_float2(-INFINITY, 0.f);
+        for (int i = 0; i < kBatch; ++i) {
+          const bool v = s0 + i < nseg;
+          const int64_t pidx = base + (int64_t)(s0 + i) * cg + p;
+          ml[i] = v ? a.part_ml[pidx] : make_float2(-INFINITY, 0.f);
 #pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          const int tt = h * 32 + lane;
-          const bool in = v && tt < ke;
-          cs[i][h] = in ? a.part_s[pidx * ke + tt] : -INFINITY;
-          ci[i][h] = in ? a.part_id[pidx * ke + tt] : INT_MAX;
+          for (int h = 0; h < 2; ++h) {
+            const int tt = h * 32 + lane;
+            const bool in = v && tt < ke;
+            cs[i][h] = in ? a.part_s[pidx * ke + tt] : -INFINITY;
+            ci[i][h] = in ? a.part_id[pidx * ke + tt] : INT_MAX;
+          }
         }
-      }
 #pragma unroll
-      for (int i = 0; i < kBatch; ++i) {
-        if (ml[i].x != -INFINITY) {
-          const float Mn = fmaxf(M, ml[i].x);
-          L = L * expf(M - Mn) + ml[i].y * expf(ml[i].x - Mn);
-          M = Mn;
-        }
-        if (ke <= 32) {
-          take32(cs[i][0], ci[i][0]);
-        } else {
+        for (int i = 0; i < kBatch; ++i) {
+          if (ml[i].x != -INFINITY) {
+            const float Mn = fmaxf(M, ml[i].x);
+            L = L * expf(M - Mn) + ml[i].y * expf(ml[i].x - Mn);
+            M = Mn;
+          }
+          if (ke <= 32) {
+            take32(cs[i][0], ci[i][0]);
+          } else {
 #pragma unroll
-          for (int h = 0; h < 2; ++h) offer(cs[i][h], ci[i][h], ke - h * 32);
+            for (int h = 0; h < 2; ++h) offer(cs[i][h], ci[i][h], ke - h * 32);
+          }
         }
       }
     }
@@ -962,7 +987,7 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   // more prefix rows than the table has.
   const bool edge_table = er && (int64_t)B * er->P > G;
   const int wpq = warps_per_query(B, m->sm_count);  // warps per query in top-k and merge
-  size_t need = Carver::round(sizeof(float) * (size_t)planes * B * G) + Carver::round(sizeof(uint32_t) * (size_t)G * W) +
+  size_t need = Carver::round(sizeof(float) * (size_t)planes * B * G) + 2 * Carver::round(sizeof(uint32_t) * (size_t)G * W) +
                 5 * Carver::round(sizeof(int32_t) * (G + 1)) + Carver::round(sizeof(int64_t) * (G + 1)) +
                 2 * Carver::round(sizeof(int32_t)) + (er ? Carver::round(sizeof(int32_t) * (size_t)B * er->P) : 0) +
                 (edge_table ? Carver::round(sizeof(float) * (size_t)G * G) : 0) +
@@ -975,6 +1000,7 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   Carver cv(m->scratch);
   float *s1 = cv.take<float>((size_t)planes * B * G);
   uint32_t *bits = cv.take<uint32_t>((size_t)G * W);
+  int32_t *wpre = cv.take<int32_t>((size_t)G * W);
   int32_t *cnt = cv.take<int32_t>(G + 1);
   int32_t *bucket_off = cv.take<int32_t>(G + 1);
   int32_t *unit_off = cv.take<int32_t>(G + 1);
@@ -1052,16 +1078,18 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   HTAM_CK(cudaMemsetAsync(bits, 0, sizeof(uint32_t) * (size_t)G * W, st));
   bucket_bits_kernel<<<(unsigned)ceil_div(rows, 256), 256, 0, st>>>(group_idx, B, kg, W, bits);
   HTAM_CK_LAUNCH("bucket_bits_kernel");
-  bucket_count_kernel<<<(unsigned)ceil_div((int64_t)G * 32, 256), 256, 0, st>>>(bits, G, W, cnt);
+  bucket_count_kernel<<<(unsigned)ceil_div((int64_t)G * 32, 256), 256, 0, st>>>(bits, G, W, cnt, wpre);
   HTAM_CK_LAUNCH("bucket_count_kernel");
+  bucket_pos_kernel<<<(unsigned)ceil_div(rows, 256), 256, 0, st>>>(bits, wpre, W, group_idx, rows, kg, pos);
+  HTAM_CK_LAUNCH("bucket_pos_kernel");
   bucket_scan_kernel<<<1, 1024, 0, st>>>(cnt, m->page_off, G, rt, m->sm_count, bucket_off, unit_off,
                                          unit_off_tc, part_off, n_units, seg_tc);
   HTAM_CK_LAUNCH("bucket_scan_kernel");
   bucket_fill_kernel<<<(unsigned)ceil_div((int64_t)G * 32, 256), 256, 0, st>>>(
-      bits, G, W, bucket_off, group_idx, kg, cnt, m->page_off, rt, seg_tc, unit_off, unit_off_tc, bucket,
-      bucket_group, pos, units, units_tc);
+      bits, G, W, bucket_off, cnt, m->page_off, rt, seg_tc, unit_off, unit_off_tc, bucket, bucket_group, units,
+      units_tc);
   HTAM_CK_LAUNCH("bucket_fill_kernel");
-  mark.launched(4);
+  mark.launched(5);
   CUtensorMap q_map;
   if (tc_ok) {
     // Queries of tensor-core buckets in bucket order (the MMA's A operand),
