@@ -64,6 +64,8 @@ def parse_args():
                     help="route stage 1 by a transition-edge table (htam_query_edges) with prefixes of this "
                          "many earlier groups; 0 = group keys")
     ap.add_argument("--edge-features", type=int, default=12, help="features per edge (12 in App. B.6)")
+    ap.add_argument("--flat", action="store_true",
+                    help="flat scan (htam_query_flat): every entry a candidate, no group stage")
     ap.add_argument("--tc-min-bucket", type=int, default=None,
                     help="smallest bucket scored on the tensor cores (library default 16)")
     return ap.parse_args()
@@ -211,7 +213,7 @@ def cuda_core_kernel(w, stream_rows) -> str:
     return "fine_simt"
 
 
-def step_work(w, counts: np.ndarray, group_idx: np.ndarray, tc_min: int):
+def step_work(w, counts: np.ndarray, group_idx: np.ndarray, tc_min: int, flat: bool = False):
     """Algorithmic bytes / flops of one query batch, from the groups it selected:
     each selected group's entries read once, the queries read once, and
     2*D flops per (query, candidate entry); split between the CUDA-core kernel
@@ -231,9 +233,11 @@ def step_work(w, counts: np.ndarray, group_idx: np.ndarray, tc_min: int):
         queries_read = float(bucket[mask].sum())          # bucket rows staged per kernel
         work[name] = {"bytes": entries_read * D * s + min(B, queries_read) * D * s,
                       "flops": 2.0 * D * float((bucket[mask] * counts[mask]).sum())}
-    coarse_flops = 2.0 * D * B * G
-    out_bytes = B * (w.k_groups * 8 + w.k_entries * 12 + 4)
-    step_bytes = float(counts[touched].sum()) * D * s + B * D * s + G * D * 4 + out_bytes
+    # The flat scan has no group stage: no group keys read, no coarse scores,
+    # no group outputs.
+    coarse_flops = 0.0 if flat else 2.0 * D * B * G
+    out_bytes = B * ((0 if flat else w.k_groups * 8) + w.k_entries * 12 + 4)
+    step_bytes = float(counts[touched].sum()) * D * s + B * D * s + (0 if flat else G * D * 4) + out_bytes
     return {"kernels": work, "step_bytes": step_bytes,
             "step_flops": 2.0 * D * float(n_b.sum()) + coarse_flops, "mean_candidates": float(n_b.mean())}
 
@@ -245,23 +249,29 @@ def make_workload(w, seed, device, rank):
     return entries, gid, centres
 
 
-def oracle_rate(w, entries_np, gid_np, queries_np, target_s, cent=None, counts=None):
+def oracle_rate(w, entries_np, gid_np, queries_np, target_s, cent=None, counts=None, flat=False):
     """Times the oracle (as it stands) on a bounded sample of the queries."""
     import oracle
 
     threads = oracle.default_threads()
-    if cent is None:
+    if cent is None and not flat:
         cent, counts = oracle.centroids(entries_np, gid_np, w.g, threads)
+
+    def call(q):
+        if flat:
+            oracle.flat(entries_np, q, w.k_entries, nthreads=threads)
+        else:
+            oracle.query(entries_np, gid_np, w.g, q, w.k_groups, w.k_entries, centroid=cent, counts=counts,
+                         nthreads=threads)
+
     probe = min(threads, queries_np.shape[0])
     t0 = time.perf_counter()
-    oracle.query(entries_np, gid_np, w.g, queries_np[:probe], w.k_groups, w.k_entries, centroid=cent,
-                 counts=counts, nthreads=threads)
+    call(queries_np[:probe])
     t_probe = max(time.perf_counter() - t0, 1e-6)
     n = int(min(queries_np.shape[0], max(probe, probe * target_s / t_probe)))
     n = max(probe, (n // threads) * threads) if n >= threads else n
     t0 = time.perf_counter()
-    oracle.query(entries_np, gid_np, w.g, queries_np[:n], w.k_groups, w.k_entries, centroid=cent,
-                 counts=counts, nthreads=threads)
+    call(queries_np[:n])
     dt = time.perf_counter() - t0
     return n / dt, n, dt, threads, cent, counts
 
@@ -280,15 +290,21 @@ def run_reference(args, world, rank):
     import oracle
 
     threads = oracle.default_threads()
-    cent, counts = oracle.centroids(entries_np, gid_np, w.g, threads)
+    cent, counts = (None, None) if args.flat else oracle.centroids(entries_np, gid_np, w.g, threads)
     per_step_target = max(0.5, 120.0 / max(1, args.steps + args.warmup))
-    _, n_sample, _, _, _, _ = oracle_rate(w, entries_np, gid_np, q_np, per_step_target, cent, counts)
+    if args.flat:  # one query per host thread per step (each scans every entry)
+        n_sample = min(threads, q_np.shape[0])
+    else:
+        _, n_sample, _, _, _, _ = oracle_rate(w, entries_np, gid_np, q_np, per_step_target, cent, counts)
     times = []
     for i in range(args.warmup + args.steps):
         off = (i * n_sample) % max(1, q_np.shape[0] - n_sample + 1)
         t0 = time.perf_counter()
-        oracle.query(entries_np, gid_np, w.g, q_np[off:off + n_sample], w.k_groups, w.k_entries, centroid=cent,
-                     counts=counts, nthreads=threads)
+        if args.flat:
+            oracle.flat(entries_np, q_np[off:off + n_sample], w.k_entries, nthreads=threads)
+        else:
+            oracle.query(entries_np, gid_np, w.g, q_np[off:off + n_sample], w.k_groups, w.k_entries,
+                         centroid=cent, counts=counts, nthreads=threads)
         if i >= args.warmup:
             times.append(time.perf_counter() - t0)
     total = sum(times)
@@ -299,10 +315,10 @@ def run_reference(args, world, rank):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic",
         "config": {"workload": w.name, "queries_per_step": n_sample, "d": w.d, "groups": w.g, "entries": w.n,
-                   "k_groups": w.k_groups, "k_entries": w.k_entries},
+                   "k_groups": w.k_groups, "k_entries": w.k_entries, **({"flat": True} if args.flat else {})},
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle",
-                         "sample": f"{n_sample} queries of {w.name} per step, float64 brute force, "
-                                   f"group keys precomputed"},
+                         "sample": f"{n_sample} queries of {w.name} per step, float64 brute force"
+                                   + (", flat retrieval" if args.flat else ", group keys precomputed")},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
@@ -353,6 +369,8 @@ def run_htam(args, world, rank, local):
     batch_of = {id(q): i for i, q in enumerate(batches)}
 
     def run_query(q, out=None):
+        if args.flat:
+            return mem.query_flat(q, w.k_entries, out=out)
         if E > 0:
             return mem.query_edges(edge_z, edge_w, edge_prefix[batch_of.get(id(q), 0)], args.prefix_lambda, q,
                                    w.k_groups, w.k_entries, out=out)
@@ -373,7 +391,11 @@ def run_htam(args, world, rank, local):
     work = []
     for q in batches:
         o = run_query(q)
-        wk = step_work(w, counts, o["group_idx"].cpu().numpy(), tc_min)
+        if args.flat:  # every query selects every non-empty group
+            gi = np.tile(np.flatnonzero(counts > 0).astype(np.int32), (q.shape[0], 1))
+        else:
+            gi = o["group_idx"].cpu().numpy()
+        wk = step_work(w, counts, gi, tc_min, flat=args.flat)
         if P > 0:  # the prefix is read once, in place of the query
             wk["step_bytes"] += (P - 1) * w.b * w.d * (2 if w.dtype == "bf16" else 4)
         if E > 0:  # stage 1 reads the referenced edge-table rows instead of the group keys
@@ -457,7 +479,7 @@ def run_htam(args, world, rank, local):
     host_q = [b.cpu().pin_memory() for b in batches]
     e2e_steps = max(3, min(args.steps, 50))
     s_elem = 2 if w.dtype == "bf16" else 4
-    if P > 0 or E > 0:
+    if P > 0 or E > 0 or args.flat:
         # No host-buffer entry point for these lookups: pinned copies on the
         # stream around the call, outputs read back every step.
         dev_q = torch.empty_like(batches[0])
@@ -471,8 +493,8 @@ def run_htam(args, world, rank, local):
             for k in host_out:
                 host_out[k].copy_(o[k], non_blocking=True)
             torch.cuda.current_stream().synchronize()
-        path = ("pinned host queries copied in, " + ("htam_query_edges" if E > 0 else "htam_query_prefix") +
-                ", outputs copied out (torch copies on the stream)")
+        entry = "htam_query_flat" if args.flat else "htam_query_edges" if E > 0 else "htam_query_prefix"
+        path = f"pinned host queries copied in, {entry}, outputs copied out (torch copies on the stream)"
     else:
         host_out = mem.query_host(host_q[0], w.k_groups, w.k_entries)
 
@@ -491,7 +513,8 @@ def run_htam(args, world, rank, local):
     e2e_s = max_over_ranks(time.perf_counter() - t0, world)
     e2e = {"value": w.b * e2e_steps * world / e2e_s, "unit": UNIT,
            "h2d_bytes_per_step": w.b * max(P, 1) * w.d * s_elem,
-           "d2h_bytes_per_step": w.b * (w.k_groups * 8 + w.k_entries * 12 + 4), "steps": e2e_steps, "path": path}
+           "d2h_bytes_per_step": sum(v.numel() * v.element_size() for v in out.values()), "steps": e2e_steps,
+           "path": path}
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -503,7 +526,15 @@ def run_htam(args, world, rank, local):
         if P > 0:  # the oracle's prefix reduction (cheap next to the lookup) happens before the timing
             q_np = oracle.round_query(oracle.prefix_reduce(q_np, args.prefix_lambda), w.dtype)
             note = f", prefixes of {P} reduced before timing"
-        if E > 0:  # the oracle's edge-routed lookup on a bounded sample of batch 0
+        if args.flat:  # the oracle's flat retrieval on one query per host thread
+            threads = oracle.default_threads()
+            n = min(w.b, threads)
+            t0 = time.perf_counter()
+            oracle.flat(entries_np, q_np[:n], w.k_entries, nthreads=threads)
+            dt = time.perf_counter() - t0
+            rate = n / dt
+            note = ", flat retrieval over all entries"
+        elif E > 0:  # the oracle's edge-routed lookup on a bounded sample of batch 0
             threads = oracle.default_threads()
             z_np, pre_np = edge_z.cpu().numpy(), edge_prefix[0]
             t0 = time.perf_counter()
@@ -520,8 +551,8 @@ def run_htam(args, world, rank, local):
         else:
             rate, n, dt, threads, _, _ = oracle_rate(w, entries_np, gid_np, q_np, args.cpu_seconds)
         cpu = {"value": rate, "unit": UNIT, "cores": threads, "kind": "oracle",
-               "sample": f"{n} queries of {w.name} ({dt:.1f} s), float64 brute force over the same memory, "
-                         f"group keys precomputed{note}"}
+               "sample": f"{n} queries of {w.name} ({dt:.1f} s), float64 brute force over the same memory"
+                         + ("" if args.flat else ", group keys precomputed") + note}
 
     if rank == 0:
         line = {
@@ -531,6 +562,7 @@ def run_htam(args, world, rank, local):
             "config": {"workload": w.name, "queries_per_step": w.b, "d": w.d, "groups": w.g, "entries": w.n,
                        "k_groups": w.k_groups, "k_entries": w.k_entries, "query_batches": len(batches),
                        "mean_candidates_per_query": float(np.mean([x["mean_candidates"] for x in work])),
+                       **({"flat": True} if args.flat else {}),
                        "l2": ("flushed between steps (2x L2 buffer write, outside the step events)" if flush_l2 else
                               f"inputs larger than L2 ({work[0]['step_bytes'] / 1e9:.2f} GB touched per step)"),
                        "parallelism": f"replicas{world}" if world > 1 else "single GPU",

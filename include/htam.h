@@ -180,6 +180,25 @@ htam_status htam_query_edges(htam_memory *m, const float *edge_features, int32_t
                              int32_t *entry_idx, float *entry_score, float *entry_weight,
                              float *lse, void *cuda_stream);
 
+/* Flat scan: stage 2 of the lookup with every entry a candidate, no group
+ * stage.  This is the flat memory retrieval the paper compares against
+ * (App. C.4, and the "w/o hierarchy" ablation of App. C.8); its result equals
+ * htam_query with k_groups = the number of non-empty groups.  The fine scores
+ * s = q . k_e over all n entries, the softmax of Eq. 11 over all of them
+ * (|C| = n in the epsilon term), and the k_entries best by Eq. 13 (ties to the
+ * lower id).
+ *  queries     : [b, d] of the memory's dtype, device, 16-byte aligned
+ *  k_entries   : 1 <= k_entries <= 64
+ *  tau, epsilon: as htam_query_params
+ *  entry_idx / entry_score / entry_weight / lse: as htam_query ([b, k_entries],
+ *                lse [b] or NULL), -1 / -inf / 0 padding when n < k_entries
+ * b * (non-empty groups) <= 2^28.  Outputs, asynchrony and errors as
+ * htam_query. */
+htam_status htam_query_flat(htam_memory *m, const void *queries, int32_t b,
+                            int32_t k_entries, float tau, float epsilon,
+                            int32_t *entry_idx, float *entry_score,
+                            float *entry_weight, float *lse, void *cuda_stream);
+
 /* Bytes of the fixed device scratch used by htam_select_groups_static. */
 #define HTAM_STATIC_SCRATCH_BYTES (16u << 20)
 

@@ -194,6 +194,18 @@ def query(entries: np.ndarray, gid: np.ndarray, n_groups: int, queries: np.ndarr
     return out
 
 
+def flat(entries: np.ndarray, queries: np.ndarray, k_entries: int, tau: float = 1.0, eps: float = 0.0,
+         nthreads: int | None = None):
+    """Flat memory retrieval (App. C.4; the "w/o hierarchy" ablation of
+    App. C.8): every entry is a candidate and there is no group stage.  Stage 2
+    over a memory of one group that holds all n entries: fine scores against
+    all of them, the softmax of Eq. 11 with |C| = n, the top-k_e of Eq. 13."""
+    n = entries.shape[0]
+    b = queries.shape[0]
+    return stage2(entries, np.zeros(n, np.int32), 1, queries, np.zeros((b, 1), np.int32), k_entries, tau, eps,
+                  nthreads)
+
+
 def prefix_reduce(prefix: np.ndarray, lam: float) -> np.ndarray:
     """Prefix-attended query (Eq. 9 over the prefix of Eq. 8, weights of
     Eq. 10): prefix [b, P, d] (q_P the most recent) -> qbar [b, d] float64,

@@ -203,6 +203,22 @@ htam_status htam_query_edges(htam_memory *m, const float *edge_features, int32_t
                     static_cast<cudaStream_t>(cuda_stream), &er);
 }
 
+htam_status htam_query_flat(htam_memory *m, const void *queries, int32_t b, int32_t k_entries, float tau,
+                            float epsilon, int32_t *entry_idx, float *entry_score, float *entry_weight, float *lse,
+                            void *cuda_stream) {
+  if (!m || b < 0 || b > (1 << 24)) return HTAM_EINVAL;
+  if (k_entries < 1 || k_entries > kMaxK) return HTAM_EINVAL;
+  if (!(tau > 0.0f) || !(epsilon >= 0.0f && epsilon <= 1.0f) || !std::isfinite(1.0f / tau)) return HTAM_EINVAL;
+  if (b > 0 && (!queries || !aligned16(queries) || !entry_idx || !entry_score || !entry_weight)) return HTAM_EINVAL;
+  if (b == 0) return HTAM_OK;
+  int64_t nonempty = 0;
+  for (int64_t c : m->h_count) nonempty += c > 0;
+  if ((int64_t)b * std::max<int64_t>(1, nonempty) > kMaxFlatRows) return HTAM_EINVAL;
+  const htam_query_params p{(int32_t)std::max<int64_t>(1, nonempty), k_entries, tau, epsilon};
+  return query_impl(m, queries, b, p, nullptr, nullptr, entry_idx, entry_score, entry_weight, lse,
+                    static_cast<cudaStream_t>(cuda_stream), nullptr, /*flat=*/true);
+}
+
 htam_status htam_query_host(htam_memory *m, const void *queries, int32_t b, const htam_query_params *p,
                             int32_t *group_idx, float *group_score, int32_t *entry_idx, float *entry_score,
                             float *entry_weight, float *lse, void *cuda_stream) {

@@ -214,7 +214,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (u >= n_units) break;
       const int4 U = a.units[u];
       const int g = U.x;
-      const int a_row = a.bucket_off[g] + U.y * kTcRows;
+      const int a_row = (a.q_direct ? 0 : a.bucket_off[g]) + U.y * kTcRows;
       const int pg0 = a.page_off[g];
       const int npg = a.page_off[g + 1] - pg0;
       const int p_beg = U.z * seg_pages, p_end = min(npg, p_beg + seg_pages);

@@ -34,6 +34,8 @@ struct TcFineArgs {
   unsigned *thr_enc;          // [B] order-preserving encoding of a lower bound of the k-th best score
   unsigned *status;           // memory status word
   uint32_t max_polls;
+  int q_direct;               // 1: every bucket holds all queries in order and the query map is the
+                              // query matrix itself (rows from 0), 0: rows from bucket_off[g]
 };
 
 // Encodes a 2-D bf16 row-major [rows, cols] tensor for TMA tile loads of

@@ -111,7 +111,9 @@ struct EdgeRoute {
 htam_status query_impl(htam_memory *m, const void *queries, int32_t b,
                        const htam_query_params &p, int32_t *group_idx, float *group_score,
                        int32_t *entry_idx, float *entry_score, float *entry_weight, float *lse,
-                       cudaStream_t st, const EdgeRoute *er = nullptr);
+                       cudaStream_t st, const EdgeRoute *er = nullptr, bool flat = false);
+// Largest b * (non-empty groups) the flat scan takes (its bucket rows).
+constexpr int64_t kMaxFlatRows = int64_t(1) << 28;
 void free_impl(htam_memory *m);
 
 // Weights alpha_1..alpha_P of a prefix (Eq. 10), passed by value to the

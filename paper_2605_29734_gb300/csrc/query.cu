@@ -275,6 +275,42 @@ __global__ void __launch_bounds__(256) edge_scores_kernel(EdgeKernelArgs a, int 
   s1[t] = acc;
 }
 
+// ---------------------------------------------------------------- flat scan
+
+// The ascending list of non-empty groups (one block, 1024 groups per pass).
+__global__ void __launch_bounds__(1024) flat_groups_kernel(const int32_t *__restrict__ count, int G,
+                                                           int32_t *__restrict__ list) {
+  __shared__ int warp_n[32];
+  __shared__ int base;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if (threadIdx.x == 0) base = 0;
+  __syncthreads();
+  for (int g0 = 0; g0 < G; g0 += 1024) {
+    const int g = g0 + (int)threadIdx.x;
+    const bool ne = g < G && count[g] > 0;
+    const unsigned bal = __ballot_sync(0xffffffffu, ne);
+    if (lane == 0) warp_n[warp] = __popc(bal);
+    __syncthreads();
+    int before = base;
+    for (int w = 0; w < warp; ++w) before += warp_n[w];
+    if (ne) list[before + __popc(bal & ((1u << lane) - 1u))] = g;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      int n = 0;
+      for (int w = 0; w < 32; ++w) n += warp_n[w];
+      base += n;
+    }
+    __syncthreads();
+  }
+}
+
+// Every query selects every non-empty group: group_idx[b][j] = list[j].
+__global__ void flat_fill_kernel(const int32_t *__restrict__ list, int64_t rows, int kg,
+                                 int32_t *__restrict__ group_idx) {
+  const int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  if (t < rows) group_idx[t] = list[t % kg];
+}
+
 // ---------------------------------------------------------------- bucketing
 
 __global__ void bucket_bits_kernel(const int32_t *__restrict__ gidx, int B, int kg, int W,
@@ -788,44 +824,71 @@ __global__ void __launch_bounds__(kMergeWarps * 32, 1) merge_kernel(MergeArgs a)
     }
     return r;
   };
-  constexpr int kBatch = 4;  // records fetched before any is combined
+  // Records are taken 32 at a time, one per lane, across group boundaries:
+  // each lane reads its record's softmax statistics and best pair, the
+  // statistics are combined by warp reductions, and only records whose best
+  // pair can still enter the top-ke are read in full (up to 4 at a time).
   const int n_t = live ? (a.kg - sw + WPQ - 1) / WPQ : 0;
-  for (int t0 = 0; t0 < n_t; t0 += 64) {
-    const GroupRecs gr0 = load_group(t0 + lane), gr1 = load_group(t0 + lane + 32);
-    const int t_end = min(n_t, t0 + 64);
-    for (int t = t0; t < t_end; ++t) {
-      const bool lo = t - t0 < 32;
-      const int src = (t - t0) & 31;
-      const int g = __shfl_sync(kFullMask, lo ? gr0.g : gr1.g, src);
-      if (g < 0) continue;  // uniform
-      const int p = __shfl_sync(kFullMask, lo ? gr0.p : gr1.p, src);
-      const int cg = __shfl_sync(kFullMask, lo ? gr0.cg : gr1.cg, src);
-      const int nseg = __shfl_sync(kFullMask, lo ? gr0.nseg : gr1.nseg, src);
-      const long long base = __shfl_sync(kFullMask, lo ? gr0.base : gr1.base, src);
-      for (int s0 = 0; s0 < nseg; s0 += kBatch) {
-        float2 ml[kBatch];
-        float cs[kBatch][2];
-        int ci[kBatch][2];
+  for (int t0 = 0; t0 < n_t; t0 += 32) {
+    const GroupRecs gr = load_group(t0 + lane);
+    const int nseg = gr.g >= 0 ? gr.nseg : 0;
+    int incl = nseg;  // inclusive prefix of the records over the lanes' groups
 #pragma unroll
-        for (int i = 0; i < kBatch; ++i) {
-          const bool v = s0 + i < nseg;
-          const int64_t pidx = base + (int64_t)(s0 + i) * cg + p;
-          ml[i] = v ? a.part_ml[pidx] : make_float2(-INFINITY, 0.f);
+    for (int o = 1; o < 32; o <<= 1) {
+      const int v = __shfl_up_sync(kFullMask, incl, o);
+      if (lane >= o) incl += v;
+    }
+    const int excl = incl - nseg;
+    const int total = __shfl_sync(kFullMask, incl, 31);
+    for (int r0 = 0; r0 < total; r0 += 32) {
+      const int r = r0 + lane;
+      // The lane whose group holds record r: the last lane with excl <= r.
+      int own = 0;
+#pragma unroll
+      for (int step = 16; step > 0; step >>= 1) {
+        if (__shfl_sync(kFullMask, excl, own + step) <= r) own += step;
+      }
+      const int seg = r - __shfl_sync(kFullMask, excl, own);
+      const int p = __shfl_sync(kFullMask, gr.p, own);
+      const int cg = __shfl_sync(kFullMask, gr.cg, own);
+      const long long base = __shfl_sync(kFullMask, gr.base, own);
+      const bool valid = r < total;
+      const long long pidx = base + (long long)seg * cg + p;
+      const float2 ml = valid ? a.part_ml[pidx] : make_float2(-INFINITY, 0.f);
+      const float hs = valid ? a.part_s[pidx * ke] : -INFINITY;
+      const int hi = valid ? a.part_id[pidx * ke] : INT_MAX;
+      const float Mb = warp_max(ml.x);
+      if (Mb != -INFINITY) {
+        const float Lb = warp_sum(ml.x == -INFINITY ? 0.f : ml.y * expf(ml.x - Mb));
+        const float Mn = fmaxf(M, Mb);
+        L = L * expf(M - Mn) + Lb * expf(Mb - Mn);
+        M = Mn;
+      }
+      unsigned todo = __ballot_sync(kFullMask, hi != INT_MAX && better(hs, hi, fs, fi));
+      while (todo) {
+        constexpr int kTake = 4;
+        int src[kTake];
+#pragma unroll
+        for (int i = 0; i < kTake; ++i) {
+          src[i] = todo ? __ffs(todo) - 1 : -1;
+          if (todo) todo &= todo - 1;
+        }
+        float cs[kTake][2];
+        int ci[kTake][2];
+#pragma unroll
+        for (int i = 0; i < kTake; ++i) {
+          const long long q = __shfl_sync(kFullMask, pidx, src[i] < 0 ? 0 : src[i]);
 #pragma unroll
           for (int h = 0; h < 2; ++h) {
             const int tt = h * 32 + lane;
-            const bool in = v && tt < ke;
-            cs[i][h] = in ? a.part_s[pidx * ke + tt] : -INFINITY;
-            ci[i][h] = in ? a.part_id[pidx * ke + tt] : INT_MAX;
+            const bool in = src[i] >= 0 && tt < ke;
+            cs[i][h] = in ? a.part_s[q * ke + tt] : -INFINITY;
+            ci[i][h] = in ? a.part_id[q * ke + tt] : INT_MAX;
           }
         }
 #pragma unroll
-        for (int i = 0; i < kBatch; ++i) {
-          if (ml[i].x != -INFINITY) {
-            const float Mn = fmaxf(M, ml[i].x);
-            L = L * expf(M - Mn) + ml[i].y * expf(ml[i].x - Mn);
-            M = Mn;
-          }
+        for (int i = 0; i < kTake; ++i) {
+          if (src[i] < 0) break;  // uniform
           if (ke <= 32) {
             take32(cs[i][0], ci[i][0]);
           } else {
@@ -833,6 +896,8 @@ __global__ void __launch_bounds__(kMergeWarps * 32, 1) merge_kernel(MergeArgs a)
             for (int h = 0; h < 2; ++h) offer(cs[i][h], ci[i][h], ke - h * 32);
           }
         }
+        // Drop the records the raised k-th best now excludes.
+        todo &= __ballot_sync(kFullMask, hi != INT_MAX && better(hs, hi, fs, fi));
       }
     }
   }
@@ -954,11 +1019,17 @@ constexpr uint32_t kMaxPolls = 1u << 24;
 htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const htam_query_params &p,
                        int32_t *group_idx, float *group_score, int32_t *entry_idx,
                        float *entry_score, float *entry_weight, float *lse, cudaStream_t st,
-                       const EdgeRoute *er) {
+                       const EdgeRoute *er, bool flat) {
   if (B == 0) return HTAM_OK;
   m->n_queries += 1;
   PhaseMark mark(m, st);
-  const int G = m->n_groups, d = m->d, kg = p.k_groups, ke = p.k_entries;
+  // The flat scan selects every non-empty group (at least one slot, -1 when
+  // the memory is empty); the group lists then live in the scratch.
+  int n_nonempty = 0;
+  if (flat) {
+    for (int64_t c : m->h_count) n_nonempty += c > 0;
+  }
+  const int G = m->n_groups, d = m->d, kg = flat ? std::max(1, n_nonempty) : p.k_groups, ke = p.k_entries;
   const int qc = simt_query_chunk(d);
   // The tensor-core path takes bf16 memories and k_entries <= 32.
   const bool tc_ok = m->dtype == HTAM_BF16 && ke <= kTcMaxK && m->tc_min <= B;
@@ -979,10 +1050,12 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   const int64_t max_units = max_parts;
   const int64_t rows = (int64_t)B * kg;  // bucket rows
   const int W = (int)ceil_div(B, 32);
-  const size_t qg_bytes = tc_ok ? sizeof(__nv_bfloat16) * (size_t)rows * d : 0;
+  // Flat scan: every bucket holds all queries in order, so the tensor-core
+  // kernel reads the query matrix itself instead of a gathered copy.
+  const size_t qg_bytes = tc_ok && !flat ? sizeof(__nv_bfloat16) * (size_t)rows * d : 0;
 
   // Coarse scores: one plane per K split of the tensor-core kernel.
-  const int planes = m->dtype == HTAM_BF16 && !er ? coarse_tc_splits(B, d, G, m->sm_count) : 1;
+  const int planes = flat ? 0 : m->dtype == HTAM_BF16 && !er ? coarse_tc_splits(B, d, G, m->sm_count) : 1;
   // Edge routing: form the whole utility table once when the batch references
   // more prefix rows than the table has.
   const bool edge_table = er && (int64_t)B * er->P > G;
@@ -994,7 +1067,7 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
                 3 * Carver::round(sizeof(int32_t) * rows) + 2 * Carver::round(sizeof(int4) * max_units) +
                 Carver::round(sizeof(float2) * max_parts) + Carver::round(sizeof(float) * max_parts * ke) +
                 Carver::round(sizeof(int32_t) * max_parts * ke) + Carver::round(sizeof(unsigned) * B) +
-                Carver::round(qg_bytes) + 8192;
+                Carver::round(qg_bytes) + (flat ? Carver::round(sizeof(int32_t) * rows) + Carver::round(sizeof(int32_t) * kg) : 0) + 8192;
   htam_status s = ensure_scratch(m, need);
   if (s != HTAM_OK) return s;
   Carver cv(m->scratch);
@@ -1020,10 +1093,25 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   float *part_s = cv.take<float>(max_parts * ke);
   int32_t *part_id = cv.take<int32_t>(max_parts * ke);
   unsigned *thr_enc = cv.take<unsigned>(B);
-  void *qg = tc_ok ? static_cast<void *>(cv.take<char>(qg_bytes)) : nullptr;
+  void *qg = tc_ok && !flat ? static_cast<void *>(cv.take<char>(qg_bytes)) : nullptr;
+  if (flat) {
+    group_idx = cv.take<int32_t>(rows);
+    int32_t *list = cv.take<int32_t>(kg);  // the non-empty groups, ascending
+    mark.begin(HTAM_PHASE_SELECT);
+    if (n_nonempty == 0) {
+      HTAM_CK(cudaMemsetAsync(group_idx, 0xff, sizeof(int32_t) * (size_t)rows, st));
+    } else {
+      flat_groups_kernel<<<1, 1024, 0, st>>>(m->count, G, list);
+      HTAM_CK_LAUNCH("flat_groups_kernel");
+      flat_fill_kernel<<<(unsigned)ceil_div(rows, 256), 256, 0, st>>>(list, rows, kg, group_idx);
+      HTAM_CK_LAUNCH("flat_fill_kernel");
+      mark.launched(2);
+    }
+    mark.end();
+  }
 
   // 1. Coarse scores and the selected groups.
-  {
+  if (!flat) {
     mark.begin(HTAM_PHASE_COARSE);
     if (er) {
       // Transition-edge scores (the prefix ids were checked on the host).
@@ -1099,13 +1187,15 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
       if (s != HTAM_OK) return s;
       m->pool_map_ready = true;
     }
-    s = make_bf16_tile_map(&q_map, qg, rows, d, kTcRows);
+    s = flat ? make_bf16_tile_map(&q_map, queries, B, d, kTcRows) : make_bf16_tile_map(&q_map, qg, rows, d, kTcRows);
     if (s != HTAM_OK) return s;
     HTAM_CK(cudaMemsetAsync(thr_enc, 0, sizeof(unsigned) * B, st));
     HTAM_CK(cudaMemsetAsync(tc_ctr, 0, sizeof(int32_t), st));
-    s = launch_gather_queries(queries, d, bucket, bucket_group, cnt, rt.tc_min, bucket_off + G, rows, qg, st);
-    if (s != HTAM_OK) return s;
-    mark.launched();
+    if (!flat) {
+      s = launch_gather_queries(queries, d, bucket, bucket_group, cnt, rt.tc_min, bucket_off + G, rows, qg, st);
+      if (s != HTAM_OK) return s;
+      mark.launched();
+    }
   }
   mark.end();
 
@@ -1133,7 +1223,7 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
     mark.begin(HTAM_PHASE_FINE_TC);
     TcFineArgs ta{units_tc, n_units + 1, tc_ctr, bucket, bucket_off, cnt, m->page_list, m->page_off, m->count, m->slot_id,
                   part_off, d, seg_tc, ke, 1.4426950408889634f / p.tau, part_ml, part_s, part_id, thr_enc,
-                  m->status, kMaxPolls};
+                  m->status, kMaxPolls, flat ? 1 : 0};
     s = launch_fine_tc(ta, q_map, m->pool_map, (int)std::min<int64_t>(max_units, m->sm_count), st);
     if (s != HTAM_OK) return s;
     mark.launched();

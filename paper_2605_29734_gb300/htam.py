@@ -24,7 +24,7 @@ HTAM_MAX_EDGE_FEATURES = 32  # most features per edge htam_query_edges takes
 # Every symbol include/htam.h declares, in declaration order.
 EXPORTS = (
     "htam_build_memory", "htam_append_transitions", "htam_query", "htam_query_host", "htam_query_prefix",
-    "htam_query_edges",
+    "htam_query_edges", "htam_query_flat",
     "htam_select_groups_static", "htam_memory_info", "htam_memory_group_counts", "htam_memory_group_keys",
     "htam_device_status", "htam_set_tuning", "htam_get_tuning", "htam_set_phase_timing",
     "htam_read_phase_timing", "htam_free_memory", "htam_status_string", "htam_last_error",
@@ -61,6 +61,7 @@ def _load() -> ctypes.CDLL:
                                       P, P, P, P, P, P, P]
     lib.htam_query_edges.argtypes = [P, P, i32, P, P, i32, ctypes.c_float, P, i32, ctypes.POINTER(QueryParams),
                                      P, P, P, P, P, P, P]
+    lib.htam_query_flat.argtypes = [P, P, i32, i32, ctypes.c_float, ctypes.c_float, P, P, P, P, P]
     lib.htam_memory_info.argtypes = [P, P, P, P, P]
     lib.htam_memory_group_counts.argtypes = [P, P]
     lib.htam_memory_group_keys.argtypes = [P, P, P]
@@ -177,6 +178,27 @@ class Memory:
                                _dev_ptr(out["entry_idx"]), _dev_ptr(out["entry_score"]),
                                _dev_ptr(out["entry_weight"]), _dev_ptr(out.get("lse")),
                                _stream_ptr(stream)), "htam_query")
+        return out
+
+    def query_flat(self, queries: torch.Tensor, k_entries: int, tau: float = 1.0, epsilon: float = 0.0,
+                   stream=None, out: dict | None = None) -> dict:
+        """Flat scan: every entry a candidate, no group stage; returns (or
+        fills) entry_idx, entry_score, entry_weight and lse."""
+        if queries.dtype != self.dtype or queries.dim() != 2 or queries.shape[1] != self.d:
+            raise ValueError("queries must be [b, d] of the memory dtype")
+        b = queries.shape[0]
+        dev = queries.device
+        if out is None:
+            out = {
+                "entry_idx": torch.empty(b, k_entries, dtype=torch.int32, device=dev),
+                "entry_score": torch.empty(b, k_entries, dtype=torch.float32, device=dev),
+                "entry_weight": torch.empty(b, k_entries, dtype=torch.float32, device=dev),
+                "lse": torch.empty(b, dtype=torch.float32, device=dev),
+            }
+        _check(_lib.htam_query_flat(self.handle, _dev_ptr(queries), b, k_entries, float(tau), float(epsilon),
+                                    _dev_ptr(out["entry_idx"]), _dev_ptr(out["entry_score"]),
+                                    _dev_ptr(out["entry_weight"]), _dev_ptr(out.get("lse")),
+                                    _stream_ptr(stream)), "htam_query_flat")
         return out
 
     def query_prefix(self, prefix: torch.Tensor, lam: float, k_groups: int, k_entries: int, tau: float = 1.0,

@@ -167,6 +167,25 @@ def compare_edge_lookup(out, entries_np, gid_np, n_groups, Z, w, prefix, lam, qu
     return problems
 
 
+def compare_flat(out, entries_np, queries_np, k_entries, tau, eps, dtype, rows=None, nthreads=None):
+    """The flat scan of the queries listed in `rows` (all by default) against
+    the oracle's flat retrieval."""
+    import oracle
+
+    ei = out["entry_idx"].cpu().numpy()
+    es = out["entry_score"].cpu().numpy()
+    ew = out["entry_weight"].cpu().numpy()
+    lse = out["lse"].cpu().numpy()
+    rows = np.arange(queries_np.shape[0]) if rows is None else np.asarray(rows)
+    q = queries_np[rows]
+    ref2 = oracle.flat(entries_np, q, k_entries + 16, tau, eps, nthreads)
+    qf = _as_f64(q)
+    problems = []
+    for r, b in enumerate(rows):
+        problems += _check_entries(ei, es, ew, lse, b, r, ref2, entries_np, qf, k_entries, tau, eps, dtype)
+    return problems
+
+
 def _as_f64(x: np.ndarray) -> np.ndarray:
     if x.dtype == np.uint16:
         return (x.astype(np.uint32) << 16).view(np.float32).astype(np.float64)

@@ -112,6 +112,14 @@ def test_uniform_4m_workload_sampled(htam):
                               "bf16", rows=rows, centroid=cent, counts=counts)
     assert not problems, "\n".join(problems[:20])
 
+    # The flat scan on the same memory, full batch, a sample of queries.
+    from parity import compare_flat
+
+    flat = mem.query_flat(q, w.k_entries)
+    torch.cuda.synchronize()
+    problems = compare_flat(flat, entries_np, to_numpy(q), w.k_entries, 1.0, 0.0, "bf16", rows=rows[::2])
+    assert not problems, "\n".join(problems[:20])
+
 
 # ------------------------------------------------------------------ edge cases
 
@@ -354,6 +362,117 @@ def test_edge_arguments_checked(htam):
                         np.ones(htam.HTAM_MAX_EDGE_FEATURES + 1, np.float32), good, 0.5, q, 2, 4)
     with pytest.raises(htam.HtamError):
         mem.query_edges(Z, np.array([1.0] * 11 + [np.nan], np.float32), good, 0.5, q, 2, 4)
+
+
+FLAT_CASES = [
+    # n, groups, d, dtype, batch, k_entries, tensor-core threshold (None = default)
+    (8000, 40, 256, torch.float32, 30, 16, None),        # fp32: CUDA-core kernel
+    (20000, 60, 512, torch.bfloat16, 150, 32, None),     # two 128-query chunks per group, the second ragged
+    (20000, 60, 512, torch.bfloat16, 150, 33, None),     # k_entries above the tensor-core limit
+    (6000, 30, 1024, torch.bfloat16, 7, 12, 1 << 30),    # bf16 rows through the CUDA-core ring
+    (30000, 30, 4096, torch.bfloat16, 64, 16, None),     # 8 KiB rows, 64 queries (the 4M workload's batch)
+    (60000, 8, 256, torch.bfloat16, 300, 20, None),      # groups spanning many page segments
+]
+
+
+@pytest.mark.parametrize("case", FLAT_CASES)
+def test_flat_scan_matches_oracle(htam, case):
+    """htam_query_flat against the oracle's flat retrieval (every entry a
+    candidate, |C| = n in the epsilon term)."""
+    from parity import compare_flat
+
+    n, g, d, dtype, b, ke, tc_min = case
+    entries, gid, centres = _rand_memory(n, d, g, dtype, seed=n + d + b)
+    q = _rand_queries(b, d, dtype, seed=n + d + b, centres=centres)
+    mem = htam.Memory(entries, gid, g)
+    if tc_min is not None:
+        mem.set_tensor_core_min_bucket(tc_min)
+    mem.read_phase_timing()
+    out = mem.query_flat(q, ke, tau=0.6, epsilon=0.05)
+    torch.cuda.synchronize()
+    dt = "bf16" if dtype == torch.bfloat16 else "f32"
+    problems = compare_flat(out, to_numpy(entries), to_numpy(q), ke, 0.6, 0.05, dt)
+    assert not problems, "\n".join(problems[:20])
+    assert mem.device_status() == htam.HTAM_OK
+    ran = mem.read_phase_timing()
+    assert ran["coarse"][1] == 0  # no group stage
+    if dtype == torch.bfloat16 and ke <= 32 and tc_min is None:
+        assert ran["fine_tc"][1] > 0
+
+
+@pytest.mark.parametrize("dtype,tc_min", [(torch.bfloat16, None), (torch.bfloat16, 1 << 30), (torch.float32, None)])
+def test_flat_scan_equals_lookup_with_every_group(htam, dtype, tc_min):
+    """With k_groups = the number of non-empty groups the two-level lookup
+    scores the same candidates with the same kernels: identical ids and
+    scores.  The softmax denominators are summed over the groups in selection
+    order there and in group-id order here, so weights and lse agree to fp32
+    rounding."""
+    gid = torch.arange(5000, device=DEV, dtype=torch.int32) % 23 * 2  # 23 of 46 groups hold entries
+    entries, gid, centres = _rand_memory(5000, 512, 46, dtype, seed=8, gid=gid)
+    q = _rand_queries(140, 512, dtype, seed=8)
+    mem = htam.Memory(entries, gid, 46)
+    if tc_min is not None:
+        mem.set_tensor_core_min_bucket(tc_min)
+    a = mem.query(q, 23, 24, tau=0.5, epsilon=0.1)
+    f = mem.query_flat(q, 24, tau=0.5, epsilon=0.1)
+    torch.cuda.synchronize()
+    assert torch.equal(a["entry_idx"], f["entry_idx"])
+    assert torch.equal(a["entry_score"], f["entry_score"])
+    torch.testing.assert_close(f["entry_weight"], a["entry_weight"], rtol=1e-5, atol=1e-9)
+    torch.testing.assert_close(f["lse"], a["lse"], rtol=1e-6, atol=1e-6)
+
+
+def test_flat_scan_short_memory_and_empty_batch(htam):
+    """Fewer entries than k_entries pads with -1 / -inf / 0; an empty batch
+    launches nothing."""
+    gid = torch.tensor([2, 5, 5, 9, 2, 2], dtype=torch.int32, device=DEV)
+    entries, gid, _ = _rand_memory(6, 32, 12, torch.float32, seed=9, clustered=False, gid=gid)
+    q = _rand_queries(5, 32, torch.float32, seed=9)
+    mem = htam.Memory(entries, gid, 12)
+    out = mem.query_flat(q, 10, tau=0.3, epsilon=0.2)
+    torch.cuda.synchronize()
+    from parity import compare_flat
+
+    problems = compare_flat(out, to_numpy(entries), to_numpy(q), 10, 0.3, 0.2, "f32")
+    assert not problems, "\n".join(problems)
+    assert (out["entry_idx"][:, 6:] == -1).all() and (out["entry_weight"][:, 6:] == 0).all()
+    assert torch.isneginf(out["entry_score"][:, 6:]).all()
+    empty = mem.query_flat(torch.empty(0, 32, device=DEV), 4)
+    torch.cuda.synchronize()
+    assert empty["entry_idx"].shape == (0, 4)
+
+
+def test_flat_scan_after_appends(htam):
+    """Appended entries (Eq. 15) are candidates of the next flat scan, also in
+    groups that were empty before."""
+    from parity import compare_flat
+
+    entries, gid, centres = _rand_memory(3000, 256, 20, torch.bfloat16, seed=10,
+                                         gid=torch.arange(3000, device=DEV, dtype=torch.int32) % 10)
+    mem = htam.Memory(entries, gid, 20, capacity=6000)
+    more, more_gid, _ = _rand_memory(1500, 256, 20, torch.bfloat16, seed=11)
+    mem.append(more, more_gid)
+    q = _rand_queries(40, 256, torch.bfloat16, seed=10, centres=centres)
+    out = mem.query_flat(q, 16, tau=0.8)
+    torch.cuda.synchronize()
+    all_e = torch.cat([entries, more])
+    problems = compare_flat(out, to_numpy(all_e), to_numpy(q), 16, 0.8, 0.0, "bf16")
+    assert not problems, "\n".join(problems[:20])
+
+
+def test_flat_arguments_checked(htam):
+    entries, gid, _ = _rand_memory(500, 64, 4, torch.float32, seed=12)
+    mem = htam.Memory(entries, gid, 4)
+    q = torch.zeros(3, 64, device=DEV)
+    for ke in (0, 65):
+        with pytest.raises(htam.HtamError):
+            mem.query_flat(q, ke)
+    for tau, eps in ((0.0, 0.0), (float("nan"), 0.0), (1.0, -0.1), (1.0, 1.5)):
+        with pytest.raises(htam.HtamError):
+            mem.query_flat(q, 4, tau=tau, epsilon=eps)
+    raw = torch.zeros(3 * 64 + 1, device=DEV)
+    with pytest.raises(htam.HtamError):  # queries not 16-byte aligned
+        mem.query_flat(raw[1:].view(3, 64), 4)
 
 
 def test_tuning_defaults_follow_row_length_and_round_trip(htam):

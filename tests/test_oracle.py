@@ -140,6 +140,30 @@ def test_all_groups_selected_equals_flat_scan(dtype):
         assert out["n_cand"][b] == n
 
 
+def test_flat_scan_matches_numpy_brute_force():
+    """The flat retrieval against numpy: matmul scores, lexsort top-k (ties to
+    the lower id, planted by duplicated rows), scipy's logsumexp, and the
+    epsilon term of Eq. 11 spread over all n entries."""
+    rng = np.random.default_rng(23)
+    n, d, b, k, tau, eps = 240, 20, 6, 30, 0.2, 0.15
+    x = _unit_rows(rng, n, d)
+    x[100:120] = x[0:20]  # equal scores: the lower id must come first
+    q = _unit_rows(rng, b, d)
+    out = oracle.flat(x, q, k, tau=tau, eps=eps)
+    scores = q.astype(np.float64) @ x.astype(np.float64).T
+    for r in range(b):
+        order = np.lexsort((np.arange(n), -scores[r]))[:k]
+        assert list(out["entry_idx"][r]) == list(order)
+        np.testing.assert_allclose(out["entry_score"][r], scores[r][order], rtol=0, atol=1e-12)
+        lse = logsumexp(scores[r] / tau)
+        assert out["lse"][r] == pytest.approx(lse, rel=1e-12)
+        np.testing.assert_allclose(out["entry_weight"][r],
+                                   eps / n + (1 - eps) * np.exp(scores[r][order] / tau - lse), rtol=1e-11)
+        assert out["n_cand"][r] == n
+    short = oracle.flat(x[:5], q, 8)
+    assert (short["entry_idx"][:, 5:] == -1).all() and (short["entry_weight"][:, 5:] == 0).all()
+
+
 def test_stage1_matches_numpy_brute_force():
     """Group keys by numpy (bincount means), coarse scores by matmul, top-k by
     lexsort: an independent computation of centroids + stage 1."""
