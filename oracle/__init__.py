@@ -68,6 +68,12 @@ def _load():
         lib.htam_oracle_edge_scores.restype = ctypes.c_int
         lib.htam_oracle_select.argtypes = [P, P, i32, i32, i32, P, P]
         lib.htam_oracle_select.restype = ctypes.c_int
+        lib.htam_oracle_philox4x32_10.argtypes = [P, P, P]
+        lib.htam_oracle_philox4x32_10.restype = None
+        lib.htam_oracle_policy_uniform.argtypes = [ctypes.c_uint64, ctypes.c_uint64, i32, i32]
+        lib.htam_oracle_policy_uniform.restype = dbl
+        lib.htam_oracle_policy_keys.argtypes = [P, P, i32, i32, dbl, dbl, ctypes.c_uint64, ctypes.c_uint64, P, P]
+        lib.htam_oracle_policy_keys.restype = ctypes.c_int
         _lib = lib
         return lib
 
@@ -277,3 +283,70 @@ def query_edges(entries: np.ndarray, gid: np.ndarray, n_groups: int, Z: np.ndarr
     out["group_idx"] = gi
     out["group_score"] = gs
     return out
+
+
+# ------------------------------------------------ sampling from the policy (Eq. 11)
+
+def philox4x32_10(ctr, key) -> np.ndarray:
+    """Philox4x32-10 (Salmon et al., SC 2011): four counter words and two key
+    words (uint32) -> four uint32 outputs."""
+    lib = _load()
+    c = np.ascontiguousarray(ctr, dtype=np.uint32)
+    k = np.ascontiguousarray(key, dtype=np.uint32)
+    if c.shape != (4,) or k.shape != (2,):
+        raise ValueError("counter has 4 words, key 2")
+    out = np.empty(4, dtype=np.uint32)
+    lib.htam_oracle_philox4x32_10(_ptr(c), _ptr(k), _ptr(out))
+    return out
+
+
+def policy_uniform(seed: int, offset: int, b: int, g: int) -> float:
+    """The uniform in (0, 1) that query b draws for group g."""
+    return float(_load().htam_oracle_policy_uniform(seed, offset, b, g))
+
+
+def coarse_scores(queries: np.ndarray, centroid: np.ndarray) -> np.ndarray:
+    """s[b][g] = q_b . c_g in float64 for every group (matrix product)."""
+    return _as_f64_input(queries) @ np.asarray(centroid, dtype=np.float64).T
+
+
+def policy_keys(scores: np.ndarray, counts: np.ndarray, tau: float, eps: float, seed: int, offset: int):
+    """Gumbel-top-k keys of the Eq. 11 policy over the non-empty groups and
+    the policy itself: returns (keys, mu), both [b, G] float64."""
+    lib = _load()
+    scores = np.ascontiguousarray(scores, dtype=np.float64)
+    counts = np.ascontiguousarray(counts, dtype=np.int64)
+    b, G = scores.shape
+    keys = np.empty((b, G), dtype=np.float64)
+    mu = np.empty((b, G), dtype=np.float64)
+    rc = lib.htam_oracle_policy_keys(_ptr(scores), _ptr(counts), b, G, float(tau), float(eps), int(seed),
+                                     int(offset), _ptr(keys), _ptr(mu))
+    if rc != 0:
+        raise ValueError("oracle policy_keys: bad argument")
+    return keys, mu
+
+
+def query_sampled(entries: np.ndarray, gid: np.ndarray, n_groups: int, queries: np.ndarray, k_groups: int,
+                  k_entries: int, tau: float, eps: float, seed: int, offset: int, centroid=None, counts=None,
+                  nthreads: int | None = None):
+    """The lookup with stage 1 drawn from the policy (Algorithm 1, step 2:
+    k_groups draws without replacement from mu_g of Eq. 11 over the group-key
+    scores), then stage 2 on the drawn groups."""
+    if centroid is None or counts is None:
+        centroid, counts = centroids(entries, gid, n_groups, nthreads)
+    keys, mu = policy_keys(coarse_scores(queries, centroid), counts, tau, eps, seed, offset)
+    gi, gk = select(keys, counts, k_groups)
+    out = stage2(entries, gid, n_groups, queries, gi, k_entries, tau, eps, nthreads)
+    out["group_idx"] = gi
+    out["group_key"] = gk
+    out["keys"] = keys
+    out["mu"] = mu
+    return out
+
+
+def _as_f64_input(x: np.ndarray) -> np.ndarray:
+    """float32 arrays or bf16 bit patterns (uint16) as float64, exactly."""
+    x = np.asarray(x)
+    if x.dtype == np.uint16:
+        return (x.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+    return x.astype(np.float64)

@@ -444,3 +444,98 @@ int htam_oracle_select(const double *scores, const int64_t *counts, int32_t n_qu
   free(cand);
   return 0;
 }
+
+/* ------------------------------------------------------------------------
+ * Sampling from the global-direction policy (Eq. 11; Algorithm 1, step 2
+ * draws g_t from it).
+ *
+ * Generator: Philox4x32-10, the counter-based generator of Salmon, Moraes,
+ * Dror and Shaw ("Parallel random numbers: as easy as 1, 2, 3", SC 2011).
+ * A 128-bit counter (four 32-bit words) and a 64-bit key (two words) map to
+ * four 32-bit outputs through ten rounds.  A round multiplies counter words 0
+ * and 2 by two fixed odd constants, giving 64-bit products; the new words are
+ * (high half of product 2) xor word 1 xor key 0, (low half of product 2),
+ * (high half of product 0) xor word 3 xor key 1, (low half of product 0).
+ * Between rounds both key words advance by fixed Weyl increments (the golden
+ * ratio and sqrt(3) - 1, scaled to 32 bits). */
+static const uint32_t kPhiloxMul0 = 0xD2511F53u, kPhiloxMul1 = 0xCD9E8D57u;
+static const uint32_t kPhiloxWeyl0 = 0x9E3779B9u, kPhiloxWeyl1 = 0xBB67AE85u;
+
+void htam_oracle_philox4x32_10(const uint32_t *ctr, const uint32_t *key, uint32_t *out) {
+  uint32_t c[4] = {ctr[0], ctr[1], ctr[2], ctr[3]};
+  uint32_t k0 = key[0], k1 = key[1];
+  for (int r = 0; r < 10; ++r) {
+    if (r > 0) {
+      k0 += kPhiloxWeyl0;
+      k1 += kPhiloxWeyl1;
+    }
+    const uint64_t p0 = (uint64_t)kPhiloxMul0 * c[0];
+    const uint64_t p1 = (uint64_t)kPhiloxMul1 * c[2];
+    const uint32_t n0 = (uint32_t)(p1 >> 32) ^ c[1] ^ k0;
+    const uint32_t n1 = (uint32_t)p1;
+    const uint32_t n2 = (uint32_t)(p0 >> 32) ^ c[3] ^ k1;
+    const uint32_t n3 = (uint32_t)p0;
+    c[0] = n0;
+    c[1] = n1;
+    c[2] = n2;
+    c[3] = n3;
+  }
+  out[0] = c[0];
+  out[1] = c[1];
+  out[2] = c[2];
+  out[3] = c[3];
+}
+
+/* The uniform of query b and group g: word (g mod 4) of Philox4x32-10 at
+ * counter (g / 4, b, low and high words of `offset`) under key (low and high
+ * words of `seed`); its top 23 bits plus one half, times 2^-23, so that
+ * u lies in (0, 1) and is exact in float32. */
+double htam_oracle_policy_uniform(uint64_t seed, uint64_t offset, int32_t b, int32_t g) {
+  const uint32_t ctr[4] = {(uint32_t)g >> 2, (uint32_t)b, (uint32_t)offset, (uint32_t)(offset >> 32)};
+  const uint32_t key[2] = {(uint32_t)seed, (uint32_t)(seed >> 32)};
+  uint32_t out[4];
+  htam_oracle_philox4x32_10(ctr, key, out);
+  return ((double)(out[g & 3] >> 9) + 0.5) * (1.0 / 8388608.0);
+}
+
+/* The policy of Eq. 11 over the candidate directions G_t = the non-empty
+ * groups (n of them), and the keys that draw from it.
+ *   mu[b][g] = eps / n + (1 - eps) * exp(s[b][g] / tau - lse_b),
+ *   lse_b = log sum_{g in G_t} exp(s[b][g] / tau)
+ * (0 for empty groups).  keys[b][g] = log mu[b][g] - log(-log u(b, g)) (log mu
+ * taken as s/tau - lse when eps = 0; -inf for empty groups).  The k groups
+ * with the largest keys (ties to the lower id) are k draws without
+ * replacement from mu, in draw order: the Gumbel-top-k construction (Kool, van
+ * Hoof and Welling, ICML 2019; k = 1 is the Gumbel-max draw of g_t ~ mu).
+ * Returns 0, or -1 on a bad argument. */
+int htam_oracle_policy_keys(const double *scores, const int64_t *counts, int32_t n_queries, int32_t G, double tau,
+                            double eps, uint64_t seed, uint64_t offset, double *keys, double *mu) {
+  if (G < 1 || n_queries < 0 || !(tau > 0.0) || !(eps >= 0.0 && eps <= 1.0)) return -1;
+  int64_t n = 0;
+  for (int32_t g = 0; g < G; ++g) n += counts[g] > 0;
+  for (int32_t b = 0; b < n_queries; ++b) {
+    const double *s = scores + (int64_t)b * G;
+    double m = -INFINITY;
+    for (int32_t g = 0; g < G; ++g) {
+      if (counts[g] > 0 && s[g] / tau > m) m = s[g] / tau;
+    }
+    double sum = 0.0;
+    for (int32_t g = 0; g < G; ++g) {
+      if (counts[g] > 0) sum += exp(s[g] / tau - m);
+    }
+    const double lse = m + log(sum);
+    for (int32_t g = 0; g < G; ++g) {
+      const int64_t o = (int64_t)b * G + g;
+      if (counts[g] == 0) {
+        mu[o] = 0.0;
+        keys[o] = -INFINITY;
+        continue;
+      }
+      mu[o] = eps / (double)n + (1.0 - eps) * exp(s[g] / tau - lse);
+      const double log_mu = eps == 0.0 ? s[g] / tau - lse : log(mu[o]);
+      const double u = htam_oracle_policy_uniform(seed, offset, b, g);
+      keys[o] = log_mu - log(-log(u));
+    }
+  }
+  return 0;
+}

@@ -9,6 +9,7 @@ sign, a transposed operand, a missing 1/n, tau multiplied instead of divided,
 a wrong tie order, a leak outside the selected groups) fails at least one.
 """
 import math
+import os
 
 import numpy as np
 import pytest
@@ -487,3 +488,98 @@ def test_select_matches_lexsort_without_empty_groups():
         assert list(gi[q, :len(order)]) == list(order)
         assert np.all(gi[q, len(order):] == -1)
         np.testing.assert_array_equal(gs[q, :len(order)], scores[q, order])
+
+
+# ------------------------------------------- sampling from the policy (Eq. 11)
+
+GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
+
+
+def test_philox_known_answers():
+    """Philox4x32-10 against the published known-answer vectors."""
+    n = 0
+    for line in open(os.path.join(GOLDEN, "philox4x32_10_kat.txt")):
+        words = line.split("#")[0].split()
+        if not words:
+            continue
+        v = [int(x, 16) for x in words]
+        assert list(oracle.philox4x32_10(v[0:4], v[4:6])) == v[6:10]
+        n += 1
+    assert n == 3
+
+
+def test_policy_uniforms_are_uniform_and_uncorrelated():
+    """Kolmogorov-Smirnov against U(0, 1); neighbouring groups (words of one
+    generator call) and neighbouring queries are uncorrelated; the seed and
+    the offset change the stream."""
+    from scipy import stats
+
+    u = np.array([[oracle.policy_uniform(7, 3, b, g) for g in range(64)] for b in range(400)])
+    assert (u > 0).all() and (u < 1).all()
+    assert stats.kstest(u.ravel(), "uniform").pvalue > 1e-4
+    assert abs(np.corrcoef(u[:, :-1].ravel(), u[:, 1:].ravel())[0, 1]) < 0.02
+    assert abs(np.corrcoef(u[:-1].ravel(), u[1:].ravel())[0, 1]) < 0.02
+    assert oracle.policy_uniform(8, 3, 0, 0) != u[0, 0]
+    assert oracle.policy_uniform(7, 4, 0, 0) != u[0, 0]
+    assert oracle.policy_uniform(7, 3 + (1 << 32), 0, 0) != u[0, 0]
+
+
+def _policy_case(B, eps, tau, seed=11):
+    scores = np.tile(np.array([0.3, -0.2, 0.9, 0.1, 0.5, 0.0]), (B, 1))
+    counts = np.array([3, 2, 4, 0, 1, 5], dtype=np.int64)
+    keys, mu = oracle.policy_keys(scores, counts, tau, eps, seed, 0)
+    ne = counts > 0
+    from scipy.special import softmax
+
+    p = np.zeros(6)
+    p[ne] = eps / ne.sum() + (1 - eps) * softmax(scores[0][ne] / tau)
+    return scores, counts, keys, mu, p
+
+
+@pytest.mark.parametrize("eps,tau", [(0.2, 0.4), (0.0, 1.0), (1.0, 0.3)])
+def test_first_draw_follows_the_policy(eps, tau):
+    """mu equals Eq. 11 by scipy's softmax over the non-empty groups, and the
+    group with the largest key (the first draw) has that distribution
+    (chi-square over 40,000 independent queries); the empty group never."""
+    from scipy import stats
+
+    B = 40000
+    _, counts, keys, mu, p = _policy_case(B, eps, tau)
+    np.testing.assert_allclose(mu[0], p, rtol=1e-12, atol=0)
+    first = keys.argmax(axis=1)
+    obs = np.bincount(first, minlength=6)
+    assert obs[3] == 0
+    ne = counts > 0
+    assert stats.chisquare(obs[ne], B * p[ne]).pvalue > 1e-4
+
+
+def test_second_draw_is_without_replacement():
+    """The second-largest key follows P(second = j) = sum_{i != j} p_i p_j / (1 - p_i),
+    the law of a second draw without replacement."""
+    from scipy import stats
+
+    B = 40000
+    _, counts, keys, mu, p = _policy_case(B, 0.1, 0.5, seed=5)
+    order = np.argsort(-keys, axis=1, kind="stable")
+    assert (order[:, 0] != order[:, 1]).all()
+    q = np.array([sum(p[i] * p[j] / (1 - p[i]) for i in range(6) if i != j and p[i] > 0) for j in range(6)])
+    np.testing.assert_allclose(q.sum(), 1.0, rtol=1e-12)
+    obs = np.bincount(order[:, 1], minlength=6)
+    ne = counts > 0
+    assert obs[3] == 0
+    assert stats.chisquare(obs[ne], B * q[ne]).pvalue > 1e-4
+
+
+def test_cold_policy_draws_the_top_groups():
+    """With a tiny temperature and no exploration the noise cannot reorder
+    groups whose scores differ by much more than tau, so the draws are
+    stage 1's ranking."""
+    rng = np.random.default_rng(9)
+    B, G, k = 50, 40, 6
+    scores = rng.permutation(G)[None, :].repeat(B, 0) * 0.1 + rng.standard_normal((B, 1))
+    counts = np.ones(G, dtype=np.int64)
+    counts[[3, 17]] = 0
+    keys, _ = oracle.policy_keys(scores, counts, 1e-3, 0.0, 3, 1)
+    gi, _ = oracle.select(keys, counts, k)
+    ref, _ = oracle.select(scores, counts, k)
+    assert (gi == ref).all()

@@ -6,7 +6,9 @@ the tie order reversed, the mean not divided by n_g, the ranking sign flipped,
 a transposed operand, a leak of entries outside the selected groups, empty
 groups allowed into stage 1, prefix weights reversed, of the wrong sign or
 missing the newest element, edge-table rows and columns swapped, an edge
-feature misread, edge-prefix weights reversed), builds it there and runs ``test_oracle.py``
+feature misread, edge-prefix weights reversed, Philox words swapped or its key
+not advanced, one uniform shared by four groups, the policy's eps term dropped
+or tau ignored, the Gumbel noise of the wrong sign, empty groups drawn), builds it there and runs ``test_oracle.py``
 against the mutant: at least one pin has to fail.
 """
 import os
@@ -38,6 +40,13 @@ MUTANTS = {
     "edge_feature_misread": ("phi += w[f] * (double)z[f];", "phi += w[f] * (double)z[(f + 1) % F];"),
     "edge_weights_reversed": ("const double alpha = exp(-lambda * (double)(p_len - i));\n      for (int32_t g",
                               "const double alpha = exp(-lambda * (double)(i - 1));\n      for (int32_t g"),
+    "philox_words_swapped": ("c[1] = n1;\n    c[2] = n2;\n    c[3] = n3;", "c[1] = n3;\n    c[2] = n2;\n    c[3] = n1;"),
+    "philox_key_not_advanced": ("k1 += kPhiloxWeyl1;", "k1 += 0;"),
+    "uniform_word_fixed": ("out[g & 3] >> 9", "out[0] >> 9"),
+    "policy_eps_dropped": ("mu[o] = eps / (double)n + (1.0 - eps)", "mu[o] = (1.0 - eps)"),
+    "policy_tau_ignored": ("if (counts[g] > 0) sum += exp(s[g] / tau - m);", "if (counts[g] > 0) sum += exp(s[g] - m);"),
+    "gumbel_sign_flipped": ("keys[o] = log_mu - log(-log(u));", "keys[o] = log_mu + log(-log(u));"),
+    "policy_empty_groups_drawn": ("      if (counts[g] == 0) {\n        mu[o] = 0.0;", "      if (0) {\n        mu[o] = 0.0;"),
 }
 
 
@@ -51,6 +60,7 @@ def test_pins_catch_planted_mistake(name, tmp_path):
     (tmp_path / "oracle" / "htam_oracle.c").write_text(src.replace(before, after))
     shutil.copy(os.path.join(ROOT, "oracle", "__init__.py"), tmp_path / "oracle" / "__init__.py")
     shutil.copy(os.path.join(ROOT, "tests", "test_oracle.py"), tmp_path / "tests" / "test_oracle.py")
+    shutil.copytree(os.path.join(ROOT, "tests", "golden"), tmp_path / "tests" / "golden")
     (tmp_path / "pytest.ini").write_text("[pytest]\naddopts = -p no:cacheprovider\n")
     env = dict(os.environ, PYTHONPATH=str(tmp_path))
     r = subprocess.run([sys.executable, "-m", "pytest", "-q", "-x", "tests/test_oracle.py"],
