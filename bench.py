@@ -66,6 +66,9 @@ def parse_args():
     ap.add_argument("--edge-features", type=int, default=12, help="features per edge (12 in App. B.6)")
     ap.add_argument("--flat", action="store_true",
                     help="flat scan (htam_query_flat): every entry a candidate, no group stage")
+    ap.add_argument("--sample", action="store_true",
+                    help="draw the groups from the policy of Eq. 11 (htam_query_sampled / "
+                         "htam_query_edges_sampled) instead of ranking them")
     ap.add_argument("--tc-min-bucket", type=int, default=None,
                     help="smallest bucket scored on the tensor cores (library default 16)")
     return ap.parse_args()
@@ -249,7 +252,7 @@ def make_workload(w, seed, device, rank):
     return entries, gid, centres
 
 
-def oracle_rate(w, entries_np, gid_np, queries_np, target_s, cent=None, counts=None, flat=False):
+def oracle_rate(w, entries_np, gid_np, queries_np, target_s, cent=None, counts=None, flat=False, sample=False):
     """Times the oracle (as it stands) on a bounded sample of the queries."""
     import oracle
 
@@ -260,6 +263,9 @@ def oracle_rate(w, entries_np, gid_np, queries_np, target_s, cent=None, counts=N
     def call(q):
         if flat:
             oracle.flat(entries_np, q, w.k_entries, nthreads=threads)
+        elif sample:
+            oracle.query_sampled(entries_np, gid_np, w.g, q, w.k_groups, w.k_entries, 1.0, 0.0, 0, 0,
+                                 centroid=cent, counts=counts, nthreads=threads)
         else:
             oracle.query(entries_np, gid_np, w.g, q, w.k_groups, w.k_entries, centroid=cent, counts=counts,
                          nthreads=threads)
@@ -373,7 +379,11 @@ def run_htam(args, world, rank, local):
             return mem.query_flat(q, w.k_entries, out=out)
         if E > 0:
             return mem.query_edges(edge_z, edge_w, edge_prefix[batch_of.get(id(q), 0)], args.prefix_lambda, q,
-                                   w.k_groups, w.k_entries, out=out)
+                                   w.k_groups, w.k_entries, out=out,
+                                   sampling=(args.seed, batch_of.get(id(q), 0)) if args.sample else None)
+        if args.sample:
+            return mem.query_sampled(q, w.k_groups, w.k_entries, seed=args.seed, offset=batch_of.get(id(q), 0),
+                                     out=out)
         if P > 0:
             return mem.query_prefix(q, args.prefix_lambda, w.k_groups, w.k_entries, out=out)
         return mem.query(q, w.k_groups, w.k_entries, out=out)
@@ -479,7 +489,7 @@ def run_htam(args, world, rank, local):
     host_q = [b.cpu().pin_memory() for b in batches]
     e2e_steps = max(3, min(args.steps, 50))
     s_elem = 2 if w.dtype == "bf16" else 4
-    if P > 0 or E > 0 or args.flat:
+    if P > 0 or E > 0 or args.flat or args.sample:
         # No host-buffer entry point for these lookups: pinned copies on the
         # stream around the call, outputs read back every step.
         dev_q = torch.empty_like(batches[0])
@@ -493,7 +503,8 @@ def run_htam(args, world, rank, local):
             for k in host_out:
                 host_out[k].copy_(o[k], non_blocking=True)
             torch.cuda.current_stream().synchronize()
-        entry = "htam_query_flat" if args.flat else "htam_query_edges" if E > 0 else "htam_query_prefix"
+        entry = ("htam_query_flat" if args.flat else "htam_query_edges" + ("_sampled" if args.sample else "")
+                 if E > 0 else "htam_query_sampled" if args.sample else "htam_query_prefix")
         path = f"pinned host queries copied in, {entry}, outputs copied out (torch copies on the stream)"
     else:
         host_out = mem.query_host(host_q[0], w.k_groups, w.k_entries)
@@ -549,7 +560,10 @@ def run_htam(args, world, rank, local):
             rate = n / dt
             note = ", edge-routed (float64 edge scores over the same table)"
         else:
-            rate, n, dt, threads, _, _ = oracle_rate(w, entries_np, gid_np, q_np, args.cpu_seconds)
+            rate, n, dt, threads, _, _ = oracle_rate(w, entries_np, gid_np, q_np, args.cpu_seconds,
+                                                     sample=args.sample)
+            if args.sample:
+                note += ", groups drawn from the policy"
         cpu = {"value": rate, "unit": UNIT, "cores": threads, "kind": "oracle",
                "sample": f"{n} queries of {w.name} ({dt:.1f} s), float64 brute force over the same memory"
                          + ("" if args.flat else ", group keys precomputed") + note}
@@ -563,6 +577,7 @@ def run_htam(args, world, rank, local):
                        "k_groups": w.k_groups, "k_entries": w.k_entries, "query_batches": len(batches),
                        "mean_candidates_per_query": float(np.mean([x["mean_candidates"] for x in work])),
                        **({"flat": True} if args.flat else {}),
+                       **({"sampled_groups": True} if args.sample else {}),
                        "l2": ("flushed between steps (2x L2 buffer write, outside the step events)" if flush_l2 else
                               f"inputs larger than L2 ({work[0]['step_bytes'] / 1e9:.2f} GB touched per step)"),
                        "parallelism": f"replicas{world}" if world > 1 else "single GPU",

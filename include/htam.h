@@ -180,6 +180,45 @@ htam_status htam_query_edges(htam_memory *m, const float *edge_features, int32_t
                              int32_t *entry_idx, float *entry_score, float *entry_weight,
                              float *lse, void *cuda_stream);
 
+/* Seed and counter offset of the policy draws below.  The draws of query i
+ * of a batch depend only on (seed, offset, i, group); pass a new offset (a
+ * step counter, say) for fresh draws. */
+typedef struct {
+  uint64_t seed;
+  uint64_t offset;
+} htam_sampling;
+
+/* Lookup with the groups DRAWN from the global-direction policy instead of
+ * ranked (Algorithm 1, step 2: g_t ~ mu_g of Eq. 11):
+ *   mu_g = epsilon / |G_t| + (1 - epsilon) * softmax(s_g / tau) over the
+ *   non-empty groups G_t, s_g = q . c_g, tau and epsilon from `p`.
+ * k_groups draws without replacement (k_groups = 1 is the paper's single
+ * draw): the groups with the k_groups largest keys log mu_g - log(-log u_g)
+ * (the Gumbel-top-k construction, Kool, van Hoof and Welling, ICML 2019),
+ * ties to the lower id.  u_g is the query's uniform for group g: word (g mod 4)
+ * of Philox4x32-10 (Salmon et al., SC 2011) at counter (g / 4, i, low and high
+ * words of offset) under key (low and high words of seed), its top 23 bits
+ * plus one half times 2^-23.  group_idx lists the draws in order and
+ * group_score holds their scores q . c_g; stage 2 and every other output are
+ * those of htam_query over the drawn groups.  Arguments, asynchrony and
+ * errors as htam_query (EINVAL also for sampling == NULL). */
+htam_status htam_query_sampled(htam_memory *m, const void *queries, int32_t b,
+                               const htam_query_params *p, const htam_sampling *sampling,
+                               int32_t *group_idx, float *group_score, int32_t *entry_idx,
+                               float *entry_score, float *entry_weight, float *lse,
+                               void *cuda_stream);
+
+/* htam_query_edges with the groups drawn from the policy of Eq. 11 over the
+ * edge-table scores of Eq. 9, as htam_query_sampled draws them (the paper's
+ * global direction choice as Algorithm 1 states it). */
+htam_status htam_query_edges_sampled(htam_memory *m, const float *edge_features, int32_t n_features,
+                                     const float *weights, const int32_t *prefix_groups, int32_t p_len,
+                                     float lambda, const void *queries, int32_t b,
+                                     const htam_query_params *p, const htam_sampling *sampling,
+                                     int32_t *group_idx, float *group_score, int32_t *entry_idx,
+                                     float *entry_score, float *entry_weight, float *lse,
+                                     void *cuda_stream);
+
 /* Flat scan: stage 2 of the lookup with every entry a candidate, no group
  * stage.  This is the flat memory retrieval the paper compares against
  * (App. C.4, and the "w/o hierarchy" ablation of App. C.8); its result equals

@@ -72,7 +72,8 @@ def _load():
         lib.htam_oracle_philox4x32_10.restype = None
         lib.htam_oracle_policy_uniform.argtypes = [ctypes.c_uint64, ctypes.c_uint64, i32, i32]
         lib.htam_oracle_policy_uniform.restype = dbl
-        lib.htam_oracle_policy_keys.argtypes = [P, P, i32, i32, dbl, dbl, ctypes.c_uint64, ctypes.c_uint64, P, P]
+        lib.htam_oracle_policy_keys.argtypes = [P, P, i32, i32, dbl, dbl, ctypes.c_uint64, ctypes.c_uint64, P, P,
+                                                P]
         lib.htam_oracle_policy_keys.restype = ctypes.c_int
         _lib = lib
         return lib
@@ -310,17 +311,22 @@ def coarse_scores(queries: np.ndarray, centroid: np.ndarray) -> np.ndarray:
     return _as_f64_input(queries) @ np.asarray(centroid, dtype=np.float64).T
 
 
-def policy_keys(scores: np.ndarray, counts: np.ndarray, tau: float, eps: float, seed: int, offset: int):
+def policy_keys(scores: np.ndarray, counts: np.ndarray, tau: float, eps: float, seed: int, offset: int,
+                query_ids=None):
     """Gumbel-top-k keys of the Eq. 11 policy over the non-empty groups and
-    the policy itself: returns (keys, mu), both [b, G] float64."""
+    the policy itself: returns (keys, mu), both [b, G] float64.  Row r draws
+    with the uniforms of query query_ids[r] (default r)."""
     lib = _load()
     scores = np.ascontiguousarray(scores, dtype=np.float64)
     counts = np.ascontiguousarray(counts, dtype=np.int64)
     b, G = scores.shape
+    ids = None if query_ids is None else np.ascontiguousarray(query_ids, dtype=np.int32)
+    if ids is not None and ids.shape != (b,):
+        raise ValueError("query_ids must have one id per row")
     keys = np.empty((b, G), dtype=np.float64)
     mu = np.empty((b, G), dtype=np.float64)
     rc = lib.htam_oracle_policy_keys(_ptr(scores), _ptr(counts), b, G, float(tau), float(eps), int(seed),
-                                     int(offset), _ptr(keys), _ptr(mu))
+                                     int(offset), _ptr(ids) if ids is not None else None, _ptr(keys), _ptr(mu))
     if rc != 0:
         raise ValueError("oracle policy_keys: bad argument")
     return keys, mu

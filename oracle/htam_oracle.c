@@ -507,9 +507,12 @@ double htam_oracle_policy_uniform(uint64_t seed, uint64_t offset, int32_t b, int
  * with the largest keys (ties to the lower id) are k draws without
  * replacement from mu, in draw order: the Gumbel-top-k construction (Kool, van
  * Hoof and Welling, ICML 2019; k = 1 is the Gumbel-max draw of g_t ~ mu).
- * Returns 0, or -1 on a bad argument. */
+ * Row b uses the uniforms of query query_ids[b] (of query b when query_ids
+ * is NULL), so that a sample of a batch's rows draws what the whole batch
+ * draws.  Returns 0, or -1 on a bad argument. */
 int htam_oracle_policy_keys(const double *scores, const int64_t *counts, int32_t n_queries, int32_t G, double tau,
-                            double eps, uint64_t seed, uint64_t offset, double *keys, double *mu) {
+                            double eps, uint64_t seed, uint64_t offset, const int32_t *query_ids, double *keys,
+                            double *mu) {
   if (G < 1 || n_queries < 0 || !(tau > 0.0) || !(eps >= 0.0 && eps <= 1.0)) return -1;
   int64_t n = 0;
   for (int32_t g = 0; g < G; ++g) n += counts[g] > 0;
@@ -533,7 +536,7 @@ int htam_oracle_policy_keys(const double *scores, const int64_t *counts, int32_t
       }
       mu[o] = eps / (double)n + (1.0 - eps) * exp(s[g] / tau - lse);
       const double log_mu = eps == 0.0 ? s[g] / tau - lse : log(mu[o]);
-      const double u = htam_oracle_policy_uniform(seed, offset, b, g);
+      const double u = htam_oracle_policy_uniform(seed, offset, query_ids ? query_ids[b] : b, g);
       keys[o] = log_mu - log(-log(u));
     }
   }

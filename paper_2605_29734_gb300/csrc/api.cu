@@ -170,10 +170,23 @@ htam_status htam_query_prefix(htam_memory *m, const void *prefix, int32_t b, int
                     st);
 }
 
-htam_status htam_query_edges(htam_memory *m, const float *edge_features, int32_t n_features, const float *weights,
-                             const int32_t *prefix_groups, int32_t p_len, float lambda, const void *queries, int32_t b,
-                             const htam_query_params *p, int32_t *group_idx, float *group_score, int32_t *entry_idx,
-                             float *entry_score, float *entry_weight, float *lse, void *cuda_stream) {
+htam_status htam_query_sampled(htam_memory *m, const void *queries, int32_t b, const htam_query_params *p,
+                               const htam_sampling *sampling, int32_t *group_idx, float *group_score,
+                               int32_t *entry_idx, float *entry_score, float *entry_weight, float *lse,
+                               void *cuda_stream) {
+  htam_status s = check_query_args(m, queries, b, p, group_idx, group_score, entry_idx, entry_score, entry_weight);
+  if (s != HTAM_OK) return s;
+  if (!sampling || (b > 0 && !aligned16(queries))) return HTAM_EINVAL;
+  const SampleSpec smp{sampling->seed, sampling->offset};
+  return query_impl(m, queries, b, *p, group_idx, group_score, entry_idx, entry_score, entry_weight, lse,
+                    static_cast<cudaStream_t>(cuda_stream), nullptr, false, &smp);
+}
+
+static htam_status query_edges_impl(htam_memory *m, const float *edge_features, int32_t n_features,
+                                    const float *weights, const int32_t *prefix_groups, int32_t p_len, float lambda,
+                                    const void *queries, int32_t b, const htam_query_params *p, int32_t *group_idx,
+                                    float *group_score, int32_t *entry_idx, float *entry_score,
+                                    float *entry_weight, float *lse, void *cuda_stream, const SampleSpec *smp) {
   htam_status s = check_query_args(m, queries, b, p, group_idx, group_score, entry_idx, entry_score, entry_weight);
   if (s != HTAM_OK) return s;
   if (b > 0 && !aligned16(queries)) return HTAM_EINVAL;
@@ -200,7 +213,27 @@ htam_status htam_query_edges(htam_memory *m, const float *edge_features, int32_t
     er.alpha[i] = i < p_len ? (float)std::exp(-(double)lambda * (double)(p_len - 1 - i)) : 0.f;
   }
   return query_impl(m, queries, b, *p, group_idx, group_score, entry_idx, entry_score, entry_weight, lse,
-                    static_cast<cudaStream_t>(cuda_stream), &er);
+                    static_cast<cudaStream_t>(cuda_stream), &er, false, smp);
+}
+
+htam_status htam_query_edges(htam_memory *m, const float *edge_features, int32_t n_features, const float *weights,
+                             const int32_t *prefix_groups, int32_t p_len, float lambda, const void *queries, int32_t b,
+                             const htam_query_params *p, int32_t *group_idx, float *group_score, int32_t *entry_idx,
+                             float *entry_score, float *entry_weight, float *lse, void *cuda_stream) {
+  return query_edges_impl(m, edge_features, n_features, weights, prefix_groups, p_len, lambda, queries, b, p,
+                          group_idx, group_score, entry_idx, entry_score, entry_weight, lse, cuda_stream, nullptr);
+}
+
+htam_status htam_query_edges_sampled(htam_memory *m, const float *edge_features, int32_t n_features,
+                                     const float *weights, const int32_t *prefix_groups, int32_t p_len,
+                                     float lambda, const void *queries, int32_t b, const htam_query_params *p,
+                                     const htam_sampling *sampling, int32_t *group_idx, float *group_score,
+                                     int32_t *entry_idx, float *entry_score, float *entry_weight, float *lse,
+                                     void *cuda_stream) {
+  if (!sampling) return HTAM_EINVAL;
+  const SampleSpec smp{sampling->seed, sampling->offset};
+  return query_edges_impl(m, edge_features, n_features, weights, prefix_groups, p_len, lambda, queries, b, p,
+                          group_idx, group_score, entry_idx, entry_score, entry_weight, lse, cuda_stream, &smp);
 }
 
 htam_status htam_query_flat(htam_memory *m, const void *queries, int32_t b, int32_t k_entries, float tau,

@@ -108,10 +108,15 @@ struct EdgeRoute {
   float w[HTAM_MAX_EDGE_FEATURES];
   float alpha[HTAM_MAX_PREFIX];
 };
+// Seed and counter offset of the policy draws (Algorithm 1, step 2).
+struct SampleSpec {
+  uint64_t seed, offset;
+};
 htam_status query_impl(htam_memory *m, const void *queries, int32_t b,
                        const htam_query_params &p, int32_t *group_idx, float *group_score,
                        int32_t *entry_idx, float *entry_score, float *entry_weight, float *lse,
-                       cudaStream_t st, const EdgeRoute *er = nullptr, bool flat = false);
+                       cudaStream_t st, const EdgeRoute *er = nullptr, bool flat = false,
+                       const SampleSpec *smp = nullptr);
 // Largest b * (non-empty groups) the flat scan takes (its bucket rows).
 constexpr int64_t kMaxFlatRows = int64_t(1) << 28;
 void free_impl(htam_memory *m);

@@ -275,6 +275,123 @@ __global__ void __launch_bounds__(256) edge_scores_kernel(EdgeKernelArgs a, int 
   s1[t] = acc;
 }
 
+// ------------------------------------------------------- policy draws (Eq. 11)
+
+// Philox4x32-10 (Salmon, Moraes, Dror and Shaw, SC 2011): ten rounds of two
+// 32x32 -> 64-bit products of counter words 0 and 2, mixed with the other
+// words and the key; the key advances by two Weyl increments between rounds.
+__device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint2 k) {
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    if (r > 0) {
+      k.x += 0x9E3779B9u;
+      k.y += 0xBB67AE85u;
+    }
+    const uint32_t p0_hi = __umulhi(0xD2511F53u, c.x), p0_lo = 0xD2511F53u * c.x;
+    const uint32_t p1_hi = __umulhi(0xCD9E8D57u, c.z), p1_lo = 0xCD9E8D57u * c.z;
+    c = make_uint4(p1_hi ^ c.y ^ k.x, p1_lo, p0_hi ^ c.w ^ k.y, p0_lo);
+  }
+  return c;
+}
+
+struct PolicyArgs {
+  const float *s1;  // [planes, B, G] scores, summed over the planes in order
+  int planes, B, G;
+  const int32_t *count;
+  int n_nonempty;   // |G_t|
+  float inv_tau, eps;
+  uint2 key;        // seed words
+  uint32_t off_lo, off_hi;
+  float *keys;      // [B, G] out
+};
+
+__device__ __forceinline__ float block_reduce(float v, bool is_max, float *red) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float w = __shfl_xor_sync(kFullMask, v, o);
+    v = is_max ? fmaxf(v, w) : v + w;
+  }
+  __syncthreads();  // the previous reduction's readers are done with red
+  if (lane == 0) red[warp] = v;
+  __syncthreads();
+  v = red[0];
+  for (int w = 1; w < (int)(blockDim.x >> 5); ++w) v = is_max ? fmaxf(v, red[w]) : v + red[w];
+  return v;
+}
+
+// One block per query: the Gumbel-top-k keys of the policy of Eq. 11 over the
+// non-empty groups, key_g = log mu_g - log(-log u_g), with mu_g = eps / |G_t|
+// + (1 - eps) softmax(s / tau)_g and u_g the query's Philox uniform for g
+// (word g mod 4 of the counter (g / 4, b, offset); top 23 bits plus one half,
+// times 2^-23).  The k largest keys are k draws without replacement from
+// mu (Kool, van Hoof and Welling, ICML 2019).  Empty groups get -inf.
+__global__ void __launch_bounds__(256) policy_keys_kernel(PolicyArgs a) {
+  __shared__ float red[32];
+  const int b = blockIdx.x;
+  const int64_t plane = (int64_t)a.B * a.G;
+  const float *src = a.s1 + (int64_t)b * a.G;
+  float *keys = a.keys + (int64_t)b * a.G;
+  // Scores (summed over the planes) into the key row, and their maximum.
+  float m = -INFINITY;
+  for (int g = threadIdx.x; g < a.G; g += blockDim.x) {
+    float s = src[g];
+    for (int p = 1; p < a.planes; ++p) s += src[p * plane + g];
+    keys[g] = s;
+    if (a.count[g] > 0) m = fmaxf(m, s * a.inv_tau);
+  }
+  m = block_reduce(m, true, red);
+  float sum = 0.f;
+  for (int g = threadIdx.x; g < a.G; g += blockDim.x) {
+    if (a.count[g] > 0) sum += expf(keys[g] * a.inv_tau - m);
+  }
+  sum = block_reduce(sum, false, red);
+  const float lse = m + logf(sum);
+  const float log_unif = a.eps > 0.f ? logf(a.eps / (float)a.n_nonempty) : -INFINITY;
+  const float log_soft = a.eps < 1.f ? log1pf(-a.eps) : -INFINITY;
+  for (int q = threadIdx.x; q * 4 < a.G; q += blockDim.x) {
+    const uint4 r = philox4x32_10(make_uint4((uint32_t)q, (uint32_t)b, a.off_lo, a.off_hi), a.key);
+    const uint32_t w[4] = {r.x, r.y, r.z, r.w};
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int g = q * 4 + j;
+      if (g >= a.G) break;
+      if (a.count[g] == 0) {
+        keys[g] = -INFINITY;
+        continue;
+      }
+      const float z = keys[g] * a.inv_tau - lse;
+      float log_mu;
+      if (a.eps == 0.f) {
+        log_mu = z;
+      } else {
+        const float c = log_soft + z;
+        const float hi = fmaxf(log_unif, c), lo = fminf(log_unif, c);
+        log_mu = hi + log1pf(expf(lo - hi));
+      }
+      const float u = ((float)(w[j] >> 9) + 0.5f) * (1.0f / 8388608.0f);
+      keys[g] = log_mu - logf(-logf(u));
+    }
+  }
+}
+
+// The drawn groups' scores: group_score[b][j] = s[b][group_idx[b][j]]
+// (planes summed in order, as the selection sums them), -inf for padding.
+__global__ void policy_scores_kernel(const float *__restrict__ s1, int planes, int B, int G, int kg,
+                                     const int32_t *__restrict__ group_idx, float *__restrict__ group_score) {
+  const int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  if (t >= (int64_t)B * kg) return;
+  const int g = group_idx[t];
+  const int64_t b = t / kg;
+  float s = -INFINITY;
+  if (g >= 0) {
+    const int64_t plane = (int64_t)B * G;
+    s = s1[b * G + g];
+    for (int p = 1; p < planes; ++p) s += s1[p * plane + b * G + g];
+  }
+  group_score[t] = s;
+}
+
 // ---------------------------------------------------------------- flat scan
 
 // The ascending list of non-empty groups (one block, 1024 groups per pass).
@@ -1019,14 +1136,14 @@ constexpr uint32_t kMaxPolls = 1u << 24;
 htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const htam_query_params &p,
                        int32_t *group_idx, float *group_score, int32_t *entry_idx,
                        float *entry_score, float *entry_weight, float *lse, cudaStream_t st,
-                       const EdgeRoute *er, bool flat) {
+                       const EdgeRoute *er, bool flat, const SampleSpec *smp) {
   if (B == 0) return HTAM_OK;
   m->n_queries += 1;
   PhaseMark mark(m, st);
   // The flat scan selects every non-empty group (at least one slot, -1 when
   // the memory is empty); the group lists then live in the scratch.
   int n_nonempty = 0;
-  if (flat) {
+  if (flat || smp) {
     for (int64_t c : m->h_count) n_nonempty += c > 0;
   }
   const int G = m->n_groups, d = m->d, kg = flat ? std::max(1, n_nonempty) : p.k_groups, ke = p.k_entries;
@@ -1067,7 +1184,7 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
                 3 * Carver::round(sizeof(int32_t) * rows) + 2 * Carver::round(sizeof(int4) * max_units) +
                 Carver::round(sizeof(float2) * max_parts) + Carver::round(sizeof(float) * max_parts * ke) +
                 Carver::round(sizeof(int32_t) * max_parts * ke) + Carver::round(sizeof(unsigned) * B) +
-                Carver::round(qg_bytes) + (flat ? Carver::round(sizeof(int32_t) * rows) + Carver::round(sizeof(int32_t) * kg) : 0) + 8192;
+                Carver::round(qg_bytes) + (smp ? Carver::round(sizeof(float) * (size_t)B * G) : 0) + (flat ? Carver::round(sizeof(int32_t) * rows) + Carver::round(sizeof(int32_t) * kg) : 0) + 8192;
   htam_status s = ensure_scratch(m, need);
   if (s != HTAM_OK) return s;
   Carver cv(m->scratch);
@@ -1094,6 +1211,7 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   int32_t *part_id = cv.take<int32_t>(max_parts * ke);
   unsigned *thr_enc = cv.take<unsigned>(B);
   void *qg = tc_ok && !flat ? static_cast<void *>(cv.take<char>(qg_bytes)) : nullptr;
+  float *policy_keys = smp ? cv.take<float>((size_t)B * G) : nullptr;
   if (flat) {
     group_idx = cv.take<int32_t>(rows);
     int32_t *list = cv.take<int32_t>(kg);  // the non-empty groups, ascending
@@ -1149,15 +1267,38 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
     mark.launched();
     mark.end();
     mark.begin(HTAM_PHASE_SELECT);
+    // Drawn groups (Algorithm 1, step 2): the top k_g of the policy keys.
+    const float *sel = s1;
+    int sel_planes = planes;
+    if (smp) {
+      if (n_nonempty > 0) {
+        PolicyArgs pa{s1, planes, B, G, m->count, n_nonempty, 1.0f / p.tau, p.epsilon,
+                      make_uint2((uint32_t)smp->seed, (uint32_t)(smp->seed >> 32)), (uint32_t)smp->offset,
+                      (uint32_t)(smp->offset >> 32), policy_keys};
+        policy_keys_kernel<<<(unsigned)B, 256, 0, st>>>(pa);
+        HTAM_CK_LAUNCH("policy_keys_kernel");
+        mark.launched();
+      } else {
+        HTAM_CK(cudaMemsetAsync(policy_keys, 0, sizeof(float) * (size_t)B * G, st));  // all groups empty
+      }
+      sel = policy_keys;
+      sel_planes = 1;
+    }
     if (wpq == 8) {
-      group_topk_kernel<8><<<(unsigned)B, kSelWarps * 32, 0, st>>>(s1, planes, B, G, m->count, kg, group_idx,
+      group_topk_kernel<8><<<(unsigned)B, kSelWarps * 32, 0, st>>>(sel, sel_planes, B, G, m->count, kg, group_idx,
                                                                    group_score);
     } else {
       group_topk_kernel<1><<<(unsigned)ceil_div(B, kSelWarps), kSelWarps * 32, 0, st>>>(
-          s1, planes, B, G, m->count, kg, group_idx, group_score);
+          sel, sel_planes, B, G, m->count, kg, group_idx, group_score);
     }
     HTAM_CK_LAUNCH("group_topk_kernel");
     mark.launched();
+    if (smp) {
+      policy_scores_kernel<<<(unsigned)ceil_div((int64_t)B * kg, 256), 256, 0, st>>>(s1, planes, B, G, kg,
+                                                                                   group_idx, group_score);
+      HTAM_CK_LAUNCH("policy_scores_kernel");
+      mark.launched();
+    }
     mark.end();
   }
 

@@ -24,7 +24,7 @@ HTAM_MAX_EDGE_FEATURES = 32  # most features per edge htam_query_edges takes
 # Every symbol include/htam.h declares, in declaration order.
 EXPORTS = (
     "htam_build_memory", "htam_append_transitions", "htam_query", "htam_query_host", "htam_query_prefix",
-    "htam_query_edges", "htam_query_flat",
+    "htam_query_edges", "htam_query_flat", "htam_query_sampled", "htam_query_edges_sampled",
     "htam_select_groups_static", "htam_memory_info", "htam_memory_group_counts", "htam_memory_group_keys",
     "htam_device_status", "htam_set_tuning", "htam_get_tuning", "htam_set_phase_timing",
     "htam_read_phase_timing", "htam_free_memory", "htam_status_string", "htam_last_error",
@@ -46,6 +46,10 @@ class QueryParams(ctypes.Structure):
                 ("tau", ctypes.c_float), ("epsilon", ctypes.c_float)]
 
 
+class Sampling(ctypes.Structure):
+    _fields_ = [("seed", ctypes.c_uint64), ("offset", ctypes.c_uint64)]
+
+
 def _load() -> ctypes.CDLL:
     if not os.path.exists(LIB_PATH):
         raise ImportError(f"{LIB_PATH} is missing: build it with paper_2605_29734_gb300.build.build()")
@@ -61,6 +65,11 @@ def _load() -> ctypes.CDLL:
                                       P, P, P, P, P, P, P]
     lib.htam_query_edges.argtypes = [P, P, i32, P, P, i32, ctypes.c_float, P, i32, ctypes.POINTER(QueryParams),
                                      P, P, P, P, P, P, P]
+    lib.htam_query_sampled.argtypes = [P, P, i32, ctypes.POINTER(QueryParams), ctypes.POINTER(Sampling),
+                                       P, P, P, P, P, P, P]
+    lib.htam_query_edges_sampled.argtypes = [P, P, i32, P, P, i32, ctypes.c_float, P, i32,
+                                             ctypes.POINTER(QueryParams), ctypes.POINTER(Sampling),
+                                             P, P, P, P, P, P, P]
     lib.htam_query_flat.argtypes = [P, P, i32, i32, ctypes.c_float, ctypes.c_float, P, P, P, P, P]
     lib.htam_memory_info.argtypes = [P, P, P, P, P]
     lib.htam_memory_group_counts.argtypes = [P, P]
@@ -159,6 +168,30 @@ class Memory:
     def query(self, queries: torch.Tensor, k_groups: int, k_entries: int, tau: float = 1.0,
               epsilon: float = 0.0, stream=None, out: dict | None = None) -> dict:
         """Device lookup; returns (or fills) a dict of device tensors."""
+        b, out = self._lookup_out(queries, k_groups, k_entries, out)
+        p = QueryParams(k_groups, k_entries, tau, epsilon)
+        _check(_lib.htam_query(self.handle, _dev_ptr(queries), b, ctypes.byref(p),
+                               _dev_ptr(out["group_idx"]), _dev_ptr(out["group_score"]),
+                               _dev_ptr(out["entry_idx"]), _dev_ptr(out["entry_score"]),
+                               _dev_ptr(out["entry_weight"]), _dev_ptr(out.get("lse")),
+                               _stream_ptr(stream)), "htam_query")
+        return out
+
+    def query_sampled(self, queries: torch.Tensor, k_groups: int, k_entries: int, seed: int, offset: int,
+                      tau: float = 1.0, epsilon: float = 0.0, stream=None, out: dict | None = None) -> dict:
+        """Lookup with the groups drawn from the policy of Eq. 11 (k_groups
+        draws without replacement; Philox uniforms from seed and offset)."""
+        b, out = self._lookup_out(queries, k_groups, k_entries, out)
+        p = QueryParams(k_groups, k_entries, tau, epsilon)
+        smp = Sampling(seed, offset)
+        _check(_lib.htam_query_sampled(self.handle, _dev_ptr(queries), b, ctypes.byref(p), ctypes.byref(smp),
+                                       _dev_ptr(out["group_idx"]), _dev_ptr(out["group_score"]),
+                                       _dev_ptr(out["entry_idx"]), _dev_ptr(out["entry_score"]),
+                                       _dev_ptr(out["entry_weight"]), _dev_ptr(out.get("lse")),
+                                       _stream_ptr(stream)), "htam_query_sampled")
+        return out
+
+    def _lookup_out(self, queries: torch.Tensor, k_groups: int, k_entries: int, out: dict | None):
         if queries.dtype != self.dtype or queries.dim() != 2 or queries.shape[1] != self.d:
             raise ValueError("queries must be [b, d] of the memory dtype")
         b = queries.shape[0]
@@ -172,13 +205,7 @@ class Memory:
                 "entry_weight": torch.empty(b, k_entries, dtype=torch.float32, device=dev),
                 "lse": torch.empty(b, dtype=torch.float32, device=dev),
             }
-        p = QueryParams(k_groups, k_entries, tau, epsilon)
-        _check(_lib.htam_query(self.handle, _dev_ptr(queries), b, ctypes.byref(p),
-                               _dev_ptr(out["group_idx"]), _dev_ptr(out["group_score"]),
-                               _dev_ptr(out["entry_idx"]), _dev_ptr(out["entry_score"]),
-                               _dev_ptr(out["entry_weight"]), _dev_ptr(out.get("lse")),
-                               _stream_ptr(stream)), "htam_query")
-        return out
+        return b, out
 
     def query_flat(self, queries: torch.Tensor, k_entries: int, tau: float = 1.0, epsilon: float = 0.0,
                    stream=None, out: dict | None = None) -> dict:
@@ -228,10 +255,12 @@ class Memory:
 
     def query_edges(self, edge_features: torch.Tensor, weights, prefix_groups, lam: float, queries: torch.Tensor,
                     k_groups: int, k_entries: int, tau: float = 1.0, epsilon: float = 0.0, stream=None,
-                    out: dict | None = None) -> dict:
+                    out: dict | None = None, sampling: tuple[int, int] | None = None) -> dict:
         """Lookup routed by transition edges: edge_features [G, G, F] float32
         on the device, weights [F] and prefix_groups [b, P] (int32, -1 = none)
-        on the host, queries [b, d] on the device for the entry level."""
+        on the host, queries [b, d] on the device for the entry level.  With
+        sampling = (seed, offset) the groups are drawn from the policy of
+        Eq. 11 over the edge scores instead of ranked."""
         if edge_features.dtype != torch.float32 or edge_features.dim() != 3:
             raise ValueError("edge_features must be a [G, G, F] float32 tensor")
         if queries.dtype != self.dtype or queries.dim() != 2 or queries.shape[1] != self.d:
@@ -252,13 +281,16 @@ class Memory:
                 "lse": torch.empty(b, dtype=torch.float32, device=dev),
             }
         p = QueryParams(k_groups, k_entries, tau, epsilon)
-        _check(_lib.htam_query_edges(self.handle, _dev_ptr(edge_features), edge_features.shape[2],
-                                     ctypes.c_void_p(w.data_ptr()), ctypes.c_void_p(pre.data_ptr()), pre.shape[1],
-                                     float(lam), _dev_ptr(queries), b, ctypes.byref(p),
-                                     _dev_ptr(out["group_idx"]), _dev_ptr(out["group_score"]),
-                                     _dev_ptr(out["entry_idx"]), _dev_ptr(out["entry_score"]),
-                                     _dev_ptr(out["entry_weight"]), _dev_ptr(out.get("lse")),
-                                     _stream_ptr(stream)), "htam_query_edges")
+        head = (self.handle, _dev_ptr(edge_features), edge_features.shape[2], ctypes.c_void_p(w.data_ptr()),
+                ctypes.c_void_p(pre.data_ptr()), pre.shape[1], float(lam), _dev_ptr(queries), b, ctypes.byref(p))
+        tail = (_dev_ptr(out["group_idx"]), _dev_ptr(out["group_score"]), _dev_ptr(out["entry_idx"]),
+                _dev_ptr(out["entry_score"]), _dev_ptr(out["entry_weight"]), _dev_ptr(out.get("lse")),
+                _stream_ptr(stream))
+        if sampling is None:
+            _check(_lib.htam_query_edges(*head, *tail), "htam_query_edges")
+        else:
+            smp = Sampling(*sampling)
+            _check(_lib.htam_query_edges_sampled(*head, ctypes.byref(smp), *tail), "htam_query_edges_sampled")
         return out
 
     def query_host(self, queries: torch.Tensor, k_groups: int, k_entries: int, tau: float = 1.0,

@@ -186,6 +186,67 @@ def compare_flat(out, entries_np, queries_np, k_entries, tau, eps, dtype, rows=N
     return problems
 
 
+def check_draws(what, gi, gs, keys, scores, counts, k, dtype, score_tol=None):
+    """Groups drawn by the GPU for one query against the oracle's policy keys
+    (the index rule on keys: the draws are the top k keys), and their
+    group_score against the oracle's float64 scores q . c_g."""
+    import oracle
+
+    ref_gi, ref_gk = oracle.select(keys[None, :], counts, min(k + 1, len(counts)))
+    ref_gi, ref_gk = ref_gi[0], ref_gk[0]
+    if len(ref_gi) == k:
+        ref_gi = np.append(ref_gi, -1)
+        ref_gk = np.append(ref_gk, -np.inf)
+    key_of = [float(keys[g]) if g >= 0 else -np.inf for g in gi]
+    problems = check_ranked(what, gi, key_of, ref_gi, ref_gk, k, lambda g: float(keys[g]), dtype)
+    for g, s in zip(gi, gs):
+        if g < 0:
+            continue
+        ok = abs(float(s) - scores[g]) <= score_tol[g] if score_tol is not None else close(s, scores[g], dtype)
+        if not ok:
+            problems.append(f"{what}: score of group {g} gpu {float(s):.7g} oracle {scores[g]:.7g}")
+            break
+    return problems
+
+
+def compare_sampled(out, entries_np, gid_np, n_groups, queries_np, k_groups, k_entries, tau, eps, dtype, seed,
+                    offset, rows=None, centroid=None, counts=None, scores=None, score_tol=None, nthreads=None):
+    """The sampled lookup of the queries in `rows` (all by default): the draws
+    against the oracle's policy keys for the same (seed, offset, query),
+    stage 2 given the GPU's draws.  `scores` ([B, G] float64) replaces the
+    group-key scores (the edge-table router), with `score_tol` ([B, G]) the
+    absolute bounds of its values."""
+    import oracle
+
+    gi = out["group_idx"].cpu().numpy()
+    gs = out["group_score"].cpu().numpy()
+    ei = out["entry_idx"].cpu().numpy()
+    es = out["entry_score"].cpu().numpy()
+    ew = out["entry_weight"].cpu().numpy()
+    lse = out["lse"].cpu().numpy()
+    B = queries_np.shape[0]
+    rows = np.arange(B) if rows is None else np.asarray(rows)
+    q = queries_np[rows]
+    if counts is None:
+        counts = np.bincount(np.asarray(gid_np, dtype=np.int64), minlength=n_groups)
+    if scores is None:
+        if centroid is None:
+            centroid, counts = oracle.centroids(entries_np, gid_np, n_groups, nthreads)
+        s_rows = oracle.coarse_scores(q, centroid)
+    else:
+        s_rows = np.asarray(scores, dtype=np.float64)[rows]
+    keys, _ = oracle.policy_keys(s_rows, counts, tau, eps, seed, offset, query_ids=rows)
+    ref2 = oracle.stage2(entries_np, gid_np, n_groups, q, gi[rows], k_entries + 16, tau, eps, nthreads)
+    qf = _as_f64(q)
+    problems = []
+    for r, b in enumerate(rows):
+        tol_r = None if score_tol is None else np.asarray(score_tol)[b]
+        problems += check_draws(f"query {b} draws", gi[b], gs[b], keys[r], s_rows[r], counts, k_groups, dtype,
+                                tol_r)
+        problems += _check_entries(ei, es, ew, lse, b, r, ref2, entries_np, qf, k_entries, tau, eps, dtype)
+    return problems
+
+
 def _as_f64(x: np.ndarray) -> np.ndarray:
     if x.dtype == np.uint16:
         return (x.astype(np.uint32) << 16).view(np.float32).astype(np.float64)

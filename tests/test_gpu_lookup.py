@@ -475,6 +475,133 @@ def test_flat_arguments_checked(htam):
         mem.query_flat(raw[1:].view(3, 64), 4)
 
 
+SAMPLED_CASES = [
+    # n, groups, d, dtype, batch, k_groups, k_entries, tau, eps
+    (8000, 40, 256, torch.float32, 30, 5, 12, 0.3, 0.1),
+    (20000, 100, 512, torch.bfloat16, 300, 1, 16, 0.05, 0.0),   # the paper's single draw; tensor-core buckets
+    (20000, 100, 512, torch.bfloat16, 70, 8, 24, 0.5, 0.3),
+    (6000, 50, 128, torch.bfloat16, 40, 6, 8, 1.0, 1.0),        # pure exploration: uniform over G_t
+    (3000, 1000, 64, torch.float32, 9, 64, 16, 0.2, 0.05),      # many groups, most of them empty or small
+]
+
+
+@pytest.mark.parametrize("case", SAMPLED_CASES)
+def test_sampled_lookup_matches_oracle(htam, case):
+    """htam_query_sampled against the oracle: the draws are the top k_groups
+    of the oracle's policy keys (Eq. 11 with the same Philox uniforms), the
+    group scores q . c_g, and stage 2 over the drawn groups."""
+    from parity import compare_sampled
+
+    n, g, d, dtype, b, kg, ke, tau, eps = case
+    entries, gid, centres = _rand_memory(n, d, g, dtype, seed=n + b)
+    q = _rand_queries(b, d, dtype, seed=n + b, centres=centres)
+    mem = htam.Memory(entries, gid, g)
+    out = mem.query_sampled(q, kg, ke, seed=1234 + n, offset=5, tau=tau, epsilon=eps)
+    torch.cuda.synchronize()
+    dt = "bf16" if dtype == torch.bfloat16 else "f32"
+    problems = compare_sampled(out, to_numpy(entries), to_numpy(gid), g, to_numpy(q), kg, ke, tau, eps, dt,
+                               seed=1234 + n, offset=5)
+    assert not problems, "\n".join(problems[:20])
+    assert mem.device_status() == htam.HTAM_OK
+
+
+def test_sampled_draws_follow_the_policy(htam):
+    """One query repeated 20,000 times: each copy draws with its own uniforms,
+    so the first draws are distributed as mu_g of Eq. 11 (chi-square against
+    the oracle's policy over the GPU's own group keys), and the empty group
+    never comes up."""
+    import oracle
+    from scipy import stats
+
+    gid = torch.tensor([0, 1, 2, 3, 5, 6] * 50, dtype=torch.int32, device=DEV)  # group 4 empty
+    entries, gid, _ = _rand_memory(300, 32, 7, torch.float32, seed=13, gid=gid)
+    q = _rand_queries(1, 32, torch.float32, seed=13).repeat(20000, 1).contiguous()
+    mem = htam.Memory(entries, gid, 7)
+    out = mem.query_sampled(q, 1, 4, seed=77, offset=0, tau=0.1, epsilon=0.2)
+    torch.cuda.synchronize()
+    first = out["group_idx"][:, 0].cpu().numpy()
+    keys_f32 = mem.group_keys().double().numpy()
+    s = oracle.coarse_scores(to_numpy(q[:1]), keys_f32)
+    counts = mem.group_counts().numpy()
+    _, mu = oracle.policy_keys(s, counts, 0.1, 0.2, 0, 0)
+    obs = np.bincount(first, minlength=7)
+    assert obs[4] == 0
+    ne = counts > 0
+    assert stats.chisquare(obs[ne], 20000 * mu[0][ne] / mu[0][ne].sum()).pvalue > 1e-4
+
+
+def test_sampled_draws_are_reproducible_and_offset_dependent(htam):
+    entries, gid, centres = _rand_memory(6000, 256, 40, torch.bfloat16, seed=14)
+    q = _rand_queries(64, 256, torch.bfloat16, seed=14, centres=centres)
+    mem = htam.Memory(entries, gid, 40)
+    a = mem.query_sampled(q, 4, 16, seed=5, offset=100, tau=0.5, epsilon=0.1)
+    b = mem.query_sampled(q, 4, 16, seed=5, offset=100, tau=0.5, epsilon=0.1)
+    c = mem.query_sampled(q, 4, 16, seed=5, offset=101, tau=0.5, epsilon=0.1)
+    d = mem.query_sampled(q, 4, 16, seed=6, offset=100, tau=0.5, epsilon=0.1)
+    torch.cuda.synchronize()
+    for k in a:
+        assert torch.equal(a[k], b[k]), k
+    assert not torch.equal(a["group_idx"], c["group_idx"])
+    assert not torch.equal(a["group_idx"], d["group_idx"])
+
+
+def test_cold_policy_draws_what_the_ranking_selects(htam):
+    """tau -> 0 with no exploration: the draws are stage 1's ranking."""
+    entries, gid, centres = _rand_memory(8000, 128, 60, torch.float32, seed=15)
+    q = _rand_queries(50, 128, torch.float32, seed=15, centres=centres)
+    mem = htam.Memory(entries, gid, 60)
+    a = mem.query(q, 6, 10, tau=1e-4)
+    s = mem.query_sampled(q, 5, 10, seed=1, offset=2, tau=1e-4)
+    torch.cuda.synchronize()
+    # Rows whose six best groups are 2e-3 apart (20 units of key next to the
+    # Gumbel noise, which exceeds that with probability about e^-20).
+    gaps = (a["group_score"][:, :-1] - a["group_score"][:, 1:]).min(dim=1).values
+    clear = gaps > 2e-3
+    assert clear.sum() > 10
+    assert torch.equal(a["group_idx"][clear][:, :5], s["group_idx"][clear])
+
+
+def test_sampled_edge_routed_lookup_matches_oracle(htam):
+    """htam_query_edges_sampled: the draws from the policy over the edge-table
+    scores (Eq. 9 with the App. B.6 utility), stage 2 over them."""
+    import oracle
+    from parity import compare_sampled
+
+    n, g, d, b, P, F, kg, ke = 12000, 60, 256, 40, 4, 12, 3, 16
+    entries, gid, centres = _rand_memory(n, d, g, torch.float32, seed=16)
+    q = _rand_queries(b, d, torch.float32, seed=16, centres=centres)
+    rng = np.random.default_rng(16)
+    Z = rng.standard_normal((g, g, F)).astype(np.float32)
+    w = rng.standard_normal(F).astype(np.float32)
+    prefix = rng.integers(-1, g, (b, P)).astype(np.int32)
+    mem = htam.Memory(entries, gid, g)
+    out = mem.query_edges(torch.from_numpy(Z).to(DEV), w, prefix, 0.5, q, kg, ke, tau=0.7, epsilon=0.1,
+                          sampling=(42, 9))
+    torch.cuda.synchronize()
+    scores = oracle.edge_scores(Z, w.astype(np.float64), prefix, 0.5)
+    mag = oracle.edge_scores(np.abs(Z), np.abs(w.astype(np.float64)), prefix, 0.5)
+    problems = compare_sampled(out, to_numpy(entries), to_numpy(gid), g, to_numpy(q), kg, ke, 0.7, 0.1, "f32",
+                               seed=42, offset=9, scores=scores, score_tol=1e-5 * mag + 1e-6)
+    assert not problems, "\n".join(problems[:20])
+
+
+def test_sampled_zipf_1m_workload_sampled_rows(htam):
+    """Full size, full batch (4,096 queries against 1,048,576 entries in
+    1,024 groups), a sample of the queries checked."""
+    from parity import compare_sampled
+
+    w = workloads.WORKLOADS["zipf_bf16_1m"]
+    entries, gid, centres = workloads.make_memory(w, seed=0, device=DEV)
+    q = workloads.make_queries(w, gid, centres, seed=0)
+    mem = htam.Memory(entries, gid, w.g)
+    out = mem.query_sampled(q, w.k_groups, w.k_entries, seed=2026, offset=3, tau=0.5, epsilon=0.05)
+    torch.cuda.synchronize()
+    rows = np.linspace(0, w.b - 1, 24).astype(int)
+    problems = compare_sampled(out, to_numpy(entries), to_numpy(gid), w.g, to_numpy(q), w.k_groups, w.k_entries,
+                               0.5, 0.05, "bf16", seed=2026, offset=3, rows=rows)
+    assert not problems, "\n".join(problems[:20])
+
+
 def test_tuning_defaults_follow_row_length_and_round_trip(htam):
     """The tensor-core threshold defaults to 2 queries for rows up to 4 KiB
     and 16 for longer rows; values set are read back; bad keys and values are

@@ -583,3 +583,17 @@ def test_cold_policy_draws_the_top_groups():
     gi, _ = oracle.select(keys, counts, k)
     ref, _ = oracle.select(scores, counts, k)
     assert (gi == ref).all()
+
+
+def test_policy_rows_keep_their_query_uniforms():
+    """A sample of a batch's rows, passed with their query ids, draws what
+    the whole batch draws for those rows."""
+    rng = np.random.default_rng(4)
+    scores = rng.standard_normal((30, 12))
+    counts = np.arange(12, dtype=np.int64) % 5
+    full, _ = oracle.policy_keys(scores, counts, 0.7, 0.1, 99, 7)
+    rows = np.array([29, 3, 17])
+    part, _ = oracle.policy_keys(scores[rows], counts, 0.7, 0.1, 99, 7, query_ids=rows)
+    np.testing.assert_array_equal(part, full[rows])
+    other, _ = oracle.policy_keys(scores[rows], counts, 0.7, 0.1, 99, 7)
+    assert not np.array_equal(other, full[rows])
