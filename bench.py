@@ -66,6 +66,9 @@ def parse_args():
     ap.add_argument("--edge-features", type=int, default=12, help="features per edge (12 in App. B.6)")
     ap.add_argument("--flat", action="store_true",
                     help="flat scan (htam_query_flat): every entry a candidate, no group stage")
+    ap.add_argument("--unassigned", type=float, default=0.0,
+                    help="streaming workloads: this share of each append's rows comes without a group id (-1) "
+                         "and joins the group with the nearest key")
     ap.add_argument("--sample", action="store_true",
                     help="draw the groups from the policy of Eq. 11 (htam_query_sampled / "
                          "htam_query_edges_sampled) instead of ranking them")
@@ -393,6 +396,10 @@ def run_htam(args, world, rank, local):
         n_rounds = args.warmup + args.steps
         append_batches = [workloads.make_append_batch(w, centres, r, seed=args.seed, device=dev)
                           for r in range(min(n_rounds, w.rounds))]
+        if args.unassigned > 0:
+            gen = torch.Generator(device=dev).manual_seed(args.seed + 31)
+            append_batches = [(e, torch.where(torch.rand(g.shape[0], generator=gen, device=dev) < args.unassigned,
+                                              torch.full_like(g, -1), g).contiguous()) for e, g in append_batches]
     out = run_query(batches[0])
     torch.cuda.synchronize()
 
@@ -578,6 +585,7 @@ def run_htam(args, world, rank, local):
                        "mean_candidates_per_query": float(np.mean([x["mean_candidates"] for x in work])),
                        **({"flat": True} if args.flat else {}),
                        **({"sampled_groups": True} if args.sample else {}),
+                       **({"unassigned_share": args.unassigned} if args.unassigned > 0 and w.rounds else {}),
                        "l2": ("flushed between steps (2x L2 buffer write, outside the step events)" if flush_l2 else
                               f"inputs larger than L2 ({work[0]['step_bytes'] / 1e9:.2f} GB touched per step)"),
                        "parallelism": f"replicas{world}" if world > 1 else "single GPU",

@@ -92,14 +92,30 @@ htam_status htam_build_memory(const void *entries, const int32_t *group_ids,
 
 /* Appends `count` entries (the memory update of Eq. 15) and updates the keys
  * of the groups they join in place.  New entries get ids n, n+1, ...
- *  entries  : [count, d] of the memory's dtype, device
- *  group_ids: [count] int32 in [0, n_groups), device
- * Synchronises `cuda_stream` once.  Errors: EINVAL (a group id out of range),
- * ECAPACITY (n + count would exceed the capacity, or the page pool is full);
- * the memory is unchanged on any error. */
+ *  entries  : [count, d] of the memory's dtype, device, 16-byte aligned
+ *  group_ids: [count] int32, device, 16-byte aligned: a group in
+ *             [0, n_groups), or -1 for an entry without a group, which joins
+ *             the group whose key scores highest against it (q . c_g with the
+ *             entry as q, stage 1's scorer; ties to the lower id; empty groups
+ *             excluded), by the keys as they stand before this call
+ * Synchronises `cuda_stream` once (twice when some id is -1).  Errors:
+ * EINVAL (a group id out of range, or an id of -1 while every group is
+ * empty), ECAPACITY (n + count would exceed the capacity, or the page pool is
+ * full), ENOMEM; the memory is unchanged on any error. */
 htam_status htam_append_transitions(htam_memory *m, const void *entries,
                                     const int32_t *group_ids, int64_t count,
                                     void *cuda_stream);
+
+/* htam_append_transitions that also reports the group each entry joined:
+ *  assigned : [count] int32, device, caller-allocated (may be group_ids
+ *             itself); receives group_ids with every -1 replaced by the group
+ *             chosen for that entry.
+ * The nearest-key choice keeps a [rows, n_groups] fp32 score buffer that the
+ * memory object owns (up to 16 MiB per K split), grown with cudaMalloc on
+ * demand. */
+htam_status htam_append_assign(htam_memory *m, const void *entries,
+                               const int32_t *group_ids, int64_t count,
+                               int32_t *assigned, void *cuda_stream);
 
 /* Answers b queries (device pointers; all outputs caller-allocated):
  *  queries     : [b, d] of the memory's dtype

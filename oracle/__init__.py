@@ -286,6 +286,20 @@ def query_edges(entries: np.ndarray, gid: np.ndarray, n_groups: int, Z: np.ndarr
     return out
 
 
+def assign_nearest(entries: np.ndarray, gid: np.ndarray, centroid: np.ndarray, counts: np.ndarray,
+                   nthreads: int | None = None) -> np.ndarray:
+    """Group ids of appended entries: ids >= 0 kept, each -1 replaced by the
+    group whose key scores highest against the entry (stage 1's scorer and
+    ranking with k_g = 1: ties to the lower id, empty groups excluded), with
+    the keys as they stand before the append."""
+    out = np.array(gid, dtype=np.int32, copy=True)
+    miss = np.flatnonzero(out == -1)
+    if len(miss):
+        gi, _ = stage1(np.ascontiguousarray(np.asarray(entries)[miss]), centroid, counts, 1, nthreads)
+        out[miss] = gi[:, 0]
+    return out
+
+
 # ------------------------------------------------ sampling from the policy (Eq. 11)
 
 def philox4x32_10(ctr, key) -> np.ndarray:

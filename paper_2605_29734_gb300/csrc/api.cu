@@ -107,7 +107,16 @@ htam_status htam_append_transitions(htam_memory *m, const void *entries, const i
   if (count == 0) return HTAM_OK;
   if (!entries || !group_ids || !aligned16(entries) || !aligned16(group_ids)) return HTAM_EINVAL;
   if (m->n + count > m->capacity) return HTAM_ECAPACITY;
-  return append_impl(m, entries, group_ids, count, static_cast<cudaStream_t>(cuda_stream));
+  return append_impl(m, entries, group_ids, count, nullptr, static_cast<cudaStream_t>(cuda_stream));
+}
+
+htam_status htam_append_assign(htam_memory *m, const void *entries, const int32_t *group_ids, int64_t count,
+                               int32_t *assigned, void *cuda_stream) {
+  if (!m || count < 0) return HTAM_EINVAL;
+  if (count == 0) return HTAM_OK;
+  if (!entries || !group_ids || !assigned || !aligned16(entries) || !aligned16(group_ids)) return HTAM_EINVAL;
+  if (m->n + count > m->capacity) return HTAM_ECAPACITY;
+  return append_impl(m, entries, group_ids, count, assigned, static_cast<cudaStream_t>(cuda_stream));
 }
 
 static htam_status check_query_args(const htam_memory *m, const void *queries, int32_t b,

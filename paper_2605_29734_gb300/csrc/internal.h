@@ -54,6 +54,8 @@ struct htam_memory {
   // Reduced queries of htam_query_prefix.
   void *prefix_buf = nullptr;
   size_t prefix_bytes = 0;
+  void *assign_buf = nullptr;  // nearest-key assignment of appended rows
+  size_t assign_bytes = 0;
 
   // Phase timing and launch counters (htam_set_phase_timing / _read_).
   bool timing = false;
@@ -98,7 +100,7 @@ htam_status build_impl(const void *entries, const int32_t *group_ids, int64_t n,
                        int32_t n_groups, htam_dtype dtype, int64_t capacity, cudaStream_t st,
                        htam_memory **out);
 htam_status append_impl(htam_memory *m, const void *entries, const int32_t *group_ids,
-                        int64_t count, cudaStream_t st);
+                        int64_t count, int32_t *assigned, cudaStream_t st);
 // Stage 1 from a transition-edge table instead of the group keys
 // (htam_query_edges).
 struct EdgeRoute {
@@ -120,6 +122,13 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t b,
 // Largest b * (non-empty groups) the flat scan takes (its bucket rows).
 constexpr int64_t kMaxFlatRows = int64_t(1) << 28;
 void free_impl(htam_memory *m);
+// ids[i] = gid[i] where gid[i] >= 0, else the group whose key scores highest
+// against row i of `entries` (stage 1's scorer and ranking with k = 1).  The
+// ids go to `dst` (`count` of them; it may be `gid` itself) or, when dst is
+// NULL, to m->assign_buf; *ids_out points at them.  The scratch is
+// m->assign_buf, grown on demand (which synchronises the device).
+htam_status assign_nearest(htam_memory *m, const void *entries, const int32_t *gid, int64_t count, int32_t *dst,
+                           const int32_t **ids_out, cudaStream_t st);
 
 // Weights alpha_1..alpha_P of a prefix (Eq. 10), passed by value to the
 // reduction kernel.

@@ -37,12 +37,17 @@ static int key_seg_rows(int64_t count) {
   return r;
 }
 
+// Per-group counts of a batch; ids of -1 (no group given) are counted apart,
+// any other id outside [0, n_groups) sets `bad`.
 __global__ void count_groups_kernel(const int32_t *__restrict__ gid, int64_t n, int32_t n_groups,
-                                    int32_t *__restrict__ counts, int32_t *__restrict__ bad) {
+                                    int32_t *__restrict__ counts, int32_t *__restrict__ bad,
+                                    int32_t *__restrict__ unassigned) {
   for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < n;
        e += (int64_t)gridDim.x * blockDim.x) {
     int32_t g = gid[e];
-    if (g < 0 || g >= n_groups) {
+    if (g == -1) {
+      atomicAdd(unassigned, 1);
+    } else if (g < 0 || g >= n_groups) {
       atomicOr(bad, 1);
     } else {
       atomicAdd(&counts[g], 1);
@@ -239,7 +244,7 @@ htam_status ensure_scratch(htam_memory *m, size_t bytes) {
 // of the groups they join.  Arguments are already validated except the group
 // id range, which is checked on the device before anything is written.
 static htam_status add_rows(htam_memory *m, const void *entries, const int32_t *gid, int64_t count,
-                            cudaStream_t st) {
+                            int32_t *assigned, cudaStream_t st) {
   if (count == 0) return HTAM_OK;
   const int32_t G = m->n_groups, d = m->d;
 
@@ -253,14 +258,14 @@ static htam_status add_rows(htam_memory *m, const void *entries, const int32_t *
   const int seg_rows = key_seg_rows(count);
   int64_t max_segs = count / seg_rows + G + 1;
 
-  size_t need = Carver::round(sizeof(int32_t) * (G + 1)) + Carver::round(sizeof(int32_t) * count) +
+  size_t need = Carver::round(sizeof(int32_t) * (G + 2)) + Carver::round(sizeof(int32_t) * count) +
                 Carver::round(sizeof(int32_t) * (size_t)G * n_chunks) +
                 Carver::round(sizeof(KeySeg) * max_segs) + Carver::round(sizeof(KeyGroup) * G) +
                 Carver::round(sizeof(double) * (size_t)max_segs * d) + 4096;
   htam_status s = ensure_scratch(m, need);
   if (s != HTAM_OK) return s;
   Carver cv(m->scratch);
-  int32_t *bcount = cv.take<int32_t>(G + 1);  // [G] counts + [1] bad flag
+  int32_t *bcount = cv.take<int32_t>(G + 2);  // [G] counts, bad flag, rows without a group
   int32_t *pos = cv.take<int32_t>(count);
   int32_t *hist = cv.take<int32_t>((size_t)G * n_chunks);
   KeySeg *segs = cv.take<KeySeg>(max_segs);
@@ -268,16 +273,34 @@ static htam_status add_rows(htam_memory *m, const void *entries, const int32_t *
   double *partial = cv.take<double>((size_t)max_segs * d);
 
   // 1. Per-group counts of the batch and the group-id range check.
-  HTAM_CK(cudaMemsetAsync(bcount, 0, sizeof(int32_t) * (G + 1), st));
-  {
+  std::vector<int32_t> h_b(G + 2);
+  auto count_batch = [&](const int32_t *ids) -> htam_status {
+    HTAM_CK(cudaMemsetAsync(bcount, 0, sizeof(int32_t) * (G + 2), st));
     int blocks = (int)std::min<int64_t>(ceil_div(count, 256), 4096);
-    count_groups_kernel<<<blocks, 256, 0, st>>>(gid, count, G, bcount, bcount + G);
+    count_groups_kernel<<<blocks, 256, 0, st>>>(ids, count, G, bcount, bcount + G, bcount + G + 1);
     HTAM_CK_LAUNCH("count_groups_kernel");
-  }
-  std::vector<int32_t> h_b(G + 1);
-  HTAM_CK(cudaMemcpyAsync(h_b.data(), bcount, sizeof(int32_t) * (G + 1), cudaMemcpyDeviceToHost, st));
-  HTAM_CK(cudaStreamSynchronize(st));
+    HTAM_CK(cudaMemcpyAsync(h_b.data(), bcount, sizeof(int32_t) * (G + 2), cudaMemcpyDeviceToHost, st));
+    HTAM_CK(cudaStreamSynchronize(st));
+    return HTAM_OK;
+  };
+  s = count_batch(gid);
+  if (s != HTAM_OK) return s;
   if (h_b[G] != 0) return HTAM_EINVAL;
+  if (h_b[G + 1] > 0) {
+    // Rows without a group join the group whose key scores highest against
+    // them, by the keys as they stand before this call (none: EINVAL).
+    bool any = false;
+    for (int64_t c : m->h_count) any |= c > 0;
+    if (!any) return HTAM_EINVAL;
+    const int32_t *ids = nullptr;
+    s = assign_nearest(m, entries, gid, count, assigned, &ids, st);
+    if (s != HTAM_OK) return s;
+    gid = ids;
+    s = count_batch(gid);
+    if (s != HTAM_OK) return s;
+  } else if (assigned && assigned != gid) {
+    HTAM_CK(cudaMemcpyAsync(assigned, gid, sizeof(int32_t) * count, cudaMemcpyDeviceToDevice, st));
+  }
 
   // 2. Page layout on the host.
   std::vector<int64_t> new_count(G);
@@ -391,6 +414,7 @@ void free_impl(htam_memory *m) {
   cudaFree(m->scratch);
   cudaFree(m->stage);
   cudaFree(m->prefix_buf);
+  cudaFree(m->assign_buf);
   for (cudaEvent_t e : m->ev_pool) cudaEventDestroy(e);
   cudaGetLastError();
   cudaSetDevice(prev);
@@ -450,16 +474,16 @@ htam_status build_impl(const void *entries, const int32_t *gid, int64_t n, int32
     set_last_error("cudaMemsetAsync", cudaGetLastError());
     return fail(HTAM_ECUDA);
   }
-  htam_status s = add_rows(m, entries, gid, n, st);
+  htam_status s = add_rows(m, entries, gid, n, nullptr, st);
   if (s != HTAM_OK) return fail(s);
   *out = m;
   return HTAM_OK;
 }
 
 htam_status append_impl(htam_memory *m, const void *entries, const int32_t *gid, int64_t count,
-                        cudaStream_t st) {
+                        int32_t *assigned, cudaStream_t st) {
   if (m->n + count > m->capacity) return HTAM_ECAPACITY;
-  return add_rows(m, entries, gid, count, st);
+  return add_rows(m, entries, gid, count, assigned, st);
 }
 
 }  // namespace htam

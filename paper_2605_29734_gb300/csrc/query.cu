@@ -1386,4 +1386,77 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   return HTAM_OK;
 }
 
+// ------------------------------------------------- nearest-key assignment
+
+namespace {
+
+// ids[i] = gid[i] when given, else the nearest group picked for row i.  gid
+// and ids may be the same array (each thread reads and writes only its row).
+__global__ void assign_fill_kernel(const int32_t *gid, const int32_t *__restrict__ pick, int64_t n, int32_t *ids) {
+  const int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  if (t < n) {
+    const int32_t g = gid[t];
+    ids[t] = g >= 0 ? g : pick[t];
+  }
+}
+
+}  // namespace
+
+htam_status assign_nearest(htam_memory *m, const void *entries, const int32_t *gid, int64_t count, int32_t *dst,
+                           const int32_t **ids_out, cudaStream_t st) {
+  const int G = m->n_groups, d = m->d;
+  // Rows per pass: the [rows, G] score matrix stays within 16 MiB per plane.
+  const int64_t R = std::max<int64_t>(1, std::min<int64_t>(count, (int64_t(1) << 22) / G));
+  const int64_t last = count - (ceil_div(count, R) - 1) * R;
+  auto planes_of = [&](int64_t rb) {
+    return m->dtype == HTAM_BF16 ? coarse_tc_splits((int)rb, d, G, m->sm_count) : 1;
+  };
+  const int64_t s1_elems = std::max<int64_t>(planes_of(R) * R, planes_of(last) * last) * G;
+  const size_t need = (dst ? 0 : Carver::round(sizeof(int32_t) * count)) + Carver::round(sizeof(float) * s1_elems) +
+                      Carver::round(sizeof(int32_t) * R) + Carver::round(sizeof(float) * R) + 1024;
+  if (need > m->assign_bytes) {
+    if (m->assign_buf) cudaFree(m->assign_buf);  // synchronises: no queued work still reads it
+    m->assign_buf = nullptr;
+    m->assign_bytes = 0;
+    const size_t want = need + need / 2;
+    if (cudaMalloc(&m->assign_buf, want) != cudaSuccess) {
+      cudaGetLastError();
+      return HTAM_ENOMEM;
+    }
+    m->assign_bytes = want;
+  }
+  Carver cv(m->assign_buf);
+  int32_t *ids = dst ? dst : cv.take<int32_t>(count);
+  float *s1 = cv.take<float>(s1_elems);
+  int32_t *pick = cv.take<int32_t>(R);
+  float *pick_score = cv.take<float>(R);
+  for (int64_t r0 = 0; r0 < count; r0 += R) {
+    const int rb = (int)std::min<int64_t>(R, count - r0);
+    const void *rows = static_cast<const char *>(entries) + r0 * d * m->elem_bytes;
+    const int planes = planes_of(rb);
+    if (m->dtype == HTAM_BF16) {
+      htam_status s = launch_coarse_tc(rows, rb, d, m->cent_hi, m->cent_lo, m->count, G, planes, s1, m->status,
+                                       kMaxPolls, st);
+      if (s != HTAM_OK) return s;
+    } else {
+      dim3 grid((unsigned)ceil_div(G, 64), (unsigned)ceil_div(rb, 64));
+      coarse_scores_simt_kernel<float><<<grid, 256, 0, st>>>(static_cast<const float *>(rows), rb, d, m->cent,
+                                                             m->count, G, s1);
+      HTAM_CK_LAUNCH("coarse_scores_simt_kernel");
+    }
+    if (warps_per_query(rb, m->sm_count) == 8) {
+      group_topk_kernel<8><<<(unsigned)rb, kSelWarps * 32, 0, st>>>(s1, planes, rb, G, m->count, 1, pick,
+                                                                    pick_score);
+    } else {
+      group_topk_kernel<1><<<(unsigned)ceil_div(rb, kSelWarps), kSelWarps * 32, 0, st>>>(
+          s1, planes, rb, G, m->count, 1, pick, pick_score);
+    }
+    HTAM_CK_LAUNCH("group_topk_kernel");
+    assign_fill_kernel<<<(unsigned)ceil_div(rb, 256), 256, 0, st>>>(gid + r0, pick, rb, ids + r0);
+    HTAM_CK_LAUNCH("assign_fill_kernel");
+  }
+  *ids_out = ids;
+  return HTAM_OK;
+}
+
 }  // namespace htam

@@ -23,8 +23,8 @@ HTAM_MAX_EDGE_FEATURES = 32  # most features per edge htam_query_edges takes
 
 # Every symbol include/htam.h declares, in declaration order.
 EXPORTS = (
-    "htam_build_memory", "htam_append_transitions", "htam_query", "htam_query_host", "htam_query_prefix",
-    "htam_query_edges", "htam_query_flat", "htam_query_sampled", "htam_query_edges_sampled",
+    "htam_build_memory", "htam_append_transitions", "htam_append_assign", "htam_query", "htam_query_host",
+    "htam_query_prefix", "htam_query_edges", "htam_query_sampled", "htam_query_edges_sampled", "htam_query_flat",
     "htam_select_groups_static", "htam_memory_info", "htam_memory_group_counts", "htam_memory_group_keys",
     "htam_device_status", "htam_set_tuning", "htam_get_tuning", "htam_set_phase_timing",
     "htam_read_phase_timing", "htam_free_memory", "htam_status_string", "htam_last_error",
@@ -58,6 +58,7 @@ def _load() -> ctypes.CDLL:
     PP = ctypes.POINTER(ctypes.c_void_p)
     lib.htam_build_memory.argtypes = [P, P, i64, i32, i32, ctypes.c_int, i64, P, PP]
     lib.htam_append_transitions.argtypes = [P, P, P, i64, P]
+    lib.htam_append_assign.argtypes = [P, P, P, i64, P, P]
     qargs = [P, P, i32, ctypes.POINTER(QueryParams), P, P, P, P, P, P, P]
     lib.htam_query.argtypes = qargs
     lib.htam_query_host.argtypes = qargs
@@ -164,6 +165,18 @@ class Memory:
         _check(_lib.htam_append_transitions(self.handle, _dev_ptr(entries), _dev_ptr(group_ids),
                                             entries.shape[0], _stream_ptr(stream)),
                "htam_append_transitions")
+
+    def append_assign(self, entries: torch.Tensor, group_ids: torch.Tensor, stream=None) -> torch.Tensor:
+        """append() that returns the group each entry joined (ids of -1 join
+        the group with the nearest key)."""
+        if entries.dtype != self.dtype or group_ids.dtype != torch.int32:
+            raise TypeError("entries must match the memory dtype; group_ids int32")
+        if entries.dim() != 2 or entries.shape[1] != self.d or group_ids.shape[0] != entries.shape[0]:
+            raise ValueError("entries [count, d] and group_ids [count] expected")
+        assigned = torch.empty_like(group_ids)
+        _check(_lib.htam_append_assign(self.handle, _dev_ptr(entries), _dev_ptr(group_ids), entries.shape[0],
+                                       _dev_ptr(assigned), _stream_ptr(stream)), "htam_append_assign")
+        return assigned
 
     def query(self, queries: torch.Tensor, k_groups: int, k_entries: int, tau: float = 1.0,
               epsilon: float = 0.0, stream=None, out: dict | None = None) -> dict:

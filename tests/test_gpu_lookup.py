@@ -718,6 +718,97 @@ def test_append_errors_leave_memory_unchanged(htam):
         assert torch.equal(before[k], after[k])
 
 
+NEAREST_CASES = [
+    # n, groups, d, dtype, appended rows, share without a group
+    (4000, 30, 64, torch.float32, 700, 0.5),
+    (6000, 40, 512, torch.bfloat16, 1500, 1.0),     # every row assigned, tensor-core scores
+    (3000, 2000, 64, torch.bfloat16, 5000, 0.7),    # rows x groups > 4M: three passes, the last ragged
+]
+
+
+@pytest.mark.parametrize("case", NEAREST_CASES)
+def test_append_without_group_joins_nearest_key(htam, case):
+    """Appended rows with group id -1 join the group whose key (before the
+    append) scores highest against them, ranked like stage 1 (the index rule
+    on the oracle's float64 scores); given ids are kept; the memory then
+    answers like the oracle rebuilt with the assigned ids."""
+    import oracle
+    from parity import check_ranked
+
+    n, g, d, dtype, add, share = case
+    entries, gid, centres = _rand_memory(n, d, g, dtype, seed=n + add)
+    mem = htam.Memory(entries, gid, g, capacity=n + add)
+    new_e, new_g, _ = _rand_memory(add, d, g, dtype, seed=n + add + 1)
+    drop = torch.rand(add, generator=torch.Generator(device=DEV).manual_seed(3), device=DEV) < share
+    new_g = torch.where(drop, torch.full_like(new_g, -1), new_g).contiguous()
+    cent, counts = oracle.centroids(to_numpy(entries), to_numpy(gid), g)
+    assigned = mem.append_assign(new_e, new_g)
+    torch.cuda.synchronize()
+    a = to_numpy(assigned)
+    given = to_numpy(new_g)
+    assert (a[given >= 0] == given[given >= 0]).all()
+    miss = np.flatnonzero(given == -1)
+    ref_gi, ref_gs = oracle.stage1(to_numpy(new_e)[miss], cent, counts, min(2, g))
+    xf = to_numpy(new_e)[miss]
+    xf = (xf.astype(np.uint32) << 16).view(np.float32).astype(np.float64) if xf.dtype == np.uint16 else xf.astype(np.float64)
+    dt = "bf16" if dtype == torch.bfloat16 else "f32"
+    problems = []
+    for r, i in enumerate(miss):
+        problems += check_ranked(f"row {i}", [a[i]], [float(cent[a[i]] @ xf[r])], ref_gi[r], ref_gs[r], 1,
+                                 lambda gg, r=r: float(cent[gg] @ xf[r]), dt)
+    assert not problems, "\n".join(problems[:20])
+    all_e = torch.cat([entries, new_e])
+    all_g = torch.cat([gid, assigned])
+    assert (mem.group_counts().numpy() == np.bincount(to_numpy(all_g), minlength=g)).all()
+    q = _rand_queries(40, d, dtype, seed=n, centres=centres)
+    _check(htam, mem, all_e, all_g, g, q, min(4, g), 12, tau=0.4)
+
+
+def test_append_without_group_in_place_and_plain_append(htam):
+    """The assigned ids may overwrite the input ids; htam_append_transitions
+    takes -1 the same way."""
+    entries, gid, _ = _rand_memory(2000, 64, 12, torch.float32, seed=21)
+    mem_a = htam.Memory(entries, gid, 12, capacity=3000)
+    mem_b = htam.Memory(entries, gid, 12, capacity=3000)
+    new_e, _, _ = _rand_memory(500, 64, 12, torch.float32, seed=22)
+    ids = torch.full((500,), -1, dtype=torch.int32, device=DEV)
+    ids[::3] = 5
+    ref = mem_a.append_assign(new_e, ids.clone())
+    mem_b.append(new_e, ids)
+    import ctypes
+
+    from paper_2605_29734_gb300.htam import _dev_ptr, _lib, _stream_ptr
+
+    mem_c = htam.Memory(entries, gid, 12, capacity=3000)
+    inplace = ids.clone()
+    assert _lib.htam_append_assign(mem_c.handle, _dev_ptr(new_e), _dev_ptr(inplace), 500, _dev_ptr(inplace),
+                                   _stream_ptr(None)) == htam.HTAM_OK
+    torch.cuda.synchronize()
+    assert torch.equal(inplace, ref)
+    assert (mem_a.group_counts() == mem_b.group_counts()).all()
+    assert (mem_c.group_counts() == mem_b.group_counts()).all()
+
+
+def test_append_without_group_errors(htam):
+    """-1 into a memory with no entries has no key to join (EINVAL); ids
+    below -1 stay invalid; the memory is unchanged."""
+    empty = htam.Memory(torch.empty(0, 32, device=DEV), torch.empty(0, dtype=torch.int32, device=DEV), 5,
+                        capacity=100)
+    e, _, _ = _rand_memory(10, 32, 5, torch.float32, seed=23)
+    with pytest.raises(htam.HtamError) as err:
+        empty.append(e, torch.full((10,), -1, dtype=torch.int32, device=DEV))
+    assert err.value.status == htam.HTAM_EINVAL
+    assert empty.info()["n"] == 0
+    entries, gid, _ = _rand_memory(100, 32, 5, torch.float32, seed=24)
+    mem = htam.Memory(entries, gid, 5, capacity=200)
+    bad = torch.full((10,), -1, dtype=torch.int32, device=DEV)
+    bad[4] = -2
+    with pytest.raises(htam.HtamError) as err:
+        mem.append(e, bad)
+    assert err.value.status == htam.HTAM_EINVAL
+    assert mem.info()["n"] == 100
+
+
 def test_stream_workload_rounds(htam):
     """The streaming workload at full size for its first rounds (append 4,096
     clustered rows, then 1,024 queries), oracle-checked on sampled queries."""

@@ -597,3 +597,30 @@ def test_policy_rows_keep_their_query_uniforms():
     np.testing.assert_array_equal(part, full[rows])
     other, _ = oracle.policy_keys(scores[rows], counts, 0.7, 0.1, 99, 7)
     assert not np.array_equal(other, full[rows])
+
+
+# ------------------------------------------------ nearest-key append (Eq. 15)
+
+def test_assign_nearest_matches_numpy_brute_force():
+    """Entries appended without a group join the non-empty group whose key
+    scores highest (numpy argmax with lexsort ties; duplicated keys force
+    ties to the lower id); given ids are kept."""
+    rng = np.random.default_rng(31)
+    d, G = 16, 9
+    keys = _unit_rows(rng, G, d).astype(np.float64)
+    keys[5] = keys[2]  # a tie: group 2 must win
+    counts = np.array([3, 0, 2, 1, 4, 2, 5, 0, 1], dtype=np.int64)
+    x = _unit_rows(rng, 200, d)
+    x[:10] = keys[2].astype(np.float32)  # rows that tie between groups 2 and 5
+    gid = np.where(rng.random(200) < 0.6, -1, rng.integers(0, G, 200)).astype(np.int32)
+    gid[:10] = -1
+    out = oracle.assign_nearest(x, gid, keys, counts)
+    s = x.astype(np.float64) @ keys.T
+    s[:, counts == 0] = -np.inf
+    for i in range(200):
+        if gid[i] >= 0:
+            assert out[i] == gid[i]
+        else:
+            assert out[i] == np.lexsort((np.arange(G), -s[i]))[0]
+    assert (out[:10] == 2).all()
+    assert not np.isin(out[gid == -1], [1, 7]).any()
