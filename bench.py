@@ -484,7 +484,10 @@ def run_htam(args, world, rank, local):
         roofline = {"kernel": kernel, "bound": "hbm", "achieved": k_bytes / k_s / 1e9, "peak": peaks["hbm_gbs"],
                     "unit": "GB/s", "alu_frac": k_flops / k_s / 1e12 / FP32_ALU_TFLOPS}
     roofline["frac"] = roofline["achieved"] / roofline["peak"]
-    roofline.update({"traffic": profiled_traffic(kernel, w.name), "peak_source": peaks["source"],
+    # Profiles are per lookup variant: the variant decides the buckets.
+    variant = ("_flat" if args.flat else "_sampled" if args.sample else "_edges" if E > 0 else
+               "_prefix" if P > 0 else "_unassigned" if args.unassigned > 0 and w.rounds else "")
+    roofline.update({"traffic": profiled_traffic(kernel, w.name + variant), "peak_source": peaks["source"],
                      "algorithmic_bytes_per_launch": k_bytes, "flops_per_launch": k_flops,
                      "mean_launch_ms": k_s * 1e3, "hbm_frac": k_bytes / k_s / 1e9 / peaks["hbm_gbs"]})
     t_roof = max(step_bytes / (peaks["hbm_gbs"] * 1e9),
