@@ -72,6 +72,8 @@ def parse_args():
     ap.add_argument("--sample", action="store_true",
                     help="draw the groups from the policy of Eq. 11 (htam_query_sampled / "
                          "htam_query_edges_sampled) instead of ranking them")
+    ap.add_argument("--tc-pairs", type=int, default=None, choices=[0, 1],
+                    help="tensor-core buckets of several chunks on SM pairs (1) or single SMs (0, library default)")
     ap.add_argument("--tc-min-bucket", type=int, default=None,
                     help="smallest bucket scored on the tensor cores (library default 16)")
     return ap.parse_args()
@@ -350,6 +352,8 @@ def run_htam(args, world, rank, local):
         mem.set_stream_rows(args.stream_rows)
     if args.tc_min_bucket is not None:
         mem.set_tensor_core_min_bucket(args.tc_min_bucket)
+    if args.tc_pairs is not None:
+        mem.set_tensor_core_pairs(args.tc_pairs)
     tc_min = mem.get_tuning(htam.HTAM_TUNE_TC_MIN_BUCKET)
     if args.no_cpu_baseline:
         del entries                  # the memory holds its own copy
@@ -466,7 +470,9 @@ def run_htam(args, world, rank, local):
     phase = max(("fine", "fine_tc"), key=lambda k: phases[k][0])
     kernel = {"fine": cuda_core_kernel(w, args.stream_rows), "fine_tc": "fine_tc"}[phase]
     k_ms, k_launches = phases[phase]
-    k_s = k_ms / 1e3 / max(1, k_launches)
+    # The phase's device time per step (one launch per step, two when the
+    # tensor-core buckets are split between the SM-pair and one-SM kernels).
+    k_s = k_ms / 1e3 / args.steps
     k_bytes = float(np.mean([x["kernels"][phase]["bytes"] for x in per_batch]))
     k_flops = float(np.mean([x["kernels"][phase]["flops"] for x in per_batch]))
     if phase == "fine_tc":
@@ -489,7 +495,8 @@ def run_htam(args, world, rank, local):
                "_prefix" if P > 0 else "_unassigned" if args.unassigned > 0 and w.rounds else "")
     roofline.update({"traffic": profiled_traffic(kernel, w.name + variant), "peak_source": peaks["source"],
                      "algorithmic_bytes_per_launch": k_bytes, "flops_per_launch": k_flops,
-                     "mean_launch_ms": k_s * 1e3, "hbm_frac": k_bytes / k_s / 1e9 / peaks["hbm_gbs"]})
+                     "mean_launch_ms": k_s * 1e3, "launches_per_step": k_launches / args.steps,
+                     "hbm_frac": k_bytes / k_s / 1e9 / peaks["hbm_gbs"]})
     t_roof = max(step_bytes / (peaks["hbm_gbs"] * 1e9),
                  step_flops / ((peaks["bf16_tflops_sustained"] or peaks["bf16_tflops"]) * 1e12))
     step_s = total_s / args.steps

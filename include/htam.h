@@ -333,8 +333,16 @@ typedef enum {
  *  HTAM_TUNE_STREAM_ROWS: 1 (default) prefetches the CUDA-core path's entry
  *    rows into per-warp shared-memory rings (bf16 memories with rows up to
  *    8 KiB and k_entries <= 32); 0 loads them directly into registers.
+ *  HTAM_TUNE_TC_PAIRS: 1 scores the tensor-core buckets of more than 128
+ *    queries on pairs of SMs (two 128-query chunks per M=256 MMA,
+ *    cta_group::2, each SM staging half of every entry tile); 0 (default)
+ *    runs every chunk on one SM.
  * Errors: EINVAL (m NULL, unknown key, value out of range). */
-typedef enum { HTAM_TUNE_TC_MIN_BUCKET = 0, HTAM_TUNE_STREAM_ROWS = 1 } htam_tuning;
+typedef enum {
+  HTAM_TUNE_TC_MIN_BUCKET = 0,
+  HTAM_TUNE_STREAM_ROWS = 1,
+  HTAM_TUNE_TC_PAIRS = 2
+} htam_tuning;
 htam_status htam_set_tuning(htam_memory *m, htam_tuning key, int32_t value);
 
 /* Reads a tuning value (the keys and defaults of htam_set_tuning) into

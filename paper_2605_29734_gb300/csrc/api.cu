@@ -348,6 +348,10 @@ htam_status htam_set_tuning(htam_memory *m, htam_tuning key, int32_t value) {
       if (value != 0 && value != 1) return HTAM_EINVAL;
       m->stream_rows = value;
       return HTAM_OK;
+    case HTAM_TUNE_TC_PAIRS:
+      if (value != 0 && value != 1) return HTAM_EINVAL;
+      m->tc_pairs = value;
+      return HTAM_OK;
   }
   return HTAM_EINVAL;
 }
@@ -360,6 +364,9 @@ htam_status htam_get_tuning(const htam_memory *m, htam_tuning key, int32_t *valu
       return HTAM_OK;
     case HTAM_TUNE_STREAM_ROWS:
       *value = m->stream_rows;
+      return HTAM_OK;
+    case HTAM_TUNE_TC_PAIRS:
+      *value = m->tc_pairs;
       return HTAM_OK;
   }
   return HTAM_EINVAL;

@@ -53,26 +53,35 @@ namespace {
 
 using namespace sm100;
 
-constexpr int kStages = 4;
 constexpr int kKBlock = 64;                        // bf16 elements per 128-byte row slice
 constexpr int kTileN = 2 * kPageRows;              // entries per tile (MMA N)
 constexpr int kABytes = kTcRows * kKBlock * 2;     // 16 KiB
 constexpr int kBBytes = kTileN * kKBlock * 2;      // 32 KiB
-constexpr int kHalfB = kBBytes / 2;
+constexpr int kHalfB = kBBytes / 2;                // one page's K slice
 constexpr int kThreads = 192;
 constexpr uint32_t kAccCols = 256;                 // fp32 columns per accumulator
 constexpr unsigned kFull = 0xffffffffu;
 
+// Operand ring per CTA: a single CTA stages A and both pages of B per K
+// slice (48 KiB, 4 stages); a CTA of a pair stages A and its own page
+// (32 KiB, 6 stages).
+template <bool PAIR>
+struct Ring {
+  static constexpr int kStages = PAIR ? 6 : 4;
+  static constexpr int kBStage = PAIR ? kHalfB : kBBytes;
+};
+constexpr int kMaxStages = 6;
+
 constexpr int kUQ = 4;  // unit queue slots (producer -> MMA and epilogue warps)
 
 struct __align__(8) TcSmem {
-  uint64_t full[kStages];
-  uint64_t empty[kStages];
+  uint64_t full[kMaxStages];
+  uint64_t empty[kMaxStages];
   uint64_t acc_full[2];
   uint64_t acc_empty[2];
   uint64_t drain;
   uint64_t uq_full[kUQ];   // a unit index was written
-  uint64_t uq_empty[kUQ];  // the MMA warp and the 4 epilogue warps have read it
+  uint64_t uq_empty[kUQ];  // every consumer of the slot has read it
   uint32_t tmem_base;
   int abort;
   int uq[kUQ];             // unit indices in the order the producer took them; -1 = no more
@@ -80,19 +89,34 @@ struct __align__(8) TcSmem {
 
 // The j-th unit of this CTA, from the producer's queue, for a whole warp:
 // -1 when there are no more units, or when the wait gave up (ok cleared).
-__device__ __forceinline__ int take_unit(TcSmem *sh, int j, volatile int *abort, uint32_t max_polls, bool &ok) {
+// Lane 0 then arrives on the slot's empty barrier, given by its
+// shared::cluster address (rank 0's barrier for a CTA pair).
+template <bool PAIR>
+__device__ __forceinline__ int take_unit(TcSmem *sh, int j, uint32_t empty_caddr0, volatile int *abort,
+                                         uint32_t max_polls, bool &ok) {
   const int slot = j % kUQ;
-  if (!mbar_wait(&sh->uq_full[slot], (uint32_t)(j / kUQ) & 1u, abort, max_polls)) {
+  const uint32_t par = (uint32_t)(j / kUQ) & 1u;
+  if (!(PAIR ? mbar_wait_cluster(&sh->uq_full[slot], par, abort, max_polls)
+             : mbar_wait(&sh->uq_full[slot], par, abort, max_polls))) {
     ok = false;
     return -1;
   }
   const int u = *reinterpret_cast<volatile int *>(&sh->uq[slot]);
   __syncwarp();
-  if ((threadIdx.x & 31) == 0) mbar_arrive(&sh->uq_empty[slot]);
+  if ((threadIdx.x & 31) == 0) {
+    if constexpr (PAIR) {
+      mbar_arrive_cluster(empty_caddr0 + slot * (uint32_t)sizeof(uint64_t));
+    } else {
+      mbar_arrive(&sh->uq_empty[slot]);
+    }
+  }
   return u;
 }
 
-constexpr size_t kSmemBytes = 1024 /* alignment slack */ + kStages * (kABytes + kBBytes) + sizeof(TcSmem);
+template <bool PAIR>
+constexpr size_t smem_bytes() {
+  return 1024 /* alignment slack */ + Ring<PAIR>::kStages * (kABytes + Ring<PAIR>::kBStage) + sizeof(TcSmem);
+}
 
 __device__ __forceinline__ unsigned enc_score(float f) {
   unsigned u = __float_as_uint(f);
@@ -137,28 +161,54 @@ struct RowTopK {
     c[0] = keep[0] ? c[0] : xc;
   }
 
-  // The score at position k-1 (k <= K): the list is sorted, so it is the
-  // smallest of the first k (a form that keeps the list in registers).
+  // The score at position k-1 (1 <= k <= K) of the sorted list, through a
+  // select tree on the bits of k-1 (log2 K levels instead of a K-long chain;
+  // register indices stay static).
   __device__ __forceinline__ float kth(int k) const {
-    float v = INFINITY;
+    if (k == K) return s[K - 1];
+    const int i = k - 1;
+    float t[K];
 #pragma unroll
-    for (int i = 0; i < K; ++i) v = (i < k) ? fminf(v, s[i]) : v;
-    return v;
+    for (int j = 0; j < K; ++j) t[j] = s[j];
+#pragma unroll
+    for (int w = K / 2, bit = 1; w >= 1; w /= 2, bit *= 2) {
+#pragma unroll
+      for (int j = 0; j < w; ++j) t[j] = (i & bit) ? t[2 * j + 1] : t[2 * j];
+    }
+    return t[0];
   }
 };
 
-template <int K>
+// PAIR = false: one CTA per unit (group, 128-query chunk, page segment).
+// PAIR = true: a cluster of two CTAs per unit (group, pair of chunks 2cp and
+// 2cp+1, page segment), multiplying with tcgen05.mma.cta_group::2 (M=256:
+// rank r holds chunk 2cp+r's 128 queries as its A rows and the tile's page r
+// as its half of B, N=256).  Each CTA reads half of the entry bytes a single
+// CTA reads per MMA, so its operand ring holds six K slices instead of four.
+// Rank 0 takes the units and passes them to both CTAs' queues, sets the
+// byte count each stage expects from both CTAs' copies, and issues the MMAs
+// and their commits to the barriers of both CTAs; each rank's epilogue
+// reads its own 128 accumulator rows.
+template <int K, bool PAIR>
 __global__ void __launch_bounds__(kThreads, 1)
     fine_tc_kernel(const __grid_constant__ CUtensorMap q_map, const __grid_constant__ CUtensorMap pool_map,
                    TcFineArgs a) {
+  constexpr int kStages = Ring<PAIR>::kStages;
+  constexpr int kBStage = Ring<PAIR>::kBStage;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t *smem = smem_raw + ((1024 - (smem_addr(smem_raw) & 1023)) & 1023);
   uint8_t *st_a = smem;
   uint8_t *st_b = st_a + kStages * kABytes;
-  TcSmem *sh = reinterpret_cast<TcSmem *>(st_b + kStages * kBBytes);
+  TcSmem *sh = reinterpret_cast<TcSmem *>(st_b + kStages * kBStage);
   volatile int *abort = &sh->abort;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = PAIR ? cluster_ctarank() : 0u;
+  const bool leader = rank == 0;
+  // Rank 0's barriers as shared::cluster addresses (this CTA's own when single).
+  const uint32_t full_c0 = PAIR ? mapa_shared(smem_addr(&sh->full[0]), 0) : smem_addr(&sh->full[0]);
+  const uint32_t acc_empty_c0 = PAIR ? mapa_shared(smem_addr(&sh->acc_empty[0]), 0) : smem_addr(&sh->acc_empty[0]);
+  const uint32_t uq_empty_c0 = PAIR ? mapa_shared(smem_addr(&sh->uq_empty[0]), 0) : smem_addr(&sh->uq_empty[0]);
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&sh->full[s], 1);
@@ -166,19 +216,26 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&sh->acc_full[i], 1);
-      mbar_init(&sh->acc_empty[i], 4);
+      mbar_init(&sh->acc_empty[i], PAIR ? 8 : 4);  // the epilogue warps of every CTA of the unit
     }
     mbar_init(&sh->drain, 1);
     for (int i = 0; i < kUQ; ++i) {
       mbar_init(&sh->uq_full[i], 1);
-      mbar_init(&sh->uq_empty[i], 5);
+      // Single: MMA warp + 4 epilogue warps.  Pair (rank 0's barrier): its
+      // MMA warp and 4 epilogue warps, rank 1's producer and 4 epilogue warps.
+      mbar_init(&sh->uq_empty[i], PAIR ? 10 : 5);
     }
     sh->abort = 0;
     fence_barrier_init();
     prefetch_tensormap(&q_map);
     prefetch_tensormap(&pool_map);
   }
-  if (warp == 1) tmem_alloc(&sh->tmem_base, 2 * kAccCols);
+  if constexpr (PAIR) {
+    cluster_sync();  // both CTAs' barriers are initialised before any remote arrival
+    if (warp == 1) tmem_alloc_pair(&sh->tmem_base, 2 * kAccCols);
+  } else {
+    if (warp == 1) tmem_alloc(&sh->tmem_base, 2 * kAccCols);
+  }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -196,25 +253,45 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t ph = 0;
     uint32_t issued = 0, issued_phase = 0;  // per stage: a copy was issued / its phase parity
     bool ok = true;
-    // Units are taken dynamically: unit blockIdx.x first, then the next one
-    // from a global counter, so CTAs that drew short units take more.  Each
-    // index goes through the queue to the MMA and epilogue warps.
-    int u = blockIdx.x;
+    // Units are taken dynamically: unit (cluster) index first, then the next
+    // one from a global counter, so CTAs that drew short units take more.
+    // Each index goes through the queue to the MMA and epilogue warps (of
+    // both CTAs of a pair; rank 1's producer reads rank 0's choice).
+    int u = PAIR ? (int)(blockIdx.x >> 1) : (int)blockIdx.x;
+    const int n_slots = PAIR ? (int)(gridDim.x >> 1) : (int)gridDim.x;
     for (int j = 0; ok; ++j) {
       const int slot = j % kUQ;
-      if (!mbar_wait(&sh->uq_empty[slot], ((uint32_t)(j / kUQ) & 1u) ^ 1u, abort, a.max_polls)) {
-        ok = false;
-        break;
+      if (leader) {
+        if (!mbar_wait(&sh->uq_empty[slot], ((uint32_t)(j / kUQ) & 1u) ^ 1u, abort, a.max_polls)) {
+          ok = false;
+          break;
+        }
+        if (lane == 0) {
+          const int v = u < n_units ? u : -1;
+          sh->uq[slot] = v;
+          mbar_arrive(&sh->uq_full[slot]);
+          if constexpr (PAIR) {
+            st_cluster_u32(mapa_shared(smem_addr(&sh->uq[slot]), 1), (uint32_t)v);
+            mbar_arrive_cluster(mapa_shared(smem_addr(&sh->uq_full[slot]), 1));
+          }
+        }
+        __syncwarp();
+      } else {
+        u = take_unit<PAIR>(sh, j, uq_empty_c0, abort, a.max_polls, ok);
+        if (!ok) break;
+        if (u < 0) u = n_units;
       }
-      if (lane == 0) {
-        sh->uq[slot] = u < n_units ? u : -1;
-        mbar_arrive(&sh->uq_full[slot]);
-      }
-      __syncwarp();
       if (u >= n_units) break;
       const int4 U = a.units[u];
       const int g = U.x;
-      const int a_row = (a.q_direct ? 0 : a.bucket_off[g]) + U.y * kTcRows;
+      // This CTA's chunk; a pair's missing second chunk re-reads the first
+      // chunk's rows (its accumulator rows are never read).
+      int c = U.y;
+      if constexpr (PAIR) {
+        c = 2 * U.y + (int)rank;
+        if (c * kTcRows >= a.cnt[g]) c = 2 * U.y;
+      }
+      const int a_row = (a.q_direct ? 0 : a.bucket_off[g]) + c * kTcRows;
       const int pg0 = a.page_off[g];
       const int npg = a.page_off[g + 1] - pg0;
       const int p_beg = U.z * seg_pages, p_end = min(npg, p_beg + seg_pages);
@@ -228,11 +305,25 @@ __global__ void __launch_bounds__(kThreads, 1)
             break;
           }
           if (lane == 0) {
-            mbar_arrive_expect_tx(&sh->full[st], kABytes + (two ? kBBytes : kHalfB));
             const int x = kb * kKBlock;
-            tma_load_2d(smem_addr(st_a + st * kABytes), &q_map, x, a_row, &sh->full[st]);
-            tma_load_2d(smem_addr(st_b + st * kBBytes), &pool_map, x, y0, &sh->full[st]);
-            if (two) tma_load_2d(smem_addr(st_b + st * kBBytes + kHalfB), &pool_map, x, y1, &sh->full[st]);
+            const uint32_t dst_a = smem_addr(st_a + st * kABytes), dst_b = smem_addr(st_b + st * kBStage);
+            if constexpr (PAIR) {
+              // Both CTAs' copies complete on rank 0's barrier; rank 0
+              // expects both ranks' A rows and the tile's pages.
+              const uint32_t bar = full_c0 + st * (uint32_t)sizeof(uint64_t);
+              if (leader) mbar_arrive_expect_tx(&sh->full[st], 2 * kABytes + (two ? 2 * kHalfB : kHalfB));
+              tma_load_2d_pair(dst_a, &q_map, x, a_row, bar);
+              if (leader) {
+                tma_load_2d_pair(dst_b, &pool_map, x, y0, bar);
+              } else if (two) {
+                tma_load_2d_pair(dst_b, &pool_map, x, y1, bar);
+              }
+            } else {
+              mbar_arrive_expect_tx(&sh->full[st], kABytes + (two ? kBBytes : kHalfB));
+              tma_load_2d(dst_a, &q_map, x, a_row, &sh->full[st]);
+              tma_load_2d(dst_b, &pool_map, x, y0, &sh->full[st]);
+              if (two) tma_load_2d(dst_b + kHalfB, &pool_map, x, y1, &sh->full[st]);
+            }
           }
           __syncwarp();
           issued |= 1u << st;
@@ -243,30 +334,39 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
       }
-      int next = 0;
-      if (lane == 0) next = (int)gridDim.x + atomicAdd(a.unit_ctr, 1);
-      u = __shfl_sync(kFull, next, 0);
+      if (leader) {
+        int next = 0;
+        if (lane == 0) next = n_slots + atomicAdd(a.unit_ctr, 1);
+        u = __shfl_sync(kFull, next, 0);
+      }
     }
     if (!ok && lane == 0) {
       atomicOr(a.status, 1u);
       sh->abort = 1;
     }
-    // Drain: every copy issued has landed before the CTA exits.
+    // Drain: every copy issued has landed before the CTA exits.  A single
+    // CTA (and rank 0) polls the stage's full barrier; rank 1's copies
+    // complete on rank 0's barrier, so rank 1 polls its empty barrier, which
+    // the MMAs release only after both CTAs' copies of the stage landed.
     for (int s = 0; s < kStages; ++s) {
       if ((issued >> s) & 1u) {
-        for (uint32_t i = 0; i < a.max_polls && !mbar_try_wait(&sh->full[s], (issued_phase >> s) & 1u); ++i) {
+        const uint32_t par = (issued_phase >> s) & 1u;
+        uint64_t *bar = leader ? &sh->full[s] : &sh->empty[s];
+        for (uint32_t i = 0; i < a.max_polls && !mbar_try_wait(bar, par); ++i) {
         }
       }
     }
     __syncwarp();
   } else if (warp == 1) {
     // --------------------------------------------------------- MMA issuer
-    const uint32_t idesc = idesc_bf16_f32(kTcRows, kTileN);
+    // (rank 0 of a pair issues for both CTAs; rank 1's MMA warp only holds
+    // its share of the tensor memory allocation)
+    const uint32_t idesc = idesc_bf16_f32(PAIR ? 2 * kTcRows : kTcRows, kTileN);
     int st = 0, acc = 0;
     uint32_t ph = 0, aph = 0;
     bool ok = true;
-    for (int j = 0; ok; ++j) {
-      const int u = take_unit(sh, j, abort, a.max_polls, ok);
+    for (int j = 0; ok && leader; ++j) {
+      const int u = take_unit<PAIR>(sh, j, uq_empty_c0, abort, a.max_polls, ok);
       if (u < 0) break;
       const int4 U = a.units[u];
       const int g = U.x;
@@ -287,12 +387,20 @@ __global__ void __launch_bounds__(kThreads, 1)
           tc_fence_after();
           if (lane == 0) {
             const uint64_t ad = sw128_kmajor_desc(smem_addr(st_a + st * kABytes));
-            const uint64_t bd = sw128_kmajor_desc(smem_addr(st_b + st * kBBytes));
+            const uint64_t bd = sw128_kmajor_desc(smem_addr(st_b + st * kBStage));
 #pragma unroll
             for (int k = 0; k < kKBlock / 16; ++k) {
-              umma_bf16(d_tmem, ad + 2 * k, bd + 2 * k, idesc, (kb | k) != 0);
+              if constexpr (PAIR) {
+                umma_bf16_pair(d_tmem, ad + 2 * k, bd + 2 * k, idesc, (kb | k) != 0);
+              } else {
+                umma_bf16(d_tmem, ad + 2 * k, bd + 2 * k, idesc, (kb | k) != 0);
+              }
             }
-            umma_commit(&sh->empty[st]);
+            if constexpr (PAIR) {
+              umma_commit_pair(&sh->empty[st], 0x3);
+            } else {
+              umma_commit(&sh->empty[st]);
+            }
           }
           __syncwarp();
           if (++st == kStages) {
@@ -301,7 +409,13 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
         if (!ok) break;
-        if (lane == 0) umma_commit(&sh->acc_full[acc]);
+        if (lane == 0) {
+          if constexpr (PAIR) {
+            umma_commit_pair(&sh->acc_full[acc], 0x3);
+          } else {
+            umma_commit(&sh->acc_full[acc]);
+          }
+        }
         __syncwarp();
         if (++acc == 2) {
           acc = 0;
@@ -314,8 +428,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       sh->abort = 1;
     }
     // Drain: all MMAs issued have completed.
-    if (lane == 0) {
-      umma_commit(&sh->drain);
+    if (leader && lane == 0) {
+      if constexpr (PAIR) {
+        umma_commit_pair(&sh->drain, 0x1);
+      } else {
+        umma_commit(&sh->drain);
+      }
       for (uint32_t i = 0; i < a.max_polls && !mbar_try_wait(&sh->drain, 0); ++i) {
       }
     }
@@ -331,15 +449,19 @@ __global__ void __launch_bounds__(kThreads, 1)
     bool ok = true;
     RowTopK<K> top;
     for (int j = 0; ok; ++j) {
-      const int u = take_unit(sh, j, abort, a.max_polls, ok);
+      const int u = take_unit<PAIR>(sh, j, uq_empty_c0, abort, a.max_polls, ok);
       if (u < 0) break;
       const int4 U = a.units[u];
-      const int g = U.x, c = U.y, sg = U.z;
+      const int g = U.x, sg = U.z;
+      const int c = PAIR ? 2 * U.y + (int)rank : U.y;
       const int cg = a.cnt[g];
-      const int nq = min(kTcRows, cg - c * kTcRows);
+      const int nq = min(kTcRows, cg - c * kTcRows);  // <= 0: a pair's missing second chunk
       const bool valid = e < nq;
       const int b = valid ? a.bucket[a.bucket_off[g] + c * kTcRows + e] : 0;
-      float thr = valid ? dec_score(a.thr_enc[b]) : INFINITY;
+      float thr = valid ? -INFINITY : INFINITY;
+      // The query's shared bound, read one tile ahead: the load's latency
+      // is spent in the previous tile's work instead of stalling this one.
+      unsigned thr_pub = valid ? a.thr_enc[b] : 0u;
       float m2 = -INFINITY, l = 0.f;
       top.init();
       const int pg0 = a.page_off[g];
@@ -349,19 +471,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int p = p_beg; ok && p < p_end; p += 2) {
         const int f0 = min(kPageRows, cnt_rows - p * kPageRows);
         const int f1 = p + 1 < p_end ? min(kPageRows, cnt_rows - (p + 1) * kPageRows) : 0;
-        if (valid) thr = fmaxf(thr, dec_score(a.thr_enc[b]));  // bounds published by other units
         if (!mbar_wait(&sh->acc_full[acc], aph, abort, a.max_polls)) ok = false;
         tc_fence_after();
-        if (ok) {
-#pragma unroll 1
-          for (int ch = 0; ch < kTileN / 32; ++ch) {
+        if (ok && nq > 0) {
+          // One 32-column chunk of the accumulator row: softmax statistics,
+          // then the pairs that reach the bound into the row's top-k.
+          auto chunk = [&](const uint32_t (&r)[32], int ch) {
             const int col0 = ch * 32;
             const int fill = ch < 4 ? f0 - col0 : f1 - (col0 - kPageRows);
-            if (fill <= 0) continue;  // uniform across the warp
-            uint32_t r[32];
-            __syncwarp();             // converged for the warp-collective load
-            tmem_ld32(lane_addr + acc * kAccCols + col0, r);
-            tmem_wait_ld();
             const int nv = min(32, fill);
             const int cbase = (p - p_beg) * kPageRows + col0;  // unit column of r[0]
             uint32_t flagged = 0;
@@ -408,17 +525,50 @@ __global__ void __launch_bounds__(kThreads, 1)
               if (any) top.insert_later(__uint_as_float(xv), cbase + j);
             }
             if (valid && most > 0) thr = fmaxf(thr, top.kth(k));
+          };
+          // The chunks holding entries are a prefix (only a group's last page
+          // is partly filled, and nothing follows it).  Each chunk's load is
+          // issued before the previous chunk is processed, so the tensor
+          // memory reads overlap the arithmetic.
+          const int n_ch = f1 > 0 ? 4 + (f1 + 31) / 32 : (f0 + 31) / 32;
+          const uint32_t acc_addr = lane_addr + acc * kAccCols;
+          uint32_t ra[32], rb[32];
+          __syncwarp();  // converged for the warp-collective loads and waits
+          tmem_ld32(acc_addr, ra);
+          tmem_wait_ld(ra);
+          if (valid) thr = fmaxf(thr, dec_score(thr_pub));  // bounds published by other units
+#pragma unroll 1
+          for (int ch = 0; ch < n_ch; ch += 2) {
+            const bool has_b = ch + 1 < n_ch;  // uniform across the warp
+            __syncwarp();
+            if (has_b) tmem_ld32(acc_addr + (ch + 1) * 32, rb);
+            chunk(ra, ch);
+            __syncwarp();
+            tmem_wait_ld(rb);
+            if (!has_b) break;
+            if (ch + 2 < n_ch) tmem_ld32(acc_addr + (ch + 2) * 32, ra);
+            chunk(rb, ch + 1);
+            __syncwarp();
+            tmem_wait_ld(ra);
           }
         }
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(&sh->acc_empty[acc]);
+        if (lane == 0) {
+          if constexpr (PAIR) {
+            mbar_arrive_cluster(acc_empty_c0 + acc * (uint32_t)sizeof(uint64_t));
+          } else {
+            mbar_arrive(&sh->acc_empty[acc]);
+          }
+        }
         if (++acc == 2) {
           acc = 0;
           aph ^= 1u;
         }
-        // Share this row's bound with the query's other units.
+        // Share this row's bound with the query's other units, and read
+        // theirs for the next tile.
         if (valid && thr != -INFINITY && top.kth(k) == thr) atomicMax(&a.thr_enc[b], enc_score(thr));
+        if (valid) thr_pub = a.thr_enc[b];
       }
       if (!ok) break;
       if (valid) {
@@ -452,9 +602,18 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   tc_fence_before();
   __syncthreads();
-  if (warp == 1) {
-    tc_fence_after();
-    tmem_dealloc(tbase, 2 * kAccCols);
+  if constexpr (PAIR) {
+    cluster_sync();  // rank 0's MMAs (which use both CTAs' memory) have drained
+    if (warp == 1) {
+      tc_fence_after();
+      tmem_dealloc_pair(tbase, 2 * kAccCols);
+    }
+    cluster_sync();
+  } else {
+    if (warp == 1) {
+      tc_fence_after();
+      tmem_dealloc(tbase, 2 * kAccCols);
+    }
   }
 }
 
@@ -488,15 +647,32 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   return fn;
 }
 
-template <int K>
+template <int K, bool PAIR>
 htam_status launch_k(const TcFineArgs &a, const CUtensorMap &q_map, const CUtensorMap &pool_map, int grid,
                      cudaStream_t st) {
   static bool attr_set = false;
   if (!attr_set) {
-    HTAM_CK(cudaFuncSetAttribute(fine_tc_kernel<K>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes));
+    HTAM_CK(cudaFuncSetAttribute(fine_tc_kernel<K, PAIR>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)smem_bytes<PAIR>()));
     attr_set = true;
   }
-  fine_tc_kernel<K><<<grid, kThreads, kSmemBytes, st>>>(q_map, pool_map, a);
+  if constexpr (PAIR) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)grid, 1, 1);
+    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.dynamicSmemBytes = smem_bytes<PAIR>();
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    HTAM_CK(cudaLaunchKernelEx(&cfg, fine_tc_kernel<K, true>, q_map, pool_map, a));
+  } else {
+    fine_tc_kernel<K, false><<<grid, kThreads, smem_bytes<false>(), st>>>(q_map, pool_map, a);
+  }
   HTAM_CK_LAUNCH("fine_tc_kernel");
   return HTAM_OK;
 }
@@ -529,11 +705,17 @@ htam_status launch_gather_queries(const void *Q, int d, const int32_t *bucket, c
 }
 
 htam_status launch_fine_tc(const TcFineArgs &a, const CUtensorMap &q_map, const CUtensorMap &pool_map, int grid,
-                           cudaStream_t st) {
+                           bool pair, cudaStream_t st) {
+  if (pair) grid &= ~1;  // whole clusters
   if (grid <= 0) return HTAM_OK;
-  if (a.ke <= 8) return launch_k<8>(a, q_map, pool_map, grid, st);
-  if (a.ke <= 16) return launch_k<16>(a, q_map, pool_map, grid, st);
-  return launch_k<32>(a, q_map, pool_map, grid, st);
+  if (pair) {
+    if (a.ke <= 8) return launch_k<8, true>(a, q_map, pool_map, grid, st);
+    if (a.ke <= 16) return launch_k<16, true>(a, q_map, pool_map, grid, st);
+    return launch_k<32, true>(a, q_map, pool_map, grid, st);
+  }
+  if (a.ke <= 8) return launch_k<8, false>(a, q_map, pool_map, grid, st);
+  if (a.ke <= 16) return launch_k<16, false>(a, q_map, pool_map, grid, st);
+  return launch_k<32, false>(a, q_map, pool_map, grid, st);
 }
 
 }  // namespace htam

@@ -48,7 +48,10 @@ htam_status launch_gather_queries(const void *Q, int d, const int32_t *bucket, c
                                   const int32_t *cnt, int tc_min, const int32_t *total_rows, int64_t max_rows,
                                   void *Qg, cudaStream_t st);
 
+// pair: the units are (group, pair of 128-query chunks, segment), run by
+// clusters of two CTAs (grid rounded down to even); otherwise (group, chunk,
+// segment), one CTA each.
 htam_status launch_fine_tc(const TcFineArgs &a, const CUtensorMap &q_map, const CUtensorMap &pool_map, int grid,
-                           cudaStream_t st);
+                           bool pair, cudaStream_t st);
 
 }  // namespace htam

@@ -71,6 +71,10 @@ struct htam_memory {
   // CUDA-core fine path: stream rows through shared memory (1) or load them
   // directly (0).
   int stream_rows = 1;
+  // Tensor-core buckets of more than one 128-query chunk on SM pairs (1) or
+  // single SMs (0).  Off by default: the epilogue, not the operand feed,
+  // limits the kernel, and the pair path measured slower.
+  int tc_pairs = 0;
   CUtensorMap pool_map;
   bool pool_map_ready = false;
 };

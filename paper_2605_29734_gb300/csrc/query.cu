@@ -482,13 +482,19 @@ __global__ void bucket_pos_kernel(const uint32_t *__restrict__ bits, const int32
 // segments of seg_tc pages, smaller ones to the SIMT kernel in chunks of
 // qc_simt queries and segments of seg_simt pages.
 struct Route {
-  int tc_min, qc_simt, seg_simt, seg_tc;
+  int tc_min, qc_simt, seg_simt, seg_tc, pairs;
   __host__ __device__ bool tc(int c) const { return c >= tc_min; }
+  // Tensor-core buckets of more than one chunk run on SM pairs (when on).
+  __host__ __device__ bool pair(int c) const { return pairs && tc(c) && c > kTcRows; }
   __host__ __device__ int qc(int c) const { return tc(c) ? kTcRows : qc_simt; }
   __host__ __device__ int seg(int c) const { return tc(c) ? seg_tc : seg_simt; }
   __host__ __device__ int nseg(int c, int pages) const { return (pages + seg(c) - 1) / seg(c); }
+  // Work units of a group: (chunk, segment) pairs, or (chunk pair, segment)
+  // pairs on SM pairs.
   __host__ __device__ int64_t units(int c, int pages) const {
-    return c > 0 ? (int64_t)((c + qc(c) - 1) / qc(c)) * nseg(c, pages) : 0;
+    if (c <= 0) return 0;
+    const int64_t nch = (c + qc(c) - 1) / qc(c);
+    return (pair(c) ? (nch + 1) / 2 : nch) * nseg(c, pages);
   }
   // Tensor-core tiles (two pages each) of a group: every chunk of the bucket
   // against every page pair.
@@ -518,8 +524,9 @@ __device__ __forceinline__ int tc_seg_pages(int64_t tiles, int sms) {
 __global__ void __launch_bounds__(1024) bucket_scan_kernel(
     const int32_t *__restrict__ cnt, const int32_t *__restrict__ page_off, int G, Route rt, int sms,
     int32_t *__restrict__ bucket_off, int32_t *__restrict__ unit_off, int32_t *__restrict__ unit_off_tc,
-    int64_t *__restrict__ part_off, int32_t *__restrict__ n_units, int32_t *__restrict__ seg_tc_dev) {
-  __shared__ int64_t sh[4][1024];
+    int32_t *__restrict__ unit_off_tc2, int64_t *__restrict__ part_off, int32_t *__restrict__ n_units,
+    int32_t *__restrict__ seg_tc_dev) {
+  __shared__ int64_t sh[5][1024];
   const int tid = threadIdx.x;
   const int per = (G + 1023) / 1024;
   const int lo = min(G, tid * per), hi = min(G, lo + per);
@@ -536,48 +543,52 @@ __global__ void __launch_bounds__(1024) bucket_scan_kernel(
     __syncthreads();  // sh is reused below
     if (tid == 0) *seg_tc_dev = rt.seg_tc;
   }
-  int64_t a = 0, u = 0, t = 0, p = 0;
-  for (int g = lo; g < hi; ++g) {
-    int c = cnt[g], pages = page_off[g + 1] - page_off[g];
+  // Per list: SIMT units (u), single-SM tensor-core units (t), SM-pair
+  // tensor-core units (t2).
+  int64_t a = 0, u = 0, t = 0, t2 = 0, p = 0;
+  auto add = [&](int c, int pages) {
     a += c;
-    (rt.tc(c) ? t : u) += rt.units(c, pages);
+    (rt.pair(c) ? t2 : rt.tc(c) ? t : u) += rt.units(c, pages);
     p += (int64_t)c * rt.nseg(c, pages);
-  }
+  };
+  for (int g = lo; g < hi; ++g) add(cnt[g], page_off[g + 1] - page_off[g]);
   sh[0][tid] = a;
   sh[1][tid] = u;
   sh[2][tid] = t;
   sh[3][tid] = p;
+  sh[4][tid] = t2;
   __syncthreads();
   for (int o = 1; o < 1024; o <<= 1) {
-    int64_t v[4] = {0, 0, 0, 0};
+    int64_t v[5] = {0, 0, 0, 0, 0};
     if (tid >= o) {
-      for (int i = 0; i < 4; ++i) v[i] = sh[i][tid - o];
+      for (int i = 0; i < 5; ++i) v[i] = sh[i][tid - o];
     }
     __syncthreads();
-    for (int i = 0; i < 4; ++i) sh[i][tid] += v[i];
+    for (int i = 0; i < 5; ++i) sh[i][tid] += v[i];
     __syncthreads();
   }
   a = sh[0][tid] - a;
   u = sh[1][tid] - u;
   t = sh[2][tid] - t;
   p = sh[3][tid] - p;
+  t2 = sh[4][tid] - t2;
   for (int g = lo; g < hi; ++g) {
-    int c = cnt[g], pages = page_off[g + 1] - page_off[g];
     bucket_off[g] = (int32_t)a;
     unit_off[g] = (int32_t)u;
     unit_off_tc[g] = (int32_t)t;
+    unit_off_tc2[g] = (int32_t)t2;
     part_off[g] = p;
-    a += c;
-    (rt.tc(c) ? t : u) += rt.units(c, pages);
-    p += (int64_t)c * rt.nseg(c, pages);
+    add(cnt[g], page_off[g + 1] - page_off[g]);
   }
   if (tid == 1023) {
     bucket_off[G] = (int32_t)a;
     unit_off[G] = (int32_t)u;
     unit_off_tc[G] = (int32_t)t;
+    unit_off_tc2[G] = (int32_t)t2;
     part_off[G] = p;
     n_units[0] = (int32_t)u;
     n_units[1] = (int32_t)t;
+    n_units[2] = (int32_t)t2;
   }
 }
 
@@ -591,9 +602,11 @@ __global__ void bucket_fill_kernel(const uint32_t *__restrict__ bits, int G, int
                                    const int32_t *__restrict__ seg_tc_dev,
                                    const int32_t *__restrict__ unit_off,
                                    const int32_t *__restrict__ unit_off_tc,
+                                   const int32_t *__restrict__ unit_off_tc2,
                                    int32_t *__restrict__ bucket, int32_t *__restrict__ bucket_group,
                                    int4 *__restrict__ units,
-                                   int4 *__restrict__ units_tc) {
+                                   int4 *__restrict__ units_tc,
+                                   int4 *__restrict__ units_tc2) {
   int g = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   int lane = threadIdx.x & 31;
   if (g >= G) return;
@@ -624,7 +637,8 @@ __global__ void bucket_fill_kernel(const uint32_t *__restrict__ bits, int G, int
   const int pages = page_off[g + 1] - page_off[g];
   const int nseg = rt.nseg(c, pages);
   const int n_u = (int)rt.units(c, pages);
-  int4 *dst = rt.tc(c) ? units_tc + unit_off_tc[g] : units + unit_off[g];
+  // (group, chunk or chunk pair, segment)
+  int4 *dst = rt.pair(c) ? units_tc2 + unit_off_tc2[g] : rt.tc(c) ? units_tc + unit_off_tc[g] : units + unit_off[g];
   for (int u = lane; u < n_u; u += 32) dst[u] = make_int4(g, u / nseg, u % nseg, 0);
 }
 
@@ -1152,7 +1166,7 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   const bool tc_ok = m->dtype == HTAM_BF16 && ke <= kTcMaxK && m->tc_min <= B;
   // seg_tc here is the shortest tensor-core segment (for the bounds below);
   // the kernels take the one bucket_scan_kernel chooses.
-  const Route rt{tc_ok ? m->tc_min : INT_MAX, qc, kSimtSegPages, kTcSegPagesMin};
+  const Route rt{tc_ok ? m->tc_min : INT_MAX, qc, kSimtSegPages, kTcSegPagesMin, m->tc_pairs};
 
   // Upper bound of the partial records: every query in the buckets of the
   // k_g groups with the most page segments (counted with the shorter
@@ -1178,10 +1192,10 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   const bool edge_table = er && (int64_t)B * er->P > G;
   const int wpq = warps_per_query(B, m->sm_count);  // warps per query in top-k and merge
   size_t need = Carver::round(sizeof(float) * (size_t)planes * B * G) + 2 * Carver::round(sizeof(uint32_t) * (size_t)G * W) +
-                5 * Carver::round(sizeof(int32_t) * (G + 1)) + Carver::round(sizeof(int64_t) * (G + 1)) +
+                6 * Carver::round(sizeof(int32_t) * (G + 4)) + Carver::round(sizeof(int64_t) * (G + 1)) +
                 2 * Carver::round(sizeof(int32_t)) + (er ? Carver::round(sizeof(int32_t) * (size_t)B * er->P) : 0) +
                 (edge_table ? Carver::round(sizeof(float) * (size_t)G * G) : 0) +
-                3 * Carver::round(sizeof(int32_t) * rows) + 2 * Carver::round(sizeof(int4) * max_units) +
+                3 * Carver::round(sizeof(int32_t) * rows) + 3 * Carver::round(sizeof(int4) * max_units) +
                 Carver::round(sizeof(float2) * max_parts) + Carver::round(sizeof(float) * max_parts * ke) +
                 Carver::round(sizeof(int32_t) * max_parts * ke) + Carver::round(sizeof(unsigned) * B) +
                 Carver::round(qg_bytes) + (smp ? Carver::round(sizeof(float) * (size_t)B * G) : 0) + (flat ? Carver::round(sizeof(int32_t) * rows) + Carver::round(sizeof(int32_t) * kg) : 0) + 8192;
@@ -1195,10 +1209,11 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   int32_t *bucket_off = cv.take<int32_t>(G + 1);
   int32_t *unit_off = cv.take<int32_t>(G + 1);
   int32_t *unit_off_tc = cv.take<int32_t>(G + 1);
+  int32_t *unit_off_tc2 = cv.take<int32_t>(G + 1);
   int64_t *part_off = cv.take<int64_t>(G + 1);
-  int32_t *n_units = cv.take<int32_t>(G + 1);  // [0] SIMT units, [1] tensor-core units
+  int32_t *n_units = cv.take<int32_t>(4);  // SIMT, single-SM and SM-pair tensor-core units
   int32_t *seg_tc = cv.take<int32_t>(1);        // pages per tensor-core unit, chosen on the device
-  int32_t *tc_ctr = cv.take<int32_t>(1);        // tensor-core units taken from the shared counter
+  int32_t *tc_ctr = cv.take<int32_t>(2);        // tensor-core units taken from the shared counters
   int32_t *edge_prefix = er ? cv.take<int32_t>((size_t)B * er->P) : nullptr;
   float *edge_u = edge_table ? cv.take<float>((size_t)G * G) : nullptr;
   int32_t *bucket = cv.take<int32_t>(rows);
@@ -1206,6 +1221,7 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   int32_t *pos = cv.take<int32_t>(rows);
   int4 *units = cv.take<int4>(max_units);
   int4 *units_tc = cv.take<int4>(max_units);
+  int4 *units_tc2 = cv.take<int4>(max_units);
   float2 *part_ml = cv.take<float2>(max_parts);
   float *part_s = cv.take<float>(max_parts * ke);
   int32_t *part_id = cv.take<int32_t>(max_parts * ke);
@@ -1312,11 +1328,11 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   bucket_pos_kernel<<<(unsigned)ceil_div(rows, 256), 256, 0, st>>>(bits, wpre, W, group_idx, rows, kg, pos);
   HTAM_CK_LAUNCH("bucket_pos_kernel");
   bucket_scan_kernel<<<1, 1024, 0, st>>>(cnt, m->page_off, G, rt, m->sm_count, bucket_off, unit_off,
-                                         unit_off_tc, part_off, n_units, seg_tc);
+                                         unit_off_tc, unit_off_tc2, part_off, n_units, seg_tc);
   HTAM_CK_LAUNCH("bucket_scan_kernel");
   bucket_fill_kernel<<<(unsigned)ceil_div((int64_t)G * 32, 256), 256, 0, st>>>(
-      bits, G, W, bucket_off, cnt, m->page_off, rt, seg_tc, unit_off, unit_off_tc, bucket, bucket_group, units,
-      units_tc);
+      bits, G, W, bucket_off, cnt, m->page_off, rt, seg_tc, unit_off, unit_off_tc, unit_off_tc2, bucket,
+      bucket_group, units, units_tc, units_tc2);
   HTAM_CK_LAUNCH("bucket_fill_kernel");
   mark.launched(5);
   CUtensorMap q_map;
@@ -1331,7 +1347,7 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
     s = flat ? make_bf16_tile_map(&q_map, queries, B, d, kTcRows) : make_bf16_tile_map(&q_map, qg, rows, d, kTcRows);
     if (s != HTAM_OK) return s;
     HTAM_CK(cudaMemsetAsync(thr_enc, 0, sizeof(unsigned) * B, st));
-    HTAM_CK(cudaMemsetAsync(tc_ctr, 0, sizeof(int32_t), st));
+    HTAM_CK(cudaMemsetAsync(tc_ctr, 0, 2 * sizeof(int32_t), st));
     if (!flat) {
       s = launch_gather_queries(queries, d, bucket, bucket_group, cnt, rt.tc_min, bucket_off + G, rows, qg, st);
       if (s != HTAM_OK) return s;
@@ -1365,7 +1381,17 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
     TcFineArgs ta{units_tc, n_units + 1, tc_ctr, bucket, bucket_off, cnt, m->page_list, m->page_off, m->count, m->slot_id,
                   part_off, d, seg_tc, ke, 1.4426950408889634f / p.tau, part_ml, part_s, part_id, thr_enc,
                   m->status, kMaxPolls, flat ? 1 : 0};
-    s = launch_fine_tc(ta, q_map, m->pool_map, (int)std::min<int64_t>(max_units, m->sm_count), st);
+    if (rt.pairs && B > kTcRows) {
+      // Buckets of several chunks on SM pairs, then the one-chunk buckets.
+      TcFineArgs tp = ta;
+      tp.units = units_tc2;
+      tp.n_units = n_units + 2;
+      tp.unit_ctr = tc_ctr + 1;
+      s = launch_fine_tc(tp, q_map, m->pool_map, 2 * (int)std::min<int64_t>(max_units, m->sm_count / 2), true, st);
+      if (s != HTAM_OK) return s;
+      mark.launched();
+    }
+    s = launch_fine_tc(ta, q_map, m->pool_map, (int)std::min<int64_t>(max_units, m->sm_count), false, st);
     if (s != HTAM_OK) return s;
     mark.launched();
     mark.end();

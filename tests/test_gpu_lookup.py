@@ -232,6 +232,25 @@ def test_tensor_core_and_cuda_core_paths(htam, case, min_bucket):
         assert ran["fine_tc"][1] == 0
 
 
+@pytest.mark.parametrize("case", TC_CASES[:2])
+def test_tensor_core_sm_pairs(htam, case):
+    """Buckets of more than 128 queries on SM pairs (cta_group::2: two
+    128-query chunks per M=256 MMA, each SM staging half of every entry tile),
+    against the oracle and bit for bit against the single-SM kernel."""
+    n, g, d, b, kg, ke = case
+    entries, gid, centres = _rand_memory(n, d, g, torch.bfloat16, seed=n + d)
+    q = _rand_queries(b, d, torch.bfloat16, seed=n + d, centres=centres)
+    mem = htam.Memory(entries, gid, g)
+    mem.set_tensor_core_min_bucket(1)
+    single = mem.query(q, kg, ke, tau=0.5, epsilon=0.05)
+    mem.set_tensor_core_pairs(True)
+    mem.read_phase_timing()
+    out = _check(htam, mem, entries, gid, g, q, kg, ke, tau=0.5, eps=0.05)
+    assert mem.read_phase_timing()["fine_tc"][1] == 2  # the pair kernel, then the one-chunk kernel
+    for k in ("group_idx", "entry_idx", "entry_score", "entry_weight", "lse"):
+        assert torch.equal(out[k], single[k]), k
+
+
 STREAM_CASES = [
     # n, groups, d, dtype, batch, k_groups, k_entries
     (6000, 30, 4096, torch.bfloat16, 20, 3, 16),   # 8 KiB rows: three ring slots per warp
@@ -611,10 +630,15 @@ def test_tuning_defaults_follow_row_length_and_round_trip(htam):
         mem = htam.Memory(e, gid, 3)
         assert mem.get_tuning(htam.HTAM_TUNE_TC_MIN_BUCKET) == want
         assert mem.get_tuning(htam.HTAM_TUNE_STREAM_ROWS) == 1
+        assert mem.get_tuning(htam.HTAM_TUNE_TC_PAIRS) == 0
         mem.set_tensor_core_min_bucket(7)
         mem.set_stream_rows(False)
+        mem.set_tensor_core_pairs(True)
         assert mem.get_tuning(htam.HTAM_TUNE_TC_MIN_BUCKET) == 7
         assert mem.get_tuning(htam.HTAM_TUNE_STREAM_ROWS) == 0
+        assert mem.get_tuning(htam.HTAM_TUNE_TC_PAIRS) == 1
+        with pytest.raises(htam.HtamError):
+            mem.set_tuning(htam.HTAM_TUNE_TC_PAIRS, 2)
         with pytest.raises(htam.HtamError):
             mem.get_tuning(99)
         with pytest.raises(htam.HtamError):
