@@ -105,6 +105,7 @@ __global__ void __launch_bounds__(256) coarse_scores_simt_kernel(
 // eight warps so that the grid fills the GPU; many take one warp each.
 constexpr int kSelWarps = 8;
 constexpr int kSelBatch = 8;
+constexpr int kSelSortMin = 4;  // more candidates than this in a chunk: sort and merge
 
 template <int WPQ>
 __global__ void __launch_bounds__(kSelWarps * 32, 1) group_topk_kernel(const float *__restrict__ s1, int planes,
@@ -146,7 +147,18 @@ __global__ void __launch_bounds__(kSelWarps * 32, 1) group_topk_kernel(const flo
       const int g0 = base + u * kStep;
       const bool valid = cv[u] > 0;
       const float sc = valid ? sv[u] : -INFINITY;
-      unsigned mask = __ballot_sync(kFullMask, valid && better(sc, g0 + lane, ts, ti));
+      const bool pass = valid && better(sc, g0 + lane, ts, ti);
+      unsigned mask = __ballot_sync(kFullMask, pass);
+      if (kg <= 32 && __popc(mask) > kSelSortMin) {
+        // Many candidates (the list is still filling): sort the chunk across
+        // the warp and merge it whole.
+        float cs = pass ? sc : -INFINITY;
+        int ci = pass ? g0 + lane : INT_MAX;
+        warp_sort32(cs, ci);
+        L.merge32(cs, ci);
+        L.kth(kg, ts, ti);
+        continue;
+      }
       while (mask) {
         const int src = __ffs(mask) - 1;
         mask &= mask - 1;
