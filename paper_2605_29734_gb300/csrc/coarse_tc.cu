@@ -9,7 +9,8 @@
 // lo (128-byte swizzle), one thread issues per slice four MMAs against hi and
 // four against lo into the same fp32 accumulator in tensor memory, and four
 // epilogue warps write the scores (-inf for empty groups) for the top-k
-// kernel.  When the tiles alone would leave SMs idle (few queries), the K
+// kernel, turned around in shared memory so that each store covers a
+// 128-byte row segment.  When the tiles alone would leave SMs idle (few queries), the K
 // slices are split over blockIdx.z: split z writes its partial dot products
 // to plane z of the output, and the top-k kernel adds the planes in order.
 // Every mbarrier wait is bounded.
@@ -144,10 +145,15 @@ __global__ void __launch_bounds__(kCThreads, 1)
     __syncwarp();
   } else {
     const int quad = warp & 3;
-    const int b = m0 + quad * 32 + lane;
     if (!mbar_wait(&sh->acc_full, 0, abort, max_polls)) ok = false;
     tc_fence_after();
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // the stages' async-proxy use is over
     if (ok) {
+      // Every MMA is done, so the operand stages are free: each warp turns
+      // its 32 rows x 32 columns around in a padded shared-memory square and
+      // writes whole 128-byte row segments (one per store instruction).
+      float *sq = reinterpret_cast<float *>(smem) + (warp - 2) * 32 * 33;
+      const int row0 = m0 + quad * 32;
       const uint32_t lane_addr = tbase + (static_cast<uint32_t>(quad * 32) << 16);
       for (int ch = 0; ch < kCN / 32; ++ch) {
         const int g0 = n0 + ch * 32;
@@ -155,14 +161,17 @@ __global__ void __launch_bounds__(kCThreads, 1)
         uint32_t r[32];
         __syncwarp();
         tmem_ld32(lane_addr + ch * 32, r);
-        tmem_wait_ld();
-        if (b < B) {
+        tmem_wait_ld(r);
 #pragma unroll
-          for (int j = 0; j < 32; ++j) {
-            const int g = g0 + j;
-            if (g < G) s1[(int64_t)b * G + g] = count[g] > 0 ? __uint_as_float(r[j]) : -INFINITY;
-          }
+        for (int j = 0; j < 32; ++j) sq[lane * 33 + j] = __uint_as_float(r[j]);
+        __syncwarp();
+        const int g = g0 + lane;
+        const bool gin = g < G;
+        const bool empty = !gin || count[g] == 0;
+        for (int i = 0; i < 32 && row0 + i < B; ++i) {
+          if (gin) s1[(int64_t)(row0 + i) * G + g] = empty ? -INFINITY : sq[i * 33 + lane];
         }
+        __syncwarp();
       }
     }
   }
