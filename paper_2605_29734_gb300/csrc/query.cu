@@ -530,77 +530,98 @@ __device__ __forceinline__ int tc_seg_pages(int64_t tiles, int sms) {
 
 // Single block: chooses the pages per tensor-core unit from the total
 // tensor-core tiles (written to seg_tc_dev), then per group the bucket size
-// c_g, its work units (in the SIMT or the tensor-core list) and its partial
-// records c_g * nseg_g, with exclusive scans over the groups.
-// n_units = {SIMT units, tensor-core units}.
+// c_g, its work units (in the SIMT, one-SM or SM-pair tensor-core list) and
+// its partial records c_g * nseg_g, with exclusive scans over the groups
+// (warp shuffles, then one pass over the 32 warp totals).
+// n_units = {SIMT units, one-SM tensor-core units, SM-pair units}.
 __global__ void __launch_bounds__(1024) bucket_scan_kernel(
     const int32_t *__restrict__ cnt, const int32_t *__restrict__ page_off, int G, Route rt, int sms,
     int32_t *__restrict__ bucket_off, int32_t *__restrict__ unit_off, int32_t *__restrict__ unit_off_tc,
     int32_t *__restrict__ unit_off_tc2, int64_t *__restrict__ part_off, int32_t *__restrict__ n_units,
     int32_t *__restrict__ seg_tc_dev) {
-  __shared__ int64_t sh[5][1024];
-  const int tid = threadIdx.x;
+  constexpr int kVals = 5;  // bucket rows, SIMT units, one-SM units, records, SM-pair units
+  __shared__ int64_t wsum[kVals][32];
+  __shared__ int64_t tiles_sh;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int per = (G + 1023) / 1024;
   const int lo = min(G, tid * per), hi = min(G, lo + per);
   {
     int64_t x = 0;
     for (int g = lo; g < hi; ++g) x += rt.tc_tiles(cnt[g], page_off[g + 1] - page_off[g]);
-    sh[0][tid] = x;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(kFullMask, x, o);
+    if (lane == 0) wsum[0][warp] = x;
     __syncthreads();
-    for (int o = 512; o > 0; o >>= 1) {
-      if (tid < o) sh[0][tid] += sh[0][tid + o];
-      __syncthreads();
+    if (tid == 0) {
+      int64_t t = 0;
+      for (int w = 0; w < 32; ++w) t += wsum[0][w];
+      tiles_sh = t;
     }
-    rt.seg_tc = tc_seg_pages(sh[0][0], sms);
-    __syncthreads();  // sh is reused below
+    __syncthreads();
+    rt.seg_tc = tc_seg_pages(tiles_sh, sms);
     if (tid == 0) *seg_tc_dev = rt.seg_tc;
   }
-  // Per list: SIMT units (u), single-SM tensor-core units (t), SM-pair
-  // tensor-core units (t2).
-  int64_t a = 0, u = 0, t = 0, t2 = 0, p = 0;
-  auto add = [&](int c, int pages) {
-    a += c;
-    (rt.pair(c) ? t2 : rt.tc(c) ? t : u) += rt.units(c, pages);
-    p += (int64_t)c * rt.nseg(c, pages);
+  int64_t v[kVals] = {0, 0, 0, 0, 0};
+  auto add = [&](int64_t (&acc)[kVals], int c, int pages) {
+    const int64_t u = rt.units(c, pages);
+    const bool pr = rt.pair(c), tc = rt.tc(c);
+    acc[0] += c;
+    acc[1] += tc ? 0 : u;
+    acc[2] += tc && !pr ? u : 0;
+    acc[3] += (int64_t)c * rt.nseg(c, pages);
+    acc[4] += pr ? u : 0;
   };
-  for (int g = lo; g < hi; ++g) add(cnt[g], page_off[g + 1] - page_off[g]);
-  sh[0][tid] = a;
-  sh[1][tid] = u;
-  sh[2][tid] = t;
-  sh[3][tid] = p;
-  sh[4][tid] = t2;
-  __syncthreads();
-  for (int o = 1; o < 1024; o <<= 1) {
-    int64_t v[5] = {0, 0, 0, 0, 0};
-    if (tid >= o) {
-      for (int i = 0; i < 5; ++i) v[i] = sh[i][tid - o];
+  for (int g = lo; g < hi; ++g) add(v, cnt[g], page_off[g + 1] - page_off[g]);
+  // Inclusive scan within the warp, then the warp totals.
+  int64_t incl[kVals];
+#pragma unroll
+  for (int i = 0; i < kVals; ++i) {
+    incl[i] = v[i];
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int64_t t = __shfl_up_sync(kFullMask, incl[i], o);
+      if (lane >= o) incl[i] += t;
     }
-    __syncthreads();
-    for (int i = 0; i < 5; ++i) sh[i][tid] += v[i];
-    __syncthreads();
   }
-  a = sh[0][tid] - a;
-  u = sh[1][tid] - u;
-  t = sh[2][tid] - t;
-  p = sh[3][tid] - p;
-  t2 = sh[4][tid] - t2;
+  __syncthreads();  // wsum[0] was read above
+  if (lane == 31) {
+#pragma unroll
+    for (int i = 0; i < kVals; ++i) wsum[i][warp] = incl[i];
+  }
+  __syncthreads();
+  if (warp == 0) {
+#pragma unroll
+    for (int i = 0; i < kVals; ++i) {
+      int64_t x = wsum[i][lane];
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int64_t t = __shfl_up_sync(kFullMask, x, o);
+        if (lane >= o) x += t;
+      }
+      wsum[i][lane] = x;  // inclusive over warps
+    }
+  }
+  __syncthreads();
+  int64_t run[kVals];
+#pragma unroll
+  for (int i = 0; i < kVals; ++i) run[i] = (warp > 0 ? wsum[i][warp - 1] : 0) + incl[i] - v[i];
   for (int g = lo; g < hi; ++g) {
-    bucket_off[g] = (int32_t)a;
-    unit_off[g] = (int32_t)u;
-    unit_off_tc[g] = (int32_t)t;
-    unit_off_tc2[g] = (int32_t)t2;
-    part_off[g] = p;
-    add(cnt[g], page_off[g + 1] - page_off[g]);
+    bucket_off[g] = (int32_t)run[0];
+    unit_off[g] = (int32_t)run[1];
+    unit_off_tc[g] = (int32_t)run[2];
+    part_off[g] = run[3];
+    unit_off_tc2[g] = (int32_t)run[4];
+    add(run, cnt[g], page_off[g + 1] - page_off[g]);
   }
   if (tid == 1023) {
-    bucket_off[G] = (int32_t)a;
-    unit_off[G] = (int32_t)u;
-    unit_off_tc[G] = (int32_t)t;
-    unit_off_tc2[G] = (int32_t)t2;
-    part_off[G] = p;
-    n_units[0] = (int32_t)u;
-    n_units[1] = (int32_t)t;
-    n_units[2] = (int32_t)t2;
+    bucket_off[G] = (int32_t)run[0];
+    unit_off[G] = (int32_t)run[1];
+    unit_off_tc[G] = (int32_t)run[2];
+    part_off[G] = run[3];
+    unit_off_tc2[G] = (int32_t)run[4];
+    n_units[0] = (int32_t)run[1];
+    n_units[1] = (int32_t)run[2];
+    n_units[2] = (int32_t)run[4];
   }
 }
 
