@@ -202,6 +202,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   TcSmem *sh = reinterpret_cast<TcSmem *>(st_b + kStages * kBStage);
   volatile int *abort = &sh->abort;
 
+  // No units (every bucket went to the CUDA cores): leave before setting up
+  // (uniform over the grid, so a CTA pair leaves together).
+  if (*a.n_units == 0) return;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t rank = PAIR ? cluster_ctarank() : 0u;
   const bool leader = rank == 0;

@@ -639,7 +639,16 @@ __global__ void bucket_fill_kernel(const uint32_t *__restrict__ bits, int G, int
                                    int32_t *__restrict__ bucket, int32_t *__restrict__ bucket_group,
                                    int4 *__restrict__ units,
                                    int4 *__restrict__ units_tc,
-                                   int4 *__restrict__ units_tc2) {
+                                   int4 *__restrict__ units_tc2,
+                                   unsigned *__restrict__ thr_zero, int B,
+                                   int32_t *__restrict__ ctr_zero) {
+  // Also clears the tensor-core kernel's shared bounds and unit counters
+  // (when given), which no earlier kernel of the query touches.
+  if (thr_zero) {
+    const int64_t t0 = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+    for (int64_t t = t0; t < B; t += (int64_t)gridDim.x * blockDim.x) thr_zero[t] = 0u;
+    if (t0 < 2) ctr_zero[t0] = 0;
+  }
   int g = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   int lane = threadIdx.x & 31;
   if (g >= G) return;
@@ -1365,7 +1374,7 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   HTAM_CK_LAUNCH("bucket_scan_kernel");
   bucket_fill_kernel<<<(unsigned)ceil_div((int64_t)G * 32, 256), 256, 0, st>>>(
       bits, G, W, bucket_off, cnt, m->page_off, rt, seg_tc, unit_off, unit_off_tc, unit_off_tc2, bucket,
-      bucket_group, units, units_tc, units_tc2);
+      bucket_group, units, units_tc, units_tc2, tc_ok ? thr_enc : nullptr, B, tc_ctr);
   HTAM_CK_LAUNCH("bucket_fill_kernel");
   mark.launched(5);
   CUtensorMap q_map;
@@ -1379,8 +1388,6 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
     }
     s = flat ? make_bf16_tile_map(&q_map, queries, B, d, kTcRows) : make_bf16_tile_map(&q_map, qg, rows, d, kTcRows);
     if (s != HTAM_OK) return s;
-    HTAM_CK(cudaMemsetAsync(thr_enc, 0, sizeof(unsigned) * B, st));
-    HTAM_CK(cudaMemsetAsync(tc_ctr, 0, 2 * sizeof(int32_t), st));
     if (!flat) {
       s = launch_gather_queries(queries, d, bucket, bucket_group, cnt, rt.tc_min, bucket_off + G, rows, qg, st);
       if (s != HTAM_OK) return s;
