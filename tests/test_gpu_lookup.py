@@ -192,6 +192,40 @@ def test_dimension_extremes(htam, d):
     _check(htam, mem, entries, gid, 12, q, 3, 9)
 
 
+def test_most_groups_and_largest_k(htam):
+    """65,536 groups (the most a memory takes), most of them empty or with a
+    few entries, k_groups = k_entries = 64; the flat scan and the policy draws
+    over all of them."""
+    from parity import compare_flat, compare_sampled
+
+    n, g, d = 150000, 65536, 64
+    gid = (torch.arange(n, device=DEV, dtype=torch.int64) * 7919 % 50000).to(torch.int32)  # 50,000 non-empty
+    entries, gid, centres = _rand_memory(n, d, g, torch.bfloat16, seed=41, gid=gid)
+    q = _rand_queries(96, d, torch.bfloat16, seed=41)
+    mem = htam.Memory(entries, gid, g)
+    rows = np.arange(0, 96, 6)
+    _check(htam, mem, entries, gid, g, q, 64, 64, tau=0.3, eps=0.01, rows=rows)
+    flat = mem.query_flat(q, 64, tau=0.3, epsilon=0.01)
+    torch.cuda.synchronize()
+    problems = compare_flat(flat, to_numpy(entries), to_numpy(q), 64, 0.3, 0.01, "bf16", rows=rows)
+    assert not problems, "\n".join(problems[:20])
+    smp = mem.query_sampled(q, 64, 32, seed=3, offset=4, tau=0.3, epsilon=0.01)
+    torch.cuda.synchronize()
+    problems = compare_sampled(smp, to_numpy(entries), to_numpy(gid), g, to_numpy(q), 64, 32, 0.3, 0.01, "bf16",
+                               seed=3, offset=4, rows=rows)
+    assert not problems, "\n".join(problems[:20])
+    assert mem.device_status() == htam.HTAM_OK
+
+
+def test_large_batch_one_warp_per_query(htam):
+    """20,000 queries: selection and merge take one warp per query, and the
+    tensor-core buckets hold thousands of queries (many 128-query chunks)."""
+    entries, gid, centres = _rand_memory(60000, 128, 400, torch.bfloat16, seed=42)
+    q = _rand_queries(20000, 128, torch.bfloat16, seed=42, centres=centres)
+    mem = htam.Memory(entries, gid, 400)
+    _check(htam, mem, entries, gid, 400, q, 8, 24, tau=0.5, eps=0.02, rows=np.linspace(0, 19999, 40).astype(int))
+
+
 def test_large_groups_many_segments_ragged_tail(htam):
     # one group of 5,000 rows (40 pages, ragged last page) and a few small ones
     gid = torch.cat([torch.zeros(5000, dtype=torch.int32), torch.arange(1, 6, dtype=torch.int32).repeat(7)])
