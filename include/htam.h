@@ -309,7 +309,8 @@ htam_status htam_memory_group_keys(const htam_memory *m, float *keys,
  * check, ECUDA if the stream reports an error, OK otherwise. */
 htam_status htam_device_status(htam_memory *m, void *cuda_stream);
 
-/* Phases of htam_query, for the timing counters below. */
+/* Phases of htam_query (and of htam_append_transitions), for the timing
+ * counters below. */
 typedef enum {
   HTAM_PHASE_COARSE = 0, /* group-key scores */
   HTAM_PHASE_SELECT = 1, /* top-k_groups per query */
@@ -318,7 +319,10 @@ typedef enum {
   HTAM_PHASE_FINE_TC = 4, /* entry scores of large buckets on the tensor cores */
   HTAM_PHASE_MERGE = 5,   /* per-query merge, weights, outputs */
   HTAM_PHASE_PREFIX = 6,  /* reduced queries of htam_query_prefix */
-  HTAM_N_PHASES = 7
+  HTAM_PHASE_APPEND = 7,  /* htam_append_transitions / htam_append_assign, from the
+                             batch's group count to the last key update (including
+                             the host round trip in between) */
+  HTAM_N_PHASES = 8
 } htam_phase;
 
 /* Tuning knobs of htam_query (all paths return the same results within the
@@ -349,9 +353,9 @@ htam_status htam_set_tuning(htam_memory *m, htam_tuning key, int32_t value);
  * *value.  Errors: EINVAL (m or value NULL, unknown key). */
 htam_status htam_get_tuning(const htam_memory *m, htam_tuning key, int32_t *value);
 
-/* Turns CUDA-event timing of each htam_query phase on (1) or off (0).  While
- * on, every query records a pair of events around each phase on its stream
- * (a few microseconds of host work per query). */
+/* Turns CUDA-event timing of each htam_query phase (and of each append) on
+ * (1) or off (0).  While on, every call records a pair of events around each
+ * phase on its stream (a few microseconds of host work per call). */
 htam_status htam_set_phase_timing(htam_memory *m, int enable);
 
 /* Synchronises `cuda_stream`, then writes, for the htam_query calls since the

@@ -205,10 +205,9 @@ htam_status launch_coarse_tc(const void *queries, int B, int d, const __nv_bfloa
   if (s == HTAM_OK) s = make_bf16_tile_map(&hi_map, hi, G, d, kPageRows);
   if (s == HTAM_OK) s = make_bf16_tile_map(&lo_map, lo, G, d, kPageRows);
   if (s != HTAM_OK) return s;
-  static bool attr_set = false;
-  if (!attr_set) {
+  static std::atomic<uint64_t> attr_set{0};
+  if (first_on_device(attr_set)) {
     HTAM_CK(cudaFuncSetAttribute(coarse_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kCSmem));
-    attr_set = true;
   }
   const int nk = (int)ceil_div((int64_t)d, kCKBlock);
   const int kb_per = (int)ceil_div((int64_t)nk, splits);

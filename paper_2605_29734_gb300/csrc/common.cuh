@@ -1,6 +1,8 @@
 // common.cuh -- shared device/host helpers of the HTAM lookup library.
 #pragma once
 
+#include <atomic>
+
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -166,5 +168,15 @@ __device__ __forceinline__ float warp_sum(float v) {
 }
 
 __host__ __device__ inline int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
+
+// True the first time it is called for the current device with this flag
+// word (one bit per device): per-device, once-only setup such as a kernel's
+// shared-memory limit, safe to call from several host threads.
+inline bool first_on_device(std::atomic<uint64_t> &done) {
+  int dev = 0;
+  cudaGetDevice(&dev);
+  const uint64_t bit = uint64_t(1) << (dev & 63);
+  return (done.fetch_or(bit) & bit) == 0;
+}
 
 }  // namespace htam

@@ -653,11 +653,10 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 template <int K, bool PAIR>
 htam_status launch_k(const TcFineArgs &a, const CUtensorMap &q_map, const CUtensorMap &pool_map, int grid,
                      cudaStream_t st) {
-  static bool attr_set = false;
-  if (!attr_set) {
+  static std::atomic<uint64_t> attr_set{0};
+  if (first_on_device(attr_set)) {
     HTAM_CK(cudaFuncSetAttribute(fine_tc_kernel<K, PAIR>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  (int)smem_bytes<PAIR>()));
-    attr_set = true;
   }
   if constexpr (PAIR) {
     cudaLaunchConfig_t cfg = {};

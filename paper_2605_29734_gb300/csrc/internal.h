@@ -131,8 +131,9 @@ void free_impl(htam_memory *m);
 // ids go to `dst` (`count` of them; it may be `gid` itself) or, when dst is
 // NULL, to m->assign_buf; *ids_out points at them.  The scratch is
 // m->assign_buf, grown on demand (which synchronises the device).
+struct PhaseMark;
 htam_status assign_nearest(htam_memory *m, const void *entries, const int32_t *gid, int64_t count, int32_t *dst,
-                           const int32_t **ids_out, cudaStream_t st);
+                           const int32_t **ids_out, cudaStream_t st, PhaseMark *mark = nullptr);
 
 // Weights alpha_1..alpha_P of a prefix (Eq. 10), passed by value to the
 // reduction kernel.
@@ -151,6 +152,10 @@ struct PhaseMark {
   cudaStream_t st;
   int phase = -1;
   PhaseMark(htam_memory *mem, cudaStream_t s) : m(mem), st(s) {}
+  // A phase begun but not ended (an error return) is dropped.
+  ~PhaseMark() {
+    if (m->timing && m->ev_phase.size() * 2 == m->ev_used + 2) m->ev_phase.pop_back();
+  }
   void begin(int p);
   void end();
   void launched(int n = 1) { m->phase_launches[phase] += n; }

@@ -272,6 +272,9 @@ static htam_status add_rows(htam_memory *m, const void *entries, const int32_t *
   KeyGroup *kgroups = cv.take<KeyGroup>(G);
   double *partial = cv.take<double>((size_t)max_segs * d);
 
+  PhaseMark mark(m, st);
+  mark.begin(HTAM_PHASE_APPEND);
+
   // 1. Per-group counts of the batch and the group-id range check.
   std::vector<int32_t> h_b(G + 2);
   auto count_batch = [&](const int32_t *ids) -> htam_status {
@@ -279,6 +282,7 @@ static htam_status add_rows(htam_memory *m, const void *entries, const int32_t *
     int blocks = (int)std::min<int64_t>(ceil_div(count, 256), 4096);
     count_groups_kernel<<<blocks, 256, 0, st>>>(ids, count, G, bcount, bcount + G, bcount + G + 1);
     HTAM_CK_LAUNCH("count_groups_kernel");
+    mark.launched();
     HTAM_CK(cudaMemcpyAsync(h_b.data(), bcount, sizeof(int32_t) * (G + 2), cudaMemcpyDeviceToHost, st));
     HTAM_CK(cudaStreamSynchronize(st));
     return HTAM_OK;
@@ -293,7 +297,7 @@ static htam_status add_rows(htam_memory *m, const void *entries, const int32_t *
     for (int64_t c : m->h_count) any |= c > 0;
     if (!any) return HTAM_EINVAL;
     const int32_t *ids = nullptr;
-    s = assign_nearest(m, entries, gid, count, assigned, &ids, st);
+    s = assign_nearest(m, entries, gid, count, assigned, &ids, st, &mark);
     if (s != HTAM_OK) return s;
     gid = ids;
     s = count_batch(gid);
@@ -357,6 +361,7 @@ static htam_status add_rows(htam_memory *m, const void *entries, const int32_t *
   HTAM_CK_LAUNCH("chunk_scan_kernel");
   chunk_place_kernel<<<(unsigned)ceil_div(n_chunks * 32, 256), 256, 0, st>>>(gid, count, chunk, n_chunks, hist, pos);
   HTAM_CK_LAUNCH("chunk_place_kernel");
+  mark.launched(3);
 
   // 4. Copy rows into their slots.
   int vec_per_row = d * m->elem_bytes / 16;
@@ -364,6 +369,7 @@ static htam_status add_rows(htam_memory *m, const void *entries, const int32_t *
       static_cast<const uint4 *>(entries), gid, pos, count, vec_per_row, m->page_list, m->page_off,
       static_cast<uint4 *>(m->pool), m->slot_id, m->n);
   HTAM_CK_LAUNCH("place_rows_kernel");
+  mark.launched();
 
   // 5. Keys of the touched groups.
   if (!h_segs.empty()) {
@@ -379,12 +385,14 @@ static htam_status add_rows(htam_memory *m, const void *entries, const int32_t *
     dim3 g2((unsigned)h_kg.size(), (unsigned)std::min<int64_t>(ceil_div(d, 256), 16));
     key_finalize_kernel<<<g2, 256, 0, st>>>(kgroups, partial, d, m->csum, m->cent, m->cent_hi, m->cent_lo);
     HTAM_CK_LAUNCH("key_finalize_kernel");
+    mark.launched(2);
   }
 
   // 6. New device counts and host mirrors.
   std::vector<int32_t> h_c32(G);
   for (int32_t g = 0; g < G; ++g) h_c32[g] = (int32_t)new_count[g];
   HTAM_CK(cudaMemcpyAsync(m->count, h_c32.data(), sizeof(int32_t) * G, cudaMemcpyHostToDevice, st));
+  mark.end();
   // The host vectors above are pageable, so cudaMemcpyAsync staged them
   // before returning; the key and segment tables in scratch are read by the
   // kernels above in stream order, before any later call on the stream can

@@ -1469,7 +1469,7 @@ __global__ void assign_fill_kernel(const int32_t *gid, const int32_t *__restrict
 }  // namespace
 
 htam_status assign_nearest(htam_memory *m, const void *entries, const int32_t *gid, int64_t count, int32_t *dst,
-                           const int32_t **ids_out, cudaStream_t st) {
+                           const int32_t **ids_out, cudaStream_t st, PhaseMark *mark) {
   const int G = m->n_groups, d = m->d;
   // Rows per pass: the [rows, G] score matrix stays within 16 MiB per plane.
   const int64_t R = std::max<int64_t>(1, std::min<int64_t>(count, (int64_t(1) << 22) / G));
@@ -1520,6 +1520,7 @@ htam_status assign_nearest(htam_memory *m, const void *entries, const int32_t *g
     HTAM_CK_LAUNCH("group_topk_kernel");
     assign_fill_kernel<<<(unsigned)ceil_div(rb, 256), 256, 0, st>>>(gid + r0, pick, rb, ids + r0);
     HTAM_CK_LAUNCH("assign_fill_kernel");
+    if (mark) mark->launched(3);
   }
   *ids_out = ids;
   return HTAM_OK;

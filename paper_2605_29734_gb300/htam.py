@@ -30,7 +30,7 @@ EXPORTS = (
     "htam_read_phase_timing", "htam_free_memory", "htam_status_string", "htam_last_error",
     "htam_selftest_wait_timeout",
 )
-PHASES = ("coarse", "select", "bucket", "fine", "fine_tc", "merge", "prefix")
+PHASES = ("coarse", "select", "bucket", "fine", "fine_tc", "merge", "prefix", "append")
 
 
 class HtamError(RuntimeError):
