@@ -279,10 +279,14 @@ def oracle_rate(w, entries_np, gid_np, queries_np, target_s, cent=None, counts=N
     t0 = time.perf_counter()
     call(queries_np[:probe])
     t_probe = max(time.perf_counter() - t0, 1e-6)
-    n = int(min(queries_np.shape[0], max(probe, probe * target_s / t_probe)))
+    # Enough queries for about target_s seconds, cycling through the batches
+    # when they hold fewer (at most 64 passes).
+    n = int(min(64 * queries_np.shape[0], max(probe, probe * target_s / t_probe)))
     n = max(probe, (n // threads) * threads) if n >= threads else n
+    reps = -(-n // queries_np.shape[0])
+    qs = np.concatenate([queries_np] * reps)[:n] if reps > 1 else queries_np[:n]
     t0 = time.perf_counter()
-    call(queries_np[:n])
+    call(qs)
     dt = time.perf_counter() - t0
     return n / dt, n, dt, threads, cent, counts
 
@@ -307,6 +311,8 @@ def run_reference(args, world, rank):
         n_sample = min(threads, q_np.shape[0])
     else:
         _, n_sample, _, _, _, _ = oracle_rate(w, entries_np, gid_np, q_np, per_step_target, cent, counts)
+        if n_sample > q_np.shape[0]:  # the sample cycles through the batches
+            q_np = np.concatenate([q_np] * -(-n_sample // q_np.shape[0]))
     times = []
     for i in range(args.warmup + args.steps):
         off = (i * n_sample) % max(1, q_np.shape[0] - n_sample + 1)
