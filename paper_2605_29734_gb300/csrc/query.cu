@@ -442,22 +442,25 @@ __global__ void flat_fill_kernel(const int32_t *__restrict__ list, int64_t rows,
 
 // ---------------------------------------------------------------- bucketing
 
+// The bucketing steps are device functions over one row or one group, run
+// by a kernel each or, for small batches, all in one block.
+__device__ __forceinline__ void bucket_bits_row(int64_t t, const int32_t *__restrict__ gidx, int kg, int W,
+                                                uint32_t *bits) {
+  const int b = (int)(t / kg);
+  const int32_t g = gidx[t];
+  if (g >= 0) atomicOr(&bits[(int64_t)g * W + (b >> 5)], 1u << (b & 31));
+}
+
 __global__ void bucket_bits_kernel(const int32_t *__restrict__ gidx, int B, int kg, int W,
                                    uint32_t *__restrict__ bits) {
-  int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-  if (t >= (int64_t)B * kg) return;
-  int b = (int)(t / kg);
-  int32_t g = gidx[t];
-  if (g >= 0) atomicOr(&bits[(int64_t)g * W + (b >> 5)], 1u << (b & 31));
+  const int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  if (t < (int64_t)B * kg) bucket_bits_row(t, gidx, kg, W, bits);
 }
 
 // One warp per group: the bucket size c_g and, per bitmap word, how many of
 // the group's queries come before it (wpre[g][w]).
-__global__ void bucket_count_kernel(const uint32_t *__restrict__ bits, int G, int W,
-                                    int32_t *__restrict__ cnt, int32_t *__restrict__ wpre) {
-  int g = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  int lane = threadIdx.x & 31;
-  if (g >= G) return;
+__device__ __forceinline__ void bucket_count_group(int g, int lane, const uint32_t *bits, int W,
+                                                   int32_t *__restrict__ cnt, int32_t *__restrict__ wpre) {
   int running = 0;
   for (int w0 = 0; w0 < W; w0 += 32) {
     const int w = w0 + lane;
@@ -474,19 +477,29 @@ __global__ void bucket_count_kernel(const uint32_t *__restrict__ bits, int G, in
   if (lane == 0) cnt[g] = running;
 }
 
+__global__ void bucket_count_kernel(const uint32_t *__restrict__ bits, int G, int W,
+                                    int32_t *__restrict__ cnt, int32_t *__restrict__ wpre) {
+  const int g = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  if (g < G) bucket_count_group(g, threadIdx.x & 31, bits, W, cnt, wpre);
+}
+
 // pos[b][j] = rank of query b in the bucket of its j-th selected group: the
 // group's queries before b's bitmap word plus those before b within it.
-__global__ void bucket_pos_kernel(const uint32_t *__restrict__ bits, const int32_t *__restrict__ wpre, int W,
-                                  const int32_t *__restrict__ gidx, int64_t rows, int kg,
-                                  int32_t *__restrict__ pos) {
-  const int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-  if (t >= rows) return;
+__device__ __forceinline__ void bucket_pos_row(int64_t t, const uint32_t *bits, const int32_t *wpre, int W,
+                                               const int32_t *__restrict__ gidx, int kg, int32_t *__restrict__ pos) {
   const int g = gidx[t];
   if (g < 0) return;
   const int b = (int)(t / kg);
   const int w = b >> 5;
   const uint32_t below = bits[(int64_t)g * W + w] & ((1u << (b & 31)) - 1u);
   pos[t] = wpre[(int64_t)g * W + w] + __popc(below);
+}
+
+__global__ void bucket_pos_kernel(const uint32_t *__restrict__ bits, const int32_t *__restrict__ wpre, int W,
+                                  const int32_t *__restrict__ gidx, int64_t rows, int kg,
+                                  int32_t *__restrict__ pos) {
+  const int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  if (t < rows) bucket_pos_row(t, bits, wpre, W, gidx, kg, pos);
 }
 
 // Which fine kernel scores a group's bucket: buckets of at least tc_min
@@ -534,7 +547,7 @@ __device__ __forceinline__ int tc_seg_pages(int64_t tiles, int sms) {
 // its partial records c_g * nseg_g, with exclusive scans over the groups
 // (warp shuffles, then one pass over the 32 warp totals).
 // n_units = {SIMT units, one-SM tensor-core units, SM-pair units}.
-__global__ void __launch_bounds__(1024) bucket_scan_kernel(
+__device__ void bucket_scan_block(
     const int32_t *__restrict__ cnt, const int32_t *__restrict__ page_off, int G, Route rt, int sms,
     int32_t *__restrict__ bucket_off, int32_t *__restrict__ unit_off, int32_t *__restrict__ unit_off_tc,
     int32_t *__restrict__ unit_off_tc2, int64_t *__restrict__ part_off, int32_t *__restrict__ n_units,
@@ -625,34 +638,25 @@ __global__ void __launch_bounds__(1024) bucket_scan_kernel(
   }
 }
 
-// One warp per group: bucket[g] lists its queries in increasing order.
-// Also writes the group's work units (group, chunk, segment) to the list of
-// the kernel that will score them, and the group of every bucket row.
-__global__ void bucket_fill_kernel(const uint32_t *__restrict__ bits, int G, int W,
-                                   const int32_t *__restrict__ bucket_off,
-                                   const int32_t *__restrict__ cnt,
-                                   const int32_t *__restrict__ page_off, Route rt,
-                                   const int32_t *__restrict__ seg_tc_dev,
-                                   const int32_t *__restrict__ unit_off,
-                                   const int32_t *__restrict__ unit_off_tc,
-                                   const int32_t *__restrict__ unit_off_tc2,
-                                   int32_t *__restrict__ bucket, int32_t *__restrict__ bucket_group,
-                                   int4 *__restrict__ units,
-                                   int4 *__restrict__ units_tc,
-                                   int4 *__restrict__ units_tc2,
-                                   unsigned *__restrict__ thr_zero, int B,
-                                   int32_t *__restrict__ ctr_zero) {
-  // Also clears the tensor-core kernel's shared bounds and unit counters
-  // (when given), which no earlier kernel of the query touches.
-  if (thr_zero) {
-    const int64_t t0 = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-    for (int64_t t = t0; t < B; t += (int64_t)gridDim.x * blockDim.x) thr_zero[t] = 0u;
-    if (t0 < 2) ctr_zero[t0] = 0;
-  }
-  int g = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  int lane = threadIdx.x & 31;
-  if (g >= G) return;
-  rt.seg_tc = *seg_tc_dev;
+__global__ void __launch_bounds__(1024) bucket_scan_kernel(
+    const int32_t *__restrict__ cnt, const int32_t *__restrict__ page_off, int G, Route rt, int sms,
+    int32_t *__restrict__ bucket_off, int32_t *__restrict__ unit_off, int32_t *__restrict__ unit_off_tc,
+    int32_t *__restrict__ unit_off_tc2, int64_t *__restrict__ part_off, int32_t *__restrict__ n_units,
+    int32_t *__restrict__ seg_tc_dev) {
+  bucket_scan_block(cnt, page_off, G, rt, sms, bucket_off, unit_off, unit_off_tc, unit_off_tc2, part_off, n_units,
+                    seg_tc_dev);
+}
+
+__device__ __forceinline__ void bucket_fill_group(int g, int lane, const uint32_t *bits, int W,
+                                                  const int32_t *__restrict__ bucket_off,
+                                                  const int32_t *__restrict__ cnt,
+                                                  const int32_t *__restrict__ page_off, const Route &rt,
+                                                  const int32_t *__restrict__ unit_off,
+                                                  const int32_t *__restrict__ unit_off_tc,
+                                                  const int32_t *__restrict__ unit_off_tc2,
+                                                  int32_t *__restrict__ bucket, int32_t *__restrict__ bucket_group,
+                                                  int4 *__restrict__ units, int4 *__restrict__ units_tc,
+                                                  int4 *__restrict__ units_tc2) {
   int running = 0;
   const int base = bucket_off[g];
   for (int w0 = 0; w0 < W; w0 += 32) {
@@ -683,6 +687,88 @@ __global__ void bucket_fill_kernel(const uint32_t *__restrict__ bits, int G, int
   int4 *dst = rt.pair(c) ? units_tc2 + unit_off_tc2[g] : rt.tc(c) ? units_tc + unit_off_tc[g] : units + unit_off[g];
   for (int u = lane; u < n_u; u += 32) dst[u] = make_int4(g, u / nseg, u % nseg, 0);
 }
+
+// One warp per group: bucket[g] lists its queries in increasing order.
+// Also writes the group's work units (group, chunk, segment) to the list of
+// the kernel that will score them, and the group of every bucket row.
+__global__ void bucket_fill_kernel(const uint32_t *__restrict__ bits, int G, int W,
+                                   const int32_t *__restrict__ bucket_off,
+                                   const int32_t *__restrict__ cnt,
+                                   const int32_t *__restrict__ page_off, Route rt,
+                                   const int32_t *__restrict__ seg_tc_dev,
+                                   const int32_t *__restrict__ unit_off,
+                                   const int32_t *__restrict__ unit_off_tc,
+                                   const int32_t *__restrict__ unit_off_tc2,
+                                   int32_t *__restrict__ bucket, int32_t *__restrict__ bucket_group,
+                                   int4 *__restrict__ units,
+                                   int4 *__restrict__ units_tc,
+                                   int4 *__restrict__ units_tc2,
+                                   unsigned *__restrict__ thr_zero, int B,
+                                   int32_t *__restrict__ ctr_zero) {
+  // Also clears the tensor-core kernel's shared bounds and unit counters
+  // (when given), which no earlier kernel of the query touches.
+  if (thr_zero) {
+    const int64_t t0 = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+    for (int64_t t = t0; t < B; t += (int64_t)gridDim.x * blockDim.x) thr_zero[t] = 0u;
+    if (t0 < 2) ctr_zero[t0] = 0;
+  }
+  const int g = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  rt.seg_tc = *seg_tc_dev;
+  if (g < G) {
+    bucket_fill_group(g, threadIdx.x & 31, bits, W, bucket_off, cnt, page_off, rt, unit_off, unit_off_tc,
+                      unit_off_tc2, bucket, bucket_group, units, units_tc, units_tc2);
+  }
+}
+
+// The whole bucketing in one block for small batches (the bitmap in shared
+// memory): the steps of the kernels above in order, a block barrier between
+// them, one launch instead of five plus a memset.
+struct BucketSmallArgs {
+  const int32_t *gidx;
+  int B, kg, G, W;
+  const int32_t *page_off;
+  Route rt;
+  int sms;
+  int32_t *cnt, *wpre, *pos, *bucket_off, *unit_off, *unit_off_tc, *unit_off_tc2;
+  int64_t *part_off;
+  int32_t *n_units, *seg_tc_dev, *bucket, *bucket_group;
+  int4 *units, *units_tc, *units_tc2;
+  unsigned *thr_zero;
+  int32_t *ctr_zero;
+};
+// One block pays off only for small problems: the 65k workload (256 groups x
+// 8 words, 2,048 rows) gains 3 us, the 8-query one 13 us, while 512 groups x
+// 32 words (8,192 rows) already run faster as five kernels.
+constexpr int kBucketSmallWords = 4096;  // bitmap words held in shared memory (16 KiB)
+constexpr int64_t kBucketSmallRows = 4096;
+
+__global__ void __launch_bounds__(1024) bucket_small_kernel(BucketSmallArgs a) {
+  extern __shared__ uint32_t sbits[];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int64_t rows = (int64_t)a.B * a.kg;
+  const int words = a.G * a.W;
+  for (int i = tid; i < words; i += 1024) sbits[i] = 0u;
+  if (a.thr_zero) {
+    for (int i = tid; i < a.B; i += 1024) a.thr_zero[i] = 0u;
+    if (tid < 2) a.ctr_zero[tid] = 0;
+  }
+  __syncthreads();
+  for (int64_t t = tid; t < rows; t += 1024) bucket_bits_row(t, a.gidx, a.kg, a.W, sbits);
+  __syncthreads();
+  for (int g = warp; g < a.G; g += 32) bucket_count_group(g, lane, sbits, a.W, a.cnt, a.wpre);
+  __syncthreads();  // counts and word prefixes (global) visible to the block
+  bucket_scan_block(a.cnt, a.page_off, a.G, a.rt, a.sms, a.bucket_off, a.unit_off, a.unit_off_tc, a.unit_off_tc2,
+                    a.part_off, a.n_units, a.seg_tc_dev);
+  __syncthreads();
+  Route rt = a.rt;
+  rt.seg_tc = *a.seg_tc_dev;
+  for (int64_t t = tid; t < rows; t += 1024) bucket_pos_row(t, sbits, a.wpre, a.W, a.gidx, a.kg, a.pos);
+  for (int g = warp; g < a.G; g += 32) {
+    bucket_fill_group(g, lane, sbits, a.W, a.bucket_off, a.cnt, a.page_off, rt, a.unit_off, a.unit_off_tc,
+                      a.unit_off_tc2, a.bucket, a.bucket_group, a.units, a.units_tc, a.units_tc2);
+  }
+}
+
 
 // ------------------------------------------------------------ fine (SIMT)
 
@@ -1362,21 +1448,35 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
 
   // 2. Buckets: group -> queries, work units, partial-record offsets.
   mark.begin(HTAM_PHASE_BUCKET);
-  HTAM_CK(cudaMemsetAsync(bits, 0, sizeof(uint32_t) * (size_t)G * W, st));
-  bucket_bits_kernel<<<(unsigned)ceil_div(rows, 256), 256, 0, st>>>(group_idx, B, kg, W, bits);
-  HTAM_CK_LAUNCH("bucket_bits_kernel");
-  bucket_count_kernel<<<(unsigned)ceil_div((int64_t)G * 32, 256), 256, 0, st>>>(bits, G, W, cnt, wpre);
-  HTAM_CK_LAUNCH("bucket_count_kernel");
-  bucket_pos_kernel<<<(unsigned)ceil_div(rows, 256), 256, 0, st>>>(bits, wpre, W, group_idx, rows, kg, pos);
-  HTAM_CK_LAUNCH("bucket_pos_kernel");
-  bucket_scan_kernel<<<1, 1024, 0, st>>>(cnt, m->page_off, G, rt, m->sm_count, bucket_off, unit_off,
-                                         unit_off_tc, unit_off_tc2, part_off, n_units, seg_tc);
-  HTAM_CK_LAUNCH("bucket_scan_kernel");
-  bucket_fill_kernel<<<(unsigned)ceil_div((int64_t)G * 32, 256), 256, 0, st>>>(
-      bits, G, W, bucket_off, cnt, m->page_off, rt, seg_tc, unit_off, unit_off_tc, unit_off_tc2, bucket,
-      bucket_group, units, units_tc, units_tc2, tc_ok ? thr_enc : nullptr, B, tc_ctr);
-  HTAM_CK_LAUNCH("bucket_fill_kernel");
-  mark.launched(5);
+  if ((int64_t)G * W <= kBucketSmallWords && rows <= kBucketSmallRows) {
+    BucketSmallArgs ba{group_idx, B, kg, G, W, m->page_off, rt, m->sm_count, cnt, wpre, pos, bucket_off, unit_off,
+                       unit_off_tc, unit_off_tc2, part_off, n_units, seg_tc, bucket, bucket_group, units, units_tc,
+                       units_tc2, tc_ok ? thr_enc : nullptr, tc_ctr};
+    static std::atomic<uint64_t> attr_set{0};
+    if (first_on_device(attr_set)) {
+      HTAM_CK(cudaFuncSetAttribute(bucket_small_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                   (int)(sizeof(uint32_t) * kBucketSmallWords)));
+    }
+    bucket_small_kernel<<<1, 1024, sizeof(uint32_t) * (size_t)G * W, st>>>(ba);
+    HTAM_CK_LAUNCH("bucket_small_kernel");
+    mark.launched();
+  } else {
+    HTAM_CK(cudaMemsetAsync(bits, 0, sizeof(uint32_t) * (size_t)G * W, st));
+    bucket_bits_kernel<<<(unsigned)ceil_div(rows, 256), 256, 0, st>>>(group_idx, B, kg, W, bits);
+    HTAM_CK_LAUNCH("bucket_bits_kernel");
+    bucket_count_kernel<<<(unsigned)ceil_div((int64_t)G * 32, 256), 256, 0, st>>>(bits, G, W, cnt, wpre);
+    HTAM_CK_LAUNCH("bucket_count_kernel");
+    bucket_pos_kernel<<<(unsigned)ceil_div(rows, 256), 256, 0, st>>>(bits, wpre, W, group_idx, rows, kg, pos);
+    HTAM_CK_LAUNCH("bucket_pos_kernel");
+    bucket_scan_kernel<<<1, 1024, 0, st>>>(cnt, m->page_off, G, rt, m->sm_count, bucket_off, unit_off,
+                                           unit_off_tc, unit_off_tc2, part_off, n_units, seg_tc);
+    HTAM_CK_LAUNCH("bucket_scan_kernel");
+    bucket_fill_kernel<<<(unsigned)ceil_div((int64_t)G * 32, 256), 256, 0, st>>>(
+        bits, G, W, bucket_off, cnt, m->page_off, rt, seg_tc, unit_off, unit_off_tc, unit_off_tc2, bucket,
+        bucket_group, units, units_tc, units_tc2, tc_ok ? thr_enc : nullptr, B, tc_ctr);
+    HTAM_CK_LAUNCH("bucket_fill_kernel");
+    mark.launched(5);
+  }
   CUtensorMap q_map;
   if (tc_ok) {
     // Queries of tensor-core buckets in bucket order (the MMA's A operand),
