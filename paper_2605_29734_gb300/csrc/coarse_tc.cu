@@ -5,7 +5,7 @@
 // MMA as the sum of two bf16 matrices, hi = bf16(c) and lo = bf16(c - hi),
 // so that q . hi + q . lo carries the key to about 2^-17 of its size while
 // both operands stay bf16 (the query itself is bf16 already).  Each CTA owns
-// one 128-query x 256-group tile: TMA stages 64-column K slices of Q, hi and
+// one 128-query x 128-group tile (two CTAs per SM): TMA stages 64-column K slices of Q, hi and
 // lo (128-byte swizzle), one thread issues per slice four MMAs against hi and
 // four against lo into the same fp32 accumulator in tensor memory, and four
 // epilogue warps write the scores (-inf for empty groups) for the top-k
@@ -31,10 +31,10 @@ using namespace sm100;
 constexpr int kCStages = 2;
 constexpr int kCKBlock = 64;
 constexpr int kCM = 128;                           // queries per tile (MMA M)
-constexpr int kCN = 256;                           // groups per tile (MMA N)
+constexpr int kCN = 128;                           // groups per tile (MMA N): one page of keys
 constexpr int kCABytes = kCM * kCKBlock * 2;       // 16 KiB
-constexpr int kCBBytes = kCN * kCKBlock * 2;       // 32 KiB (hi or lo)
-constexpr int kCHalf = kCBBytes / 2;
+constexpr int kCBBytes = kCN * kCKBlock * 2;       // 16 KiB (hi or lo)
+constexpr int kCPerSM = 2;                         // CTAs resident per SM (96 KiB of stages each)
 constexpr int kCThreads = 192;
 
 struct __align__(8) CoarseBars {
@@ -47,7 +47,7 @@ struct __align__(8) CoarseBars {
 
 constexpr size_t kCSmem = 1024 + kCStages * (kCABytes + 2 * kCBBytes) + sizeof(CoarseBars);
 
-__global__ void __launch_bounds__(kCThreads, 1)
+__global__ void __launch_bounds__(kCThreads, kCPerSM)
     coarse_tc_kernel(const __grid_constant__ CUtensorMap q_map, const __grid_constant__ CUtensorMap hi_map,
                      const __grid_constant__ CUtensorMap lo_map, int d, int kb_per, const int32_t *__restrict__ count,
                      int B, int G, float *__restrict__ s1, unsigned *status, uint32_t max_polls) {
@@ -60,7 +60,6 @@ __global__ void __launch_bounds__(kCThreads, 1)
   volatile int *abort = &sh->abort;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int m0 = blockIdx.x * kCM, n0 = blockIdx.y * kCN;
-  const bool two = n0 + kPageRows < G;  // second half of the group tile exists
   const int nk_all = (d + kCKBlock - 1) / kCKBlock;
   const int kb0 = blockIdx.z * kb_per;                // this split's K slices: [kb0, kb0 + nk)
   const int nk = min(nk_all, kb0 + kb_per) - kb0;     // >= 1 by the launch
@@ -91,16 +90,12 @@ __global__ void __launch_bounds__(kCThreads, 1)
         break;
       }
       if (lane == 0) {
-        const uint32_t bytes = kCABytes + 2u * (two ? kCBBytes : kCHalf);
+        const uint32_t bytes = kCABytes + 2u * kCBBytes;
         mbar_arrive_expect_tx(&sh->full[st], bytes);
         const int x = (kb0 + kb) * kCKBlock;
         tma_load_2d(smem_addr(st_a + st * kCABytes), &q_map, x, m0, &sh->full[st]);
         tma_load_2d(smem_addr(st_hi + st * kCBBytes), &hi_map, x, n0, &sh->full[st]);
         tma_load_2d(smem_addr(st_lo + st * kCBBytes), &lo_map, x, n0, &sh->full[st]);
-        if (two) {
-          tma_load_2d(smem_addr(st_hi + st * kCBBytes + kCHalf), &hi_map, x, n0 + kPageRows, &sh->full[st]);
-          tma_load_2d(smem_addr(st_lo + st * kCBBytes + kCHalf), &lo_map, x, n0 + kPageRows, &sh->full[st]);
-        }
       }
       __syncwarp();
       if (++st == kCStages) {
@@ -192,7 +187,8 @@ __global__ void __launch_bounds__(kCThreads, 1)
 int coarse_tc_splits(int B, int d, int G, int sm_count) {
   const int64_t tiles = ceil_div((int64_t)B, kCM) * ceil_div((int64_t)G, kCN);
   const int nk = (int)ceil_div((int64_t)d, kCKBlock);
-  const int want = (int)std::max<int64_t>(1, std::min<int64_t>(nk, sm_count / std::max<int64_t>(1, tiles)));
+  const int want =
+      (int)std::max<int64_t>(1, std::min<int64_t>(nk, kCPerSM * sm_count / std::max<int64_t>(1, tiles)));
   const int kb_per = (int)ceil_div((int64_t)nk, want);
   return (int)ceil_div((int64_t)nk, kb_per);
 }
