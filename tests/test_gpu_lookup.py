@@ -285,6 +285,47 @@ def test_tensor_core_sm_pairs(htam, case):
         assert torch.equal(out[k], single[k]), k
 
 
+@pytest.mark.parametrize("b,g,kg", [(512, 64, 8), (513, 64, 8), (64, 2048, 4), (33, 4096, 8)])
+def test_bucketing_in_one_block_and_in_five_kernels(htam, b, g, kg):
+    """Batches on both sides of the one-block bucketing limits (4,096 rows,
+    4,096 bitmap words) against the oracle."""
+    entries, gid, centres = _rand_memory(20000, 64, g, torch.bfloat16, seed=b + g)
+    q = _rand_queries(b, 64, torch.bfloat16, seed=b + g, centres=centres)
+    mem = htam.Memory(entries, gid, g)
+    _check(htam, mem, entries, gid, g, q, kg, 12, tau=0.6, eps=0.02, rows=np.linspace(0, b - 1, 24).astype(int))
+
+
+def test_flat_scan_on_sm_pairs(htam):
+    """The flat scan with the SM-pair kernel: every group's bucket holds all
+    300 queries (three chunks, the pair of the third one half empty)."""
+    from parity import compare_flat
+
+    entries, gid, centres = _rand_memory(30000, 256, 20, torch.bfloat16, seed=51)
+    q = _rand_queries(300, 256, torch.bfloat16, seed=51, centres=centres)
+    mem = htam.Memory(entries, gid, 20)
+    single = mem.query_flat(q, 16, tau=0.5)
+    mem.set_tensor_core_pairs(True)
+    out = mem.query_flat(q, 16, tau=0.5)
+    torch.cuda.synchronize()
+    problems = compare_flat(out, to_numpy(entries), to_numpy(q), 16, 0.5, 0.0, "bf16", rows=np.arange(0, 300, 7))
+    assert not problems, "\n".join(problems[:20])
+    for k in single:
+        assert torch.equal(out[k], single[k]), k
+
+
+def test_append_phase_is_timed_and_counted(htam):
+    entries, gid, _ = _rand_memory(2000, 64, 10, torch.bfloat16, seed=52)
+    mem = htam.Memory(entries, gid, 10, capacity=3000)
+    mem.read_phase_timing()
+    mem.set_phase_timing(True)
+    e, g, _ = _rand_memory(500, 64, 10, torch.bfloat16, seed=53)
+    mem.append(e, g)
+    ran = mem.read_phase_timing()
+    mem.set_phase_timing(False)
+    assert ran["append"][0] > 0 and ran["append"][1] >= 7
+    assert ran["queries"] == 0
+
+
 STREAM_CASES = [
     # n, groups, d, dtype, batch, k_groups, k_entries
     (6000, 30, 4096, torch.bfloat16, 20, 3, 16),   # 8 KiB rows: three ring slots per warp
