@@ -107,16 +107,16 @@ constexpr int kSelWarps = 8;
 constexpr int kSelBatch = 8;
 constexpr int kSelSortMin = 4;  // more candidates than this in a chunk: sort and merge
 
-template <int WPQ>
-__global__ void __launch_bounds__(kSelWarps * 32, 1) group_topk_kernel(const float *__restrict__ s1, int planes,
-                                                                    int B, int G,
-                                                                    const int32_t *__restrict__ count, int kg,
-                                                                    int32_t *__restrict__ gidx,
-                                                                    float *__restrict__ gscore) {
-  __shared__ float ls[kSelWarps][64];
-  __shared__ int li[kSelWarps][64];
+template <int WPQ, int NW = (WPQ > kSelWarps ? WPQ : kSelWarps)>
+__global__ void __launch_bounds__(NW * 32, 1) group_topk_kernel(const float *__restrict__ s1, int planes,
+                                                             int B, int G,
+                                                             const int32_t *__restrict__ count, int kg,
+                                                             int32_t *__restrict__ gidx,
+                                                             float *__restrict__ gscore) {
+  __shared__ float ls[NW][64];
+  __shared__ int li[NW][64];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int b = blockIdx.x * (kSelWarps / WPQ) + warp / WPQ;
+  const int b = blockIdx.x * (NW / WPQ) + warp / WPQ;
   const int sw = warp % WPQ;  // this warp's place in the team
   const bool live = b < B;    // uniform per warp
   const int64_t plane = (int64_t)B * G;
@@ -219,6 +219,11 @@ __global__ void __launch_bounds__(kSelWarps * 32, 1) group_topk_kernel(const flo
 // Warps per query for B queries: eight while B * 8 warps stay under about
 // two full waves of the GPU (16 warps per SM), else one.
 static int warps_per_query(int B, int sm_count) { return (int64_t)B * 8 <= 2LL * 16 * sm_count ? 8 : 1; }
+// Group selection: teams of 32 warps (one 1,024-thread block per query) when
+// even that keeps the grid within two blocks per SM.
+static int select_warps_per_query(int B, int sm_count) {
+  return (int64_t)B <= sm_count ? 32 : warps_per_query(B, sm_count);
+}
 
 // Stage-1 scores from a transition-edge table (the router of Eq. 9 with the
 // linear utility of App. B.6 and the weights of Eq. 10): one thread per
@@ -575,7 +580,8 @@ __device__ void bucket_scan_block(
     if (tid == 0) *seg_tc_dev = rt.seg_tc;
   }
   int64_t v[kVals] = {0, 0, 0, 0, 0};
-  auto add = [&](int64_t (&acc)[kVals], int c, int pages) {
+  auto add = [&](int64_t (&acc)[kVals], int g) {
+    const int c = cnt[g], pages = page_off[g + 1] - page_off[g];
     const int64_t u = rt.units(c, pages);
     const bool pr = rt.pair(c), tc = rt.tc(c);
     acc[0] += c;
@@ -584,7 +590,7 @@ __device__ void bucket_scan_block(
     acc[3] += (int64_t)c * rt.nseg(c, pages);
     acc[4] += pr ? u : 0;
   };
-  for (int g = lo; g < hi; ++g) add(v, cnt[g], page_off[g + 1] - page_off[g]);
+  for (int g = lo; g < hi; ++g) add(v, g);
   // Inclusive scan within the warp, then the warp totals.
   int64_t incl[kVals];
 #pragma unroll
@@ -624,7 +630,7 @@ __device__ void bucket_scan_block(
     unit_off_tc[g] = (int32_t)run[2];
     part_off[g] = run[3];
     unit_off_tc2[g] = (int32_t)run[4];
-    add(run, cnt[g], page_off[g + 1] - page_off[g]);
+    add(run, g);
   }
   if (tid == 1023) {
     bucket_off[G] = (int32_t)run[0];
@@ -1428,7 +1434,11 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
       sel = policy_keys;
       sel_planes = 1;
     }
-    if (wpq == 8) {
+    const int swpq = select_warps_per_query(B, m->sm_count);
+    if (swpq == 32) {
+      group_topk_kernel<32><<<(unsigned)B, 32 * 32, 0, st>>>(sel, sel_planes, B, G, m->count, kg, group_idx,
+                                                            group_score);
+    } else if (swpq == 8) {
       group_topk_kernel<8><<<(unsigned)B, kSelWarps * 32, 0, st>>>(sel, sel_planes, B, G, m->count, kg, group_idx,
                                                                    group_score);
     } else {
