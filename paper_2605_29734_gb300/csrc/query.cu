@@ -220,7 +220,7 @@ __global__ void __launch_bounds__(NW * 32, 1) group_topk_kernel(const float *__r
 // two full waves of the GPU (16 warps per SM), else one.
 static int warps_per_query(int B, int sm_count) { return (int64_t)B * 8 <= 2LL * 16 * sm_count ? 8 : 1; }
 // Group selection: teams of 32 warps (one 1,024-thread block per query) when
-// even that keeps the grid within two blocks per SM.
+// the batch has no more queries than there are SMs.
 static int select_warps_per_query(int B, int sm_count) {
   return (int64_t)B <= sm_count ? 32 : warps_per_query(B, sm_count);
 }
