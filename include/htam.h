@@ -330,10 +330,9 @@ typedef enum {
  *  HTAM_TUNE_TC_MIN_BUCKET: when a group was selected by at least this many
  *    queries of a batch, its entries are scored against them on the tensor
  *    cores (tcgen05, 128 queries per tile); smaller buckets are scored on the
- *    CUDA cores.  Needs a bf16 memory and k_entries <= 32.  Default 2 for
- *    d <= 2048 (the CUDA cores are compute-bound there when they score
- *    several queries per row) and 16 for longer rows; a value above the
- *    batch size turns the tensor-core path off.  >= 1.
+ *    CUDA cores.  Needs a bf16 memory and k_entries <= 32.  Default 2 (a
+ *    bucket of one query is matrix-vector work, streamed on the CUDA cores);
+ *    a value above the batch size turns the tensor-core path off.  >= 1.
  *  HTAM_TUNE_STREAM_ROWS: 1 (default) prefetches the CUDA-core path's entry
  *    rows into per-warp shared-memory rings (bf16 memories with rows up to
  *    8 KiB and k_entries <= 32); 0 loads them directly into registers.

@@ -437,11 +437,12 @@ htam_status build_impl(const void *entries, const int32_t *gid, int64_t n, int32
   HTAM_CK(cudaGetDevice(&m->device));
   HTAM_CK(cudaDeviceGetAttribute(&m->sm_count, cudaDevAttrMultiProcessorCount, m->device));
   m->d = d;
-  // Rows up to 4 KiB (d <= 2048 bf16) are scored against 4-8 queries at a
-  // time on the CUDA cores, which is compute-bound there: a padded 128-row
-  // tensor-core tile is faster from two queries up.  Longer rows stream at
-  // HBM speed on the CUDA cores until a bucket has 16 queries.
-  m->tc_min = d <= 2048 ? 2 : 16;
+  // Buckets of two or more queries go to the tensor cores: a padded 128-row
+  // tile still streams its entries at HBM speed, while the CUDA cores are
+  // compute-bound with several queries per row for d <= 2048 and, for
+  // longer rows, score at most two queries per pass (the rest re-read the
+  // rows).  Measured: 2 is the fastest threshold on every workload tried.
+  m->tc_min = 2;
   m->n_groups = n_groups;
   m->dtype = dtype;
   m->elem_bytes = dtype == HTAM_BF16 ? 2 : 4;

@@ -697,10 +697,9 @@ def test_sampled_zipf_1m_workload_sampled_rows(htam):
 
 
 def test_tuning_defaults_follow_row_length_and_round_trip(htam):
-    """The tensor-core threshold defaults to 2 queries for rows up to 4 KiB
-    and 16 for longer rows; values set are read back; bad keys and values are
-    refused."""
-    for d, want in ((1024, 2), (2048, 2), (4096, 16)):
+    """The tensor-core threshold defaults to 2 queries for every row length;
+    values set are read back; bad keys and values are refused."""
+    for d, want in ((1024, 2), (2048, 2), (4096, 2)):
         e, gid, _ = _rand_memory(300, d, 3, torch.bfloat16, seed=d)
         mem = htam.Memory(e, gid, 3)
         assert mem.get_tuning(htam.HTAM_TUNE_TC_MIN_BUCKET) == want
