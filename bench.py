@@ -75,7 +75,9 @@ def parse_args():
     ap.add_argument("--tc-pairs", type=int, default=None, choices=[0, 1],
                     help="tensor-core buckets of several chunks on SM pairs (1) or single SMs (0, library default)")
     ap.add_argument("--tc-min-bucket", type=int, default=None,
-                    help="smallest bucket scored on the tensor cores (library default 16)")
+                    help="smallest bucket scored on the tensor cores (library default 2)")
+    ap.add_argument("--ref-seconds", type=float, default=120.0,
+                    help="reference arm: seconds of oracle work over all warm-up and timed steps")
     return ap.parse_args()
 
 
@@ -306,7 +308,7 @@ def run_reference(args, world, rank):
 
     threads = oracle.default_threads()
     cent, counts = (None, None) if args.flat else oracle.centroids(entries_np, gid_np, w.g, threads)
-    per_step_target = max(0.5, 120.0 / max(1, args.steps + args.warmup))
+    per_step_target = max(0.5, args.ref_seconds / max(1, args.steps + args.warmup))
     if args.flat:  # one query per host thread per step (each scans every entry)
         n_sample = min(threads, q_np.shape[0])
     else:
