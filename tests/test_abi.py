@@ -95,3 +95,30 @@ def test_null_memory_is_rejected(htam):
     assert lib.htam_memory_group_counts(z, z) == htam.HTAM_EINVAL
     assert lib.htam_device_status(z, z) == htam.HTAM_EINVAL
     lib.htam_free_memory(z)  # no-op
+
+
+def test_binding_without_the_library_fails_loudly(tmp_path):
+    """No CPU fallback: a binding whose library is absent refuses to import."""
+    import importlib.util
+    import shutil
+
+    pkg = tmp_path / "htam_copy"
+    pkg.mkdir()
+    shutil.copy(os.path.join(ROOT, "paper_2605_29734_gb300", "htam.py"), pkg / "htam.py")
+    spec = importlib.util.spec_from_file_location("htam_copy_binding", pkg / "htam.py")
+    module = importlib.util.module_from_spec(spec)
+    with pytest.raises(ImportError, match="libhtam.so is missing"):
+        spec.loader.exec_module(module)
+
+
+def test_product_package_never_reaches_the_oracle():
+    """The oracle is test infrastructure: nothing in the package imports it
+    or names its library (the shared input generators only mention it)."""
+    pkg = os.path.join(ROOT, "paper_2605_29734_gb300")
+    for dirpath, _, files in os.walk(pkg):
+        if "_build" in dirpath or "__pycache__" in dirpath:
+            continue
+        for name in files:
+            if name.endswith((".py", ".cu", ".cuh", ".h", ".c")):
+                text = open(os.path.join(dirpath, name)).read()
+                assert not re.search(r"(import\s+oracle|from\s+oracle|htam_oracle)", text), os.path.join(dirpath, name)
