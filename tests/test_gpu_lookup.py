@@ -783,6 +783,59 @@ def test_append_rounds_match_rebuilt_oracle(htam, dtype):
         _check(htam, mem, all_e, all_g, 30, q, 4, 12, tau=0.3)
 
 
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+def test_memory_built_empty_then_filled_by_appends(htam, dtype):
+    """A memory built with no entries has no non-empty group, so a lookup
+    returns padding only (lse = -inf: an empty candidate set).  Appends then
+    fill half of the groups, and later all of them: groups that were empty
+    become selectable, and each lookup matches the oracle on the rows
+    appended so far (ids count from 0 in append order).  The appends fill
+    the capacity exactly; one more row is refused."""
+    d, g = 64, 12
+    mem = htam.Memory(torch.empty(0, d, dtype=dtype, device=DEV), torch.empty(0, dtype=torch.int32, device=DEV),
+                      g, capacity=2400)  # the two appends below fill it exactly
+    gen = torch.Generator(device=DEV).manual_seed(21)
+    centres = torch.randn(g, d, generator=gen, device=DEV)
+    q = _rand_queries(40, d, dtype, seed=21, centres=centres)
+    out = mem.query(q, 3, 5)
+    torch.cuda.synchronize()
+    assert (out["group_idx"] == -1).all() and torch.isneginf(out["group_score"]).all()
+    assert (out["entry_idx"] == -1).all() and (out["entry_weight"] == 0).all()
+    assert torch.isneginf(out["entry_score"]).all() and torch.isneginf(out["lse"]).all()
+    assert mem.device_status() == htam.HTAM_OK
+
+    half = torch.randint(0, g // 2, (900,), generator=gen, device=DEV, dtype=torch.int64).to(torch.int32)
+    rounds = [half, torch.randint(0, g, (1500,), generator=gen, device=DEV, dtype=torch.int64).to(torch.int32)]
+    all_e, all_g = [], []
+    for r, gid in enumerate(rounds):
+        x = centres[gid.long()] + 0.3 * torch.randn(gid.shape[0], d, generator=gen, device=DEV)
+        e = _unit(x).to(dtype).contiguous()
+        mem.append(e, gid)
+        all_e.append(e)
+        all_g.append(gid)
+        ents, gids = torch.cat(all_e), torch.cat(all_g)
+        assert mem.info()["n"] == ents.shape[0]
+        counts = np.bincount(to_numpy(gids), minlength=g)
+        assert (mem.group_counts().numpy() == counts).all()
+        import oracle
+
+        keys = mem.group_keys().double().numpy()
+        ref, _ = oracle.centroids(to_numpy(ents), to_numpy(gids), g)
+        filled = counts > 0  # the oracle's mean of an empty group is NaN
+        np.testing.assert_allclose(keys[filled], ref[filled], rtol=1e-5, atol=1e-6)  # fp32 means
+        assert (keys[~filled] == 0).all()  # the library's rows of empty groups are zero
+        out = _check(htam, mem, ents, gids, g, q, 4, 8, tau=0.5, eps=0.05)
+        selected = out["group_idx"].cpu()
+        if r == 0:  # only the filled half can be selected; the rest pads
+            assert ((selected >= 0) & (selected < g // 2)).sum(1).eq(4).all()
+        else:
+            assert (selected >= g // 2).any()
+    one = torch.zeros(1, d, dtype=dtype, device=DEV)
+    with pytest.raises(htam.HtamError) as err:
+        mem.append(one, torch.zeros(1, dtype=torch.int32, device=DEV))
+    assert err.value.status == htam.HTAM_ECAPACITY and mem.info()["n"] == 2400
+
+
 def test_append_updates_group_keys_in_place(htam):
     import oracle
 
