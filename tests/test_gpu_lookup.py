@@ -183,6 +183,42 @@ def test_duplicate_rows_tie_to_lower_id(htam):
                 assert ids[b, i] < ids[b, i + 1]
 
 
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+@pytest.mark.parametrize("min_bucket", [1, 1 << 30])
+def test_zero_queries_tie_everything_to_the_lowest_ids(htam, dtype, min_bucket):
+    """A zero query scores exactly 0 against every key and entry, in any
+    summation order, so both levels are pure ties: the selected groups are
+    the lowest non-empty group ids, the entries the lowest entry ids of
+    those groups, every candidate weighs 1/n_b and lse = log n_b (any tau).
+    Checked exactly on both fine routes (tensor cores / CUDA cores) with
+    buckets of several 128-query chunks, and on the flat scan."""
+    n, d, g, kg, ke = 5000, 256, 40, 6, 20
+    gen = torch.Generator(device=DEV).manual_seed(31)
+    pool = torch.tensor([x for x in range(g) if x not in (0, 3, 4)], device=DEV)  # 0, 3, 4 stay empty
+    gid = pool[torch.randint(0, pool.numel(), (n,), generator=gen, device=DEV)].to(torch.int32)
+    entries, gid, _ = _rand_memory(n, d, g, dtype, seed=31, gid=gid)
+    mem = htam.Memory(entries, gid, g)
+    mem.set_tensor_core_min_bucket(min_bucket)
+    q = torch.zeros(300, d, dtype=dtype, device=DEV)
+    out = mem.query(q, kg, ke, tau=0.3, epsilon=0.1)
+    flat = mem.query_flat(q, ke, tau=0.3, epsilon=0.1)
+    torch.cuda.synchronize()
+    gid_np = to_numpy(gid)
+    groups = sorted(set(gid_np.tolist()))[:kg]
+    cand = np.flatnonzero(np.isin(gid_np, groups))
+    assert (out["group_idx"].cpu().numpy() == np.array(groups)).all()
+    assert (out["group_score"] == 0).all()
+    assert (out["entry_idx"].cpu().numpy() == cand[:ke]).all()
+    assert (out["entry_score"] == 0).all()
+    torch.testing.assert_close(out["entry_weight"], torch.full_like(out["entry_weight"], 1.0 / cand.size),
+                               rtol=1e-5, atol=0)
+    torch.testing.assert_close(out["lse"], torch.full_like(out["lse"], float(np.log(cand.size))), rtol=1e-6, atol=0)
+    assert (flat["entry_idx"].cpu().numpy() == np.arange(ke)).all()
+    torch.testing.assert_close(flat["entry_weight"], torch.full_like(flat["entry_weight"], 1.0 / n), rtol=1e-5, atol=0)
+    torch.testing.assert_close(flat["lse"], torch.full_like(flat["lse"], float(np.log(n))), rtol=1e-6, atol=0)
+    assert mem.device_status() == htam.HTAM_OK
+
+
 @pytest.mark.parametrize("d", [8, 24, 4096, 16384])
 def test_dimension_extremes(htam, d):
     n = 2000 if d <= 4096 else 400
