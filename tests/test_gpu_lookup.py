@@ -219,6 +219,32 @@ def test_zero_queries_tie_everything_to_the_lowest_ids(htam, dtype, min_bucket):
     assert mem.device_status() == htam.HTAM_OK
 
 
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+@pytest.mark.parametrize("min_bucket", [1, 1 << 30])
+def test_large_scores_are_max_shifted(htam, dtype, min_bucket):
+    """Rows of norm sqrt(40) and tau = 0.1 give s / tau up to 400, far past
+    where exp overflows in fp32 (about 88): the online maximum of the fine
+    kernels and the merge's log-sum-exp must keep every weight and lse
+    finite and equal to the oracle's.  The tolerance is the bf16 one for
+    both dtypes: at this temperature a score's last-place error is
+    amplified 10x in the weights."""
+    n, d, g, b, kg, ke = 6000, 128, 24, 200, 4, 16
+    entries, gid, centres = _rand_memory(n, d, g, torch.float32, seed=41)
+    q = _rand_queries(b, d, torch.float32, seed=41, centres=centres)
+    scale = float(np.sqrt(40.0))
+    entries = (entries * scale).to(dtype).contiguous()
+    q = (q * scale).to(dtype).contiguous()
+    mem = htam.Memory(entries, gid, g)
+    mem.set_tensor_core_min_bucket(min_bucket)
+    out = mem.query(q, kg, ke, tau=0.1, epsilon=0.05)
+    torch.cuda.synchronize()
+    assert mem.device_status() == htam.HTAM_OK
+    assert torch.isfinite(out["lse"]).all() and torch.isfinite(out["entry_weight"]).all()
+    assert out["lse"].max().item() > 300.0  # the unshifted exponentials would overflow
+    problems = compare_lookup(out, to_numpy(entries), to_numpy(gid), g, to_numpy(q), kg, ke, 0.1, 0.05, "bf16")
+    assert not problems, "\n".join(problems[:20])
+
+
 @pytest.mark.parametrize("d", [8, 24, 4096, 16384])
 def test_dimension_extremes(htam, d):
     n = 2000 if d <= 4096 else 400
