@@ -624,3 +624,98 @@ def test_assign_nearest_matches_numpy_brute_force():
             assert out[i] == np.lexsort((np.arange(G), -s[i]))[0]
     assert (out[:10] == 2).all()
     assert not np.isin(out[gid == -1], [1, 7]).any()
+
+
+# ------------------------------------------------ composed lookups (N2, N4)
+
+def _brute_stage2(x, gid, q, groups, k, tau, eps):
+    """Stage 2 written out with numpy: candidates = entries of `groups`,
+    matmul scores, lexsort top-k (ties to the lower id), scipy logsumexp."""
+    cand = np.flatnonzero(np.isin(gid, groups))
+    s = x[cand].astype(np.float64) @ q.astype(np.float64)
+    order = np.lexsort((cand, -s))[:k]
+    lse = logsumexp(s / tau)
+    w = eps / cand.size + (1 - eps) * np.exp(s[order] / tau - lse)
+    return cand[order], s[order], w, lse
+
+
+def test_edge_routed_lookup_by_inspection():
+    """One feature, w = 1 and Z[p, g] = -(g - p)^2: a query whose prefix is
+    the single group p ranks p first, then its neighbours by distance, the
+    lower id first on ties, skipping empty groups (3 here).  The group
+    scores are -(g - p)^2 exactly (a one-element prefix weighs 1), and the
+    entries are the brute-force stage 2 over exactly those groups."""
+    G, d, n, kg, ke, tau, eps = 10, 8, 500, 4, 6, 0.7, 0.1
+    rng = np.random.default_rng(43)
+    Z = np.zeros((G, G, 1), np.float32)
+    for p in range(G):
+        for g in range(G):
+            Z[p, g, 0] = -float((g - p) ** 2)
+    x = _unit_rows(rng, n, d)
+    gid = rng.integers(0, G, n).astype(np.int32)
+    gid[gid == 3] = 2
+    prefix = np.array([[5], [0], [9]], np.int32)
+    q = _unit_rows(rng, 3, d)
+    out = oracle.query_edges(x, gid, G, Z, np.array([1.0]), prefix, 0.5, q, kg, ke, tau=tau, eps=eps)
+    want = [[5, 4, 6, 7], [0, 1, 2, 4], [9, 8, 7, 6]]
+    for r, p in enumerate(prefix[:, 0]):
+        assert list(out["group_idx"][r]) == want[r]
+        assert list(out["group_score"][r]) == [-float((g - p) ** 2) for g in want[r]]
+        ids, s, w, lse = _brute_stage2(x, gid, q[r], want[r], ke, tau, eps)
+        assert list(out["entry_idx"][r]) == list(ids)
+        np.testing.assert_allclose(out["entry_score"][r], s, rtol=0, atol=1e-12)
+        np.testing.assert_allclose(out["entry_weight"][r], w, rtol=1e-11)
+        assert out["lse"][r] == pytest.approx(lse, rel=1e-12)
+
+
+def test_sampled_lookup_cold_limit_is_the_ranked_lookup():
+    """As tau -> 0 the policy of Eq. 11 puts all its mass on the best group:
+    with score gaps of at least 5e-3 and tau = 1e-4, log-probability gaps
+    (>= 50) exceed any Gumbel spread (about 20 for 23-bit uniforms).  So the
+    draws are stage 1's ranking, and the sampled lookup returns the ranked
+    lookup's groups, entries, weights and lse, for every seed."""
+    rng = np.random.default_rng(44)
+    n, d, G, b, kg, ke, tau = 600, 12, 10, 8, 3, 7, 1e-4
+    x = _unit_rows(rng, n, d)
+    gid = rng.integers(0, G, n).astype(np.int32)
+    cent, counts = oracle.centroids(x, gid, G)
+    q = _unit_rows(rng, 64, d)
+    s = -np.sort(-(q.astype(np.float64) @ cent.T), axis=1)
+    gaps = (s[:, :kg] - s[:, 1:kg + 1]).min(axis=1)
+    q = q[gaps > 5e-3][:b]
+    assert q.shape[0] == b
+    ref = oracle.query(x, gid, G, q, kg, ke, tau=tau)
+    for seed in (0, 1, 7):
+        out = oracle.query_sampled(x, gid, G, q, kg, ke, tau, 0.0, seed, 3, centroid=cent, counts=counts)
+        assert np.array_equal(out["group_idx"], ref["group_idx"])
+        assert np.array_equal(out["entry_idx"], ref["entry_idx"])
+        np.testing.assert_allclose(out["entry_weight"], ref["entry_weight"], rtol=1e-12)
+        np.testing.assert_allclose(out["lse"], ref["lse"], rtol=1e-12)
+
+
+def test_sampled_lookup_draws_uniformly_at_full_exploration():
+    """With eps = 1 the policy of Eq. 11 is uniform over the non-empty groups,
+    whatever the scores: over many seeds the sampled lookup's first group is
+    uniform (chi-square), its groups are distinct and never empty, and its
+    entries are the brute-force stage 2 over the drawn groups."""
+    from scipy.stats import chisquare
+
+    rng = np.random.default_rng(45)
+    n, d, G, kg, ke = 300, 8, 6, 2, 5
+    x = _unit_rows(rng, n, d)
+    gid = rng.integers(0, G, n).astype(np.int32)
+    gid[gid == 4] = 5  # group 4 empty
+    q = _unit_rows(rng, 1, d)
+    cent, counts = oracle.centroids(x, gid, G)
+    first = []
+    for seed in range(1500):
+        out = oracle.query_sampled(x, gid, G, q, kg, ke, 0.5, 1.0, seed, 0, centroid=cent, counts=counts)
+        gi = out["group_idx"][0]
+        assert len(set(gi.tolist())) == kg and 4 not in gi and (gi >= 0).all()
+        if seed < 20:
+            ids, s, w, lse = _brute_stage2(x, gid, q[0], gi, ke, 0.5, 1.0)
+            assert list(out["entry_idx"][0]) == list(ids)
+            np.testing.assert_allclose(out["entry_weight"][0], w, rtol=1e-11)
+        first.append(gi[0])
+    obs = np.bincount(first, minlength=G)[[0, 1, 2, 3, 5]]
+    assert chisquare(obs).pvalue > 1e-3

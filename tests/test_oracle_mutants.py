@@ -8,8 +8,12 @@ groups allowed into stage 1, prefix weights reversed, of the wrong sign or
 missing the newest element, edge-table rows and columns swapped, an edge
 feature misread, edge-prefix weights reversed, Philox words swapped or its key
 not advanced, one uniform shared by four groups, the policy's eps term dropped
-or tau ignored, the Gumbel noise of the wrong sign, empty groups drawn), builds it there and runs ``test_oracle.py``
-against the mutant: at least one pin has to fail.
+or tau ignored, the Gumbel noise of the wrong sign, empty groups drawn), or one
+in the Python layer that composes the C routines (the sampled lookup ranking
+instead of drawing or dropping tau in stage 2, the edge-routed lookup counting
+empty groups, the flat scan ignoring tau, the nearest-key assignment
+overwriting given ids), builds it there and runs ``test_oracle.py`` against
+the mutant: at least one pin has to fail.
 """
 import os
 import shutil
@@ -47,18 +51,33 @@ MUTANTS = {
     "policy_tau_ignored": ("if (counts[g] > 0) sum += exp(s[g] / tau - m);", "if (counts[g] > 0) sum += exp(s[g] - m);"),
     "gumbel_sign_flipped": ("keys[o] = log_mu - log(-log(u));", "keys[o] = log_mu + log(-log(u));"),
     "policy_empty_groups_drawn": ("      if (counts[g] == 0) {\n        mu[o] = 0.0;", "      if (0) {\n        mu[o] = 0.0;"),
+    # Slips in the Python layer that composes the C routines.
+    "sampled_lookup_ranks_instead_of_drawing": ("__init__.py", "gi, gk = select(keys, counts, k_groups)",
+                                                "gi, gk = select(coarse_scores(queries, centroid), counts, k_groups)"),
+    "sampled_stage2_tau_dropped": ("__init__.py",
+                                   "gi, k_entries, tau, eps, nthreads)\n    out[\"group_idx\"] = gi\n    out[\"group_key\"]",
+                                   "gi, k_entries, 1.0, eps, nthreads)\n    out[\"group_idx\"] = gi\n    out[\"group_key\"]"),
+    "edge_lookup_counts_every_group": ("__init__.py",
+                                       "counts = np.bincount(np.asarray(gid, dtype=np.int64), minlength=n_groups)",
+                                       "counts = np.ones(n_groups, dtype=np.int64)"),
+    "flat_tau_ignored": ("__init__.py", "np.zeros((b, 1), np.int32), k_entries, tau, eps,",
+                         "np.zeros((b, 1), np.int32), k_entries, 1.0, eps,"),
+    "assign_overwrites_given_ids": ("__init__.py", "miss = np.flatnonzero(out == -1)", "miss = np.arange(out.size)"),
 }
 
 
 @pytest.mark.parametrize("name", sorted(MUTANTS))
 def test_pins_catch_planted_mistake(name, tmp_path):
-    before, after = MUTANTS[name]
-    src = open(os.path.join(ROOT, "oracle", "htam_oracle.c")).read()
-    assert before in src, "mutation site moved; update the mutant"
+    spec = MUTANTS[name]
+    target, before, after = spec if len(spec) == 3 else ("htam_oracle.c", *spec)
     (tmp_path / "oracle").mkdir()
     (tmp_path / "tests").mkdir()
-    (tmp_path / "oracle" / "htam_oracle.c").write_text(src.replace(before, after))
-    shutil.copy(os.path.join(ROOT, "oracle", "__init__.py"), tmp_path / "oracle" / "__init__.py")
+    for fname in ("htam_oracle.c", "__init__.py"):
+        src = open(os.path.join(ROOT, "oracle", fname)).read()
+        if fname == target:
+            assert before in src, "mutation site moved; update the mutant"
+            src = src.replace(before, after)  # every occurrence
+        (tmp_path / "oracle" / fname).write_text(src)
     shutil.copy(os.path.join(ROOT, "tests", "test_oracle.py"), tmp_path / "tests" / "test_oracle.py")
     shutil.copytree(os.path.join(ROOT, "tests", "golden"), tmp_path / "tests" / "golden")
     (tmp_path / "pytest.ini").write_text("[pytest]\naddopts = -p no:cacheprovider\n")
