@@ -127,9 +127,9 @@ htam_status htam_append_assign(htam_memory *m, const void *entries,
  *  entry_score : [b, k_entries] fp32, q . k_e (-inf for padding)
  *  entry_weight: [b, k_entries] fp32, w_e as above (0 for padding)
  *  lse         : [b] fp32 or NULL, log-sum-exp of s/tau over the candidates
- * Fully asynchronous: nothing is read back.  b may be 0.  A device-side
- * timeout is reported by htam_device_status.  Errors: EINVAL, ENOMEM (scratch
- * growth), ECUDA. */
+ * Fully asynchronous: nothing is read back.  0 <= b <= 2^24 (b may be 0).  A
+ * device-side timeout is reported by htam_device_status.  Errors: EINVAL,
+ * ENOMEM (scratch growth), ECUDA. */
 htam_status htam_query(htam_memory *m, const void *queries, int32_t b,
                        const htam_query_params *p, int32_t *group_idx,
                        float *group_score, int32_t *entry_idx,
@@ -247,8 +247,8 @@ htam_status htam_query_edges_sampled(htam_memory *m, const float *edge_features,
  *  tau, epsilon: as htam_query_params
  *  entry_idx / entry_score / entry_weight / lse: as htam_query ([b, k_entries],
  *                lse [b] or NULL), -1 / -inf / 0 padding when n < k_entries
- * b * (non-empty groups) <= 2^28.  Outputs, asynchrony and errors as
- * htam_query. */
+ * 0 <= b <= 2^24 and b * (non-empty groups) <= 2^28.  Outputs, asynchrony
+ * and errors as htam_query. */
 htam_status htam_query_flat(htam_memory *m, const void *queries, int32_t b,
                             int32_t k_entries, float tau, float epsilon,
                             int32_t *entry_idx, float *entry_score,
