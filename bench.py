@@ -76,6 +76,8 @@ def parse_args():
                     help="tensor-core buckets of several chunks on SM pairs (1) or single SMs (0, library default)")
     ap.add_argument("--tc-min-bucket", type=int, default=None,
                     help="smallest bucket scored on the tensor cores (library default 2)")
+    ap.add_argument("--no-secondary", action="store_true",
+                    help="default workload only: skip the secondary (4,096-query, 1M-entry) measurement")
     ap.add_argument("--ref-seconds", type=float, default=120.0,
                     help="reference arm: seconds of oracle work over all warm-up and timed steps")
     return ap.parse_args()
@@ -343,7 +345,10 @@ def run_reference(args, world, rank):
     print(json.dumps(line), flush=True)
 
 
-def run_htam(args, world, rank, local):
+def measure(args, world, rank, local, full=True):
+    """One workload's timed steps on this rank.  Returns the JSON line's
+    fields on rank 0 (None elsewhere).  full=False leaves out the end-to-end
+    leg and the CPU baseline (the secondary workload of the default run)."""
     from paper_2605_29734_gb300 import htam
 
     w = workload_of(args)
@@ -510,6 +515,23 @@ def run_htam(args, world, rank, local):
     step_s = total_s / args.steps
     launches = sum(v[1] for k, v in phases.items() if k != "queries")
 
+    if not full:
+        mem.close()
+        if rank != 0:
+            return None
+        return {"workload": w.name, "value": value, "unit": UNIT, "ms_per_step": 1e3 * step_s, "dtype": w.dtype,
+                "config": {"workload": w.name, "queries_per_step": w.b, "d": w.d, "groups": w.g, "entries": w.n,
+                           "k_groups": w.k_groups, "k_entries": w.k_entries, "query_batches": len(batches),
+                           "l2": ("flushed between steps (2x L2 buffer write, outside the step events)"
+                                  if flush_l2 else
+                                  f"inputs larger than L2 ({work[0]['step_bytes'] / 1e9:.2f} GB touched per step)")},
+                "steps": args.steps, "warmup": args.warmup, "roofline": roofline,
+                "step_roofline": {"algorithmic_bytes": step_bytes, "algorithmic_flops": step_flops,
+                                  "t_roof_ms": 1e3 * t_roof, "frac": t_roof / step_s,
+                                  "phase_ms_per_step": {k: v[0] / args.steps for k, v in phases.items()
+                                                        if k != "queries"}},
+                "clocks": clocks, "gpu_launches": launches, "wall_s_timed_region": wall}
+
     # End to end: host (pinned) queries in, host results out, through the C ABI.
     host_q = [b.cpu().pin_memory() for b in batches]
     e2e_steps = max(3, min(args.steps, 50))
@@ -623,8 +645,30 @@ def run_htam(args, world, rank, local):
             "gpu_launches": launches,
             "wall_s_timed_region": wall,
         }
-        print(json.dumps(line), flush=True)
     mem.close()
+    return line if rank == 0 else None
+
+
+# The default run also times the contraction-bound workload (4,096 queries
+# against 1,048,576 entries, d = 1,024) after the headline one, in the same
+# process, and reports it under "secondary".
+SECONDARY_WORKLOAD = "zipf_bf16_1m"
+
+
+def run_htam(args, world, rank, local):
+    line = measure(args, world, rank, local)
+    plain = not (args.flat or args.sample or args.prefix or args.edges or args.unassigned > 0 or args.shrink > 1)
+    if plain and args.workload == DEFAULT_WORKLOAD and not args.no_secondary:
+        import copy
+
+        torch.cuda.empty_cache()
+        sec_args = copy.copy(args)
+        sec_args.workload = SECONDARY_WORKLOAD
+        sec = measure(sec_args, world, rank, local, full=False)
+        if line is not None:
+            line["secondary"] = sec
+    if line is not None:
+        print(json.dumps(line), flush=True)
 
 
 def main():

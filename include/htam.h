@@ -273,7 +273,7 @@ htam_status htam_query_flat(htam_memory *m, const void *queries, int32_t b,
  * fp32 rounding (so groups whose scores differ by less than that may come
  * out in the other order).  Arguments are those
  * of htam_query: device pointers, queries [b, d] of the memory's dtype,
- * outputs [b, k_groups].
+ * outputs [b, k_groups], 0 <= b <= 2^24.
  *
  * Scratch: the [b, n_groups] fp32 score matrix lives in one fixed array of
  * HTAM_STATIC_SCRATCH_BYTES compiled into the library; every GPU that loads

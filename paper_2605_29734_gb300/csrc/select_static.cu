@@ -60,7 +60,8 @@ htam_status static_scores_on(int device, float **out) {
 // s1[b][g] = q_b . cent_g, each output accumulated with fmaf over k = 0..d-1
 // in order against the fp32 group key (htam_query reaches the same scores
 // within fp32 rounding, on the tensor cores for bf16 memories); -inf for empty
-// groups.  32x32 tiles.
+// groups.  32x32 tiles: query tiles on grid.x (up to 2^31 - 1 blocks), group
+// tiles on grid.y (at most 2,048 for 65,536 groups).
 template <typename T>
 __global__ void __launch_bounds__(256) static_coarse_kernel(const T *__restrict__ Q, int B, int d,
                                                             const float *__restrict__ cent,
@@ -69,7 +70,7 @@ __global__ void __launch_bounds__(256) static_coarse_kernel(const T *__restrict_
   __shared__ float qs[32][33];
   __shared__ float cs[32][33];
   const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;  // 32 x 8 threads
-  const int b0 = blockIdx.y * 32, g0 = blockIdx.x * 32;
+  const int b0 = blockIdx.x * 32, g0 = blockIdx.y * 32;
   float acc[4] = {0.f, 0.f, 0.f, 0.f};
   for (int k0 = 0; k0 < d; k0 += 32) {
     for (int r = ty; r < 32; r += 8) {
@@ -136,7 +137,9 @@ using namespace htam;
 extern "C" htam_status htam_select_groups_static(const htam_memory *m, const void *queries, int32_t b,
                                                  int32_t k_groups, int32_t *group_idx, float *group_score,
                                                  void *cuda_stream) {
-  if (!m || b < 0 || k_groups < 1 || k_groups > kMaxK || k_groups > m->n_groups) return HTAM_EINVAL;
+  if (!m || b < 0 || b > (1 << 24) || k_groups < 1 || k_groups > kMaxK || k_groups > m->n_groups) {
+    return HTAM_EINVAL;
+  }
   if (b == 0) return HTAM_OK;
   if (!queries || !group_idx || !group_score) return HTAM_EINVAL;
   if ((reinterpret_cast<uintptr_t>(queries) & 15u) != 0) return HTAM_EINVAL;
@@ -150,7 +153,10 @@ extern "C" htam_status htam_select_groups_static(const htam_memory *m, const voi
   if (s != HTAM_OK) return s;
   cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
   const int G = m->n_groups, d = m->d;
-  dim3 grid((unsigned)ceil_div(G, 32), (unsigned)ceil_div(b, 32));
+  // b <= 2^24 gives at most 2^19 query tiles on grid.x and G <= 65,536 at
+  // most 2,048 group tiles on grid.y: both within the launch limits, so no
+  // argument that passed the checks above fails at launch.
+  dim3 grid((unsigned)ceil_div(b, 32), (unsigned)ceil_div(G, 32));
   if (m->dtype == HTAM_BF16) {
     static_coarse_kernel<__nv_bfloat16><<<grid, 256, 0, st>>>(static_cast<const __nv_bfloat16 *>(queries), b, d,
                                                               m->cent, m->count, G, s1);

@@ -136,11 +136,28 @@ def _check_entries(ei, es, ew, lse, b, r, ref2, entries_np, qf, k_entries, tau, 
     return problems
 
 
+def edge_score_tol(scores, mag, n_features, p_len):
+    """Absolute bounds for the fp32 edge-table scores of Eq. 9 (App. B.6
+    utility): the fp32 value gate 1e-5 |ref| + 1e-7 wherever the sum is well
+    conditioned, widened where it cancels to the textbook bound of an fp32
+    sum of n rounded terms, gamma_n * sum |terms| with gamma_n = n u / (1 - n u)
+    and u = 2^-24 (Higham, Accuracy and Stability of Numerical Algorithms,
+    §3.1).  The kernels take, per prefix element, n_features fused
+    multiply-adds for w . z, then one more to add alpha_i times it, and alpha_i
+    is rounded once to fp32: n = n_features + p_len + 1.  mag is the oracle's
+    score with |Z| and |w|, i.e. sum_i alpha_i sum_f |w_f| |Z_f|."""
+    rtol, atol = TOL["f32"]
+    n = n_features + p_len + 1
+    u = 2.0 ** -24
+    gamma = n * u / (1.0 - n * u)
+    return np.maximum(rtol * np.abs(np.asarray(scores, dtype=np.float64)) + atol,
+                      gamma * np.asarray(mag, dtype=np.float64))
+
+
 def compare_edge_lookup(out, entries_np, gid_np, n_groups, Z, w, prefix, lam, queries_np, k_groups, k_entries,
                         tau, eps, dtype, nthreads=None):
     """The edge-routed lookup: stage 1 against the oracle's edge-table scores
-    (values within 1e-5 of the sum of the magnitudes of their terms, the fp32
-    rounding bound of the sum, plus 1e-6), stage 2 given the GPU's groups."""
+    (values within edge_score_tol), stage 2 given the GPU's groups."""
     import oracle
 
     gi = out["group_idx"].cpu().numpy()
@@ -152,6 +169,7 @@ def compare_edge_lookup(out, entries_np, gid_np, n_groups, Z, w, prefix, lam, qu
     counts = np.bincount(np.asarray(gid_np, dtype=np.int64), minlength=n_groups)
     scores = oracle.edge_scores(Z, w, prefix, lam)
     mag = oracle.edge_scores(np.abs(Z), np.abs(np.asarray(w, dtype=np.float64)), prefix, lam)
+    stol = edge_score_tol(scores, mag, Z.shape[2], prefix.shape[1])
     ref_gi, ref_gs = oracle.select(scores, counts, min(k_groups + 1, n_groups))
     if ref_gi.shape[1] == k_groups:
         ref_gi = np.concatenate([ref_gi, -np.ones((len(ref_gi), 1), np.int32)], axis=1)
@@ -162,7 +180,7 @@ def compare_edge_lookup(out, entries_np, gid_np, n_groups, Z, w, prefix, lam, qu
     for b in range(queries_np.shape[0]):
         problems += check_ranked(f"query {b} groups", gi[b], gs[b], ref_gi[b], ref_gs[b], k_groups,
                                  lambda g, b=b: float(scores[b, g]), dtype,
-                                 tol=lambda g, b=b: 1e-5 * float(mag[b, g]) + 1e-6)
+                                 tol=lambda g, b=b: float(stol[b, g]))
         problems += _check_entries(ei, es, ew, lse, b, b, ref2, entries_np, qf, k_entries, tau, eps, dtype)
     return problems
 

@@ -427,6 +427,39 @@ def test_prefix_scores_are_weighted_stage1_scores():
     np.testing.assert_allclose(got, want, rtol=0, atol=2e-6)
 
 
+def test_round_query_bf16_is_round_to_nearest_even():
+    """The reduced query is rounded to bf16 the way any bf16 query is made:
+    float64 -> float32 -> bf16, each step to nearest, ties to even.  Checked
+    against torch's float32 -> bfloat16 conversion (an independent library
+    routine) on random values over many binades, and on hand-made float32
+    patterns whose dropped half is exactly 0x8000 (a tie: even lsb stays,
+    odd lsb rounds up), just below and just above it, and carries that ripple
+    into the exponent."""
+    import torch
+
+    rng = np.random.default_rng(41)
+    x = rng.standard_normal(20000) * np.exp2(rng.integers(-30, 30, 20000))
+    got = oracle.round_query(x, "bf16")
+    want = torch.from_numpy(x.astype(np.float32)).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    assert np.array_equal(got, want)
+    cases = {
+        0x3F808000: 0x3F80,  # tie, even lsb: stays
+        0x3F818000: 0x3F82,  # tie, odd lsb: up to even
+        0x3F807FFF: 0x3F80,  # just below the half: down
+        0x3F808001: 0x3F81,  # just above the half: up
+        0xBF818000: 0xBF82,  # negative tie, odd lsb: magnitude up
+        0x3F7FFFFF: 0x3F80,  # carry into the exponent
+        0x00008000: 0x0000,  # subnormal tie, even lsb
+        0x00018000: 0x0002,  # subnormal tie, odd lsb
+    }
+    bits = np.array(list(cases), dtype=np.uint32)
+    got = oracle.round_query(bits.view(np.float32).astype(np.float64), "bf16")
+    assert [int(v) for v in got] == list(cases.values())
+    # The float64 -> float32 step rounds to nearest too: a double just above
+    # the float32 midpoint of 1 and 1 + 2^-23 goes up, bf16 then keeps 1.0.
+    assert oracle.round_query(np.array([1.0 + 2.0 ** -24 + 2.0 ** -40]), "f32").view(np.uint32)[0] == 0x3F800001
+
+
 # ------------------------------------------------ edge-table routing (N2)
 
 def test_edge_scores_one_hot_weights_read_the_feature_slice():

@@ -12,7 +12,8 @@ or tau ignored, the Gumbel noise of the wrong sign, empty groups drawn), or one
 in the Python layer that composes the C routines (the sampled lookup ranking
 instead of drawing or dropping tau in stage 2, the edge-routed lookup counting
 empty groups, the flat scan ignoring tau, the nearest-key assignment
-overwriting given ids), builds it there and runs ``test_oracle.py`` against
+overwriting given ids, the bf16 rounding of a reduced query truncating or
+rounding ties away from zero), builds it there and runs ``test_oracle.py`` against
 the mutant: at least one pin has to fail.
 """
 import os
@@ -63,6 +64,10 @@ MUTANTS = {
     "flat_tau_ignored": ("__init__.py", "np.zeros((b, 1), np.int32), k_entries, tau, eps,",
                          "np.zeros((b, 1), np.int32), k_entries, 1.0, eps,"),
     "assign_overwrites_given_ids": ("__init__.py", "miss = np.flatnonzero(out == -1)", "miss = np.arange(out.size)"),
+    "bf16_rounding_truncates": ("__init__.py", "rounded = (u + 0x7FFF + ((u >> 16) & 1)) >> 16",
+                                "rounded = u >> 16"),
+    "bf16_ties_away_from_zero": ("__init__.py", "rounded = (u + 0x7FFF + ((u >> 16) & 1)) >> 16",
+                                 "rounded = (u + 0x8000) >> 16"),
 }
 
 
