@@ -87,8 +87,12 @@ def _against_query(gi, gs, ref_gi, ref_gs, dtype):
     problems = []
     for b in range(gi.shape[0]):
         for i in range(gi.shape[1]):
+            if ref_gi[b, i] < 0:  # padding: -1 / -inf on both sides
+                if gi[b, i] != -1 or not np.isneginf(gs[b, i]):
+                    problems.append(f"query {b} slot {i}: padding {gi[b, i]} {gs[b, i]}")
+                continue
             clear_above = i == 0 or ref_gs[b, i - 1] - ref_gs[b, i] > 1e-3
-            clear_below = i + 1 == gi.shape[1] or ref_gs[b, i] - ref_gs[b, i + 1] > 1e-3
+            clear_below = i + 1 == gi.shape[1] or ref_gi[b, i + 1] < 0 or ref_gs[b, i] - ref_gs[b, i + 1] > 1e-3
             if clear_above and clear_below and gi[b, i] != ref_gi[b, i]:
                 problems.append(f"query {b} slot {i}: {gi[b, i]} vs htam_query {ref_gi[b, i]}")
             if not close(gs[b, i], ref_gs[b, i], dt):
