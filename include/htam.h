@@ -33,6 +33,9 @@
  *    the library copies entries into its own storage.
  *  - Functions return a status and never abort or throw.  Argument errors are
  *    detected before anything is launched and leave the memory unchanged.
+ *    The one check made on the device is that of an append's group ids (see
+ *    htam_append_transitions): a rejected batch leaves the memory unchanged
+ *    and is reported by htam_device_status.
  *  - One memory object is used from one stream at a time: htam_query does
  *    not modify the stored entries or keys, but it uses scratch space owned by
  *    the memory object, so two queries on the same object must not overlap.
@@ -82,26 +85,37 @@ typedef struct {
  *  capacity : most entries the memory will ever hold (>= n, < 2^31); storage
  *             is reserved up front so that appends never reallocate
  *  out      : receives the new memory (NULL on failure)
- * Synchronises `cuda_stream` once (the group sizes are read back to lay out
- * the pages).  Errors: EINVAL (arguments, a group id out of range), ENOMEM,
- * ECUDA, ENODEV. */
+ * The rows are laid out on the device as an append lays them out; the call
+ * then synchronises `cuda_stream` once to read the group-id check, so a
+ * build with a group id outside [0, n_groups) fails with EINVAL.  Errors:
+ * EINVAL (arguments, a group id out of range), ENOMEM, ECUDA, ENODEV. */
 htam_status htam_build_memory(const void *entries, const int32_t *group_ids,
                               int64_t n, int32_t d, int32_t n_groups,
                               htam_dtype dtype, int64_t capacity,
                               void *cuda_stream, htam_memory **out);
 
 /* Appends `count` entries (the memory update of Eq. 15) and updates the keys
- * of the groups they join in place.  New entries get ids n, n+1, ...
+ * of the groups they join in place.  New entries get ids n, n+1, ... where n
+ * counts the entries of every batch accepted before this one.
  *  entries  : [count, d] of the memory's dtype, device, 16-byte aligned
  *  group_ids: [count] int32, device, 16-byte aligned: a group in
  *             [0, n_groups), or -1 for an entry without a group, which joins
  *             the group whose key scores highest against it (q . c_g with the
  *             entry as q, stage 1's scorer; ties to the lower id; empty groups
  *             excluded), by the keys as they stand before this call
- * Synchronises `cuda_stream` once (twice when some id is -1).  Errors:
- * EINVAL (a group id out of range, or an id of -1 while every group is
- * empty), ECAPACITY (n + count would exceed the capacity, or the page pool is
- * full), ENOMEM; the memory is unchanged on any error. */
+ * Fully asynchronous: the batch's group sizes, the nearest-key choices, the
+ * page layout and the key updates are all computed on the device, with no
+ * host round trip (a growth of the memory object's scratch, on the first
+ * append of a new size, synchronises the device once).  Page space never
+ * runs out: the pages reserved at build hold any `capacity` entries.
+ * The group ids are checked on the device.  A batch with an id out of range,
+ * or an id of -1 while every group is empty, is rejected there: the memory
+ * is left unchanged (no entry, key, size or id number is used up) and the
+ * next htam_device_status call returns EINVAL.  Later calls queued behind a
+ * rejected batch see the memory as it was.
+ * Errors returned by the call itself: EINVAL (arguments), ECAPACITY (n +
+ * count would exceed the capacity; appends the device rejected are
+ * subtracted first), ENOMEM, ECUDA; the memory is unchanged on any of them. */
 htam_status htam_append_transitions(htam_memory *m, const void *entries,
                                     const int32_t *group_ids, int64_t count,
                                     void *cuda_stream);
@@ -109,10 +123,12 @@ htam_status htam_append_transitions(htam_memory *m, const void *entries,
 /* htam_append_transitions that also reports the group each entry joined:
  *  assigned : [count] int32, device, caller-allocated (may be group_ids
  *             itself); receives group_ids with every -1 replaced by the group
- *             chosen for that entry.
+ *             chosen for that entry (left as it was if the device rejects the
+ *             batch).
  * The nearest-key choice keeps a [rows, n_groups] fp32 score buffer that the
  * memory object owns (up to 16 MiB per K split), grown with cudaMalloc on
- * demand. */
+ * demand; its kernels are queued with every append and do nothing when no id
+ * is -1. */
 htam_status htam_append_assign(htam_memory *m, const void *entries,
                                const int32_t *group_ids, int64_t count,
                                int32_t *assigned, void *cuda_stream);
@@ -216,8 +232,10 @@ typedef struct {
  * words of offset) under key (low and high words of seed), its top 23 bits
  * plus one half times 2^-23.  group_idx lists the draws in order and
  * group_score holds their scores q . c_g; stage 2 and every other output are
- * those of htam_query over the drawn groups.  Arguments, asynchrony and
- * errors as htam_query (EINVAL also for sampling == NULL). */
+ * those of htam_query over the drawn groups.  Arguments and errors as
+ * htam_query (EINVAL also for sampling == NULL); the call waits for the group
+ * sizes of the last queued append (the policy's |G_t| is the exact number of
+ * non-empty groups), otherwise it is asynchronous. */
 htam_status htam_query_sampled(htam_memory *m, const void *queries, int32_t b,
                                const htam_query_params *p, const htam_sampling *sampling,
                                int32_t *group_idx, float *group_score, int32_t *entry_idx,
@@ -247,8 +265,9 @@ htam_status htam_query_edges_sampled(htam_memory *m, const float *edge_features,
  *  tau, epsilon: as htam_query_params
  *  entry_idx / entry_score / entry_weight / lse: as htam_query ([b, k_entries],
  *                lse [b] or NULL), -1 / -inf / 0 padding when n < k_entries
- * 0 <= b <= 2^24 and b * (non-empty groups) <= 2^28.  Outputs, asynchrony
- * and errors as htam_query. */
+ * 0 <= b <= 2^24 and b * (non-empty groups) <= 2^28.  Outputs and errors as
+ * htam_query; the call waits for the group sizes of the last queued append
+ * (it needs the exact non-empty groups), otherwise it is asynchronous. */
 htam_status htam_query_flat(htam_memory *m, const void *queries, int32_t b,
                             int32_t k_entries, float tau, float epsilon,
                             int32_t *entry_idx, float *entry_score,
@@ -292,11 +311,14 @@ htam_status htam_select_groups_static(const htam_memory *m, const void *queries,
                                       int32_t *group_idx, float *group_score,
                                       void *cuda_stream);
 
-/* Sizes of a memory; any output pointer may be NULL (host pointers). */
+/* Sizes of a memory; any output pointer may be NULL (host pointers).  *n
+ * waits for the last queued append to finish (and excludes any batch the
+ * device rejected). */
 htam_status htam_memory_info(const htam_memory *m, int64_t *n, int32_t *d,
                              int32_t *n_groups, int64_t *capacity);
 
-/* Copies the current group sizes n_g into counts[n_groups] (host). */
+/* Copies the current group sizes n_g into counts[n_groups] (host), after
+ * waiting for the last queued append to finish. */
 htam_status htam_memory_group_counts(const htam_memory *m, int64_t *counts);
 
 /* Copies the current group keys (fp32 means, [n_groups, d]) into host
@@ -306,7 +328,9 @@ htam_status htam_memory_group_keys(const htam_memory *m, float *keys,
 
 /* Synchronises `cuda_stream`, reads and clears the memory's device status
  * word.  Returns ETIMEOUT if a bounded device wait gave up since the last
- * check, ECUDA if the stream reports an error, OK otherwise. */
+ * check, else EINVAL if the device rejected an append's group ids since the
+ * last check (see htam_append_transitions), ECUDA if the stream reports an
+ * error, OK otherwise. */
 htam_status htam_device_status(htam_memory *m, void *cuda_stream);
 
 /* Phases of htam_query (and of htam_append_transitions), for the timing
@@ -320,8 +344,7 @@ typedef enum {
   HTAM_PHASE_MERGE = 5,   /* per-query merge, weights, outputs */
   HTAM_PHASE_PREFIX = 6,  /* reduced queries of htam_query_prefix */
   HTAM_PHASE_APPEND = 7,  /* htam_append_transitions / htam_append_assign, from the
-                             batch's group count to the last key update (including
-                             the host round trip in between) */
+                             batch's group count to the last key update */
   HTAM_N_PHASES = 8
 } htam_phase;
 

@@ -106,7 +106,6 @@ htam_status htam_append_transitions(htam_memory *m, const void *entries, const i
   if (!m || count < 0) return HTAM_EINVAL;
   if (count == 0) return HTAM_OK;
   if (!entries || !group_ids || !aligned16(entries) || !aligned16(group_ids)) return HTAM_EINVAL;
-  if (m->n + count > m->capacity) return HTAM_ECAPACITY;
   return append_impl(m, entries, group_ids, count, nullptr, static_cast<cudaStream_t>(cuda_stream));
 }
 
@@ -115,7 +114,6 @@ htam_status htam_append_assign(htam_memory *m, const void *entries, const int32_
   if (!m || count < 0) return HTAM_EINVAL;
   if (count == 0) return HTAM_OK;
   if (!entries || !group_ids || !assigned || !aligned16(entries) || !aligned16(group_ids)) return HTAM_EINVAL;
-  if (m->n + count > m->capacity) return HTAM_ECAPACITY;
   return append_impl(m, entries, group_ids, count, assigned, static_cast<cudaStream_t>(cuda_stream));
 }
 
@@ -253,6 +251,8 @@ htam_status htam_query_flat(htam_memory *m, const void *queries, int32_t b, int3
   if (!(tau > 0.0f) || !(epsilon >= 0.0f && epsilon <= 1.0f) || !std::isfinite(1.0f / tau)) return HTAM_EINVAL;
   if (b > 0 && (!queries || !aligned16(queries) || !entry_idx || !entry_score || !entry_weight)) return HTAM_EINVAL;
   if (b == 0) return HTAM_OK;
+  htam_status s = refresh_mirror(m, true);  // the exact non-empty groups (after any queued append)
+  if (s != HTAM_OK) return s;
   int64_t nonempty = 0;
   for (int64_t c : m->h_count) nonempty += c > 0;
   if ((int64_t)b * std::max<int64_t>(1, nonempty) > kMaxFlatRows) return HTAM_EINVAL;
@@ -306,7 +306,13 @@ htam_status htam_query_host(htam_memory *m, const void *queries, int32_t b, cons
 htam_status htam_memory_info(const htam_memory *m, int64_t *n, int32_t *d, int32_t *n_groups,
                              int64_t *capacity) {
   if (!m) return HTAM_EINVAL;
-  if (n) *n = m->n;
+  if (n) {
+    // The host mirror is a cache of device state: waiting for the last
+    // append's copy updates it, not the memory.
+    htam_status s = refresh_mirror(const_cast<htam_memory *>(m), true);
+    if (s != HTAM_OK) return s;
+    *n = m->n;
+  }
   if (d) *d = m->d;
   if (n_groups) *n_groups = m->n_groups;
   if (capacity) *capacity = m->capacity;
@@ -315,6 +321,8 @@ htam_status htam_memory_info(const htam_memory *m, int64_t *n, int32_t *d, int32
 
 htam_status htam_memory_group_counts(const htam_memory *m, int64_t *counts) {
   if (!m || !counts) return HTAM_EINVAL;
+  htam_status s = refresh_mirror(const_cast<htam_memory *>(m), true);  // a cache of device state
+  if (s != HTAM_OK) return s;
   std::memcpy(counts, m->h_count.data(), sizeof(int64_t) * m->n_groups);
   return HTAM_OK;
 }
@@ -334,7 +342,11 @@ htam_status htam_device_status(htam_memory *m, void *cuda_stream) {
   HTAM_CK(cudaMemcpyAsync(&word, m->status, sizeof word, cudaMemcpyDeviceToHost, st));
   HTAM_CK(cudaMemsetAsync(m->status, 0, sizeof(unsigned int), st));
   HTAM_CK(cudaStreamSynchronize(st));
-  return word ? HTAM_ETIMEOUT : HTAM_OK;
+  htam_status s = refresh_mirror(m, true);
+  if (s != HTAM_OK) return s;
+  if (word & 1u) return HTAM_ETIMEOUT;
+  if (word & 2u) return HTAM_EINVAL;  // an append was rejected on the device
+  return HTAM_OK;
 }
 
 htam_status htam_set_tuning(htam_memory *m, htam_tuning key, int32_t value) {

@@ -50,7 +50,12 @@ constexpr size_t kCSmem = 1024 + kCStages * (kCABytes + 2 * kCBBytes) + sizeof(C
 __global__ void __launch_bounds__(kCThreads, kCPerSM)
     coarse_tc_kernel(const __grid_constant__ CUtensorMap q_map, const __grid_constant__ CUtensorMap hi_map,
                      const __grid_constant__ CUtensorMap lo_map, int d, int kb_per, const int32_t *__restrict__ count,
-                     int B, int G, float *__restrict__ s1, unsigned *status, uint32_t max_polls) {
+                     int B, int G, float *__restrict__ s1, unsigned *status, uint32_t max_polls,
+                     const int32_t *__restrict__ gate) {
+  // Gated launch (rows appended without a group): nothing to score.  The
+  // exit is uniform over the grid and comes before any barrier or tensor
+  // memory is set up.
+  if (gate && *gate == 0) return;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t *smem = smem_raw + ((1024 - (smem_addr(smem_raw) & 1023)) & 1023);
   uint8_t *st_a = smem;
@@ -195,7 +200,7 @@ int coarse_tc_splits(int B, int d, int G, int sm_count) {
 
 htam_status launch_coarse_tc(const void *queries, int B, int d, const __nv_bfloat16 *hi, const __nv_bfloat16 *lo,
                              const int32_t *count, int G, int splits, float *s1, unsigned *status,
-                             uint32_t max_polls, cudaStream_t st) {
+                             uint32_t max_polls, cudaStream_t st, const int32_t *gate) {
   CUtensorMap q_map, hi_map, lo_map;
   htam_status s = make_bf16_tile_map(&q_map, queries, B, d, kCM);
   if (s == HTAM_OK) s = make_bf16_tile_map(&hi_map, hi, G, d, kPageRows);
@@ -210,7 +215,7 @@ htam_status launch_coarse_tc(const void *queries, int B, int d, const __nv_bfloa
   if (splits < 1 || (int)ceil_div((int64_t)nk, kb_per) != splits) return HTAM_EINVAL;  // no empty split
   dim3 grid((unsigned)ceil_div(B, kCM), (unsigned)ceil_div(G, kCN), (unsigned)splits);
   coarse_tc_kernel<<<grid, kCThreads, kCSmem, st>>>(q_map, hi_map, lo_map, d, kb_per, count, B, G, s1, status,
-                                                     max_polls);
+                                                     max_polls, gate);
   HTAM_CK_LAUNCH("coarse_tc_kernel");
   return HTAM_OK;
 }

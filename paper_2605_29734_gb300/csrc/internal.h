@@ -17,10 +17,12 @@ struct htam_memory {
   int32_t n_groups = 0;
   htam_dtype dtype = HTAM_BF16;
   int elem_bytes = 2;
-  int64_t n = 0;           // entries stored
+  // Entries stored, as the host sees it: the device's count at the last
+  // adopted mirror plus the rows of every append queued since (an append the
+  // device rejects is subtracted once a later mirror shows it).
+  int64_t n = 0;
   int64_t capacity = 0;    // most entries ever stored
   int64_t n_pages_max = 0; // pages reserved: ceil(capacity/128) + n_groups
-  int64_t n_pages_used = 0;
 
   // Paged storage: page p holds rows [p*128, p*128+128) of `pool`; each row
   // is d elements of dtype.  Group g owns pages page_list[page_off[g] ..
@@ -30,7 +32,13 @@ struct htam_memory {
   int32_t *slot_id = nullptr;    // [n_pages_max*128] entry id of each row, -1 if empty
   int32_t *page_list = nullptr;  // [n_pages_max]
   int32_t *page_off = nullptr;   // [n_groups+1]
+  // The layout an append writes (it reads the one above); the host swaps the
+  // two pairs after queueing each append, so the pair above is always the
+  // current one in stream order.
+  int32_t *page_list_alt = nullptr;
+  int32_t *page_off_alt = nullptr;
   int32_t *count = nullptr;      // [n_groups] entries per group (device copy)
+  int64_t *dev_ctr = nullptr;    // [2] entries stored, pages used (device)
 
   // Group keys: fp64 running sums (exact enough to update in place), the
   // fp32 mean, and the mean split into bf16 hi + lo parts.
@@ -41,9 +49,24 @@ struct htam_memory {
 
   unsigned int *status = nullptr;   // device status word (bit 0: a wait gave up)
 
-  // Host mirrors of the layout.
+  // Host mirror of the group sizes, exact as of the append numbered
+  // mirror_seq; rows_pending rows were queued after it.  Appends run on the
+  // device without a host round trip: each one ends by copying the device
+  // sizes and entry count into a pinned slot of a small ring and recording an
+  // event; a later call adopts the newest slot whose event has completed
+  // (htam_device_status and the introspection calls wait for it).
+  static constexpr int kMirrorSlots = 4;
   std::vector<int64_t> h_count;
-  std::vector<std::vector<int32_t>> h_pages;
+  int64_t rows_pending = 0;
+  int64_t rows_issued = 0;       // rows of all appends queued (and the build)
+  int64_t append_seq = 0;        // appends queued
+  int64_t mirror_seq = 0;        // the append the mirror reflects
+  void *h_pin = nullptr;         // kMirrorSlots x (int64 n, int32 counts[G])
+  size_t pin_slot_bytes = 0;
+  cudaEvent_t mirror_ev[kMirrorSlots] = {};
+  int64_t slot_seq[kMirrorSlots] = {};       // append number each slot holds (0 = none)
+  int64_t slot_rows_issued[kMirrorSlots] = {};
+  cudaStream_t last_stream = nullptr;        // stream of the last append
 
   // Scratch owned by the object, grown on demand (never shrinks).
   void *scratch = nullptr;
@@ -100,6 +123,11 @@ struct Carver {
   static size_t round(size_t bytes) { return (bytes + 255) & ~size_t(255); }
 };
 
+// Adopts the newest completed mirror slot.  wait = true first waits for the
+// newest slot's event (the mirror is then exact unless a later append was
+// queued meanwhile).  Returns HTAM_ECUDA if waiting failed.
+htam_status refresh_mirror(htam_memory *m, bool wait);
+
 htam_status build_impl(const void *entries, const int32_t *group_ids, int64_t n, int32_t d,
                        int32_t n_groups, htam_dtype dtype, int64_t capacity, cudaStream_t st,
                        htam_memory **out);
@@ -126,14 +154,18 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t b,
 // Largest b * (non-empty groups) the flat scan takes (its bucket rows).
 constexpr int64_t kMaxFlatRows = int64_t(1) << 28;
 void free_impl(htam_memory *m);
-// ids[i] = gid[i] where gid[i] >= 0, else the group whose key scores highest
-// against row i of `entries` (stage 1's scorer and ranking with k = 1).  The
-// ids go to `dst` (`count` of them; it may be `gid` itself) or, when dst is
-// NULL, to m->assign_buf; *ids_out points at them.  The scratch is
-// m->assign_buf, grown on demand (which synchronises the device).
+// Rows of `entries` whose id in gid is -1 join the group whose key scores
+// highest against them (stage 1's scorer and ranking with k = 1, by the keys
+// as they stand before the append).  Queued without a host round trip: every
+// kernel is gated on *n_unassigned (the batch's tally of such rows, on the
+// device) and does nothing when it is zero.  For each such row e: ids[e] =
+// the chosen group and bcount[that group] += 1; a row that finds no
+// non-empty group sets *bad.  Scratch: m->assign_buf, grown with cudaMalloc
+// on demand (a growth synchronises the device).
 struct PhaseMark;
-htam_status assign_nearest(htam_memory *m, const void *entries, const int32_t *gid, int64_t count, int32_t *dst,
-                           const int32_t **ids_out, cudaStream_t st, PhaseMark *mark = nullptr);
+htam_status assign_unassigned(htam_memory *m, const void *entries, const int32_t *gid, int64_t count,
+                              const int32_t *n_unassigned, int32_t *ids, int32_t *bcount, int32_t *bad,
+                              cudaStream_t st, PhaseMark *mark = nullptr);
 
 // Weights alpha_1..alpha_P of a prefix (Eq. 10), passed by value to the
 // reduction kernel.

@@ -37,15 +37,18 @@ static int key_seg_rows(int64_t count) {
   return r;
 }
 
-// Per-group counts of a batch; ids of -1 (no group given) are counted apart,
-// any other id outside [0, n_groups) sets `bad`.
+// Per-group counts of a batch.  Ids of -1 (no group given) are counted
+// apart when `allow_unassigned`, and count as bad otherwise; any other id
+// outside [0, n_groups) sets `bad`.  The same grid also clears the stable
+// sort's (group, chunk) counters.
 __global__ void count_groups_kernel(const int32_t *__restrict__ gid, int64_t n, int32_t n_groups,
-                                    int32_t *__restrict__ counts, int32_t *__restrict__ bad,
-                                    int32_t *__restrict__ unassigned) {
-  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < n;
-       e += (int64_t)gridDim.x * blockDim.x) {
+                                    int allow_unassigned, int32_t *__restrict__ counts, int32_t *__restrict__ bad,
+                                    int32_t *__restrict__ unassigned, int32_t *__restrict__ hist,
+                                    int64_t hist_len) {
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < n; e += stride) {
     int32_t g = gid[e];
-    if (g == -1) {
+    if (g == -1 && allow_unassigned) {
       atomicAdd(unassigned, 1);
     } else if (g < 0 || g >= n_groups) {
       atomicOr(bad, 1);
@@ -53,21 +56,154 @@ __global__ void count_groups_kernel(const int32_t *__restrict__ gid, int64_t n, 
       atomicAdd(&counts[g], 1);
     }
   }
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < hist_len; i += stride) hist[i] = 0;
+}
+
+// The group of row e: its given id, or for a row given -1 the group the
+// nearest-key assignment chose.
+__device__ __forceinline__ int32_t row_group(const int32_t *__restrict__ gid, const int32_t *__restrict__ ids,
+                                             int64_t e) {
+  const int32_t g = gid[e];
+  return g >= 0 ? g : ids[e];
+}
+
+struct KeySeg {
+  int32_t g, r0, r1, pad;
+};
+struct KeyGroup {
+  int32_t g, seg0, seg1, count;
+};
+
+// Inclusive scan of one value per thread over a block of kLayoutThreads.
+constexpr int kLayoutThreads = 1024;
+__device__ __forceinline__ int64_t block_scan_incl(int64_t v, int64_t *sh /* [32] */) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int64_t t = __shfl_up_sync(kFullMask, v, o);
+    if (lane >= o) v += t;
+  }
+  if (lane == 31) sh[warp] = v;
+  __syncthreads();
+  if (warp == 0) {
+    int64_t w = lane < kLayoutThreads / 32 ? sh[lane] : 0;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int64_t t = __shfl_up_sync(kFullMask, w, o);
+      if (lane >= o) w += t;
+    }
+    sh[lane] = w;
+  }
+  __syncthreads();
+  const int64_t r = v + (warp > 0 ? sh[warp - 1] : 0);
+  __syncthreads();  // sh is reused by the next scan
+  return r;
+}
+
+// One block lays out a batch on the device (the page layout, the key
+// segments, the new sizes), so an append needs no host round trip.
+//   per group g: old = count[g], add = bcount[g], new = old + add;
+//   pages: ceil(new/128) in total, of which the ones beyond ceil(old/128)
+//     are fresh pages taken from the pool cursor dev_ctr[1] in group order;
+//   page_off_new = the exclusive scan of the page totals; first_new[g] =
+//     g's first fresh page;
+//   key segments over the new rows of every touched group (rows old.. new in
+//     steps of seg_rows) and one KeyGroup per touched group;
+//   base[g] = old (the stable sort's starting slot), count[g] = new;
+//   meta[0..1] = segment and touched-group counts, *id_base = the entry count
+//     before the batch, and the entry count grows by `rows`.
+// A bad batch changes nothing: the current offsets are copied to the new
+// layout, no segment is listed, and status bit 1 records the rejection.
+__global__ void __launch_bounds__(kLayoutThreads, 1)
+    layout_kernel(int32_t G, int64_t rows, int seg_rows, const int32_t *__restrict__ bcount,
+                  const int32_t *__restrict__ bad, int32_t *__restrict__ count,
+                  const int32_t *__restrict__ page_off_cur, int32_t *__restrict__ page_off_new,
+                  int32_t *__restrict__ first_new, int32_t *__restrict__ base, KeySeg *__restrict__ segs,
+                  KeyGroup *__restrict__ kgroups, int32_t *__restrict__ meta, int64_t *__restrict__ id_base,
+                  int64_t *__restrict__ dev_ctr, unsigned *__restrict__ status) {
+  __shared__ int64_t sh[32];
+  if (*bad) {
+    for (int g = threadIdx.x; g <= G; g += blockDim.x) page_off_new[g] = page_off_cur[g];
+    if (threadIdx.x == 0) {
+      meta[0] = 0;
+      meta[1] = 0;
+      atomicOr(status, 2u);
+    }
+    return;
+  }
+  const int per = (int)ceil_div(G, kLayoutThreads);
+  const int g0 = min(G, (int)threadIdx.x * per), g1 = min(G, g0 + per);
+  int64_t tp = 0, np = 0, ns = 0, nt = 0;  // this thread's pages, fresh pages, segments, touched groups
+  for (int g = g0; g < g1; ++g) {
+    const int64_t old = count[g], add = bcount[g], nw = old + add;
+    tp += ceil_div(nw, kPageRows);
+    np += ceil_div(nw, kPageRows) - ceil_div(old, kPageRows);
+    ns += ceil_div(add, seg_rows);
+    nt += add > 0;
+  }
+  int64_t o_tp = block_scan_incl(tp, sh) - tp;
+  int64_t o_np = block_scan_incl(np, sh) - np;
+  int64_t o_ns = block_scan_incl(ns, sh) - ns;
+  int64_t o_nt = block_scan_incl(nt, sh) - nt;
+  const int64_t pages_used = dev_ctr[1];
+  for (int g = g0; g < g1; ++g) {
+    const int64_t old = count[g], add = bcount[g], nw = old + add;
+    page_off_new[g] = (int32_t)o_tp;
+    first_new[g] = (int32_t)(pages_used + o_np);
+    base[g] = (int32_t)old;
+    o_tp += ceil_div(nw, kPageRows);
+    o_np += ceil_div(nw, kPageRows) - ceil_div(old, kPageRows);
+    if (add > 0) {
+      const int32_t s0 = (int32_t)o_ns;
+      for (int64_t r = old; r < nw; r += seg_rows) {
+        segs[o_ns++] = KeySeg{g, (int32_t)r, (int32_t)min(nw, r + seg_rows), 0};
+      }
+      kgroups[o_nt++] = KeyGroup{g, s0, (int32_t)o_ns, (int32_t)nw};
+      count[g] = (int32_t)nw;
+    }
+  }
+  // The last thread's running offsets are the totals.
+  if (threadIdx.x == kLayoutThreads - 1) {
+    page_off_new[G] = (int32_t)o_tp;
+    meta[0] = (int32_t)o_ns;
+    meta[1] = (int32_t)o_nt;
+    *id_base = dev_ctr[0];
+    dev_ctr[0] += rows;
+    dev_ctr[1] = pages_used + o_np;
+  }
+}
+
+// One warp per group: the group's page list in the new layout (its current
+// pages, then its fresh ones).
+__global__ void page_copy_kernel(int32_t G, const int32_t *__restrict__ page_off_cur,
+                                 const int32_t *__restrict__ page_list_cur, const int32_t *__restrict__ page_off_new,
+                                 const int32_t *__restrict__ first_new, int32_t *__restrict__ page_list_new) {
+  const int g = (int)((blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5);
+  const int lane = threadIdx.x & 31;
+  if (g >= G) return;
+  const int32_t c0 = page_off_cur[g], n_old = page_off_cur[g + 1] - c0;
+  const int32_t n0 = page_off_new[g], n_tot = page_off_new[g + 1] - n0;
+  for (int32_t i = lane; i < n_tot; i += 32) {
+    page_list_new[n0 + i] = i < n_old ? page_list_cur[c0 + i] : first_new[g] + (i - n_old);
+  }
 }
 
 // hist[g * n_chunks + c] = number of rows of group g in chunk c.
-__global__ void chunk_hist_kernel(const int32_t *__restrict__ gid, int64_t n, int64_t chunk,
-                                  int64_t n_chunks, int32_t *__restrict__ hist) {
+__global__ void chunk_hist_kernel(const int32_t *__restrict__ gid, const int32_t *__restrict__ ids, int64_t n,
+                                  int64_t chunk, int64_t n_chunks, int32_t *__restrict__ hist,
+                                  const int32_t *__restrict__ bad) {
+  if (*bad) return;
   int64_t c = blockIdx.x;
   int64_t lo = c * chunk, hi = min(n, lo + chunk);
   for (int64_t e = lo + threadIdx.x; e < hi; e += blockDim.x) {
-    atomicAdd(&hist[(int64_t)gid[e] * n_chunks + c], 1);
+    atomicAdd(&hist[(int64_t)row_group(gid, ids, e) * n_chunks + c], 1);
   }
 }
 
 // Per group (one warp each): hist[g][c] <- base[g] + sum_{c' < c} hist[g][c'].
 __global__ void chunk_scan_kernel(int32_t *__restrict__ hist, int64_t n_chunks, int32_t n_groups,
-                                  const int32_t *__restrict__ base) {
+                                  const int32_t *__restrict__ base, const int32_t *__restrict__ bad) {
+  if (*bad) return;
   int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   int lane = threadIdx.x & 31;
   if (warp >= n_groups) return;
@@ -89,9 +225,10 @@ __global__ void chunk_scan_kernel(int32_t *__restrict__ hist, int64_t n_chunks, 
 
 // One warp per chunk walks its rows in order; rows of the same group take
 // consecutive slots (stable), so pos[e] = slot of row e within its group.
-__global__ void chunk_place_kernel(const int32_t *__restrict__ gid, int64_t n, int64_t chunk,
-                                   int64_t n_chunks, int32_t *__restrict__ hist,
-                                   int32_t *__restrict__ pos) {
+__global__ void chunk_place_kernel(const int32_t *__restrict__ gid, const int32_t *__restrict__ ids, int64_t n,
+                                   int64_t chunk, int64_t n_chunks, int32_t *__restrict__ hist,
+                                   int32_t *__restrict__ pos, const int32_t *__restrict__ bad) {
+  if (*bad) return;
   int64_t c = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
   int lane = threadIdx.x & 31;
   if (c >= n_chunks) return;
@@ -101,7 +238,7 @@ __global__ void chunk_place_kernel(const int32_t *__restrict__ gid, int64_t n, i
     int64_t e = b0 + lane;
     unsigned act = __ballot_sync(kFullMask, e < hi);
     if (e < hi) {
-      int32_t g = gid[e];
+      int32_t g = row_group(gid, ids, e);
       unsigned peers = __match_any_sync(act, g);
       int leader = __ffs(peers) - 1;
       int rank = __popc(peers & lt);
@@ -118,31 +255,34 @@ __global__ void chunk_place_kernel(const int32_t *__restrict__ gid, int64_t n, i
   }
 }
 
-// One warp per row: copy into its page slot, record its entry id.
-__global__ void place_rows_kernel(const uint4 *__restrict__ src, const int32_t *__restrict__ gid,
+// One warp per row: copy into its page slot, record its entry id (and, when
+// asked, the group it joined).
+__global__ void place_rows_kernel(const uint4 *__restrict__ src, const int32_t *gid, const int32_t *__restrict__ ids,
                                   const int32_t *__restrict__ pos, int64_t n, int vec_per_row,
-                                  const int32_t *__restrict__ page_list,
-                                  const int32_t *__restrict__ page_off, uint4 *__restrict__ pool,
-                                  int32_t *__restrict__ slot_id, int64_t id_base) {
+                                  const int32_t *__restrict__ page_list, const int32_t *__restrict__ page_off,
+                                  uint4 *__restrict__ pool, int32_t *__restrict__ slot_id,
+                                  const int64_t *__restrict__ id_base, int32_t *assigned,
+                                  const int32_t *__restrict__ bad) {
+  if (*bad) return;
   int64_t e = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
   int lane = threadIdx.x & 31;
-  if (e >= n) return;
-  int32_t g = gid[e];
+  if (e >= n) return;  // uniform per warp
+  // Lane 0 reads the group and hands it to the warp, so no lane reads gid[e]
+  // after lane 0 may have overwritten it through `assigned`.
+  int32_t g = lane == 0 ? row_group(gid, ids, e) : 0;
+  g = __shfl_sync(kFullMask, g, 0);
   int32_t p = pos[e];
   int64_t page = page_list[page_off[g] + p / kPageRows];
   int64_t slot = page * kPageRows + (p % kPageRows);
   const uint4 *s = src + e * vec_per_row;
   uint4 *dst = pool + slot * vec_per_row;
   for (int v = lane; v < vec_per_row; v += 32) dst[v] = s[v];
-  if (lane == 0) slot_id[slot] = (int32_t)(id_base + e);
+  if (lane == 0) {
+    slot_id[slot] = (int32_t)(*id_base + e);
+    if (assigned) assigned[e] = g;  // after this row's own read of gid[e] (assigned may be gid)
+  }
 }
 
-struct KeySeg {
-  int32_t g, r0, r1, pad;
-};
-struct KeyGroup {
-  int32_t g, seg0, seg1, count;
-};
 
 // partial[s][j] = sum over rows r0..r1-1 of group g of row[j], accumulated
 // in fp32 with Kahan compensation and returned as fp64 (sum + compensation),
@@ -152,8 +292,10 @@ template <typename T>
 __global__ void key_partial_kernel(const T *__restrict__ pool, int32_t d,
                                    const int32_t *__restrict__ page_list,
                                    const int32_t *__restrict__ page_off,
-                                   const KeySeg *__restrict__ segs, double *__restrict__ partial) {
+                                   const KeySeg *__restrict__ segs, const int32_t *__restrict__ n_segs,
+                                   double *__restrict__ partial) {
   constexpr int kBatch = 8;
+  if ((int)blockIdx.x >= *n_segs) return;  // the grid covers the host's bound on the segments
   const KeySeg sg = segs[blockIdx.x];
   const int j0 = (blockIdx.y * blockDim.x + threadIdx.x) * 8;
   if (j0 >= d) return;
@@ -199,10 +341,11 @@ __global__ void key_partial_kernel(const T *__restrict__ pool, int32_t d,
 
 // csum[g] += partials in segment order; refresh the fp32 mean and its bf16
 // hi/lo split for the group.
-__global__ void key_finalize_kernel(const KeyGroup *__restrict__ groups,
+__global__ void key_finalize_kernel(const KeyGroup *__restrict__ groups, const int32_t *__restrict__ n_groups,
                                     const double *__restrict__ partial, int32_t d,
                                     double *__restrict__ csum, float *__restrict__ cent,
                                     __nv_bfloat16 *__restrict__ hi, __nv_bfloat16 *__restrict__ lo) {
+  if ((int)blockIdx.x >= *n_groups) return;  // the grid covers every group
   KeyGroup kg = groups[blockIdx.x];
   for (int j = blockIdx.y * blockDim.x + threadIdx.x; j < d; j += gridDim.y * blockDim.x) {
     double add = 0.0;
@@ -240,11 +383,46 @@ htam_status ensure_scratch(htam_memory *m, size_t bytes) {
   return HTAM_OK;
 }
 
-// Files `count` rows (ids id_base..) under their groups and updates the keys
-// of the groups they join.  Arguments are already validated except the group
-// id range, which is checked on the device before anything is written.
+htam_status refresh_mirror(htam_memory *m, bool wait) {
+  if (m->mirror_seq == m->append_seq) return HTAM_OK;
+  constexpr int S = htam_memory::kMirrorSlots;
+  if (wait) {
+    const int newest = (int)(m->append_seq % S);
+    HTAM_CK(cudaEventSynchronize(m->mirror_ev[newest]));
+  }
+  // The newest slot whose copies have landed.
+  for (int64_t q = m->append_seq; q > m->mirror_seq && q > m->append_seq - S; --q) {
+    const int slot = (int)(q % S);
+    if (m->slot_seq[slot] != q) continue;
+    cudaError_t e = cudaEventQuery(m->mirror_ev[slot]);
+    if (e == cudaErrorNotReady) continue;
+    if (e != cudaSuccess) {
+      set_last_error("cudaEventQuery", e);
+      return HTAM_ECUDA;
+    }
+    const char *p = static_cast<const char *>(m->h_pin) + slot * m->pin_slot_bytes;
+    const int64_t n_dev = *reinterpret_cast<const int64_t *>(p);
+    const int32_t *c = reinterpret_cast<const int32_t *>(p + sizeof(int64_t));
+    for (int32_t g = 0; g < m->n_groups; ++g) m->h_count[g] = c[g];
+    m->mirror_seq = q;
+    m->rows_pending = m->rows_issued - m->slot_rows_issued[slot];
+    m->n = n_dev + m->rows_pending;
+    return HTAM_OK;
+  }
+  return HTAM_OK;
+}
+
+// Files `count` rows under their groups and updates the keys of the groups
+// they join (the memory update of Eq. 15), entirely on the device: the batch's
+// group sizes, the nearest-key choice for rows given -1 (appends only), the
+// page layout, the stable slot order and the key sums are all computed by
+// kernels queued on `st`, with no host round trip.  Group ids are checked on
+// the device: a bad batch (an id out of range, or -1 with no non-empty group
+// to join) is skipped by every kernel after the check and recorded in status
+// bit 1, leaving the memory unchanged.  `build` (the first batch of a new
+// memory) takes no -1 ids.
 static htam_status add_rows(htam_memory *m, const void *entries, const int32_t *gid, int64_t count,
-                            int32_t *assigned, cudaStream_t st) {
+                            int32_t *assigned, cudaStream_t st, bool build, int32_t **bad_out = nullptr) {
   if (count == 0) return HTAM_OK;
   const int32_t G = m->n_groups, d = m->d;
 
@@ -253,154 +431,118 @@ static htam_status add_rows(htam_memory *m, const void *entries, const int32_t *
   chunk = ceil_div(chunk, 32) * 32;
   int64_t n_chunks = ceil_div(count, chunk);
 
-  // Key segments need the final layout; their number is bounded by
-  // count/seg_rows + number of groups.
+  // Key segments: at most count/seg_rows + (touched groups) of them.
   const int seg_rows = key_seg_rows(count);
-  int64_t max_segs = count / seg_rows + G + 1;
+  int64_t max_segs = std::min<int64_t>(count, count / seg_rows + G + 1);
 
-  size_t need = Carver::round(sizeof(int32_t) * (G + 2)) + Carver::round(sizeof(int32_t) * count) +
-                Carver::round(sizeof(int32_t) * (size_t)G * n_chunks) +
+  size_t need = Carver::round(sizeof(int32_t) * (G + 2)) + Carver::round(sizeof(int32_t) * 4) +
+                Carver::round(sizeof(int64_t)) + (build ? 0 : Carver::round(sizeof(int32_t) * count)) +
+                Carver::round(sizeof(int32_t) * count) + Carver::round(sizeof(int32_t) * (size_t)G * n_chunks) +
                 Carver::round(sizeof(KeySeg) * max_segs) + Carver::round(sizeof(KeyGroup) * G) +
-                Carver::round(sizeof(double) * (size_t)max_segs * d) + 4096;
+                2 * Carver::round(sizeof(int32_t) * G) + Carver::round(sizeof(double) * (size_t)max_segs * d) + 4096;
   htam_status s = ensure_scratch(m, need);
   if (s != HTAM_OK) return s;
   Carver cv(m->scratch);
   int32_t *bcount = cv.take<int32_t>(G + 2);  // [G] counts, bad flag, rows without a group
+  int32_t *meta = cv.take<int32_t>(4);         // key segments, touched groups
+  int64_t *id_base = cv.take<int64_t>(1);
+  int32_t *ids = build ? nullptr : cv.take<int32_t>(count);  // groups chosen for rows given -1
   int32_t *pos = cv.take<int32_t>(count);
   int32_t *hist = cv.take<int32_t>((size_t)G * n_chunks);
   KeySeg *segs = cv.take<KeySeg>(max_segs);
   KeyGroup *kgroups = cv.take<KeyGroup>(G);
+  int32_t *first_new = cv.take<int32_t>(G);
+  int32_t *base = cv.take<int32_t>(G);
   double *partial = cv.take<double>((size_t)max_segs * d);
+  int32_t *bad = bcount + G;
+  if (bad_out) *bad_out = bad;
 
   PhaseMark mark(m, st);
   mark.begin(HTAM_PHASE_APPEND);
 
-  // 1. Per-group counts of the batch and the group-id range check.
-  std::vector<int32_t> h_b(G + 2);
-  auto count_batch = [&](const int32_t *ids) -> htam_status {
-    HTAM_CK(cudaMemsetAsync(bcount, 0, sizeof(int32_t) * (G + 2), st));
-    int blocks = (int)std::min<int64_t>(ceil_div(count, 256), 4096);
-    count_groups_kernel<<<blocks, 256, 0, st>>>(ids, count, G, bcount, bcount + G, bcount + G + 1);
+  // 1. Per-group counts of the batch and the group-id range check (the same
+  //    grid clears the slot counters).
+  HTAM_CK(cudaMemsetAsync(bcount, 0, sizeof(int32_t) * (G + 2), st));
+  {
+    const int blocks = (int)std::min<int64_t>(ceil_div(std::max<int64_t>(count, (int64_t)G * n_chunks), 256), 4096);
+    count_groups_kernel<<<blocks, 256, 0, st>>>(gid, count, G, build ? 0 : 1, bcount, bad, bcount + G + 1, hist,
+                                                (int64_t)G * n_chunks);
     HTAM_CK_LAUNCH("count_groups_kernel");
     mark.launched();
-    HTAM_CK(cudaMemcpyAsync(h_b.data(), bcount, sizeof(int32_t) * (G + 2), cudaMemcpyDeviceToHost, st));
-    HTAM_CK(cudaStreamSynchronize(st));
-    return HTAM_OK;
-  };
-  s = count_batch(gid);
-  if (s != HTAM_OK) return s;
-  if (h_b[G] != 0) return HTAM_EINVAL;
-  if (h_b[G + 1] > 0) {
-    // Rows without a group join the group whose key scores highest against
-    // them, by the keys as they stand before this call (none: EINVAL).
-    bool any = false;
-    for (int64_t c : m->h_count) any |= c > 0;
-    if (!any) return HTAM_EINVAL;
-    const int32_t *ids = nullptr;
-    s = assign_nearest(m, entries, gid, count, assigned, &ids, st, &mark);
+  }
+  // 2. Rows without a group join the group whose key scores highest against
+  //    them, by the keys as they stand before this call.  The kernels run
+  //    only when the count above found such rows.
+  if (!build) {
+    s = assign_unassigned(m, entries, gid, count, bcount + G + 1, ids, bcount, bad, st, &mark);
     if (s != HTAM_OK) return s;
-    gid = ids;
-    s = count_batch(gid);
-    if (s != HTAM_OK) return s;
-  } else if (assigned && assigned != gid) {
-    HTAM_CK(cudaMemcpyAsync(assigned, gid, sizeof(int32_t) * count, cudaMemcpyDeviceToDevice, st));
   }
+  // 3. Page layout, key segments and new sizes; then the page lists.
+  layout_kernel<<<1, kLayoutThreads, 0, st>>>(G, count, seg_rows, bcount, bad, m->count, m->page_off,
+                                              m->page_off_alt, first_new, base, segs, kgroups, meta, id_base,
+                                              m->dev_ctr, m->status);
+  HTAM_CK_LAUNCH("layout_kernel");
+  page_copy_kernel<<<(unsigned)ceil_div((int64_t)G * 32, 256), 256, 0, st>>>(G, m->page_off, m->page_list,
+                                                                             m->page_off_alt, first_new,
+                                                                             m->page_list_alt);
+  HTAM_CK_LAUNCH("page_copy_kernel");
+  mark.launched(2);
 
-  // 2. Page layout on the host.
-  std::vector<int64_t> new_count(G);
-  int64_t new_pages = 0;
-  for (int32_t g = 0; g < G; ++g) {
-    new_count[g] = m->h_count[g] + h_b[g];
-    new_pages += ceil_div(new_count[g], kPageRows) - ceil_div(m->h_count[g], kPageRows);
-  }
-  if (m->n + count > m->capacity || m->n_pages_used + new_pages > m->n_pages_max) {
-    return HTAM_ECAPACITY;
-  }
-  // Every check has passed: from here on the layout is extended in place.
-  std::vector<std::vector<int32_t>> &pages = m->h_pages;
-  int64_t next_page = m->n_pages_used;
-  std::vector<int32_t> h_off(G + 1), h_list;
-  h_list.reserve((size_t)(m->n_pages_used + new_pages));
-  for (int32_t g = 0; g < G; ++g) {
-    int64_t want = ceil_div(new_count[g], kPageRows);
-    while ((int64_t)pages[g].size() < want) pages[g].push_back((int32_t)next_page++);
-    h_off[g] = (int32_t)h_list.size();
-    h_list.insert(h_list.end(), pages[g].begin(), pages[g].end());
-  }
-  h_off[G] = (int32_t)h_list.size();
-
-  // Key segments over the new rows of every touched group.
-  std::vector<KeySeg> h_segs;
-  std::vector<KeyGroup> h_kg;
-  for (int32_t g = 0; g < G; ++g) {
-    if (h_b[g] == 0) continue;
-    KeyGroup kg{g, (int32_t)h_segs.size(), 0, (int32_t)new_count[g]};
-    for (int64_t r = m->h_count[g]; r < new_count[g]; r += seg_rows) {
-      h_segs.push_back(KeySeg{g, (int32_t)r, (int32_t)std::min<int64_t>(new_count[g], r + seg_rows), 0});
-    }
-    kg.seg1 = (int32_t)h_segs.size();
-    h_kg.push_back(kg);
-  }
-
-  // From here on the memory is modified.  Upload the layout (stream
-  // ordered after any earlier query on this stream).
-  HTAM_CK(cudaMemcpyAsync(m->page_off, h_off.data(), sizeof(int32_t) * (G + 1), cudaMemcpyHostToDevice, st));
-  if (!h_list.empty()) {
-    HTAM_CK(cudaMemcpyAsync(m->page_list, h_list.data(), sizeof(int32_t) * h_list.size(),
-                            cudaMemcpyHostToDevice, st));
-  }
-  HTAM_CK(cudaMemcpyAsync(segs, h_segs.data(), sizeof(KeySeg) * h_segs.size(), cudaMemcpyHostToDevice, st));
-  HTAM_CK(cudaMemcpyAsync(kgroups, h_kg.data(), sizeof(KeyGroup) * h_kg.size(), cudaMemcpyHostToDevice, st));
-
-  // 3. Stable slot assignment: pos[e] = old count of its group + rank among
+  // 4. Stable slot assignment: pos[e] = old size of its group + rank among
   //    earlier rows of the batch with the same group.
-  HTAM_CK(cudaMemsetAsync(hist, 0, sizeof(int32_t) * (size_t)G * n_chunks, st));
-  chunk_hist_kernel<<<(unsigned)n_chunks, 256, 0, st>>>(gid, count, chunk, n_chunks, hist);
+  chunk_hist_kernel<<<(unsigned)n_chunks, 256, 0, st>>>(gid, ids, count, chunk, n_chunks, hist, bad);
   HTAM_CK_LAUNCH("chunk_hist_kernel");
-  chunk_scan_kernel<<<(unsigned)ceil_div((int64_t)G * 32, 256), 256, 0, st>>>(hist, n_chunks, G, m->count);
+  chunk_scan_kernel<<<(unsigned)ceil_div((int64_t)G * 32, 256), 256, 0, st>>>(hist, n_chunks, G, base, bad);
   HTAM_CK_LAUNCH("chunk_scan_kernel");
-  chunk_place_kernel<<<(unsigned)ceil_div(n_chunks * 32, 256), 256, 0, st>>>(gid, count, chunk, n_chunks, hist, pos);
+  chunk_place_kernel<<<(unsigned)ceil_div(n_chunks * 32, 256), 256, 0, st>>>(gid, ids, count, chunk, n_chunks, hist,
+                                                                             pos, bad);
   HTAM_CK_LAUNCH("chunk_place_kernel");
   mark.launched(3);
 
-  // 4. Copy rows into their slots.
+  // 5. Copy rows into their slots.
   int vec_per_row = d * m->elem_bytes / 16;
   place_rows_kernel<<<(unsigned)ceil_div(count * 32, 256), 256, 0, st>>>(
-      static_cast<const uint4 *>(entries), gid, pos, count, vec_per_row, m->page_list, m->page_off,
-      static_cast<uint4 *>(m->pool), m->slot_id, m->n);
+      static_cast<const uint4 *>(entries), gid, ids, pos, count, vec_per_row, m->page_list_alt, m->page_off_alt,
+      static_cast<uint4 *>(m->pool), m->slot_id, id_base, assigned, bad);
   HTAM_CK_LAUNCH("place_rows_kernel");
   mark.launched();
 
-  // 5. Keys of the touched groups.
-  if (!h_segs.empty()) {
-    dim3 grid((unsigned)h_segs.size(), (unsigned)ceil_div(d, 256 * 8));
+  // 6. Keys of the touched groups.
+  {
+    dim3 grid((unsigned)max_segs, (unsigned)ceil_div(d, 256 * 8));
     if (m->dtype == HTAM_BF16) {
-      key_partial_kernel<__nv_bfloat16><<<grid, 256, 0, st>>>(
-          static_cast<const __nv_bfloat16 *>(m->pool), d, m->page_list, m->page_off, segs, partial);
+      key_partial_kernel<__nv_bfloat16><<<grid, 256, 0, st>>>(static_cast<const __nv_bfloat16 *>(m->pool), d,
+                                                              m->page_list_alt, m->page_off_alt, segs, meta,
+                                                              partial);
     } else {
-      key_partial_kernel<float><<<grid, 256, 0, st>>>(static_cast<const float *>(m->pool), d,
-                                                      m->page_list, m->page_off, segs, partial);
+      key_partial_kernel<float><<<grid, 256, 0, st>>>(static_cast<const float *>(m->pool), d, m->page_list_alt,
+                                                      m->page_off_alt, segs, meta, partial);
     }
     HTAM_CK_LAUNCH("key_partial_kernel");
-    dim3 g2((unsigned)h_kg.size(), (unsigned)std::min<int64_t>(ceil_div(d, 256), 16));
-    key_finalize_kernel<<<g2, 256, 0, st>>>(kgroups, partial, d, m->csum, m->cent, m->cent_hi, m->cent_lo);
+    dim3 g2((unsigned)G, (unsigned)std::min<int64_t>(ceil_div(d, 256), 16));
+    key_finalize_kernel<<<g2, 256, 0, st>>>(kgroups, meta + 1, partial, d, m->csum, m->cent, m->cent_hi,
+                                            m->cent_lo);
     HTAM_CK_LAUNCH("key_finalize_kernel");
     mark.launched(2);
   }
 
-  // 6. New device counts and host mirrors.
-  std::vector<int32_t> h_c32(G);
-  for (int32_t g = 0; g < G; ++g) h_c32[g] = (int32_t)new_count[g];
-  HTAM_CK(cudaMemcpyAsync(m->count, h_c32.data(), sizeof(int32_t) * G, cudaMemcpyHostToDevice, st));
-  mark.end();
-  // The host vectors above are pageable, so cudaMemcpyAsync staged them
-  // before returning; the key and segment tables in scratch are read by the
-  // kernels above in stream order, before any later call on the stream can
-  // reuse the scratch (a reallocation frees it only after a device
-  // synchronisation).  Nothing here needs to wait for the GPU.
-  m->h_count.swap(new_count);
-  m->n_pages_used = next_page;
+  // 7. The new layout is current from here on in stream order; the sizes
+  //    and the entry count go to the next mirror slot.
+  std::swap(m->page_list, m->page_list_alt);
+  std::swap(m->page_off, m->page_off_alt);
+  m->append_seq += 1;
+  m->rows_issued += count;
+  m->rows_pending += count;
   m->n += count;
+  const int slot = (int)(m->append_seq % htam_memory::kMirrorSlots);
+  char *pin = static_cast<char *>(m->h_pin) + slot * m->pin_slot_bytes;
+  HTAM_CK(cudaMemcpyAsync(pin, m->dev_ctr, sizeof(int64_t), cudaMemcpyDeviceToHost, st));
+  HTAM_CK(cudaMemcpyAsync(pin + sizeof(int64_t), m->count, sizeof(int32_t) * G, cudaMemcpyDeviceToHost, st));
+  HTAM_CK(cudaEventRecord(m->mirror_ev[slot], st));
+  m->slot_seq[slot] = m->append_seq;
+  m->slot_rows_issued[slot] = m->rows_issued;
+  m->last_stream = st;
+  mark.end();
   return HTAM_OK;
 }
 
@@ -413,6 +555,13 @@ void free_impl(htam_memory *m) {
   cudaFree(m->slot_id);
   cudaFree(m->page_list);
   cudaFree(m->page_off);
+  cudaFree(m->page_list_alt);
+  cudaFree(m->page_off_alt);
+  cudaFree(m->dev_ctr);
+  if (m->h_pin) cudaFreeHost(m->h_pin);
+  for (cudaEvent_t e : m->mirror_ev) {
+    if (e) cudaEventDestroy(e);
+  }
   cudaFree(m->count);
   cudaFree(m->csum);
   cudaFree(m->cent);
@@ -449,7 +598,6 @@ htam_status build_impl(const void *entries, const int32_t *gid, int64_t n, int32
   m->capacity = capacity;
   m->n_pages_max = ceil_div(capacity, kPageRows) + n_groups;
   m->h_count.assign(n_groups, 0);
-  m->h_pages.assign(n_groups, {});
 
   auto fail = [&](htam_status s) {
     free_impl(m);
@@ -461,6 +609,9 @@ htam_status build_impl(const void *entries, const int32_t *gid, int64_t n, int32
       cudaMalloc(&m->slot_id, sizeof(int32_t) * m->n_pages_max * kPageRows) != cudaSuccess ||
       cudaMalloc(&m->page_list, sizeof(int32_t) * m->n_pages_max) != cudaSuccess ||
       cudaMalloc(&m->page_off, sizeof(int32_t) * (n_groups + 1)) != cudaSuccess ||
+      cudaMalloc(&m->page_list_alt, sizeof(int32_t) * m->n_pages_max) != cudaSuccess ||
+      cudaMalloc(&m->page_off_alt, sizeof(int32_t) * (n_groups + 1)) != cudaSuccess ||
+      cudaMalloc(&m->dev_ctr, sizeof(int64_t) * 2) != cudaSuccess ||
       cudaMalloc(&m->count, sizeof(int32_t) * n_groups) != cudaSuccess ||
       cudaMalloc(&m->csum, sizeof(double) * gd) != cudaSuccess ||
       cudaMalloc(&m->cent, sizeof(float) * gd) != cudaSuccess ||
@@ -470,10 +621,26 @@ htam_status build_impl(const void *entries, const int32_t *gid, int64_t n, int32
     cudaGetLastError();
     return fail(HTAM_ENOMEM);
   }
+  // Pinned mirror slots (entry count + group sizes) and their events.
+  m->pin_slot_bytes = Carver::round(sizeof(int64_t) + sizeof(int32_t) * (size_t)n_groups);
+  if (cudaMallocHost(&m->h_pin, m->pin_slot_bytes * htam_memory::kMirrorSlots) != cudaSuccess) {
+    cudaGetLastError();
+    m->h_pin = nullptr;
+    return fail(HTAM_ENOMEM);
+  }
+  for (cudaEvent_t &e : m->mirror_ev) {
+    if (cudaEventCreateWithFlags(&e, cudaEventDisableTiming) != cudaSuccess) {
+      cudaGetLastError();
+      e = nullptr;
+      return fail(HTAM_ECUDA);
+    }
+  }
   // Empty rows are zero (never NaN), empty slots have id -1, keys start at 0.
   if (cudaMemsetAsync(m->pool, 0, pool_bytes, st) != cudaSuccess ||
       cudaMemsetAsync(m->slot_id, 0xff, sizeof(int32_t) * m->n_pages_max * kPageRows, st) != cudaSuccess ||
       cudaMemsetAsync(m->page_off, 0, sizeof(int32_t) * (n_groups + 1), st) != cudaSuccess ||
+      cudaMemsetAsync(m->page_off_alt, 0, sizeof(int32_t) * (n_groups + 1), st) != cudaSuccess ||
+      cudaMemsetAsync(m->dev_ctr, 0, sizeof(int64_t) * 2, st) != cudaSuccess ||
       cudaMemsetAsync(m->count, 0, sizeof(int32_t) * n_groups, st) != cudaSuccess ||
       cudaMemsetAsync(m->csum, 0, sizeof(double) * gd, st) != cudaSuccess ||
       cudaMemsetAsync(m->cent, 0, sizeof(float) * gd, st) != cudaSuccess ||
@@ -483,7 +650,19 @@ htam_status build_impl(const void *entries, const int32_t *gid, int64_t n, int32
     set_last_error("cudaMemsetAsync", cudaGetLastError());
     return fail(HTAM_ECUDA);
   }
-  htam_status s = add_rows(m, entries, gid, n, nullptr, st);
+  // The build is the one synchronous batch: a group id out of range fails
+  // the call (and frees the memory) instead of being reported later.
+  int32_t *bad = nullptr;
+  htam_status s = add_rows(m, entries, gid, n, nullptr, st, /*build=*/true, &bad);
+  if (s != HTAM_OK) return fail(s);
+  int32_t h_bad = 0;
+  if (bad && (cudaMemcpyAsync(&h_bad, bad, sizeof h_bad, cudaMemcpyDeviceToHost, st) != cudaSuccess ||
+              cudaStreamSynchronize(st) != cudaSuccess)) {
+    set_last_error("htam_build_memory: reading the group-id check", cudaGetLastError());
+    return fail(HTAM_ECUDA);
+  }
+  if (h_bad) return fail(HTAM_EINVAL);
+  s = refresh_mirror(m, true);
   if (s != HTAM_OK) return fail(s);
   *out = m;
   return HTAM_OK;
@@ -491,8 +670,14 @@ htam_status build_impl(const void *entries, const int32_t *gid, int64_t n, int32
 
 htam_status append_impl(htam_memory *m, const void *entries, const int32_t *gid, int64_t count,
                         int32_t *assigned, cudaStream_t st) {
-  if (m->n + count > m->capacity) return HTAM_ECAPACITY;
-  return add_rows(m, entries, gid, count, assigned, st);
+  if (m->n + count > m->capacity) {
+    // The host's count may still include appends the device rejected: look
+    // at the device's before refusing.
+    htam_status s = refresh_mirror(m, true);
+    if (s != HTAM_OK) return s;
+    if (m->n + count > m->capacity) return HTAM_ECAPACITY;
+  }
+  return add_rows(m, entries, gid, count, assigned, st, /*build=*/false);
 }
 
 }  // namespace htam

@@ -34,7 +34,8 @@ namespace {
 template <typename T>
 __global__ void __launch_bounds__(256) coarse_scores_simt_kernel(
     const T *__restrict__ Q, int B, int d, const float *__restrict__ cent,
-    const int32_t *__restrict__ count, int G, float *__restrict__ s1) {
+    const int32_t *__restrict__ count, int G, float *__restrict__ s1, const int32_t *__restrict__ gate = nullptr) {
+  if (gate && *gate == 0) return;  // gated launch with nothing to score
   __shared__ float qs[32][68];
   __shared__ float cs[32][68];
   const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
@@ -112,7 +113,9 @@ __global__ void __launch_bounds__(NW * 32, 1) group_topk_kernel(const float *__r
                                                              int B, int G,
                                                              const int32_t *__restrict__ count, int kg,
                                                              int32_t *__restrict__ gidx,
-                                                             float *__restrict__ gscore) {
+                                                             float *__restrict__ gscore,
+                                                             const int32_t *__restrict__ gate = nullptr) {
+  if (gate && *gate == 0) return;  // gated launch with nothing to select
   __shared__ float ls[NW][64];
   __shared__ int li[NW][64];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -1286,6 +1289,12 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
                        float *entry_score, float *entry_weight, float *lse, cudaStream_t st,
                        const EdgeRoute *er, bool flat, const SampleSpec *smp) {
   if (B == 0) return HTAM_OK;
+  // The host mirror of the group sizes bounds the scratch below; the flat
+  // scan and the policy draws need the exact non-empty groups, so they wait
+  // for the mirror of the last append (the others take the newest one that
+  // has landed and bound the rows queued since).
+  htam_status s = refresh_mirror(m, flat || smp);
+  if (s != HTAM_OK) return s;
   m->n_queries += 1;
   PhaseMark mark(m, st);
   // The flat scan selects every non-empty group (at least one slot, -1 when
@@ -1304,13 +1313,16 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
 
   // Upper bound of the partial records: every query in the buckets of the
   // k_g groups with the most page segments (counted with the shorter
-  // segments of the two kernels).
+  // segments of the two kernels).  Rows queued after the mirror add at most
+  // pending/128 + k_g pages to any k_g groups, so at most
+  // (pending/128 + k_g)/seg_min + k_g segments.
   const int seg_min = std::min(kSimtSegPages, kTcSegPagesMin);
   std::vector<int64_t> nseg(G);
-  for (int g = 0; g < G; ++g) nseg[g] = ceil_div((int64_t)m->h_pages[g].size(), seg_min);
+  for (int g = 0; g < G; ++g) nseg[g] = ceil_div(ceil_div(m->h_count[g], kPageRows), seg_min);
   std::nth_element(nseg.begin(), nseg.begin() + (kg - 1), nseg.end(), std::greater<int64_t>());
   int64_t seg_sum = 0;
   for (int i = 0; i < kg; ++i) seg_sum += nseg[i];
+  if (m->rows_pending > 0) seg_sum += ceil_div(ceil_div(m->rows_pending, kPageRows) + kg, seg_min) + kg;
   const int64_t max_parts = std::max<int64_t>(1, (int64_t)B * seg_sum);
   const int64_t max_units = max_parts;
   const int64_t rows = (int64_t)B * kg;  // bucket rows
@@ -1333,7 +1345,7 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
                 Carver::round(sizeof(float2) * max_parts) + Carver::round(sizeof(float) * max_parts * ke) +
                 Carver::round(sizeof(int32_t) * max_parts * ke) + Carver::round(sizeof(unsigned) * B) +
                 Carver::round(qg_bytes) + (smp ? Carver::round(sizeof(float) * (size_t)B * G) : 0) + (flat ? Carver::round(sizeof(int32_t) * rows) + Carver::round(sizeof(int32_t) * kg) : 0) + 8192;
-  htam_status s = ensure_scratch(m, need);
+  s = ensure_scratch(m, need);
   if (s != HTAM_OK) return s;
   Carver cv(m->scratch);
   float *s1 = cv.take<float>((size_t)planes * B * G);
@@ -1568,18 +1580,30 @@ namespace {
 
 // ids[i] = gid[i] when given, else the nearest group picked for row i.  gid
 // and ids may be the same array (each thread reads and writes only its row).
-__global__ void assign_fill_kernel(const int32_t *gid, const int32_t *__restrict__ pick, int64_t n, int32_t *ids) {
-  const int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-  if (t < n) {
-    const int32_t g = gid[t];
-    ids[t] = g >= 0 ? g : pick[t];
+// Rows appended without a group (id -1): the group picked for each, counted
+// into the batch's group sizes; a row with no non-empty group to join marks
+// the batch bad.  Gated on the batch's count of such rows.
+__global__ void assign_resolve_kernel(const int32_t *__restrict__ gid, const int32_t *__restrict__ pick, int64_t n,
+                                      const int32_t *__restrict__ gate, int32_t *__restrict__ ids,
+                                      int32_t *__restrict__ bcount, int32_t *__restrict__ bad) {
+  if (*gate == 0) return;
+  for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < n; t += (int64_t)gridDim.x * blockDim.x) {
+    if (gid[t] != -1) continue;
+    const int32_t p = pick[t];
+    if (p < 0) {
+      atomicOr(bad, 1);
+    } else {
+      ids[t] = p;
+      atomicAdd(&bcount[p], 1);
+    }
   }
 }
 
 }  // namespace
 
-htam_status assign_nearest(htam_memory *m, const void *entries, const int32_t *gid, int64_t count, int32_t *dst,
-                           const int32_t **ids_out, cudaStream_t st, PhaseMark *mark) {
+htam_status assign_unassigned(htam_memory *m, const void *entries, const int32_t *gid, int64_t count,
+                              const int32_t *n_unassigned, int32_t *ids, int32_t *bcount, int32_t *bad,
+                              cudaStream_t st, PhaseMark *mark) {
   const int G = m->n_groups, d = m->d;
   // Rows per pass: the [rows, G] score matrix stays within 16 MiB per plane.
   const int64_t R = std::max<int64_t>(1, std::min<int64_t>(count, (int64_t(1) << 22) / G));
@@ -1588,8 +1612,8 @@ htam_status assign_nearest(htam_memory *m, const void *entries, const int32_t *g
     return m->dtype == HTAM_BF16 ? coarse_tc_splits((int)rb, d, G, m->sm_count) : 1;
   };
   const int64_t s1_elems = std::max<int64_t>(planes_of(R) * R, planes_of(last) * last) * G;
-  const size_t need = (dst ? 0 : Carver::round(sizeof(int32_t) * count)) + Carver::round(sizeof(float) * s1_elems) +
-                      Carver::round(sizeof(int32_t) * R) + Carver::round(sizeof(float) * R) + 1024;
+  const size_t need = Carver::round(sizeof(float) * s1_elems) + Carver::round(sizeof(int32_t) * R) +
+                      Carver::round(sizeof(float) * R) + 1024;
   if (need > m->assign_bytes) {
     if (m->assign_buf) cudaFree(m->assign_buf);  // synchronises: no queued work still reads it
     m->assign_buf = nullptr;
@@ -1602,7 +1626,6 @@ htam_status assign_nearest(htam_memory *m, const void *entries, const int32_t *g
     m->assign_bytes = want;
   }
   Carver cv(m->assign_buf);
-  int32_t *ids = dst ? dst : cv.take<int32_t>(count);
   float *s1 = cv.take<float>(s1_elems);
   int32_t *pick = cv.take<int32_t>(R);
   float *pick_score = cv.take<float>(R);
@@ -1612,27 +1635,27 @@ htam_status assign_nearest(htam_memory *m, const void *entries, const int32_t *g
     const int planes = planes_of(rb);
     if (m->dtype == HTAM_BF16) {
       htam_status s = launch_coarse_tc(rows, rb, d, m->cent_hi, m->cent_lo, m->count, G, planes, s1, m->status,
-                                       kMaxPolls, st);
+                                       kMaxPolls, st, n_unassigned);
       if (s != HTAM_OK) return s;
     } else {
       dim3 grid((unsigned)ceil_div(G, 64), (unsigned)ceil_div(rb, 64));
       coarse_scores_simt_kernel<float><<<grid, 256, 0, st>>>(static_cast<const float *>(rows), rb, d, m->cent,
-                                                             m->count, G, s1);
+                                                             m->count, G, s1, n_unassigned);
       HTAM_CK_LAUNCH("coarse_scores_simt_kernel");
     }
     if (warps_per_query(rb, m->sm_count) == 8) {
       group_topk_kernel<8><<<(unsigned)rb, kSelWarps * 32, 0, st>>>(s1, planes, rb, G, m->count, 1, pick,
-                                                                    pick_score);
+                                                                    pick_score, n_unassigned);
     } else {
       group_topk_kernel<1><<<(unsigned)ceil_div(rb, kSelWarps), kSelWarps * 32, 0, st>>>(
-          s1, planes, rb, G, m->count, 1, pick, pick_score);
+          s1, planes, rb, G, m->count, 1, pick, pick_score, n_unassigned);
     }
     HTAM_CK_LAUNCH("group_topk_kernel");
-    assign_fill_kernel<<<(unsigned)ceil_div(rb, 256), 256, 0, st>>>(gid + r0, pick, rb, ids + r0);
-    HTAM_CK_LAUNCH("assign_fill_kernel");
+    const unsigned blocks = (unsigned)std::min<int64_t>(ceil_div(rb, 256), 1024);
+    assign_resolve_kernel<<<blocks, 256, 0, st>>>(gid + r0, pick, rb, n_unassigned, ids + r0, bcount, bad);
+    HTAM_CK_LAUNCH("assign_resolve_kernel");
     if (mark) mark->launched(3);
   }
-  *ids_out = ids;
   return HTAM_OK;
 }
 

@@ -157,7 +157,10 @@ class Memory:
             raise RuntimeError("memory already freed")
         return self._h
 
-    def append(self, entries: torch.Tensor, group_ids: torch.Tensor, stream=None) -> None:
+    def append(self, entries: torch.Tensor, group_ids: torch.Tensor, stream=None, check: bool = False) -> None:
+        """Queues an append (no host round trip).  Group ids are checked on
+        the device: a rejected batch changes nothing and is reported by
+        device_status(); check=True waits for that report and raises it."""
         if entries.dtype != self.dtype or group_ids.dtype != torch.int32:
             raise TypeError("entries must match the memory dtype; group_ids int32")
         if entries.dim() != 2 or entries.shape[1] != self.d or group_ids.shape[0] != entries.shape[0]:
@@ -165,8 +168,11 @@ class Memory:
         _check(_lib.htam_append_transitions(self.handle, _dev_ptr(entries), _dev_ptr(group_ids),
                                             entries.shape[0], _stream_ptr(stream)),
                "htam_append_transitions")
+        if check:
+            _check(self.device_status(stream), "htam_append_transitions (device check)")
 
-    def append_assign(self, entries: torch.Tensor, group_ids: torch.Tensor, stream=None) -> torch.Tensor:
+    def append_assign(self, entries: torch.Tensor, group_ids: torch.Tensor, stream=None,
+                      check: bool = False) -> torch.Tensor:
         """append() that returns the group each entry joined (ids of -1 join
         the group with the nearest key)."""
         if entries.dtype != self.dtype or group_ids.dtype != torch.int32:
@@ -176,6 +182,8 @@ class Memory:
         assigned = torch.empty_like(group_ids)
         _check(_lib.htam_append_assign(self.handle, _dev_ptr(entries), _dev_ptr(group_ids), entries.shape[0],
                                        _dev_ptr(assigned), _stream_ptr(stream)), "htam_append_assign")
+        if check:
+            _check(self.device_status(stream), "htam_append_assign (device check)")
         return assigned
 
     def query(self, queries: torch.Tensor, k_groups: int, k_entries: int, tau: float = 1.0,

@@ -917,6 +917,39 @@ def test_memory_built_empty_then_filled_by_appends(htam, dtype):
     assert err.value.status == htam.HTAM_ECAPACITY and mem.info()["n"] == 2400
 
 
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+def test_appends_queued_back_to_back_grow_one_group(htam, dtype):
+    """Appends run on the device with no host round trip, so the host sizes
+    a query's scratch from group sizes that may lag behind the queued
+    appends.  Eight batches of 3,000 rows all go to group 0 (24,000 rows,
+    188 new pages), each followed at once by a lookup that selects it, with
+    nothing synchronised in between; every lookup is then checked against
+    the oracle over the memory as it stood at that point."""
+    d, g = 64, 10
+    entries, gid, centres = _rand_memory(2000, d, g, dtype, seed=40)
+    mem = htam.Memory(entries, gid, g, capacity=2000 + 8 * 3000)
+    gen = torch.Generator(device=DEV).manual_seed(41)
+    q = _rand_queries(48, d, dtype, seed=40, centres=centres)
+    all_e, all_g, outs = [entries], [gid], []
+    for r in range(8):
+        new_g = torch.zeros(3000, dtype=torch.int32, device=DEV)
+        x = centres[0] + 0.3 * torch.randn(3000, d, generator=gen, device=DEV)
+        new_e = _unit(x).to(dtype).contiguous()
+        mem.append(new_e, new_g)
+        all_e.append(new_e)
+        all_g.append(new_g)
+        outs.append(({k: v.clone() for k, v in mem.query(q, 3, 12, tau=0.5).items()}, len(all_e)))
+    torch.cuda.synchronize()
+    assert mem.device_status() == htam.HTAM_OK
+    dt = "bf16" if dtype == torch.bfloat16 else "f32"
+    for r, (out, upto) in enumerate(outs):
+        ents, gids = torch.cat(all_e[:upto]), torch.cat(all_g[:upto])
+        assert (out["group_idx"] == 0).any()  # the grown group is selected
+        problems = compare_lookup(out, to_numpy(ents), to_numpy(gids), g, to_numpy(q), 3, 12, 0.5, 0.0, dt)
+        assert not problems, f"lookup after append {r}:\n" + "\n".join(problems[:20])
+    assert mem.info()["n"] == 2000 + 8 * 3000
+
+
 def test_append_updates_group_keys_in_place(htam):
     import oracle
 
@@ -935,9 +968,13 @@ def test_append_errors_leave_memory_unchanged(htam):
     q = _rand_queries(8, 32, torch.bfloat16, seed=12, centres=centres)
     before = {k: v.clone() for k, v in mem.query(q, 3, 5).items()}
     bad_e, bad_g, _ = _rand_memory(50, 32, 10, torch.bfloat16, seed=13)
-    bad_g[17] = 10  # out of range
+    bad_g[17] = 10  # out of range: found on the device, reported by the status call
+    mem.append(bad_e, bad_g)
+    after_bad = {k: v.clone() for k, v in mem.query(q, 3, 5).items()}  # queued behind the rejected batch
+    assert mem.device_status() == htam.HTAM_EINVAL
+    assert mem.device_status() == htam.HTAM_OK  # read and cleared
     with pytest.raises(htam.HtamError) as err:
-        mem.append(bad_e, bad_g)
+        mem.append(bad_e, bad_g, check=True)
     assert err.value.status == htam.HTAM_EINVAL
     big_e, big_g, _ = _rand_memory(101, 32, 10, torch.bfloat16, seed=14)
     with pytest.raises(htam.HtamError) as err:
@@ -946,8 +983,13 @@ def test_append_errors_leave_memory_unchanged(htam):
     after = mem.query(q, 3, 5)
     torch.cuda.synchronize()
     assert mem.info()["n"] == 1000
+    assert (mem.group_counts().numpy() == np.bincount(to_numpy(gid), minlength=10)).all()
     for k in before:
-        assert torch.equal(before[k], after[k])
+        assert torch.equal(before[k], after[k]) and torch.equal(before[k], after_bad[k])
+    # The rejected batches left the id numbering alone: the next rows are 1000..
+    ok_e, ok_g, _ = _rand_memory(100, 32, 10, torch.bfloat16, seed=15)
+    mem.append(ok_e, ok_g, check=True)
+    _check(htam, mem, torch.cat([entries, ok_e]), torch.cat([gid, ok_g]), 10, q, 3, 5)
 
 
 NEAREST_CASES = [
@@ -1028,7 +1070,7 @@ def test_append_without_group_errors(htam):
                         capacity=100)
     e, _, _ = _rand_memory(10, 32, 5, torch.float32, seed=23)
     with pytest.raises(htam.HtamError) as err:
-        empty.append(e, torch.full((10,), -1, dtype=torch.int32, device=DEV))
+        empty.append(e, torch.full((10,), -1, dtype=torch.int32, device=DEV), check=True)
     assert err.value.status == htam.HTAM_EINVAL
     assert empty.info()["n"] == 0
     entries, gid, _ = _rand_memory(100, 32, 5, torch.float32, seed=24)
@@ -1036,9 +1078,10 @@ def test_append_without_group_errors(htam):
     bad = torch.full((10,), -1, dtype=torch.int32, device=DEV)
     bad[4] = -2
     with pytest.raises(htam.HtamError) as err:
-        mem.append(e, bad)
+        mem.append(e, bad, check=True)
     assert err.value.status == htam.HTAM_EINVAL
     assert mem.info()["n"] == 100
+    assert (mem.group_counts().numpy() == np.bincount(to_numpy(gid), minlength=5)).all()
 
 
 def test_stream_workload_all_rounds(htam):
