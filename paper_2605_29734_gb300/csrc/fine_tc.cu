@@ -113,9 +113,16 @@ __device__ __forceinline__ int take_unit(TcSmem *sh, int j, uint32_t empty_caddr
   return u;
 }
 
+// Per epilogue warp, a 32 x 32 fp32 staging area: a lane writes its row's
+// 32-column accumulator chunk there when some lane of the warp has pairs to
+// insert, and reads back the flagged columns one at a time by index.
+constexpr int kEpiWarps = 4;
+constexpr int kStageFloats = 32 * 32;
+
 template <bool PAIR>
 constexpr size_t smem_bytes() {
-  return 1024 /* alignment slack */ + Ring<PAIR>::kStages * (kABytes + Ring<PAIR>::kBStage) + sizeof(TcSmem);
+  return 1024 /* alignment slack */ + Ring<PAIR>::kStages * (kABytes + Ring<PAIR>::kBStage) +
+         sizeof(float) * kEpiWarps * kStageFloats + sizeof(TcSmem);
 }
 
 __device__ __forceinline__ unsigned enc_score(float f) {
@@ -199,7 +206,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t *smem = smem_raw + ((1024 - (smem_addr(smem_raw) & 1023)) & 1023);
   uint8_t *st_a = smem;
   uint8_t *st_b = st_a + kStages * kABytes;
-  TcSmem *sh = reinterpret_cast<TcSmem *>(st_b + kStages * kBStage);
+  float *st_epi = reinterpret_cast<float *>(st_b + kStages * kBStage);  // [kEpiWarps][32][32]
+  TcSmem *sh = reinterpret_cast<TcSmem *>(st_epi + kEpiWarps * kStageFloats);
   volatile int *abort = &sh->abort;
 
   // No units (every bucket went to the CUDA cores): leave before setting up
@@ -447,6 +455,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int e = quad * 32 + lane;           // this thread's row of the chunk
     const uint32_t lane_addr = tbase + (static_cast<uint32_t>(quad * 32) << 16);
     const int k = a.ke;
+    const int kj = (k + kThrSlots - 1) / kThrSlots;  // the rank each segment class publishes
+    // This lane's staging row (16-byte groups swizzled by the lane so that
+    // the warp's row writes spread over the banks).
+    float *stg = st_epi + (warp - 2) * kStageFloats + lane * 32;
     int acc = 0;
     uint32_t aph = 0;
     bool ok = true;
@@ -461,10 +473,26 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int nq = min(kTcRows, cg - c * kTcRows);  // <= 0: a pair's missing second chunk
       const bool valid = e < nq;
       const int b = valid ? a.bucket[a.bucket_off[g] + c * kTcRows + e] : 0;
+      unsigned *tb = a.thr_enc + (int64_t)b * kThrWords;
+      const int cls = 1 + sg % kThrSlots;
       float thr = valid ? -INFINITY : INFINITY;
-      // The query's shared bound, read one tile ahead: the load's latency
+      // The query's shared bounds, read one tile ahead: the loads' latency
       // is spent in the previous tile's work instead of stalling this one.
-      unsigned thr_pub = valid ? a.thr_enc[b] : 0u;
+      // (L2 loads: other CTAs raise the words with atomics.)
+      unsigned w0 = 0u, w1 = 0u, w2 = 0u, w3 = 0u, w4 = 0u;
+      auto load_bounds = [&]() {
+        w0 = __ldcg(tb);
+        w1 = __ldcg(tb + 1);
+        w2 = __ldcg(tb + 2);
+        w3 = __ldcg(tb + 3);
+        w4 = __ldcg(tb + 4);
+      };
+      auto shared_bound = [&]() {
+        const float slots = fminf(fminf(dec_score(w1), dec_score(w2)), fminf(dec_score(w3), dec_score(w4)));
+        return fmaxf(dec_score(w0), slots);
+      };
+      if (valid) load_bounds();
+      float pub_k = -INFINITY, pub_j = -INFINITY;  // what this unit has published
       float m2 = -INFINITY, l = 0.f;
       top.init();
       const int pg0 = a.page_off[g];
@@ -509,23 +537,22 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int o = 16; o > 0; o >>= 1) most = max(most, __shfl_xor_sync(kFull, most, o));
             // Insert the flagged pairs one at a time.  (A sorting network over
             // the chunk costs more here: its unrolled code is large and runs
-            // rarely, while this loop body is small.)
+            // rarely, while this loop body is small.)  The chunk goes through
+            // this lane's staging row, so a flagged column is one indexed
+            // load; each lane reads only what it wrote, so no barrier.
+            if (most > 0) {
+#pragma unroll
+              for (int i = 0; i < 8; ++i) {
+                *reinterpret_cast<uint4 *>(stg + ((i ^ (lane & 7)) << 2)) =
+                    make_uint4(r[4 * i], r[4 * i + 1], r[4 * i + 2], r[4 * i + 3]);
+              }
+            }
             for (int it = 0; it < most; ++it) {
               const bool any = flagged != 0u;
               const int j = any ? __ffs(flagged) - 1 : 0;
               flagged &= flagged - 1;
-              // r[j] through a 5-level select tree on the bits of j.
-              uint32_t t16[16], t8[8], t4[4], t2[2];
-#pragma unroll
-              for (int i = 0; i < 16; ++i) t16[i] = (j & 1) ? r[2 * i + 1] : r[2 * i];
-#pragma unroll
-              for (int i = 0; i < 8; ++i) t8[i] = (j & 2) ? t16[2 * i + 1] : t16[2 * i];
-#pragma unroll
-              for (int i = 0; i < 4; ++i) t4[i] = (j & 4) ? t8[2 * i + 1] : t8[2 * i];
-#pragma unroll
-              for (int i = 0; i < 2; ++i) t2[i] = (j & 8) ? t4[2 * i + 1] : t4[2 * i];
-              const uint32_t xv = (j & 16) ? t2[1] : t2[0];
-              if (any) top.insert_later(__uint_as_float(xv), cbase + j);
+              const float xv = stg[(((j >> 2) ^ (lane & 7)) << 2) | (j & 3)];
+              if (any) top.insert_later(xv, cbase + j);
             }
             if (valid && most > 0) thr = fmaxf(thr, top.kth(k));
           };
@@ -539,7 +566,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           __syncwarp();  // converged for the warp-collective loads and waits
           tmem_ld32(acc_addr, ra);
           tmem_wait_ld(ra);
-          if (valid) thr = fmaxf(thr, dec_score(thr_pub));  // bounds published by other units
+          if (valid) thr = fmaxf(thr, shared_bound());  // bounds published by other units
 #pragma unroll 1
           for (int ch = 0; ch < n_ch; ch += 2) {
             const bool has_b = ch + 1 < n_ch;  // uniform across the warp
@@ -568,10 +595,22 @@ __global__ void __launch_bounds__(kThreads, 1)
           acc = 0;
           aph ^= 1u;
         }
-        // Share this row's bound with the query's other units, and read
-        // theirs for the next tile.
-        if (valid && thr != -INFINITY && top.kth(k) == thr) atomicMax(&a.thr_enc[b], enc_score(thr));
-        if (valid) thr_pub = a.thr_enc[b];
+        // Share this row's bounds with the query's other units (its k-th
+        // score, and its kj-th score in its segment class), and read theirs
+        // for the next tile.
+        if (valid) {
+          const float kv = top.kth(k);
+          if (kv > pub_k) {
+            atomicMax(tb, enc_score(kv));
+            pub_k = kv;
+          }
+          const float jv = top.kth(kj);
+          if (jv > pub_j) {
+            atomicMax(tb + cls, enc_score(jv));
+            pub_j = jv;
+          }
+          load_bounds();
+        }
       }
       if (!ok) break;
       if (valid) {

@@ -12,6 +12,15 @@ namespace htam {
 constexpr int kTcRows = 128;      // queries per tensor-core work unit (MMA M)
 constexpr int kTcMaxK = 32;       // largest k_entries the tensor-core path keeps
 
+// Per-query shared score bounds of the tensor-core units: word 0 is the best
+// k-th score any unit's own list has reached; word 1 + s is the best
+// ceil(k / kThrSlots)-th score of the units whose page segment index is s
+// modulo kThrSlots.  Units of different classes hold disjoint entries, so
+// kThrSlots * ceil(k / kThrSlots) >= k candidates score at least the smallest
+// of those words: both are lower bounds of the query's final k-th best score.
+constexpr int kThrSlots = 4;
+constexpr int kThrWords = 1 + kThrSlots;
+
 struct TcFineArgs {
   const int4 *units;          // (group, bucket chunk, page segment)
   const int32_t *n_units;     // device count of units
@@ -31,7 +40,7 @@ struct TcFineArgs {
   float2 *part_ml;
   float *part_s;
   int32_t *part_id;
-  unsigned *thr_enc;          // [B] order-preserving encoding of a lower bound of the k-th best score
+  unsigned *thr_enc;          // [B][kThrWords] order-preserving encodings of the shared bounds above
   unsigned *status;           // memory status word
   uint32_t max_polls;
   int q_direct;               // 1: every bucket holds all queries in order and the query map is the

@@ -24,7 +24,7 @@ namespace htam {
 
 namespace {
 
-constexpr int kKeySegRowsMin = 64;     // rows per key partial-sum segment: at least this,
+constexpr int kKeySegRowsMin = 16;     // rows per key partial-sum segment: at least this,
 constexpr int kKeySegRowsMax = 1024;   // at most this,
 constexpr int64_t kKeySegTarget = 4096;  // and about count / this (bounds the partial-sum buffer)
 
@@ -347,17 +347,21 @@ __global__ void key_finalize_kernel(const KeyGroup *__restrict__ groups, const i
                                     __nv_bfloat16 *__restrict__ hi, __nv_bfloat16 *__restrict__ lo) {
   if ((int)blockIdx.x >= *n_groups) return;  // the grid covers every group
   KeyGroup kg = groups[blockIdx.x];
+  // One fp64 reciprocal per group instead of a division per column (fp64
+  // arithmetic is slow on this part); the mean is then rounded to fp32 and
+  // split in fp32: hi = bf16(mean), lo = bf16(mean - hi).
+  const double inv = kg.count > 0 ? 1.0 / (double)kg.count : 0.0;
   for (int j = blockIdx.y * blockDim.x + threadIdx.x; j < d; j += gridDim.y * blockDim.x) {
     double add = 0.0;
     for (int s = kg.seg0; s < kg.seg1; ++s) add += partial[(int64_t)s * d + j];
     int64_t o = (int64_t)kg.g * d + j;
     double sum = csum[o] + add;
     csum[o] = sum;
-    double mean = kg.count > 0 ? sum / (double)kg.count : 0.0;
-    cent[o] = (float)mean;
-    __nv_bfloat16 h = __double2bfloat16(mean);
+    const float mean = (float)(sum * inv);
+    cent[o] = mean;
+    const __nv_bfloat16 h = __float2bfloat16_rn(mean);
     hi[o] = h;
-    lo[o] = __double2bfloat16(mean - (double)__bfloat162float(h));
+    lo[o] = __float2bfloat16_rn(mean - __bfloat162float(h));
   }
 }
 
@@ -426,8 +430,10 @@ static htam_status add_rows(htam_memory *m, const void *entries, const int32_t *
   if (count == 0) return HTAM_OK;
   const int32_t G = m->n_groups, d = m->d;
 
-  // Chunking of the stable sort: at most ~16M (group, chunk) counters.
-  int64_t chunk = std::max<int64_t>(256, ceil_div((int64_t)count * G, int64_t(1) << 24));
+  // Chunking of the stable sort: at most ~16M (group, chunk) counters; one
+  // warp-wide step per chunk for batches of up to 64K rows (an append), so
+  // the placing warps do not walk long chunks one after another.
+  int64_t chunk = std::max<int64_t>(count <= 65536 ? 32 : 256, ceil_div((int64_t)count * G, int64_t(1) << 24));
   chunk = ceil_div(chunk, 32) * 32;
   int64_t n_chunks = ceil_div(count, chunk);
 
@@ -509,13 +515,15 @@ static htam_status add_rows(htam_memory *m, const void *entries, const int32_t *
 
   // 6. Keys of the touched groups.
   {
-    dim3 grid((unsigned)max_segs, (unsigned)ceil_div(d, 256 * 8));
+    // 8 columns per thread: 128 threads cover d = 1,024.
+    const int kp_threads = (int)std::min<int64_t>(256, ceil_div(ceil_div(d, 8), 32) * 32);
+    dim3 grid((unsigned)max_segs, (unsigned)ceil_div(d, kp_threads * 8));
     if (m->dtype == HTAM_BF16) {
-      key_partial_kernel<__nv_bfloat16><<<grid, 256, 0, st>>>(static_cast<const __nv_bfloat16 *>(m->pool), d,
+      key_partial_kernel<__nv_bfloat16><<<grid, kp_threads, 0, st>>>(static_cast<const __nv_bfloat16 *>(m->pool), d,
                                                               m->page_list_alt, m->page_off_alt, segs, meta,
                                                               partial);
     } else {
-      key_partial_kernel<float><<<grid, 256, 0, st>>>(static_cast<const float *>(m->pool), d, m->page_list_alt,
+      key_partial_kernel<float><<<grid, kp_threads, 0, st>>>(static_cast<const float *>(m->pool), d, m->page_list_alt,
                                                       m->page_off_alt, segs, meta, partial);
     }
     HTAM_CK_LAUNCH("key_partial_kernel");

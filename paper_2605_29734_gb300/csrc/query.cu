@@ -712,13 +712,13 @@ __global__ void bucket_fill_kernel(const uint32_t *__restrict__ bits, int G, int
                                    int4 *__restrict__ units,
                                    int4 *__restrict__ units_tc,
                                    int4 *__restrict__ units_tc2,
-                                   unsigned *__restrict__ thr_zero, int B,
+                                   unsigned *__restrict__ thr_zero, int thr_words,
                                    int32_t *__restrict__ ctr_zero) {
   // Also clears the tensor-core kernel's shared bounds and unit counters
   // (when given), which no earlier kernel of the query touches.
   if (thr_zero) {
     const int64_t t0 = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-    for (int64_t t = t0; t < B; t += (int64_t)gridDim.x * blockDim.x) thr_zero[t] = 0u;
+    for (int64_t t = t0; t < thr_words; t += (int64_t)gridDim.x * blockDim.x) thr_zero[t] = 0u;
     if (t0 < 2) ctr_zero[t0] = 0;
   }
   const int g = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
@@ -743,6 +743,7 @@ struct BucketSmallArgs {
   int32_t *n_units, *seg_tc_dev, *bucket, *bucket_group;
   int4 *units, *units_tc, *units_tc2;
   unsigned *thr_zero;
+  int thr_words;  // words of thr_zero
   int32_t *ctr_zero;
 };
 // One block pays off only for small problems: the 65k workload (256 groups x
@@ -758,7 +759,7 @@ __global__ void __launch_bounds__(1024) bucket_small_kernel(BucketSmallArgs a) {
   const int words = a.G * a.W;
   for (int i = tid; i < words; i += 1024) sbits[i] = 0u;
   if (a.thr_zero) {
-    for (int i = tid; i < a.B; i += 1024) a.thr_zero[i] = 0u;
+    for (int i = tid; i < a.thr_words; i += 1024) a.thr_zero[i] = 0u;
     if (tid < 2) a.ctr_zero[tid] = 0;
   }
   __syncthreads();
@@ -1343,7 +1344,7 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
                 (edge_table ? Carver::round(sizeof(float) * (size_t)G * G) : 0) +
                 3 * Carver::round(sizeof(int32_t) * rows) + 3 * Carver::round(sizeof(int4) * max_units) +
                 Carver::round(sizeof(float2) * max_parts) + Carver::round(sizeof(float) * max_parts * ke) +
-                Carver::round(sizeof(int32_t) * max_parts * ke) + Carver::round(sizeof(unsigned) * B) +
+                Carver::round(sizeof(int32_t) * max_parts * ke) + Carver::round(sizeof(unsigned) * (size_t)B * kThrWords) +
                 Carver::round(qg_bytes) + (smp ? Carver::round(sizeof(float) * (size_t)B * G) : 0) + (flat ? Carver::round(sizeof(int32_t) * rows) + Carver::round(sizeof(int32_t) * kg) : 0) + 8192;
   s = ensure_scratch(m, need);
   if (s != HTAM_OK) return s;
@@ -1371,7 +1372,7 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   float2 *part_ml = cv.take<float2>(max_parts);
   float *part_s = cv.take<float>(max_parts * ke);
   int32_t *part_id = cv.take<int32_t>(max_parts * ke);
-  unsigned *thr_enc = cv.take<unsigned>(B);
+  unsigned *thr_enc = cv.take<unsigned>((size_t)B * kThrWords);
   void *qg = tc_ok && !flat ? static_cast<void *>(cv.take<char>(qg_bytes)) : nullptr;
   float *policy_keys = smp ? cv.take<float>((size_t)B * G) : nullptr;
   if (flat) {
@@ -1473,7 +1474,7 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   if ((int64_t)G * W <= kBucketSmallWords && rows <= kBucketSmallRows) {
     BucketSmallArgs ba{group_idx, B, kg, G, W, m->page_off, rt, m->sm_count, cnt, wpre, pos, bucket_off, unit_off,
                        unit_off_tc, unit_off_tc2, part_off, n_units, seg_tc, bucket, bucket_group, units, units_tc,
-                       units_tc2, tc_ok ? thr_enc : nullptr, tc_ctr};
+                       units_tc2, tc_ok ? thr_enc : nullptr, B * kThrWords, tc_ctr};
     static std::atomic<uint64_t> attr_set{0};
     if (first_on_device(attr_set)) {
       HTAM_CK(cudaFuncSetAttribute(bucket_small_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -1495,7 +1496,7 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
     HTAM_CK_LAUNCH("bucket_scan_kernel");
     bucket_fill_kernel<<<(unsigned)ceil_div((int64_t)G * 32, 256), 256, 0, st>>>(
         bits, G, W, bucket_off, cnt, m->page_off, rt, seg_tc, unit_off, unit_off_tc, unit_off_tc2, bucket,
-        bucket_group, units, units_tc, units_tc2, tc_ok ? thr_enc : nullptr, B, tc_ctr);
+        bucket_group, units, units_tc, units_tc2, tc_ok ? thr_enc : nullptr, B * kThrWords, tc_ctr);
     HTAM_CK_LAUNCH("bucket_fill_kernel");
     mark.launched(5);
   }
