@@ -42,6 +42,7 @@
 #include <cudaTypedefs.h>
 
 #include <algorithm>
+#include <type_traits>
 
 #include "common.cuh"
 #include "fine_tc.h"
@@ -514,27 +515,49 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int cbase = (p - p_beg) * kPageRows + col0;  // unit column of r[0]
             uint32_t flagged = 0;
             if (valid) {
-              float cmax = -INFINITY;
+              // With one epilogue warp per scheduler the chunk's arithmetic
+              // is latency-bound, so it runs as short independent chains:
+              // the maximum by a tree of three-input maxima, the sum of
+              // exponentials in four interleaved partial sums, the flags
+              // only on a lane whose maximum reaches its bound, built in
+              // four partial masks.  A full chunk (every page row filled,
+              // uniform across the warp) skips the per-column fill test.
+              auto body = [&](auto full_tag) {
+                constexpr bool kFullChunk = decltype(full_tag)::value;
+                auto val = [&](int j) {
+                  return (kFullChunk || j < nv) ? __uint_as_float(r[j]) : -INFINITY;
+                };
+                float t[11];
 #pragma unroll
-              for (int j = 0; j < 32; ++j)
-                if (j < nv) cmax = fmaxf(cmax, __uint_as_float(r[j]));
-              const float mz = cmax * a.k2;
-              if (mz > m2) {
-                l *= ex2(m2 - mz);
-                m2 = mz;
-              }
-#pragma unroll
-              for (int j = 0; j < 32; ++j) {
-                if (j < nv) {
-                  const float s = __uint_as_float(r[j]);
-                  l += ex2(fmaf(s, a.k2, -m2));
-                  if (s >= thr) flagged |= 1u << j;
+                for (int i = 0; i < 10; ++i) t[i] = max3f(val(3 * i), val(3 * i + 1), val(3 * i + 2));
+                t[10] = fmaxf(val(30), val(31));
+                const float cmax = max3f(max3f(t[0], t[1], t[2]), max3f(t[3], t[4], t[5]),
+                                         max3f(max3f(t[6], t[7], t[8]), t[9], t[10]));
+                const float mz = cmax * a.k2;
+                if (mz > m2) {
+                  l *= ex2(m2 - mz);
+                  m2 = mz;
                 }
+                float l4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+                for (int j = 0; j < 32; ++j) l4[j & 3] += ex2(fmaf(val(j), a.k2, -m2));
+                l += (l4[0] + l4[1]) + (l4[2] + l4[3]);
+                if (cmax >= thr) {
+                  uint32_t f4[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+                  for (int j = 0; j < 32; ++j) {
+                    if ((kFullChunk || j < nv) && val(j) >= thr) f4[j & 3] |= 1u << j;
+                  }
+                  flagged = (f4[0] | f4[1]) | (f4[2] | f4[3]);
+                }
+              };
+              if (nv == 32) {
+                body(std::true_type{});
+              } else {
+                body(std::false_type{});
               }
             }
-            int most = __popc(flagged);
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1) most = max(most, __shfl_xor_sync(kFull, most, o));
+            const int most = (int)__reduce_max_sync(kFull, (unsigned)__popc(flagged));
             // Insert the flagged pairs one at a time.  (A sorting network over
             // the chunk costs more here: its unrolled code is large and runs
             // rarely, while this loop body is small.)  The chunk goes through
