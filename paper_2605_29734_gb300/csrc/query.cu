@@ -541,7 +541,7 @@ struct Route {
 // kTcSegPagesMax].  Long segments mean fewer cold top-k lists and fewer
 // partial records; short ones keep every SM busy when the tensor-core work
 // is small (units are taken dynamically, so a few long ones balance out).
-constexpr int kTcSegPagesMin = 16;
+constexpr int kTcSegPagesMin = 4;
 constexpr int kTcSegPagesMax = 256;
 __device__ __forceinline__ int tc_seg_pages(int64_t tiles, int sms) {
   int seg = kTcSegPagesMin;
