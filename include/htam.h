@@ -363,11 +363,17 @@ typedef enum {
  *    queries on pairs of SMs (two 128-query chunks per M=256 MMA,
  *    cta_group::2, each SM staging half of every entry tile); 0 (default)
  *    runs every chunk on one SM.
+ *  HTAM_TUNE_PDL: 1 (default) launches the kernels of a query or an append
+ *    with programmatic stream serialisation, so that each kernel's blocks
+ *    are scheduled while the previous kernel finishes (every such kernel
+ *    waits for its predecessor before touching memory); 0 launches them
+ *    plainly.  The results are the same either way.
  * Errors: EINVAL (m NULL, unknown key, value out of range). */
 typedef enum {
   HTAM_TUNE_TC_MIN_BUCKET = 0,
   HTAM_TUNE_STREAM_ROWS = 1,
-  HTAM_TUNE_TC_PAIRS = 2
+  HTAM_TUNE_TC_PAIRS = 2,
+  HTAM_TUNE_PDL = 3
 } htam_tuning;
 htam_status htam_set_tuning(htam_memory *m, htam_tuning key, int32_t value);
 

@@ -12,6 +12,7 @@
 namespace htam {
 
 static thread_local char g_last_error[256] = "";
+thread_local bool g_launch_pdl = false;
 
 void set_last_error(const char *what, cudaError_t err) {
   std::snprintf(g_last_error, sizeof g_last_error, "%s: %s", what, cudaGetErrorString(err));
@@ -165,6 +166,7 @@ htam_status htam_query_prefix(htam_memory *m, const void *prefix, int32_t b, int
     }
     m->prefix_bytes = want;
   }
+  PdlScope pdl(m->pdl != 0);
   PrefixWeights w;
   for (int i = 1; i <= p_len; ++i) w.alpha[i - 1] = (float)std::exp(-(double)lambda * (double)(p_len - i));
   PhaseMark mark(m, st);
@@ -364,6 +366,10 @@ htam_status htam_set_tuning(htam_memory *m, htam_tuning key, int32_t value) {
       if (value != 0 && value != 1) return HTAM_EINVAL;
       m->tc_pairs = value;
       return HTAM_OK;
+    case HTAM_TUNE_PDL:
+      if (value != 0 && value != 1) return HTAM_EINVAL;
+      m->pdl = value;
+      return HTAM_OK;
   }
   return HTAM_EINVAL;
 }
@@ -379,6 +385,9 @@ htam_status htam_get_tuning(const htam_memory *m, htam_tuning key, int32_t *valu
       return HTAM_OK;
     case HTAM_TUNE_TC_PAIRS:
       *value = m->tc_pairs;
+      return HTAM_OK;
+    case HTAM_TUNE_PDL:
+      *value = m->pdl;
       return HTAM_OK;
   }
   return HTAM_EINVAL;

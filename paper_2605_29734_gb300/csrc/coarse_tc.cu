@@ -52,6 +52,7 @@ __global__ void __launch_bounds__(kCThreads, kCPerSM)
                      const __grid_constant__ CUtensorMap lo_map, int d, int kb_per, const int32_t *__restrict__ count,
                      int B, int G, float *__restrict__ s1, unsigned *status, uint32_t max_polls,
                      const int32_t *__restrict__ gate) {
+  pdl_entry();  // after the previous kernel of the stream (see common.cuh)
   // Gated launch (rows appended without a group): nothing to score.  The
   // exit is uniform over the grid and comes before any barrier or tensor
   // memory is set up.
@@ -214,7 +215,7 @@ htam_status launch_coarse_tc(const void *queries, int B, int d, const __nv_bfloa
   const int kb_per = (int)ceil_div((int64_t)nk, splits);
   if (splits < 1 || (int)ceil_div((int64_t)nk, kb_per) != splits) return HTAM_EINVAL;  // no empty split
   dim3 grid((unsigned)ceil_div(B, kCM), (unsigned)ceil_div(G, kCN), (unsigned)splits);
-  coarse_tc_kernel<<<grid, kCThreads, kCSmem, st>>>(q_map, hi_map, lo_map, d, kb_per, count, B, G, s1, status,
+  launch_kernel(coarse_tc_kernel, grid, kCThreads, kCSmem, st, q_map, hi_map, lo_map, d, kb_per, count, B, G, s1, status,
                                                      max_polls, gate);
   HTAM_CK_LAUNCH("coarse_tc_kernel");
   return HTAM_OK;

@@ -169,6 +169,61 @@ __device__ __forceinline__ float warp_sum(float v) {
 
 __host__ __device__ inline int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
 
+// ------------------------------------------------ programmatic dependent launch
+// The kernels of a query (and of an append) run back to back on one stream.
+// Launched with programmatic stream serialisation, a kernel's blocks may be
+// scheduled while the previous kernel is still finishing; every kernel of
+// those paths therefore starts with griddepcontrol.wait (returns once the
+// previous kernel has completed and its writes are visible; a no-op when the
+// launch had no programmatic dependency) before it touches device memory,
+// and then lets its own dependents start launching.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void pdl_entry() {
+  pdl_wait();
+  pdl_trigger();
+}
+
+// Whether the launches made by this host thread use programmatic stream
+// serialisation (set for the duration of a query or append from the memory
+// object's tuning).
+extern thread_local bool g_launch_pdl;
+struct PdlScope {
+  bool prev;
+  explicit PdlScope(bool on) : prev(g_launch_pdl) { g_launch_pdl = on; }
+  ~PdlScope() { g_launch_pdl = prev; }
+};
+
+template <typename... P, typename... A>
+inline cudaError_t launch_kernel(void (*kernel)(P...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                                 A &&...args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  if (g_launch_pdl) {
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+  }
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<A &&>(args)...);
+}
+
+// Launches `kernel` (parenthesise template kernels) and returns HTAM_ECUDA
+// from the enclosing function if the launch fails.
+#define HTAM_LAUNCH(what, kernel, grid, block, smem, st, ...)                                   \
+  do {                                                                                        \
+    cudaError_t err__ = ::htam::launch_kernel(kernel, dim3(grid), dim3(block), (size_t)(smem), \
+                                              st, __VA_ARGS__);                               \
+    if (err__ != cudaSuccess) {                                                               \
+      ::htam::set_last_error(what, err__);                                                    \
+      return HTAM_ECUDA;                                                                      \
+    }                                                                                         \
+  } while (0)
+
 // True the first time it is called for the current device with this flag
 // word (one bit per device): per-device, once-only setup such as a kernel's
 // shared-memory limit, safe to call from several host threads.

@@ -125,6 +125,7 @@ __device__ __forceinline__ UnitRows unit_rows(const StreamArgs &a, int u, int wa
 
 template <int QC, int KV>
 __global__ void __launch_bounds__(kWarps * 32, 1) fine_ring_kernel(StreamArgs a) {
+  pdl_entry();  // after the previous kernel of the stream (see common.cuh)
   // Slice t of a lane is row slice lane + 32 t, and query register qr[j][t]
   // holds the same slice of query j.
   constexpr int S = ring_slots<QC, KV>();
@@ -356,7 +357,7 @@ htam_status launch_qk(const StreamArgs &a, int sm_count, cudaStream_t st) {
   const size_t smem = (size_t)kWarps * ring_slots<QC, KV>() * 32 * KV * 16 + side_bytes(QC);
   auto kernel = fine_ring_kernel<QC, KV>;
   HTAM_CK(cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
-  kernel<<<sm_count, kWarps * 32, smem, st>>>(a);
+  launch_kernel(kernel, sm_count, kWarps * 32, smem, st, a);
   HTAM_CK_LAUNCH("fine_ring_kernel");
   return HTAM_OK;
 }

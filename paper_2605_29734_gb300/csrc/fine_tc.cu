@@ -201,6 +201,7 @@ template <int K, bool PAIR>
 __global__ void __launch_bounds__(kThreads, 1)
     fine_tc_kernel(const __grid_constant__ CUtensorMap q_map, const __grid_constant__ CUtensorMap pool_map,
                    TcFineArgs a) {
+  pdl_entry();  // after the previous kernel of the stream (see common.cuh)
   constexpr int kStages = Ring<PAIR>::kStages;
   constexpr int kBStage = Ring<PAIR>::kBStage;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
@@ -687,6 +688,7 @@ __global__ void gather_queries_kernel(const uint4 *__restrict__ Q, int vec_per_r
                                       const int32_t *__restrict__ bucket_group, const int32_t *__restrict__ cnt,
                                       int tc_min, const int32_t *__restrict__ total_rows, int64_t max_rows,
                                       uint4 *__restrict__ Qg) {
+  pdl_entry();  // after the previous kernel of the stream (see common.cuh)
   const int64_t r = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (r >= max_rows || r >= *total_rows) return;
@@ -726,16 +728,18 @@ htam_status launch_k(const TcFineArgs &a, const CUtensorMap &q_map, const CUtens
     cfg.blockDim = dim3(kThreads, 1, 1);
     cfg.dynamicSmemBytes = smem_bytes<PAIR>();
     cfg.stream = st;
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = 2;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = g_launch_pdl ? 2 : 1;
     HTAM_CK(cudaLaunchKernelEx(&cfg, fine_tc_kernel<K, true>, q_map, pool_map, a));
   } else {
-    fine_tc_kernel<K, false><<<grid, kThreads, smem_bytes<false>(), st>>>(q_map, pool_map, a);
+    launch_kernel(fine_tc_kernel<K, false>, grid, kThreads, smem_bytes<false>(), st, q_map, pool_map, a);
   }
   HTAM_CK_LAUNCH("fine_tc_kernel");
   return HTAM_OK;
@@ -761,7 +765,7 @@ htam_status launch_gather_queries(const void *Q, int d, const int32_t *bucket, c
                                   void *Qg, cudaStream_t st) {
   if (max_rows <= 0) return HTAM_OK;
   const int vec = d * 2 / 16;
-  gather_queries_kernel<<<(unsigned)ceil_div(max_rows * 32, 256), 256, 0, st>>>(
+  launch_kernel(gather_queries_kernel, (unsigned)ceil_div(max_rows * 32, 256), 256, 0, st, 
       static_cast<const uint4 *>(Q), vec, bucket, bucket_group, cnt, tc_min, total_rows, max_rows,
       static_cast<uint4 *>(Qg));
   HTAM_CK_LAUNCH("gather_queries_kernel");

@@ -98,6 +98,9 @@ struct htam_memory {
   // single SMs (0).  Off by default: the epilogue, not the operand feed,
   // limits the kernel, and the pair path measured slower.
   int tc_pairs = 0;
+  // Kernels of a query or append launched with programmatic stream
+  // serialisation (1, default) or as plain launches (0).
+  int pdl = 1;
   CUtensorMap pool_map;
   bool pool_map_ready = false;
 };

@@ -45,6 +45,7 @@ __global__ void count_groups_kernel(const int32_t *__restrict__ gid, int64_t n, 
                                     int allow_unassigned, int32_t *__restrict__ counts, int32_t *__restrict__ bad,
                                     int32_t *__restrict__ unassigned, int32_t *__restrict__ hist,
                                     int64_t hist_len) {
+  pdl_entry();  // after the previous kernel of the stream (see common.cuh)
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < n; e += stride) {
     int32_t g = gid[e];
@@ -121,6 +122,7 @@ __global__ void __launch_bounds__(kLayoutThreads, 1)
                   int32_t *__restrict__ first_new, int32_t *__restrict__ base, KeySeg *__restrict__ segs,
                   KeyGroup *__restrict__ kgroups, int32_t *__restrict__ meta, int64_t *__restrict__ id_base,
                   int64_t *__restrict__ dev_ctr, unsigned *__restrict__ status) {
+  pdl_entry();  // after the previous kernel of the stream (see common.cuh)
   __shared__ int64_t sh[32];
   if (*bad) {
     for (int g = threadIdx.x; g <= G; g += blockDim.x) page_off_new[g] = page_off_cur[g];
@@ -178,6 +180,7 @@ __global__ void __launch_bounds__(kLayoutThreads, 1)
 __global__ void page_copy_kernel(int32_t G, const int32_t *__restrict__ page_off_cur,
                                  const int32_t *__restrict__ page_list_cur, const int32_t *__restrict__ page_off_new,
                                  const int32_t *__restrict__ first_new, int32_t *__restrict__ page_list_new) {
+  pdl_entry();  // after the previous kernel of the stream (see common.cuh)
   const int g = (int)((blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5);
   const int lane = threadIdx.x & 31;
   if (g >= G) return;
@@ -192,6 +195,7 @@ __global__ void page_copy_kernel(int32_t G, const int32_t *__restrict__ page_off
 __global__ void chunk_hist_kernel(const int32_t *__restrict__ gid, const int32_t *__restrict__ ids, int64_t n,
                                   int64_t chunk, int64_t n_chunks, int32_t *__restrict__ hist,
                                   const int32_t *__restrict__ bad) {
+  pdl_entry();  // after the previous kernel of the stream (see common.cuh)
   if (*bad) return;
   int64_t c = blockIdx.x;
   int64_t lo = c * chunk, hi = min(n, lo + chunk);
@@ -203,6 +207,7 @@ __global__ void chunk_hist_kernel(const int32_t *__restrict__ gid, const int32_t
 // Per group (one warp each): hist[g][c] <- base[g] + sum_{c' < c} hist[g][c'].
 __global__ void chunk_scan_kernel(int32_t *__restrict__ hist, int64_t n_chunks, int32_t n_groups,
                                   const int32_t *__restrict__ base, const int32_t *__restrict__ bad) {
+  pdl_entry();  // after the previous kernel of the stream (see common.cuh)
   if (*bad) return;
   int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   int lane = threadIdx.x & 31;
@@ -228,6 +233,7 @@ __global__ void chunk_scan_kernel(int32_t *__restrict__ hist, int64_t n_chunks, 
 __global__ void chunk_place_kernel(const int32_t *__restrict__ gid, const int32_t *__restrict__ ids, int64_t n,
                                    int64_t chunk, int64_t n_chunks, int32_t *__restrict__ hist,
                                    int32_t *__restrict__ pos, const int32_t *__restrict__ bad) {
+  pdl_entry();  // after the previous kernel of the stream (see common.cuh)
   if (*bad) return;
   int64_t c = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
   int lane = threadIdx.x & 31;
@@ -263,6 +269,7 @@ __global__ void place_rows_kernel(const uint4 *__restrict__ src, const int32_t *
                                   uint4 *__restrict__ pool, int32_t *__restrict__ slot_id,
                                   const int64_t *__restrict__ id_base, int32_t *assigned,
                                   const int32_t *__restrict__ bad) {
+  pdl_entry();  // after the previous kernel of the stream (see common.cuh)
   if (*bad) return;
   int64_t e = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
   int lane = threadIdx.x & 31;
@@ -294,6 +301,7 @@ __global__ void key_partial_kernel(const T *__restrict__ pool, int32_t d,
                                    const int32_t *__restrict__ page_off,
                                    const KeySeg *__restrict__ segs, const int32_t *__restrict__ n_segs,
                                    double *__restrict__ partial) {
+  pdl_entry();  // after the previous kernel of the stream (see common.cuh)
   constexpr int kBatch = 8;
   if ((int)blockIdx.x >= *n_segs) return;  // the grid covers the host's bound on the segments
   const KeySeg sg = segs[blockIdx.x];
@@ -345,6 +353,7 @@ __global__ void key_finalize_kernel(const KeyGroup *__restrict__ groups, const i
                                     const double *__restrict__ partial, int32_t d,
                                     double *__restrict__ csum, float *__restrict__ cent,
                                     __nv_bfloat16 *__restrict__ hi, __nv_bfloat16 *__restrict__ lo) {
+  pdl_entry();  // after the previous kernel of the stream (see common.cuh)
   if ((int)blockIdx.x >= *n_groups) return;  // the grid covers every group
   KeyGroup kg = groups[blockIdx.x];
   // One fp64 reciprocal per group instead of a division per column (fp64
@@ -428,6 +437,7 @@ htam_status refresh_mirror(htam_memory *m, bool wait) {
 static htam_status add_rows(htam_memory *m, const void *entries, const int32_t *gid, int64_t count,
                             int32_t *assigned, cudaStream_t st, bool build, int32_t **bad_out = nullptr) {
   if (count == 0) return HTAM_OK;
+  PdlScope pdl(m->pdl != 0);
   const int32_t G = m->n_groups, d = m->d;
 
   // Chunking of the stable sort: at most ~16M (group, chunk) counters; one
@@ -471,7 +481,7 @@ static htam_status add_rows(htam_memory *m, const void *entries, const int32_t *
   HTAM_CK(cudaMemsetAsync(bcount, 0, sizeof(int32_t) * (G + 2), st));
   {
     const int blocks = (int)std::min<int64_t>(ceil_div(std::max<int64_t>(count, (int64_t)G * n_chunks), 256), 4096);
-    count_groups_kernel<<<blocks, 256, 0, st>>>(gid, count, G, build ? 0 : 1, bcount, bad, bcount + G + 1, hist,
+    launch_kernel(count_groups_kernel, blocks, 256, 0, st, gid, count, G, build ? 0 : 1, bcount, bad, bcount + G + 1, hist,
                                                 (int64_t)G * n_chunks);
     HTAM_CK_LAUNCH("count_groups_kernel");
     mark.launched();
@@ -484,11 +494,11 @@ static htam_status add_rows(htam_memory *m, const void *entries, const int32_t *
     if (s != HTAM_OK) return s;
   }
   // 3. Page layout, key segments and new sizes; then the page lists.
-  layout_kernel<<<1, kLayoutThreads, 0, st>>>(G, count, seg_rows, bcount, bad, m->count, m->page_off,
+  launch_kernel(layout_kernel, 1, kLayoutThreads, 0, st, G, count, seg_rows, bcount, bad, m->count, m->page_off,
                                               m->page_off_alt, first_new, base, segs, kgroups, meta, id_base,
                                               m->dev_ctr, m->status);
   HTAM_CK_LAUNCH("layout_kernel");
-  page_copy_kernel<<<(unsigned)ceil_div((int64_t)G * 32, 256), 256, 0, st>>>(G, m->page_off, m->page_list,
+  launch_kernel(page_copy_kernel, (unsigned)ceil_div((int64_t)G * 32, 256), 256, 0, st, G, m->page_off, m->page_list,
                                                                              m->page_off_alt, first_new,
                                                                              m->page_list_alt);
   HTAM_CK_LAUNCH("page_copy_kernel");
@@ -496,18 +506,18 @@ static htam_status add_rows(htam_memory *m, const void *entries, const int32_t *
 
   // 4. Stable slot assignment: pos[e] = old size of its group + rank among
   //    earlier rows of the batch with the same group.
-  chunk_hist_kernel<<<(unsigned)n_chunks, 256, 0, st>>>(gid, ids, count, chunk, n_chunks, hist, bad);
+  launch_kernel(chunk_hist_kernel, (unsigned)n_chunks, 256, 0, st, gid, ids, count, chunk, n_chunks, hist, bad);
   HTAM_CK_LAUNCH("chunk_hist_kernel");
-  chunk_scan_kernel<<<(unsigned)ceil_div((int64_t)G * 32, 256), 256, 0, st>>>(hist, n_chunks, G, base, bad);
+  launch_kernel(chunk_scan_kernel, (unsigned)ceil_div((int64_t)G * 32, 256), 256, 0, st, hist, n_chunks, G, base, bad);
   HTAM_CK_LAUNCH("chunk_scan_kernel");
-  chunk_place_kernel<<<(unsigned)ceil_div(n_chunks * 32, 256), 256, 0, st>>>(gid, ids, count, chunk, n_chunks, hist,
+  launch_kernel(chunk_place_kernel, (unsigned)ceil_div(n_chunks * 32, 256), 256, 0, st, gid, ids, count, chunk, n_chunks, hist,
                                                                              pos, bad);
   HTAM_CK_LAUNCH("chunk_place_kernel");
   mark.launched(3);
 
   // 5. Copy rows into their slots.
   int vec_per_row = d * m->elem_bytes / 16;
-  place_rows_kernel<<<(unsigned)ceil_div(count * 32, 256), 256, 0, st>>>(
+  launch_kernel(place_rows_kernel, (unsigned)ceil_div(count * 32, 256), 256, 0, st, 
       static_cast<const uint4 *>(entries), gid, ids, pos, count, vec_per_row, m->page_list_alt, m->page_off_alt,
       static_cast<uint4 *>(m->pool), m->slot_id, id_base, assigned, bad);
   HTAM_CK_LAUNCH("place_rows_kernel");
@@ -519,16 +529,16 @@ static htam_status add_rows(htam_memory *m, const void *entries, const int32_t *
     const int kp_threads = (int)std::min<int64_t>(256, ceil_div(ceil_div(d, 8), 32) * 32);
     dim3 grid((unsigned)max_segs, (unsigned)ceil_div(d, kp_threads * 8));
     if (m->dtype == HTAM_BF16) {
-      key_partial_kernel<__nv_bfloat16><<<grid, kp_threads, 0, st>>>(static_cast<const __nv_bfloat16 *>(m->pool), d,
+      launch_kernel(key_partial_kernel<__nv_bfloat16>, grid, kp_threads, 0, st, static_cast<const __nv_bfloat16 *>(m->pool), d,
                                                               m->page_list_alt, m->page_off_alt, segs, meta,
                                                               partial);
     } else {
-      key_partial_kernel<float><<<grid, kp_threads, 0, st>>>(static_cast<const float *>(m->pool), d, m->page_list_alt,
+      launch_kernel(key_partial_kernel<float>, grid, kp_threads, 0, st, static_cast<const float *>(m->pool), d, m->page_list_alt,
                                                       m->page_off_alt, segs, meta, partial);
     }
     HTAM_CK_LAUNCH("key_partial_kernel");
     dim3 g2((unsigned)G, (unsigned)std::min<int64_t>(ceil_div(d, 256), 16));
-    key_finalize_kernel<<<g2, 256, 0, st>>>(kgroups, meta + 1, partial, d, m->csum, m->cent, m->cent_hi,
+    launch_kernel(key_finalize_kernel, g2, 256, 0, st, kgroups, meta + 1, partial, d, m->csum, m->cent, m->cent_hi,
                                             m->cent_lo);
     HTAM_CK_LAUNCH("key_finalize_kernel");
     mark.launched(2);

@@ -20,6 +20,7 @@ namespace {
 template <typename T>
 __global__ void __launch_bounds__(256) prefix_reduce_kernel(const T *__restrict__ prefix, int32_t b, int32_t p_len,
                                                             int32_t d, PrefixWeights w, T *__restrict__ out) {
+  pdl_entry();  // after the previous kernel of the stream (see common.cuh)
   const int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   const int per_row = d / 8;
   if (t >= (int64_t)b * per_row) return;
@@ -67,10 +68,10 @@ htam_status launch_prefix_reduce(const htam_memory *m, const void *prefix, int32
   const int64_t threads = (int64_t)b * (m->d / 8);
   const unsigned blocks = (unsigned)ceil_div(threads, 256);
   if (m->dtype == HTAM_BF16) {
-    prefix_reduce_kernel<__nv_bfloat16><<<blocks, 256, 0, st>>>(static_cast<const __nv_bfloat16 *>(prefix), b,
+    launch_kernel(prefix_reduce_kernel<__nv_bfloat16>, blocks, 256, 0, st, static_cast<const __nv_bfloat16 *>(prefix), b,
                                                                  p_len, m->d, w, static_cast<__nv_bfloat16 *>(out));
   } else {
-    prefix_reduce_kernel<float><<<blocks, 256, 0, st>>>(static_cast<const float *>(prefix), b, p_len, m->d, w,
+    launch_kernel(prefix_reduce_kernel<float>, blocks, 256, 0, st, static_cast<const float *>(prefix), b, p_len, m->d, w,
                                                         static_cast<float *>(out));
   }
   HTAM_CK_LAUNCH("prefix_reduce_kernel");

@@ -35,6 +35,7 @@ template <typename T>
 __global__ void __launch_bounds__(256) coarse_scores_simt_kernel(
     const T *__restrict__ Q, int B, int d, const float *__restrict__ cent,
     const int32_t *__restrict__ count, int G, float *__restrict__ s1, const int32_t *__restrict__ gate = nullptr) {
+  pdl_entry();  // after the previous kernel of the stream (see common.cuh)
   if (gate && *gate == 0) return;  // gated launch with nothing to score
   __shared__ float qs[32][68];
   __shared__ float cs[32][68];
@@ -115,6 +116,7 @@ __global__ void __launch_bounds__(NW * 32, 1) group_topk_kernel(const float *__r
                                                              int32_t *__restrict__ gidx,
                                                              float *__restrict__ gscore,
                                                              const int32_t *__restrict__ gate = nullptr) {
+  pdl_entry();  // after the previous kernel of the stream (see common.cuh)
   if (gate && *gate == 0) return;  // gated launch with nothing to select
   __shared__ float ls[NW][64];
   __shared__ int li[NW][64];
@@ -262,6 +264,7 @@ __device__ __forceinline__ float edge_phi(const EdgeKernelArgs &a, const float *
 // of every edge is formed once (U[from][to] = phi) and the scores gather
 // from U: the same products and sums in the same order, so the same results.
 __global__ void __launch_bounds__(256) edge_phi_kernel(EdgeKernelArgs a, int G, float *__restrict__ U) {
+  pdl_entry();  // after the previous kernel of the stream (see common.cuh)
   const int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   if (t >= (int64_t)G * G) return;
   U[t] = edge_phi(a, a.Z + t * a.F);
@@ -269,6 +272,7 @@ __global__ void __launch_bounds__(256) edge_phi_kernel(EdgeKernelArgs a, int G, 
 
 __global__ void __launch_bounds__(256) edge_gather_kernel(EdgeKernelArgs a, const float *__restrict__ U, int B, int G,
                                                           float *__restrict__ s1) {
+  pdl_entry();  // after the previous kernel of the stream (see common.cuh)
   const int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   if (t >= (int64_t)B * G) return;
   const int64_t b = t / G;
@@ -282,6 +286,7 @@ __global__ void __launch_bounds__(256) edge_gather_kernel(EdgeKernelArgs a, cons
 }
 
 __global__ void __launch_bounds__(256) edge_scores_kernel(EdgeKernelArgs a, int B, int G, float *__restrict__ s1) {
+  pdl_entry();  // after the previous kernel of the stream (see common.cuh)
   const int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   if (t >= (int64_t)B * G) return;
   const int64_t b = t / G;
@@ -347,6 +352,7 @@ __device__ __forceinline__ float block_reduce(float v, bool is_max, float *red) 
 // times 2^-23).  The k largest keys are k draws without replacement from
 // mu (Kool, van Hoof and Welling, ICML 2019).  Empty groups get -inf.
 __global__ void __launch_bounds__(256) policy_keys_kernel(PolicyArgs a) {
+  pdl_entry();  // after the previous kernel of the stream (see common.cuh)
   __shared__ float red[32];
   const int b = blockIdx.x;
   const int64_t plane = (int64_t)a.B * a.G;
@@ -399,6 +405,7 @@ __global__ void __launch_bounds__(256) policy_keys_kernel(PolicyArgs a) {
 // (planes summed in order, as the selection sums them), -inf for padding.
 __global__ void policy_scores_kernel(const float *__restrict__ s1, int planes, int B, int G, int kg,
                                      const int32_t *__restrict__ group_idx, float *__restrict__ group_score) {
+  pdl_entry();  // after the previous kernel of the stream (see common.cuh)
   const int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   if (t >= (int64_t)B * kg) return;
   const int g = group_idx[t];
@@ -417,6 +424,7 @@ __global__ void policy_scores_kernel(const float *__restrict__ s1, int planes, i
 // The ascending list of non-empty groups (one block, 1024 groups per pass).
 __global__ void __launch_bounds__(1024) flat_groups_kernel(const int32_t *__restrict__ count, int G,
                                                            int32_t *__restrict__ list) {
+  pdl_entry();  // after the previous kernel of the stream (see common.cuh)
   __shared__ int warp_n[32];
   __shared__ int base;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -444,6 +452,7 @@ __global__ void __launch_bounds__(1024) flat_groups_kernel(const int32_t *__rest
 // Every query selects every non-empty group: group_idx[b][j] = list[j].
 __global__ void flat_fill_kernel(const int32_t *__restrict__ list, int64_t rows, int kg,
                                  int32_t *__restrict__ group_idx) {
+  pdl_entry();  // after the previous kernel of the stream (see common.cuh)
   const int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   if (t < rows) group_idx[t] = list[t % kg];
 }
@@ -461,6 +470,7 @@ __device__ __forceinline__ void bucket_bits_row(int64_t t, const int32_t *__rest
 
 __global__ void bucket_bits_kernel(const int32_t *__restrict__ gidx, int B, int kg, int W,
                                    uint32_t *__restrict__ bits) {
+  pdl_entry();  // after the previous kernel of the stream (see common.cuh)
   const int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   if (t < (int64_t)B * kg) bucket_bits_row(t, gidx, kg, W, bits);
 }
@@ -487,6 +497,7 @@ __device__ __forceinline__ void bucket_count_group(int g, int lane, const uint32
 
 __global__ void bucket_count_kernel(const uint32_t *__restrict__ bits, int G, int W,
                                     int32_t *__restrict__ cnt, int32_t *__restrict__ wpre) {
+  pdl_entry();  // after the previous kernel of the stream (see common.cuh)
   const int g = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   if (g < G) bucket_count_group(g, threadIdx.x & 31, bits, W, cnt, wpre);
 }
@@ -506,6 +517,7 @@ __device__ __forceinline__ void bucket_pos_row(int64_t t, const uint32_t *bits, 
 __global__ void bucket_pos_kernel(const uint32_t *__restrict__ bits, const int32_t *__restrict__ wpre, int W,
                                   const int32_t *__restrict__ gidx, int64_t rows, int kg,
                                   int32_t *__restrict__ pos) {
+  pdl_entry();  // after the previous kernel of the stream (see common.cuh)
   const int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   if (t < rows) bucket_pos_row(t, bits, wpre, W, gidx, kg, pos);
 }
@@ -652,6 +664,7 @@ __global__ void __launch_bounds__(1024) bucket_scan_kernel(
     int32_t *__restrict__ bucket_off, int32_t *__restrict__ unit_off, int32_t *__restrict__ unit_off_tc,
     int32_t *__restrict__ unit_off_tc2, int64_t *__restrict__ part_off, int32_t *__restrict__ n_units,
     int32_t *__restrict__ seg_tc_dev) {
+  pdl_entry();  // after the previous kernel of the stream (see common.cuh)
   bucket_scan_block(cnt, page_off, G, rt, sms, bucket_off, unit_off, unit_off_tc, unit_off_tc2, part_off, n_units,
                     seg_tc_dev);
 }
@@ -714,6 +727,7 @@ __global__ void bucket_fill_kernel(const uint32_t *__restrict__ bits, int G, int
                                    int4 *__restrict__ units_tc2,
                                    unsigned *__restrict__ thr_zero, int thr_words,
                                    int32_t *__restrict__ ctr_zero) {
+  pdl_entry();  // after the previous kernel of the stream (see common.cuh)
   // Also clears the tensor-core kernel's shared bounds and unit counters
   // (when given), which no earlier kernel of the query touches.
   if (thr_zero) {
@@ -753,6 +767,7 @@ constexpr int kBucketSmallWords = 4096;  // bitmap words held in shared memory (
 constexpr int64_t kBucketSmallRows = 4096;
 
 __global__ void __launch_bounds__(1024) bucket_small_kernel(BucketSmallArgs a) {
+  pdl_entry();  // after the previous kernel of the stream (see common.cuh)
   extern __shared__ uint32_t sbits[];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int64_t rows = (int64_t)a.B * a.kg;
@@ -834,6 +849,7 @@ struct Unpack<float> {
 // and one partial record per (query, unit) is written.
 template <typename T, int QC, int B>
 __global__ void __launch_bounds__(kFineWarps * 32, 2) fine_simt_kernel(FineArgs a) {
+  pdl_entry();  // after the previous kernel of the stream (see common.cuh)
   extern __shared__ __align__(16) unsigned char smem_raw[];
   constexpr int kN = Unpack<T>::kN;
   const int d = a.d;
@@ -1036,6 +1052,7 @@ constexpr int kMergeWarps = 8;
 
 template <int WPQ>
 __global__ void __launch_bounds__(kMergeWarps * 32, 1) merge_kernel(MergeArgs a) {
+  pdl_entry();  // after the previous kernel of the stream (see common.cuh)
   __shared__ float ls[kMergeWarps][64];
   __shared__ int li[kMergeWarps][64];
   __shared__ float wM[kMergeWarps], wL[kMergeWarps];
@@ -1239,7 +1256,7 @@ htam_status launch_fine_simt(const FineArgs &fa, int sm_count, int64_t max_units
   per_sm = std::max(per_sm, 1);
   int64_t grid = std::min<int64_t>(max_units, (int64_t)sm_count * per_sm);
   if (grid <= 0) return HTAM_OK;
-  kernel<<<(unsigned)grid, kFineWarps * 32, smem, st>>>(fa);
+  launch_kernel(kernel, (unsigned)grid, kFineWarps * 32, smem, st, fa);
   HTAM_CK_LAUNCH("fine_simt_kernel");
   return HTAM_OK;
 }
@@ -1290,6 +1307,7 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
                        float *entry_score, float *entry_weight, float *lse, cudaStream_t st,
                        const EdgeRoute *er, bool flat, const SampleSpec *smp) {
   if (B == 0) return HTAM_OK;
+  PdlScope pdl(m->pdl != 0);
   // The host mirror of the group sizes bounds the scratch below; the flat
   // scan and the policy draws need the exact non-empty groups, so they wait
   // for the mirror of the last append (the others take the newest one that
@@ -1382,9 +1400,9 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
     if (n_nonempty == 0) {
       HTAM_CK(cudaMemsetAsync(group_idx, 0xff, sizeof(int32_t) * (size_t)rows, st));
     } else {
-      flat_groups_kernel<<<1, 1024, 0, st>>>(m->count, G, list);
+      launch_kernel(flat_groups_kernel, 1, 1024, 0, st, m->count, G, list);
       HTAM_CK_LAUNCH("flat_groups_kernel");
-      flat_fill_kernel<<<(unsigned)ceil_div(rows, 256), 256, 0, st>>>(list, rows, kg, group_idx);
+      launch_kernel(flat_fill_kernel, (unsigned)ceil_div(rows, 256), 256, 0, st, list, rows, kg, group_idx);
       HTAM_CK_LAUNCH("flat_fill_kernel");
       mark.launched(2);
     }
@@ -1406,13 +1424,13 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
       for (int f = 0; f < HTAM_MAX_EDGE_FEATURES; ++f) ea.w[f] = er->w[f];
       for (int i = 0; i < HTAM_MAX_PREFIX; ++i) ea.alpha[i] = er->alpha[i];
       if (edge_table) {
-        edge_phi_kernel<<<(unsigned)ceil_div((int64_t)G * G, 256), 256, 0, st>>>(ea, G, edge_u);
+        launch_kernel(edge_phi_kernel, (unsigned)ceil_div((int64_t)G * G, 256), 256, 0, st, ea, G, edge_u);
         HTAM_CK_LAUNCH("edge_phi_kernel");
-        edge_gather_kernel<<<(unsigned)ceil_div((int64_t)B * G, 256), 256, 0, st>>>(ea, edge_u, B, G, s1);
+        launch_kernel(edge_gather_kernel, (unsigned)ceil_div((int64_t)B * G, 256), 256, 0, st, ea, edge_u, B, G, s1);
         HTAM_CK_LAUNCH("edge_gather_kernel");
         mark.launched();
       } else {
-        edge_scores_kernel<<<(unsigned)ceil_div((int64_t)B * G, 256), 256, 0, st>>>(ea, B, G, s1);
+        launch_kernel(edge_scores_kernel, (unsigned)ceil_div((int64_t)B * G, 256), 256, 0, st, ea, B, G, s1);
         HTAM_CK_LAUNCH("edge_scores_kernel");
       }
     } else if (m->dtype == HTAM_BF16) {
@@ -1423,8 +1441,8 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
     } else {
       // fp32 memories: CUDA cores against the fp32 keys.
       dim3 grid((unsigned)ceil_div(G, 64), (unsigned)ceil_div(B, 64));
-      coarse_scores_simt_kernel<float><<<grid, 256, 0, st>>>(static_cast<const float *>(queries), B, d,
-                                                             m->cent, m->count, G, s1);
+      launch_kernel(coarse_scores_simt_kernel<float>, grid, 256, 0, st, static_cast<const float *>(queries), B, d,
+                                                             m->cent, m->count, G, s1, nullptr);
       HTAM_CK_LAUNCH("coarse_scores_simt_kernel");
     }
     mark.launched();
@@ -1438,7 +1456,7 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
         PolicyArgs pa{s1, planes, B, G, m->count, n_nonempty, 1.0f / p.tau, p.epsilon,
                       make_uint2((uint32_t)smp->seed, (uint32_t)(smp->seed >> 32)), (uint32_t)smp->offset,
                       (uint32_t)(smp->offset >> 32), policy_keys};
-        policy_keys_kernel<<<(unsigned)B, 256, 0, st>>>(pa);
+        launch_kernel(policy_keys_kernel, (unsigned)B, 256, 0, st, pa);
         HTAM_CK_LAUNCH("policy_keys_kernel");
         mark.launched();
       } else {
@@ -1449,19 +1467,19 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
     }
     const int swpq = select_warps_per_query(B, m->sm_count);
     if (swpq == 32) {
-      group_topk_kernel<32><<<(unsigned)B, 32 * 32, 0, st>>>(sel, sel_planes, B, G, m->count, kg, group_idx,
-                                                            group_score);
+      launch_kernel(group_topk_kernel<32>, (unsigned)B, 32 * 32, 0, st, sel, sel_planes, B, G, m->count, kg, group_idx,
+                                                            group_score, nullptr);
     } else if (swpq == 8) {
-      group_topk_kernel<8><<<(unsigned)B, kSelWarps * 32, 0, st>>>(sel, sel_planes, B, G, m->count, kg, group_idx,
-                                                                   group_score);
+      launch_kernel(group_topk_kernel<8>, (unsigned)B, kSelWarps * 32, 0, st, sel, sel_planes, B, G, m->count, kg, group_idx,
+                                                                   group_score, nullptr);
     } else {
-      group_topk_kernel<1><<<(unsigned)ceil_div(B, kSelWarps), kSelWarps * 32, 0, st>>>(
-          sel, sel_planes, B, G, m->count, kg, group_idx, group_score);
+      launch_kernel(group_topk_kernel<1>, (unsigned)ceil_div(B, kSelWarps), kSelWarps * 32, 0, st,
+          sel, sel_planes, B, G, m->count, kg, group_idx, group_score, nullptr);
     }
     HTAM_CK_LAUNCH("group_topk_kernel");
     mark.launched();
     if (smp) {
-      policy_scores_kernel<<<(unsigned)ceil_div((int64_t)B * kg, 256), 256, 0, st>>>(s1, planes, B, G, kg,
+      launch_kernel(policy_scores_kernel, (unsigned)ceil_div((int64_t)B * kg, 256), 256, 0, st, s1, planes, B, G, kg,
                                                                                    group_idx, group_score);
       HTAM_CK_LAUNCH("policy_scores_kernel");
       mark.launched();
@@ -1480,21 +1498,21 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
       HTAM_CK(cudaFuncSetAttribute(bucket_small_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                    (int)(sizeof(uint32_t) * kBucketSmallWords)));
     }
-    bucket_small_kernel<<<1, 1024, sizeof(uint32_t) * (size_t)G * W, st>>>(ba);
+    launch_kernel(bucket_small_kernel, 1, 1024, sizeof(uint32_t) * (size_t)G * W, st, ba);
     HTAM_CK_LAUNCH("bucket_small_kernel");
     mark.launched();
   } else {
     HTAM_CK(cudaMemsetAsync(bits, 0, sizeof(uint32_t) * (size_t)G * W, st));
-    bucket_bits_kernel<<<(unsigned)ceil_div(rows, 256), 256, 0, st>>>(group_idx, B, kg, W, bits);
+    launch_kernel(bucket_bits_kernel, (unsigned)ceil_div(rows, 256), 256, 0, st, group_idx, B, kg, W, bits);
     HTAM_CK_LAUNCH("bucket_bits_kernel");
-    bucket_count_kernel<<<(unsigned)ceil_div((int64_t)G * 32, 256), 256, 0, st>>>(bits, G, W, cnt, wpre);
+    launch_kernel(bucket_count_kernel, (unsigned)ceil_div((int64_t)G * 32, 256), 256, 0, st, bits, G, W, cnt, wpre);
     HTAM_CK_LAUNCH("bucket_count_kernel");
-    bucket_pos_kernel<<<(unsigned)ceil_div(rows, 256), 256, 0, st>>>(bits, wpre, W, group_idx, rows, kg, pos);
+    launch_kernel(bucket_pos_kernel, (unsigned)ceil_div(rows, 256), 256, 0, st, bits, wpre, W, group_idx, rows, kg, pos);
     HTAM_CK_LAUNCH("bucket_pos_kernel");
-    bucket_scan_kernel<<<1, 1024, 0, st>>>(cnt, m->page_off, G, rt, m->sm_count, bucket_off, unit_off,
+    launch_kernel(bucket_scan_kernel, 1, 1024, 0, st, cnt, m->page_off, G, rt, m->sm_count, bucket_off, unit_off,
                                            unit_off_tc, unit_off_tc2, part_off, n_units, seg_tc);
     HTAM_CK_LAUNCH("bucket_scan_kernel");
-    bucket_fill_kernel<<<(unsigned)ceil_div((int64_t)G * 32, 256), 256, 0, st>>>(
+    launch_kernel(bucket_fill_kernel, (unsigned)ceil_div((int64_t)G * 32, 256), 256, 0, st,
         bits, G, W, bucket_off, cnt, m->page_off, rt, seg_tc, unit_off, unit_off_tc, unit_off_tc2, bucket,
         bucket_group, units, units_tc, units_tc2, tc_ok ? thr_enc : nullptr, B * kThrWords, tc_ctr);
     HTAM_CK_LAUNCH("bucket_fill_kernel");
@@ -1565,9 +1583,9 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   MergeArgs ma{group_idx, B, kg, ke, m->count, pos, cnt, m->page_off, rt, seg_tc, part_off, part_ml, part_s,
                part_id, 1.0f / p.tau, p.epsilon, entry_idx, entry_score, entry_weight, lse};
   if (wpq == 8) {
-    merge_kernel<8><<<(unsigned)B, kMergeWarps * 32, 0, st>>>(ma);
+    launch_kernel(merge_kernel<8>, (unsigned)B, kMergeWarps * 32, 0, st, ma);
   } else {
-    merge_kernel<1><<<(unsigned)ceil_div(B, kMergeWarps), kMergeWarps * 32, 0, st>>>(ma);
+    launch_kernel(merge_kernel<1>, (unsigned)ceil_div(B, kMergeWarps), kMergeWarps * 32, 0, st, ma);
   }
   HTAM_CK_LAUNCH("merge_kernel");
   mark.launched();
@@ -1587,6 +1605,7 @@ namespace {
 __global__ void assign_resolve_kernel(const int32_t *__restrict__ gid, const int32_t *__restrict__ pick, int64_t n,
                                       const int32_t *__restrict__ gate, int32_t *__restrict__ ids,
                                       int32_t *__restrict__ bcount, int32_t *__restrict__ bad) {
+  pdl_entry();  // after the previous kernel of the stream (see common.cuh)
   if (*gate == 0) return;
   for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < n; t += (int64_t)gridDim.x * blockDim.x) {
     if (gid[t] != -1) continue;
@@ -1640,20 +1659,20 @@ htam_status assign_unassigned(htam_memory *m, const void *entries, const int32_t
       if (s != HTAM_OK) return s;
     } else {
       dim3 grid((unsigned)ceil_div(G, 64), (unsigned)ceil_div(rb, 64));
-      coarse_scores_simt_kernel<float><<<grid, 256, 0, st>>>(static_cast<const float *>(rows), rb, d, m->cent,
+      launch_kernel(coarse_scores_simt_kernel<float>, grid, 256, 0, st, static_cast<const float *>(rows), rb, d, m->cent,
                                                              m->count, G, s1, n_unassigned);
       HTAM_CK_LAUNCH("coarse_scores_simt_kernel");
     }
     if (warps_per_query(rb, m->sm_count) == 8) {
-      group_topk_kernel<8><<<(unsigned)rb, kSelWarps * 32, 0, st>>>(s1, planes, rb, G, m->count, 1, pick,
+      launch_kernel(group_topk_kernel<8>, (unsigned)rb, kSelWarps * 32, 0, st, s1, planes, rb, G, m->count, 1, pick,
                                                                     pick_score, n_unassigned);
     } else {
-      group_topk_kernel<1><<<(unsigned)ceil_div(rb, kSelWarps), kSelWarps * 32, 0, st>>>(
+      launch_kernel(group_topk_kernel<1>, (unsigned)ceil_div(rb, kSelWarps), kSelWarps * 32, 0, st,
           s1, planes, rb, G, m->count, 1, pick, pick_score, n_unassigned);
     }
     HTAM_CK_LAUNCH("group_topk_kernel");
     const unsigned blocks = (unsigned)std::min<int64_t>(ceil_div(rb, 256), 1024);
-    assign_resolve_kernel<<<blocks, 256, 0, st>>>(gid + r0, pick, rb, n_unassigned, ids + r0, bcount, bad);
+    launch_kernel(assign_resolve_kernel, blocks, 256, 0, st, gid + r0, pick, rb, n_unassigned, ids + r0, bcount, bad);
     HTAM_CK_LAUNCH("assign_resolve_kernel");
     if (mark) mark->launched(3);
   }

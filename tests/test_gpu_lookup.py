@@ -1146,6 +1146,28 @@ def test_repeated_queries_are_bitwise_deterministic(htam):
         assert torch.equal(a[k], b[k]) and torch.equal(a[k], c[k]), k
 
 
+def test_programmatic_launch_on_and_off_agree_bitwise(htam):
+    """Kernels launched with programmatic stream serialisation (the default)
+    and plainly give bit-identical lookups and appends: every kernel waits
+    for its predecessor before touching memory either way."""
+    entries, gid, centres = _rand_memory(30000, 256, 64, torch.bfloat16, seed=26)
+    q = _rand_queries(300, 256, torch.bfloat16, seed=26, centres=centres)
+    extra, extra_g, _ = _rand_memory(2000, 256, 64, torch.bfloat16, seed=27)
+    outs = []
+    for pdl in (1, 0):
+        mem = htam.Memory(entries, gid, 64, capacity=32000)
+        mem.set_programmatic_launch(pdl)
+        a = {k: v.clone() for k, v in mem.query(q, 8, 16).items()}
+        mem.append(extra, extra_g)
+        b = {k: v.clone() for k, v in mem.query(q, 8, 16).items()}
+        outs.append((a, b, mem.group_keys()))
+        assert mem.device_status() == htam.HTAM_OK
+    for x, y in zip(outs[0][:2], outs[1][:2]):
+        for k in x:
+            assert torch.equal(x[k], y[k]), k
+    assert torch.equal(outs[0][2], outs[1][2])
+
+
 def test_bad_query_arguments(htam):
     entries, gid, _ = _rand_memory(100, 16, 4, torch.float32, seed=17)
     mem = htam.Memory(entries, gid, 4)
