@@ -77,6 +77,8 @@ def parse_args():
     ap.add_argument("--pdl", type=int, default=None, choices=[0, 1],
                     help="programmatic dependent launch of the query's kernels (1, library default) or plain "
                          "launches (0)")
+    ap.add_argument("--fine-overlap", type=int, default=None, choices=[0, 1],
+                    help="CUDA-core and tensor-core fine kernels concurrently (1, library default) or in turn (0)")
     ap.add_argument("--tc-min-bucket", type=int, default=None,
                     help="smallest bucket scored on the tensor cores (library default 2)")
     ap.add_argument("--no-secondary", action="store_true",
@@ -372,6 +374,8 @@ def measure(args, world, rank, local, full=True):
         mem.set_tensor_core_pairs(args.tc_pairs)
     if args.pdl is not None:
         mem.set_programmatic_launch(args.pdl)
+    if args.fine_overlap is not None:
+        mem.set_fine_overlap(args.fine_overlap)
     tc_min = mem.get_tuning(htam.HTAM_TUNE_TC_MIN_BUCKET)
     if args.no_cpu_baseline:
         del entries                  # the memory holds its own copy
@@ -475,9 +479,13 @@ def measure(args, world, rank, local, full=True):
     launches = sum(v[1] for k, v in mem.read_phase_timing().items() if k != "queries")
     step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
     # Per-phase device times from a second pass of the same steps with CUDA
-    # events recorded around every phase on the launching stream.  The events
-    # separate the kernels (no programmatic overlap across them), so this
-    # pass is not the timed region; it gives the dominant kernel's duration.
+    # events recorded around every phase on the launching stream, and the two
+    # fine kernels run one after the other, so that each kernel's duration is
+    # its own (in the timed region they share the SMs).  The events separate
+    # the kernels, so this pass is not the timed region; it gives the
+    # dominant kernel's duration.
+    overlap = mem.get_tuning(htam.HTAM_TUNE_FINE_OVERLAP)
+    mem.set_fine_overlap(False)
     mem.set_phase_timing(True)
     for i in range(args.steps):
         if flush is not None:
@@ -485,6 +493,7 @@ def measure(args, world, rank, local, full=True):
         one_step(args.warmup + args.steps + i)
     torch.cuda.synchronize()
     mem.set_phase_timing(False)
+    mem.set_fine_overlap(bool(overlap))
     phases = mem.read_phase_timing()
     value, total_s = whole_job_rate(sum(step_ms) / 1e3, w.b * args.steps, world)
 

@@ -368,12 +368,19 @@ typedef enum {
  *    are scheduled while the previous kernel finishes (every such kernel
  *    waits for its predecessor before touching memory); 0 launches them
  *    plainly.  The results are the same either way.
+ *  HTAM_TUNE_FINE_OVERLAP: 1 (default) runs the CUDA-core and tensor-core
+ *    fine kernels of a query concurrently: the CUDA-core kernel goes to an
+ *    internal stream of the memory object, forked from `cuda_stream` and
+ *    joined back to it by events inside the call (so the call still orders
+ *    as one unit of work on `cuda_stream`, and stream capture records the
+ *    fork and join); 0 runs them one after the other on `cuda_stream`.
  * Errors: EINVAL (m NULL, unknown key, value out of range). */
 typedef enum {
   HTAM_TUNE_TC_MIN_BUCKET = 0,
   HTAM_TUNE_STREAM_ROWS = 1,
   HTAM_TUNE_TC_PAIRS = 2,
-  HTAM_TUNE_PDL = 3
+  HTAM_TUNE_PDL = 3,
+  HTAM_TUNE_FINE_OVERLAP = 4
 } htam_tuning;
 htam_status htam_set_tuning(htam_memory *m, htam_tuning key, int32_t value);
 

@@ -370,6 +370,10 @@ htam_status htam_set_tuning(htam_memory *m, htam_tuning key, int32_t value) {
       if (value != 0 && value != 1) return HTAM_EINVAL;
       m->pdl = value;
       return HTAM_OK;
+    case HTAM_TUNE_FINE_OVERLAP:
+      if (value != 0 && value != 1) return HTAM_EINVAL;
+      m->fine_overlap = value;
+      return HTAM_OK;
   }
   return HTAM_EINVAL;
 }
@@ -388,6 +392,9 @@ htam_status htam_get_tuning(const htam_memory *m, htam_tuning key, int32_t *valu
       return HTAM_OK;
     case HTAM_TUNE_PDL:
       *value = m->pdl;
+      return HTAM_OK;
+    case HTAM_TUNE_FINE_OVERLAP:
+      *value = m->fine_overlap;
       return HTAM_OK;
   }
   return HTAM_EINVAL;

@@ -101,6 +101,12 @@ struct htam_memory {
   // Kernels of a query or append launched with programmatic stream
   // serialisation (1, default) or as plain launches (0).
   int pdl = 1;
+  // The CUDA-core and tensor-core fine kernels of a query run concurrently
+  // (1: the CUDA-core kernel on an internal stream forked from and joined
+  // back to the caller's by events) or one after the other (0).
+  int fine_overlap = 1;
+  cudaStream_t side = nullptr;   // created on first use
+  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
   CUtensorMap pool_map;
   bool pool_map_ready = false;
 };

@@ -580,6 +580,9 @@ void free_impl(htam_memory *m) {
   for (cudaEvent_t e : m->mirror_ev) {
     if (e) cudaEventDestroy(e);
   }
+  if (m->ev_fork) cudaEventDestroy(m->ev_fork);
+  if (m->ev_join) cudaEventDestroy(m->ev_join);
+  if (m->side) cudaStreamDestroy(m->side);
   cudaFree(m->count);
   cudaFree(m->csum);
   cudaFree(m->cent);

@@ -760,11 +760,12 @@ struct BucketSmallArgs {
   int thr_words;  // words of thr_zero
   int32_t *ctr_zero;
 };
-// One block pays off only for small problems: the 65k workload (256 groups x
-// 8 words, 2,048 rows) gains 3 us, the 8-query one 13 us, while 512 groups x
-// 32 words (8,192 rows) already run faster as five kernels.
+// One block pays off only for small problems: with programmatic dependent
+// launch the five kernels already win on the 65k workload (256 groups x 8
+// words, 2,048 rows: 20 us against 28 us), while the 8-query one (32 rows)
+// still saves launches in one block.
 constexpr int kBucketSmallWords = 4096;  // bitmap words held in shared memory (16 KiB)
-constexpr int64_t kBucketSmallRows = 4096;
+constexpr int64_t kBucketSmallRows = 1024;
 
 __global__ void __launch_bounds__(1024) bucket_small_kernel(BucketSmallArgs a) {
   pdl_entry();  // after the previous kernel of the stream (see common.cuh)
@@ -1537,24 +1538,45 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   }
   mark.end();
 
-  // 3a. Fine scores of small buckets on the CUDA cores.
-  mark.begin(HTAM_PHASE_FINE);
+  // 3a. Fine scores of small buckets on the CUDA cores.  When both fine
+  // kernels run, the CUDA-core one goes to the memory's internal stream,
+  // forked from the caller's stream here and joined back before the merge,
+  // so that it shares the SMs with the tensor-core kernel instead of running
+  // before it (the two write disjoint partial records).
+  const bool overlap = tc_ok && m->fine_overlap;
+  cudaStream_t fst = st;
+  if (overlap) {
+    if (!m->side) {
+      if (cudaStreamCreateWithFlags(&m->side, cudaStreamNonBlocking) != cudaSuccess ||
+          cudaEventCreateWithFlags(&m->ev_fork, cudaEventDisableTiming) != cudaSuccess ||
+          cudaEventCreateWithFlags(&m->ev_join, cudaEventDisableTiming) != cudaSuccess) {
+        set_last_error("creating the internal stream", cudaGetLastError());
+        return HTAM_ECUDA;
+      }
+    }
+    HTAM_CK(cudaEventRecord(m->ev_fork, st));
+    HTAM_CK(cudaStreamWaitEvent(m->side, m->ev_fork, 0));
+    fst = m->side;
+  }
+  PhaseMark fmark(m, fst);
+  fmark.begin(HTAM_PHASE_FINE);
   {
     // Rows prefetched into per-warp shared-memory rings; rows or query
     // blocks too large for the rings take direct 16-byte loads.
     StreamArgs sa{m->pool, d, m->slot_id, m->page_list, m->page_off, m->count, queries, bucket, bucket_off,
                   cnt, units, n_units, part_off, ke, 1.0f / p.tau, kSimtSegPages, part_ml, part_s, part_id};
-    s = m->stream_rows ? launch_fine_stream(sa, qc, m->dtype, m->sm_count, st) : HTAM_EINVAL;
+    s = m->stream_rows ? launch_fine_stream(sa, qc, m->dtype, m->sm_count, fst) : HTAM_EINVAL;
     if (s == HTAM_EINVAL) {
       FineArgs fa{m->pool, d, m->slot_id, m->page_list, m->page_off, m->count, queries, bucket, bucket_off,
                   cnt, units, n_units, part_off, ke, 1.0f / p.tau, kSimtSegPages, part_ml, part_s, part_id};
-      s = m->dtype == HTAM_BF16 ? dispatch_fine_simt<__nv_bfloat16>(qc, fa, m->sm_count, max_units, st)
-                                : dispatch_fine_simt<float>(qc, fa, m->sm_count, max_units, st);
+      s = m->dtype == HTAM_BF16 ? dispatch_fine_simt<__nv_bfloat16>(qc, fa, m->sm_count, max_units, fst)
+                                : dispatch_fine_simt<float>(qc, fa, m->sm_count, max_units, fst);
     }
   }
   if (s != HTAM_OK) return s;
-  mark.launched();
-  mark.end();
+  fmark.launched();
+  fmark.end();
+  if (overlap) HTAM_CK(cudaEventRecord(m->ev_join, fst));
 
   // 3b. Fine scores of large buckets on the tensor cores.
   if (tc_ok) {
@@ -1577,6 +1599,8 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
     mark.launched();
     mark.end();
   }
+
+  if (overlap) HTAM_CK(cudaStreamWaitEvent(st, m->ev_join, 0));
 
   // 4. Merge per query.
   mark.begin(HTAM_PHASE_MERGE);

@@ -18,6 +18,7 @@ LIB_PATH = os.path.join(_PKG, "_lib", "libhtam.so")
 HTAM_OK, HTAM_EINVAL, HTAM_ENOMEM, HTAM_ECAPACITY, HTAM_ECUDA, HTAM_ETIMEOUT, HTAM_ENODEV = range(7)
 HTAM_F32, HTAM_BF16 = 0, 1
 HTAM_TUNE_TC_MIN_BUCKET, HTAM_TUNE_STREAM_ROWS, HTAM_TUNE_TC_PAIRS, HTAM_TUNE_PDL = 0, 1, 2, 3
+HTAM_TUNE_FINE_OVERLAP = 4
 HTAM_MAX_PREFIX = 64  # longest prefix htam_query_prefix takes
 HTAM_MAX_EDGE_FEATURES = 32  # most features per edge htam_query_edges takes
 
@@ -378,6 +379,11 @@ class Memory:
         """Tensor-core buckets of more than 128 queries on SM pairs (True) or
         single SMs (False)."""
         self.set_tuning(HTAM_TUNE_TC_PAIRS, int(bool(enable)))
+
+    def set_fine_overlap(self, enable: bool) -> None:
+        """CUDA-core and tensor-core fine kernels concurrently (True, default)
+        or one after the other (False)."""
+        self.set_tuning(HTAM_TUNE_FINE_OVERLAP, int(bool(enable)))
 
     def set_programmatic_launch(self, enable: bool) -> None:
         """Kernels of a query or append launched with programmatic stream
