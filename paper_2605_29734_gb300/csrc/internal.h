@@ -168,13 +168,15 @@ void free_impl(htam_memory *m);
 // as they stand before the append).  Queued without a host round trip: every
 // kernel is gated on *n_unassigned (the batch's tally of such rows, on the
 // device) and does nothing when it is zero.  For each such row e: ids[e] =
-// the chosen group and bcount[that group] += 1; a row that finds no
+// the chosen group, bcount[that group] += 1 and hist[that group * n_chunks
+// + e / chunk] += 1 (the stable sort's counts); a row that finds no
 // non-empty group sets *bad.  Scratch: m->assign_buf, grown with cudaMalloc
 // on demand (a growth synchronises the device).
 struct PhaseMark;
 htam_status assign_unassigned(htam_memory *m, const void *entries, const int32_t *gid, int64_t count,
                               const int32_t *n_unassigned, int32_t *ids, int32_t *bcount, int32_t *bad,
-                              cudaStream_t st, PhaseMark *mark = nullptr);
+                              int32_t *hist, int64_t chunk, int64_t n_chunks, cudaStream_t st,
+                              PhaseMark *mark = nullptr);
 
 // Weights alpha_1..alpha_P of a prefix (Eq. 10), passed by value to the
 // reduction kernel.

@@ -37,14 +37,15 @@ static int key_seg_rows(int64_t count) {
   return r;
 }
 
-// Per-group counts of a batch.  Ids of -1 (no group given) are counted
-// apart when `allow_unassigned`, and count as bad otherwise; any other id
-// outside [0, n_groups) sets `bad`.  The same grid also clears the stable
-// sort's (group, chunk) counters.
+// Per-group counts of a batch, and the stable sort's per (group, chunk of
+// `chunk` rows) counts hist[g * n_chunks + c] (both zeroed before).  Ids of
+// -1 (no group given) are counted apart when `allow_unassigned` (the
+// nearest-key assignment adds them later), and count as bad otherwise; any
+// other id outside [0, n_groups) sets `bad`.
 __global__ void count_groups_kernel(const int32_t *__restrict__ gid, int64_t n, int32_t n_groups,
                                     int allow_unassigned, int32_t *__restrict__ counts, int32_t *__restrict__ bad,
-                                    int32_t *__restrict__ unassigned, int32_t *__restrict__ hist,
-                                    int64_t hist_len) {
+                                    int32_t *__restrict__ unassigned, int32_t *__restrict__ hist, int64_t chunk,
+                                    int64_t n_chunks) {
   pdl_entry();  // after the previous kernel of the stream (see common.cuh)
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < n; e += stride) {
@@ -55,9 +56,9 @@ __global__ void count_groups_kernel(const int32_t *__restrict__ gid, int64_t n, 
       atomicOr(bad, 1);
     } else {
       atomicAdd(&counts[g], 1);
+      atomicAdd(&hist[(int64_t)g * n_chunks + e / chunk], 1);
     }
   }
-  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < hist_len; i += stride) hist[i] = 0;
 }
 
 // The group of row e: its given id, or for a row given -1 the group the
@@ -115,21 +116,35 @@ __device__ __forceinline__ int64_t block_scan_incl(int64_t v, int64_t *sh /* [32
 //     before the batch, and the entry count grows by `rows`.
 // A bad batch changes nothing: the current offsets are copied to the new
 // layout, no segment is listed, and status bit 1 records the rejection.
+// For small batches and layouts the same block then does what
+// chunk_scan_kernel (fuse_scan) and page_copy_kernel (fuse_copy) do.
+__device__ void chunk_scan_group(int g, int lane, int32_t *hist, int64_t n_chunks, const int32_t *base);
+__device__ void page_copy_group(int g, int lane, const int32_t *page_off_cur, const int32_t *page_list_cur,
+                                const int32_t *page_off_new, const int32_t *first_new, int32_t *page_list_new);
+
 __global__ void __launch_bounds__(kLayoutThreads, 1)
     layout_kernel(int32_t G, int64_t rows, int seg_rows, const int32_t *__restrict__ bcount,
                   const int32_t *__restrict__ bad, int32_t *__restrict__ count,
                   const int32_t *__restrict__ page_off_cur, int32_t *__restrict__ page_off_new,
                   int32_t *__restrict__ first_new, int32_t *__restrict__ base, KeySeg *__restrict__ segs,
                   KeyGroup *__restrict__ kgroups, int32_t *__restrict__ meta, int64_t *__restrict__ id_base,
-                  int64_t *__restrict__ dev_ctr, unsigned *__restrict__ status) {
+                  int64_t *__restrict__ dev_ctr, unsigned *__restrict__ status, int fuse_scan, int32_t *hist,
+                  int64_t n_chunks, int fuse_copy, const int32_t *page_list_cur, int32_t *page_list_new) {
   pdl_entry();  // after the previous kernel of the stream (see common.cuh)
   __shared__ int64_t sh[32];
-  if (*bad) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if (*bad) {  // uniform over the block
     for (int g = threadIdx.x; g <= G; g += blockDim.x) page_off_new[g] = page_off_cur[g];
     if (threadIdx.x == 0) {
       meta[0] = 0;
       meta[1] = 0;
       atomicOr(status, 2u);
+    }
+    if (fuse_copy) {
+      __syncthreads();
+      for (int g = warp; g < G; g += kLayoutThreads / 32) {
+        page_copy_group(g, lane, page_off_cur, page_list_cur, page_off_new, first_new, page_list_new);
+      }
     }
     return;
   }
@@ -173,17 +188,18 @@ __global__ void __launch_bounds__(kLayoutThreads, 1)
     dev_ctr[0] += rows;
     dev_ctr[1] = pages_used + o_np;
   }
+  if (!fuse_scan && !fuse_copy) return;
+  __syncthreads();  // base, page_off_new and first_new of every group are written
+  for (int g = warp; g < G; g += kLayoutThreads / 32) {
+    if (fuse_scan) chunk_scan_group(g, lane, hist, n_chunks, base);
+    if (fuse_copy) page_copy_group(g, lane, page_off_cur, page_list_cur, page_off_new, first_new, page_list_new);
+  }
 }
 
-// One warp per group: the group's page list in the new layout (its current
-// pages, then its fresh ones).
-__global__ void page_copy_kernel(int32_t G, const int32_t *__restrict__ page_off_cur,
-                                 const int32_t *__restrict__ page_list_cur, const int32_t *__restrict__ page_off_new,
-                                 const int32_t *__restrict__ first_new, int32_t *__restrict__ page_list_new) {
-  pdl_entry();  // after the previous kernel of the stream (see common.cuh)
-  const int g = (int)((blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5);
-  const int lane = threadIdx.x & 31;
-  if (g >= G) return;
+// One warp: group g's page list in the new layout (its current pages, then
+// its fresh ones).
+__device__ void page_copy_group(int g, int lane, const int32_t *page_off_cur, const int32_t *page_list_cur,
+                                const int32_t *page_off_new, const int32_t *first_new, int32_t *page_list_new) {
   const int32_t c0 = page_off_cur[g], n_old = page_off_cur[g + 1] - c0;
   const int32_t n0 = page_off_new[g], n_tot = page_off_new[g + 1] - n0;
   for (int32_t i = lane; i < n_tot; i += 32) {
@@ -191,29 +207,19 @@ __global__ void page_copy_kernel(int32_t G, const int32_t *__restrict__ page_off
   }
 }
 
-// hist[g * n_chunks + c] = number of rows of group g in chunk c.
-__global__ void chunk_hist_kernel(const int32_t *__restrict__ gid, const int32_t *__restrict__ ids, int64_t n,
-                                  int64_t chunk, int64_t n_chunks, int32_t *__restrict__ hist,
-                                  const int32_t *__restrict__ bad) {
+__global__ void page_copy_kernel(int32_t G, const int32_t *__restrict__ page_off_cur,
+                                 const int32_t *__restrict__ page_list_cur, const int32_t *__restrict__ page_off_new,
+                                 const int32_t *__restrict__ first_new, int32_t *__restrict__ page_list_new) {
   pdl_entry();  // after the previous kernel of the stream (see common.cuh)
-  if (*bad) return;
-  int64_t c = blockIdx.x;
-  int64_t lo = c * chunk, hi = min(n, lo + chunk);
-  for (int64_t e = lo + threadIdx.x; e < hi; e += blockDim.x) {
-    atomicAdd(&hist[(int64_t)row_group(gid, ids, e) * n_chunks + c], 1);
-  }
+  const int g = (int)((blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5);
+  if (g >= G) return;
+  page_copy_group(g, threadIdx.x & 31, page_off_cur, page_list_cur, page_off_new, first_new, page_list_new);
 }
 
-// Per group (one warp each): hist[g][c] <- base[g] + sum_{c' < c} hist[g][c'].
-__global__ void chunk_scan_kernel(int32_t *__restrict__ hist, int64_t n_chunks, int32_t n_groups,
-                                  const int32_t *__restrict__ base, const int32_t *__restrict__ bad) {
-  pdl_entry();  // after the previous kernel of the stream (see common.cuh)
-  if (*bad) return;
-  int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  int lane = threadIdx.x & 31;
-  if (warp >= n_groups) return;
-  int32_t *row = hist + (int64_t)warp * n_chunks;
-  int32_t running = base[warp];
+// One warp: hist[g][c] <- base[g] + sum_{c' < c} hist[g][c'].
+__device__ void chunk_scan_group(int g, int lane, int32_t *hist, int64_t n_chunks, const int32_t *base) {
+  int32_t *row = hist + (int64_t)g * n_chunks;
+  int32_t running = base[g];
   for (int64_t c0 = 0; c0 < n_chunks; c0 += 32) {
     int64_t c = c0 + lane;
     int32_t v = c < n_chunks ? row[c] : 0;
@@ -226,6 +232,17 @@ __global__ void chunk_scan_kernel(int32_t *__restrict__ hist, int64_t n_chunks, 
     if (c < n_chunks) row[c] = running + incl - v;
     running += __shfl_sync(kFullMask, incl, 31);
   }
+}
+
+// Per group (one warp each), for large layouts.
+__global__ void chunk_scan_kernel(int32_t *__restrict__ hist, int64_t n_chunks, int32_t n_groups,
+                                  const int32_t *__restrict__ base, const int32_t *__restrict__ bad) {
+  pdl_entry();  // after the previous kernel of the stream (see common.cuh)
+  if (*bad) return;
+  int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  int lane = threadIdx.x & 31;
+  if (warp >= n_groups) return;
+  chunk_scan_group(warp, lane, hist, n_chunks, base);
 }
 
 // One warp per chunk walks its rows in order; rows of the same group take
@@ -361,8 +378,18 @@ __global__ void key_finalize_kernel(const KeyGroup *__restrict__ groups, const i
   // split in fp32: hi = bf16(mean), lo = bf16(mean - hi).
   const double inv = kg.count > 0 ? 1.0 / (double)kg.count : 0.0;
   for (int j = blockIdx.y * blockDim.x + threadIdx.x; j < d; j += gridDim.y * blockDim.x) {
+    // The segments' partial sums added in segment order, loaded eight at a
+    // time so that a group of many segments is not one load per step.
     double add = 0.0;
-    for (int s = kg.seg0; s < kg.seg1; ++s) add += partial[(int64_t)s * d + j];
+    for (int s0 = kg.seg0; s0 < kg.seg1; s0 += 8) {
+      double v[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) v[u] = s0 + u < kg.seg1 ? partial[(int64_t)(s0 + u) * d + j] : 0.0;
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        if (s0 + u < kg.seg1) add += v[u];
+      }
+    }
     int64_t o = (int64_t)kg.g * d + j;
     double sum = csum[o] + add;
     csum[o] = sum;
@@ -451,20 +478,24 @@ static htam_status add_rows(htam_memory *m, const void *entries, const int32_t *
   const int seg_rows = key_seg_rows(count);
   int64_t max_segs = std::min<int64_t>(count, count / seg_rows + G + 1);
 
-  size_t need = Carver::round(sizeof(int32_t) * (G + 2)) + Carver::round(sizeof(int32_t) * 4) +
-                Carver::round(sizeof(int64_t)) + (build ? 0 : Carver::round(sizeof(int32_t) * count)) +
-                Carver::round(sizeof(int32_t) * count) + Carver::round(sizeof(int32_t) * (size_t)G * n_chunks) +
+  size_t need = Carver::round(sizeof(int32_t) * (ceil_div(G + 2, 64) * 64 + (size_t)G * n_chunks)) +
+                Carver::round(sizeof(int32_t) * 4) + Carver::round(sizeof(int64_t)) +
+                (build ? 0 : Carver::round(sizeof(int32_t) * count)) + Carver::round(sizeof(int32_t) * count) +
                 Carver::round(sizeof(KeySeg) * max_segs) + Carver::round(sizeof(KeyGroup) * G) +
                 2 * Carver::round(sizeof(int32_t) * G) + Carver::round(sizeof(double) * (size_t)max_segs * d) + 4096;
   htam_status s = ensure_scratch(m, need);
   if (s != HTAM_OK) return s;
   Carver cv(m->scratch);
-  int32_t *bcount = cv.take<int32_t>(G + 2);  // [G] counts, bad flag, rows without a group
+  // Cleared by one memset: the batch's counts, the bad flag, the count of
+  // rows without a group, then the (group, chunk) counts of the stable sort.
+  const int64_t hist_off = ceil_div(G + 2, 64) * 64;
+  const int64_t n_zero = hist_off + (int64_t)G * n_chunks;
+  int32_t *bcount = cv.take<int32_t>(n_zero);  // [G] counts, bad flag, rows without a group
   int32_t *meta = cv.take<int32_t>(4);         // key segments, touched groups
   int64_t *id_base = cv.take<int64_t>(1);
   int32_t *ids = build ? nullptr : cv.take<int32_t>(count);  // groups chosen for rows given -1
   int32_t *pos = cv.take<int32_t>(count);
-  int32_t *hist = cv.take<int32_t>((size_t)G * n_chunks);
+  int32_t *hist = bcount + hist_off;
   KeySeg *segs = cv.take<KeySeg>(max_segs);
   KeyGroup *kgroups = cv.take<KeyGroup>(G);
   int32_t *first_new = cv.take<int32_t>(G);
@@ -476,13 +507,13 @@ static htam_status add_rows(htam_memory *m, const void *entries, const int32_t *
   PhaseMark mark(m, st);
   mark.begin(HTAM_PHASE_APPEND);
 
-  // 1. Per-group counts of the batch and the group-id range check (the same
-  //    grid clears the slot counters).
-  HTAM_CK(cudaMemsetAsync(bcount, 0, sizeof(int32_t) * (G + 2), st));
+  // 1. Per-group and per-(group, chunk) counts of the batch and the
+  //    group-id range check.
+  HTAM_CK(cudaMemsetAsync(bcount, 0, sizeof(int32_t) * n_zero, st));
   {
-    const int blocks = (int)std::min<int64_t>(ceil_div(std::max<int64_t>(count, (int64_t)G * n_chunks), 256), 4096);
-    launch_kernel(count_groups_kernel, blocks, 256, 0, st, gid, count, G, build ? 0 : 1, bcount, bad, bcount + G + 1, hist,
-                                                (int64_t)G * n_chunks);
+    const int blocks = (int)std::min<int64_t>(ceil_div(count, 256), 4096);
+    launch_kernel(count_groups_kernel, blocks, 256, 0, st, gid, count, G, build ? 0 : 1, bcount, bad, bcount + G + 1,
+                  hist, chunk, n_chunks);
     HTAM_CK_LAUNCH("count_groups_kernel");
     mark.launched();
   }
@@ -490,30 +521,43 @@ static htam_status add_rows(htam_memory *m, const void *entries, const int32_t *
   //    them, by the keys as they stand before this call.  The kernels run
   //    only when the count above found such rows.
   if (!build) {
-    s = assign_unassigned(m, entries, gid, count, bcount + G + 1, ids, bcount, bad, st, &mark);
+    s = assign_unassigned(m, entries, gid, count, bcount + G + 1, ids, bcount, bad, hist, chunk, n_chunks, st,
+                          &mark);
     if (s != HTAM_OK) return s;
   }
-  // 3. Page layout, key segments and new sizes; then the page lists.
+  // 3. Page layout, key segments and new sizes; then the page lists and the
+  //    scan of the (group, chunk) counts from each group's old size (in the
+  //    same block when they are small, one warp per group, else by kernels
+  //    of their own).
+  // (One block walks each warp's groups one after another, so this pays
+  // only for a few counters and pages; the 512-group streaming workload
+  // runs faster with the separate kernels.)
+  const bool fuse_scan = (int64_t)G * n_chunks <= 2048;
+  const bool fuse_copy = m->n_pages_max <= 2048;
   launch_kernel(layout_kernel, 1, kLayoutThreads, 0, st, G, count, seg_rows, bcount, bad, m->count, m->page_off,
-                                              m->page_off_alt, first_new, base, segs, kgroups, meta, id_base,
-                                              m->dev_ctr, m->status);
+                m->page_off_alt, first_new, base, segs, kgroups, meta, id_base, m->dev_ctr, m->status,
+                fuse_scan ? 1 : 0, hist, n_chunks, fuse_copy ? 1 : 0, m->page_list, m->page_list_alt);
   HTAM_CK_LAUNCH("layout_kernel");
-  launch_kernel(page_copy_kernel, (unsigned)ceil_div((int64_t)G * 32, 256), 256, 0, st, G, m->page_off, m->page_list,
-                                                                             m->page_off_alt, first_new,
-                                                                             m->page_list_alt);
-  HTAM_CK_LAUNCH("page_copy_kernel");
-  mark.launched(2);
+  mark.launched();
+  if (!fuse_copy) {
+    launch_kernel(page_copy_kernel, (unsigned)ceil_div((int64_t)G * 32, 256), 256, 0, st, G, m->page_off,
+                  m->page_list, m->page_off_alt, first_new, m->page_list_alt);
+    HTAM_CK_LAUNCH("page_copy_kernel");
+    mark.launched();
+  }
 
   // 4. Stable slot assignment: pos[e] = old size of its group + rank among
   //    earlier rows of the batch with the same group.
-  launch_kernel(chunk_hist_kernel, (unsigned)n_chunks, 256, 0, st, gid, ids, count, chunk, n_chunks, hist, bad);
-  HTAM_CK_LAUNCH("chunk_hist_kernel");
-  launch_kernel(chunk_scan_kernel, (unsigned)ceil_div((int64_t)G * 32, 256), 256, 0, st, hist, n_chunks, G, base, bad);
-  HTAM_CK_LAUNCH("chunk_scan_kernel");
+  if (!fuse_scan) {
+    launch_kernel(chunk_scan_kernel, (unsigned)ceil_div((int64_t)G * 32, 256), 256, 0, st, hist, n_chunks, G, base,
+                  bad);
+    HTAM_CK_LAUNCH("chunk_scan_kernel");
+    mark.launched();
+  }
   launch_kernel(chunk_place_kernel, (unsigned)ceil_div(n_chunks * 32, 256), 256, 0, st, gid, ids, count, chunk, n_chunks, hist,
                                                                              pos, bad);
   HTAM_CK_LAUNCH("chunk_place_kernel");
-  mark.launched(3);
+  mark.launched();
 
   // 5. Copy rows into their slots.
   int vec_per_row = d * m->elem_bytes / 16;

@@ -1628,7 +1628,8 @@ namespace {
 // the batch bad.  Gated on the batch's count of such rows.
 __global__ void assign_resolve_kernel(const int32_t *__restrict__ gid, const int32_t *__restrict__ pick, int64_t n,
                                       const int32_t *__restrict__ gate, int32_t *__restrict__ ids,
-                                      int32_t *__restrict__ bcount, int32_t *__restrict__ bad) {
+                                      int32_t *__restrict__ bcount, int32_t *__restrict__ bad,
+                                      int32_t *__restrict__ hist, int64_t row0, int64_t chunk, int64_t n_chunks) {
   pdl_entry();  // after the previous kernel of the stream (see common.cuh)
   if (*gate == 0) return;
   for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < n; t += (int64_t)gridDim.x * blockDim.x) {
@@ -1639,6 +1640,7 @@ __global__ void assign_resolve_kernel(const int32_t *__restrict__ gid, const int
     } else {
       ids[t] = p;
       atomicAdd(&bcount[p], 1);
+      atomicAdd(&hist[(int64_t)p * n_chunks + (row0 + t) / chunk], 1);
     }
   }
 }
@@ -1647,7 +1649,7 @@ __global__ void assign_resolve_kernel(const int32_t *__restrict__ gid, const int
 
 htam_status assign_unassigned(htam_memory *m, const void *entries, const int32_t *gid, int64_t count,
                               const int32_t *n_unassigned, int32_t *ids, int32_t *bcount, int32_t *bad,
-                              cudaStream_t st, PhaseMark *mark) {
+                              int32_t *hist, int64_t chunk, int64_t n_chunks, cudaStream_t st, PhaseMark *mark) {
   const int G = m->n_groups, d = m->d;
   // Rows per pass: the [rows, G] score matrix stays within 16 MiB per plane.
   const int64_t R = std::max<int64_t>(1, std::min<int64_t>(count, (int64_t(1) << 22) / G));
@@ -1696,7 +1698,8 @@ htam_status assign_unassigned(htam_memory *m, const void *entries, const int32_t
     }
     HTAM_CK_LAUNCH("group_topk_kernel");
     const unsigned blocks = (unsigned)std::min<int64_t>(ceil_div(rb, 256), 1024);
-    launch_kernel(assign_resolve_kernel, blocks, 256, 0, st, gid + r0, pick, rb, n_unassigned, ids + r0, bcount, bad);
+    launch_kernel(assign_resolve_kernel, blocks, 256, 0, st, gid + r0, pick, rb, n_unassigned, ids + r0, bcount, bad, hist, r0, chunk,
+                  n_chunks);
     HTAM_CK_LAUNCH("assign_resolve_kernel");
     if (mark) mark->launched(3);
   }
