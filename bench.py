@@ -194,6 +194,26 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
+def read_probe_gbs(dev, gib: int = 4, reps: int = 5) -> float:
+    """Context for the HBM roofline: a read-only stream (torch's sum of a
+    4 GiB int32 tensor), which a gather that only reads can exceed the
+    measured copy peak by.  Best of `reps`, CUDA events."""
+    x = torch.ones((gib << 30) // 4, dtype=torch.int32, device=dev)
+    x.sum()
+    best = float("inf")
+    for _ in range(reps):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        x.sum()
+        b.record()
+        torch.cuda.synchronize()
+        best = min(best, a.elapsed_time(b) / 1e3)
+    n = x.numel() * 4
+    del x
+    torch.cuda.empty_cache()
+    return n / best / 1e9
+
+
 def source_sha(*names) -> str:
     h = hashlib.sha256()
     for n in names:
@@ -527,6 +547,10 @@ def measure(args, world, rank, local, full=True):
         roofline = {"kernel": kernel, "bound": "hbm", "achieved": k_bytes / k_s / 1e9, "peak": peaks["hbm_gbs"],
                     "unit": "GB/s", "alu_frac": k_flops / k_s / 1e12 / FP32_ALU_TFLOPS}
     roofline["frac"] = roofline["achieved"] / roofline["peak"]
+    if roofline["bound"] == "hbm" and full:
+        probe = read_probe_gbs(dev)
+        roofline.update({"read_probe_gbs": probe, "frac_of_read_probe": roofline["achieved"] / probe,
+                         "read_probe_note": "context only: torch sum of 4 GiB, read-only, best of 5"})
     # Profiles are per lookup variant: the variant decides the buckets.
     variant = ("_flat" if args.flat else "_sampled" if args.sample else "_edges" if E > 0 else
                "_prefix" if P > 0 else "_unassigned" if args.unassigned > 0 and w.rounds else "")
