@@ -195,16 +195,16 @@ class ClockSampler:
 
 
 def read_probe_gbs(dev, gib: int = 4, reps: int = 5) -> float:
-    """Context for the HBM roofline: a read-only stream (torch's sum of a
-    4 GiB int32 tensor), which a gather that only reads can exceed the
+    """Context for the HBM roofline: a read-only stream (torch's max of a
+    4 GiB fp32 tensor), which a gather that only reads can exceed the
     measured copy peak by.  Best of `reps`, CUDA events."""
-    x = torch.ones((gib << 30) // 4, dtype=torch.int32, device=dev)
-    x.sum()
+    x = torch.ones((gib << 30) // 4, dtype=torch.float32, device=dev)
+    x.amax()
     best = float("inf")
     for _ in range(reps):
         a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         a.record()
-        x.sum()
+        x.amax()
         b.record()
         torch.cuda.synchronize()
         best = min(best, a.elapsed_time(b) / 1e3)
@@ -550,7 +550,7 @@ def measure(args, world, rank, local, full=True):
     if roofline["bound"] == "hbm" and full:
         probe = read_probe_gbs(dev)
         roofline.update({"read_probe_gbs": probe, "frac_of_read_probe": roofline["achieved"] / probe,
-                         "read_probe_note": "context only: torch sum of 4 GiB, read-only, best of 5"})
+                         "read_probe_note": "context only: torch amax over 4 GiB of fp32, read-only, best of 5"})
     # Profiles are per lookup variant: the variant decides the buckets.
     variant = ("_flat" if args.flat else "_sampled" if args.sample else "_edges" if E > 0 else
                "_prefix" if P > 0 else "_unassigned" if args.unassigned > 0 and w.rounds else "")
