@@ -74,6 +74,7 @@ struct KeySeg {
 };
 struct KeyGroup {
   int32_t g, seg0, seg1, count;
+  double inv;  // 1 / count (0 for an empty group), taken once per group by the layout block
 };
 
 // Inclusive scan of one value per thread over a block of kLayoutThreads.
@@ -117,7 +118,8 @@ __device__ __forceinline__ int64_t block_scan_incl(int64_t v, int64_t *sh /* [32
 // A bad batch changes nothing: the current offsets are copied to the new
 // layout, no segment is listed, and status bit 1 records the rejection.
 // For small batches and layouts the same block then does what
-// chunk_scan_kernel (fuse_scan) and page_copy_kernel (fuse_copy) do.
+// group_lists_kernel does (the chunk scan when fuse_scan, the page list copy
+// when fuse_copy).
 __device__ void chunk_scan_group(int g, int lane, int32_t *hist, int64_t n_chunks, const int32_t *base);
 __device__ void page_copy_group(int g, int lane, const int32_t *page_off_cur, const int32_t *page_list_cur,
                                 const int32_t *page_off_new, const int32_t *first_new, int32_t *page_list_new);
@@ -175,7 +177,7 @@ __global__ void __launch_bounds__(kLayoutThreads, 1)
       for (int64_t r = old; r < nw; r += seg_rows) {
         segs[o_ns++] = KeySeg{g, (int32_t)r, (int32_t)min(nw, r + seg_rows), 0};
       }
-      kgroups[o_nt++] = KeyGroup{g, s0, (int32_t)o_ns, (int32_t)nw};
+      kgroups[o_nt++] = KeyGroup{g, s0, (int32_t)o_ns, (int32_t)nw, nw > 0 ? 1.0 / (double)nw : 0.0};
       count[g] = (int32_t)nw;
     }
   }
@@ -207,15 +209,6 @@ __device__ void page_copy_group(int g, int lane, const int32_t *page_off_cur, co
   }
 }
 
-__global__ void page_copy_kernel(int32_t G, const int32_t *__restrict__ page_off_cur,
-                                 const int32_t *__restrict__ page_list_cur, const int32_t *__restrict__ page_off_new,
-                                 const int32_t *__restrict__ first_new, int32_t *__restrict__ page_list_new) {
-  pdl_entry();  // after the previous kernel of the stream (see common.cuh)
-  const int g = (int)((blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5);
-  if (g >= G) return;
-  page_copy_group(g, threadIdx.x & 31, page_off_cur, page_list_cur, page_off_new, first_new, page_list_new);
-}
-
 // One warp: hist[g][c] <- base[g] + sum_{c' < c} hist[g][c'].
 __device__ void chunk_scan_group(int g, int lane, int32_t *hist, int64_t n_chunks, const int32_t *base) {
   int32_t *row = hist + (int64_t)g * n_chunks;
@@ -234,15 +227,19 @@ __device__ void chunk_scan_group(int g, int lane, int32_t *hist, int64_t n_chunk
   }
 }
 
-// Per group (one warp each), for large layouts.
-__global__ void chunk_scan_kernel(int32_t *__restrict__ hist, int64_t n_chunks, int32_t n_groups,
-                                  const int32_t *__restrict__ base, const int32_t *__restrict__ bad) {
+// Per group (one warp each), for large layouts: the page list copy and, for a
+// batch that passed the check, the chunk scan, in one launch.
+__global__ void group_lists_kernel(int32_t G, const int32_t *__restrict__ page_off_cur,
+                                   const int32_t *__restrict__ page_list_cur, const int32_t *__restrict__ page_off_new,
+                                   const int32_t *__restrict__ first_new, int32_t *__restrict__ page_list_new,
+                                   int do_copy, int32_t *__restrict__ hist, int64_t n_chunks, int do_scan,
+                                   const int32_t *__restrict__ base, const int32_t *__restrict__ bad) {
   pdl_entry();  // after the previous kernel of the stream (see common.cuh)
-  if (*bad) return;
-  int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  int lane = threadIdx.x & 31;
-  if (warp >= n_groups) return;
-  chunk_scan_group(warp, lane, hist, n_chunks, base);
+  const int g = (int)((blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5);
+  const int lane = threadIdx.x & 31;
+  if (g >= G) return;
+  if (do_copy) page_copy_group(g, lane, page_off_cur, page_list_cur, page_off_new, first_new, page_list_new);
+  if (do_scan && !*bad) chunk_scan_group(g, lane, hist, n_chunks, base);
 }
 
 // One warp per chunk walks its rows in order; rows of the same group take
@@ -275,6 +272,60 @@ __global__ void chunk_place_kernel(const int32_t *__restrict__ gid, const int32_
       pos[e] = old + rank;
     }
     __syncwarp();
+  }
+}
+
+// Chunks of 32 rows (appends): one block per chunk.  Its first warp takes
+// the chunk's rows in order and gives each its slot as chunk_place_kernel
+// does; then the block's eight warps copy the rows into their slots as
+// place_rows_kernel does, four rows each.  (Every group id of the chunk is
+// read before the barrier, so `assigned` may alias `gid`.)
+constexpr int kPlaceWarps = 8;
+__global__ void __launch_bounds__(kPlaceWarps * 32)
+    place_chunk_kernel(const uint4 *__restrict__ src, const int32_t *gid, const int32_t *__restrict__ ids, int64_t n,
+                       int64_t n_chunks, int32_t *__restrict__ hist, int vec_per_row,
+                       const int32_t *__restrict__ page_list, const int32_t *__restrict__ page_off,
+                       uint4 *__restrict__ pool, int32_t *__restrict__ slot_id, const int64_t *__restrict__ id_base,
+                       int32_t *assigned, const int32_t *__restrict__ bad) {
+  pdl_entry();  // after the previous kernel of the stream (see common.cuh)
+  __shared__ int32_t s_grp[32], s_pos[32];
+  if (*bad) return;  // uniform over the grid
+  const int64_t c = blockIdx.x;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t lo = c * 32, hi = min(n, lo + 32);
+  if (warp == 0) {
+    const int64_t e = lo + lane;
+    const unsigned act = __ballot_sync(kFullMask, e < hi);
+    if (e < hi) {
+      const int32_t g = row_group(gid, ids, e);
+      const unsigned peers = __match_any_sync(act, g);
+      const int leader = __ffs(peers) - 1;
+      const int rank = __popc(peers & ((1u << lane) - 1u));
+      int32_t old = 0;
+      int32_t *slot = &hist[(int64_t)g * n_chunks + c];
+      if (lane == leader) {
+        old = *slot;
+        *slot = old + __popc(peers);
+      }
+      old = __shfl_sync(act, old, leader);
+      s_grp[lane] = g;
+      s_pos[lane] = old + rank;
+    }
+  }
+  __syncthreads();
+  const int rows = (int)(hi - lo);
+  for (int i = warp; i < rows; i += kPlaceWarps) {
+    const int64_t e = lo + i;
+    const int32_t g = s_grp[i], p = s_pos[i];
+    const int64_t page = page_list[page_off[g] + p / kPageRows];
+    const int64_t sl = page * kPageRows + (p % kPageRows);
+    const uint4 *s = src + e * vec_per_row;
+    uint4 *dst = pool + sl * vec_per_row;
+    for (int v = lane; v < vec_per_row; v += 32) dst[v] = s[v];
+    if (lane == 0) {
+      slot_id[sl] = (int32_t)(*id_base + e);
+      if (assigned) assigned[e] = g;
+    }
   }
 }
 
@@ -373,10 +424,10 @@ __global__ void key_finalize_kernel(const KeyGroup *__restrict__ groups, const i
   pdl_entry();  // after the previous kernel of the stream (see common.cuh)
   if ((int)blockIdx.x >= *n_groups) return;  // the grid covers every group
   KeyGroup kg = groups[blockIdx.x];
-  // One fp64 reciprocal per group instead of a division per column (fp64
-  // arithmetic is slow on this part); the mean is then rounded to fp32 and
-  // split in fp32: hi = bf16(mean), lo = bf16(mean - hi).
-  const double inv = kg.count > 0 ? 1.0 / (double)kg.count : 0.0;
+  // The group's fp64 reciprocal comes from the layout block (fp64
+  // arithmetic is slow on this part, a division most of all); the mean is
+  // then rounded to fp32 and split in fp32: hi = bf16(mean), lo = bf16(mean - hi).
+  const double inv = kg.inv;
   for (int j = blockIdx.y * blockDim.x + threadIdx.x; j < d; j += gridDim.y * blockDim.x) {
     // The segments' partial sums added in segment order, loaded eight at a
     // time so that a group of many segments is not one load per step.
@@ -539,33 +590,39 @@ static htam_status add_rows(htam_memory *m, const void *entries, const int32_t *
                 fuse_scan ? 1 : 0, hist, n_chunks, fuse_copy ? 1 : 0, m->page_list, m->page_list_alt);
   HTAM_CK_LAUNCH("layout_kernel");
   mark.launched();
-  if (!fuse_copy) {
-    launch_kernel(page_copy_kernel, (unsigned)ceil_div((int64_t)G * 32, 256), 256, 0, st, G, m->page_off,
-                  m->page_list, m->page_off_alt, first_new, m->page_list_alt);
-    HTAM_CK_LAUNCH("page_copy_kernel");
+  // 4. The page lists of the new layout and the scan of the (group, chunk)
+  //    counts from each group's old size, one warp per group, when the
+  //    layout block did not do them.
+  if (!fuse_copy || !fuse_scan) {
+    launch_kernel(group_lists_kernel, (unsigned)ceil_div((int64_t)G * 32, 256), 256, 0, st, G, m->page_off,
+                  m->page_list, m->page_off_alt, first_new, m->page_list_alt, fuse_copy ? 0 : 1, hist, n_chunks,
+                  fuse_scan ? 0 : 1, base, bad);
+    HTAM_CK_LAUNCH("group_lists_kernel");
     mark.launched();
   }
 
-  // 4. Stable slot assignment: pos[e] = old size of its group + rank among
-  //    earlier rows of the batch with the same group.
-  if (!fuse_scan) {
-    launch_kernel(chunk_scan_kernel, (unsigned)ceil_div((int64_t)G * 32, 256), 256, 0, st, hist, n_chunks, G, base,
-                  bad);
-    HTAM_CK_LAUNCH("chunk_scan_kernel");
-    mark.launched();
-  }
-  launch_kernel(chunk_place_kernel, (unsigned)ceil_div(n_chunks * 32, 256), 256, 0, st, gid, ids, count, chunk, n_chunks, hist,
-                                                                             pos, bad);
-  HTAM_CK_LAUNCH("chunk_place_kernel");
-  mark.launched();
-
-  // 5. Copy rows into their slots.
+  // 5. Stable slot assignment (pos[e] = old size of its group + rank among
+  //    earlier rows of the batch with the same group), then the rows copied
+  //    into their slots: one launch for chunks of 32 rows (appends), two
+  //    for the long chunks of large builds.
   int vec_per_row = d * m->elem_bytes / 16;
-  launch_kernel(place_rows_kernel, (unsigned)ceil_div(count * 32, 256), 256, 0, st, 
-      static_cast<const uint4 *>(entries), gid, ids, pos, count, vec_per_row, m->page_list_alt, m->page_off_alt,
-      static_cast<uint4 *>(m->pool), m->slot_id, id_base, assigned, bad);
-  HTAM_CK_LAUNCH("place_rows_kernel");
-  mark.launched();
+  if (chunk == 32) {
+    launch_kernel(place_chunk_kernel, (unsigned)n_chunks, kPlaceWarps * 32, 0, st,
+                  static_cast<const uint4 *>(entries), gid, ids, count, n_chunks, hist, vec_per_row,
+                  m->page_list_alt, m->page_off_alt, static_cast<uint4 *>(m->pool), m->slot_id, id_base, assigned,
+                  bad);
+    HTAM_CK_LAUNCH("place_chunk_kernel");
+    mark.launched();
+  } else {
+    launch_kernel(chunk_place_kernel, (unsigned)ceil_div(n_chunks * 32, 256), 256, 0, st, gid, ids, count, chunk,
+                  n_chunks, hist, pos, bad);
+    HTAM_CK_LAUNCH("chunk_place_kernel");
+    launch_kernel(place_rows_kernel, (unsigned)ceil_div(count * 32, 256), 256, 0, st,
+                  static_cast<const uint4 *>(entries), gid, ids, pos, count, vec_per_row, m->page_list_alt,
+                  m->page_off_alt, static_cast<uint4 *>(m->pool), m->slot_id, id_base, assigned, bad);
+    HTAM_CK_LAUNCH("place_rows_kernel");
+    mark.launched(2);
+  }
 
   // 6. Keys of the touched groups.
   {
