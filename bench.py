@@ -397,7 +397,7 @@ def measure(args, world, rank, local, full=True):
     if args.fine_overlap is not None:
         mem.set_fine_overlap(args.fine_overlap)
     tc_min = mem.get_tuning(htam.HTAM_TUNE_TC_MIN_BUCKET)
-    if args.no_cpu_baseline:
+    if args.no_cpu_baseline and not w.rounds:
         del entries                  # the memory holds its own copy
         torch.cuda.empty_cache()
     q_seed = args.seed + 1000 * rank
@@ -423,19 +423,20 @@ def measure(args, world, rank, local, full=True):
         edge_prefix = [rng.integers(0, w.g, (w.b, E)).astype(np.int32) for _ in range(args.batches)]
     batch_of = {id(q): i for i, q in enumerate(batches)}
 
-    def run_query(q, out=None):
+    def run_query(q, out=None, m=None):
+        m = mem if m is None else m
         if args.flat:
-            return mem.query_flat(q, w.k_entries, out=out)
+            return m.query_flat(q, w.k_entries, out=out)
         if E > 0:
-            return mem.query_edges(edge_z, edge_w, edge_prefix[batch_of.get(id(q), 0)], args.prefix_lambda, q,
-                                   w.k_groups, w.k_entries, out=out,
-                                   sampling=(args.seed, batch_of.get(id(q), 0)) if args.sample else None)
+            return m.query_edges(edge_z, edge_w, edge_prefix[batch_of.get(id(q), 0)], args.prefix_lambda, q,
+                                 w.k_groups, w.k_entries, out=out,
+                                 sampling=(args.seed, batch_of.get(id(q), 0)) if args.sample else None)
         if args.sample:
-            return mem.query_sampled(q, w.k_groups, w.k_entries, seed=args.seed, offset=batch_of.get(id(q), 0),
-                                     out=out)
+            return m.query_sampled(q, w.k_groups, w.k_entries, seed=args.seed, offset=batch_of.get(id(q), 0),
+                                   out=out)
         if P > 0:
-            return mem.query_prefix(q, args.prefix_lambda, w.k_groups, w.k_entries, out=out)
-        return mem.query(q, w.k_groups, w.k_entries, out=out)
+            return m.query_prefix(q, args.prefix_lambda, w.k_groups, w.k_entries, out=out)
+        return m.query(q, w.k_groups, w.k_entries, out=out)
 
     append_batches = []
     if w.rounds:
@@ -466,6 +467,36 @@ def measure(args, world, rank, local, full=True):
             wk["step_bytes"] += rows * w.g * args.edge_features * 4 - w.g * w.d * 4
             wk["step_flops"] += 2.0 * args.edge_features * E * w.b * w.g - 2.0 * w.d * w.b * w.g
         work.append(wk)
+    # The streaming workload's memory grows by one append per step, so the
+    # work of step a (append a, then query batch a) is measured on a second
+    # memory that replays the same appends and queries: the timed region is
+    # steps warmup .. warmup+steps-1, the per-phase pass the next `steps`.
+    # Its bytes include the append's: the new rows read and stored, and the
+    # touched groups' keys (fp64 sums read and written, fp32 mean and the
+    # bf16 halves written).
+    stream_work = None
+    if w.rounds:
+        mem2 = htam.Memory(entries, gid, w.g, capacity=capacity)
+        for setter, val in ((mem2.set_stream_rows, args.stream_rows), (mem2.set_tensor_core_min_bucket,
+                            args.tc_min_bucket), (mem2.set_tensor_core_pairs, args.tc_pairs)):
+            if val is not None:
+                setter(val)
+        s_elem = 2 if w.dtype == "bf16" else 4
+        stream_work = []
+        for a in range(args.warmup + 2 * args.steps):
+            e, g = append_batches[a % len(append_batches)]
+            mem2.append(e, g)
+            o = run_query(batches[a % len(batches)], m=mem2)
+            counts_a = mem2.group_counts().numpy()
+            wk = step_work(w, counts_a, o["group_idx"].cpu().numpy(), tc_min, flat=args.flat)
+            touched = int(torch.unique(g[g >= 0]).numel()) if args.unassigned == 0 else w.g
+            wk["step_bytes"] += 2.0 * e.shape[0] * w.d * s_elem + touched * w.d * (8 + 8 + 4 + 2 + 2)
+            stream_work.append(wk)
+        mem2.close()
+        if args.no_cpu_baseline:
+            del entries
+            torch.cuda.empty_cache()
+
     flush_l2 = work[0]["step_bytes"] < 4 * l2_bytes
     flush = torch.empty(2 * l2_bytes, dtype=torch.uint8, device=dev) if flush_l2 else None
 
@@ -519,7 +550,12 @@ def measure(args, world, rank, local, full=True):
 
     # Dominant kernel roofline (live CUDA events on the launching stream).
     peaks = load_peaks()
-    per_batch = [work[(args.warmup + i) % len(work)] for i in range(args.steps)]
+    if stream_work is not None:
+        per_batch = stream_work[args.warmup:args.warmup + args.steps]
+        phase_batch = stream_work[args.warmup + args.steps:]
+    else:
+        per_batch = [work[(args.warmup + i) % len(work)] for i in range(args.steps)]
+        phase_batch = per_batch
     step_bytes = float(np.mean([x["step_bytes"] for x in per_batch]))
     step_flops = float(np.mean([x["step_flops"] for x in per_batch]))
     # The dominant kernel: the fine kernel (CUDA-core or tensor-core) with the
@@ -530,8 +566,8 @@ def measure(args, world, rank, local, full=True):
     # The phase's device time per step (one launch per step, two when the
     # tensor-core buckets are split between the SM-pair and one-SM kernels).
     k_s = k_ms / 1e3 / args.steps
-    k_bytes = float(np.mean([x["kernels"][phase]["bytes"] for x in per_batch]))
-    k_flops = float(np.mean([x["kernels"][phase]["flops"] for x in per_batch]))
+    k_bytes = float(np.mean([x["kernels"][phase]["bytes"] for x in phase_batch]))
+    k_flops = float(np.mean([x["kernels"][phase]["flops"] for x in phase_batch]))
     if phase == "fine_tc":
         tensor_peak = peaks["bf16_tflops_sustained"] or peaks["bf16_tflops"]
         t_hbm = k_bytes / (peaks["hbm_gbs"] * 1e9)
