@@ -62,6 +62,10 @@ struct htam_memory {
   int64_t append_seq = 0;        // appends queued
   int64_t mirror_seq = 0;        // the append the mirror reflects
   void *h_pin = nullptr;         // kMirrorSlots x (int64 n, int32 counts[G])
+  void *d_pin = nullptr;         // h_pin as the device sees it (the last append kernel writes the slots)
+  int32_t *batch_ctr = nullptr;  // batch counters of add_rows, zero between batches
+  int64_t batch_ctr_len = 0;
+  bool batch_dirty = false;       // a batch stopped before clearing them
   size_t pin_slot_bytes = 0;
   cudaEvent_t mirror_ev[kMirrorSlots] = {};
   int64_t slot_seq[kMirrorSlots] = {};       // append number each slot holds (0 = none)

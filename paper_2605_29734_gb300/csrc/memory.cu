@@ -125,7 +125,7 @@ __device__ void page_copy_group(int g, int lane, const int32_t *page_off_cur, co
                                 const int32_t *page_off_new, const int32_t *first_new, int32_t *page_list_new);
 
 __global__ void __launch_bounds__(kLayoutThreads, 1)
-    layout_kernel(int32_t G, int64_t rows, int seg_rows, const int32_t *__restrict__ bcount,
+    layout_kernel(int32_t G, int64_t rows, int seg_rows, int32_t *__restrict__ bcount,
                   const int32_t *__restrict__ bad, int32_t *__restrict__ count,
                   const int32_t *__restrict__ page_off_cur, int32_t *__restrict__ page_off_new,
                   int32_t *__restrict__ first_new, int32_t *__restrict__ base, KeySeg *__restrict__ segs,
@@ -137,10 +137,14 @@ __global__ void __launch_bounds__(kLayoutThreads, 1)
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   if (*bad) {  // uniform over the block
     for (int g = threadIdx.x; g <= G; g += blockDim.x) page_off_new[g] = page_off_cur[g];
+    // The batch's group counts and its count of rows without a group are
+    // read by nothing after this block: cleared here for the next batch.
+    for (int g = threadIdx.x; g < G; g += blockDim.x) bcount[g] = 0;
     if (threadIdx.x == 0) {
       meta[0] = 0;
       meta[1] = 0;
       atomicOr(status, 2u);
+      bcount[G + 1] = 0;
     }
     if (fuse_copy) {
       __syncthreads();
@@ -180,7 +184,9 @@ __global__ void __launch_bounds__(kLayoutThreads, 1)
       kgroups[o_nt++] = KeyGroup{g, s0, (int32_t)o_ns, (int32_t)nw, nw > 0 ? 1.0 / (double)nw : 0.0};
       count[g] = (int32_t)nw;
     }
+    bcount[g] = 0;  // read for the last time: cleared for the next batch
   }
+  if (threadIdx.x == 0) bcount[G + 1] = 0;
   // The last thread's running offsets are the totals.
   if (threadIdx.x == kLayoutThreads - 1) {
     page_off_new[G] = (int32_t)o_tp;
@@ -417,11 +423,30 @@ __global__ void key_partial_kernel(const T *__restrict__ pool, int32_t d,
 
 // csum[g] += partials in segment order; refresh the fp32 mean and its bf16
 // hi/lo split for the group.
+// Also writes the host mirror slot (pinned host memory, mapped): the entry
+// count and every group's size after the batch, one group per block of the
+// first column range, so that no copy follows the append in the stream.
 __global__ void key_finalize_kernel(const KeyGroup *__restrict__ groups, const int32_t *__restrict__ n_groups,
                                     const double *__restrict__ partial, int32_t d,
                                     double *__restrict__ csum, float *__restrict__ cent,
-                                    __nv_bfloat16 *__restrict__ hi, __nv_bfloat16 *__restrict__ lo) {
+                                    __nv_bfloat16 *__restrict__ hi, __nv_bfloat16 *__restrict__ lo,
+                                    const int32_t *__restrict__ count, const int64_t *__restrict__ dev_ctr,
+                                    char *mirror, int32_t *__restrict__ bad, int32_t *__restrict__ hist,
+                                    int64_t hist_len) {
   pdl_entry();  // after the previous kernel of the stream (see common.cuh)
+  // The batch's remaining counters (read by nothing after the row placement):
+  // the check flag and the (group, chunk) counts, cleared for the next batch.
+  {
+    const int64_t t0 = ((int64_t)blockIdx.y * gridDim.x + blockIdx.x) * blockDim.x + threadIdx.x;
+    const int64_t nt = (int64_t)gridDim.x * gridDim.y * blockDim.x;
+    for (int64_t t = t0; t < hist_len; t += nt) hist[t] = 0;
+    if (t0 == 0) *bad = 0;
+  }
+  if (blockIdx.y == 0 && threadIdx.x == 0) {
+    if (blockIdx.x == 0) *reinterpret_cast<volatile int64_t *>(mirror) = dev_ctr[0];
+    reinterpret_cast<volatile int32_t *>(mirror + sizeof(int64_t))[blockIdx.x] = count[blockIdx.x];
+    __threadfence_system();
+  }
   if ((int)blockIdx.x >= *n_groups) return;  // the grid covers every group
   KeyGroup kg = groups[blockIdx.x];
   // The group's fp64 reciprocal comes from the layout block (fp64
@@ -513,7 +538,7 @@ htam_status refresh_mirror(htam_memory *m, bool wait) {
 // bit 1, leaving the memory unchanged.  `build` (the first batch of a new
 // memory) takes no -1 ids.
 static htam_status add_rows(htam_memory *m, const void *entries, const int32_t *gid, int64_t count,
-                            int32_t *assigned, cudaStream_t st, bool build, int32_t **bad_out = nullptr) {
+                            int32_t *assigned, cudaStream_t st, bool build) {
   if (count == 0) return HTAM_OK;
   PdlScope pdl(m->pdl != 0);
   const int32_t G = m->n_groups, d = m->d;
@@ -529,19 +554,36 @@ static htam_status add_rows(htam_memory *m, const void *entries, const int32_t *
   const int seg_rows = key_seg_rows(count);
   int64_t max_segs = std::min<int64_t>(count, count / seg_rows + G + 1);
 
-  size_t need = Carver::round(sizeof(int32_t) * (ceil_div(G + 2, 64) * 64 + (size_t)G * n_chunks)) +
-                Carver::round(sizeof(int32_t) * 4) + Carver::round(sizeof(int64_t)) +
+  size_t need = Carver::round(sizeof(int32_t) * 4) + Carver::round(sizeof(int64_t)) +
                 (build ? 0 : Carver::round(sizeof(int32_t) * count)) + Carver::round(sizeof(int32_t) * count) +
                 Carver::round(sizeof(KeySeg) * max_segs) + Carver::round(sizeof(KeyGroup) * G) +
                 2 * Carver::round(sizeof(int32_t) * G) + Carver::round(sizeof(double) * (size_t)max_segs * d) + 4096;
   htam_status s = ensure_scratch(m, need);
   if (s != HTAM_OK) return s;
-  Carver cv(m->scratch);
-  // Cleared by one memset: the batch's counts, the bad flag, the count of
+  // The batch counters live in a buffer of the memory object that is zero
+  // between batches: the batch's group counts, the check flag, the count of
   // rows without a group, then the (group, chunk) counts of the stable sort.
+  // The layout block clears the first and the last of the three, the key
+  // finalisation the flag and the (group, chunk) counts, so no memset
+  // starts a batch; a batch that stopped early leaves them marked dirty and
+  // the next one clears them first.
   const int64_t hist_off = ceil_div(G + 2, 64) * 64;
-  const int64_t n_zero = hist_off + (int64_t)G * n_chunks;
-  int32_t *bcount = cv.take<int32_t>(n_zero);  // [G] counts, bad flag, rows without a group
+  const int64_t n_ctr = hist_off + (int64_t)G * n_chunks;
+  if (n_ctr > m->batch_ctr_len) {
+    if (m->batch_ctr) cudaFree(m->batch_ctr);  // synchronises: no queued work still uses it
+    m->batch_ctr = nullptr;
+    m->batch_ctr_len = 0;
+    const int64_t want = n_ctr + n_ctr / 2;
+    if (cudaMalloc(&m->batch_ctr, sizeof(int32_t) * want) != cudaSuccess) {
+      cudaGetLastError();
+      m->batch_ctr = nullptr;
+      return HTAM_ENOMEM;
+    }
+    m->batch_ctr_len = want;
+    m->batch_dirty = true;
+  }
+  Carver cv(m->scratch);
+  int32_t *bcount = m->batch_ctr;              // [G] counts, bad flag, rows without a group
   int32_t *meta = cv.take<int32_t>(4);         // key segments, touched groups
   int64_t *id_base = cv.take<int64_t>(1);
   int32_t *ids = build ? nullptr : cv.take<int32_t>(count);  // groups chosen for rows given -1
@@ -553,14 +595,14 @@ static htam_status add_rows(htam_memory *m, const void *entries, const int32_t *
   int32_t *base = cv.take<int32_t>(G);
   double *partial = cv.take<double>((size_t)max_segs * d);
   int32_t *bad = bcount + G;
-  if (bad_out) *bad_out = bad;
 
   PhaseMark mark(m, st);
   mark.begin(HTAM_PHASE_APPEND);
 
   // 1. Per-group and per-(group, chunk) counts of the batch and the
   //    group-id range check.
-  HTAM_CK(cudaMemsetAsync(bcount, 0, sizeof(int32_t) * n_zero, st));
+  if (m->batch_dirty) HTAM_CK(cudaMemsetAsync(bcount, 0, sizeof(int32_t) * m->batch_ctr_len, st));
+  m->batch_dirty = true;  // until the key finalisation below is queued
   {
     const int blocks = (int)std::min<int64_t>(ceil_div(count, 256), 4096);
     launch_kernel(count_groups_kernel, blocks, 256, 0, st, gid, count, G, build ? 0 : 1, bcount, bad, bcount + G + 1,
@@ -639,9 +681,12 @@ static htam_status add_rows(htam_memory *m, const void *entries, const int32_t *
     }
     HTAM_CK_LAUNCH("key_partial_kernel");
     dim3 g2((unsigned)G, (unsigned)std::min<int64_t>(ceil_div(d, 256), 16));
+    const int slot = (int)((m->append_seq + 1) % htam_memory::kMirrorSlots);
+    char *mirror = static_cast<char *>(m->d_pin) + slot * m->pin_slot_bytes;
     launch_kernel(key_finalize_kernel, g2, 256, 0, st, kgroups, meta + 1, partial, d, m->csum, m->cent, m->cent_hi,
-                                            m->cent_lo);
+                  m->cent_lo, m->count, m->dev_ctr, mirror, bad, hist, (int64_t)G * n_chunks);
     HTAM_CK_LAUNCH("key_finalize_kernel");
+    m->batch_dirty = false;
     mark.launched(2);
   }
 
@@ -653,10 +698,8 @@ static htam_status add_rows(htam_memory *m, const void *entries, const int32_t *
   m->rows_issued += count;
   m->rows_pending += count;
   m->n += count;
+  // (key_finalize_kernel wrote the slot; its event marks it complete.)
   const int slot = (int)(m->append_seq % htam_memory::kMirrorSlots);
-  char *pin = static_cast<char *>(m->h_pin) + slot * m->pin_slot_bytes;
-  HTAM_CK(cudaMemcpyAsync(pin, m->dev_ctr, sizeof(int64_t), cudaMemcpyDeviceToHost, st));
-  HTAM_CK(cudaMemcpyAsync(pin + sizeof(int64_t), m->count, sizeof(int32_t) * G, cudaMemcpyDeviceToHost, st));
   HTAM_CK(cudaEventRecord(m->mirror_ev[slot], st));
   m->slot_seq[slot] = m->append_seq;
   m->slot_rows_issued[slot] = m->rows_issued;
@@ -677,6 +720,7 @@ void free_impl(htam_memory *m) {
   cudaFree(m->page_list_alt);
   cudaFree(m->page_off_alt);
   cudaFree(m->dev_ctr);
+  cudaFree(m->batch_ctr);
   if (m->h_pin) cudaFreeHost(m->h_pin);
   for (cudaEvent_t e : m->mirror_ev) {
     if (e) cudaEventDestroy(e);
@@ -750,6 +794,10 @@ htam_status build_impl(const void *entries, const int32_t *gid, int64_t n, int32
     m->h_pin = nullptr;
     return fail(HTAM_ENOMEM);
   }
+  if (cudaHostGetDevicePointer(&m->d_pin, m->h_pin, 0) != cudaSuccess) {
+    set_last_error("cudaHostGetDevicePointer", cudaGetLastError());
+    return fail(HTAM_ECUDA);
+  }
   for (cudaEvent_t &e : m->mirror_ev) {
     if (cudaEventCreateWithFlags(&e, cudaEventDisableTiming) != cudaSuccess) {
       cudaGetLastError();
@@ -774,16 +822,17 @@ htam_status build_impl(const void *entries, const int32_t *gid, int64_t n, int32
   }
   // The build is the one synchronous batch: a group id out of range fails
   // the call (and frees the memory) instead of being reported later.
-  int32_t *bad = nullptr;
-  htam_status s = add_rows(m, entries, gid, n, nullptr, st, /*build=*/true, &bad);
+  // The check's outcome is status bit 1 (set by the layout block for a
+  // rejected batch).
+  htam_status s = add_rows(m, entries, gid, n, nullptr, st, /*build=*/true);
   if (s != HTAM_OK) return fail(s);
-  int32_t h_bad = 0;
-  if (bad && (cudaMemcpyAsync(&h_bad, bad, sizeof h_bad, cudaMemcpyDeviceToHost, st) != cudaSuccess ||
-              cudaStreamSynchronize(st) != cudaSuccess)) {
+  unsigned h_status = 0;
+  if (cudaMemcpyAsync(&h_status, m->status, sizeof h_status, cudaMemcpyDeviceToHost, st) != cudaSuccess ||
+      cudaStreamSynchronize(st) != cudaSuccess) {
     set_last_error("htam_build_memory: reading the group-id check", cudaGetLastError());
     return fail(HTAM_ECUDA);
   }
-  if (h_bad) return fail(HTAM_EINVAL);
+  if (h_status & 2u) return fail(HTAM_EINVAL);
   s = refresh_mirror(m, true);
   if (s != HTAM_OK) return fail(s);
   *out = m;
