@@ -66,6 +66,9 @@ struct htam_memory {
   int32_t *batch_ctr = nullptr;  // batch counters of add_rows, zero between batches
   int64_t batch_ctr_len = 0;
   bool batch_dirty = false;       // a batch stopped before clearing them
+  uint32_t *qbits = nullptr;      // bucket bitmap of the multi-kernel bucketing, zero between queries
+  int64_t qbits_len = 0;
+  bool qbits_dirty = false;       // a query stopped before clearing it
   size_t pin_slot_bytes = 0;
   cudaEvent_t mirror_ev[kMirrorSlots] = {};
   int64_t slot_seq[kMirrorSlots] = {};       // append number each slot holds (0 = none)

@@ -721,6 +721,7 @@ void free_impl(htam_memory *m) {
   cudaFree(m->page_off_alt);
   cudaFree(m->dev_ctr);
   cudaFree(m->batch_ctr);
+  cudaFree(m->qbits);
   if (m->h_pin) cudaFreeHost(m->h_pin);
   for (cudaEvent_t e : m->mirror_ev) {
     if (e) cudaEventDestroy(e);

@@ -674,7 +674,7 @@ __global__ void __launch_bounds__(1024) bucket_scan_kernel(
                     seg_tc_dev);
 }
 
-__device__ __forceinline__ void bucket_fill_group(int g, int lane, const uint32_t *bits, int W,
+__device__ __forceinline__ void bucket_fill_group(int g, int lane, uint32_t *bits, bool clear, int W,
                                                   const int32_t *__restrict__ bucket_off,
                                                   const int32_t *__restrict__ cnt,
                                                   const int32_t *__restrict__ page_off, const Route &rt,
@@ -688,6 +688,11 @@ __device__ __forceinline__ void bucket_fill_group(int g, int lane, const uint32_
   const int base = bucket_off[g];
   for (int w0 = 0; w0 < W; w0 += 32) {
     uint32_t word = w0 + lane < W ? bits[(int64_t)g * W + w0 + lane] : 0u;
+    // The global bitmap of the multi-kernel bucketing is zero between
+    // queries: read here for the last time, so cleared for the next query.
+    // (The one-block bucketing's bitmap is in shared memory, where other
+    // threads may still be reading it.)
+    if (clear && w0 + lane < W) bits[(int64_t)g * W + w0 + lane] = 0u;
     int pc = __popc(word), incl = pc;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
@@ -718,7 +723,7 @@ __device__ __forceinline__ void bucket_fill_group(int g, int lane, const uint32_
 // One warp per group: bucket[g] lists its queries in increasing order.
 // Also writes the group's work units (group, chunk, segment) to the list of
 // the kernel that will score them, and the group of every bucket row.
-__global__ void bucket_fill_kernel(const uint32_t *__restrict__ bits, int G, int W,
+__global__ void bucket_fill_kernel(uint32_t *__restrict__ bits, int G, int W,
                                    const int32_t *__restrict__ bucket_off,
                                    const int32_t *__restrict__ cnt,
                                    const int32_t *__restrict__ page_off, Route rt,
@@ -743,7 +748,7 @@ __global__ void bucket_fill_kernel(const uint32_t *__restrict__ bits, int G, int
   const int g = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   rt.seg_tc = *seg_tc_dev;
   if (g < G) {
-    bucket_fill_group(g, threadIdx.x & 31, bits, W, bucket_off, cnt, page_off, rt, unit_off, unit_off_tc,
+    bucket_fill_group(g, threadIdx.x & 31, bits, true, W, bucket_off, cnt, page_off, rt, unit_off, unit_off_tc,
                       unit_off_tc2, bucket, bucket_group, units, units_tc, units_tc2);
   }
 }
@@ -795,7 +800,7 @@ __global__ void __launch_bounds__(1024) bucket_small_kernel(BucketSmallArgs a) {
   rt.seg_tc = *a.seg_tc_dev;
   for (int64_t t = tid; t < rows; t += 1024) bucket_pos_row(t, sbits, a.wpre, a.W, a.gidx, a.kg, a.pos);
   for (int g = warp; g < a.G; g += 32) {
-    bucket_fill_group(g, lane, sbits, a.W, a.bucket_off, a.cnt, a.page_off, rt, a.unit_off, a.unit_off_tc,
+    bucket_fill_group(g, lane, sbits, false, a.W, a.bucket_off, a.cnt, a.page_off, rt, a.unit_off, a.unit_off_tc,
                       a.unit_off_tc2, a.bucket, a.bucket_group, a.units, a.units_tc, a.units_tc2);
   }
 }
@@ -1362,7 +1367,7 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   // more prefix rows than the table has.
   const bool edge_table = er && (int64_t)B * er->P > G;
   const int wpq = warps_per_query(B, m->sm_count);  // warps per query in top-k and merge
-  size_t need = Carver::round(sizeof(float) * (size_t)planes * B * G) + 2 * Carver::round(sizeof(uint32_t) * (size_t)G * W) +
+  size_t need = Carver::round(sizeof(float) * (size_t)planes * B * G) + Carver::round(sizeof(uint32_t) * (size_t)G * W) +
                 6 * Carver::round(sizeof(int32_t) * (G + 4)) + Carver::round(sizeof(int64_t) * (G + 1)) +
                 2 * Carver::round(sizeof(int32_t)) + (er ? Carver::round(sizeof(int32_t) * (size_t)B * er->P) : 0) +
                 (edge_table ? Carver::round(sizeof(float) * (size_t)G * G) : 0) +
@@ -1374,7 +1379,12 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   if (s != HTAM_OK) return s;
   Carver cv(m->scratch);
   float *s1 = cv.take<float>((size_t)planes * B * G);
-  uint32_t *bits = cv.take<uint32_t>((size_t)G * W);
+  // The bitmap of the multi-kernel bucketing (group -> queries) lives in the
+  // memory object and is zero between queries: the fill kernel clears each
+  // word after its last read, so no memset precedes the bucketing.  A query
+  // that stopped before the fill leaves it marked dirty; the next one clears
+  // it first.
+  uint32_t *bits = nullptr;
   int32_t *wpre = cv.take<int32_t>((size_t)G * W);
   int32_t *cnt = cv.take<int32_t>(G + 1);
   int32_t *bucket_off = cv.take<int32_t>(G + 1);
@@ -1511,7 +1521,22 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
     HTAM_CK_LAUNCH("bucket_small_kernel");
     mark.launched();
   } else {
-    HTAM_CK(cudaMemsetAsync(bits, 0, sizeof(uint32_t) * (size_t)G * W, st));
+    if ((int64_t)G * W > m->qbits_len) {
+      if (m->qbits) cudaFree(m->qbits);  // synchronises: no queued work still uses it
+      m->qbits = nullptr;
+      m->qbits_len = 0;
+      const int64_t want = (int64_t)G * W + (int64_t)G * W / 2;
+      if (cudaMalloc(&m->qbits, sizeof(uint32_t) * want) != cudaSuccess) {
+        cudaGetLastError();
+        m->qbits = nullptr;
+        return HTAM_ENOMEM;
+      }
+      m->qbits_len = want;
+      m->qbits_dirty = true;
+    }
+    bits = m->qbits;
+    if (m->qbits_dirty) HTAM_CK(cudaMemsetAsync(bits, 0, sizeof(uint32_t) * (size_t)m->qbits_len, st));
+    m->qbits_dirty = true;  // until the fill below is queued
     launch_kernel(bucket_bits_kernel, (unsigned)ceil_div(rows, 256), 256, 0, st, group_idx, B, kg, W, bits);
     HTAM_CK_LAUNCH("bucket_bits_kernel");
     launch_kernel(bucket_count_kernel, (unsigned)ceil_div((int64_t)G * 32, 256), 256, 0, st, bits, G, W, cnt, wpre);
@@ -1525,6 +1550,7 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
         bits, G, W, bucket_off, cnt, m->page_off, rt, seg_tc, unit_off, unit_off_tc, unit_off_tc2, bucket,
         bucket_group, units, units_tc, units_tc2, tc_ok ? thr_enc : nullptr, B * kThrWords, tc_ctr);
     HTAM_CK_LAUNCH("bucket_fill_kernel");
+    m->qbits_dirty = false;
     mark.launched(5);
   }
   CUtensorMap q_map;
