@@ -32,10 +32,15 @@
 // and passes its index to the MMA and epilogue warps through a small
 // shared-memory queue guarded by mbarriers.
 //
-// Warp roles (192 threads, one CTA per SM, persistent over units):
+// Warp roles (224 threads, one CTA per SM, persistent over units):
 //   warp 0   TMA producer (lane 0 issues)
 //   warp 1   TMEM owner, MMA issuer (lane 0 issues)
 //   warps 2..5  epilogue (TMEM lane quadrant = warp % 4)
+//   warp 6   A copier: the chunk's query rows, straight from the query
+//            matrix with cp.async into the swizzled A stages, two stages
+//            ahead of their release (one-SM units of batches it is chosen
+//            for; otherwise the block has 192 threads and the producer loads
+//            bucket-ordered A tiles by TMA)
 // Every mbarrier wait is bounded; a give-up sets the memory's status word and
 // the CTA drains its own copies and MMAs before releasing tensor memory.
 
@@ -59,7 +64,9 @@ constexpr int kTileN = 2 * kPageRows;              // entries per tile (MMA N)
 constexpr int kABytes = kTcRows * kKBlock * 2;     // 16 KiB
 constexpr int kBBytes = kTileN * kKBlock * 2;      // 32 KiB
 constexpr int kHalfB = kBBytes / 2;                // one page's K slice
-constexpr int kThreads = 192;
+constexpr int kThreads = 224;     // with the A copier (warp 6)
+constexpr int kThreadsTma = 192;  // without it: the A tiles come by TMA
+constexpr int kALag = 2;  // stages the A copier keeps in flight before releasing the oldest
 constexpr uint32_t kAccCols = 256;                 // fp32 columns per accumulator
 constexpr unsigned kFull = 0xffffffffu;
 
@@ -112,6 +119,22 @@ __device__ __forceinline__ int take_unit(TcSmem *sh, int j, uint32_t empty_caddr
     }
   }
   return u;
+}
+
+// Copies of query rows into an A stage by the copier warp's lanes: 16 bytes
+// each, zero-filled past the row's end (src_bytes 0).
+__device__ __forceinline__ void cp_async16_zfill(uint32_t dst, const void *src, uint32_t src_bytes) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+// Makes this thread's completed generic-proxy writes to shared memory (the
+// copies above) visible to the async proxy that tcgen05.mma reads through.
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
 // Per epilogue warp, a 32 x 32 fp32 staging area: a lane writes its row's
@@ -224,7 +247,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t uq_empty_c0 = PAIR ? mapa_shared(smem_addr(&sh->uq_empty[0]), 0) : smem_addr(&sh->uq_empty[0]);
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
-      mbar_init(&sh->full[s], 1);
+      // With the A copier, a stage is full once its B pages' bytes landed
+      // and the copier has arrived for its A rows.
+      mbar_init(&sh->full[s], (!PAIR && a.a_rows) ? 2 : 1);
       mbar_init(&sh->empty[s], 1);
     }
     for (int i = 0; i < 2; ++i) {
@@ -234,9 +259,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(&sh->drain, 1);
     for (int i = 0; i < kUQ; ++i) {
       mbar_init(&sh->uq_full[i], 1);
-      // Single: MMA warp + 4 epilogue warps.  Pair (rank 0's barrier): its
-      // MMA warp and 4 epilogue warps, rank 1's producer and 4 epilogue warps.
-      mbar_init(&sh->uq_empty[i], PAIR ? 10 : 5);
+      // Single: MMA warp + 4 epilogue warps (+ the A copier).  Pair (rank 0's
+      // barrier): its MMA warp and 4 epilogue warps, rank 1's producer and 4
+      // epilogue warps.
+      mbar_init(&sh->uq_empty[i], PAIR ? 10 : (a.a_rows ? 6 : 5));
     }
     sh->abort = 0;
     fence_barrier_init();
@@ -331,6 +357,10 @@ __global__ void __launch_bounds__(kThreads, 1)
               } else if (two) {
                 tma_load_2d_pair(dst_b, &pool_map, x, y1, bar);
               }
+            } else if (a.a_rows) {
+              mbar_arrive_expect_tx(&sh->full[st], two ? kBBytes : kHalfB);
+              tma_load_2d(dst_b, &pool_map, x, y0, &sh->full[st]);
+              if (two) tma_load_2d(dst_b + kHalfB, &pool_map, x, y1, &sh->full[st]);
             } else {
               mbar_arrive_expect_tx(&sh->full[st], kABytes + (two ? kBBytes : kHalfB));
               tma_load_2d(dst_a, &q_map, x, a_row, &sh->full[st]);
@@ -451,6 +481,86 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
     __syncwarp();
+  } else if (warp == 6) {
+    // ---------------------------------------------------------- A copier
+    // Walks the same units, tiles and K slices as the producer (so the
+    // same stages and phases), waits for each stage to be free, copies the
+    // K slice of the chunk's 128 query rows into it (lane l: rows l, l+32,
+    // l+64, l+96), and releases a stage kALag stages later: once the lane's
+    // copy group of that stage completed, a proxy fence, then one arrival.
+    if (!PAIR && a.a_rows) {
+      int st = 0;
+      uint32_t ph = 0;
+      bool ok = true;
+      int64_t n_iss = 0;  // stages issued (their stage indices run in order)
+      int qid[4];         // query ids of the chunk's rows lane, lane+32, lane+64, lane+96
+      for (int j = 0; ok; ++j) {
+        const int u = take_unit<PAIR>(sh, j, uq_empty_c0, abort, a.max_polls, ok);
+        if (u < 0) break;
+        const int4 U = a.units[u];
+        const int g = U.x, c = U.y;
+        const int a_row = a.bucket_off[g] + c * kTcRows;
+        const int nq = min(kTcRows, a.cnt[g] - c * kTcRows);
+        // Rows past the chunk's queries repeat its first query (in bounds;
+        // their accumulator rows are never read).
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const int r = lane + 32 * i;
+          qid[i] = a.bucket[a_row + (r < nq ? r : 0)];
+        }
+        const int npg = a.page_off[g + 1] - a.page_off[g];
+        const int p_beg = U.z * seg_pages, p_end = min(npg, p_beg + seg_pages);
+        const int n_stages = (p_end - p_beg + 1) / 2 * nk;
+        for (int i_st = 0; i_st < n_stages; ++i_st) {
+          const int kb = i_st % nk;
+          if (!mbar_wait(&sh->empty[st], ph ^ 1u, abort, a.max_polls)) {
+            ok = false;
+            break;
+          }
+          // K slice kb of the 128 rows, four rows per instruction: eight lanes
+          // take the eight 16-byte vectors of one row (128 contiguous bytes),
+          // stored where the 128-byte swizzle puts them (vector v of row r at
+          // 16 * (v ^ (r % 8))).  The row's query id comes from the lane that
+          // holds it.
+          const uint32_t dst_a = smem_addr(st_a + st * kABytes);
+          const int v = lane & 7;
+          const bool in = kb * (kKBlock / 8) + v < a.qvec;
+          const int vsrc = in ? kb * (kKBlock / 8) + v : 0;
+#pragma unroll
+          for (int i = 0; i < kTcRows / 4; ++i) {
+            const int r = 4 * i + (lane >> 3);
+            const int q = __shfl_sync(kFull, qid[i / 8], r & 31);
+            cp_async16_zfill(dst_a + r * 128 + ((v ^ (r & 7)) << 4), a.queries + (int64_t)q * a.qvec + vsrc,
+                             in ? 16u : 0u);
+          }
+          cp_async_commit();
+          if (++n_iss > kALag) {
+            // The stage issued kALag stages ago: its group has completed.
+            cp_async_wait<kALag>();
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&sh->full[(st + kStages - kALag) % kStages]);
+          }
+          if (++st == kStages) {
+            st = 0;
+            ph ^= 1u;
+          }
+        }
+      }
+      // The stages still waiting: every copy of the lane completed, fenced,
+      // then their arrivals.
+      cp_async_wait<0>();
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) {
+        const int left = (int)(n_iss < kALag ? n_iss : kALag);
+        for (int q = left; q >= 1; --q) mbar_arrive(&sh->full[(st + kStages - q) % kStages]);
+      }
+      if (!ok && lane == 0) {
+        atomicOr(a.status, 1u);
+        sh->abort = 1;
+      }
+    }
   } else {
     // ----------------------------------------------------------- epilogue
     const int quad = warp & 3;                // TMEM lane quadrant
@@ -725,7 +835,7 @@ htam_status launch_k(const TcFineArgs &a, const CUtensorMap &q_map, const CUtens
   if constexpr (PAIR) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)grid, 1, 1);
-    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.blockDim = dim3(kThreadsTma, 1, 1);
     cfg.dynamicSmemBytes = smem_bytes<PAIR>();
     cfg.stream = st;
     cudaLaunchAttribute attr[2];
@@ -739,7 +849,8 @@ htam_status launch_k(const TcFineArgs &a, const CUtensorMap &q_map, const CUtens
     cfg.numAttrs = g_launch_pdl ? 2 : 1;
     HTAM_CK(cudaLaunchKernelEx(&cfg, fine_tc_kernel<K, true>, q_map, pool_map, a));
   } else {
-    launch_kernel(fine_tc_kernel<K, false>, grid, kThreads, smem_bytes<false>(), st, q_map, pool_map, a);
+    launch_kernel(fine_tc_kernel<K, false>, grid, a.a_rows ? kThreads : kThreadsTma, smem_bytes<false>(), st, q_map,
+                  pool_map, a);
   }
   HTAM_CK_LAUNCH("fine_tc_kernel");
   return HTAM_OK;

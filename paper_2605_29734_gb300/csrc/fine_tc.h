@@ -45,6 +45,13 @@ struct TcFineArgs {
   uint32_t max_polls;
   int q_direct;               // 1: every bucket holds all queries in order and the query map is the
                               // query matrix itself (rows from 0), 0: rows from bucket_off[g]
+  // a_rows = 1 (one-SM units): a copier warp copies each chunk's query rows
+  // from the query matrix `queries` (`qvec` 16-byte vectors a row) with
+  // cp.async into the swizzled A stages; the query map is then unused.
+  // 0: the A tiles come from the query map by TMA.
+  int a_rows;
+  const uint4 *queries;
+  int qvec;
 };
 
 // Encodes a 2-D bf16 row-major [rows, cols] tensor for TMA tile loads of

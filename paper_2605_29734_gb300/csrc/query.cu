@@ -1357,9 +1357,18 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   const int64_t max_units = max_parts;
   const int64_t rows = (int64_t)B * kg;  // bucket rows
   const int W = (int)ceil_div(B, 32);
-  // Flat scan: every bucket holds all queries in order, so the tensor-core
-  // kernel reads the query matrix itself instead of a gathered copy.
-  const size_t qg_bytes = tc_ok && !flat ? sizeof(__nv_bfloat16) * (size_t)rows * d : 0;
+  // The tensor-core kernel's A rows.  The flat scan's buckets hold every
+  // query in order, so TMA reads the query matrix itself.  Otherwise, for
+  // batches of up to 2,048 queries of up to 1,024 dims on one-SM units, a
+  // copier warp of the kernel copies them from the query matrix (no
+  // bucket-ordered copy: 65k workload 0.113 -> 0.110 ms, stream 0.341 ->
+  // 0.335 ms); larger batches, longer rows and SM pairs read a
+  // bucket-ordered copy by TMA (the copier's 32 copies a lane per K slice
+  // made the 4,096-query 1M workload's kernel 0.657 -> 0.797 ms).
+  const bool tc_pairs_run = tc_ok && rt.pairs && B > kTcRows;
+  const bool a_rows = tc_ok && !flat && !tc_pairs_run && B <= 2048 && d <= 1024;
+  const bool q_gather = tc_ok && !flat && !a_rows;
+  const size_t qg_bytes = q_gather ? sizeof(__nv_bfloat16) * (size_t)rows * d : 0;
 
   // Coarse scores: one plane per K split of the tensor-core kernel.
   const int planes = flat ? 0 : m->dtype == HTAM_BF16 && !er ? coarse_tc_splits(B, d, G, m->sm_count) : 1;
@@ -1407,7 +1416,7 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
   float *part_s = cv.take<float>(max_parts * ke);
   int32_t *part_id = cv.take<int32_t>(max_parts * ke);
   unsigned *thr_enc = cv.take<unsigned>((size_t)B * kThrWords);
-  void *qg = tc_ok && !flat ? static_cast<void *>(cv.take<char>(qg_bytes)) : nullptr;
+  void *qg = q_gather ? static_cast<void *>(cv.take<char>(qg_bytes)) : nullptr;
   float *policy_keys = smp ? cv.take<float>((size_t)B * G) : nullptr;
   if (flat) {
     group_idx = cv.take<int32_t>(rows);
@@ -1562,9 +1571,11 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
       if (s != HTAM_OK) return s;
       m->pool_map_ready = true;
     }
-    s = flat ? make_bf16_tile_map(&q_map, queries, B, d, kTcRows) : make_bf16_tile_map(&q_map, qg, rows, d, kTcRows);
+    // (A map of the query matrix when no bucket-ordered copy is made; the
+    // kernel then ignores it unless the scan is flat.)
+    s = q_gather ? make_bf16_tile_map(&q_map, qg, rows, d, kTcRows) : make_bf16_tile_map(&q_map, queries, B, d, kTcRows);
     if (s != HTAM_OK) return s;
-    if (!flat) {
+    if (q_gather) {
       s = launch_gather_queries(queries, d, bucket, bucket_group, cnt, rt.tc_min, bucket_off + G, rows, qg, st);
       if (s != HTAM_OK) return s;
       mark.launched();
@@ -1617,9 +1628,12 @@ htam_status query_impl(htam_memory *m, const void *queries, int32_t B, const hta
     mark.begin(HTAM_PHASE_FINE_TC);
     TcFineArgs ta{units_tc, n_units + 1, tc_ctr, bucket, bucket_off, cnt, m->page_list, m->page_off, m->count, m->slot_id,
                   part_off, d, seg_tc, ke, 1.4426950408889634f / p.tau, part_ml, part_s, part_id, thr_enc,
-                  m->status, kMaxPolls, flat ? 1 : 0};
-    if (rt.pairs && B > kTcRows) {
-      // Buckets of several chunks on SM pairs, then the one-chunk buckets.
+                  m->status, kMaxPolls, flat ? 1 : 0, a_rows ? 1 : 0,
+                  static_cast<const uint4 *>(queries), d * 2 / 16};
+    if (tc_pairs_run) {
+      // Buckets of several chunks on SM pairs, then the one-chunk buckets
+      // (both by TMA: from the bucket-ordered copy, or the query matrix in a
+      // flat scan).
       TcFineArgs tp = ta;
       tp.units = units_tc2;
       tp.n_units = n_units + 2;
