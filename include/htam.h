@@ -105,8 +105,9 @@ htam_status htam_build_memory(const void *entries, const int32_t *group_ids,
  *             excluded), by the keys as they stand before this call
  * Fully asynchronous: the batch's group sizes, the nearest-key choices, the
  * page layout and the key updates are all computed on the device, with no
- * host round trip (a growth of the memory object's scratch, on the first
- * append of a new size, synchronises the device once).  Page space never
+ * host round trip and no memset or copy in the stream (a growth of the
+ * memory object's scratch or batch counters, on the first append of a new
+ * size, synchronises the device once).  Page space never
  * runs out: the pages reserved at build hold any `capacity` entries.
  * The group ids are checked on the device.  A batch with an id out of range,
  * or an id of -1 while every group is empty, is rejected there: the memory
