@@ -485,9 +485,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ---------------------------------------------------------- A copier
     // Walks the same units, tiles and K slices as the producer (so the
     // same stages and phases), waits for each stage to be free, copies the
-    // K slice of the chunk's 128 query rows into it (lane l: rows l, l+32,
-    // l+64, l+96), and releases a stage kALag stages later: once the lane's
-    // copy group of that stage completed, a proxy fence, then one arrival.
+    // K slice of the chunk's 128 query rows into it, and releases a stage
+    // kALag stages later: once the lane's copy group of that stage
+    // completed, a proxy fence, then one arrival.  Lane l holds the query
+    // ids of rows l, l+32, l+64 and l+96.
     if (!PAIR && a.a_rows) {
       int st = 0;
       uint32_t ph = 0;
