@@ -1168,6 +1168,25 @@ def test_programmatic_launch_on_and_off_agree_bitwise(htam):
     assert torch.equal(outs[0][2], outs[1][2])
 
 
+def test_query_rows_copied_or_gathered_agree_bitwise(htam):
+    """The tensor-core kernel takes its query rows from the query matrix by
+    its copier warp for batches of up to 2,048 queries, and from a
+    bucket-ordered copy by TMA above that.  The same 2,048 queries give
+    bit-identical results either way: once alone (copier), once followed by
+    a repeat of the batch (4,096 queries, TMA), every bucket on the tensor
+    cores in both."""
+    entries, gid, centres = _rand_memory(40000, 256, 96, torch.bfloat16, seed=61)
+    q = _rand_queries(2048, 256, torch.bfloat16, seed=61, centres=centres)
+    mem = htam.Memory(entries, gid, 96)
+    mem.set_tensor_core_min_bucket(1)
+    a = {k: v.clone() for k, v in mem.query(q, 6, 16, tau=0.5, epsilon=0.05).items()}
+    b = mem.query(torch.cat([q, q]).contiguous(), 6, 16, tau=0.5, epsilon=0.05)
+    torch.cuda.synchronize()
+    for k in a:
+        assert torch.equal(a[k], b[k][:2048]) and torch.equal(a[k], b[k][2048:]), k
+    assert mem.device_status() == htam.HTAM_OK
+
+
 def test_bad_query_arguments(htam):
     entries, gid, _ = _rand_memory(100, 16, 4, torch.float32, seed=17)
     mem = htam.Memory(entries, gid, 4)
