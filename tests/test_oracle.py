@@ -110,6 +110,24 @@ def test_single_candidate_has_weight_one():
     assert np.isneginf(out["entry_score"][0][1:]).all()
 
 
+def test_cold_softmax_keeps_the_closed_form():
+    """Eq. 11 at a temperature where exp(s/tau) overflows a double: scores 0
+    and 1 at tau = 1e-3 give lse = 1000 + log(1 + e^-1000) = 1000 and
+    weights eps/2 + (1-eps) * {e^-1000, 1}.  The weaker candidate comes first
+    in entry order, so the softmax has to shift by the largest s/tau, not by
+    whichever candidate it met first."""
+    entries = np.array([[1.0, 0, 0, 0], [0, 1.0, 0, 0], [0, 0, 1.0, 0]], dtype=np.float32)
+    gid = np.array([0, 0, 1], dtype=np.int32)
+    q = np.array([[0, 1.0, 0, 0]], dtype=np.float32)
+    eps = 0.1
+    out = oracle.query(entries, gid, 2, q, k_groups=1, k_entries=2, tau=1e-3, eps=eps)
+    assert list(out["group_idx"][0]) == [0]
+    assert list(out["entry_idx"][0]) == [1, 0]
+    assert out["lse"][0] == pytest.approx(1000.0, rel=1e-15)
+    assert out["entry_weight"][0][0] == pytest.approx(eps / 2 + (1 - eps), rel=1e-15)
+    assert out["entry_weight"][0][1] == pytest.approx(eps / 2, rel=1e-15)
+
+
 # ---------------------------------------------------- library-routine special cases
 
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])

@@ -8,7 +8,12 @@ groups allowed into stage 1, prefix weights reversed, of the wrong sign or
 missing the newest element, edge-table rows and columns swapped, an edge
 feature misread, edge-prefix weights reversed, Philox words swapped or its key
 not advanced, one uniform shared by four groups, the policy's eps term dropped
-or tau ignored, the Gumbel noise of the wrong sign, empty groups drawn), or one
+or tau ignored, the Gumbel noise of the wrong sign, empty groups drawn, the
+softmax's log-sum-exp missing its shift or shifted by the first candidate
+instead of the largest, the eps/|C| term spread over k_entries, padding slots
+weighted, the last candidate dropped from the top-k, stage 1 padding with
+group 0, stage 2 reading only the first selected group, a coordinate split
+that skips a column of the key sums, group sizes not accumulated), or one
 in the Python layer that composes the C routines (the sampled lookup ranking
 instead of drawing or dropping tau in stage 2, the edge-routed lookup counting
 empty groups, the flat scan ignoring tau, the nearest-key assignment
@@ -52,6 +57,18 @@ MUTANTS = {
     "policy_tau_ignored": ("if (counts[g] > 0) sum += exp(s[g] / tau - m);", "if (counts[g] > 0) sum += exp(s[g] - m);"),
     "gumbel_sign_flipped": ("keys[o] = log_mu - log(-log(u));", "keys[o] = log_mu + log(-log(u));"),
     "policy_empty_groups_drawn": ("      if (counts[g] == 0) {\n        mu[o] = 0.0;", "      if (0) {\n        mu[o] = 0.0;"),
+    "lse_shift_dropped": ("lse_b = m + log(sum);", "lse_b = log(sum);"),
+    "softmax_shift_not_max": ("if (z > m) m = z;", "if (i == 0) m = z;"),
+    "eps_spread_over_k": ("job->eps / (double)n_cand +", "job->eps / (double)job->k_entries +"),
+    "entry_pad_weighted": ("job->entry_weight[o] = 0.0;", "job->entry_weight[o] = job->eps / (double)n_cand;"),
+    "topk_drops_last_candidate": ("if (j < n_cand) {\n        job->entry_idx[o]",
+                                  "if (j + 1 < n_cand) {\n        job->entry_idx[o]"),
+    "stage1_pads_with_group_zero": ("job->group_idx[o] = -1;", "job->group_idx[o] = 0;"),
+    "stage2_first_group_only": ("for (int32_t j = 0; j < job->k_groups; ++j) {\n      int32_t g = job->groups",
+                                "for (int32_t j = 0; j < 1; ++j) {\n      int32_t g = job->groups"),
+    "key_columns_split_short": ("(int32_t)((int64_t)d * (t + 1) / nthreads)",
+                                "(int32_t)((int64_t)d * (t + 1) / nthreads) - 1"),
+    "counts_not_accumulated": ("counts[gid[e]] += 1;", "counts[gid[e]] = 1;"),
     # Slips in the Python layer that composes the C routines.
     "sampled_lookup_ranks_instead_of_drawing": ("__init__.py", "gi, gk = select(keys, counts, k_groups)",
                                                 "gi, gk = select(coarse_scores(queries, centroid), counts, k_groups)"),
