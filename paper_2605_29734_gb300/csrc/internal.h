@@ -51,9 +51,10 @@ struct htam_memory {
 
   // Host mirror of the group sizes, exact as of the append numbered
   // mirror_seq; rows_pending rows were queued after it.  Appends run on the
-  // device without a host round trip: each one ends by copying the device
-  // sizes and entry count into a pinned slot of a small ring and recording an
-  // event; a later call adopts the newest slot whose event has completed
+  // device without a host round trip: in each one the key finalisation
+  // kernel writes the device sizes and entry count into a slot of a small
+  // ring of mapped pinned memory, and an event is recorded after it; a later
+  // call adopts the newest slot whose event has completed
   // (htam_device_status and the introspection calls wait for it).
   static constexpr int kMirrorSlots = 4;
   std::vector<int64_t> h_count;
